@@ -1,0 +1,108 @@
+"""Workload driver for the oracle: weight preparation, prefill, decode steps.
+
+Weight preparation (offline in the paper, Sec. 3.1 and the Sec. 4 setup):
+the tiny layer factors a Gaussian W_qkv by the joint SVD (Eq. 2-4, beta = 0.5
+since the paper learns beta per layer and prints no value); every layer's
+fp32 W_d is quantized per output channel to int8 (RTN, clip ratio 1.0), and
+the up-projections are stored in bf16.
+
+Decode order per step (every sequence gets one new token): project the new
+tokens (Eq. 12), append their latent codes at position len[b], then attend
+over positions 0..len[b] (Eq. 5).  K and V rows are computed once per token
+when the token enters the cache: row t of C W^u depends only on row t of C,
+so this is the definition evaluated row by row.
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict, Iterable, Optional
+
+import numpy as np
+
+from synthetic import LayerInputs, bf16_bits, bf16_from_bits
+
+from . import attention, latent, quant, svd
+
+TINY_BETA = 0.5
+
+
+def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1.0):
+    """Returns dict(W_d fp32 values [d, r], Wq int64 [d, r], s_w [r],
+    U_q/U_k/U_v bf16 bits [r, d])."""
+    s = inp.workload.shape
+    if inp.W_qkv is not None:
+        d = s.d
+        W_d, Uq, Uk, Uv, _ = svd.joint_qkv_factors(
+            inp.W_qkv[:, :d], inp.W_qkv[:, d:2 * d], inp.W_qkv[:, 2 * d:], s.r, beta)
+        W_d = quant.f32(W_d)
+        U_q, U_k, U_v = bf16_bits(Uq), bf16_bits(Uk), bf16_bits(Uv)
+    else:
+        W_d, U_q, U_k, U_v = inp.W_d, inp.U_q, inp.U_k, inp.U_v
+    Wq, s_w = quant.quantize_columns(W_d, 8, w_clip)
+    return dict(W_d=W_d, Wq=Wq, s_w=s_w, U_q=U_q, U_k=U_k, U_v=U_v)
+
+
+class OracleLayer:
+    """One layer's latent cache plus explicit K/V rows for tracked sequences."""
+
+    def __init__(self, shape, weights: Dict, B: int, tmax: int, lat_bits: int,
+                 act_clip: float = 1.0, lat_clip: float = 1.0,
+                 track: Optional[Iterable[int]] = None):
+        self.s = shape
+        self.w = weights
+        self.U_q = bf16_from_bits(weights["U_q"])
+        self.U_k = bf16_from_bits(weights["U_k"])
+        self.U_v = bf16_from_bits(weights["U_v"])
+        self.B, self.tmax, self.bits = B, tmax, lat_bits
+        self.act_clip, self.lat_clip = act_clip, lat_clip
+        self.cache = latent.LatentCache(B, tmax, shape.r, lat_bits)
+        self.len = np.zeros(B, dtype=np.int64)
+        self.track = set(range(B)) if track is None else set(track)
+        self.K = {b: np.zeros((tmax, shape.d)) for b in self.track}
+        self.V = {b: np.zeros((tmax, shape.d)) for b in self.track}
+
+    def project(self, X_bits):
+        """Eq. 12 for a block of tokens given as bf16 bits [T, d]."""
+        X = bf16_from_bits(X_bits)
+        return latent.latent_project(X, self.w["Wq"], self.w["s_w"],
+                                     self.act_clip, self.bits, self.lat_clip)
+
+    def _append(self, seq, pos, codes, scale):
+        self.cache.append(seq, pos, codes, scale)
+        for b in set(int(x) for x in seq) & self.track:
+            sel = np.asarray(seq) == b
+            rows = latent.dequantize_latent(codes[sel], scale[sel], self.bits)
+            p = np.asarray(pos)[sel]
+            self.K[b][p] = rows @ self.U_k
+            self.V[b][p] = rows @ self.U_v
+
+    def prefill(self, b: int, X_bits):
+        """Project and cache the prompt of sequence b (positions len[b]...)."""
+        out = self.project(X_bits)
+        T = X_bits.shape[0]
+        pos = self.len[b] + np.arange(T)
+        self._append(np.full(T, b), pos, out["codes"], out["scale"])
+        self.len[b] += T
+        return out
+
+    def attend(self, b: int):
+        L = int(self.len[b])
+        C = self.cache.rows(b, L)
+        if b in self.track:
+            return attention.decode_attention(C, self.U_q, self.U_k, self.U_v,
+                                              self.s.H, self.s.dh,
+                                              1.0 / math.sqrt(self.s.dh),
+                                              K=self.K[b][:L], V=self.V[b][:L])
+        return attention.decode_attention(C, self.U_q, self.U_k, self.U_v,
+                                          self.s.H, self.s.dh)
+
+    def decode_step(self, x_bits, attend: Optional[Iterable[int]] = None):
+        """One decode step: x_bits [B, d] bf16 bits, one token per sequence.
+        Returns (projection dict, {b: o_b}) for the sequences in ``attend``
+        (default: the tracked ones)."""
+        out = self.project(x_bits)
+        seq = np.arange(self.B)
+        self._append(seq, self.len.copy(), out["codes"], out["scale"])
+        self.len += 1
+        targets = sorted(self.track) if attend is None else list(attend)
+        return out, {b: self.attend(b) for b in targets}
