@@ -1,0 +1,513 @@
+#!/usr/bin/env python
+"""Benchmark of the QSVD latent-attention hot path (arxiv 2510.16292) on GB300.
+
+One step = one pass of the whole path over the LLaVA-7B-shaped layer
+(d=4096, H=32, dh=128, r=1536): prefill of 640 tokens (576 image-like + 64
+text-like; per-token int8 X, exact int8 GEMM with W_d, per-token latent
+requantization fused into the cache store), then 128 decode steps (project
+the new token, append it, attend over the int8 latent cache with U_k absorbed
+and U_v applied last).  Inputs are seeded synthetic arrays resident in HBM
+before timing.  L2 is flushed (a 256 MiB write) before the prefill and before
+every decode step; the flush sits outside the timed intervals, which are CUDA
+events on the launching stream around each sub-step.
+
+value = decode tokens/s (all ranks' tokens / max-over-ranks decode time).
+Secondary figures: prefill TOPS (2*T*d*r over the projection call), latent
+cache GB/s, and the decode step's fraction of its HBM roofline.
+
+--impl reference times the CPU oracle (the plain fp64 definition) on a
+bounded sample of the same workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synthetic  # noqa: E402
+
+METRIC = "decode tokens/s + latent-cache HBM GB/s; prefill int8 TOPS (LLaVA-7B shape)"
+WORKLOAD = "llava7b"
+FLUSH_BYTES = 256 << 20
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["native", "reference"], default="native")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            m = json.load(f)
+        return float(m["hbm_gbs"]), float(m["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+def workload_desc(wl):
+    s = wl.shape
+    return (f"{wl.name}: d={s.d} H={s.H} dh={s.dh} r={s.r}, B={wl.B}, prefill {wl.n_image} image-like + "
+            f"{wl.n_text} text-like tokens, {wl.decode_steps} decode steps, int{wl.lat_bits} latent cache")
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) >= 9:
+                rows.append(f)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------
+# native arm
+# ---------------------------------------------------------------------------
+class NativeBench:
+    def __init__(self, wl, rank):
+        import torch
+        import paper_2510_16292_gb300 as q
+        self.torch, self.q, self.wl = torch, q, wl
+        s = wl.shape
+        self.dev = torch.device("cuda", torch.cuda.current_device())
+        inp = synthetic.gen_layer(wl, seed=rank)
+        self.inp = inp
+        dev = self.dev
+
+        def bf16(bits):
+            a = np.ascontiguousarray(bits).view(np.int16)
+            return torch.from_numpy(a).view(torch.bfloat16).to(dev)
+
+        self.W = q.qsvd_quantize_weight(torch.from_numpy(inp.W_d.astype(np.float32)).to(dev))
+        self.U = [bf16(u) for u in (inp.U_q, inp.U_k, inp.U_v)]
+        B, P, S = wl.B, wl.prefill, wl.decode_steps
+        self.B, self.P, self.S = B, P, S
+        self.Xp = bf16(inp.X_prefill.reshape(B * P, s.d))
+        self.Xd = bf16(inp.X_decode)                       # [S, B, d]
+        self.cache = q.LatentCache.empty(B, wl.tmax, s.r, wl.lat_bits, dev)
+        i32 = lambda a: torch.as_tensor(np.asarray(a, dtype=np.int32), device=dev)  # noqa: E731
+        self.pseq = i32(np.repeat(np.arange(B), P))
+        self.ppos = i32(np.tile(np.arange(P), B))
+        self.dseq = i32(np.arange(B))
+        self.dpos = [i32(np.full(B, P + t)) for t in range(S)]
+        self.dlen = [i32(np.full(B, P + t + 1)) for t in range(S)]
+        self.O = torch.empty((B, s.d), dtype=torch.float32, device=dev)
+        self.wsp = torch.empty(q.qsvd_project_workspace_bytes(B * P, s.d, s.r), dtype=torch.uint8, device=dev)
+        self.wsd = torch.empty(q.qsvd_decode_workspace_bytes(B, wl.tmax, s.r, s.H, s.dh), dtype=torch.uint8,
+                               device=dev)
+        self.flushbuf = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+        self.stream = torch.cuda.current_stream()
+        self._marshal()
+
+    def _marshal(self):
+        """Pre-build the ctypes argument tuples of every C-ABI call of a step."""
+        q, wl, s = self.q, self.wl, self.wl.shape
+        lib = q._lib
+        self.lib = lib
+        self.cW = self.W._c()
+        self.cC = self.cache._c()
+        st = self.stream.cuda_stream
+        P = ctypes.c_void_p
+        self.pre_args = (ctypes.byref(self.cW), self.Xp.data_ptr(), self.B * self.P, 1.0, wl.lat_bits, 1.0,
+                         None, None, ctypes.byref(self.cC), self.pseq.data_ptr(), self.ppos.data_ptr(),
+                         None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st)
+        self.dec_proj = []
+        self.dec_attn = []
+        for t in range(self.S):
+            self.dec_proj.append((ctypes.byref(self.cW), self.Xd[t].data_ptr(), self.B, 1.0, wl.lat_bits, 1.0,
+                                  None, None, ctypes.byref(self.cC), self.dseq.data_ptr(), self.dpos[t].data_ptr(),
+                                  None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st))
+            self.dec_attn.append((ctypes.byref(self.cC), self.dlen[t].data_ptr(), self.P + t + 1,
+                                  self.U[0].data_ptr(), self.U[1].data_ptr(), self.U[2].data_ptr(), s.H, s.dh,
+                                  1.0 / math.sqrt(s.dh), self.O.data_ptr(), self.wsd.data_ptr(),
+                                  self.wsd.numel(), st))
+        del P
+
+    def _call(self, fn, args):
+        stt = fn(*args)
+        if stt != 0:
+            raise RuntimeError(f"qsvd status {stt}: {self.lib.qsvd_last_error().decode()}")
+
+    def prefill(self):
+        self._call(self.lib.qsvd_latent_project, self.pre_args)
+
+    def decode(self, t):
+        self._call(self.lib.qsvd_latent_project, self.dec_proj[t])
+        self._call(self.lib.qsvd_latent_decode_attn, self.dec_attn[t])
+
+    def flush(self):
+        self.flushbuf.fill_(1)
+
+    def run_step(self, evs):
+        """evs: list of (start, end) event pairs, one per sub-step (prefill, decode 0..S-1)."""
+        self.flush()
+        evs[0][0].record(self.stream)
+        self.prefill()
+        evs[0][1].record(self.stream)
+        for t in range(self.S):
+            self.flush()
+            evs[t + 1][0].record(self.stream)
+            self.decode(t)
+            evs[t + 1][1].record(self.stream)
+
+    def make_events(self):
+        E = self.torch.cuda.Event
+        return [(E(enable_timing=True), E(enable_timing=True)) for _ in range(self.S + 1)]
+
+    # ---- kernel-level profile (CUDA events the library records between its kernels) ----
+    def profile(self, steps=1):
+        torch = self.torch
+        n = steps * (self.S * 12 + 8)
+        events = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+        handles = (ctypes.c_void_p * n)(*[ctypes.c_void_p(e.cuda_event) for e in events])
+        ctx = []          # sub-step of each recorded event
+        lib = self.lib
+        lib.qsvd_profile_count.restype = ctypes.c_int32
+        lib.qsvd_profile_label.restype = ctypes.c_char_p
+        lib.qsvd_profile_events(handles, n)
+        try:
+            for _ in range(steps):
+                self.flush()
+                c0 = lib.qsvd_profile_count()
+                self.prefill()
+                ctx += [("prefill", None)] * (lib.qsvd_profile_count() - c0)
+                for t in range(self.S):
+                    self.flush()
+                    c0 = lib.qsvd_profile_count()
+                    self.decode(t)
+                    ctx += [("decode", t)] * (lib.qsvd_profile_count() - c0)
+            torch.cuda.synchronize()
+            cnt = lib.qsvd_profile_count()
+            labels = [lib.qsvd_profile_label(i).decode() for i in range(cnt)]
+        finally:
+            lib.qsvd_profile_events(None, 0)
+        launches = []
+        for i in range(1, cnt):
+            if labels[i] == "begin":
+                continue
+            launches.append((labels[i], ctx[i], events[i - 1].elapsed_time(events[i]) * 1e-3))
+        return launches
+
+    def alg_bytes(self, label, ctx):
+        """Minimal HBM bytes of one launch: every input read once, every output written once."""
+        s, B, P = self.wl.shape, self.B, self.P
+        d, r, H = s.d, s.r, s.H
+        tok = r if self.wl.lat_bits == 8 else r // 2 + 2 * (r // 128)
+        stok = 4 if self.wl.lat_bits == 8 else 0
+        T = B * P if ctx[0] == "prefill" else B
+        L = P + ctx[1] + 1 if ctx[0] == "decode" else 0
+        if label == "xquant":
+            return T * d * 2 + T * d + 4 * T
+        if label == "proj_dp4a":
+            return r * d + T * d + 4 * r + 4 * T + 4 * T * r
+        if label == "requant":
+            return 4 * T * r + T * (tok + stok) + 8 * T
+        if label == "qproj":
+            return r * d * 2 + B * (tok + stok) + 4 * B * d
+        if label == "qabsorb":
+            return r * d * 2 + 4 * B * d + 4 * B * H * r
+        if label == "attn_split":
+            ns = (L + 255) // 256
+            return B * L * (tok + stok) + 4 * B * H * r + 4 * B * ns * H * (r + 2)
+        if label == "combine_uv":
+            ns = (L + 255) // 256
+            return r * d * 2 + 4 * B * ns * H * (r + 2) + 4 * B * d
+        return 0
+
+    def step_roofline_bytes(self, t):
+        """Bytes one decode step must move (per the path's definition): cache read,
+        append, U_q/U_k/U_v, W_d codes and scales, x in, O out."""
+        s, B = self.wl.shape, self.B
+        d, r = s.d, s.r
+        tok = (r + 4) if self.wl.lat_bits == 8 else (r // 2 + 2 * (r // 128))
+        L = self.P + t + 1
+        return B * L * tok + B * tok + 3 * r * d * 2 + d * r + 4 * r + B * d * 2 + 4 * B * d
+
+    # ---- end to end through the public binding with host buffers ----
+    def e2e(self, steps, warmup):
+        torch, q, s = self.torch, self.q, self.wl.shape
+        hx_p = torch.empty(self.Xp.shape, dtype=torch.bfloat16, pin_memory=True)
+        hx_p.copy_(self.Xp.cpu())
+        hx_d = torch.empty(self.Xd.shape, dtype=torch.bfloat16, pin_memory=True)
+        hx_d.copy_(self.Xd.cpu())
+        hO = torch.empty((self.S, self.B, s.d), dtype=torch.float32, pin_memory=True)
+        dXp = torch.empty_like(self.Xp)
+        dXd = torch.empty((self.B, s.d), dtype=torch.bfloat16, device=self.dev)
+        E = torch.cuda.Event
+        tot = []
+        for it in range(warmup + steps):
+            evs = [(E(enable_timing=True), E(enable_timing=True)) for _ in range(self.S + 1)]
+            self.flush()
+            evs[0][0].record()
+            dXp.copy_(hx_p, non_blocking=True)
+            q.qsvd_latent_project(self.W, dXp, 1.0, self.wl.lat_bits, 1.0, dst=self.cache, dst_seq=self.pseq,
+                                  dst_pos=self.ppos, workspace=self.wsp)
+            evs[0][1].record()
+            for t in range(self.S):
+                self.flush()
+                evs[t + 1][0].record()
+                dXd.copy_(hx_d[t], non_blocking=True)
+                q.qsvd_latent_project(self.W, dXd, 1.0, self.wl.lat_bits, 1.0, dst=self.cache,
+                                      dst_seq=self.dseq, dst_pos=self.dpos[t], workspace=self.wsp)
+                q.qsvd_latent_decode_attn(self.cache, self.dlen[t], self.P + t + 1, *self.U, s.H, s.dh, self.O,
+                                          workspace=self.wsd)
+                hO[t].copy_(self.O, non_blocking=True)
+                evs[t + 1][1].record()
+            torch.cuda.synchronize()
+            if it >= warmup:
+                tot.append(sum(a.elapsed_time(b) for a, b in evs[1:]) * 1e-3)
+        dec_s = statistics.mean(tot)
+        h2d = self.B * self.P * s.d * 2 + self.S * self.B * s.d * 2
+        d2h = self.S * self.B * s.d * 4
+        return self.B * self.S / dec_s, h2d, d2h
+
+
+def run_native(args, rank, world, local_rank):
+    import torch
+    torch.cuda.set_device(local_rank)
+    wl = synthetic.WORKLOADS[WORKLOAD]
+    nb = NativeBench(wl, rank)
+    S = wl.decode_steps
+    hbm, _, peak_kind = peaks()
+
+    # warm-up
+    for _ in range(args.warmup):
+        nb.run_step(nb.make_events())
+    torch.cuda.synchronize()
+    step_events = [nb.make_events() for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    t_wall = time.perf_counter()
+    for k in range(args.steps):
+        nb.run_step(step_events[k])
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    t_wall = time.perf_counter() - t_wall
+    clk = clocks.stop()
+    pre = [step_events[k][0][0].elapsed_time(step_events[k][0][1]) * 1e-3 for k in range(args.steps)]
+    dec = [sum(a.elapsed_time(b) for a, b in step_events[k][1:]) * 1e-3 for k in range(args.steps)]
+    per_dec = [[step_events[k][t + 1][0].elapsed_time(step_events[k][t + 1][1]) * 1e-3 for t in range(S)]
+               for k in range(args.steps)]
+    dec_total, pre_total = sum(dec), sum(pre)
+    if world > 1:
+        tt = torch.tensor([dec_total, pre_total], dtype=torch.float64, device=nb.dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        dec_total, pre_total = float(tt[0]), float(tt[1])
+    dec_tokens = world * wl.B * S * args.steps
+    value = dec_tokens / dec_total
+    s = wl.shape
+    prefill_ops = 2 * wl.B * wl.prefill * s.d * s.r
+    prefill_tops = world * prefill_ops * args.steps / pre_total / 1e12
+    tok_bytes = (s.r + 4) if wl.lat_bits == 8 else (s.r // 2 + 2 * (s.r // 128))
+    cache_bytes = sum(wl.B * (wl.prefill + t + 1) * tok_bytes for t in range(S))
+    roof_s = sum(nb.step_roofline_bytes(t) for t in range(S)) / (hbm * 1e9)
+    step_frac = roof_s / statistics.mean(dec)
+
+    # kernel-level profile (separate pass of the same step) -> dominant kernel + roofline
+    launches = nb.profile(steps=1)
+    by = {}
+    for lab, ctx, dt in launches:
+        e = by.setdefault(lab, {"launches": 0, "time_s": 0.0, "bytes": 0})
+        e["launches"] += 1
+        e["time_s"] += dt
+        e["bytes"] += nb.alg_bytes(lab, ctx)
+    tot_t = sum(e["time_s"] for e in by.values())
+    dom = max(by, key=lambda k: by[k]["time_s"])
+    de = by[dom]
+    achieved = de["bytes"] / de["time_s"] / 1e9
+    kernels = {k: {"launches": v["launches"], "avg_us": round(v["time_s"] / v["launches"] * 1e6, 2),
+                   "share": round(v["time_s"] / tot_t, 4),
+                   "gbs": round(v["bytes"] / v["time_s"] / 1e9, 1)} for k, v in sorted(by.items())}
+    launches_per_step = len(launches)
+
+    e2e = None
+    if not args.no_e2e:
+        e2e_val, h2d, d2h = nb.e2e(steps=min(args.steps, 3), warmup=1)
+        if world > 1:
+            tt = torch.tensor([e2e_val], dtype=torch.float64, device=nb.dev)
+            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MIN)
+            e2e_val = float(tt[0]) * world
+        e2e = {"value": round(e2e_val, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h}
+
+    if rank != 0:
+        return
+    out = {
+        "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round((dec_total + pre_total) / args.steps * 1e3, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int8/fp32",
+        "data": "synthetic",
+        "config": {"workload": workload_desc(wl), "global_batch": world * wl.B,
+                   "seq_len": wl.tmax, "parallelism": f"replicas x{world} (one independent layer per GPU)",
+                   "l2": "flushed (256 MiB write) before the prefill and before every decode step; "
+                         "flushes outside the timed intervals"},
+        "secondary": {
+            "decode_ms_per_step": round(dec_total / args.steps * 1e3, 4),
+            "prefill_ms_per_step": round(pre_total / args.steps * 1e3, 4),
+            "decode_us_per_token_step": round(statistics.mean(sum(per_dec, [])) * 1e6, 3),
+            "prefill_tops": round(prefill_tops, 3),
+            "latent_cache_gbs": round(cache_bytes * args.steps * world / dec_total / 1e9, 2),
+            "decode_step_roofline_frac": round(step_frac, 4),
+            "decode_step_roofline_us": round(roof_s / S * 1e6, 3),
+            "wall_s_timed_region": round(t_wall, 3),
+            "kernels": kernels,
+        },
+        "roofline": {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
+                     "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": None,
+                     "peak_kind": peak_kind},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk,
+    }
+    if e2e:
+        out["e2e"] = e2e
+    if world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(wl, budget_s=15.0)
+    print(json.dumps(out), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (baseline leg and reference arm)
+# ---------------------------------------------------------------------------
+def _oracle_layer(wl, seed=0):
+    from oracle import pipeline
+    inp = synthetic.gen_layer(wl, seed=seed)
+    w = pipeline.prepare_weights(inp)
+    lay = pipeline.OracleLayer(wl.shape, w, wl.B, wl.tmax, wl.lat_bits)
+    for b in range(wl.B):
+        lay.prefill(b, inp.X_prefill[b])
+    return inp, w, lay
+
+
+def cpu_baseline(wl, budget_s=15.0):
+    """Decode tokens/s of the oracle on a bounded sample: prefill, then decode
+    steps until `budget_s` seconds of decode work (at most all steps)."""
+    inp, w, lay = _oracle_layer(wl)
+    t0 = time.perf_counter()
+    n = 0
+    while n < wl.decode_steps and time.perf_counter() - t0 < budget_s:
+        lay.decode_step(inp.X_decode[n])
+        n += 1
+    dt = time.perf_counter() - t0
+    return {"value": round(wl.B * n / dt, 2), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{n} of {wl.decode_steps} decode steps of {wl.name} after its full prefill "
+                      f"(numpy fp64, BLAS on all host cores)"}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    wl = synthetic.WORKLOADS[WORKLOAD]
+    inp, w, lay = _oracle_layer(wl)
+    per = 4                                   # decode steps per reference step
+    times = []
+    pos = 0
+    for k in range(args.warmup + args.steps):
+        if pos + per > wl.decode_steps:       # restart the decode from the prefilled cache
+            inp, w, lay = _oracle_layer(wl)
+            pos = 0
+        t0 = time.perf_counter()
+        for t in range(per):
+            lay.decode_step(inp.X_decode[pos + t])
+        dt = time.perf_counter() - t0
+        pos += per
+        if k >= args.warmup:
+            times.append(dt)
+    total = sum(times)
+    value = wl.B * per * args.steps / total
+    sample = f"{per} decode steps of {wl.name} per step (numpy fp64 oracle, BLAS on all host cores)"
+    out = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 3),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "config": {"workload": workload_desc(wl)},
+           "cpu_baseline": {"value": round(value, 2), "unit": "tokens/s", "cores": os.cpu_count(),
+                            "kind": "oracle", "sample": sample},
+           "e2e": {"value": round(value, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    try:
+        run_native(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,201 @@
+/*
+ * qsvd.h -- C ABI of the QSVD latent-attention hot path on GB300 (sm_103a).
+ *
+ * QSVD (arxiv 2510.16292) factors the concatenated query/key/value weight
+ * [W_q, W_k, W_v] of an attention layer into one shared down-projection W_d
+ * (E x r) and three up-projections U_q, U_k, U_v (r x E each) (Sec. 3.1,
+ * Eq. 2-4).  Only the latent C = X W_d of each token is cached; keys and
+ * values are recomputed from it as K = C U_k, V = C U_v (Eq. 5).  With
+ * quantization, C is computed from int8 X and int8 W_d and is itself stored
+ * in low precision (Eq. 11-12).
+ *
+ * This library implements, on the caller's CUDA stream:
+ *   qsvd_quantize_weight     offline per-channel int8 RTN of W_d (Sec. 4 setup)
+ *   qsvd_latent_project      C = Q(X) Q(W_d), requantized per token (Eq. 11-12)
+ *   qsvd_cache_append        store latent rows in the latent cache (Fig. 2(f))
+ *   qsvd_latent_decode_attn  one decode step of attention over that cache (Eq. 5)
+ *
+ * Conventions shared by every entry point:
+ *   - Row-vector convention Y = X W, as in the paper.  E = d = H * dh.
+ *   - Every pointer is device memory owned by the caller unless stated
+ *     otherwise.  The library never allocates device memory; scratch space is
+ *     a caller-provided workspace whose size the *_workspace_bytes calls give.
+ *   - Calls are asynchronous on `stream` and never synchronize it, except
+ *     qsvd_check.  A return of QSVD_OK means the work was enqueued.
+ *   - bf16 buffers are passed as uint16_t bit patterns.
+ *   - Every device pointer must be 16-byte aligned; row lengths in bytes must
+ *     be multiples of 16.
+ *   - Errors: argument problems are detected on the host before anything is
+ *     enqueued and return a negative status; the message of the last failure
+ *     on the calling thread is in qsvd_last_error().  Out-of-range cache
+ *     positions and expired bounded waits are detected on the device: the
+ *     offending write is skipped, a device error word is set, and qsvd_check
+ *     reports it.  Nothing traps or aborts.
+ *
+ * Quantizer (all entry points; the paper says per-token symmetric for
+ * activations, RTN per-channel symmetric for weights, and fixes no
+ * arithmetic, so this is the library's definition):
+ *   m = max|v| over the row (or channel, or int4 group);
+ *   s = fp32(fp32(clip * m) / q_max),  q_max = 127 (int8) or 7 (int4);
+ *   code = clamp(round_half_even(fp32(v / s)), -q_max, q_max), IEEE division;
+ *   s == 0 gives all-zero codes.  int4 scales are fp16: s is rounded to fp16
+ *   (nearest even, saturated at 65504) and the codes divide by that value.
+ */
+#ifndef QSVD_H_
+#define QSVD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define QSVD_OK             0
+#define QSVD_EINVAL        -1  /* null pointer, bad shape, misaligned pointer */
+#define QSVD_EUNSUPPORTED  -2  /* device is not sm_103, or a shape the kernels do not cover */
+#define QSVD_ECUDA         -3  /* a CUDA runtime call or launch failed */
+#define QSVD_ETIMEOUT      -4  /* a bounded device-side wait expired (from qsvd_check) */
+#define QSVD_ERANGE        -5  /* a cache position or sequence index out of range */
+#define QSVD_ENOSPC        -6  /* workspace smaller than the *_workspace_bytes figure */
+
+/*
+ * Quantized shared down-projection W^d_qkv (Eq. 3), stored per output
+ * channel.  codes[j * d + k] is the int8 code of W_d[k, j] (row j of `codes`
+ * is column j of W_d: the reduction dimension d is contiguous).  scale[j] is
+ * its fp32 scale.  codes_bf16 holds the same integer codes as bf16 bit
+ * patterns in the same layout; it is the tensor-core operand of the prefill
+ * GEMM (every int8 code is exact in bf16).  All three are produced by
+ * qsvd_quantize_weight.  Requirements: d % 64 == 0, r % 16 == 0.
+ */
+typedef struct qsvd_down_weight {
+    const int8_t   *codes;       /* [r, d] */
+    const uint16_t *codes_bf16;  /* [r, d] */
+    const float    *scale;       /* [r]    */
+    int32_t d;
+    int32_t r;
+} qsvd_down_weight;
+
+/*
+ * Latent cache of one layer (Fig. 2(f): the buffered C_qkv, eta = r L per
+ * sequence), laid out [B, Tmax, ...]:
+ *   bits == 8: codes int8 [B, Tmax, r];  scales fp32 [B, Tmax] (one per token)
+ *   bits == 4: codes uint8 [B, Tmax, r/2], element 2i in the low nibble of
+ *              byte i, two's complement;  scales fp16 [B, Tmax, r/128]
+ *              (one per token and 128-channel group).  Requires r % 128 == 0.
+ */
+typedef struct qsvd_cache {
+    void   *codes;
+    void   *scales;
+    int32_t bits;
+    int32_t B;
+    int32_t Tmax;
+    int32_t r;
+} qsvd_cache;
+
+/*
+ * Offline weight preparation (Sec. 4 setup: RTN, per-channel symmetric, with
+ * a clipping ratio `clip` in (0, 1]).
+ *   W_d        fp32 [d, r] row-major (W_d[k, j] at k * r + j).
+ *   codes      int8 [r, d] out;  codes_bf16 bf16 [r, d] out (may be NULL);
+ *   scale      fp32 [r] out.
+ */
+int qsvd_quantize_weight(const float *W_d, int32_t d, int32_t r, float clip,
+                         int8_t *codes, uint16_t *codes_bf16, float *scale,
+                         cudaStream_t stream);
+
+/*
+ * Quantized joint down-projection with the latent requantization fused
+ * behind it (Eq. 12 with H1 = H2 = I, then Eq. 11's Q(C_qkv)):
+ *   1. X [T, d] bf16 is quantized per token to int8 (clip `act_clip`);
+ *   2. acc[t, j] = sum_k xq[t, k] * codes[j, k]    exact int32;
+ *   3. c[t, j] = fp32(fp32(fp32(acc) * s_x[t]) * scale[j])   (no FMA);
+ *   4. c[t, :] is requantized per token to `lat_bits` (8: one fp32 scale per
+ *      token; 4: one fp16 scale per 128 channels), clip `lat_clip`.
+ * Destinations (at least one must be given):
+ *   lat_codes/lat_scales  token-major: int8 [T, r] + fp32 [T], or packed
+ *                         uint8 [T, r/2] + fp16 [T, r/128];
+ *   dst/dst_seq/dst_pos   fused cache append: row t goes to sequence
+ *                         dst_seq[t] at position dst_pos[t] (device int32
+ *                         arrays of length T); dst->bits must equal lat_bits.
+ * Optional intermediates for inspection (NULL skips the write):
+ *   xq_out int8 [T, d], xs_out fp32 [T], acc_out int32 [T, r].
+ * workspace: at least qsvd_project_workspace_bytes(T, d, r) bytes, 256-byte
+ * aligned.  T may be 0 (nothing is enqueued).
+ */
+int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
+                        float act_clip, int32_t lat_bits, float lat_clip,
+                        void *lat_codes, void *lat_scales,
+                        const qsvd_cache *dst, const int32_t *dst_seq, const int32_t *dst_pos,
+                        int8_t *xq_out, float *xs_out, int32_t *acc_out,
+                        void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r);
+
+/*
+ * Latent cache append (the store of Fig. 2(f)): row i of the token-major
+ * latent (codes + scales, in the cache's format) is copied to sequence
+ * seq[i], position pos[i].  seq and pos are device int32 [n].  Rows whose
+ * (seq, pos) fall outside [0, B) x [0, Tmax) are skipped and flag QSVD_ERANGE
+ * for qsvd_check.
+ */
+int qsvd_cache_append(const qsvd_cache *cache, const int32_t *seq, const int32_t *pos,
+                      int64_t n, const void *lat_codes, const void *lat_scales,
+                      cudaStream_t stream);
+
+/*
+ * One decode step of attention over the latent cache (Eq. 5 and the decode
+ * remark after it).  For every sequence b with L = seq_len[b] cached tokens
+ * (the current token, already appended, at position L-1) and every head h
+ * (columns h*dh .. h*dh+dh-1 of each up-projection):
+ *   c_t  = dequantized latent of token t;     q_h = c_{L-1} U_q[:, h]
+ *   o_h  = softmax_t( (c_t U_k[:, h]) . q_h * softmax_scale ) . (c_t U_v[:, h])
+ * computed without forming K or V: U_k is absorbed into the query
+ * (qt_h = U_k[:, h] q_h, scores c_t . qt_h) and U_v is applied after the
+ * softmax-weighted sum of latent rows.
+ *   seq_len      device int32 [B], 1 <= seq_len[b] <= max_seq_len <= Tmax;
+ *   max_seq_len  host-side bound used to size the launch;
+ *   U_q, U_k, U_v  bf16 [r, H*dh] row-major;
+ *   O            fp32 [B, H*dh] out.
+ * workspace: qsvd_decode_workspace_bytes(B, max_seq_len, r, H, dh) bytes.
+ * Requirements: dh in {64, 128}; r % 16 == 0 and r <= 3072.
+ */
+int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int32_t max_seq_len,
+                            const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v,
+                            int32_t H, int32_t dh, float softmax_scale, float *O,
+                            void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+size_t qsvd_decode_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t r, int32_t H, int32_t dh);
+
+/*
+ * Synchronizes `stream`, then reads and clears the device error word.
+ * Returns QSVD_OK, QSVD_ERANGE, QSVD_ETIMEOUT or QSVD_ECUDA.
+ */
+int qsvd_check(cudaStream_t stream);
+
+/* Message of the last failure on the calling thread ("" if none). */
+const char *qsvd_last_error(void);
+
+/*
+ * Kernel-level timing for benchmarks (not part of the paper's method).
+ * qsvd_profile_events(events, n) hands the calling thread an array of n
+ * caller-created cudaEvent_t handles (passed as void*).  From then on every
+ * entry point records the next event on its stream once before its first
+ * kernel (label "begin") and once after each kernel it launches (label = the
+ * kernel's name), until the array is full.  The elapsed time between event
+ * i-1 and event i is the duration of kernel i whenever label i is not
+ * "begin".  qsvd_profile_events(NULL, 0) switches recording off.  Nothing is
+ * recorded while profiling is off.
+ */
+int qsvd_profile_events(void **events, int32_t capacity);
+int32_t qsvd_profile_count(void);
+const char *qsvd_profile_label(int32_t i);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int qsvd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* QSVD_H_ */

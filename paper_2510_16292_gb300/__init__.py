@@ -1,0 +1,205 @@
+"""Python binding of the QSVD latent-attention library (include/qsvd.h).
+
+Argument marshalling only: every function below forwards device pointers of
+torch tensors and the current CUDA stream to the C ABI of ``libqsvd.so`` and
+raises ``QsvdError`` on a non-zero status.  All arithmetic runs in the CUDA
+kernels; there is no host fallback.  Importing this package fails loudly if
+the library has not been built (``python paper_2510_16292_gb300/build.py``).
+
+Names follow the C ABI: ``qsvd_quantize_weight``, ``qsvd_latent_project``,
+``qsvd_cache_append``, ``qsvd_latent_decode_attn``, ``qsvd_check``, plus the
+workspace-size queries.  ``DownWeight`` and ``LatentCache`` hold the torch
+tensors behind the two C structs.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import math
+import os
+from typing import Optional
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_build", "libqsvd.so")
+if not os.path.exists(_LIB_PATH):
+    raise ImportError(f"QSVD CUDA library not built ({_LIB_PATH} missing); "
+                      "run `python paper_2510_16292_gb300/build.py`")
+_lib = ctypes.CDLL(_LIB_PATH)
+
+QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
+QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
+EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspace_bytes",
+           "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
+           "qsvd_check", "qsvd_last_error", "qsvd_version")
+
+
+class QsvdError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"qsvd status {status}: {msg}")
+        self.status = status
+
+
+class _DownWeight(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_void_p), ("codes_bf16", ctypes.c_void_p), ("scale", ctypes.c_void_p),
+                ("d", ctypes.c_int32), ("r", ctypes.c_int32)]
+
+
+class _Cache(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p), ("bits", ctypes.c_int32),
+                ("B", ctypes.c_int32), ("Tmax", ctypes.c_int32), ("r", ctypes.c_int32)]
+
+
+_vp, _i32, _i64, _f32, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+_lib.qsvd_quantize_weight.argtypes = [_vp, _i32, _i32, _f32, _vp, _vp, _vp, _vp]
+_lib.qsvd_latent_project.argtypes = [ctypes.POINTER(_DownWeight), _vp, _i64, _f32, _i32, _f32, _vp, _vp,
+                                     ctypes.POINTER(_Cache), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+_lib.qsvd_project_workspace_bytes.argtypes = [_i64, _i32, _i32]
+_lib.qsvd_project_workspace_bytes.restype = _sz
+_lib.qsvd_cache_append.argtypes = [ctypes.POINTER(_Cache), _vp, _vp, _i64, _vp, _vp, _vp]
+_lib.qsvd_latent_decode_attn.argtypes = [ctypes.POINTER(_Cache), _vp, _i32, _vp, _vp, _vp, _i32, _i32, _f32,
+                                         _vp, _vp, _sz, _vp]
+_lib.qsvd_decode_workspace_bytes.argtypes = [_i32, _i32, _i32, _i32, _i32]
+_lib.qsvd_decode_workspace_bytes.restype = _sz
+_lib.qsvd_check.argtypes = [_vp]
+_lib.qsvd_last_error.restype = ctypes.c_char_p
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("device tensor expected")
+    if not t.is_contiguous():
+        raise ValueError("contiguous tensor expected")
+    return t.data_ptr()
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def _check(status: int):
+    if status != QSVD_OK:
+        raise QsvdError(status, _lib.qsvd_last_error().decode(errors="replace"))
+
+
+@dataclasses.dataclass
+class DownWeight:
+    """Quantized W_d: codes int8 [r, d], codes_bf16 bf16 [r, d], scale fp32 [r]."""
+    codes: torch.Tensor
+    codes_bf16: torch.Tensor
+    scale: torch.Tensor
+
+    @property
+    def d(self):
+        return self.codes.shape[1]
+
+    @property
+    def r(self):
+        return self.codes.shape[0]
+
+    def _c(self):
+        return _DownWeight(_ptr(self.codes), _ptr(self.codes_bf16), _ptr(self.scale), self.d, self.r)
+
+
+@dataclasses.dataclass
+class LatentCache:
+    """Latent cache tensors: int8 codes [B, Tmax, r] + fp32 scales [B, Tmax],
+    or packed uint8 codes [B, Tmax, r/2] + fp16 scales [B, Tmax, r/128]."""
+    codes: torch.Tensor
+    scales: torch.Tensor
+    bits: int
+    B: int
+    Tmax: int
+    r: int
+
+    @staticmethod
+    def empty(B: int, Tmax: int, r: int, bits: int, device="cuda") -> "LatentCache":
+        if bits == 8:
+            codes = torch.zeros((B, Tmax, r), dtype=torch.int8, device=device)
+            scales = torch.zeros((B, Tmax), dtype=torch.float32, device=device)
+        else:
+            codes = torch.zeros((B, Tmax, r // 2), dtype=torch.uint8, device=device)
+            scales = torch.zeros((B, Tmax, r // 128), dtype=torch.float16, device=device)
+        return LatentCache(codes, scales, bits, B, Tmax, r)
+
+    def _c(self):
+        return _Cache(_ptr(self.codes), _ptr(self.scales), self.bits, self.B, self.Tmax, self.r)
+
+    def nbytes_per_token(self) -> int:
+        return self.r if self.bits == 8 else self.r // 2 + 2 * (self.r // 128)
+
+
+def qsvd_quantize_weight(W_d: torch.Tensor, clip: float = 1.0, stream=None) -> DownWeight:
+    """W_d fp32 [d, r] -> DownWeight (per-output-channel int8 RTN)."""
+    d, r = W_d.shape
+    dev = W_d.device
+    codes = torch.empty((r, d), dtype=torch.int8, device=dev)
+    codes_bf16 = torch.empty((r, d), dtype=torch.bfloat16, device=dev)
+    scale = torch.empty((r,), dtype=torch.float32, device=dev)
+    _check(_lib.qsvd_quantize_weight(_ptr(W_d), d, r, clip, _ptr(codes), _ptr(codes_bf16), _ptr(scale),
+                                     _stream(stream)))
+    return DownWeight(codes, codes_bf16, scale)
+
+
+def qsvd_project_workspace_bytes(T: int, d: int, r: int) -> int:
+    return int(_lib.qsvd_project_workspace_bytes(T, d, r))
+
+
+def qsvd_decode_workspace_bytes(B: int, max_seq_len: int, r: int, H: int, dh: int) -> int:
+    return int(_lib.qsvd_decode_workspace_bytes(B, max_seq_len, r, H, dh))
+
+
+def qsvd_latent_project(W: DownWeight, X: torch.Tensor, act_clip: float = 1.0, lat_bits: int = 8,
+                        lat_clip: float = 1.0, lat_codes=None, lat_scales=None,
+                        dst: Optional[LatentCache] = None, dst_seq=None, dst_pos=None,
+                        xq_out=None, xs_out=None, acc_out=None, workspace=None, stream=None) -> None:
+    T = X.shape[0]
+    if workspace is None:
+        workspace = torch.empty(max(1, qsvd_project_workspace_bytes(T, W.d, W.r)), dtype=torch.uint8,
+                                device=X.device)
+    cw = W._c()
+    cc = dst._c() if dst is not None else None
+    _check(_lib.qsvd_latent_project(ctypes.byref(cw), _ptr(X), T, act_clip, lat_bits, lat_clip,
+                                    _ptr(lat_codes), _ptr(lat_scales),
+                                    ctypes.byref(cc) if cc is not None else None,
+                                    _ptr(dst_seq), _ptr(dst_pos), _ptr(xq_out), _ptr(xs_out), _ptr(acc_out),
+                                    _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def qsvd_cache_append(cache: LatentCache, seq: torch.Tensor, pos: torch.Tensor, lat_codes: torch.Tensor,
+                      lat_scales: torch.Tensor, stream=None) -> None:
+    cc = cache._c()
+    _check(_lib.qsvd_cache_append(ctypes.byref(cc), _ptr(seq), _ptr(pos), seq.numel(), _ptr(lat_codes),
+                                  _ptr(lat_scales), _stream(stream)))
+
+
+def qsvd_latent_decode_attn(cache: LatentCache, seq_len: torch.Tensor, max_seq_len: int, U_q, U_k, U_v,
+                            H: int, dh: int, O: torch.Tensor, softmax_scale: Optional[float] = None,
+                            workspace=None, stream=None) -> None:
+    if softmax_scale is None:
+        softmax_scale = 1.0 / math.sqrt(dh)
+    if workspace is None:
+        workspace = torch.empty(qsvd_decode_workspace_bytes(cache.B, max_seq_len, cache.r, H, dh),
+                                dtype=torch.uint8, device=O.device)
+    cc = cache._c()
+    _check(_lib.qsvd_latent_decode_attn(ctypes.byref(cc), _ptr(seq_len), max_seq_len, _ptr(U_q), _ptr(U_k),
+                                        _ptr(U_v), H, dh, softmax_scale, _ptr(O), _ptr(workspace),
+                                        workspace.numel(), _stream(stream)))
+
+
+def qsvd_check(stream=None) -> int:
+    """Synchronize the stream and return the device status (raises on error)."""
+    st = _lib.qsvd_check(_stream(stream))
+    _check(st)
+    return st
+
+
+def qsvd_version() -> int:
+    return int(_lib.qsvd_version())

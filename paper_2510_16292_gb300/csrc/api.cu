@@ -1,0 +1,261 @@
+// C ABI of the QSVD latent-attention path (declared in include/qsvd.h):
+// argument validation, workspace carving and kernel launch order.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <vector>
+
+#include "launch.h"
+#include "qsvd.h"
+
+namespace qsvd {
+
+// Device error word: bit kErrRange / kErrTimeout set by kernels, read and
+// cleared by qsvd_check.  It is a module-scope variable (no allocation).
+__device__ int g_error_word;
+
+namespace {
+
+thread_local char g_msg[512];
+
+int fail(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_msg, sizeof(g_msg), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char *where) {
+    return fail(QSVD_ECUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+constexpr int kMaxDevices = 64;
+int g_arch_ok[kMaxDevices];          // 0 unknown, 1 sm_103, -1 other
+int *g_err_ptr[kMaxDevices];
+
+// Checks that the current device is an sm_103 part and returns the address
+// of its error word.
+int device_setup(int **err) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(QSVD_EUNSUPPORTED, "device index %d", dev);
+    if (g_arch_ok[dev] == 0) {
+        int major = 0, minor = 0;
+        e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+        void *p = nullptr;
+        if (major == 10 && minor == 3) {
+            e = cudaGetSymbolAddress(&p, g_error_word);
+            if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(error word)");
+            g_err_ptr[dev] = static_cast<int *>(p);
+            g_arch_ok[dev] = 1;
+        } else {
+            g_arch_ok[dev] = -1;
+        }
+    }
+    if (g_arch_ok[dev] < 0)
+        return fail(QSVD_EUNSUPPORTED, "this library is built for sm_103 (GB300) only");
+    *err = g_err_ptr[dev];
+    return QSVD_OK;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+int check_cache(const qsvd_cache *c) {
+    if (!c || !c->codes || !c->scales) return fail(QSVD_EINVAL, "cache: null pointer");
+    if (!aligned16(c->codes) || !aligned16(c->scales)) return fail(QSVD_EINVAL, "cache: pointers must be 16-byte aligned");
+    if (c->bits != 8 && c->bits != 4) return fail(QSVD_EINVAL, "cache: bits must be 8 or 4");
+    if (c->B <= 0 || c->Tmax <= 0 || c->r <= 0) return fail(QSVD_EINVAL, "cache: B, Tmax, r must be positive");
+    if (c->r % 16) return fail(QSVD_EINVAL, "cache: r must be a multiple of 16");
+    if (c->bits == 4 && c->r % 128) return fail(QSVD_EUNSUPPORTED, "cache: int4 needs r %% 128 == 0");
+    return QSVD_OK;
+}
+
+CacheView view(const qsvd_cache *c) { return CacheView{c->codes, c->scales, c->bits, c->B, c->Tmax, c->r}; }
+
+// Profiling state of the calling thread (see qsvd_profile_events).
+thread_local cudaEvent_t *t_prof_events = nullptr;
+thread_local int t_prof_capacity = 0;
+thread_local std::vector<const char *> t_prof_labels;
+
+}  // namespace
+
+void prof_mark(cudaStream_t s, const char *label) {
+    if (!t_prof_events || int(t_prof_labels.size()) >= t_prof_capacity) return;
+    if (cudaEventRecord(t_prof_events[t_prof_labels.size()], s) == cudaSuccess) t_prof_labels.push_back(label);
+}
+
+}  // namespace qsvd
+
+using namespace qsvd;
+
+extern "C" {
+
+const char *qsvd_last_error(void) { return g_msg; }
+
+int qsvd_version(void) { return 100; }
+
+int qsvd_profile_events(void **events, int32_t capacity) {
+    t_prof_labels.clear();
+    if (!events || capacity <= 0) {
+        t_prof_events = nullptr;
+        t_prof_capacity = 0;
+        return QSVD_OK;
+    }
+    t_prof_events = reinterpret_cast<cudaEvent_t *>(events);
+    t_prof_capacity = capacity;
+    t_prof_labels.reserve(size_t(capacity));
+    return QSVD_OK;
+}
+
+int32_t qsvd_profile_count(void) { return int32_t(t_prof_labels.size()); }
+
+const char *qsvd_profile_label(int32_t i) {
+    return (i >= 0 && i < int32_t(t_prof_labels.size())) ? t_prof_labels[size_t(i)] : "";
+}
+
+int qsvd_check(cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    cudaError_t e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    int word = 0;
+    e = cudaMemcpyFromSymbol(&word, g_error_word, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "read error word");
+    if (word) {
+        const int zero = 0;
+        e = cudaMemcpyToSymbol(g_error_word, &zero, sizeof(int));
+        if (e != cudaSuccess) return cuda_fail(e, "clear error word");
+    }
+    if (word & kErrTimeout) return fail(QSVD_ETIMEOUT, "a bounded device wait expired");
+    if (word & kErrRange) return fail(QSVD_ERANGE, "a cache position, sequence index or length was out of range");
+    g_msg[0] = 0;
+    return QSVD_OK;
+}
+
+int qsvd_quantize_weight(const float *W_d, int32_t d, int32_t r, float clip, int8_t *codes,
+                         uint16_t *codes_bf16, float *scale, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!W_d || !codes || !scale) return fail(QSVD_EINVAL, "quantize_weight: null pointer");
+    if (d <= 0 || r <= 0) return fail(QSVD_EINVAL, "quantize_weight: d and r must be positive");
+    if (!(clip > 0.0f && clip <= 1.0f)) return fail(QSVD_EINVAL, "quantize_weight: clip must lie in (0, 1]");
+    prof_mark(stream, "begin");
+    cudaError_t e = launch_quantize_weight(W_d, d, r, clip, codes, codes_bf16, scale, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "quantize_weight launch");
+}
+
+size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r) {
+    if (T < 0 || d <= 0 || r <= 0) return 0;
+    return align256(size_t(T) * d) +            // int8 codes of X
+           align256(size_t(T) * 4) +            // s_x
+           align256(size_t(T) * r * 4);         // dequantized latent c_hat
+}
+
+int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T, float act_clip,
+                        int32_t lat_bits, float lat_clip, void *lat_codes, void *lat_scales,
+                        const qsvd_cache *dst, const int32_t *dst_seq, const int32_t *dst_pos,
+                        int8_t *xq_out, float *xs_out, int32_t *acc_out, void *workspace,
+                        size_t workspace_bytes, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!W || !W->codes || !W->scale) return fail(QSVD_EINVAL, "latent_project: null weight pointer");
+    if (T < 0) return fail(QSVD_EINVAL, "latent_project: T < 0");
+    const int d = W->d, r = W->r;
+    if (d <= 0 || r <= 0 || d % 64 || r % 16) return fail(QSVD_EINVAL, "latent_project: need d %% 64 == 0 and r %% 16 == 0");
+    if (r > 4096) return fail(QSVD_EUNSUPPORTED, "latent_project: r > 4096");
+    if (lat_bits != 8 && lat_bits != 4) return fail(QSVD_EINVAL, "latent_project: lat_bits must be 8 or 4");
+    if (lat_bits == 4 && r % 128) return fail(QSVD_EUNSUPPORTED, "latent_project: int4 needs r %% 128 == 0");
+    if (!(act_clip > 0.0f && act_clip <= 1.0f) || !(lat_clip > 0.0f && lat_clip <= 1.0f))
+        return fail(QSVD_EINVAL, "latent_project: clip ratios must lie in (0, 1]");
+    const bool tok = lat_codes != nullptr || lat_scales != nullptr;
+    if (tok && (!lat_codes || !lat_scales)) return fail(QSVD_EINVAL, "latent_project: give both lat_codes and lat_scales");
+    if (!tok && !dst) return fail(QSVD_EINVAL, "latent_project: no destination for the latent");
+    if (dst) {
+        if ((st = check_cache(dst))) return st;
+        if (dst->bits != lat_bits || dst->r != r) return fail(QSVD_EINVAL, "latent_project: cache format differs");
+        if (!dst_seq || !dst_pos) return fail(QSVD_EINVAL, "latent_project: dst_seq/dst_pos required with dst");
+    }
+    if (T == 0) return QSVD_OK;
+    if (!X) return fail(QSVD_EINVAL, "latent_project: X is null");
+    const void *ptrs[] = {X, W->codes, W->scale, lat_codes, lat_scales, xq_out, xs_out, acc_out, workspace};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(QSVD_EINVAL, "latent_project: pointers must be 16-byte aligned");
+    const size_t need = qsvd_project_workspace_bytes(T, d, r);
+    if (!workspace || workspace_bytes < need)
+        return fail(QSVD_ENOSPC, "latent_project: workspace needs %zu bytes", need);
+
+    char *wsp = static_cast<char *>(workspace);
+    int8_t *xq = xq_out ? xq_out : reinterpret_cast<int8_t *>(wsp);
+    wsp += align256(size_t(T) * d);
+    float *xs = xs_out ? xs_out : reinterpret_cast<float *>(wsp);
+    wsp += align256(size_t(T) * 4);
+    float *c_hat = reinterpret_cast<float *>(wsp);
+
+    prof_mark(stream, "begin");
+    cudaError_t e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
+    e = launch_proj_dp4a(xq, T, d, W->codes, W->scale, xs, r, c_hat, acc_out, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "projection launch");
+    CacheView dv{};
+    if (dst) dv = view(dst);
+    e = launch_requant(c_hat, T, r, lat_bits, lat_clip, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
+                       dst_pos, err, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "requant launch");
+    return QSVD_OK;
+}
+
+int qsvd_cache_append(const qsvd_cache *cache, const int32_t *seq, const int32_t *pos, int64_t n,
+                      const void *lat_codes, const void *lat_scales, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if ((st = check_cache(cache))) return st;
+    if (n < 0) return fail(QSVD_EINVAL, "cache_append: n < 0");
+    if (n == 0) return QSVD_OK;
+    if (!seq || !pos || !lat_codes || !lat_scales) return fail(QSVD_EINVAL, "cache_append: null pointer");
+    if (!aligned16(lat_codes)) return fail(QSVD_EINVAL, "cache_append: lat_codes must be 16-byte aligned");
+    prof_mark(stream, "begin");
+    cudaError_t e = launch_append(view(cache), seq, pos, n, lat_codes, lat_scales, err, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "cache_append launch");
+}
+
+size_t qsvd_decode_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t r, int32_t H, int32_t dh) {
+    if (B <= 0 || max_seq_len <= 0 || r <= 0 || H <= 0 || dh <= 0) return 0;
+    return decode_workspace_bytes(B, max_seq_len, r, H, dh);
+}
+
+int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int32_t max_seq_len,
+                            const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v, int32_t H,
+                            int32_t dh, float softmax_scale, float *O, void *workspace, size_t workspace_bytes,
+                            cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if ((st = check_cache(cache))) return st;
+    if (!seq_len || !U_q || !U_k || !U_v || !O) return fail(QSVD_EINVAL, "decode_attn: null pointer");
+    if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "decode_attn: dh must be 64 or 128");
+    if (H <= 0) return fail(QSVD_EINVAL, "decode_attn: H must be positive");
+    if (cache->r > 3072) return fail(QSVD_EUNSUPPORTED, "decode_attn: r > 3072");
+    if (max_seq_len < 1 || max_seq_len > cache->Tmax) return fail(QSVD_EINVAL, "decode_attn: max_seq_len outside [1, Tmax]");
+    const void *ptrs[] = {U_q, U_k, U_v, O, workspace};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(QSVD_EINVAL, "decode_attn: pointers must be 16-byte aligned");
+    const size_t need = qsvd_decode_workspace_bytes(cache->B, max_seq_len, cache->r, H, dh);
+    if (!workspace || workspace_bytes < need)
+        return fail(QSVD_ENOSPC, "decode_attn: workspace needs %zu bytes", need);
+    DecodeArgs a{view(cache), seq_len, max_seq_len, U_q, U_k, U_v, H, dh, softmax_scale, O};
+    prof_mark(stream, "begin");
+    cudaError_t e = launch_decode(a, workspace, workspace_bytes, err, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "decode_attn launch");
+}
+
+}  // extern "C"

@@ -1,0 +1,71 @@
+// Host-side launchers of the QSVD kernels (internal to the library; the
+// public surface is include/qsvd.h).  Every launcher only enqueues work on
+// `stream` and returns the launch status.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace qsvd {
+
+// Bits of the device error word (read and cleared by qsvd_check).
+enum : int { kErrRange = 1, kErrTimeout = 2 };
+
+// Plain description of a latent cache (mirrors qsvd_cache).
+struct CacheView {
+    void *codes;
+    void *scales;
+    int bits;
+    int B;
+    int Tmax;
+    int r;
+};
+
+// Profiling marker: when the calling thread has enabled profiling
+// (qsvd_profile_events), records the next caller-provided event on `s` and
+// remembers `label`; otherwise does nothing.  Every launcher calls it right
+// after each kernel launch, and each entry point once before its first one.
+void prof_mark(cudaStream_t s, const char *label);
+
+// Per-token int8 quantization of X [T, d] bf16 (a1).
+cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip,
+                          int8_t *xq, uint16_t *xq_bf16, float *xs, cudaStream_t s);
+
+// Per-output-channel int8 RTN of W_d [d, r] fp32 -> codes [r, d] (+ bf16 image).
+cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int8_t *codes,
+                                   uint16_t *codes_bf16, float *scale, cudaStream_t s);
+
+// Exact int8 GEMM on the CUDA cores (dp4a) with the dequant epilogue (a2, a3 first half):
+// c_hat[t, j] = (fp32(acc) * xs[t]) * ws[j].
+cudaError_t launch_proj_dp4a(const int8_t *xq, int64_t T, int d, const int8_t *wcodes,
+                             const float *ws, const float *xs, int r, float *c_hat,
+                             int32_t *acc_out, cudaStream_t s);
+
+// Per-token requantization of c_hat [T, r] into the latent format (a3 second
+// half), written token-major and/or into the cache (a4).
+cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float clip,
+                           void *lat_codes, void *lat_scales, const CacheView *dst,
+                           const int32_t *dst_seq, const int32_t *dst_pos, int *err,
+                           cudaStream_t s);
+
+// Copy token-major latent rows into the cache (a4).
+cudaError_t launch_append(const CacheView &c, const int32_t *seq, const int32_t *pos, int64_t n,
+                          const void *lat_codes, const void *lat_scales, int *err,
+                          cudaStream_t s);
+
+// Decode attention (a5-a8).
+struct DecodeArgs {
+    CacheView cache;
+    const int32_t *seq_len;
+    int max_seq_len;
+    const uint16_t *U_q, *U_k, *U_v;
+    int H, dh;
+    float softmax_scale;
+    float *O;
+};
+size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
+cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *err,
+                          cudaStream_t s);
+
+}  // namespace qsvd

@@ -1,0 +1,244 @@
+// Quantization, requantization and cache-append kernels.
+//
+//   xquant_kernel       a1: per-token symmetric int8 RTN of X (Sec. 4 setup;
+//                       Q(X H1^T) of Eq. 12 with H1 = I).
+//   weight_quant_kernel offline per-output-channel int8 RTN of W_d.
+//   requant_kernel      a3/a4: Eq. 11's Q(C_qkv), per token (int8) or per
+//                       128-channel group (int4), written token-major and/or
+//                       straight into the latent cache.
+//   append_kernel       a4: latent rows -> cache slots.
+#include "common.cuh"
+#include "launch.h"
+
+namespace qsvd {
+
+// ---------------------------------------------------------------------------
+// a1: one CTA per token row.  The row is staged in shared memory as fp32
+// (bf16 -> fp32 is exact), reduced to its absmax, then quantized.
+// ---------------------------------------------------------------------------
+constexpr int kXqThreads = 256;
+
+__global__ void __launch_bounds__(kXqThreads)
+xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int8_t *__restrict__ xq,
+              uint16_t *__restrict__ xq_bf16, float *__restrict__ xs) {
+    extern __shared__ float row[];
+    __shared__ float red[kXqThreads / 32];
+    const int64_t t = blockIdx.x;
+    const uint16_t *x = X + t * d;
+    float m = 0.0f;
+    for (int i = threadIdx.x * 8; i < d; i += kXqThreads * 8) {
+        float f[8];
+        unpack8_bf16(*reinterpret_cast<const uint4 *>(x + i), f);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            row[i + e] = f[e];
+            m = fmaxf(m, fabsf(f[e]));
+        }
+    }
+    m = block_max<kXqThreads>(m, red);
+    const float s = quant_scale(m, clip, 127.0f);
+    for (int i = threadIdx.x * 8; i < d; i += kXqThreads * 8) {
+        uint32_t packed[2] = {0u, 0u};
+        uint32_t bfw[4];
+#pragma unroll
+        for (int e = 0; e < 8; e += 2) {
+            const int c0 = quant_code(row[i + e], s, 127);
+            const int c1 = quant_code(row[i + e + 1], s, 127);
+            packed[e >> 2] |= (uint32_t(c0 & 0xff) << ((e & 3) * 8)) |
+                              (uint32_t(c1 & 0xff) << (((e & 3) + 1) * 8));
+            bfw[e >> 1] = uint32_t(int_to_bf16_bits(c0)) | (uint32_t(int_to_bf16_bits(c1)) << 16);
+        }
+        if (xq) *reinterpret_cast<uint2 *>(xq + t * d + i) = make_uint2(packed[0], packed[1]);
+        if (xq_bf16)
+            *reinterpret_cast<uint4 *>(xq_bf16 + t * d + i) = make_uint4(bfw[0], bfw[1], bfw[2], bfw[3]);
+    }
+    if (threadIdx.x == 0 && xs) xs[t] = s;
+}
+
+cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip, int8_t *xq,
+                          uint16_t *xq_bf16, float *xs, cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    const size_t smem = size_t(d) * sizeof(float);
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(xquant_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             int(smem));
+        if (e != cudaSuccess) return e;
+    }
+    xquant_kernel<<<dim3(unsigned(T)), kXqThreads, smem, s>>>(X, d, clip, xq, xq_bf16, xs);
+    prof_mark(s, "xquant");
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Offline: W_d [d, r] fp32 row-major -> per-column codes [r, d] int8 (+bf16).
+// CTA = 32 columns x 8 row lanes; coalesced reads along a row of W_d.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256)
+weight_quant_kernel(const float *__restrict__ W, int d, int r, float clip, int8_t *__restrict__ codes,
+                    uint16_t *__restrict__ codes_bf16, float *__restrict__ scale) {
+    __shared__ float red[8][33];
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int j = blockIdx.x * 32 + tx;
+    float m = 0.0f;
+    if (j < r)
+        for (int k = ty; k < d; k += 8) m = fmaxf(m, fabsf(W[size_t(k) * r + j]));
+    red[ty][tx] = m;
+    __syncthreads();
+    if (ty == 0) {
+        for (int i = 1; i < 8; ++i) m = fmaxf(m, red[i][tx]);
+        red[0][tx] = quant_scale(m, clip, 127.0f);
+    }
+    __syncthreads();
+    const float s = red[0][tx];
+    if (j >= r) return;
+    if (ty == 0) scale[j] = s;
+    for (int k = ty; k < d; k += 8) {
+        const int c = quant_code(W[size_t(k) * r + j], s, 127);
+        codes[size_t(j) * d + k] = int8_t(c);
+        if (codes_bf16) codes_bf16[size_t(j) * d + k] = int_to_bf16_bits(c);
+    }
+}
+
+cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int8_t *codes,
+                                   uint16_t *codes_bf16, float *scale, cudaStream_t s) {
+    weight_quant_kernel<<<dim3((r + 31) / 32), 256, 0, s>>>(W, d, r, clip, codes, codes_bf16, scale);
+    prof_mark(s, "weight_quant");
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// a3/a4: requantize one latent row per CTA.  Each thread owns groups of 4
+// consecutive channels (one float4); an int4 group of 128 channels is one
+// warp's float4 row (32 lanes x 4), so its absmax is a warp reduction.
+// ---------------------------------------------------------------------------
+constexpr int kRqThreads = 256;
+constexpr int kRqMaxQuads = 4;     // r <= 4096
+
+__global__ void __launch_bounds__(kRqThreads)
+requant_kernel(const float *__restrict__ c_hat, int r, int bits, float clip,
+               void *__restrict__ lat_codes, void *__restrict__ lat_scales, CacheView dst,
+               const int32_t *__restrict__ dst_seq, const int32_t *__restrict__ dst_pos,
+               int *err) {
+    __shared__ float red[kRqThreads / 32];
+    const int64_t t = blockIdx.x;
+    const float *row = c_hat + t * r;
+    const int nq = r / 4;
+    float4 v[kRqMaxQuads];
+#pragma unroll
+    for (int k = 0; k < kRqMaxQuads; ++k) {
+        const int qi = threadIdx.x + k * kRqThreads;
+        v[k] = qi < nq ? reinterpret_cast<const float4 *>(row)[qi] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    // cache destination of this row (if any), bounds-checked
+    uint8_t *cache_codes = nullptr;
+    void *cache_scale = nullptr;
+    if (dst.codes) {
+        const int b = dst_seq[t], p = dst_pos[t];
+        if (b < 0 || b >= dst.B || p < 0 || p >= dst.Tmax) {
+            if (threadIdx.x == 0) flag_error(err, kErrRange);
+        } else {
+            const size_t slot = size_t(b) * dst.Tmax + p;
+            if (bits == 8) {
+                cache_codes = static_cast<uint8_t *>(dst.codes) + slot * r;
+                cache_scale = static_cast<float *>(dst.scales) + slot;
+            } else {
+                cache_codes = static_cast<uint8_t *>(dst.codes) + slot * (r / 2);
+                cache_scale = static_cast<__half *>(dst.scales) + slot * (r / 128);
+            }
+        }
+    }
+    uint8_t *tok_codes = lat_codes ? static_cast<uint8_t *>(lat_codes) + t * (bits == 8 ? r : r / 2)
+                                   : nullptr;
+
+    if (bits == 8) {
+        float m = 0.0f;
+#pragma unroll
+        for (int k = 0; k < kRqMaxQuads; ++k)
+            m = fmaxf(m, fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w))));
+        m = block_max<kRqThreads>(m, red);
+        const float s = quant_scale(m, clip, 127.0f);
+#pragma unroll
+        for (int k = 0; k < kRqMaxQuads; ++k) {
+            const int qi = threadIdx.x + k * kRqThreads;
+            if (qi >= nq) break;
+            const uint32_t w = uint32_t(quant_code(v[k].x, s, 127) & 0xff) |
+                               (uint32_t(quant_code(v[k].y, s, 127) & 0xff) << 8) |
+                               (uint32_t(quant_code(v[k].z, s, 127) & 0xff) << 16) |
+                               (uint32_t(quant_code(v[k].w, s, 127) & 0xff) << 24);
+            if (tok_codes) reinterpret_cast<uint32_t *>(tok_codes)[qi] = w;
+            if (cache_codes) reinterpret_cast<uint32_t *>(cache_codes)[qi] = w;
+        }
+        if (threadIdx.x == 0) {
+            if (lat_scales) static_cast<float *>(lat_scales)[t] = s;
+            if (cache_scale) *static_cast<float *>(cache_scale) = s;
+        }
+    } else {
+        // quad qi covers channels 4qi..4qi+3; its group is qi / 32 = one warp row
+#pragma unroll
+        for (int k = 0; k < kRqMaxQuads; ++k) {
+            const int qi = threadIdx.x + k * kRqThreads;
+            if (qi - (threadIdx.x & 31) >= nq) break;       // warp-uniform
+            float m = fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w)));
+            m = warp_max(m);
+            const __half hs = int4_group_scale(m, clip);
+            const float s = __half2float(hs);
+            const int c0 = quant_code(v[k].x, s, 7), c1 = quant_code(v[k].y, s, 7);
+            const int c2 = quant_code(v[k].z, s, 7), c3 = quant_code(v[k].w, s, 7);
+            const uint16_t w = uint16_t((c0 & 0xf) | ((c1 & 0xf) << 4) | ((c2 & 0xf) << 8) | ((c3 & 0xf) << 12));
+            if (tok_codes) reinterpret_cast<uint16_t *>(tok_codes)[qi] = w;
+            if (cache_codes) reinterpret_cast<uint16_t *>(cache_codes)[qi] = w;
+            if ((threadIdx.x & 31) == 0) {
+                const int g = qi >> 5;
+                if (lat_scales) static_cast<__half *>(lat_scales)[t * (r / 128) + g] = hs;
+                if (cache_scale) static_cast<__half *>(cache_scale)[g] = hs;
+            }
+        }
+    }
+}
+
+cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float clip, void *lat_codes,
+                           void *lat_scales, const CacheView *dst, const int32_t *dst_seq,
+                           const int32_t *dst_pos, int *err, cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    CacheView d{};
+    if (dst) d = *dst;
+    requant_kernel<<<dim3(unsigned(T)), kRqThreads, 0, s>>>(c_hat, r, bits, clip, lat_codes, lat_scales, d,
+                                                             dst_seq, dst_pos, err);
+    prof_mark(s, "requant");
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// a4: copy rows into the cache.  One warp per row, 16-byte vectors.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256)
+append_kernel(CacheView c, const int32_t *__restrict__ seq, const int32_t *__restrict__ pos, int64_t n,
+              const uint8_t *__restrict__ codes, const uint8_t *__restrict__ scales, int *err) {
+    const int64_t i = int64_t(blockIdx.x) * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (i >= n) return;
+    const int b = seq[i], p = pos[i];
+    if (b < 0 || b >= c.B || p < 0 || p >= c.Tmax) {
+        if (lane == 0) flag_error(err, kErrRange);
+        return;
+    }
+    const size_t slot = size_t(b) * c.Tmax + p;
+    const int row_bytes = c.bits == 8 ? c.r : c.r / 2;
+    const int scale_bytes = c.bits == 8 ? 4 : 2 * (c.r / 128);
+    const uint4 *src = reinterpret_cast<const uint4 *>(codes + i * row_bytes);
+    uint4 *dstc = reinterpret_cast<uint4 *>(static_cast<uint8_t *>(c.codes) + slot * row_bytes);
+    for (int k = lane; k < row_bytes / 16; k += 32) dstc[k] = src[k];
+    uint8_t *dsts = static_cast<uint8_t *>(c.scales) + slot * scale_bytes;
+    for (int k = lane; k < scale_bytes; k += 32) dsts[k] = scales[i * scale_bytes + k];
+}
+
+cudaError_t launch_append(const CacheView &c, const int32_t *seq, const int32_t *pos, int64_t n,
+                          const void *lat_codes, const void *lat_scales, int *err, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    append_kernel<<<dim3(unsigned((n + 7) / 8)), 256, 0, s>>>(
+        c, seq, pos, n, static_cast<const uint8_t *>(lat_codes), static_cast<const uint8_t *>(lat_scales), err);
+    prof_mark(s, "append");
+    return cudaGetLastError();
+}
+
+}  // namespace qsvd
