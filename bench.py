@@ -217,6 +217,9 @@ class NativeBench:
         torch = self.torch
         n = steps * (self.S * 12 + 8)
         events = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+        for e in events:            # torch creates the CUDA event lazily, on first record
+            e.record(self.stream)
+        torch.cuda.synchronize()
         handles = (ctypes.c_void_p * n)(*[ctypes.c_void_p(e.cuda_event) for e in events])
         ctx = []          # sub-step of each recorded event
         lib = self.lib

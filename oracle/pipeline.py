@@ -39,7 +39,8 @@ def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1
     else:
         W_d, U_q, U_k, U_v = inp.W_d, inp.U_q, inp.U_k, inp.U_v
     Wq, s_w = quant.quantize_columns(W_d, 8, w_clip)
-    return dict(W_d=W_d, Wq=Wq, s_w=s_w, U_q=U_q, U_k=U_k, U_v=U_v)
+    c = np.ascontiguousarray
+    return dict(W_d=c(W_d), Wq=c(Wq), s_w=c(s_w), U_q=c(U_q), U_k=c(U_k), U_v=c(U_v))
 
 
 class OracleLayer:

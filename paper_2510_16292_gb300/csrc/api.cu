@@ -87,7 +87,10 @@ thread_local std::vector<const char *> t_prof_labels;
 
 void prof_mark(cudaStream_t s, const char *label) {
     if (!t_prof_events || int(t_prof_labels.size()) >= t_prof_capacity) return;
-    if (cudaEventRecord(t_prof_events[t_prof_labels.size()], s) == cudaSuccess) t_prof_labels.push_back(label);
+    if (cudaEventRecord(t_prof_events[t_prof_labels.size()], s) == cudaSuccess)
+        t_prof_labels.push_back(label);
+    else
+        (void)cudaGetLastError();     // a bad event handle must not surface as a launch error
 }
 
 }  // namespace qsvd
@@ -182,9 +185,9 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
     if (dst) {
         if ((st = check_cache(dst))) return st;
         if (dst->bits != lat_bits || dst->r != r) return fail(QSVD_EINVAL, "latent_project: cache format differs");
-        if (!dst_seq || !dst_pos) return fail(QSVD_EINVAL, "latent_project: dst_seq/dst_pos required with dst");
     }
     if (T == 0) return QSVD_OK;
+    if (dst && (!dst_seq || !dst_pos)) return fail(QSVD_EINVAL, "latent_project: dst_seq/dst_pos required with dst");
     if (!X) return fail(QSVD_EINVAL, "latent_project: X is null");
     const void *ptrs[] = {X, W->codes, W->scale, lat_codes, lat_scales, xq_out, xs_out, acc_out, workspace};
     for (const void *p : ptrs)
