@@ -7,7 +7,7 @@ text-like; per-token int8 X, exact int8 GEMM with W_d, per-token latent
 requantization fused into the cache store), then 128 decode steps (project
 the new token, append it, attend over the int8 latent cache with U_k absorbed
 and U_v applied last).  Inputs are seeded synthetic arrays resident in HBM
-before timing.  L2 is flushed (a 256 MiB write) before the prefill and before
+before timing.  L2 is flushed (a 256 MiB read) before the prefill and before
 every decode step; the flush sits outside the timed intervals, which are CUDA
 events on the launching stream around each sub-step.
 
@@ -150,22 +150,23 @@ class NativeBench:
         self.dpos = [i32(np.full(B, P + t)) for t in range(S)]
         self.dlen = [i32(np.full(B, P + t + 1)) for t in range(S)]
         self.O = torch.empty((B, s.d), dtype=torch.float32, device=dev)
-        self.wsp = torch.empty(q.qsvd_project_workspace_bytes(B * P, s.d, s.r), dtype=torch.uint8, device=dev)
-        self.wsd = torch.empty(q.qsvd_decode_workspace_bytes(B, wl.tmax, s.r, s.H, s.dh), dtype=torch.uint8,
+        self.wsp = torch.zeros(q.qsvd_project_workspace_bytes(B * P, s.d, s.r), dtype=torch.uint8, device=dev)
+        self.wsd = torch.zeros(q.qsvd_decode_workspace_bytes(B, wl.tmax, s.r, s.H, s.dh), dtype=torch.uint8,
                                device=dev)
-        self.flushbuf = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+        self.flushbuf = torch.ones(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+        self.flush_out = torch.zeros((), dtype=torch.int64, device=dev)
         self.stream = torch.cuda.current_stream()
         self._marshal()
 
-    def _marshal(self):
-        """Pre-build the ctypes argument tuples of every C-ABI call of a step."""
+    def _marshal(self, stream=None):
+        """Pre-build the ctypes argument tuples of every C-ABI call of a step,
+        bound to `stream` (default: the current stream)."""
         q, wl, s = self.q, self.wl, self.wl.shape
         lib = q._lib
         self.lib = lib
         self.cW = self.W._c()
         self.cC = self.cache._c()
-        st = self.stream.cuda_stream
-        P = ctypes.c_void_p
+        st = (stream or self.stream).cuda_stream
         self.pre_args = (ctypes.byref(self.cW), self.Xp.data_ptr(), self.B * self.P, 1.0, wl.lat_bits, 1.0,
                          None, None, ctypes.byref(self.cC), self.pseq.data_ptr(), self.ppos.data_ptr(),
                          None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st)
@@ -179,7 +180,25 @@ class NativeBench:
                                   self.U[0].data_ptr(), self.U[1].data_ptr(), self.U[2].data_ptr(), s.H, s.dh,
                                   1.0 / math.sqrt(s.dh), self.O.data_ptr(), self.wsd.data_ptr(),
                                   self.wsd.numel(), st))
-        del P
+
+    def build_graph(self):
+        """Capture one whole step (flushes, sub-step events and every C-ABI
+        call) into a CUDA graph; replaying it removes host launch overhead."""
+        torch = self.torch
+        gs = torch.cuda.Stream()
+        self._marshal(stream=gs)
+        E = lambda: torch.cuda.Event(enable_timing=True, external=True)  # noqa: E731
+        self.gevs = [(E(), E()) for _ in range(self.S + 1)]
+        gs.wait_stream(self.stream)
+        with torch.cuda.stream(gs):
+            self.run_step(self.make_events(), gs)          # eager warm-up on the capture stream
+        gs.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=gs):
+            self.run_step(self.gevs, gs)
+        torch.cuda.synchronize()
+        self.graph = g
+        self._marshal()                                    # eager calls go back to the default stream
 
     def _call(self, fn, args):
         stt = fn(*args)
@@ -194,19 +213,26 @@ class NativeBench:
         self._call(self.lib.qsvd_latent_decode_attn, self.dec_attn[t])
 
     def flush(self):
-        self.flushbuf.fill_(1)
+        """Evict L2 by reading a 256 MiB buffer (leaves L2 clean, unlike a write)."""
+        torch = self.torch
+        torch.sum(self.flushbuf, dim=(0,), dtype=torch.int64, out=self.flush_out)
 
-    def run_step(self, evs):
+    def run_step(self, evs, stream=None):
         """evs: list of (start, end) event pairs, one per sub-step (prefill, decode 0..S-1)."""
+        st = stream or self.stream
         self.flush()
-        evs[0][0].record(self.stream)
+        evs[0][0].record(st)
         self.prefill()
-        evs[0][1].record(self.stream)
+        evs[0][1].record(st)
         for t in range(self.S):
             self.flush()
-            evs[t + 1][0].record(self.stream)
+            evs[t + 1][0].record(st)
             self.decode(t)
-            evs[t + 1][1].record(self.stream)
+            evs[t + 1][1].record(st)
+
+    def replay(self):
+        self.graph.replay()
+        return self.gevs
 
     def make_events(self):
         E = self.torch.cuda.Event
@@ -267,12 +293,10 @@ class NativeBench:
             return r * d * 2 + B * (tok + stok) + 4 * B * d
         if label == "qabsorb":
             return r * d * 2 + 4 * B * d + 4 * B * H * r
-        if label == "attn_split":
-            ns = (L + 255) // 256
-            return B * L * (tok + stok) + 4 * B * H * r + 4 * B * ns * H * (r + 2)
+        if label == "attn_chunk":
+            return B * L * (tok + stok) + 4 * B * H * r
         if label == "combine_uv":
-            ns = (L + 255) // 256
-            return r * d * 2 + 4 * B * ns * H * (r + 2) + 4 * B * d
+            return r * d * 2 + 4 * B * d
         return 0
 
     def step_roofline_bytes(self, t):
@@ -331,28 +355,28 @@ def run_native(args, rank, world, local_rank):
     S = wl.decode_steps
     hbm, _, peak_kind = peaks()
 
-    # warm-up
+    nb.build_graph()
     for _ in range(args.warmup):
-        nb.run_step(nb.make_events())
+        nb.replay()
     torch.cuda.synchronize()
-    step_events = [nb.make_events() for _ in range(args.steps)]
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     clocks = ClockSampler(local_rank)
     clocks.start()
     t_wall = time.perf_counter()
+    pre, dec, per_dec = [], [], []
     for k in range(args.steps):
-        nb.run_step(step_events[k])
-    torch.cuda.synchronize()
+        evs = nb.replay()
+        torch.cuda.synchronize()                   # events are re-recorded by the next replay
+        pre.append(evs[0][0].elapsed_time(evs[0][1]) * 1e-3)
+        d_t = [evs[t + 1][0].elapsed_time(evs[t + 1][1]) * 1e-3 for t in range(S)]
+        per_dec.append(d_t)
+        dec.append(sum(d_t))
     if world > 1:
         torch.distributed.barrier()
     t_wall = time.perf_counter() - t_wall
     clk = clocks.stop()
-    pre = [step_events[k][0][0].elapsed_time(step_events[k][0][1]) * 1e-3 for k in range(args.steps)]
-    dec = [sum(a.elapsed_time(b) for a, b in step_events[k][1:]) * 1e-3 for k in range(args.steps)]
-    per_dec = [[step_events[k][t + 1][0].elapsed_time(step_events[k][t + 1][1]) * 1e-3 for t in range(S)]
-               for k in range(args.steps)]
     dec_total, pre_total = sum(dec), sum(pre)
     if world > 1:
         tt = torch.tensor([dec_total, pre_total], dtype=torch.float64, device=nb.dev)
@@ -405,8 +429,9 @@ def run_native(args, rank, world, local_rank):
         "data": "synthetic",
         "config": {"workload": workload_desc(wl), "global_batch": world * wl.B,
                    "seq_len": wl.tmax, "parallelism": f"replicas x{world} (one independent layer per GPU)",
-                   "l2": "flushed (256 MiB write) before the prefill and before every decode step; "
-                         "flushes outside the timed intervals"},
+                   "l2": "flushed (256 MiB read) before the prefill and before every decode step; "
+                         "flushes outside the timed intervals",
+                   "launch": "one CUDA graph per step (captured C-ABI calls, PDL-chained kernels)"},
         "secondary": {
             "decode_ms_per_step": round(dec_total / args.steps * 1e3, 4),
             "prefill_ms_per_step": round(pre_total / args.steps * 1e3, 4),

@@ -20,6 +20,14 @@
  *   - Every pointer is device memory owned by the caller unless stated
  *     otherwise.  The library never allocates device memory; scratch space is
  *     a caller-provided workspace whose size the *_workspace_bytes calls give.
+ *     A workspace must be zero-filled before its first use; every call leaves
+ *     the workspace's completion counters at zero again, so a workspace can be
+ *     reused by later calls on the same stream, but two calls that may run
+ *     concurrently on the GPU need separate workspaces.
+ *   - Kernels are launched with programmatic dependent launch: a call may
+ *     begin prefetching its (read-only) weights into L2 while the previous
+ *     kernel in the stream is still running; every read of data produced by
+ *     earlier stream work happens after that work has completed.
  *   - Calls are asynchronous on `stream` and never synchronize it, except
  *     qsvd_check.  A return of QSVD_OK means the work was enqueued.
  *   - bf16 buffers are passed as uint16_t bit patterns.
@@ -159,7 +167,8 @@ int qsvd_cache_append(const qsvd_cache *cache, const int32_t *seq, const int32_t
  *   U_q, U_k, U_v  bf16 [r, H*dh] row-major;
  *   O            fp32 [B, H*dh] out.
  * workspace: qsvd_decode_workspace_bytes(B, max_seq_len, r, H, dh) bytes.
- * Requirements: dh in {64, 128}; r % 16 == 0 and r <= 3072.
+ * Requirements: dh in {64, 128}; r % 16 == 0 and r <= 3072; H*dh % 256 == 0
+ * and H*dh <= 6144.
  */
 int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int32_t max_seq_len,
                             const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v,

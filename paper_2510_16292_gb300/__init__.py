@@ -162,7 +162,7 @@ def qsvd_latent_project(W: DownWeight, X: torch.Tensor, act_clip: float = 1.0, l
                         xq_out=None, xs_out=None, acc_out=None, workspace=None, stream=None) -> None:
     T = X.shape[0]
     if workspace is None:
-        workspace = torch.empty(max(1, qsvd_project_workspace_bytes(T, W.d, W.r)), dtype=torch.uint8,
+        workspace = torch.zeros(max(1, qsvd_project_workspace_bytes(T, W.d, W.r)), dtype=torch.uint8,
                                 device=X.device)
     cw = W._c()
     cc = dst._c() if dst is not None else None
@@ -186,7 +186,7 @@ def qsvd_latent_decode_attn(cache: LatentCache, seq_len: torch.Tensor, max_seq_l
     if softmax_scale is None:
         softmax_scale = 1.0 / math.sqrt(dh)
     if workspace is None:
-        workspace = torch.empty(qsvd_decode_workspace_bytes(cache.B, max_seq_len, cache.r, H, dh),
+        workspace = torch.zeros(qsvd_decode_workspace_bytes(cache.B, max_seq_len, cache.r, H, dh),
                                 dtype=torch.uint8, device=O.device)
     cc = cache._c()
     _check(_lib.qsvd_latent_decode_attn(ctypes.byref(cc), _ptr(seq_len), max_seq_len, _ptr(U_q), _ptr(U_k),

@@ -3,6 +3,8 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
+#include <unordered_map>
 #include <vector>
 
 #include "launch.h"
@@ -85,6 +87,29 @@ thread_local std::vector<const char *> t_prof_labels;
 
 }  // namespace
 
+cudaError_t ensure_smem_ptr(const void *kernel, size_t bytes) {
+    static std::mutex mu;
+    static std::unordered_map<const void *, int> done;     // kernel -> device bitmask
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    int &mask = done[kernel];
+    if (dev < 31 && (mask >> dev) & 1) return cudaSuccess;
+    // the opt-in limit covers static + dynamic shared memory of the kernel
+    int optin = 0;
+    e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e != cudaSuccess) return e;
+    cudaFuncAttributes fa{};
+    e = cudaFuncGetAttributes(&fa, kernel);
+    if (e != cudaSuccess) return e;
+    const int max_dyn = optin - int(fa.sharedSizeBytes);
+    if (int64_t(bytes) > max_dyn) return cudaErrorInvalidValue;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, max_dyn);
+    if (e == cudaSuccess && dev < 31) mask |= 1 << dev;
+    return e;
+}
+
 void prof_mark(cudaStream_t s, const char *label) {
     if (!t_prof_events || int(t_prof_labels.size()) >= t_prof_capacity) return;
     if (cudaEventRecord(t_prof_events[t_prof_labels.size()], s) == cudaSuccess)
@@ -157,7 +182,8 @@ int qsvd_quantize_weight(const float *W_d, int32_t d, int32_t r, float clip, int
 
 size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r) {
     if (T < 0 || d <= 0 || r <= 0) return 0;
-    return align256(size_t(T) * d) +            // int8 codes of X
+    return 256 +                                // completion counter (zero at rest)
+           align256(size_t(T) * d) +            // int8 codes of X
            align256(size_t(T) * 4) +            // s_x
            align256(size_t(T) * r * 4);         // dequantized latent c_hat
 }
@@ -197,19 +223,28 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
         return fail(QSVD_ENOSPC, "latent_project: workspace needs %zu bytes", need);
 
     char *wsp = static_cast<char *>(workspace);
+    int *counter = reinterpret_cast<int *>(wsp);
+    wsp += 256;
     int8_t *xq = xq_out ? xq_out : reinterpret_cast<int8_t *>(wsp);
     wsp += align256(size_t(T) * d);
     float *xs = xs_out ? xs_out : reinterpret_cast<float *>(wsp);
     wsp += align256(size_t(T) * 4);
     float *c_hat = reinterpret_cast<float *>(wsp);
+    CacheView dv{};
+    if (dst) dv = view(dst);
 
     prof_mark(stream, "begin");
-    cudaError_t e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream);
+    cudaError_t e;
+    if (T <= kPsMaxTok && d <= 6144 && d % 256 == 0) {
+        e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
+                              xq_out, xs_out, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq, dst_pos,
+                              err, stream);
+        return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "projection launch");
+    }
+    e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream);
     if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
     e = launch_proj_dp4a(xq, T, d, W->codes, W->scale, xs, r, c_hat, acc_out, stream);
     if (e != cudaSuccess) return cuda_fail(e, "projection launch");
-    CacheView dv{};
-    if (dst) dv = view(dst);
     e = launch_requant(c_hat, T, r, lat_bits, lat_clip, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
                        dst_pos, err, stream);
     if (e != cudaSuccess) return cuda_fail(e, "requant launch");
@@ -248,6 +283,7 @@ int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int
     if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "decode_attn: dh must be 64 or 128");
     if (H <= 0) return fail(QSVD_EINVAL, "decode_attn: H must be positive");
     if (cache->r > 3072) return fail(QSVD_EUNSUPPORTED, "decode_attn: r > 3072");
+    if ((H * dh) % 256 || H * dh > 6144) return fail(QSVD_EUNSUPPORTED, "decode_attn: need H*dh %% 256 == 0 and H*dh <= 6144");
     if (max_seq_len < 1 || max_seq_len > cache->Tmax) return fail(QSVD_EINVAL, "decode_attn: max_seq_len outside [1, Tmax]");
     const void *ptrs[] = {U_q, U_k, U_v, O, workspace};
     for (const void *p : ptrs)

@@ -10,8 +10,82 @@
 
 namespace qsvd {
 
+// Programmatic dependent launch: let the next kernel in the stream start its
+// prologue now / wait until every earlier kernel in the stream has finished
+// and its writes are visible.  Both are no-ops without the launch attribute.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Bulk prefetch of [p, p + bytes) into L2 (16-byte aligned, bytes % 16 == 0).
+// A hint only: data written later by an earlier kernel is still read
+// correctly, because later loads go through the coherent L2.
+__device__ __forceinline__ void prefetch_l2_bulk(const void *p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+// CTA `i` of `n` prefetches its 1/n share of a buffer into L2 (thread 0 only,
+// in pieces of at most 64 KiB).
+__device__ __forceinline__ void prefetch_share_l2(const void *base, size_t bytes, size_t i, size_t n) {
+    if (threadIdx.x != 0 || bytes == 0) return;
+    size_t per = ((bytes + n - 1) / n + 15) & ~size_t(15);
+    size_t lo = i * per;
+    if (lo >= bytes) return;
+    size_t hi = lo + per < bytes ? lo + per : bytes;
+    hi &= ~size_t(15);
+    const char *c = static_cast<const char *>(base);
+    for (size_t o = lo; o < hi; o += 65536) {
+        const size_t len = hi - o < 65536 ? hi - o : 65536;
+        prefetch_l2_bulk(c + o, uint32_t(len));
+    }
+}
+
 __device__ __forceinline__ void flag_error(int *err, int bit) {
     if (err) atomicOr(err, bit);
+}
+
+// ---------------------------------------------------------------------------
+// mbarrier + bulk (TMA, non-tensor) copies global -> shared
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_init_fence() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+// One arrival that also announces `bytes` of transactions for this phase.
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+                 : "memory");
+}
+// Bulk copy of `bytes` (multiple of 16; both addresses 16-byte aligned).
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(smem_addr(dst)), "l"(src), "r"(bytes), "r"(smem_addr(bar))
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+                 "selp.u32 %0, 1, 0, p;\n}\n"
+                 : "=r"(ok)
+                 : "r"(smem_addr(bar)), "r"(parity)
+                 : "memory");
+    return ok != 0;
+}
+// Bounded wait for phase `parity`.  On expiry the error word gets
+// kErrTimeout, then the wait continues (bounded again) so that copies still in
+// flight land before the CTA may exit; returns whether the phase completed.
+constexpr long kWaitLimit = 1L << 24;
+static __device__ __noinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int *err) {
+    for (long i = 0; i < kWaitLimit; ++i)
+        if (mbar_try_wait(bar, parity)) return true;
+    flag_error(err, kErrTimeout);
+    for (long i = 0; i < kWaitLimit; ++i)
+        if (mbar_try_wait(bar, parity)) return false;
+    return false;
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -83,6 +157,97 @@ __device__ __forceinline__ float block_max(float v, float *red) {
 #pragma unroll
     for (int i = 1; i < NT / 32; ++i) m = fmaxf(m, red[i]);
     return m;
+}
+
+
+// ---------------------------------------------------------------------------
+// Per-token requantization of latent row t of c_hat [T, r] by one CTA of
+// kRqThreads threads (Eq. 11's Q(C_qkv)): int8 with one fp32 scale per token,
+// or int4 with one fp16 scale per 128-channel group (one warp row of float4).
+// Writes token-major outputs and/or the cache slot (seq, pos) of row t;
+// out-of-range slots are skipped and flagged.  `red` holds kRqThreads/32 floats.
+// ---------------------------------------------------------------------------
+constexpr int kRqThreads = 256;
+constexpr int kRqMaxQuads = 4;     // r <= 4096
+
+__device__ __forceinline__ void requant_row_cta(const float *__restrict__ c_hat, int64_t t, int r, int bits,
+                                                float clip, void *__restrict__ lat_codes,
+                                                void *__restrict__ lat_scales, const CacheView &dst,
+                                                const int32_t *__restrict__ dst_seq,
+                                                const int32_t *__restrict__ dst_pos, int *err, float *red) {
+    const float *row = c_hat + t * r;
+    const int nq = r / 4;
+    float4 v[kRqMaxQuads];
+#pragma unroll
+    for (int k = 0; k < kRqMaxQuads; ++k) {
+        const int qi = threadIdx.x + k * kRqThreads;
+        v[k] = qi < nq ? reinterpret_cast<const float4 *>(row)[qi] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    // cache destination of this row (if any), bounds-checked
+    uint8_t *cache_codes = nullptr;
+    void *cache_scale = nullptr;
+    if (dst.codes) {
+        const int b = dst_seq[t], p = dst_pos[t];
+        if (b < 0 || b >= dst.B || p < 0 || p >= dst.Tmax) {
+            if (threadIdx.x == 0) flag_error(err, kErrRange);
+        } else {
+            const size_t slot = size_t(b) * dst.Tmax + p;
+            if (bits == 8) {
+                cache_codes = static_cast<uint8_t *>(dst.codes) + slot * r;
+                cache_scale = static_cast<float *>(dst.scales) + slot;
+            } else {
+                cache_codes = static_cast<uint8_t *>(dst.codes) + slot * (r / 2);
+                cache_scale = static_cast<__half *>(dst.scales) + slot * (r / 128);
+            }
+        }
+    }
+    uint8_t *tok_codes = lat_codes ? static_cast<uint8_t *>(lat_codes) + t * (bits == 8 ? r : r / 2)
+                                   : nullptr;
+
+    if (bits == 8) {
+        float m = 0.0f;
+#pragma unroll
+        for (int k = 0; k < kRqMaxQuads; ++k)
+            m = fmaxf(m, fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w))));
+        m = block_max<kRqThreads>(m, red);
+        const float s = quant_scale(m, clip, 127.0f);
+#pragma unroll
+        for (int k = 0; k < kRqMaxQuads; ++k) {
+            const int qi = threadIdx.x + k * kRqThreads;
+            if (qi >= nq) break;
+            const uint32_t w = uint32_t(quant_code(v[k].x, s, 127) & 0xff) |
+                               (uint32_t(quant_code(v[k].y, s, 127) & 0xff) << 8) |
+                               (uint32_t(quant_code(v[k].z, s, 127) & 0xff) << 16) |
+                               (uint32_t(quant_code(v[k].w, s, 127) & 0xff) << 24);
+            if (tok_codes) reinterpret_cast<uint32_t *>(tok_codes)[qi] = w;
+            if (cache_codes) reinterpret_cast<uint32_t *>(cache_codes)[qi] = w;
+        }
+        if (threadIdx.x == 0) {
+            if (lat_scales) static_cast<float *>(lat_scales)[t] = s;
+            if (cache_scale) *static_cast<float *>(cache_scale) = s;
+        }
+    } else {
+        // quad qi covers channels 4qi..4qi+3; its group is qi / 32 = one warp row
+#pragma unroll
+        for (int k = 0; k < kRqMaxQuads; ++k) {
+            const int qi = threadIdx.x + k * kRqThreads;
+            if (qi - (threadIdx.x & 31) >= nq) break;       // warp-uniform
+            float m = fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w)));
+            m = warp_max(m);
+            const __half hs = int4_group_scale(m, clip);
+            const float s = __half2float(hs);
+            const int c0 = quant_code(v[k].x, s, 7), c1 = quant_code(v[k].y, s, 7);
+            const int c2 = quant_code(v[k].z, s, 7), c3 = quant_code(v[k].w, s, 7);
+            const uint16_t w = uint16_t((c0 & 0xf) | ((c1 & 0xf) << 4) | ((c2 & 0xf) << 8) | ((c3 & 0xf) << 12));
+            if (tok_codes) reinterpret_cast<uint16_t *>(tok_codes)[qi] = w;
+            if (cache_codes) reinterpret_cast<uint16_t *>(cache_codes)[qi] = w;
+            if ((threadIdx.x & 31) == 0) {
+                const int g = qi >> 5;
+                if (lat_scales) static_cast<__half *>(lat_scales)[t * (r / 128) + g] = hs;
+                if (cache_scale) static_cast<__half *>(cache_scale)[g] = hs;
+            }
+        }
+    }
 }
 
 }  // namespace qsvd

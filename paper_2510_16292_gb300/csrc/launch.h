@@ -5,9 +5,38 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 #include <cuda_runtime.h>
 
 namespace qsvd {
+
+// Raise a kernel's dynamic shared memory limit to the maximum the first time
+// it needs more than the default (so that no attribute call happens while a
+// stream is being captured into a graph).  Defined in api.cu.
+cudaError_t ensure_smem_ptr(const void *kernel, size_t bytes);
+template <typename K>
+cudaError_t ensure_smem(K kernel, size_t bytes) {
+    return bytes <= 48 * 1024 ? cudaSuccess : ensure_smem_ptr(reinterpret_cast<const void *>(kernel), bytes);
+}
+
+// Launch with programmatic stream serialization: the kernel may start while
+// the previous kernel in the stream is still running; it must execute
+// pdl_wait() before reading anything an earlier stream operation produced.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // Bits of the device error word (read and cleared by qsvd_check).
 enum : int { kErrRange = 1, kErrTimeout = 2 };
@@ -41,6 +70,15 @@ cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int
 cudaError_t launch_proj_dp4a(const int8_t *xq, int64_t T, int d, const int8_t *wcodes,
                              const float *ws, const float *xs, int r, float *c_hat,
                              int32_t *acc_out, cudaStream_t s);
+
+// Decode-size projection (T <= kPsMaxTok): a1, a2, a3 and a4 in one launch.
+// `counter` must be zero before the first call; the kernel leaves it at zero.
+constexpr int kPsMaxTok = 16;
+cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, const int8_t *wcodes,
+                              const float *ws, int r, int lat_bits, float lat_clip, float *c_hat, int *counter,
+                              int8_t *xq_out, float *xs_out, int32_t *acc_out, void *lat_codes, void *lat_scales,
+                              const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
+                              cudaStream_t s);
 
 // Per-token requantization of c_hat [T, r] into the latent format (a3 second
 // half), written token-major and/or into the cache (a4).

@@ -2,9 +2,10 @@
 // the dequantization of Eq. 12's product fused behind it:
 //   acc[t, j]   = sum_k xq[t, k] * w[j, k]          (exact: |acc| < 2^31)
 //   c_hat[t, j] = fp32(fp32(fp32(acc) * s_x[t]) * s_w[j])
-// This is the small-T path (decode: one token per sequence), where the GEMM
-// is bound by reading W_d's int8 codes once; prefill-sized T goes to the
-// tensor-core kernel.
+// proj_dp4a_kernel is the general CUDA-core path; proj_small_kernel is the
+// decode path (T <= kPsMaxTok tokens): it quantizes X itself, streams its 8
+// rows of W_d codes into shared memory with one bulk copy, and the last CTA
+// to finish requantizes the latent rows and stores them (a1-a4 in one launch).
 #include "common.cuh"
 #include "launch.h"
 
@@ -19,6 +20,9 @@ proj_dp4a_kernel(const int8_t *__restrict__ xq, int64_t T, int d, const int8_t *
                  float *__restrict__ c_hat, int32_t *__restrict__ acc_out) {
     const int lane = threadIdx.x & 31;
     const int j = blockIdx.x * kPjWarps + (threadIdx.x >> 5);
+    pdl_trigger();
+    if (blockIdx.y == 0) prefetch_share_l2(w, size_t(r) * d, blockIdx.x, gridDim.x);
+    pdl_wait();
     if (j >= r) return;
     const int64_t t0 = int64_t(blockIdx.y) * kPjTokens;
     const int64_t t1 = (T < t0 + kPjTokens) ? T : t0 + kPjTokens;
@@ -38,13 +42,135 @@ proj_dp4a_kernel(const int8_t *__restrict__ xq, int64_t T, int d, const int8_t *
     }
 }
 
+// ---------------------------------------------------------------------------
+// Decode path.  CTA = 8 output channels (one warp each); every CTA quantizes
+// the T <= kPsMaxTok token rows itself (redundantly, they are tiny).
+// ---------------------------------------------------------------------------
+constexpr int kPsWarps = 8;
+constexpr int kPsMaxD = 6144;          // d <= 6144: 24 x 16-byte vectors per lane
+
+__global__ void __launch_bounds__(kPsWarps * 32)
+proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, const int8_t *__restrict__ w,
+                  const float *__restrict__ ws, int r, int lat_bits, float lat_clip, float *__restrict__ c_hat,
+                  int *__restrict__ counter, int8_t *__restrict__ xq_out, float *__restrict__ xs_out,
+                  int32_t *__restrict__ acc_out, void *__restrict__ lat_codes, void *__restrict__ lat_scales,
+                  CacheView dst, const int32_t *__restrict__ dst_seq, const int32_t *__restrict__ dst_pos,
+                  int *err) {
+    extern __shared__ __align__(16) uint8_t smem[];
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ float xs_s[kPsMaxTok];
+    __shared__ float red[kPsWarps];
+    __shared__ int last;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j0 = blockIdx.x * kPsWarps;
+    const int rows = min(kPsWarps, r - j0);
+    int8_t *w_s = reinterpret_cast<int8_t *>(smem);                  // [kPsWarps][d]
+    int8_t *xq_s = reinterpret_cast<int8_t *>(smem) + kPsWarps * d;  // [T][d]
+    pdl_trigger();
+    prefetch_share_l2(w, size_t(r) * d, blockIdx.x, gridDim.x);
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        mbar_init_fence();
+    }
+    __syncthreads();
+    pdl_wait();
+    if (threadIdx.x == 0) {
+        mbar_arrive_expect_tx(&bar, uint32_t(rows) * d);
+        bulk_g2s(w_s, w + size_t(j0) * d, uint32_t(rows) * d, &bar);
+    }
+    // a1: per-token int8 quantization; the whole CTA works on one token at a time
+    for (int t = 0; t < T; ++t) {
+        float f[kPsMaxD / 2048][8];
+        float m = 0.0f;
+#pragma unroll
+        for (int k = 0; k < kPsMaxD / 2048; ++k) {
+            const int col = (k * 256 + threadIdx.x) * 8;
+            if (col < d) {
+                unpack8_bf16(*reinterpret_cast<const uint4 *>(X + size_t(t) * d + col), f[k]);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(f[k][e]));
+            }
+        }
+        m = block_max<kPsWarps * 32>(m, red);
+        const float s = quant_scale(m, act_clip, 127.0f);
+#pragma unroll
+        for (int k = 0; k < kPsMaxD / 2048; ++k) {
+            const int col = (k * 256 + threadIdx.x) * 8;
+            if (col < d) {
+                uint32_t lo = 0, hi = 0;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    lo |= uint32_t(quant_code(f[k][e], s, 127) & 0xff) << (8 * e);
+                    hi |= uint32_t(quant_code(f[k][e + 4], s, 127) & 0xff) << (8 * e);
+                }
+                *reinterpret_cast<uint2 *>(xq_s + size_t(t) * d + col) = make_uint2(lo, hi);
+                if (xq_out && blockIdx.x == 0)
+                    *reinterpret_cast<uint2 *>(xq_out + size_t(t) * d + col) = make_uint2(lo, hi);
+            }
+        }
+        if (threadIdx.x == 0) {
+            xs_s[t] = s;
+            if (xs_out && blockIdx.x == 0) xs_out[t] = s;
+        }
+    }
+    __syncthreads();
+    mbar_wait(&bar, 0, err);
+    // a2 + first half of a3: exact int32 dot products, then the fp32 dequantization
+    if (warp < rows) {
+        const int j = j0 + warp;
+        const int *wrow = reinterpret_cast<const int *>(w_s + size_t(warp) * d);
+        const float sw = ws[j];
+        for (int t = 0; t < T; ++t) {
+            const int *xrow = reinterpret_cast<const int *>(xq_s + size_t(t) * d);
+            int acc = 0;
+#pragma unroll 8
+            for (int i = lane; i < d / 4; i += 32) acc = __dp4a(wrow[i], xrow[i], acc);
+            acc = warp_sum_int(acc);
+            if (lane == 0) {
+                c_hat[size_t(t) * r + j] = __fmul_rn(__fmul_rn(__int2float_rn(acc), xs_s[t]), sw);
+                if (acc_out) acc_out[size_t(t) * r + j] = acc;
+            }
+        }
+    }
+    // second half of a3 + a4: the last CTA requantizes every row of c_hat
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) last = atomicAdd(counter, 1) == int(gridDim.x) - 1;
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    float *red8 = red;
+    static_assert(kRqThreads == kPsWarps * 32, "requant_row_cta expects one full CTA");
+    for (int t = 0; t < T; ++t)
+        requant_row_cta(c_hat, t, r, lat_bits, lat_clip, lat_codes, lat_scales, dst, dst_seq, dst_pos, err, red8);
+    if (threadIdx.x == 0) *counter = 0;
+}
+
+cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, const int8_t *wcodes,
+                              const float *ws, int r, int lat_bits, float lat_clip, float *c_hat, int *counter,
+                              int8_t *xq_out, float *xs_out, int32_t *acc_out, void *lat_codes, void *lat_scales,
+                              const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
+                              cudaStream_t s) {
+    CacheView dv{};
+    if (dst) dv = *dst;
+    const size_t smem = size_t(kPsWarps) * d + size_t(T) * d;
+    cudaError_t e = ensure_smem(proj_small_kernel, smem);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(proj_small_kernel, dim3((r + kPsWarps - 1) / kPsWarps), dim3(kPsWarps * 32), smem, s, X, T, d,
+                   act_clip, wcodes, ws, r, lat_bits, lat_clip, c_hat, counter, xq_out, xs_out, acc_out, lat_codes,
+                   lat_scales, dv, dst_seq, dst_pos, err);
+    prof_mark(s, "proj_small");
+    return e;
+}
+
 cudaError_t launch_proj_dp4a(const int8_t *xq, int64_t T, int d, const int8_t *wcodes, const float *ws,
                              const float *xs, int r, float *c_hat, int32_t *acc_out, cudaStream_t s) {
     if (T == 0) return cudaSuccess;
     dim3 grid((r + kPjWarps - 1) / kPjWarps, unsigned((T + kPjTokens - 1) / kPjTokens));
-    proj_dp4a_kernel<<<grid, kPjWarps * 32, 0, s>>>(xq, T, d, wcodes, ws, xs, r, c_hat, acc_out);
+    cudaError_t e = launch_pdl(proj_dp4a_kernel, grid, dim3(kPjWarps * 32), 0, s, xq, T, d, wcodes, ws, xs, r,
+                               c_hat, acc_out);
     prof_mark(s, "proj_dp4a");
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace qsvd

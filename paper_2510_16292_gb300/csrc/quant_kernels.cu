@@ -25,6 +25,8 @@ xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int8_t *__restr
     __shared__ float red[kXqThreads / 32];
     const int64_t t = blockIdx.x;
     const uint16_t *x = X + t * d;
+    pdl_trigger();
+    pdl_wait();
     float m = 0.0f;
     for (int i = threadIdx.x * 8; i < d; i += kXqThreads * 8) {
         float f[8];
@@ -60,13 +62,13 @@ cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip, int8_
     if (T == 0) return cudaSuccess;
     const size_t smem = size_t(d) * sizeof(float);
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(xquant_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             int(smem));
+        cudaError_t e = ensure_smem(xquant_kernel, smem);
         if (e != cudaSuccess) return e;
     }
-    xquant_kernel<<<dim3(unsigned(T)), kXqThreads, smem, s>>>(X, d, clip, xq, xq_bf16, xs);
+    cudaError_t e = launch_pdl(xquant_kernel, dim3(unsigned(T)), dim3(kXqThreads), smem, s, X, d, clip, xq,
+                               xq_bf16, xs);
     prof_mark(s, "xquant");
-    return cudaGetLastError();
+    return e;
 }
 
 // ---------------------------------------------------------------------------
@@ -107,93 +109,17 @@ cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int
 }
 
 // ---------------------------------------------------------------------------
-// a3/a4: requantize one latent row per CTA.  Each thread owns groups of 4
-// consecutive channels (one float4); an int4 group of 128 channels is one
-// warp's float4 row (32 lanes x 4), so its absmax is a warp reduction.
+// a3/a4: requantize one latent row per CTA (requant_row_cta, common.cuh).
 // ---------------------------------------------------------------------------
-constexpr int kRqThreads = 256;
-constexpr int kRqMaxQuads = 4;     // r <= 4096
-
 __global__ void __launch_bounds__(kRqThreads)
 requant_kernel(const float *__restrict__ c_hat, int r, int bits, float clip,
                void *__restrict__ lat_codes, void *__restrict__ lat_scales, CacheView dst,
                const int32_t *__restrict__ dst_seq, const int32_t *__restrict__ dst_pos,
                int *err) {
     __shared__ float red[kRqThreads / 32];
-    const int64_t t = blockIdx.x;
-    const float *row = c_hat + t * r;
-    const int nq = r / 4;
-    float4 v[kRqMaxQuads];
-#pragma unroll
-    for (int k = 0; k < kRqMaxQuads; ++k) {
-        const int qi = threadIdx.x + k * kRqThreads;
-        v[k] = qi < nq ? reinterpret_cast<const float4 *>(row)[qi] : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    // cache destination of this row (if any), bounds-checked
-    uint8_t *cache_codes = nullptr;
-    void *cache_scale = nullptr;
-    if (dst.codes) {
-        const int b = dst_seq[t], p = dst_pos[t];
-        if (b < 0 || b >= dst.B || p < 0 || p >= dst.Tmax) {
-            if (threadIdx.x == 0) flag_error(err, kErrRange);
-        } else {
-            const size_t slot = size_t(b) * dst.Tmax + p;
-            if (bits == 8) {
-                cache_codes = static_cast<uint8_t *>(dst.codes) + slot * r;
-                cache_scale = static_cast<float *>(dst.scales) + slot;
-            } else {
-                cache_codes = static_cast<uint8_t *>(dst.codes) + slot * (r / 2);
-                cache_scale = static_cast<__half *>(dst.scales) + slot * (r / 128);
-            }
-        }
-    }
-    uint8_t *tok_codes = lat_codes ? static_cast<uint8_t *>(lat_codes) + t * (bits == 8 ? r : r / 2)
-                                   : nullptr;
-
-    if (bits == 8) {
-        float m = 0.0f;
-#pragma unroll
-        for (int k = 0; k < kRqMaxQuads; ++k)
-            m = fmaxf(m, fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w))));
-        m = block_max<kRqThreads>(m, red);
-        const float s = quant_scale(m, clip, 127.0f);
-#pragma unroll
-        for (int k = 0; k < kRqMaxQuads; ++k) {
-            const int qi = threadIdx.x + k * kRqThreads;
-            if (qi >= nq) break;
-            const uint32_t w = uint32_t(quant_code(v[k].x, s, 127) & 0xff) |
-                               (uint32_t(quant_code(v[k].y, s, 127) & 0xff) << 8) |
-                               (uint32_t(quant_code(v[k].z, s, 127) & 0xff) << 16) |
-                               (uint32_t(quant_code(v[k].w, s, 127) & 0xff) << 24);
-            if (tok_codes) reinterpret_cast<uint32_t *>(tok_codes)[qi] = w;
-            if (cache_codes) reinterpret_cast<uint32_t *>(cache_codes)[qi] = w;
-        }
-        if (threadIdx.x == 0) {
-            if (lat_scales) static_cast<float *>(lat_scales)[t] = s;
-            if (cache_scale) *static_cast<float *>(cache_scale) = s;
-        }
-    } else {
-        // quad qi covers channels 4qi..4qi+3; its group is qi / 32 = one warp row
-#pragma unroll
-        for (int k = 0; k < kRqMaxQuads; ++k) {
-            const int qi = threadIdx.x + k * kRqThreads;
-            if (qi - (threadIdx.x & 31) >= nq) break;       // warp-uniform
-            float m = fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w)));
-            m = warp_max(m);
-            const __half hs = int4_group_scale(m, clip);
-            const float s = __half2float(hs);
-            const int c0 = quant_code(v[k].x, s, 7), c1 = quant_code(v[k].y, s, 7);
-            const int c2 = quant_code(v[k].z, s, 7), c3 = quant_code(v[k].w, s, 7);
-            const uint16_t w = uint16_t((c0 & 0xf) | ((c1 & 0xf) << 4) | ((c2 & 0xf) << 8) | ((c3 & 0xf) << 12));
-            if (tok_codes) reinterpret_cast<uint16_t *>(tok_codes)[qi] = w;
-            if (cache_codes) reinterpret_cast<uint16_t *>(cache_codes)[qi] = w;
-            if ((threadIdx.x & 31) == 0) {
-                const int g = qi >> 5;
-                if (lat_scales) static_cast<__half *>(lat_scales)[t * (r / 128) + g] = hs;
-                if (cache_scale) static_cast<__half *>(cache_scale)[g] = hs;
-            }
-        }
-    }
+    pdl_trigger();
+    pdl_wait();
+    requant_row_cta(c_hat, blockIdx.x, r, bits, clip, lat_codes, lat_scales, dst, dst_seq, dst_pos, err, red);
 }
 
 cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float clip, void *lat_codes,
@@ -202,10 +128,10 @@ cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float
     if (T == 0) return cudaSuccess;
     CacheView d{};
     if (dst) d = *dst;
-    requant_kernel<<<dim3(unsigned(T)), kRqThreads, 0, s>>>(c_hat, r, bits, clip, lat_codes, lat_scales, d,
-                                                             dst_seq, dst_pos, err);
+    cudaError_t e = launch_pdl(requant_kernel, dim3(unsigned(T)), dim3(kRqThreads), 0, s, c_hat, r, bits, clip,
+                               lat_codes, lat_scales, d, dst_seq, dst_pos, err);
     prof_mark(s, "requant");
-    return cudaGetLastError();
+    return e;
 }
 
 // ---------------------------------------------------------------------------
@@ -216,6 +142,8 @@ append_kernel(CacheView c, const int32_t *__restrict__ seq, const int32_t *__res
               const uint8_t *__restrict__ codes, const uint8_t *__restrict__ scales, int *err) {
     const int64_t i = int64_t(blockIdx.x) * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
+    pdl_trigger();
+    pdl_wait();
     if (i >= n) return;
     const int b = seq[i], p = pos[i];
     if (b < 0 || b >= c.B || p < 0 || p >= c.Tmax) {
@@ -235,10 +163,10 @@ append_kernel(CacheView c, const int32_t *__restrict__ seq, const int32_t *__res
 cudaError_t launch_append(const CacheView &c, const int32_t *seq, const int32_t *pos, int64_t n,
                           const void *lat_codes, const void *lat_scales, int *err, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
-    append_kernel<<<dim3(unsigned((n + 7) / 8)), 256, 0, s>>>(
-        c, seq, pos, n, static_cast<const uint8_t *>(lat_codes), static_cast<const uint8_t *>(lat_scales), err);
+    cudaError_t e = launch_pdl(append_kernel, dim3(unsigned((n + 7) / 8)), dim3(256), 0, s, c, seq, pos, n,
+                               static_cast<const uint8_t *>(lat_codes), static_cast<const uint8_t *>(lat_scales), err);
     prof_mark(s, "append");
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace qsvd
