@@ -153,6 +153,9 @@ class NativeBench:
         self.wsp = torch.zeros(q.qsvd_project_workspace_bytes(B * P, s.d, s.r), dtype=torch.uint8, device=dev)
         self.wsd = torch.zeros(q.qsvd_decode_workspace_bytes(B, wl.tmax, s.r, s.H, s.dh), dtype=torch.uint8,
                                device=dev)
+        self.fused = False          # the PDL-chained calls are faster than the fused step today
+        self.wsf = torch.zeros(max(1, q.qsvd_decode_step_workspace_bytes(B, wl.tmax, s.d, s.r, s.H, s.dh)),
+                               dtype=torch.uint8, device=dev)
         self.flushbuf = torch.ones(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
         self.flush_out = torch.zeros((), dtype=torch.int64, device=dev)
         self.stream = torch.cuda.current_stream()
@@ -172,6 +175,7 @@ class NativeBench:
                          None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st)
         self.dec_proj = []
         self.dec_attn = []
+        self.dec_fused = []
         for t in range(self.S):
             self.dec_proj.append((ctypes.byref(self.cW), self.Xd[t].data_ptr(), self.B, 1.0, wl.lat_bits, 1.0,
                                   None, None, ctypes.byref(self.cC), self.dseq.data_ptr(), self.dpos[t].data_ptr(),
@@ -180,6 +184,11 @@ class NativeBench:
                                   self.U[0].data_ptr(), self.U[1].data_ptr(), self.U[2].data_ptr(), s.H, s.dh,
                                   1.0 / math.sqrt(s.dh), self.O.data_ptr(), self.wsd.data_ptr(),
                                   self.wsd.numel(), st))
+            self.dec_fused.append((ctypes.byref(self.cW), self.Xd[t].data_ptr(), ctypes.byref(self.cC),
+                                   self.dlen[t].data_ptr(), self.P + t + 1, self.U[0].data_ptr(),
+                                   self.U[1].data_ptr(), self.U[2].data_ptr(), s.H, s.dh, 1.0, 1.0,
+                                   1.0 / math.sqrt(s.dh), self.O.data_ptr(), self.wsf.data_ptr(),
+                                   self.wsf.numel(), st))
 
     def build_graph(self):
         """Capture one whole step (flushes, sub-step events and every C-ABI
@@ -209,8 +218,11 @@ class NativeBench:
         self._call(self.lib.qsvd_latent_project, self.pre_args)
 
     def decode(self, t):
-        self._call(self.lib.qsvd_latent_project, self.dec_proj[t])
-        self._call(self.lib.qsvd_latent_decode_attn, self.dec_attn[t])
+        if self.fused:
+            self._call(self.lib.qsvd_decode_step, self.dec_fused[t])
+        else:
+            self._call(self.lib.qsvd_latent_project, self.dec_proj[t])
+            self._call(self.lib.qsvd_latent_decode_attn, self.dec_attn[t])
 
     def flush(self):
         """Evict L2 by reading a 256 MiB buffer (leaves L2 clean, unlike a write)."""
@@ -297,6 +309,8 @@ class NativeBench:
             return B * L * (tok + stok) + 4 * B * H * r
         if label == "combine_uv":
             return r * d * 2 + 4 * B * d
+        if label == "decode_step":
+            return self.step_roofline_bytes(ctx[1])
         return 0
 
     def step_roofline_bytes(self, t):

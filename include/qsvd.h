@@ -178,6 +178,30 @@ int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int
 size_t qsvd_decode_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t r, int32_t H, int32_t dh);
 
 /*
+ * One whole decode step for a small batch, in a single launch: for each of
+ * the B = cache->B sequences, the new token X[b] (bf16 [B, d]) is quantized
+ * and projected (Eq. 12), its latent is requantized and stored at position
+ * seq_len[b] - 1 of sequence b (Eq. 11, Fig. 2(f)), and attention over
+ * positions 0 .. seq_len[b]-1 is computed as in qsvd_latent_decode_attn
+ * (Eq. 5).  The result equals qsvd_latent_project(dst = cache,
+ * dst_seq = b, dst_pos = seq_len[b] - 1) followed by qsvd_latent_decode_attn,
+ * with the same arithmetic; it exists because a small-batch decode step is
+ * bound by launch latency rather than by its bytes.
+ * The launch is cooperative (one CTA per SM, grid-wide barriers whose waits
+ * are bounded: an expired wait abandons the step and flags QSVD_ETIMEOUT).
+ * Requirements: B <= 8; d = H*dh, d % 256 == 0, d <= 6144; r <= 3072;
+ * dh in {64, 128}.  workspace: qsvd_decode_step_workspace_bytes(...) bytes.
+ */
+int qsvd_decode_step(const qsvd_down_weight *W, const uint16_t *X, const qsvd_cache *cache,
+                     const int32_t *seq_len, int32_t max_seq_len,
+                     const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v,
+                     int32_t H, int32_t dh, float act_clip, float lat_clip, float softmax_scale,
+                     float *O, void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+size_t qsvd_decode_step_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t d, int32_t r,
+                                        int32_t H, int32_t dh);
+
+/*
  * Synchronizes `stream`, then reads and clears the device error word.
  * Returns QSVD_OK, QSVD_ERANGE, QSVD_ETIMEOUT or QSVD_ECUDA.
  */

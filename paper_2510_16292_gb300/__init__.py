@@ -31,6 +31,7 @@ QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
 EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
+           "qsvd_decode_step", "qsvd_decode_step_workspace_bytes",
            "qsvd_check", "qsvd_last_error", "qsvd_version")
 
 
@@ -61,6 +62,10 @@ _lib.qsvd_latent_decode_attn.argtypes = [ctypes.POINTER(_Cache), _vp, _i32, _vp,
                                          _vp, _vp, _sz, _vp]
 _lib.qsvd_decode_workspace_bytes.argtypes = [_i32, _i32, _i32, _i32, _i32]
 _lib.qsvd_decode_workspace_bytes.restype = _sz
+_lib.qsvd_decode_step.argtypes = [ctypes.POINTER(_DownWeight), _vp, ctypes.POINTER(_Cache), _vp, _i32, _vp, _vp,
+                                  _vp, _i32, _i32, _f32, _f32, _f32, _vp, _vp, _sz, _vp]
+_lib.qsvd_decode_step_workspace_bytes.argtypes = [_i32, _i32, _i32, _i32, _i32, _i32]
+_lib.qsvd_decode_step_workspace_bytes.restype = _sz
 _lib.qsvd_check.argtypes = [_vp]
 _lib.qsvd_last_error.restype = ctypes.c_char_p
 
@@ -192,6 +197,27 @@ def qsvd_latent_decode_attn(cache: LatentCache, seq_len: torch.Tensor, max_seq_l
     _check(_lib.qsvd_latent_decode_attn(ctypes.byref(cc), _ptr(seq_len), max_seq_len, _ptr(U_q), _ptr(U_k),
                                         _ptr(U_v), H, dh, softmax_scale, _ptr(O), _ptr(workspace),
                                         workspace.numel(), _stream(stream)))
+
+
+def qsvd_decode_step_workspace_bytes(B: int, max_seq_len: int, d: int, r: int, H: int, dh: int) -> int:
+    return int(_lib.qsvd_decode_step_workspace_bytes(B, max_seq_len, d, r, H, dh))
+
+
+def qsvd_decode_step(W: DownWeight, X: torch.Tensor, cache: LatentCache, seq_len: torch.Tensor, max_seq_len: int,
+                     U_q, U_k, U_v, H: int, dh: int, O: torch.Tensor, act_clip: float = 1.0,
+                     lat_clip: float = 1.0, softmax_scale: Optional[float] = None, workspace=None,
+                     stream=None) -> None:
+    """Fused decode step: project the new token of every sequence, store its
+    latent at position seq_len[b] - 1, attend over positions < seq_len[b]."""
+    if softmax_scale is None:
+        softmax_scale = 1.0 / math.sqrt(dh)
+    if workspace is None:
+        workspace = torch.zeros(qsvd_decode_step_workspace_bytes(cache.B, max_seq_len, W.d, W.r, H, dh),
+                                dtype=torch.uint8, device=O.device)
+    cw, cc = W._c(), cache._c()
+    _check(_lib.qsvd_decode_step(ctypes.byref(cw), _ptr(X), ctypes.byref(cc), _ptr(seq_len), max_seq_len,
+                                 _ptr(U_q), _ptr(U_k), _ptr(U_v), H, dh, act_clip, lat_clip, softmax_scale,
+                                 _ptr(O), _ptr(workspace), workspace.numel(), _stream(stream)))
 
 
 def qsvd_check(stream=None) -> int:

@@ -297,4 +297,43 @@ int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "decode_attn launch");
 }
 
+size_t qsvd_decode_step_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t d, int32_t r, int32_t H,
+                                        int32_t dh) {
+    if (B <= 0 || max_seq_len <= 0 || d <= 0 || r <= 0 || H <= 0 || dh <= 0) return 0;
+    return fused_workspace_bytes(B, max_seq_len, d, r, H, dh);
+}
+
+int qsvd_decode_step(const qsvd_down_weight *W, const uint16_t *X, const qsvd_cache *cache, const int32_t *seq_len,
+                     int32_t max_seq_len, const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v, int32_t H,
+                     int32_t dh, float act_clip, float lat_clip, float softmax_scale, float *O, void *workspace,
+                     size_t workspace_bytes, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if ((st = check_cache(cache))) return st;
+    if (!W || !W->codes || !W->scale || !X || !seq_len || !U_q || !U_k || !U_v || !O)
+        return fail(QSVD_EINVAL, "decode_step: null pointer");
+    const int d = W->d, r = W->r;
+    if (r != cache->r) return fail(QSVD_EINVAL, "decode_step: weight rank differs from the cache's");
+    if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "decode_step: dh must be 64 or 128");
+    if (H <= 0 || H * dh != d) return fail(QSVD_EINVAL, "decode_step: H * dh must equal d");
+    if (d % 256 || d > 6144) return fail(QSVD_EUNSUPPORTED, "decode_step: need d %% 256 == 0 and d <= 6144");
+    if (r > 3072) return fail(QSVD_EUNSUPPORTED, "decode_step: r > 3072");
+    if (cache->B > kFuseMaxB) return fail(QSVD_EUNSUPPORTED, "decode_step: more than %d sequences", kFuseMaxB);
+    if (max_seq_len < 1 || max_seq_len > cache->Tmax)
+        return fail(QSVD_EINVAL, "decode_step: max_seq_len outside [1, Tmax]");
+    if (!(act_clip > 0.0f && act_clip <= 1.0f) || !(lat_clip > 0.0f && lat_clip <= 1.0f))
+        return fail(QSVD_EINVAL, "decode_step: clip ratios must lie in (0, 1]");
+    const void *ptrs[] = {X, W->codes, W->scale, U_q, U_k, U_v, O, workspace};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(QSVD_EINVAL, "decode_step: pointers must be 16-byte aligned");
+    const size_t need = fused_workspace_bytes(cache->B, max_seq_len, d, r, H, dh);
+    if (!workspace || workspace_bytes < need) return fail(QSVD_ENOSPC, "decode_step: workspace needs %zu bytes", need);
+    FusedArgs a{X, W->codes, W->scale, view(cache), seq_len, max_seq_len, U_q, U_k, U_v, d, H, dh,
+                act_clip, lat_clip, softmax_scale, O};
+    prof_mark(stream, "begin");
+    cudaError_t e = launch_decode_fused(a, workspace, workspace_bytes, err, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "decode_step launch");
+}
+
 }  // extern "C"

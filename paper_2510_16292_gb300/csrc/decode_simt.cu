@@ -461,16 +461,19 @@ combine_uv_kernel(const int32_t *__restrict__ seq_len, int B, int Tmax, int H, i
         const int ns = (L + chunk - 1) / chunk;
         const size_t base = size_t(b) * n_split * H + h;
         __syncthreads();
-        if (threadIdx.x == 0) {
-            float M = -FLT_MAX;
-            for (int s = 0; s < ns; ++s) M = fmaxf(M, pm[base + size_t(s) * H]);
-            float l = 0.0f;
-            for (int s = 0; s < ns; ++s) {
-                const float w = expf(pm[base + size_t(s) * H] - M);
-                wsp[s] = w;
-                l += w * pl[base + size_t(s) * H];
-            }
-            inv_l = 1.0f / l;
+        if (threadIdx.x < 32) {                 // ns <= 64: two partials per lane
+            const int lane = threadIdx.x;
+            const float m0 = lane < ns ? pm[base + size_t(lane) * H] : -FLT_MAX;
+            const float m1 = lane + 32 < ns ? pm[base + size_t(lane + 32) * H] : -FLT_MAX;
+            const float l0 = lane < ns ? pl[base + size_t(lane) * H] : 0.0f;
+            const float l1 = lane + 32 < ns ? pl[base + size_t(lane + 32) * H] : 0.0f;
+            const float M = warp_max(fmaxf(m0, m1));
+            const float w0 = lane < ns ? expf(m0 - M) : 0.0f;
+            const float w1 = lane + 32 < ns ? expf(m1 - M) : 0.0f;
+            wsp[lane] = w0;
+            wsp[lane + 32] = w1;
+            const float l = warp_sum(w0 * l0 + w1 * l1);
+            if (lane == 0) inv_l = 1.0f / l;
         }
         __syncthreads();
         for (int jj = threadIdx.x; jj < rows; jj += blockDim.x) {

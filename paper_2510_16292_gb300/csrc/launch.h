@@ -103,6 +103,23 @@ struct DecodeArgs {
     float *O;
 };
 size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
+
+// One fused decode step (a1-a8) for B <= kFuseMaxB sequences, one new token each.
+constexpr int kFuseMaxB = 8;
+struct FusedArgs {
+    const uint16_t *X;
+    const int8_t *w_codes;
+    const float *w_scale;
+    CacheView cache;
+    const int32_t *seq_len;
+    int max_seq_len;
+    const uint16_t *U_q, *U_k, *U_v;
+    int d, H, dh;
+    float act_clip, lat_clip, softmax_scale;
+    float *O;
+};
+size_t fused_workspace_bytes(int B, int max_seq_len, int d, int r, int H, int dh);
+cudaError_t launch_decode_fused(const FusedArgs &a, void *ws, size_t ws_bytes, int *err, cudaStream_t s);
 cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *err,
                           cudaStream_t s);
 

@@ -72,6 +72,15 @@ class GpuLayer:
                                      dst=self.cache, dst_seq=i32(np.full(T, b)), dst_pos=i32(pos))
         self.len[b] += T
 
+    def decode_step_fused(self, x_bits):
+        """One decode step through the single-launch entry point."""
+        B = self.B
+        self.len += 1
+        O = torch.empty((B, self.s.d), dtype=torch.float32, device=dev())
+        self.lib.qsvd_decode_step(self.W, bf16(x_bits), self.cache, i32(self.len), int(self.len.max()), self.U_q,
+                                  self.U_k, self.U_v, self.s.H, self.s.dh, O, self.act_clip, self.lat_clip)
+        return O
+
     def decode_step(self, x_bits):
         B = self.B
         self.lib.qsvd_latent_project(self.W, bf16(x_bits), self.act_clip, self.bits, self.lat_clip,

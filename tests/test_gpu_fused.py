@@ -1,0 +1,71 @@
+"""GPU parity of the single-launch decode step (qsvd_decode_step) against the
+CPU oracle: cache codes bit-exact, outputs within 2e-3 * ||o_ref||_2."""
+import numpy as np
+import pytest
+
+import synthetic
+from oracle import pipeline
+
+from gpu_util import GpuLayer, assert_rows_close, q
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(wl, inp, w, steps, check, lens=None):
+    s = wl.shape
+    ref = pipeline.OracleLayer(s, w, wl.B, wl.tmax, wl.lat_bits)
+    gpu = GpuLayer(s, w, wl.B, wl.tmax, wl.lat_bits)
+    for b in range(wl.B):
+        n = wl.prefill if lens is None else lens[b]
+        ref.prefill(b, inp.X_prefill[b][:n])
+        gpu.prefill(b, inp.X_prefill[b][:n])
+    for step in range(steps):
+        _, outs = ref.decode_step(inp.X_decode[step], attend=None if step in check else [])
+        O = gpu.decode_step_fused(inp.X_decode[step])
+        if step in check:
+            q().qsvd_check()
+            assert_rows_close(O.cpu().numpy(), np.stack([outs[b] for b in range(wl.B)]), f"step {step}")
+    q().qsvd_check()
+    for b in range(wl.B):
+        L = int(ref.len[b])
+        np.testing.assert_array_equal(gpu.cache.codes[b, :L].cpu().numpy().view(np.uint8),
+                                      ref.cache.packed_codes()[b, :L].view(np.uint8))
+        np.testing.assert_array_equal(gpu.cache.scales[b, :L].cpu().numpy().astype(np.float64), ref.cache.scale[b, :L])
+
+
+def test_fused_tiny_all_steps():
+    wl = synthetic.WORKLOADS["tiny"]
+    inp = synthetic.gen_layer(wl, seed=0)
+    _run(wl, inp, pipeline.prepare_weights(inp), wl.decode_steps, set(range(wl.decode_steps)))
+
+
+def test_fused_7b_sampled():
+    wl = synthetic.WORKLOADS["llava7b"]
+    inp = synthetic.gen_layer(wl, seed=0)
+    _run(wl, inp, pipeline.prepare_weights(inp), wl.decode_steps, {0, 64, wl.decode_steps - 1})
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_fused_batch_ragged(bits):
+    base = synthetic.WORKLOADS["llava7b"]
+    wl = synthetic.Workload("ragged", base.shape, B=3, n_image=0, n_text=300, decode_steps=2, lat_bits=bits)
+    inp = synthetic.gen_layer(wl, seed=7)
+    _run(wl, inp, pipeline.prepare_weights(inp), 2, {0, 1}, lens=[1, 63, 300])
+
+
+def test_fused_13b_shape():
+    base = synthetic.WORKLOADS["llava13b"]
+    wl = synthetic.Workload("13b_small", base.shape, B=2, n_image=200, n_text=40, decode_steps=2, lat_bits=8)
+    inp = synthetic.gen_layer(wl, seed=4)
+    _run(wl, inp, pipeline.prepare_weights(inp), 2, {0, 1})
+
+
+def test_fused_rejects_large_batch():
+    lib = q()
+    base = synthetic.WORKLOADS["llava7b"]
+    wl = synthetic.Workload("big", base.shape, B=9, n_image=0, n_text=4, decode_steps=1, lat_bits=8)
+    inp = synthetic.gen_layer(wl, seed=1)
+    gpu = GpuLayer(wl.shape, pipeline.prepare_weights(inp), wl.B, wl.tmax, 8)
+    with pytest.raises(lib.QsvdError) as e:
+        gpu.decode_step_fused(inp.X_decode[0])
+    assert e.value.status == lib.QSVD_EUNSUPPORTED
