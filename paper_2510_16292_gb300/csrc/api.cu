@@ -185,7 +185,8 @@ size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r) {
     return 256 +                                // completion counter (zero at rest)
            align256(size_t(T) * d) +            // int8 codes of X
            align256(size_t(T) * 4) +            // s_x
-           align256(size_t(T) * r * 4);         // dequantized latent c_hat
+           align256(size_t(T) * r * 4) +        // dequantized latent c_hat
+           align256(size_t(T) * d * 2);         // bf16 image of the X codes (tensor-core operand)
 }
 
 int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T, float act_clip,
@@ -230,6 +231,8 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
     float *xs = xs_out ? xs_out : reinterpret_cast<float *>(wsp);
     wsp += align256(size_t(T) * 4);
     float *c_hat = reinterpret_cast<float *>(wsp);
+    wsp += align256(size_t(T) * r * 4);
+    uint16_t *xq_bf16 = reinterpret_cast<uint16_t *>(wsp);
     CacheView dv{};
     if (dst) dv = view(dst);
 
@@ -241,10 +244,18 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
                               err, stream);
         return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "projection launch");
     }
-    e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
-    e = launch_proj_dp4a(xq, T, d, W->codes, W->scale, xs, r, c_hat, acc_out, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "projection launch");
+    if (W->codes_bf16 && gemm_tc_supported(d, r)) {
+        if (!aligned16(W->codes_bf16)) return fail(QSVD_EINVAL, "latent_project: codes_bf16 must be 16-byte aligned");
+        e = launch_xquant(X, T, d, act_clip, xq_out, xq_bf16, xs, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
+        e = launch_gemm_tc(xq_bf16, T, d, W->codes_bf16, W->scale, xs, r, c_hat, acc_out, err, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "tensor-core projection launch");
+    } else {
+        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
+        e = launch_proj_dp4a(xq, T, d, W->codes, W->scale, xs, r, c_hat, acc_out, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "projection launch");
+    }
     e = launch_requant(c_hat, T, r, lat_bits, lat_clip, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
                        dst_pos, err, stream);
     if (e != cudaSuccess) return cuda_fail(e, "requant launch");

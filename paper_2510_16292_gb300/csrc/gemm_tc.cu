@@ -1,0 +1,266 @@
+// Exact int8 x int8 -> int32 down-projection on the 5th-generation tensor
+// cores (a2 + the fp32 dequantization of a3), for prefill-sized T.
+//
+// sm_103a has no integer tcgen05 MMA, so the int8 codes are fed as bf16
+// values (every integer in [-127, 127] is exact in bf16, every product
+// |x w| <= 127^2 is exact in fp32) to tcgen05.mma.kind::f16 with an fp32
+// accumulator in tensor memory.  A partial sum of up to 1024 such products
+// stays below 2^24, so it is an exact integer in fp32 regardless of the
+// order the tensor core adds in; the accumulator is therefore drained into
+// int32 registers every kChunkK = 1024 of the reduction dimension, and the
+// int32 sum over chunks is the exact integer product.
+//
+// CTA tile 128 (tokens) x 128 (latent channels), K staged 64 at a time.
+//   warp 0      TMA producer: 2D tiles of X-codes [T, d] and W-codes [r, d]
+//               (both K-major, 128-byte swizzle) into a kStages-deep ring
+//   warp 1      allocates tensor memory; lane 0 issues the MMAs (M=128,
+//               N=128, K=16) and commits stage releases / chunk completions
+//   warps 2-5   epilogue: drain each chunk's accumulator (tcgen05.ld) into
+//               int32 registers, then c_hat = (fp32(acc) * s_x[t]) * s_w[j]
+// Two 128-column accumulators alternate between chunks so that the MMA of
+// chunk c+1 overlaps the drain of chunk c.
+#include <cuda.h>
+
+#include "common.cuh"
+#include "launch.h"
+
+namespace qsvd {
+
+constexpr int kBM = 128, kBN = 128, kBK = 64;
+constexpr int kStages = 6;
+constexpr int kChunkK = 1024;                  // <= 2^24 / 127^2 products per exact fp32 partial
+constexpr int kGemmThreads = 192;
+constexpr int kStageA = kBM * kBK * 2;         // 16 KiB
+constexpr int kStageB = kBN * kBK * 2;         // 16 KiB
+constexpr size_t kGemmSmem = size_t(kStages) * (kStageA + kStageB) + 1024;   // + alignment slack
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(smem_addr(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+        : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (the layout TMA's 128B swizzle writes for 64 bf16 per row).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    return uint64_t((saddr & 0x3FFFF) >> 4) | (uint64_t(1) << 16) | (uint64_t(1024 >> 4) << 32) |
+           (uint64_t(1) << 46) | (uint64_t(2) << 61);
+}
+
+// Instruction descriptor: bf16 x bf16 -> f32, both K-major, M=128, N=128.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kBN >> 3) << 17) | (uint32_t(kBM >> 4) << 24);
+
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
+    asm volatile("{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+                 ::"r"(d_tmem), "l"(a), "l"(b), "r"(kIdesc), "r"(accumulate));
+}
+__device__ __forceinline__ void umma_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+                 ::"r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// 32 consecutive columns of this warp's 32 lanes.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kGemmThreads, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_w, int64_t T, int d,
+               int r, const float *__restrict__ xs, const float *__restrict__ ws, float *__restrict__ c_hat,
+               int32_t *__restrict__ acc_out, int *err) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sA = smem;                                    // [kStages][128 x 64] bf16, SW128
+    uint8_t *sB = smem + size_t(kStages) * kStageA;        // [kStages][128 x 64] bf16, SW128
+    __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages];
+    __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2];
+    __shared__ uint32_t tmem_base;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * kBN;
+    const int n_k = d / kBK;
+    const int stages_per_chunk = kChunkK / kBK;
+    const int n_chunks = (n_k + stages_per_chunk - 1) / stages_per_chunk;
+
+    pdl_trigger();
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&acc_full[s], 1);
+            mbar_init(&acc_empty[s], 4);      // one arrival per epilogue warp
+        }
+        mbar_init_fence();
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_x)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_w)) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                     ::"r"(smem_addr(&tmem_base)), "r"(2 * kBN));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+    pdl_wait();
+
+    if (warp == 0) {
+        // ---------------- TMA producer ----------------
+        if (lane == 0) {
+            for (int i = 0; i < n_k; ++i) {
+                const int s = i % kStages;
+                if (i >= kStages && !mbar_wait(&empty_bar[s], ((i / kStages) - 1) & 1, err)) break;
+                mbar_arrive_expect_tx(&full_bar[s], kStageA + kStageB);
+                tma_load_2d(sA + size_t(s) * kStageA, &map_x, i * kBK, m0, &full_bar[s]);
+                tma_load_2d(sB + size_t(s) * kStageB, &map_w, i * kBK, n0, &full_bar[s]);
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer ----------------
+        if (lane == 0) {
+            bool ok = true;
+            for (int c = 0; c < n_chunks && ok; ++c) {
+                const int buf = c & 1;
+                if (c >= 2) {
+                    ok = mbar_wait(&acc_empty[buf], ((c >> 1) - 1) & 1, err);
+                    tc_fence_after();
+                }
+                const uint32_t d_tmem = tmem + uint32_t(buf * kBN);
+                const int i0 = c * stages_per_chunk, i1 = min(n_k, i0 + stages_per_chunk);
+                for (int i = i0; i < i1 && ok; ++i) {
+                    const int s = i % kStages;
+                    ok = mbar_wait(&full_bar[s], (i / kStages) & 1, err);
+                    if (!ok) break;
+                    tc_fence_after();
+                    const uint32_t a0 = smem_addr(sA + size_t(s) * kStageA);
+                    const uint32_t b0 = smem_addr(sB + size_t(s) * kStageB);
+#pragma unroll
+                    for (int ks = 0; ks < kBK / 16; ++ks)
+                        umma_bf16(d_tmem, sw128_desc(a0 + ks * 32), sw128_desc(b0 + ks * 32), (i > i0 || ks > 0) ? 1u : 0u);
+                    umma_commit(&empty_bar[s]);          // stage s may be refilled once these MMAs finish
+                }
+                if (ok) umma_commit(&acc_full[buf]);     // chunk c's partial sum is complete
+            }
+        }
+    } else {
+        // ---------------- epilogue (warps 2-5) ----------------
+        const int quad = warp & 3;                        // TMEM lane quadrant of this warp
+        const int row = quad * 32 + lane;                 // row of the tile (token)
+        int32_t acc[kBN];
+#pragma unroll
+        for (int j = 0; j < kBN; ++j) acc[j] = 0;
+        bool ok = true;
+        for (int c = 0; c < n_chunks && ok; ++c) {
+            const int buf = c & 1;
+            ok = mbar_wait(&acc_full[buf], (c >> 1) & 1, err);
+            tc_fence_after();
+            if (!ok) break;
+            const uint32_t taddr = tmem + (uint32_t(quad * 32) << 16) + uint32_t(buf * kBN);
+#pragma unroll
+            for (int j0 = 0; j0 < kBN; j0 += 32) {
+                uint32_t v[32];
+                tmem_ld32(taddr + j0, v);
+                tmem_ld_wait();
+#pragma unroll
+                for (int j = 0; j < 32; ++j) acc[j0 + j] += __float2int_rn(__uint_as_float(v[j]));
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&acc_empty[buf])) : "memory");
+        }
+        const int64_t t = m0 + row;
+        if (ok && t < T) {
+            const float sx = xs[t];
+            float *out = c_hat + t * r + n0;
+#pragma unroll
+            for (int j = 0; j < kBN; j += 4) {
+                float4 v;
+                v.x = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 0]), sx), ws[n0 + j + 0]);
+                v.y = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 1]), sx), ws[n0 + j + 1]);
+                v.z = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 2]), sx), ws[n0 + j + 2]);
+                v.w = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 3]), sx), ws[n0 + j + 3]);
+                *reinterpret_cast<float4 *>(out + j) = v;
+            }
+            if (acc_out) {
+                int32_t *ao = acc_out + t * r + n0;
+#pragma unroll
+                for (int j = 0; j < kBN; j += 4)
+                    *reinterpret_cast<int4 *>(ao + j) = make_int4(acc[j], acc[j + 1], acc[j + 2], acc[j + 3]);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * kBN));
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &p, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// bf16 matrix [rows, cols] row-major (cols contiguous), box [box_rows x 64 cols], 128B swizzle.
+static bool make_map(CUtensorMap *map, const void *base, int64_t rows, int cols, int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {cuuint64_t(cols), cuuint64_t(rows)};
+    const cuuint64_t strides[1] = {cuuint64_t(cols) * 2};
+    const cuuint32_t box[2] = {cuuint32_t(kBK), cuuint32_t(box_rows)};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool gemm_tc_supported(int d, int r) { return d % kBK == 0 && r % kBN == 0 && encode_fn() != nullptr; }
+
+cudaError_t launch_gemm_tc(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
+                           const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    CUtensorMap mx, mw;
+    if (!make_map(&mx, xq_bf16, T, d, kBM) || !make_map(&mw, w_bf16, r, d, kBN)) return cudaErrorInvalidValue;
+    cudaError_t e = ensure_smem(gemm_tc_kernel, kGemmSmem);
+    if (e != cudaSuccess) return e;
+    dim3 grid(unsigned((T + kBM - 1) / kBM), unsigned(r / kBN));
+    e = launch_pdl(gemm_tc_kernel, grid, dim3(kGemmThreads), kGemmSmem, s, mx, mw, T, d, r, xs, ws, c_hat, acc_out,
+                   err);
+    prof_mark(s, "gemm_tc");
+    return e;
+}
+
+}  // namespace qsvd

@@ -80,6 +80,12 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
                               const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
                               cudaStream_t s);
 
+// Exact int8 GEMM on the tensor cores (bf16 images of the codes, fp32 TMEM
+// accumulators drained to int32 every 1024 of K) + the fp32 dequantization.
+bool gemm_tc_supported(int d, int r);
+cudaError_t launch_gemm_tc(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
+                           const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s);
+
 // Per-token requantization of c_hat [T, r] into the latent format (a3 second
 // half), written token-major and/or into the cache (a4).
 cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float clip,

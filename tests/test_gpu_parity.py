@@ -253,3 +253,40 @@ def test_error_paths(tiny):
     with pytest.raises(lib.QsvdError) as e:
         lib.qsvd_check()
     assert e.value.status == lib.QSVD_ERANGE
+
+
+# ---------------------------------------------------------------------------
+# tensor-core projection: exactness at the extremes of the int8 range
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("d,r,T", [(4096, 1536, 200), (5120, 2048, 131)])
+def test_project_tc_worst_case_exact(d, r, T):
+    """Every code at +-127: |acc| = 127^2 d exceeds 2^24, so the result is
+    exact only if the fp32 tensor-core partial sums are drained to int32
+    before they leave the exact-integer range of fp32."""
+    lib = q()
+    rng = np.random.default_rng(d + r)
+    W = np.full((d, r), 0.01, dtype=np.float32)
+    W[:, 1::3] = -0.02                       # a third of the channels at -127
+    X = np.ones((T, d))
+    X[1::2, ::2] = -1.0                      # alternate signs along K on odd tokens
+    X[5] = rng.standard_normal(d)            # one ordinary row
+    Xb = synthetic.bf16_bits(X)
+    Wq = lib.qsvd_quantize_weight(torch.from_numpy(W).to(dev()))
+    got = _project_outputs(Wq, Xb, r, 8)
+    Wc, s_w = quant.quantize_columns(W.astype(np.float64), 8)
+    ref = latent.latent_project(synthetic.bf16_from_bits(Xb), Wc, s_w, lat_bits=8)
+    assert np.abs(ref["acc"]).max() > 2 ** 24
+    _assert_project_exact(got, ref, 8)
+
+
+def test_project_13b_shape_tc():
+    base = synthetic.WORKLOADS["llava13b"]
+    wl = synthetic.Workload("13b_proj", base.shape, B=1, n_image=300, n_text=0, decode_steps=0, lat_bits=8)
+    inp = synthetic.gen_layer(wl, seed=2)
+    w = pipeline.prepare_weights(inp)
+    W = q().qsvd_quantize_weight(torch.from_numpy(w["W_d"].astype(np.float32)).to(dev()))
+    X = inp.X_prefill[0]
+    for bits in (8, 4):
+        got = _project_outputs(W, X, wl.shape.r, bits)
+        ref = latent.latent_project(synthetic.bf16_from_bits(X), w["Wq"], w["s_w"], lat_bits=bits)
+        _assert_project_exact(got, ref, bits)
