@@ -52,6 +52,7 @@ def parse():
     p.add_argument("--impl", choices=["native", "reference"], default="native")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-prefill13", action="store_true")
     return p.parse_args()
 
 
@@ -361,6 +362,61 @@ class NativeBench:
         return self.B * self.S / dec_s, h2d, d2h
 
 
+def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
+    """Prefill projection at the LLaVA-13B batch shape (8 x (5 x 576 + 128)
+    tokens, d=5120, r=2048): time of the whole qsvd_latent_project call and of
+    its tensor-core GEMM kernel (library events), cold L2 before each call.
+    Inputs: seeded torch Gaussians (X with the outlier-channel pattern of the
+    synthetic recipe), W_d columns scaled by j^-0.5."""
+    import torch
+    import paper_2510_16292_gb300 as q
+    dev = torch.device("cuda", torch.cuda.current_device())
+    g = torch.Generator(device=dev)
+    g.manual_seed(1234)
+    X = torch.randn((T, d), generator=g, device=dev)
+    X[:, torch.randperm(d, generator=g, device=dev)[: d // 100]] *= 20
+    X = X.to(torch.bfloat16)
+    Wd = torch.randn((d, r), generator=g, device=dev) / math.sqrt(d)
+    Wd *= torch.arange(1, r + 1, device=dev, dtype=torch.float32) ** -0.5
+    W = q.qsvd_quantize_weight(Wd.contiguous())
+    lc = torch.empty((T, r), dtype=torch.int8, device=dev)
+    ls = torch.empty((T,), dtype=torch.float32, device=dev)
+    ws = torch.zeros(q.qsvd_project_workspace_bytes(T, d, r), dtype=torch.uint8, device=dev)
+    flush = torch.ones((256 << 20) // 4, dtype=torch.int32, device=dev)
+    sink = torch.zeros((), dtype=torch.int64, device=dev)
+    n = 16
+    events = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+    for e in events:
+        e.record()
+    torch.cuda.synchronize()
+    handles = (ctypes.c_void_p * n)(*[ctypes.c_void_p(e.cuda_event) for e in events])
+    lib = q._lib
+    lib.qsvd_profile_count.restype = ctypes.c_int32
+    lib.qsvd_profile_label.restype = ctypes.c_char_p
+    gemm, call = [], []
+    for it in range(iters + 1):
+        torch.sum(flush, dim=(0,), dtype=torch.int64, out=sink)
+        lib.qsvd_profile_events(handles, n)
+        q.qsvd_latent_project(W, X, lat_codes=lc, lat_scales=ls, workspace=ws)
+        torch.cuda.synchronize()
+        cnt = lib.qsvd_profile_count()
+        labels = [lib.qsvd_profile_label(i).decode() for i in range(cnt)]
+        lib.qsvd_profile_events(None, 0)
+        if it == 0:
+            continue
+        gi = labels.index("gemm_tc")
+        gemm.append(events[gi - 1].elapsed_time(events[gi]) * 1e-3)
+        call.append(events[0].elapsed_time(events[cnt - 1]) * 1e-3)
+    ops = 2.0 * T * d * r
+    _, bf16_peak, kind = peaks()
+    g_s, c_s = min(gemm), min(call)
+    del X, W, lc, ls, ws, flush
+    return {"shape": f"T={T} d={d} r={r} (8 x 3008 tokens, LLaVA-13B layer)", "gemm_us": round(g_s * 1e6, 2),
+            "gemm_tops": round(ops / g_s / 1e12, 1), "gemm_frac_of_bf16_peak": round(ops / g_s / 1e12 / bf16_peak, 4),
+            "project_call_us": round(c_s * 1e6, 2), "project_call_tops": round(ops / c_s / 1e12, 1),
+            "peak_kind": kind}
+
+
 def run_native(args, rank, world, local_rank):
     import torch
     torch.cuda.set_device(local_rank)
@@ -433,6 +489,7 @@ def run_native(args, rank, world, local_rank):
         e2e = {"value": round(e2e_val, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h}
 
+    pre13 = prefill_gemm_probe() if not args.no_prefill13 else None
     if rank != 0:
         return
     out = {
@@ -456,6 +513,7 @@ def run_native(args, rank, world, local_rank):
             "decode_step_roofline_us": round(roof_s / S * 1e6, 3),
             "wall_s_timed_region": round(t_wall, 3),
             "kernels": kernels,
+            "prefill_13b": pre13,
         },
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": None,

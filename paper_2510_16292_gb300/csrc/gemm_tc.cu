@@ -10,15 +10,19 @@
 // int32 registers every kChunkK = 1024 of the reduction dimension, and the
 // int32 sum over chunks is the exact integer product.
 //
-// CTA tile 128 (tokens) x 128 (latent channels), K staged 64 at a time.
+// CTA tile 128 (tokens) x BN (latent channels, 128 or 256), K staged 64 at
+// a time.
 //   warp 0      TMA producer: 2D tiles of X-codes [T, d] and W-codes [r, d]
-//               (both K-major, 128-byte swizzle) into a kStages-deep ring
+//               (both K-major, 128-byte swizzle) into a ring of stages
 //   warp 1      allocates tensor memory; lane 0 issues the MMAs (M=128,
-//               N=128, K=16) and commits stage releases / chunk completions
-//   warps 2-5   epilogue: drain each chunk's accumulator (tcgen05.ld) into
-//               int32 registers, then c_hat = (fp32(acc) * s_x[t]) * s_w[j]
-// Two 128-column accumulators alternate between chunks so that the MMA of
-// chunk c+1 overlaps the drain of chunk c.
+//               N=BN, K=16) and commits stage releases / chunk completions
+//   warps 2..   epilogue, BN/32 warps: warp w drains TMEM lane quadrant w%4,
+//               columns 128*((w-2)/4) .. +127, of each chunk's accumulator
+//               into int32 registers, then c_hat = (fp32(acc) s_x[t]) s_w[j]
+// Two BN-column accumulators alternate between chunks so that the MMA of
+// chunk c+1 overlaps the drain of chunk c.  A wide tile (BN=256) halves the
+// number of MMA instructions per byte and cuts L2 traffic per MAC by a
+// quarter; narrow tiles are kept for small T, where they give more CTAs.
 #include <cuda.h>
 
 #include "common.cuh"
@@ -26,13 +30,21 @@
 
 namespace qsvd {
 
-constexpr int kBM = 128, kBN = 128, kBK = 64;
-constexpr int kStages = 6;
+constexpr int kBM = 128, kBK = 64;
 constexpr int kChunkK = 1024;                  // <= 2^24 / 127^2 products per exact fp32 partial
-constexpr int kGemmThreads = 192;
 constexpr int kStageA = kBM * kBK * 2;         // 16 KiB
-constexpr int kStageB = kBN * kBK * 2;         // 16 KiB
-constexpr size_t kGemmSmem = size_t(kStages) * (kStageA + kStageB) + 1024;   // + alignment slack
+constexpr int kRingBytes = 192 * 1024;         // TMA ring (stages of A + B tiles)
+
+template <int BN> struct GemmCfg {
+    static constexpr int kStageB = BN * kBK * 2;
+    static constexpr int kStages = kRingBytes / (kStageA + kStageB);
+    static constexpr int kEpiWarps = BN / 32;
+    static constexpr int kThreads = 64 + 32 * kEpiWarps;
+    static constexpr size_t kSmem = size_t(kStages) * (kStageA + kStageB) + 1024;   // + alignment slack
+    // bf16 x bf16 -> f32, both K-major, M=128, N=BN
+    static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BN >> 3) << 17) |
+                                       (uint32_t(kBM >> 4) << 24);
+};
 
 // ---------------------------------------------------------------------------
 // PTX wrappers
@@ -51,13 +63,16 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
            (uint64_t(1) << 46) | (uint64_t(2) << 61);
 }
 
-// Instruction descriptor: bf16 x bf16 -> f32, both K-major, M=128, N=128.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(kBN >> 3) << 17) | (uint32_t(kBM >> 4) << 24);
-
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
     asm volatile("{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
                  "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
-                 ::"r"(d_tmem), "l"(a), "l"(b), "r"(kIdesc), "r"(accumulate));
+                 ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
+}
+// Spin on an mbarrier phase inline (no call), bounded; false on expiry.
+__device__ __forceinline__ bool spin_wait(uint64_t *bar, uint32_t parity, int *err) {
+    for (long i = 0; i < kWaitLimit; ++i)
+        if (mbar_try_wait(bar, parity)) return true;
+    return mbar_wait(bar, parity, err);     // flags the timeout, then a last bounded wait
 }
 __device__ __forceinline__ void umma_commit(uint64_t *bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
@@ -81,19 +96,22 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kGemmThreads, 1)
+template <int BN>
+__global__ void __launch_bounds__(GemmCfg<BN>::kThreads, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_w, int64_t T, int d,
                int r, const float *__restrict__ xs, const float *__restrict__ ws, float *__restrict__ c_hat,
                int32_t *__restrict__ acc_out, int *err) {
+    using C = GemmCfg<BN>;
+    constexpr int kStages = C::kStages, kStageB = C::kStageB;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sA = smem;                                    // [kStages][128 x 64] bf16, SW128
-    uint8_t *sB = smem + size_t(kStages) * kStageA;        // [kStages][128 x 64] bf16, SW128
+    uint8_t *sB = smem + size_t(kStages) * kStageA;        // [kStages][BN x 64] bf16, SW128
     __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages];
     __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2];
     __shared__ uint32_t tmem_base;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * kBN;
+    const int m0 = blockIdx.y * kBM, n0 = blockIdx.x * BN;      // N fastest: a wave shares X tiles
     const int n_k = d / kBK;
     const int stages_per_chunk = kChunkK / kBK;
     const int n_chunks = (n_k + stages_per_chunk - 1) / stages_per_chunk;
@@ -106,7 +124,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&acc_full[s], 1);
-            mbar_init(&acc_empty[s], 4);      // one arrival per epilogue warp
+            mbar_init(&acc_empty[s], C::kEpiWarps);   // one arrival per epilogue warp
         }
         mbar_init_fence();
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&map_x)) : "memory");
@@ -114,7 +132,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
-                     ::"r"(smem_addr(&tmem_base)), "r"(2 * kBN));
+                     ::"r"(smem_addr(&tmem_base)), "r"(2 * BN));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     tc_fence_before();
@@ -128,7 +146,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
         if (lane == 0) {
             for (int i = 0; i < n_k; ++i) {
                 const int s = i % kStages;
-                if (i >= kStages && !mbar_wait(&empty_bar[s], ((i / kStages) - 1) & 1, err)) break;
+                if (i >= kStages && !spin_wait(&empty_bar[s], ((i / kStages) - 1) & 1, err)) break;
                 mbar_arrive_expect_tx(&full_bar[s], kStageA + kStageB);
                 tma_load_2d(sA + size_t(s) * kStageA, &map_x, i * kBK, m0, &full_bar[s]);
                 tma_load_2d(sB + size_t(s) * kStageB, &map_w, i * kBK, n0, &full_bar[s]);
@@ -141,42 +159,44 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
             for (int c = 0; c < n_chunks && ok; ++c) {
                 const int buf = c & 1;
                 if (c >= 2) {
-                    ok = mbar_wait(&acc_empty[buf], ((c >> 1) - 1) & 1, err);
+                    ok = spin_wait(&acc_empty[buf], ((c >> 1) - 1) & 1, err);
                     tc_fence_after();
                 }
-                const uint32_t d_tmem = tmem + uint32_t(buf * kBN);
+                const uint32_t d_tmem = tmem + uint32_t(buf * BN);
                 const int i0 = c * stages_per_chunk, i1 = min(n_k, i0 + stages_per_chunk);
                 for (int i = i0; i < i1 && ok; ++i) {
                     const int s = i % kStages;
-                    ok = mbar_wait(&full_bar[s], (i / kStages) & 1, err);
+                    ok = spin_wait(&full_bar[s], (i / kStages) & 1, err);
                     if (!ok) break;
                     tc_fence_after();
                     const uint32_t a0 = smem_addr(sA + size_t(s) * kStageA);
                     const uint32_t b0 = smem_addr(sB + size_t(s) * kStageB);
 #pragma unroll
                     for (int ks = 0; ks < kBK / 16; ++ks)
-                        umma_bf16(d_tmem, sw128_desc(a0 + ks * 32), sw128_desc(b0 + ks * 32), (i > i0 || ks > 0) ? 1u : 0u);
+                        umma_bf16(d_tmem, sw128_desc(a0 + ks * 32), sw128_desc(b0 + ks * 32), C::kIdesc,
+                                  (i > i0 || ks > 0) ? 1u : 0u);
                     umma_commit(&empty_bar[s]);          // stage s may be refilled once these MMAs finish
                 }
                 if (ok) umma_commit(&acc_full[buf]);     // chunk c's partial sum is complete
             }
         }
     } else {
-        // ---------------- epilogue (warps 2-5) ----------------
+        // ---------------- epilogue (warps 2 .. 2 + kEpiWarps - 1) ----------------
         const int quad = warp & 3;                        // TMEM lane quadrant of this warp
+        const int col0 = ((warp - 2) >> 2) * 128;         // this warp's 128 columns of the tile
         const int row = quad * 32 + lane;                 // row of the tile (token)
-        int32_t acc[kBN];
+        int32_t acc[128];
 #pragma unroll
-        for (int j = 0; j < kBN; ++j) acc[j] = 0;
+        for (int j = 0; j < 128; ++j) acc[j] = 0;
         bool ok = true;
         for (int c = 0; c < n_chunks && ok; ++c) {
             const int buf = c & 1;
-            ok = mbar_wait(&acc_full[buf], (c >> 1) & 1, err);
+            ok = spin_wait(&acc_full[buf], (c >> 1) & 1, err);
             tc_fence_after();
             if (!ok) break;
-            const uint32_t taddr = tmem + (uint32_t(quad * 32) << 16) + uint32_t(buf * kBN);
+            const uint32_t taddr = tmem + (uint32_t(quad * 32) << 16) + uint32_t(buf * BN + col0);
 #pragma unroll
-            for (int j0 = 0; j0 < kBN; j0 += 32) {
+            for (int j0 = 0; j0 < 128; j0 += 32) {
                 uint32_t v[32];
                 tmem_ld32(taddr + j0, v);
                 tmem_ld_wait();
@@ -190,20 +210,21 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
         const int64_t t = m0 + row;
         if (ok && t < T) {
             const float sx = xs[t];
-            float *out = c_hat + t * r + n0;
+            const int nc = n0 + col0;
+            float *out = c_hat + t * r + nc;
 #pragma unroll
-            for (int j = 0; j < kBN; j += 4) {
+            for (int j = 0; j < 128; j += 4) {
                 float4 v;
-                v.x = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 0]), sx), ws[n0 + j + 0]);
-                v.y = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 1]), sx), ws[n0 + j + 1]);
-                v.z = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 2]), sx), ws[n0 + j + 2]);
-                v.w = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 3]), sx), ws[n0 + j + 3]);
+                v.x = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 0]), sx), ws[nc + j + 0]);
+                v.y = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 1]), sx), ws[nc + j + 1]);
+                v.z = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 2]), sx), ws[nc + j + 2]);
+                v.w = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 3]), sx), ws[nc + j + 3]);
                 *reinterpret_cast<float4 *>(out + j) = v;
             }
             if (acc_out) {
-                int32_t *ao = acc_out + t * r + n0;
+                int32_t *ao = acc_out + t * r + nc;
 #pragma unroll
-                for (int j = 0; j < kBN; j += 4)
+                for (int j = 0; j < 128; j += 4)
                     *reinterpret_cast<int4 *>(ao + j) = make_int4(acc[j], acc[j + 1], acc[j + 2], acc[j + 3]);
             }
         }
@@ -212,7 +233,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
     __syncthreads();
     tc_fence_after();
     if (warp == 1)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * kBN));
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * BN));
 }
 
 // ---------------------------------------------------------------------------
@@ -247,20 +268,32 @@ static bool make_map(CUtensorMap *map, const void *base, int64_t rows, int cols,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-bool gemm_tc_supported(int d, int r) { return d % kBK == 0 && r % kBN == 0 && encode_fn() != nullptr; }
+bool gemm_tc_supported(int d, int r) { return d % kBK == 0 && r % 128 == 0 && encode_fn() != nullptr; }
+
+template <int BN>
+static cudaError_t launch_bn(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
+                             const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s) {
+    using C = GemmCfg<BN>;
+    CUtensorMap mx, mw;
+    if (!make_map(&mx, xq_bf16, T, d, kBM) || !make_map(&mw, w_bf16, r, d, BN)) return cudaErrorInvalidValue;
+    cudaError_t e = ensure_smem(gemm_tc_kernel<BN>, C::kSmem);
+    if (e != cudaSuccess) return e;
+    dim3 grid(unsigned(r / BN), unsigned((T + kBM - 1) / kBM));
+    e = launch_pdl(gemm_tc_kernel<BN>, grid, dim3(C::kThreads), C::kSmem, s, mx, mw, T, d, r, xs, ws, c_hat, acc_out,
+                   err);
+    prof_mark(s, "gemm_tc");
+    return e;
+}
 
 cudaError_t launch_gemm_tc(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
                            const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s) {
     if (T == 0) return cudaSuccess;
-    CUtensorMap mx, mw;
-    if (!make_map(&mx, xq_bf16, T, d, kBM) || !make_map(&mw, w_bf16, r, d, kBN)) return cudaErrorInvalidValue;
-    cudaError_t e = ensure_smem(gemm_tc_kernel, kGemmSmem);
-    if (e != cudaSuccess) return e;
-    dim3 grid(unsigned((T + kBM - 1) / kBM), unsigned(r / kBN));
-    e = launch_pdl(gemm_tc_kernel, grid, dim3(kGemmThreads), kGemmSmem, s, mx, mw, T, d, r, xs, ws, c_hat, acc_out,
-                   err);
-    prof_mark(s, "gemm_tc");
-    return e;
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t wide_tiles = ((T + kBM - 1) / kBM) * (r / 256);
+    if (r % 256 == 0 && wide_tiles >= 2 * sms)
+        return launch_bn<256>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, err, s);
+    return launch_bn<128>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, err, s);
 }
 
 }  // namespace qsvd
