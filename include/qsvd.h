@@ -202,6 +202,32 @@ size_t qsvd_decode_step_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t 
                                         int32_t H, int32_t dh);
 
 /*
+ * Allocation-free variant of qsvd_latent_project for decode-size calls
+ * (T <= 16 tokens, r <= 4096, d % 256 == 0, d <= 6144).  The paper has no
+ * counterpart; it exists for callers that cannot allocate device memory when
+ * they project a token, such as a serving process whose device memory was
+ * reserved in full at start-up by another allocator, or code running while a
+ * stream is captured into a graph (cudaMalloc is not allowed there), and
+ * that therefore cannot supply the workspace qsvd_latent_project needs.
+ * Arguments and results are those of qsvd_latent_project without the
+ * inspection outputs and the workspace.  The scratch lives in a fixed
+ * 264 KiB device array inside the library, held by every GPU that loads the
+ * library until the process exits; the call allocates nothing.
+ *   - The first call on a device looks up that array's device address, so
+ *     make it before any stream capture on that device.
+ *   - T > 16 or r > 4096 returns QSVD_ENOSPC with a message.
+ *   - All calls share the one array: calls that may overlap on the GPU (on
+ *     different streams, or on the same device from several threads without
+ *     ordering) race and must not be issued.
+ *   - Each call clears the array's completion counter before it launches.
+ */
+int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
+                               float act_clip, int32_t lat_bits, float lat_clip,
+                               void *lat_codes, void *lat_scales,
+                               const qsvd_cache *dst, const int32_t *dst_seq, const int32_t *dst_pos,
+                               cudaStream_t stream);
+
+/*
  * Synchronizes `stream`, then reads and clears the device error word.
  * Returns QSVD_OK, QSVD_ERANGE, QSVD_ETIMEOUT or QSVD_ECUDA.
  */

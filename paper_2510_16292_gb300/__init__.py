@@ -31,7 +31,7 @@ QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
 EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
-           "qsvd_decode_step", "qsvd_decode_step_workspace_bytes",
+           "qsvd_decode_step", "qsvd_decode_step_workspace_bytes", "qsvd_latent_project_static",
            "qsvd_check", "qsvd_last_error", "qsvd_version")
 
 
@@ -66,6 +66,8 @@ _lib.qsvd_decode_step.argtypes = [ctypes.POINTER(_DownWeight), _vp, ctypes.POINT
                                   _vp, _i32, _i32, _f32, _f32, _f32, _vp, _vp, _sz, _vp]
 _lib.qsvd_decode_step_workspace_bytes.argtypes = [_i32, _i32, _i32, _i32, _i32, _i32]
 _lib.qsvd_decode_step_workspace_bytes.restype = _sz
+_lib.qsvd_latent_project_static.argtypes = [ctypes.POINTER(_DownWeight), _vp, _i64, _f32, _i32, _f32, _vp, _vp,
+                                            ctypes.POINTER(_Cache), _vp, _vp, _vp]
 _lib.qsvd_check.argtypes = [_vp]
 _lib.qsvd_last_error.restype = ctypes.c_char_p
 
@@ -218,6 +220,19 @@ def qsvd_decode_step(W: DownWeight, X: torch.Tensor, cache: LatentCache, seq_len
     _check(_lib.qsvd_decode_step(ctypes.byref(cw), _ptr(X), ctypes.byref(cc), _ptr(seq_len), max_seq_len,
                                  _ptr(U_q), _ptr(U_k), _ptr(U_v), H, dh, act_clip, lat_clip, softmax_scale,
                                  _ptr(O), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def qsvd_latent_project_static(W: DownWeight, X: torch.Tensor, act_clip: float = 1.0, lat_bits: int = 8,
+                               lat_clip: float = 1.0, lat_codes=None, lat_scales=None,
+                               dst: Optional[LatentCache] = None, dst_seq=None, dst_pos=None, stream=None) -> None:
+    """Decode-size projection (T <= 16) that uses the library's fixed device
+    scratch instead of a workspace; nothing is allocated on the device."""
+    cw = W._c()
+    cc = dst._c() if dst is not None else None
+    _check(_lib.qsvd_latent_project_static(ctypes.byref(cw), _ptr(X), X.shape[0], act_clip, lat_bits, lat_clip,
+                                           _ptr(lat_codes), _ptr(lat_scales),
+                                           ctypes.byref(cc) if cc is not None else None, _ptr(dst_seq),
+                                           _ptr(dst_pos), _stream(stream)))
 
 
 def qsvd_check(stream=None) -> int:

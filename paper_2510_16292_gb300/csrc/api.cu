@@ -87,6 +87,13 @@ thread_local std::vector<const char *> t_prof_labels;
 
 }  // namespace
 
+int *error_word_for_current_device() {
+    int *err = nullptr;
+    return device_setup(&err) == QSVD_OK ? err : nullptr;
+}
+
+int set_last_error(int code, const char *msg) { return fail(code, "%s", msg); }
+
 cudaError_t ensure_smem_ptr(const void *kernel, size_t bytes) {
     static std::mutex mu;
     static std::unordered_map<const void *, int> done;     // kernel -> device bitmask

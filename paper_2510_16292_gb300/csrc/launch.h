@@ -41,6 +41,11 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 // Bits of the device error word (read and cleared by qsvd_check).
 enum : int { kErrRange = 1, kErrTimeout = 2 };
 
+// Device address of the error word for the current device (nullptr if the
+// device is unusable), and the thread's last-error message setter.
+int *error_word_for_current_device();
+int set_last_error(int code, const char *msg);
+
 // Plain description of a latent cache (mirrors qsvd_cache).
 struct CacheView {
     void *codes;
