@@ -22,6 +22,7 @@ from __future__ import annotations
 
 import argparse
 import ctypes
+import dataclasses
 import json
 import math
 import os
@@ -53,6 +54,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-prefill13", action="store_true")
+    p.add_argument("--workload", default=WORKLOAD, choices=sorted(synthetic.WORKLOADS))
+    p.add_argument("--decode-steps", type=int, default=0, help="override the workload's decode steps")
     return p.parse_args()
 
 
@@ -420,7 +423,9 @@ def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
 def run_native(args, rank, world, local_rank):
     import torch
     torch.cuda.set_device(local_rank)
-    wl = synthetic.WORKLOADS[WORKLOAD]
+    wl = synthetic.WORKLOADS[args.workload]
+    if args.decode_steps:
+        wl = dataclasses.replace(wl, decode_steps=args.decode_steps)
     nb = NativeBench(wl, rank)
     S = wl.decode_steps
     hbm, _, peak_kind = peaks()
@@ -523,7 +528,7 @@ def run_native(args, rank, world, local_rank):
     }
     if e2e:
         out["e2e"] = e2e
-    if world == 1 and not args.no_cpu_baseline:
+    if world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
         out["cpu_baseline"] = cpu_baseline(wl, budget_s=15.0)
     print(json.dumps(out), flush=True)
 
