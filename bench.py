@@ -309,7 +309,7 @@ class NativeBench:
             return r * d * 2 + B * (tok + stok) + 4 * B * d
         if label == "qabsorb":
             return r * d * 2 + 4 * B * d + 4 * B * H * r
-        if label == "attn_chunk":
+        if label in ("attn_chunk", "attn_tc"):
             return B * L * (tok + stok) + 4 * B * H * r
         if label == "combine_uv":
             return r * d * 2 + 4 * B * d

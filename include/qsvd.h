@@ -167,7 +167,7 @@ int qsvd_cache_append(const qsvd_cache *cache, const int32_t *seq, const int32_t
  *   U_q, U_k, U_v  bf16 [r, H*dh] row-major;
  *   O            fp32 [B, H*dh] out.
  * workspace: qsvd_decode_workspace_bytes(B, max_seq_len, r, H, dh) bytes.
- * Requirements: dh in {64, 128}; r % 16 == 0 and r <= 3072; H*dh % 256 == 0
+ * Requirements: dh in {64, 128}; r % 32 == 0 and r <= 3072; H*dh % 256 == 0
  * and H*dh <= 6144.
  */
 int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int32_t max_seq_len,
@@ -226,6 +226,20 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
                                void *lat_codes, void *lat_scales,
                                const qsvd_cache *dst, const int32_t *dst_seq, const int32_t *dst_pos,
                                cudaStream_t stream);
+
+/*
+ * Choice of attention kernels for qsvd_latent_decode_attn (a library setting,
+ * not part of the paper's method; process-wide, not thread-safe):
+ *   0  automatic (default): the tensor-core kernel when the shape allows it
+ *      and B * max_seq_len >= 4096, else the CUDA-core kernels;
+ *   1  always the CUDA-core kernels;
+ *   2  the tensor-core kernel whenever the shape allows it.
+ * The tensor-core kernel needs r % 256 == 0, r <= 1536, H <= 32 and
+ * (r / 256) * ceil16(H) <= 192; other shapes always use the CUDA-core
+ * kernels.  Both give the same results up to floating-point rounding.
+ * Returns the previous setting, or QSVD_EINVAL for another value.
+ */
+int qsvd_set_decode_attn_path(int32_t path);
 
 /*
  * Synchronizes `stream`, then reads and clears the device error word.

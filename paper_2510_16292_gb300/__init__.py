@@ -32,7 +32,7 @@ QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
 EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
            "qsvd_decode_step", "qsvd_decode_step_workspace_bytes", "qsvd_latent_project_static",
-           "qsvd_check", "qsvd_last_error", "qsvd_version")
+           "qsvd_set_decode_attn_path", "qsvd_check", "qsvd_last_error", "qsvd_version")
 
 
 class QsvdError(RuntimeError):
@@ -244,3 +244,15 @@ def qsvd_check(stream=None) -> int:
 
 def qsvd_version() -> int:
     return int(_lib.qsvd_version())
+
+
+_lib.qsvd_set_decode_attn_path.argtypes = [_i32]
+
+
+def qsvd_set_decode_attn_path(path: int) -> int:
+    """0 automatic, 1 CUDA-core kernels, 2 tensor-core kernel where the shape
+    allows it.  Returns the previous setting."""
+    st = _lib.qsvd_set_decode_attn_path(path)
+    if st < 0:
+        _check(st)
+    return st

@@ -117,6 +117,36 @@ cudaError_t ensure_smem_ptr(const void *kernel, size_t bytes) {
     return e;
 }
 
+namespace {
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *q = nullptr;
+        cudaDriverEntryPointQueryResult res;
+        if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &q, cudaEnableDefault, &res) == cudaSuccess &&
+            res == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(q);
+    });
+    return fn;
+}
+}  // namespace
+
+bool encode_map_2d(CUtensorMap *map, CUtensorMapDataType type, const void *base, uint64_t inner, uint64_t outer,
+                   uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swizzle) {
+    EncodeTiledFn fn = encode_tiled();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {inner, outer};
+    const cuuint64_t strides[1] = {row_bytes};
+    const cuuint32_t box[2] = {box_inner, box_outer};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, type, 2, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 void prof_mark(cudaStream_t s, const char *label) {
     if (!t_prof_events || int(t_prof_labels.size()) >= t_prof_capacity) return;
     if (cudaEventRecord(t_prof_events[t_prof_labels.size()], s) == cudaSuccess)
@@ -134,6 +164,13 @@ extern "C" {
 const char *qsvd_last_error(void) { return g_msg; }
 
 int qsvd_version(void) { return 100; }
+
+int qsvd_set_decode_attn_path(int32_t path) {
+    if (path < 0 || path > 2) return fail(QSVD_EINVAL, "set_decode_attn_path: path must be 0, 1 or 2");
+    const int prev = attn_path();
+    set_attn_path(path);
+    return prev;
+}
 
 int qsvd_profile_events(void **events, int32_t capacity) {
     t_prof_labels.clear();
@@ -300,7 +337,7 @@ int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int
     if (!seq_len || !U_q || !U_k || !U_v || !O) return fail(QSVD_EINVAL, "decode_attn: null pointer");
     if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "decode_attn: dh must be 64 or 128");
     if (H <= 0) return fail(QSVD_EINVAL, "decode_attn: H must be positive");
-    if (cache->r > 3072) return fail(QSVD_EUNSUPPORTED, "decode_attn: r > 3072");
+    if (cache->r > 3072 || cache->r % 32) return fail(QSVD_EUNSUPPORTED, "decode_attn: need r %% 32 == 0 and r <= 3072");
     if ((H * dh) % 256 || H * dh > 6144) return fail(QSVD_EUNSUPPORTED, "decode_attn: need H*dh %% 256 == 0 and H*dh <= 6144");
     if (max_seq_len < 1 || max_seq_len > cache->Tmax) return fail(QSVD_EINVAL, "decode_attn: max_seq_len outside [1, Tmax]");
     const void *ptrs[] = {U_q, U_k, U_v, O, workspace};

@@ -1,0 +1,890 @@
+// Decode attention over the latent cache on the 5th-generation tensor cores
+// (Eq. 5 with W^u_k absorbed into the query: scores c_t . q~_h, softmax, and
+// the softmax-weighted latent sum sum_t p_t c_t; W^u_v is applied afterwards
+// by combine_uv_kernel).
+//
+// Work unit: a cluster of two CTAs takes a contiguous range of 128-token tiles
+// of one sequence.  CTA k of the pair owns the latent channels
+// [k r/2, (k+1) r/2).  Per tile it computes partial scores over its channels,
+// the pair swaps them through distributed shared memory and both add them in
+// the same order, so both run the identical online softmax; each then
+// accumulates o_lat for its own channels.  Splitting the channels halves the
+// tensor-memory footprint of the o_lat accumulator and the bytes each SM
+// reads.
+//
+// Per tile the CTA streams its channels twice (the second stream hits L2):
+//   pass 1  warp 0 loads 128-token x 128-channel chunks with TMA; warpgroup 1
+//           (one thread per token) converts 64 channels at a time to fp16 and
+//           stores them into tensor memory; warp 1 issues
+//              S[t, h] += C[t, ch] Q[ch, h]      (M = 128 tokens, N = heads,
+//           A from tensor memory, B = the fp16 query block in shared memory).
+//   softmax warpgroup 3 reads S, swaps partials with the peer, applies the
+//           token scale and 1/sqrt(dh), runs the online softmax (o_lat is
+//           rescaled lazily, only when the running maximum of a head grows by
+//           more than kRescale2) and writes P (fp16, [heads x tokens]).
+//   pass 2  warp 3 loads the same chunks again; warpgroup 2 converts them to
+//           an fp16 tile in shared memory; warp 2 issues
+//              O^T[ch, h] += C^T[ch, t] P[t, h]  (M = 128 channels, K = tokens,
+//           A = the tile read channel-major, B = P).
+// int8 codes are exact in fp16; the per-token scale multiplies the scores and
+// is folded into P.  int4 codes are converted to code * group-scale in fp16.
+// The query block is scaled per head by a power of two so that its largest
+// entry sits just below 2^14 (the scale is undone on the scores).
+//
+// Every wait is bounded in time (on expiry the error word gets kErrTimeout and
+// the CTA abandons its tiles); a CTA always drains its own copies and MMAs,
+// meets its peer at the final cluster barrier, and frees its tensor memory.
+#include <cfloat>
+#include <cuda.h>
+#include <cuda_fp16.h>
+
+#include "common.cuh"
+#include "launch.h"
+
+namespace qsvd {
+
+namespace atc {
+
+constexpr int kTile = 128;        // tokens per tile
+constexpr int kChunk = 128;       // channels per TMA chunk
+constexpr int kThreads = 512;     // 16 warps
+constexpr int kRing = 2;          // TMA slots per pass
+constexpr int kMaxN = 32;         // heads (padded to a multiple of 16)
+constexpr int kMaxRc = 768;       // channels per CTA
+constexpr float kRescale2 = 11.5f;  // lazy rescale threshold (log2 units, about 8 in natural-log units)
+constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per wait
+
+// dynamic shared memory (byte offsets from a 1024-aligned base)
+constexpr int kQtBytes = kMaxN * kMaxRc * 2;       // query block, fp16, 128-byte swizzled, K-major
+constexpr int kSlotBytes = kTile * kChunk;         // one int8 chunk (int4 uses half)
+constexpr int kPvaBytes = kTile * kChunk * 2;      // fp16 tile of one chunk
+constexpr int kPBytes = kMaxN * kTile * 2;         // P, fp16, 128-byte swizzled, K-major
+constexpr int kXchBytes = kTile * kMaxN * 4;       // the peer's partial scores
+constexpr int kOffQt = 0;
+constexpr int kOffT1 = kOffQt + kQtBytes;
+constexpr int kOffT2 = kOffT1 + kRing * kSlotBytes;
+constexpr int kOffPva = kOffT2 + kRing * kSlotBytes;
+constexpr int kOffP = kOffPva + 2 * kPvaBytes;
+constexpr int kOffXch = kOffP + 2 * kPBytes;
+constexpr int kSmemBytes = kOffXch + kXchBytes + 1024;
+
+// tensor memory columns
+constexpr uint32_t kColO = 0;      // o_lat^T: (r_c / 128) x Np       (<= 192)
+constexpr uint32_t kColS = 192;    // scores: 2 buffers x 32
+constexpr int kABufs = 4;          // scores A operand buffers (64 channels each)
+constexpr uint32_t kColA = 256;    // scores A operand: kABufs x 32 columns
+constexpr uint32_t kTmemCols = 512;
+
+struct Params {
+    CacheView c;
+    const int32_t *seq_len;
+    const float *qt;        // [B, H, r] fp32
+    const unsigned *qmax;   // [B, H] bit patterns of max_j |qt[b, h, j]| (non-negative floats)
+    int H, Np;              // heads, heads padded to a multiple of 16
+    float softmax_scale;
+    int tiles_per_split, n_split;
+    float *pm, *pl, *po;    // [B, n_split, H] and [B, n_split, H, r]
+    int *err;
+};
+
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t map_peer(uint32_t local, uint32_t peer) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(peer));
+    return r;
+}
+// Asynchronous 16-byte store into the peer's shared memory; its completion
+// counts 16 bytes on the peer's mbarrier `bar` (both cluster addresses).
+__device__ __forceinline__ void st_async_v4(uint32_t addr, float a, float b, float c, float d, uint32_t bar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];"
+                 ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d), "r"(bar)
+                 : "memory");
+}
+__device__ __forceinline__ void arrive_peer(uint32_t bar_cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster_addr) : "memory");
+}
+__device__ __forceinline__ void arrive_local(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ bool try_wait_acq_cluster(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+                 "selp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(ok)
+                 : "r"(smem_addr(bar)), "r"(parity)
+                 : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ unsigned long long now_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+// Wait for phase `parity` of `bar`, for at most kWaitNs.  `cluster`: acquire
+// at cluster scope (the phase is completed by the peer CTA).
+__device__ __noinline__ bool wait_bar(uint64_t *bar, uint32_t parity, int *err, bool cluster) {
+    if (cluster ? try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = now_ns();
+    for (;;) {
+        for (int i = 0; i < 64; ++i)
+            if (cluster ? try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
+        if (now_ns() - t0 > kWaitNs) {
+            flag_error(err, kErrTimeout);
+            return false;
+        }
+    }
+}
+__device__ __forceinline__ bool wait(uint64_t *bar, uint32_t parity, int *err) {
+    return mbar_try_wait(bar, parity) || wait_bar(bar, parity, err, false);
+}
+// Warp-uniform forms: every lane waits (and acquires); the warp agrees on the outcome.
+__device__ __forceinline__ bool wwait(uint64_t *bar, uint32_t parity, int *err) {
+    return __all_sync(0xffffffffu, wait(bar, parity, err));
+}
+__device__ __forceinline__ bool wwait_cluster(uint64_t *bar, uint32_t parity, int *err) {
+    return __all_sync(0xffffffffu, try_wait_acq_cluster(bar, parity) || wait_bar(bar, parity, err, true));
+}
+// Named barrier 1 over the 128 softmax threads, returning the OR of `v` over them.
+__device__ __forceinline__ bool group_any(bool v) {
+    uint32_t r;
+    asm volatile("{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.or.pred q, 1, 128, p;\n\t"
+                 "selp.u32 %0, 1, 0, q;\n\t}"
+                 : "=r"(r)
+                 : "r"(uint32_t(v))
+                 : "memory");
+    return r != 0;
+}
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(smem_addr(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+        : "memory");
+}
+// L2 prefetch of one box of a tensor map (no shared memory, no completion).
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap *map, int x, int y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];"
+                 ::"l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y)
+                 : "memory");
+}
+// Shared-memory matrix descriptor, 128-byte swizzle.
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return uint64_t((saddr & 0x3FFFF) >> 4) | (uint64_t((lbo >> 4) & 0x3FFF) << 16) |
+           (uint64_t((sbo >> 4) & 0x3FFF) << 32) | (uint64_t(1) << 46) | (uint64_t(2) << 61);
+}
+// Instruction descriptor: f16 x f16 -> f32, M = 128, N = n; a_mn: A is M-major.
+__host__ __device__ constexpr uint32_t idesc_f16(int n, int a_mn) {
+    return (1u << 4) | (uint32_t(a_mn) << 15) | (uint32_t(n >> 3) << 17) | (uint32_t(128 >> 4) << 24);
+}
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}"
+                 ::"r"(d), "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc));
+}
+__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+                 ::"r"(d), "l"(a), "l"(b), "r"(idesc), "r"(acc));
+}
+__device__ __forceinline__ void commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_addr(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};"
+        ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),
+        "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]),
+        "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31]));
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+        ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]));
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// Four int8 codes -> two fp16 pairs, exact: the half with bits 0x64xx is
+// 1024 + xx, so (code + 128) placed in the low byte gives 1152 + code.
+__device__ __forceinline__ void i8x4_to_h2x2(uint32_t w, uint32_t &lo, uint32_t &hi) {
+    const uint32_t u = w ^ 0x80808080u;
+    const uint32_t a = __byte_perm(u, 0x64646464u, 0x5150);
+    const uint32_t b = __byte_perm(u, 0x64646464u, 0x5352);
+    const __half2 bias = __half2half2(__ushort_as_half(0x6480));      // 1152
+    const __half2 ha = __hsub2(*reinterpret_cast<const __half2 *>(&a), bias);
+    const __half2 hb = __hsub2(*reinterpret_cast<const __half2 *>(&b), bias);
+    lo = *reinterpret_cast<const uint32_t *>(&ha);
+    hi = *reinterpret_cast<const uint32_t *>(&hb);
+}
+// Eight int4 codes (element i in bits 4i..4i+3, two's complement) times an
+// fp16 group scale -> four fp16 pairs (products rounded to nearest).
+__device__ __forceinline__ void i4x8_to_h2x4(uint32_t w, __half2 s2, uint32_t *o) {
+    const __half2 bias = __half2half2(__ushort_as_half(0x6408));      // 1032 = 1024 + 8
+    const uint32_t x = w ^ 0x88888888u;                               // code + 8 in every nibble
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint32_t n0 = (x >> (8 * k)) & 0xfu, n1 = (x >> (8 * k + 4)) & 0xfu;
+        const uint32_t p = (0x6400u | n0) | ((0x6400u | n1) << 16);
+        const __half2 h = __hmul2(__hsub2(*reinterpret_cast<const __half2 *>(&p), bias), s2);
+        o[k] = *reinterpret_cast<const uint32_t *>(&h);
+    }
+}
+
+// Byte offset of 16-byte chunk q of row `row` in a 128-byte-swizzled tile
+// (rows of 128 bytes, tile base 1024-aligned).
+__device__ __forceinline__ uint32_t sw128(uint32_t row, uint32_t q) { return row * 128u + ((q ^ (row & 7u)) << 4); }
+// The same for a 64-byte-swizzled tile (rows of 64 bytes).
+__device__ __forceinline__ uint32_t sw64(uint32_t row, uint32_t q) {
+    return row * 64u + ((q ^ ((row >> 1) & 3u)) << 4);
+}
+
+__device__ __forceinline__ uint16_t load_group_scale(const CacheView &c, size_t slot, int group, bool live) {
+    return live ? static_cast<const uint16_t *>(c.scales)[slot * (c.r / 128) + group] : uint16_t(0);
+}
+
+}  // namespace atc
+
+// ---------------------------------------------------------------------------
+template <int BITS>
+__global__ void __launch_bounds__(atc::kThreads, 1)
+attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
+    using namespace atc;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t t1_full[kRing], t1_empty[kRing], t2_full[kRing], t2_empty[kRing];
+    __shared__ __align__(8) uint64_t a_full[kABufs], a_empty[kABufs], s_full[2], s_empty[2];
+    __shared__ __align__(8) uint64_t pva_full[2], pva_empty[2], p_full[2], p_empty[2];
+    __shared__ __align__(8) uint64_t xch_full, xch_empty, mma_done[2];
+    __shared__ uint32_t tmem_base;
+    __shared__ float red_max[4][kMaxN];
+    __shared__ float m_ref[kMaxN], alpha[kMaxN], q_exp[kMaxN], qfac[kMaxN];
+    __shared__ volatile int abort_flag;
+
+    const CacheView &c = p.c;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_rank(), peer = rank ^ 1u;
+    const int split = blockIdx.x >> 1, b = blockIdx.y;
+    const int r = c.r, rc = r / 2, ch0 = int(rank) * rc;
+    const int n_chunks = rc / kChunk;
+    const int Np = p.Np, H = p.H;
+    constexpr uint32_t kLoadBytes = BITS == 8 ? kTile * kChunk : kTile * kChunk / 2;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kRing; ++i) {
+            mbar_init(&t1_full[i], 1);
+            mbar_init(&t1_empty[i], 4);
+            mbar_init(&t2_full[i], 1);
+            mbar_init(&t2_empty[i], 4);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&s_full[i], 1);
+            mbar_init(&s_empty[i], 4);
+            mbar_init(&pva_full[i], 4);
+            mbar_init(&pva_empty[i], 1);
+            mbar_init(&p_full[i], 4);
+            mbar_init(&p_empty[i], 1);
+            mbar_init(&mma_done[i], 1);
+        }
+        for (int i = 0; i < kABufs; ++i) {
+            mbar_init(&a_full[i], 4);
+            mbar_init(&a_empty[i], 1);
+        }
+        mbar_init(&xch_full, 1);     // one local expect-tx arrival + the peer's st.async bytes
+        mbar_init(&xch_empty, 128);  // every softmax thread of the peer, after reading
+        mbar_init_fence();
+        abort_flag = 0;
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                     ::"r"(smem_addr(&tmem_base)), "r"(kTmemCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    fence_before();
+    __syncthreads();
+    fence_after();
+    cluster_sync();                  // the peer's barriers exist before any remote arrive
+    const uint32_t tmem = tmem_base;
+    pdl_trigger();
+    pdl_wait();
+
+    const int L = p.seq_len[b];
+    const bool valid = L >= 1 && L <= c.Tmax;
+    const int t_begin = split * p.tiles_per_split * kTile;
+    const int t_end = valid ? min(L, t_begin + p.tiles_per_split * kTile) : t_begin;
+    const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
+    const size_t row0 = size_t(b) * c.Tmax;          // cache slot of token 0 of the sequence
+    const int total = n_tiles * n_chunks;             // chunk loads per pass
+
+    // ---- query block: per-head power-of-two scale from the max over all r
+    // channels (both CTAs of the pair get the same scale), then the fp16
+    // block Q^T [heads][channels of this CTA], 128-byte swizzled, 64 channels
+    // per 128-byte row, blocks of Np rows.
+    if (n_tiles > 0) {
+        if (threadIdx.x < kMaxN) {
+            const int h = threadIdx.x;
+            int e = 0;
+            if (h < H) {
+                const float m = __uint_as_float(p.qmax[size_t(b) * H + h]);   // max_j |q~[b, h, j]|
+                if (m > 0.0f) frexpf(m, &e);                                   // m < 2^e
+            }
+            q_exp[h] = float(14 - e);                                          // |q~| * 2^(14-e) < 2^14
+            // scores -> logits in log2 units: undo the query scale, times softmax_scale * log2(e)
+            qfac[h] = exp2f(float(e - 14)) * p.softmax_scale * 1.4426950408889634f;
+            m_ref[h] = -INFINITY;
+        }
+        __syncthreads();
+        if (warp >= 4) {
+            // 8 channels per item; all loads of a thread are issued before its first conversion
+            constexpr int kPer = 8;
+            const int items = Np * (rc / 8);
+            for (int i0 = threadIdx.x - 128; i0 < items; i0 += kPer * (kThreads - 128)) {
+                float4 va[kPer], vb[kPer];
+#pragma unroll
+                for (int k = 0; k < kPer; ++k) {
+                    const int i = i0 + k * (kThreads - 128);
+                    const int h = i / (rc / 8), q8 = i % (rc / 8);
+                    va[k] = vb[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (i < items && h < H) {
+                        const float4 *src = reinterpret_cast<const float4 *>(p.qt + (size_t(b) * H + h) * r + ch0 + q8 * 8);
+                        va[k] = src[0];
+                        vb[k] = src[1];
+                    }
+                }
+#pragma unroll
+                for (int k = 0; k < kPer; ++k) {
+                    const int i = i0 + k * (kThreads - 128);
+                    if (i >= items) break;
+                    const int h = i / (rc / 8), q8 = i % (rc / 8);
+                    const int kc = q8 >> 3, q = q8 & 7;
+                    const float sc = exp2f(q_exp[h]);
+                    const float4 a = va[k], bq = vb[k];
+                    const __half2 v0 = __floats2half2_rn(a.x * sc, a.y * sc), v1 = __floats2half2_rn(a.z * sc, a.w * sc);
+                    const __half2 v2 = __floats2half2_rn(bq.x * sc, bq.y * sc), v3 = __floats2half2_rn(bq.z * sc, bq.w * sc);
+                    *reinterpret_cast<uint4 *>(sm + kOffQt + kc * (Np * 128) + sw128(h, q)) =
+                        make_uint4(*reinterpret_cast<const uint32_t *>(&v0), *reinterpret_cast<const uint32_t *>(&v1),
+                                   *reinterpret_cast<const uint32_t *>(&v2), *reinterpret_cast<const uint32_t *>(&v3));
+                }
+            }
+            fence_async_smem();
+        }
+    }
+    __syncthreads();
+
+    if (warp == 0 || warp == 3) {
+        // ---------------- TMA producers: warp 0 pass 1, warp 3 pass 2 ----------------
+        if (lane == 0 && total > 0) {
+            uint64_t *full = warp == 0 ? t1_full : t2_full;
+            uint64_t *empty = warp == 0 ? t1_empty : t2_empty;
+            uint8_t *ring = sm + (warp == 0 ? kOffT1 : kOffT2);
+            int issued = 0;
+            // pass 1 keeps the chunks of the next two tiles streaming into L2
+            const int ahead = 2 * n_chunks;
+            auto prefetch = [&](int j) {
+                tma_prefetch_2d(&map_c, (ch0 + (j % n_chunks) * kChunk) * BITS / 8,
+                                int(row0) + t_begin + (j / n_chunks) * kTile);
+            };
+            if (warp == 0)
+                for (int j = 0; j < ahead && j < total; ++j) prefetch(j);
+            for (int i = 0; i < total && !abort_flag; ++i) {
+                const int s = i % kRing, tile = i / n_chunks, ck = i % n_chunks;
+                if (warp == 0 && i + ahead < total) prefetch(i + ahead);
+                if (i >= kRing && !wait(&empty[s], ((i / kRing) - 1) & 1, p.err)) { abort_flag = 1; break; }
+                mbar_arrive_expect_tx(&full[s], kLoadBytes);
+                tma_load_2d(ring + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
+                            int(row0) + t_begin + tile * kTile, &full[s]);
+                ++issued;
+            }
+            // every issued copy has landed before the CTA may finish
+            for (int i = issued - kRing > 0 ? issued - kRing : 0; i < issued; ++i)
+                wait(&full[i % kRing], (i / kRing) & 1, p.err);
+        }
+    } else if (warp == 1) {
+        // ---------------- scores MMA ----------------
+        if (lane == 0 && n_tiles > 0) {
+            const uint32_t idesc = idesc_f16(Np, 0);
+            int half = 0;
+            for (int tile = 0; tile < n_tiles && !abort_flag; ++tile) {
+                const int sb = tile & 1;
+                if (tile >= 2 && !wait(&s_empty[sb], ((tile >> 1) - 1) & 1, p.err)) { abort_flag = 1; break; }
+                fence_after();
+                bool ok = true;
+                for (int hh = 0; hh < 2 * n_chunks; ++hh, ++half) {
+                    const int ab = half % kABufs;
+                    if (!wait(&a_full[ab], (half / kABufs) & 1, p.err)) { ok = false; break; }
+                    fence_after();
+                    const uint32_t qblk = smem_addr(sm + kOffQt + hh * (Np * 128));
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        mma_ts(tmem + kColS + sb * 32, tmem + kColA + ab * 32 + k * 8, sdesc(qblk + k * 32, 16, 1024),
+                               idesc, (hh > 0 || k > 0) ? 1u : 0u);
+                    commit(&a_empty[ab]);
+                }
+                if (!ok) { abort_flag = 1; break; }
+                commit(&s_full[sb]);
+            }
+            commit(&mma_done[0]);
+            wait(&mma_done[0], 0, p.err);
+        }
+    } else if (warp == 2) {
+        // ---------------- PV MMA: O^T += C^T P ----------------
+        if (lane == 0 && n_tiles > 0) {
+            const uint32_t idesc = idesc_f16(Np, 1);
+            int chunk = 0;
+            for (int tile = 0; tile < n_tiles && !abort_flag; ++tile) {
+                const int pb = tile & 1;
+                if (!wait(&p_full[pb], (tile >> 1) & 1, p.err)) { abort_flag = 1; break; }
+                fence_after();
+                const uint32_t pbase = smem_addr(sm + kOffP + pb * kPBytes);
+                bool ok = true;
+                for (int ck = 0; ck < n_chunks; ++ck, ++chunk) {
+                    const int vb = chunk & 1;
+                    if (!wait(&pva_full[vb], (chunk >> 1) & 1, p.err)) { ok = false; break; }
+                    fence_after();
+                    const uint32_t abase = smem_addr(sm + kOffPva + vb * kPvaBytes);
+#pragma unroll
+                    for (int k = 0; k < kTile / 16; ++k) {
+                        // A: channel-major fp16 tile; 64-channel halves 16 KiB apart, 8-token groups 1 KiB apart
+                        const uint64_t a = sdesc(abase + k * 16 * 128, kTile * 128, 1024);
+                        // B: P^T rows = heads; 64-token blocks Np * 128 bytes apart
+                        const uint64_t bb = sdesc(pbase + (k >> 2) * (Np * 128) + (k & 3) * 32, 16, 1024);
+                        mma_ss(tmem + kColO + ck * Np, a, bb, idesc, (tile > 0 || k > 0) ? 1u : 0u);
+                    }
+                    commit(&pva_empty[vb]);
+                }
+                if (!ok) { abort_flag = 1; break; }
+                commit(&p_empty[pb]);
+            }
+            commit(&mma_done[1]);
+            wait(&mma_done[1], 0, p.err);
+        }
+    } else if (warp < 8) {
+        // ---------------- warpgroup 1: pass-1 converter, one thread per token ----------------
+        const int quad = warp & 3, t = quad * 32 + lane;
+        const uint32_t trow = tmem + (uint32_t(quad * 32) << 16);
+        int half = 0;
+        uint16_t sc_next = 0;
+        if (BITS == 4 && total > 0) {
+            const int tok = t_begin + t;
+            sc_next = load_group_scale(c, row0 + tok, ch0 / 128, tok < t_end);
+        }
+        for (int i = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0); ++i) {
+            const int s = i % kRing;
+            const uint16_t sc_cur = sc_next;
+            if (BITS == 4 && i + 1 < total) {      // next chunk's group scale, loaded ahead
+                const int tok = t_begin + ((i + 1) / n_chunks) * kTile + t;
+                sc_next = load_group_scale(c, row0 + tok, (ch0 / 128) + (i + 1) % n_chunks, tok < t_end);
+            }
+            if (!wwait(&t1_full[s], (i / kRing) & 1, p.err)) { abort_flag = 1; break; }
+            const uint8_t *slot = sm + kOffT1 + s * kSlotBytes;
+            bool ok = true;
+            for (int hh = 0; hh < 2; ++hh, ++half) {
+                const int ab = half % kABufs;
+                if (half >= kABufs && !wwait(&a_empty[ab], ((half / kABufs) - 1) & 1, p.err)) { ok = false; break; }
+                uint32_t v[32];
+                if (BITS == 8) {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {           // 4 x 16 codes = 64 channels
+                        const uint4 w = *reinterpret_cast<const uint4 *>(slot + sw128(t, hh * 4 + q));
+                        i8x4_to_h2x2(w.x, v[q * 8 + 0], v[q * 8 + 1]);
+                        i8x4_to_h2x2(w.y, v[q * 8 + 2], v[q * 8 + 3]);
+                        i8x4_to_h2x2(w.z, v[q * 8 + 4], v[q * 8 + 5]);
+                        i8x4_to_h2x2(w.w, v[q * 8 + 6], v[q * 8 + 7]);
+                    }
+                } else {
+                    const __half2 s2 = __half2half2(__ushort_as_half(sc_cur));
+#pragma unroll
+                    for (int q = 0; q < 2; ++q) {           // 2 x 32 codes = 64 channels
+                        const uint4 w = *reinterpret_cast<const uint4 *>(slot + sw64(t, hh * 2 + q));
+                        i4x8_to_h2x4(w.x, s2, &v[q * 16 + 0]);
+                        i4x8_to_h2x4(w.y, s2, &v[q * 16 + 4]);
+                        i4x8_to_h2x4(w.z, s2, &v[q * 16 + 8]);
+                        i4x8_to_h2x4(w.w, s2, &v[q * 16 + 12]);
+                    }
+                }
+                tmem_st32(trow + kColA + ab * 32, v);
+                tmem_wait_st();
+                fence_before();
+                __syncwarp();
+                if (lane == 0) arrive_local(&a_full[ab]);
+            }
+            __syncwarp();
+            if (lane == 0) arrive_local(&t1_empty[s]);
+            if (!ok) { abort_flag = 1; break; }
+        }
+    } else if (warp < 12) {
+        // ---------------- warpgroup 2: pass-2 converter (fp16 tile in shared memory) ----------------
+        // thread: 16-channel group g of the chunk, tokens tb + 16 k (k = 0..7)
+        const int tid = threadIdx.x - 256, g = tid & 7, tb = tid >> 3;
+        uint16_t scn[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        auto load_scales = [&](int i) {
+            const int tile = i / n_chunks, grp = ch0 / 128 + i % n_chunks;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int tok = t_begin + tile * kTile + tb + 16 * k;
+                scn[k] = load_group_scale(c, row0 + tok, grp, tok < t_end);
+            }
+        };
+        if (BITS == 4 && total > 0) load_scales(0);
+        for (int i = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0); ++i) {
+            const int s = i % kRing, vb = i & 1;
+            uint16_t scl[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) scl[k] = scn[k];
+            if (BITS == 4 && i + 1 < total) load_scales(i + 1);
+            if (!wwait(&t2_full[s], (i / kRing) & 1, p.err)) { abort_flag = 1; break; }
+            if (i >= 2 && !wwait(&pva_empty[vb], ((i >> 1) - 1) & 1, p.err)) { abort_flag = 1; break; }
+            const uint8_t *src = sm + kOffT2 + s * kSlotBytes;
+            uint8_t *dst = sm + kOffPva + vb * kPvaBytes + (g >> 2) * (kTile * 128);
+            const int q0 = (g & 3) * 2;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int t = tb + 16 * k;
+                uint32_t o[8];
+                if (BITS == 8) {
+                    const uint4 w = *reinterpret_cast<const uint4 *>(src + sw128(t, g));
+                    i8x4_to_h2x2(w.x, o[0], o[1]);
+                    i8x4_to_h2x2(w.y, o[2], o[3]);
+                    i8x4_to_h2x2(w.z, o[4], o[5]);
+                    i8x4_to_h2x2(w.w, o[6], o[7]);
+                } else {
+                    const __half2 s2 = __half2half2(__ushort_as_half(scl[k]));
+                    const uint2 w = *reinterpret_cast<const uint2 *>(src + sw64(t, g >> 1) + (g & 1) * 8);
+                    i4x8_to_h2x4(w.x, s2, &o[0]);
+                    i4x8_to_h2x4(w.y, s2, &o[4]);
+                }
+                // [64-channel half][token][64 channels], 128-byte rows, swizzled
+                *reinterpret_cast<uint4 *>(dst + sw128(t, q0)) = make_uint4(o[0], o[1], o[2], o[3]);
+                *reinterpret_cast<uint4 *>(dst + sw128(t, q0 + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
+            }
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                arrive_local(&pva_full[vb]);
+                arrive_local(&t2_empty[s]);
+            }
+        }
+    } else {
+        // ---------------- warpgroup 3: exchange, online softmax, P ----------------
+        // Logits are kept in log2 units.  Each thread (one token) accumulates
+        // its own sums of p per head over the tiles; the sums over tokens are
+        // formed once, at the end.  The reference maximum m_ref of a head only
+        // moves when a logit exceeds it by more than kRescale2 (one vote per
+        // tile); then the tile maximum is reduced through shared memory, and
+        // o_lat and the sums are rescaled.  A failed wait marks the warp
+        // `bad`; the group leaves the tile loop together at its next named
+        // barrier (bar.red.or), so no warp is left at a barrier the others skip.
+        const int quad = warp & 3, t = quad * 32 + lane, wq = warp - 12;
+        const uint32_t trow = tmem + (uint32_t(quad * 32) << 16);
+        const uint32_t xch_remote = map_peer(smem_addr(sm + kOffXch), peer);
+        const uint32_t xfull_remote = map_peer(smem_addr(&xch_full), peer);
+        const uint32_t xempty_remote = map_peer(smem_addr(&xch_empty), peer);
+        float *xr = reinterpret_cast<float *>(sm + kOffXch);   // peer partials, then transposed reductions
+        const float *tscale = static_cast<const float *>(c.scales);
+        float tsc_next = 0.0f;
+        if (BITS == 8 && n_tiles > 0) tsc_next = t_begin + t < t_end ? tscale[row0 + t_begin + t] : 0.0f;
+        float lt[kMaxN];
+#pragma unroll
+        for (int h = 0; h < kMaxN; ++h) lt[h] = 0.0f;
+        bool failed = false;
+        for (int tile = 0; tile < n_tiles; ++tile) {
+            const int sb = tile & 1;
+            const int tok = t_begin + tile * kTile + t;
+            const bool live = tok < t_end;
+            const float tsc = tsc_next;
+            if (BITS == 8 && tile + 1 < n_tiles)
+                tsc_next = tok + kTile < t_end ? tscale[row0 + tok + kTile] : 0.0f;
+            bool bad = __any_sync(0xffffffffu, abort_flag != 0);
+            if (!bad) bad = !wwait(&s_full[sb], (tile >> 1) & 1, p.err);
+            float s[kMaxN];
+            if (!bad) {
+                fence_after();
+                uint32_t v[32];
+                tmem_ld32(trow + kColS + sb * 32, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int h = 0; h < kMaxN; ++h) s[h] = __uint_as_float(v[h]);
+                fence_before();
+                __syncwarp();
+                if (lane == 0) arrive_local(&s_empty[sb]);
+            } else {
+#pragma unroll
+                for (int h = 0; h < kMaxN; ++h) s[h] = 0.0f;
+            }
+            // swap partial scores with the peer: asynchronous stores that
+            // count their bytes on the peer's xch_full, whose phase also needs
+            // the peer's own expect-tx arrival
+            if (t == 0 && !bad) mbar_arrive_expect_tx(&xch_full, kTile * kMaxN * 4);
+            if (!bad && tile > 0) bad = !wwait_cluster(&xch_empty, (tile - 1) & 1, p.err);
+            if (!bad) {
+#pragma unroll
+                for (int h = 0; h < kMaxN; h += 4)
+                    st_async_v4(xch_remote + (t * kMaxN + h) * 4, s[h], s[h + 1], s[h + 2], s[h + 3], xfull_remote);
+                bad = !wwait_cluster(&xch_full, tile & 1, p.err);
+            }
+            bool exceed = false;
+            if (!bad) {
+#pragma unroll
+                for (int h = 0; h < kMaxN; h += 4) {
+                    const float4 o = *reinterpret_cast<const float4 *>(xr + t * kMaxN + h);
+                    // rank 0 computes own + peer, rank 1 peer + own: the same sums on both CTAs
+                    if (rank == 0) { s[h] += o.x; s[h + 1] += o.y; s[h + 2] += o.z; s[h + 3] += o.w; }
+                    else { s[h] = o.x + s[h]; s[h + 1] = o.y + s[h + 1]; s[h + 2] = o.z + s[h + 2]; s[h + 3] = o.w + s[h + 3]; }
+                }
+                // logits in log2 units; dead tokens and padding heads get -inf
+#pragma unroll
+                for (int h = 0; h < kMaxN; ++h) {
+                    const float lg = s[h] * qfac[h] * (BITS == 8 ? tsc : 1.0f);
+                    s[h] = (live && h < H) ? lg : -INFINITY;
+                    exceed |= s[h] > m_ref[h] + kRescale2;
+                }
+            }
+            if (group_any(bad)) { failed = true; break; }
+            if (group_any(exceed)) {
+                // tile maximum per head: the logits, transposed through the exchange buffer
+#pragma unroll
+                for (int h = 0; h < kMaxN; ++h) xr[t * kMaxN + (h ^ lane)] = s[h];
+                asm volatile("bar.sync 1, 128;" ::: "memory");
+                {
+                    float m = -INFINITY;
+#pragma unroll 8
+                    for (int k = 0; k < 32; ++k) m = fmaxf(m, xr[(wq * 32 + k) * kMaxN + (lane ^ k)]);
+                    red_max[wq][lane] = m;
+                }
+                asm volatile("bar.sync 1, 128;" ::: "memory");
+                if (t < kMaxN) {
+                    float a = 1.0f;
+                    if (t < H) {
+                        const float tm = fmaxf(fmaxf(red_max[0][t], red_max[1][t]), fmaxf(red_max[2][t], red_max[3][t]));
+                        const float mr = m_ref[t];
+                        if (tm > mr + kRescale2) {
+                            a = mr == -INFINITY ? 0.0f : exp2f(mr - tm);
+                            m_ref[t] = tm;
+                        }
+                    }
+                    alpha[t] = a;
+                }
+                asm volatile("bar.sync 1, 128;" ::: "memory");
+#pragma unroll
+                for (int h = 0; h < kMaxN; ++h) lt[h] *= alpha[h];
+                if (tile > 0) {
+                    // the PV MMAs of the previous tile must be complete before o_lat is scaled
+                    bad = !wwait(&p_empty[(tile - 1) & 1], ((tile - 1) >> 1) & 1, p.err);
+                    if (!bad) {
+                        fence_after();
+                        for (int ck = 0; ck < n_chunks; ++ck) {
+                            for (int h0 = 0; h0 < Np; h0 += 16) {
+                                uint32_t v[16];
+                                tmem_ld16(trow + kColO + ck * Np + h0, v);
+                                tmem_wait_ld();
+#pragma unroll
+                                for (int e = 0; e < 16; ++e)
+                                    v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha[h0 + e]);
+                                tmem_st16(trow + kColO + ck * Np + h0, v);
+                            }
+                        }
+                        tmem_wait_st();
+                        fence_before();
+                    }
+                }
+            }
+            arrive_peer(xempty_remote);     // this thread is done with the exchange buffer (release)
+            if (!bad && tile >= 2) bad = !wwait(&p_empty[sb], ((tile >> 1) - 1) & 1, p.err);
+            // P^T [heads][tokens], 64-token blocks of Np rows x 128 bytes, swizzled
+            uint8_t *pbuf = sm + kOffP + sb * kPBytes + (t >> 6) * (Np * 128);
+            const int col = t & 63;
+#pragma unroll
+            for (int h = 0; h < kMaxN; ++h) {
+                const float pe = h < H ? exp2f(s[h] - m_ref[h]) : 0.0f;
+                lt[h] += pe;
+                if (!bad && h < Np) {
+                    const __half hv = __float2half_rn(BITS == 8 ? pe * tsc : pe);
+                    *reinterpret_cast<__half *>(pbuf + h * 128 + ((((col >> 3) ^ (h & 7))) << 4) + (col & 7) * 2) = hv;
+                }
+            }
+            fence_async_smem();
+            if (group_any(bad)) { failed = true; break; }
+            __syncwarp();
+            if (lane == 0) arrive_local(&p_full[sb]);
+        }
+        if (failed) abort_flag = 1;
+        // ---- after the last PV MMA: this CTA's channel slice of o_lat, then (rank 0) m and l
+        if (!failed && n_tiles > 0) {
+            const int lt_last = n_tiles - 1;
+            const bool ok = wwait(&p_empty[lt_last & 1], (lt_last >> 1) & 1, p.err);
+            // sums over the tokens, transposed through the exchange buffer (the peer sends no more)
+#pragma unroll
+            for (int h = 0; h < kMaxN; ++h) xr[t * kMaxN + (h ^ lane)] = lt[h];
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            {
+                float sum = 0.0f;
+#pragma unroll 8
+                for (int k = 0; k < 32; ++k) sum += xr[(wq * 32 + k) * kMaxN + (lane ^ k)];
+                red_max[wq][lane] = sum;
+            }
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            if (!group_any(!ok)) {
+                fence_after();
+                const size_t pb = (size_t(b) * p.n_split + split) * H;
+                for (int ck = 0; ck < n_chunks; ++ck) {
+                    const int ch = ch0 + ck * kChunk + t;
+                    for (int h0 = 0; h0 < Np; h0 += 16) {
+                        uint32_t v[16];
+                        tmem_ld16(trow + kColO + ck * Np + h0, v);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 16; ++e)
+                            if (h0 + e < H) p.po[(pb + h0 + e) * r + ch] = __uint_as_float(v[e]);
+                    }
+                }
+                if (rank == 0 && t < H) {
+                    p.pm[pb + t] = m_ref[t] * 0.6931471805599453f;       // natural-log units
+                    p.pl[pb + t] = (red_max[0][t] + red_max[1][t]) + (red_max[2][t] + red_max[3][t]);
+                }
+            } else {
+                abort_flag = 1;
+            }
+        }
+    }
+
+    fence_before();
+    __syncthreads();
+    cluster_sync();                  // the peer has finished every access to this CTA's shared memory
+    fence_after();
+    if (warp == 1) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *q = nullptr;
+        cudaDriverEntryPointQueryResult res;
+        if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &q, cudaEnableDefault, &res) == cudaSuccess &&
+            res == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(q);
+    }
+    return fn;
+}
+
+int g_attn_path = 0;     // 0 automatic, 1 CUDA cores, 2 tensor cores
+
+}  // namespace
+
+void set_attn_path(int path) { g_attn_path = path; }
+int attn_path() { return g_attn_path; }
+
+bool attn_tc_shape_ok(int r, int bits, int H) {
+    const int Np = (H + 15) / 16 * 16;
+    if (bits != 8 && bits != 4) return false;
+    if (r % 256 || r / 2 > atc::kMaxRc || Np > atc::kMaxN) return false;
+    return (r / 2 / atc::kChunk) * Np <= int(atc::kColS - atc::kColO);
+}
+
+bool attn_tc_use(const CacheView &c, int H, int max_seq_len) {
+    if (g_attn_path == 1 || !attn_tc_shape_ok(c.r, c.bits, H) || !encode_fn()) return false;
+    if (g_attn_path == 2) return true;
+    return int64_t(c.B) * max_seq_len >= 4096;      // short caches stay on the CUDA-core kernels
+}
+
+int attn_tc_splits(int B, int max_seq_len, int *tiles_per_split) {
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int tiles = (max_seq_len + atc::kTile - 1) / atc::kTile;
+    const int64_t pairs = sms / 2;                   // CTA pairs resident at once
+    int per = int((int64_t(B) * tiles + 2 * pairs - 1) / (2 * pairs));   // about two waves
+    if (per < 1) per = 1;
+    while ((tiles + per - 1) / per > 64) ++per;      // at most 64 partials per sequence
+    *tiles_per_split = per;
+    return (tiles + per - 1) / per;
+}
+
+cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const float *qt, const unsigned *qmax, int H,
+                           float softmax_scale,
+                           int tiles_per_split, int n_split, float *pm, float *pl, float *po, int *err,
+                           cudaStream_t s) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return cudaErrorNotSupported;
+    // the cache as a byte matrix [B * Tmax rows, row_bytes]; a box is 128 rows
+    // x one chunk (128 bytes of int8, 128-byte swizzle; 64 bytes of int4, 64-byte swizzle)
+    const int row_bytes = c.bits == 8 ? c.r : c.r / 2;
+    CUtensorMap map;
+    const cuuint64_t dims[2] = {cuuint64_t(row_bytes), cuuint64_t(int64_t(c.B) * c.Tmax)};
+    const cuuint64_t strides[1] = {cuuint64_t(row_bytes)};
+    const cuuint32_t box[2] = {c.bits == 8 ? 128u : 64u, 128u};
+    const cuuint32_t estr[2] = {1, 1};
+    if (fn(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, c.codes, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+           c.bits == 8 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return cudaErrorInvalidValue;
+    const atc::Params prm{c, seq_len, qt, qmax, H, (H + 15) / 16 * 16, softmax_scale, tiles_per_split, n_split,
+                          pm, pl, po, err};
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * n_split, c.B);
+    cfg.blockDim = dim3(atc::kThreads);
+    cfg.dynamicSmemBytes = atc::kSmemBytes;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    cudaError_t e;
+    if (c.bits == 8) {
+        e = ensure_smem(attn_tc_kernel<8>, atc::kSmemBytes);
+        if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, attn_tc_kernel<8>, map, prm);
+    } else {
+        e = ensure_smem(attn_tc_kernel<4>, atc::kSmemBytes);
+        if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, attn_tc_kernel<4>, map, prm);
+    }
+    return e;
+}
+
+}  // namespace qsvd

@@ -1,0 +1,537 @@
+// The per-step products with the up-projections around decode attention
+// (Eq. 5 with W^u_k absorbed into the query and W^u_v applied last), for all
+// B sequences of a step at once:
+//
+//   qproj_kernel      a5: q[b] = c_{L_b - 1} U_q
+//   qabsorb_kernel    a5: q~[b, h, j] = U_k[j, h-block] . q[b, h-block], and the
+//                     per-(b, h) maximum of |q~| (it scales the fp16 query of
+//                     the tensor-core attention)
+//   combine_uv_kernel a7/a8: merge the per-split softmax partials of every
+//                     sequence and multiply by U_v[:, h-block]
+//
+// Each is a skinny product (B rows) that streams one up-projection once.  A
+// CTA's weight tile arrives by one or two TMA boxes (or a few large bulk
+// copies); all global loads of a phase are issued before the first use; each
+// thread keeps the sums of NB sequences in registers (NB = the batch rounded up
+// to a power of two, at most 16).  The products over the r latent channels
+// (qproj, combine) are split over a cluster of kCl CTAs, whose partial results
+// are added in rank order through distributed shared memory: the sums are
+// deterministic and need no global scratch.
+#include <cfloat>
+
+#include "common.cuh"
+#include "launch.h"
+
+namespace qsvd {
+
+namespace {
+
+constexpr int kBC = 16;          // largest NB
+constexpr int kCl = 8;           // CTAs per cluster (split of the r latent rows)
+constexpr int kQaRows = 32;      // U_k rows per qabsorb CTA (one per lane)
+constexpr int kMaxSplitsG = 64;  // softmax partials per sequence
+
+__device__ __forceinline__ uint32_t cl_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cl_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Load a float from the same shared-memory offset in CTA `rank` of the cluster.
+__device__ __forceinline__ float ld_rank(const float *p, uint32_t rank) {
+    uint32_t a;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_addr(p)), "r"(rank));
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(smem_addr(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+        : "memory");
+}
+__device__ __forceinline__ void tma_prefetch(const CUtensorMap *map, int x, int y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];"
+                 ::"l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool len_ok(int L, int Tmax) { return L >= 1 && L <= Tmax; }
+
+// Rows of a weight tile per TMA box (box dimensions are at most 256).
+__host__ __device__ __forceinline__ int box_rows(int rs) { return rs / ((rs + 255) / 256); }
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// a5 first half.  Grid (kCl, d / ncol), cluster (kCl, 1, 1), ncol / 2 threads
+// (two columns each).  CTA k of a cluster takes rows [k rs, (k+1) rs) of U_q
+// (rs = r / kCl) and the cluster's ncol columns; rank k then adds the kCl
+// partials of columns [k ncol/kCl, (k+1) ncol/kCl) in rank order.
+// CTA (0, 0) also clears qmax for qabsorb_kernel.
+// ---------------------------------------------------------------------------
+template <int NB>
+__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(128)
+qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32_t *__restrict__ seq_len, int B,
+             int d, float *__restrict__ q, unsigned *__restrict__ qmax, int n_qmax, int *err) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int L_s[NB];
+    const int r = c.r, rs = r / kCl, ncol = 2 * blockDim.x, br = box_rows(rs);
+    const uint32_t rank = cl_rank();
+    const int c0 = blockIdx.y * ncol, j0 = int(rank) * rs;
+    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                          // [rs][ncol] bf16
+    float *c_s = reinterpret_cast<float *>(smem + size_t(rs) * ncol * 2);        // [NB][rs]
+    float *p_s = c_s + NB * rs;                                                  // [NB][ncol]
+    const int tid = threadIdx.x;
+    pdl_trigger();
+    if (tid == 0) {
+        for (int k = 0; k < rs / br; ++k) tma_prefetch(&map_u, c0, j0 + k * br);
+        mbar_init(&bar, 1);
+        mbar_init_fence();
+    }
+    __syncthreads();
+    pdl_wait();
+    if (tid == 0) {
+        mbar_arrive_expect_tx(&bar, uint32_t(rs) * ncol * 2);
+        for (int k = 0; k < rs / br; ++k) tma_2d(u_s + size_t(k) * br * ncol, &map_u, c0, j0 + k * br, &bar);
+    }
+    if (rank == 0 && blockIdx.y == 0)
+        for (int i = tid; i < n_qmax; i += blockDim.x) qmax[i] = 0u;
+    bool ready = false;
+    const int per_rank = ncol / kCl;
+    const int wpr = c.bits == 8 ? rs / 4 : rs / 8;        // 32-bit code words per latent row slice
+    for (int b0 = 0; b0 < B; b0 += NB) {
+        const int nb = min(NB, B - b0);
+        __syncthreads();
+        if (tid < NB) {
+            int L = tid < nb ? seq_len[b0 + tid] : 0;
+            if (tid < nb && !len_ok(L, c.Tmax)) {
+                if (rank == 0 && blockIdx.y == 0) flag_error(err, kErrRange);
+                L = 0;
+            }
+            L_s[tid] = L;
+        }
+        __syncthreads();
+        // dequantized latent rows c_{L-1}: code words and scales, every load issued first
+        // words per thread: nb * wpr / blockDim <= NB * 96 / 64 (rs <= 384; 64 threads when r > 1536)
+        constexpr int kPer = NB * 96 / 64;
+        uint32_t wv[kPer];
+        float sv[kPer];
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) {
+            const int w = tid + k * int(blockDim.x);
+            wv[k] = 0u;
+            sv[k] = 0.0f;
+            if (w < nb * wpr) {
+                const int bi = w / wpr, x = w - bi * wpr;
+                const int L = L_s[bi];
+                if (L > 0) {
+                    const size_t slot = size_t(b0 + bi) * c.Tmax + (L - 1);
+                    if (c.bits == 8) {
+                        wv[k] = reinterpret_cast<const uint32_t *>(static_cast<const int8_t *>(c.codes) + slot * r + j0)[x];
+                        sv[k] = static_cast<const float *>(c.scales)[slot];
+                    } else {
+                        wv[k] = reinterpret_cast<const uint32_t *>(static_cast<const uint8_t *>(c.codes) + slot * (r / 2) + j0 / 2)[x];
+                        sv[k] = __half2float(static_cast<const __half *>(c.scales)[slot * (r / 128) + (j0 + 8 * x) / 128]);
+                    }
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) {
+            const int w = tid + k * int(blockDim.x);
+            if (w >= nb * wpr) break;
+            const int bi = w / wpr, x = w - bi * wpr;
+            if (c.bits == 8) {
+                float4 o;
+                o.x = float(int8_t(wv[k] & 0xff)) * sv[k];
+                o.y = float(int8_t((wv[k] >> 8) & 0xff)) * sv[k];
+                o.z = float(int8_t((wv[k] >> 16) & 0xff)) * sv[k];
+                o.w = float(int8_t(wv[k] >> 24)) * sv[k];
+                *reinterpret_cast<float4 *>(c_s + bi * rs + 4 * x) = o;
+            } else {
+                float f[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) f[e] = float((int((wv[k] >> (4 * e)) & 0xf) ^ 8) - 8) * sv[k];
+                *reinterpret_cast<float4 *>(c_s + bi * rs + 8 * x) = make_float4(f[0], f[1], f[2], f[3]);
+                *reinterpret_cast<float4 *>(c_s + bi * rs + 8 * x + 4) = make_float4(f[4], f[5], f[6], f[7]);
+            }
+        }
+        for (int i = nb * rs + tid; i < NB * rs; i += blockDim.x) c_s[i] = 0.0f;
+        __syncthreads();
+        if (!ready) {
+            mbar_wait(&bar, 0, err);
+            ready = true;
+        }
+        float a0[NB], a1[NB];
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi) a0[bi] = a1[bi] = 0.0f;
+        for (int i = 0; i < rs; i += 2) {            // rs is even (r % 32 == 0)
+            const uint32_t w0 = *reinterpret_cast<const uint32_t *>(u_s + size_t(i) * ncol + 2 * tid);
+            const uint32_t w1 = *reinterpret_cast<const uint32_t *>(u_s + size_t(i + 1) * ncol + 2 * tid);
+            const float u00 = bf16_lo(w0), u01 = bf16_hi(w0), u10 = bf16_lo(w1), u11 = bf16_hi(w1);
+#pragma unroll
+            for (int bi = 0; bi < NB; ++bi) {
+                const float2 cv = *reinterpret_cast<const float2 *>(c_s + bi * rs + i);
+                a0[bi] = fmaf(cv.y, u10, fmaf(cv.x, u00, a0[bi]));
+                a1[bi] = fmaf(cv.y, u11, fmaf(cv.x, u01, a1[bi]));
+            }
+        }
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi)
+            if (bi < nb) *reinterpret_cast<float2 *>(p_s + bi * ncol + 2 * tid) = make_float2(a0[bi], a1[bi]);
+        cl_sync();                                   // every rank's partials are complete
+        for (int o = tid; o < nb * per_rank; o += blockDim.x) {
+            const int bi = o / per_rank, col = int(rank) * per_rank + (o - bi * per_rank);
+            float v = 0.0f;
+#pragma unroll
+            for (int k = 0; k < kCl; ++k) v += ld_rank(p_s + bi * ncol + col, uint32_t(k));
+            q[size_t(b0 + bi) * d + c0 + col] = v;
+        }
+        cl_sync();                                   // partials read before they are overwritten / the CTA exits
+    }
+}
+
+// ---------------------------------------------------------------------------
+// a5 second half.  Grid (ceil(r / 32), H / hg), 32 * hg threads: lane = row j
+// of U_k, warp = head.  The head block of the 32 rows sits in shared memory
+// with rows padded by 16 bytes (conflict-free 16-byte reads).
+// ---------------------------------------------------------------------------
+template <int NB>
+__global__ void __launch_bounds__(256)
+qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int B, int r, int d, int H, int dh,
+               int hg, float *__restrict__ qt, unsigned *__restrict__ qmax, int *err) {
+    extern __shared__ __align__(16) uint8_t smem[];
+    __shared__ __align__(8) uint64_t bar;
+    const int ustride = hg * dh + 8;                                             // bf16 per padded row
+    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                          // [32][ustride]
+    float *q_s = reinterpret_cast<float *>(smem + size_t(kQaRows) * ustride * 2); // [NB][hg * dh]
+    const int j0 = blockIdx.x * kQaRows, h0 = blockIdx.y * hg;
+    const int rows = min(kQaRows, r - j0);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int w = hg * dh;
+    pdl_trigger();
+    if (threadIdx.x < 32)
+        for (int i = lane; i < rows; i += 32)
+            prefetch_l2_bulk(Uk + size_t(j0 + i) * d + size_t(h0) * dh, uint32_t(w) * 2);
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        mbar_init_fence();
+    }
+    __syncthreads();
+    pdl_wait();
+    if (warp == 0) {
+        if (lane == 0) mbar_arrive_expect_tx(&bar, uint32_t(rows) * w * 2);
+        __syncwarp();
+        for (int i = lane; i < rows; i += 32)
+            bulk_g2s(u_s + size_t(i) * ustride, Uk + size_t(j0 + i) * d + size_t(h0) * dh, uint32_t(w) * 2, &bar);
+    }
+    bool ready = false;
+    const int h = h0 + warp;
+    for (int b0 = 0; b0 < B; b0 += NB) {
+        const int nb = min(NB, B - b0);
+        __syncthreads();
+        // q block of the pass, every load issued first (at most NB float4 per thread: dh <= 128)
+        {
+            float4 v[NB];
+            const int n4 = nb * (w / 4);
+#pragma unroll
+            for (int k = 0; k < NB; ++k) {
+                const int idx = threadIdx.x + k * blockDim.x;
+                v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (idx < n4) {
+                    const int bi = idx / (w / 4), c4 = idx - bi * (w / 4);
+                    v[k] = reinterpret_cast<const float4 *>(q + size_t(b0 + bi) * d + size_t(h0) * dh)[c4];
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < NB; ++k) {
+                const int idx = threadIdx.x + k * blockDim.x;
+                if (idx < n4) reinterpret_cast<float4 *>(q_s)[idx] = v[k];
+            }
+        }
+        __syncthreads();
+        if (!ready) {
+            mbar_wait(&bar, 0, err);
+            ready = true;
+        }
+        float acc[NB];
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi) acc[bi] = 0.0f;
+        const uint16_t *urow = u_s + size_t(lane) * ustride + warp * dh;
+        for (int i = 0; i < dh; i += 8) {
+            float f[8];
+            unpack8_bf16(*reinterpret_cast<const uint4 *>(urow + i), f);
+#pragma unroll
+            for (int bi = 0; bi < NB; ++bi) {
+                if (bi >= nb) break;
+                const float4 qa = *reinterpret_cast<const float4 *>(q_s + bi * w + warp * dh + i);
+                const float4 qb = *reinterpret_cast<const float4 *>(q_s + bi * w + warp * dh + i + 4);
+                float a = acc[bi];
+                a = fmaf(f[0], qa.x, a); a = fmaf(f[1], qa.y, a); a = fmaf(f[2], qa.z, a); a = fmaf(f[3], qa.w, a);
+                a = fmaf(f[4], qb.x, a); a = fmaf(f[5], qb.y, a); a = fmaf(f[6], qb.z, a); a = fmaf(f[7], qb.w, a);
+                acc[bi] = a;
+            }
+        }
+        const bool live = lane < rows;
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi) {
+            if (bi >= nb) break;
+            if (live) qt[(size_t(b0 + bi) * H + h) * r + j0 + lane] = acc[bi];
+            const float m = warp_max(live ? fabsf(acc[bi]) : 0.0f);
+            if (lane == 0) atomicMax(qmax + size_t(b0 + bi) * H + h, __float_as_uint(m));
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// a7/a8.  Grid (kCl, H), cluster (kCl, 1, 1), 128 threads.  CTA k of head h's
+// cluster merges, for every sequence, the softmax partials of latent rows
+// [k rs, (k+1) rs) (weights exp(m_s - M) / l), multiplies them by those rows
+// of U_v[:, h-block], and rank k adds the kCl products for its share of the
+// dh output columns in rank order.
+// ---------------------------------------------------------------------------
+template <int NB>
+__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(128)
+combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__restrict__ seq_len, int B, int Tmax,
+                  int H, int dh, int r, int chunk, int n_split, const float *__restrict__ pm,
+                  const float *__restrict__ pl, const float *__restrict__ po, float *__restrict__ O, int *err) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ float w_s[NB][kMaxSplitsG];
+    __shared__ float inv_s[NB];
+    __shared__ int ns_s[NB];
+    const int rs = r / kCl, d = H * dh, h = blockIdx.y, br = box_rows(rs);
+    const uint32_t rank = cl_rank();
+    const int j0 = int(rank) * rs;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                          // [rs][dh] bf16
+    float *ol_s = reinterpret_cast<float *>(smem + size_t(rs) * dh * 2);         // [NB][rs]
+    float *p_s = ol_s + NB * rs;                                                 // [2][NB][dh]
+    pdl_trigger();
+    if (tid == 0) {
+        for (int k = 0; k < rs / br; ++k) tma_prefetch(&map_v, h * dh, j0 + k * br);
+        mbar_init(&bar, 1);
+        mbar_init_fence();
+    }
+    __syncthreads();
+    pdl_wait();
+    if (tid == 0) {
+        mbar_arrive_expect_tx(&bar, uint32_t(rs) * dh * 2);
+        for (int k = 0; k < rs / br; ++k) tma_2d(u_s + size_t(k) * br * dh, &map_v, h * dh, j0 + k * br, &bar);
+    }
+    bool ready = false;
+    const int nq = rs / 4;                           // row quads (r % 32 == 0)
+    const int nsub = 128 / dh, sub = tid / dh, col = tid - sub * dh;
+    const int per_rank = dh / kCl;
+    constexpr int kWB = NB / 4 > 0 ? NB / 4 : 1;     // sequences per warp in the weight phase
+    for (int b0 = 0; b0 < B; b0 += NB) {
+        const int nb = min(NB, B - b0);
+        __syncthreads();
+        // merge weights of every sequence of the pass: warp w takes sequences w, w+4, ...
+        {
+            int ns[kWB];
+            float m0[kWB], m1[kWB], l0[kWB], l1[kWB];
+#pragma unroll
+            for (int k = 0; k < kWB; ++k) {
+                const int bi = warp + 4 * k;
+                const int L = bi < nb ? seq_len[b0 + bi] : 0;
+                ns[k] = len_ok(L, Tmax) ? (L + chunk - 1) / chunk : 0;
+            }
+#pragma unroll
+            for (int k = 0; k < kWB; ++k) {
+                const size_t base = size_t(b0 + warp + 4 * k) * n_split * H + h;
+                m0[k] = lane < ns[k] ? pm[base + size_t(lane) * H] : -FLT_MAX;
+                m1[k] = lane + 32 < ns[k] ? pm[base + size_t(lane + 32) * H] : -FLT_MAX;
+                l0[k] = lane < ns[k] ? pl[base + size_t(lane) * H] : 0.0f;
+                l1[k] = lane + 32 < ns[k] ? pl[base + size_t(lane + 32) * H] : 0.0f;
+            }
+#pragma unroll
+            for (int k = 0; k < kWB; ++k) {
+                const int bi = warp + 4 * k;
+                if (bi >= NB) break;
+                const float M = warp_max(fmaxf(m0[k], m1[k]));
+                const float e0 = lane < ns[k] ? expf(m0[k] - M) : 0.0f;
+                const float e1 = lane + 32 < ns[k] ? expf(m1[k] - M) : 0.0f;
+                w_s[bi][lane] = e0;
+                w_s[bi][lane + 32] = e1;
+                const float l = warp_sum(e0 * l0[k] + e1 * l1[k]);
+                if (lane == 0) {
+                    inv_s[bi] = ns[k] ? 1.0f / l : 0.0f;
+                    ns_s[bi] = ns[k];
+                }
+            }
+        }
+        __syncthreads();
+        // merged o_lat rows: thread = (sequence, row quad); up to 16 partial loads in flight
+        for (int idx = tid; idx < NB * nq; idx += blockDim.x) {
+            const int bi = idx / nq, q4 = idx - bi * nq;
+            const int ns = bi < nb ? ns_s[bi] : 0;
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            const float *src = po + (size_t(b0 + bi) * n_split * H + h) * r + j0 + 4 * q4;
+            for (int s0 = 0; s0 < ns; s0 += 16) {
+                float4 v[16];
+#pragma unroll
+                for (int k = 0; k < 16; ++k)
+                    v[k] = s0 + k < ns ? *reinterpret_cast<const float4 *>(src + size_t(s0 + k) * H * r)
+                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    const float wk = s0 + k < ns ? w_s[bi][s0 + k] : 0.0f;
+                    acc.x = fmaf(wk, v[k].x, acc.x);
+                    acc.y = fmaf(wk, v[k].y, acc.y);
+                    acc.z = fmaf(wk, v[k].z, acc.z);
+                    acc.w = fmaf(wk, v[k].w, acc.w);
+                }
+            }
+            const float il = bi < nb ? inv_s[bi] : 0.0f;
+            *reinterpret_cast<float4 *>(ol_s + bi * rs + 4 * q4) = make_float4(acc.x * il, acc.y * il, acc.z * il, acc.w * il);
+        }
+        __syncthreads();
+        if (!ready) {
+            mbar_wait(&bar, 0, err);
+            ready = true;
+        }
+        // this rank's rows times U_v: thread = (row subset `sub`, output column `col`)
+        float acc[NB];
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi) acc[bi] = 0.0f;
+        for (int i = 4 * sub; i < rs; i += 4 * nsub) {
+            const float u0 = bf16_to_f32(u_s[size_t(i) * dh + col]), u1 = bf16_to_f32(u_s[size_t(i + 1) * dh + col]);
+            const float u2 = bf16_to_f32(u_s[size_t(i + 2) * dh + col]), u3 = bf16_to_f32(u_s[size_t(i + 3) * dh + col]);
+#pragma unroll
+            for (int bi = 0; bi < NB; ++bi) {
+                const float4 o = *reinterpret_cast<const float4 *>(ol_s + bi * rs + i);
+                acc[bi] = fmaf(o.w, u3, fmaf(o.z, u2, fmaf(o.y, u1, fmaf(o.x, u0, acc[bi]))));
+            }
+        }
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi)
+            if (bi < nb) p_s[(sub * NB + bi) * dh + col] = acc[bi];
+        __syncthreads();
+        if (nsub == 2)
+            for (int o = tid; o < nb * dh; o += blockDim.x) p_s[o] += p_s[NB * dh + o];
+        cl_sync();                                   // every rank's products are complete
+        for (int o = tid; o < nb * per_rank; o += blockDim.x) {
+            const int bi = o / per_rank, cc = int(rank) * per_rank + (o - bi * per_rank);
+            float v = 0.0f;
+#pragma unroll
+            for (int k = 0; k < kCl; ++k) v += ld_rank(p_s + bi * dh + cc, uint32_t(k));
+            O[size_t(b0 + bi) * d + size_t(h) * dh + cc] = v;
+        }
+        cl_sync();
+    }
+}
+
+// ---------------------------------------------------------------------------
+namespace {
+
+int qproj_cols(int r) { return r <= 1536 ? 256 : 128; }
+
+int qabsorb_hg(int H) {
+    for (int g = 8; g > 1; g >>= 1)
+        if (H % g == 0) return g;
+    return 1;
+}
+
+// Sequences per pass: the batch rounded up to a power of two, at most kBC.
+int pass_nb(int B) {
+    int nb = 1;
+    while (nb < B && nb < kBC) nb <<= 1;
+    return nb;
+}
+
+template <int NB>
+cudaError_t qproj_nb(const CUtensorMap &map, const CacheView &c, const int32_t *seq_len, int d, float *q,
+                     unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
+    const int rs = c.r / kCl, ncol = qproj_cols(c.r);
+    const size_t smem = size_t(rs) * ncol * 2 + size_t(NB) * rs * 4 + size_t(NB) * ncol * 4;
+    cudaError_t e = ensure_smem(qproj_kernel<NB>, smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(qproj_kernel<NB>, dim3(kCl, d / ncol), dim3(ncol / 2), smem, s, map, c, seq_len, c.B, d, q,
+                      qmax, n_qmax, err);
+}
+
+template <int NB>
+cudaError_t qabsorb_nb(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
+                       unsigned *qmax, int *err, cudaStream_t s) {
+    const int hg = qabsorb_hg(H);
+    const size_t smem = size_t(kQaRows) * (hg * dh + 8) * 2 + size_t(NB) * hg * dh * 4;
+    cudaError_t e = ensure_smem(qabsorb_kernel<NB>, smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(qabsorb_kernel<NB>, dim3((r + kQaRows - 1) / kQaRows, H / hg), dim3(32 * hg), smem, s, q, Uk,
+                      B, r, d, H, dh, hg, qt, qmax, err);
+}
+
+template <int NB>
+cudaError_t combine_nb(const CUtensorMap &map, const int32_t *seq_len, int B, int Tmax, int H, int dh, int r,
+                       int chunk, int n_split, const float *pm, const float *pl, const float *po, float *O, int *err,
+                       cudaStream_t s) {
+    const int rs = r / kCl;
+    const size_t smem = size_t(rs) * dh * 2 + size_t(NB) * rs * 4 + size_t(2) * NB * dh * 4;
+    cudaError_t e = ensure_smem(combine_uv_kernel<NB>, smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(combine_uv_kernel<NB>, dim3(kCl, H), dim3(128), smem, s, map, seq_len, B, Tmax, H, dh, r, chunk,
+                      n_split, pm, pl, po, O, err);
+}
+
+}  // namespace
+
+cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
+                         unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
+    const int rs = c.r / kCl, ncol = qproj_cols(c.r);
+    CUtensorMap map;
+    if (!encode_map_2d(&map, CU_TENSOR_MAP_DATA_TYPE_UINT16, Uq, uint64_t(d), uint64_t(c.r), uint64_t(d) * 2,
+                       uint32_t(ncol), uint32_t(box_rows(rs)), CU_TENSOR_MAP_SWIZZLE_NONE))
+        return cudaErrorInvalidValue;
+    cudaError_t e;
+    switch (pass_nb(c.B)) {
+        case 1: e = qproj_nb<1>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        case 2: e = qproj_nb<2>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        case 4: e = qproj_nb<4>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        case 8: e = qproj_nb<8>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        default: e = qproj_nb<16>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+    }
+    prof_mark(s, "qproj");
+    return e;
+}
+
+cudaError_t launch_qabsorb(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
+                           unsigned *qmax, int *err, cudaStream_t s) {
+    cudaError_t e;
+    switch (pass_nb(B)) {
+        case 1: e = qabsorb_nb<1>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
+        case 2: e = qabsorb_nb<2>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
+        case 4: e = qabsorb_nb<4>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
+        case 8: e = qabsorb_nb<8>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
+        default: e = qabsorb_nb<16>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
+    }
+    prof_mark(s, "qabsorb");
+    return e;
+}
+
+cudaError_t launch_combine_uv(const int32_t *seq_len, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
+                              const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
+                              int *err, cudaStream_t s) {
+    const int rs = r / kCl, d = H * dh;
+    CUtensorMap map;
+    if (!encode_map_2d(&map, CU_TENSOR_MAP_DATA_TYPE_UINT16, Uv, uint64_t(d), uint64_t(r), uint64_t(d) * 2,
+                       uint32_t(dh), uint32_t(box_rows(rs)), CU_TENSOR_MAP_SWIZZLE_NONE))
+        return cudaErrorInvalidValue;
+    cudaError_t e;
+    switch (pass_nb(B)) {
+        case 1: e = combine_nb<1>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 2: e = combine_nb<2>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 4: e = combine_nb<4>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 8: e = combine_nb<8>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        default: e = combine_nb<16>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+    }
+    prof_mark(s, "combine_uv");
+    return e;
+}
+
+}  // namespace qsvd

@@ -6,9 +6,17 @@
 #include <cstddef>
 #include <cstdint>
 #include <utility>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace qsvd {
+
+// 2D tiled TMA descriptor over a row-major matrix of `outer` rows x `inner`
+// elements (rows `row_bytes` apart), box = box_outer rows x box_inner
+// elements.  Returns false if the driver entry point is missing or refuses
+// the parameters.  Defined in api.cu.
+bool encode_map_2d(CUtensorMap *map, CUtensorMapDataType type, const void *base, uint64_t inner, uint64_t outer,
+                   uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swizzle);
 
 // Raise a kernel's dynamic shared memory limit to the maximum the first time
 // it needs more than the default (so that no attribute call happens while a
@@ -114,6 +122,28 @@ struct DecodeArgs {
     float *O;
 };
 size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
+
+// a5 and a7/a8 for all B sequences of a step (decode_gemv.cu).
+cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
+                         unsigned *qmax, int n_qmax, int *err, cudaStream_t s);
+cudaError_t launch_qabsorb(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
+                           unsigned *qmax, int *err, cudaStream_t s);
+cudaError_t launch_combine_uv(const int32_t *seq_len, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
+                              const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
+                              int *err, cudaStream_t s);
+
+// Tensor-core latent attention (a6/a7): choice of kernel, split of each
+// sequence into partials (tiles of 128 tokens), and the launcher, which writes
+// the same (m, l, o_lat) partials as the CUDA-core kernel.
+void set_attn_path(int path);      // 0 automatic, 1 CUDA cores, 2 tensor cores where the shape allows
+int attn_path();
+bool attn_tc_shape_ok(int r, int bits, int H);
+bool attn_tc_use(const CacheView &c, int H, int max_seq_len);
+int attn_tc_splits(int B, int max_seq_len, int *tiles_per_split);
+cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const float *qt, const unsigned *qmax, int H,
+                           float softmax_scale,
+                           int tiles_per_split, int n_split, float *pm, float *pl, float *po, int *err,
+                           cudaStream_t s);
 
 // One fused decode step (a1-a8) for B <= kFuseMaxB sequences, one new token each.
 constexpr int kFuseMaxB = 8;

@@ -206,3 +206,14 @@ def gen_layer(wl: Workload, seed: int = 0, layer: int = 0,
         X_decode = np.stack([_activations(wl.B, s.d, 1.0 if wl.tiny_svd else 0.5, outl, rng)
                              for _ in range(steps)], axis=0)
     return LayerInputs(wl, seed, W_qkv, W_d, U_q, U_k, U_v, outl, X_prefill, X_decode)
+
+
+def latent_rows(n_rows: int, r: int, rng) -> np.ndarray:
+    """Latent rows shaped like x W_d of the synthetic layers: channel j has
+    standard deviation (j+1)^-0.5 (the spectrum decay of the down-projection)
+    times a per-token magnitude drawn log-uniformly from [0.5, 2]; fp32
+    values as fp64 [n_rows, r]."""
+    decay = np.arange(1, r + 1, dtype=np.float64) ** -0.5
+    mag = np.exp(rng.uniform(math.log(0.5), math.log(2.0), size=(n_rows, 1)))
+    x = rng.standard_normal((n_rows, r)) * decay[None, :] * mag
+    return x.astype(np.float32).astype(np.float64)

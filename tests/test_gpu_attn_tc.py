@@ -1,0 +1,124 @@
+"""GPU parity of the tensor-core latent attention (Eq. 5, U_k absorbed into
+the query, U_v applied last) against the oracle.
+
+The cache content is an input here: seeded latent rows quantized by the
+oracle's own quantizer (per-token int8, or int4 with fp16 scales per 128
+channels), written into the device cache as is.  A few tokens repeat the
+current token's latent row, so that their scores stand far above the rest and
+the running softmax maximum jumps late in the sequence.  Every case runs the
+tensor-core kernel (path 2) and, where stated, the CUDA-core kernels (path 1)
+on the same cache; both must match the oracle to 2e-3 * ||o_ref||_2 per row.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import synthetic
+from oracle import attention, quant
+
+from gpu_util import assert_rows_close, bf16, dev, i32, q
+
+pytestmark = pytest.mark.gpu
+
+
+def _up_weights(H, dh, r, seed):
+    shape = synthetic.LayerShape(H * dh, H, dh, r)
+    wl = synthetic.Workload("attn", shape, B=1, n_image=0, n_text=0, decode_steps=0, lat_bits=8)
+    inp = synthetic.gen_layer(wl, seed=seed, prefill_rows=0, decode_steps=0)
+    return inp.U_q, inp.U_k, inp.U_v
+
+
+def _cache_rows(lens, r, seed, hot):
+    """fp64 latent rows per sequence; rows at the `hot` fractions of the
+    length repeat the last (current) row."""
+    rng = np.random.default_rng(seed)
+    rows = []
+    for L in lens:
+        x = synthetic.latent_rows(L, r, rng)
+        for f in hot:
+            t = int(f * (L - 1))
+            if 0 <= t < L - 1:
+                x[t] = x[L - 1]
+        rows.append(x)
+    return rows
+
+
+def _run(H, dh, r, bits, lens, paths=(2, 1), seed=0, hot=(0.3, 0.8), tmax=None):
+    lib = q()
+    B = len(lens)
+    tmax = tmax or max(lens)
+    U_q, U_k, U_v = _up_weights(H, dh, r, seed)
+    rows = _cache_rows(lens, r, seed + 1, hot)
+    cache = lib.LatentCache.empty(B, tmax, r, bits, dev())
+    refs = []
+    for b, (L, x) in enumerate(zip(lens, rows)):
+        if bits == 8:
+            codes, s = quant.quantize_rows(x, 8)
+            C = quant.dequantize_rows(codes, s)
+            cache.codes[b, :L] = torch.from_numpy(codes.astype(np.int8)).to(dev())
+            cache.scales[b, :L] = torch.from_numpy(s.astype(np.float32)).to(dev())
+        else:
+            codes, s16 = quant.quantize_int4_groups(x)
+            C = quant.dequantize_int4_groups(codes, s16)
+            cache.codes[b, :L] = torch.from_numpy(quant.pack_int4(codes)).to(dev())
+            cache.scales[b, :L] = torch.from_numpy(s16.astype(np.float16)).to(dev())
+        refs.append(attention.decode_attention_absorbed(
+            C, synthetic.bf16_from_bits(U_q), synthetic.bf16_from_bits(U_k), synthetic.bf16_from_bits(U_v), H, dh))
+    ref = np.stack(refs)
+    Uq, Uk, Uv = bf16(U_q), bf16(U_k), bf16(U_v)
+    seq_len = i32(lens)
+    outs = {}
+    for path in paths:
+        prev = lib.qsvd_set_decode_attn_path(path)
+        try:
+            O = torch.full((B, H * dh), float("nan"), dtype=torch.float32, device=dev())
+            lib.qsvd_latent_decode_attn(cache, seq_len, max(lens), Uq, Uk, Uv, H, dh, O)
+            lib.qsvd_check()
+        finally:
+            lib.qsvd_set_decode_attn_path(prev)
+        got = O.cpu().numpy()
+        assert np.isfinite(got).all(), f"path {path}: non-finite output"
+        assert_rows_close(got, ref, f"path {path}")
+        outs[path] = got
+    return outs, ref
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_attn_tc_7b_ragged(bits):
+    """r = 1536, H = 32, dh = 128: lengths 1 (the current token alone), one
+    tile minus one, one tile plus one, and several tiles with a ragged tail."""
+    _run(32, 128, 1536, bits, [1, 127, 129, 700])
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_attn_tc_long_sequence_multi_tile_splits(bits):
+    """One 20000-token sequence: each CTA pair walks several tiles, reusing
+    its double buffers, and the late high scores force o_lat rescaling."""
+    _run(32, 128, 1536, bits, [20000], paths=(2,), hot=(0.1, 0.55, 0.97))
+
+
+@pytest.mark.parametrize("H,dh,r,bits", [(8, 128, 512, 8), (20, 64, 768, 8), (20, 64, 768, 4), (16, 64, 256, 4)])
+def test_attn_tc_head_and_rank_shapes(H, dh, r, bits):
+    """N = 16 (H = 8, 16), padded heads (H = 20 -> 32), 1-3 chunks per CTA."""
+    _run(H, dh, r, bits, [300, 64, 1000], seed=2)
+
+
+def test_attn_tc_cache_larger_than_lengths():
+    """Tmax above every length: the rows after each sequence's end belong to
+    no token and must not contribute."""
+    _run(32, 128, 1536, 8, [200, 513], tmax=900, seed=4)
+
+
+def test_attn_tc_path_selection():
+    """The automatic choice uses the tensor cores for a large batch x length
+    and the setting is restored; an unsupported shape falls back silently."""
+    lib = q()
+    assert lib.qsvd_set_decode_attn_path(0) == 0
+    assert lib.qsvd_set_decode_attn_path(2) == 0
+    assert lib.qsvd_set_decode_attn_path(0) == 2
+    with pytest.raises(lib.QsvdError):
+        lib.qsvd_set_decode_attn_path(3)
+    # r = 2048 exceeds the tensor-core kernel's limit: path 2 still answers correctly
+    _run(40, 128, 2048, 8, [300, 40], paths=(2,), seed=6)
