@@ -250,4 +250,80 @@ __device__ __forceinline__ void requant_row_cta(const float *__restrict__ c_hat,
     }
 }
 
+
+// The same per-token requantization by one warp (no block barriers): two
+// passes over the row, the second reading it back from L1/L2.  Codes and
+// scales are identical to requant_row_cta's (the maximum does not depend on
+// the order of reduction).
+__device__ __forceinline__ void requant_row_warp(const float *__restrict__ c_hat, int64_t t, int r, int bits,
+                                                 float clip, void *__restrict__ lat_codes,
+                                                 void *__restrict__ lat_scales, const CacheView &dst,
+                                                 const int32_t *__restrict__ dst_seq,
+                                                 const int32_t *__restrict__ dst_pos, int *err) {
+    const int lane = threadIdx.x & 31;
+    const float4 *row = reinterpret_cast<const float4 *>(c_hat + t * r);
+    const int nq = r / 4;
+    uint8_t *cache_codes = nullptr;
+    void *cache_scale = nullptr;
+    if (dst.codes) {
+        const int b = dst_seq[t], p = dst_pos[t];
+        if (b < 0 || b >= dst.B || p < 0 || p >= dst.Tmax) {
+            if (lane == 0) flag_error(err, kErrRange);
+        } else {
+            const size_t slot = size_t(b) * dst.Tmax + p;
+            if (bits == 8) {
+                cache_codes = static_cast<uint8_t *>(dst.codes) + slot * r;
+                cache_scale = static_cast<float *>(dst.scales) + slot;
+            } else {
+                cache_codes = static_cast<uint8_t *>(dst.codes) + slot * (r / 2);
+                cache_scale = static_cast<__half *>(dst.scales) + slot * (r / 128);
+            }
+        }
+    }
+    uint8_t *tok_codes = lat_codes ? static_cast<uint8_t *>(lat_codes) + t * (bits == 8 ? r : r / 2) : nullptr;
+    if (bits == 8) {
+        float m = 0.0f;
+#pragma unroll 4
+        for (int qi = lane; qi < nq; qi += 32) {
+            const float4 v = row[qi];
+            m = fmaxf(m, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
+        }
+        m = warp_max(m);
+        const float s = quant_scale(m, clip, 127.0f);
+#pragma unroll 4
+        for (int qi = lane; qi < nq; qi += 32) {
+            const float4 v = row[qi];
+            const uint32_t w = uint32_t(quant_code(v.x, s, 127) & 0xff) | (uint32_t(quant_code(v.y, s, 127) & 0xff) << 8) |
+                               (uint32_t(quant_code(v.z, s, 127) & 0xff) << 16) |
+                               (uint32_t(quant_code(v.w, s, 127) & 0xff) << 24);
+            if (tok_codes) reinterpret_cast<uint32_t *>(tok_codes)[qi] = w;
+            if (cache_codes) reinterpret_cast<uint32_t *>(cache_codes)[qi] = w;
+        }
+        if (lane == 0) {
+            if (lat_scales) static_cast<float *>(lat_scales)[t] = s;
+            if (cache_scale) *static_cast<float *>(cache_scale) = s;
+        }
+    } else {
+        // group g = quads 32 g .. 32 g + 31: one quad per lane
+#pragma unroll 4
+        for (int g = 0; g < r / 128; ++g) {
+            const int qi = g * 32 + lane;
+            const float4 v = row[qi];
+            float m = fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w)));
+            m = warp_max(m);
+            const __half hs = int4_group_scale(m, clip);
+            const float s = __half2float(hs);
+            const int c0 = quant_code(v.x, s, 7), c1 = quant_code(v.y, s, 7);
+            const int c2 = quant_code(v.z, s, 7), c3 = quant_code(v.w, s, 7);
+            const uint16_t w = uint16_t((c0 & 0xf) | ((c1 & 0xf) << 4) | ((c2 & 0xf) << 8) | ((c3 & 0xf) << 12));
+            if (tok_codes) reinterpret_cast<uint16_t *>(tok_codes)[qi] = w;
+            if (cache_codes) reinterpret_cast<uint16_t *>(cache_codes)[qi] = w;
+            if (lane == 0) {
+                if (lat_scales) static_cast<__half *>(lat_scales)[t * (r / 128) + g] = hs;
+                if (cache_scale) static_cast<__half *>(cache_scale)[g] = hs;
+            }
+        }
+    }
+}
+
 }  // namespace qsvd

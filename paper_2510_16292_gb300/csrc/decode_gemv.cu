@@ -67,25 +67,27 @@ __host__ __device__ __forceinline__ int box_rows(int rs) { return rs / ((rs + 25
 }  // namespace
 
 // ---------------------------------------------------------------------------
-// a5 first half.  Grid (kCl, d / ncol), cluster (kCl, 1, 1), ncol / 2 threads
-// (two columns each).  CTA k of a cluster takes rows [k rs, (k+1) rs) of U_q
-// (rs = r / kCl) and the cluster's ncol columns; rank k then adds the kCl
-// partials of columns [k ncol/kCl, (k+1) ncol/kCl) in rank order.
-// CTA (0, 0) also clears qmax for qabsorb_kernel.
+// a5 first half.  Grid (kCl, d / ncol), cluster (kCl, 1, 1), 256 threads.
+// CTA k of a cluster takes rows [k rs, (k+1) rs) of U_q (rs = r / kCl) and the
+// cluster's ncol columns.  Thread = (column quad, row group): it accumulates 4
+// columns x NB sequences over its row group; the row groups are added in
+// shared memory, then rank k adds the kCl partials of columns
+// [k ncol/kCl, (k+1) ncol/kCl) in rank order.  CTA (0, 0) also clears qmax.
 // ---------------------------------------------------------------------------
 template <int NB>
-__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(128)
+__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
 qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32_t *__restrict__ seq_len, int B,
-             int d, float *__restrict__ q, unsigned *__restrict__ qmax, int n_qmax, int *err) {
+             int d, int ncol, float *__restrict__ q, unsigned *__restrict__ qmax, int n_qmax, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ int L_s[NB];
-    const int r = c.r, rs = r / kCl, ncol = 2 * blockDim.x, br = box_rows(rs);
+    const int r = c.r, rs = r / kCl, br = box_rows(rs);
+    const int ncq = ncol / 4, G = 256 / ncq, rpg = rs / G;
     const uint32_t rank = cl_rank();
     const int c0 = blockIdx.y * ncol, j0 = int(rank) * rs;
     uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                          // [rs][ncol] bf16
     float *c_s = reinterpret_cast<float *>(smem + size_t(rs) * ncol * 2);        // [NB][rs]
-    float *p_s = c_s + NB * rs;                                                  // [NB][ncol]
+    float *part = c_s + NB * rs;                                                 // [G][NB][ncol]
     const int tid = threadIdx.x;
     pdl_trigger();
     if (tid == 0) {
@@ -104,6 +106,7 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32
     bool ready = false;
     const int per_rank = ncol / kCl;
     const int wpr = c.bits == 8 ? rs / 4 : rs / 8;        // 32-bit code words per latent row slice
+    const int cq = tid % ncq, g = tid / ncq;
     for (int b0 = 0; b0 < B; b0 += NB) {
         const int nb = min(NB, B - b0);
         __syncthreads();
@@ -117,13 +120,12 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32
         }
         __syncthreads();
         // dequantized latent rows c_{L-1}: code words and scales, every load issued first
-        // words per thread: nb * wpr / blockDim <= NB * 96 / 64 (rs <= 384; 64 threads when r > 1536)
-        constexpr int kPer = NB * 96 / 64;
+        constexpr int kPer = (NB * 96 + 255) / 256;      // >= words per thread (rs <= 384)
         uint32_t wv[kPer];
         float sv[kPer];
 #pragma unroll
         for (int k = 0; k < kPer; ++k) {
-            const int w = tid + k * int(blockDim.x);
+            const int w = tid + k * 256;
             wv[k] = 0u;
             sv[k] = 0.0f;
             if (w < nb * wpr) {
@@ -143,7 +145,7 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32
         }
 #pragma unroll
         for (int k = 0; k < kPer; ++k) {
-            const int w = tid + k * int(blockDim.x);
+            const int w = tid + k * 256;
             if (w >= nb * wpr) break;
             const int bi = w / wpr, x = w - bi * wpr;
             if (c.bits == 8) {
@@ -167,29 +169,55 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32
             mbar_wait(&bar, 0, err);
             ready = true;
         }
-        float a0[NB], a1[NB];
+        // 4 columns x NB sequences over rows [g rpg, (g+1) rpg)
+        float acc[NB][4];
 #pragma unroll
-        for (int bi = 0; bi < NB; ++bi) a0[bi] = a1[bi] = 0.0f;
-        for (int i = 0; i < rs; i += 2) {            // rs is even (r % 32 == 0)
-            const uint32_t w0 = *reinterpret_cast<const uint32_t *>(u_s + size_t(i) * ncol + 2 * tid);
-            const uint32_t w1 = *reinterpret_cast<const uint32_t *>(u_s + size_t(i + 1) * ncol + 2 * tid);
-            const float u00 = bf16_lo(w0), u01 = bf16_hi(w0), u10 = bf16_lo(w1), u11 = bf16_hi(w1);
+        for (int bi = 0; bi < NB; ++bi) acc[bi][0] = acc[bi][1] = acc[bi][2] = acc[bi][3] = 0.0f;
+        const int i0 = g * rpg, i1 = i0 + rpg;
+        int i = i0;
+        for (; i + 4 <= i1; i += 4) {
+            float u[4][4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const uint2 w2 = *reinterpret_cast<const uint2 *>(u_s + size_t(i + k) * ncol + 4 * cq);
+                u[k][0] = bf16_lo(w2.x); u[k][1] = bf16_hi(w2.x); u[k][2] = bf16_lo(w2.y); u[k][3] = bf16_hi(w2.y);
+            }
 #pragma unroll
             for (int bi = 0; bi < NB; ++bi) {
-                const float2 cv = *reinterpret_cast<const float2 *>(c_s + bi * rs + i);
-                a0[bi] = fmaf(cv.y, u10, fmaf(cv.x, u00, a0[bi]));
-                a1[bi] = fmaf(cv.y, u11, fmaf(cv.x, u01, a1[bi]));
+                const float4 cv = *reinterpret_cast<const float4 *>(c_s + bi * rs + i);
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    acc[bi][e] = fmaf(cv.w, u[3][e], fmaf(cv.z, u[2][e], fmaf(cv.y, u[1][e], fmaf(cv.x, u[0][e], acc[bi][e]))));
+            }
+        }
+        for (; i < i1; ++i) {                          // rows left over when rpg % 4 != 0
+            const uint2 w2 = *reinterpret_cast<const uint2 *>(u_s + size_t(i) * ncol + 4 * cq);
+            const float u0 = bf16_lo(w2.x), u1 = bf16_hi(w2.x), u2 = bf16_lo(w2.y), u3 = bf16_hi(w2.y);
+#pragma unroll
+            for (int bi = 0; bi < NB; ++bi) {
+                const float cv = c_s[bi * rs + i];
+                acc[bi][0] = fmaf(cv, u0, acc[bi][0]);
+                acc[bi][1] = fmaf(cv, u1, acc[bi][1]);
+                acc[bi][2] = fmaf(cv, u2, acc[bi][2]);
+                acc[bi][3] = fmaf(cv, u3, acc[bi][3]);
             }
         }
 #pragma unroll
         for (int bi = 0; bi < NB; ++bi)
-            if (bi < nb) *reinterpret_cast<float2 *>(p_s + bi * ncol + 2 * tid) = make_float2(a0[bi], a1[bi]);
+            *reinterpret_cast<float4 *>(part + (size_t(g) * NB + bi) * ncol + 4 * cq) =
+                make_float4(acc[bi][0], acc[bi][1], acc[bi][2], acc[bi][3]);
+        __syncthreads();
+        for (int o = tid; o < nb * ncol; o += blockDim.x) {     // row groups in order
+            float v = part[o];
+            for (int k = 1; k < G; ++k) v += part[size_t(k) * NB * ncol + o];
+            part[o] = v;
+        }
         cl_sync();                                   // every rank's partials are complete
         for (int o = tid; o < nb * per_rank; o += blockDim.x) {
             const int bi = o / per_rank, col = int(rank) * per_rank + (o - bi * per_rank);
             float v = 0.0f;
 #pragma unroll
-            for (int k = 0; k < kCl; ++k) v += ld_rank(p_s + bi * ncol + col, uint32_t(k));
+            for (int k = 0; k < kCl; ++k) v += ld_rank(part + bi * ncol + col, uint32_t(k));
             q[size_t(b0 + bi) * d + c0 + col] = v;
         }
         cl_sync();                                   // partials read before they are overwritten / the CTA exits
@@ -289,14 +317,14 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
 }
 
 // ---------------------------------------------------------------------------
-// a7/a8.  Grid (kCl, H), cluster (kCl, 1, 1), 128 threads.  CTA k of head h's
+// a7/a8.  Grid (kCl, H), cluster (kCl, 1, 1), 256 threads.  CTA k of head h's
 // cluster merges, for every sequence, the softmax partials of latent rows
 // [k rs, (k+1) rs) (weights exp(m_s - M) / l), multiplies them by those rows
 // of U_v[:, h-block], and rank k adds the kCl products for its share of the
 // dh output columns in rank order.
 // ---------------------------------------------------------------------------
 template <int NB>
-__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(128)
+__global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
 combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__restrict__ seq_len, int B, int Tmax,
                   int H, int dh, int r, int chunk, int n_split, const float *__restrict__ pm,
                   const float *__restrict__ pl, const float *__restrict__ po, float *__restrict__ O, int *err) {
@@ -309,9 +337,10 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__re
     const uint32_t rank = cl_rank();
     const int j0 = int(rank) * rs;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int nsub = 256 / dh;
     uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                          // [rs][dh] bf16
     float *ol_s = reinterpret_cast<float *>(smem + size_t(rs) * dh * 2);         // [NB][rs]
-    float *p_s = ol_s + NB * rs;                                                 // [2][NB][dh]
+    float *p_s = ol_s + NB * rs;                                                 // [nsub][NB][dh]
     pdl_trigger();
     if (tid == 0) {
         for (int k = 0; k < rs / br; ++k) tma_prefetch(&map_v, h * dh, j0 + k * br);
@@ -326,25 +355,26 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__re
     }
     bool ready = false;
     const int nq = rs / 4;                           // row quads (r % 32 == 0)
-    const int nsub = 128 / dh, sub = tid / dh, col = tid - sub * dh;
+    const int sub = tid / dh, col = tid - sub * dh;
     const int per_rank = dh / kCl;
-    constexpr int kWB = NB / 4 > 0 ? NB / 4 : 1;     // sequences per warp in the weight phase
+    constexpr int kWB = (NB + 7) / 8;                // sequences per warp in the weight phase
+    constexpr int kParts = NB >= 4 ? 1 : 4 / NB;     // lanes sharing one (sequence, row quad)
     for (int b0 = 0; b0 < B; b0 += NB) {
         const int nb = min(NB, B - b0);
         __syncthreads();
-        // merge weights of every sequence of the pass: warp w takes sequences w, w+4, ...
+        // merge weights of every sequence of the pass: warp w takes sequences w, w+8
         {
             int ns[kWB];
             float m0[kWB], m1[kWB], l0[kWB], l1[kWB];
 #pragma unroll
             for (int k = 0; k < kWB; ++k) {
-                const int bi = warp + 4 * k;
+                const int bi = warp + 8 * k;
                 const int L = bi < nb ? seq_len[b0 + bi] : 0;
                 ns[k] = len_ok(L, Tmax) ? (L + chunk - 1) / chunk : 0;
             }
 #pragma unroll
             for (int k = 0; k < kWB; ++k) {
-                const size_t base = size_t(b0 + warp + 4 * k) * n_split * H + h;
+                const size_t base = size_t(b0 + warp + 8 * k) * n_split * H + h;
                 m0[k] = lane < ns[k] ? pm[base + size_t(lane) * H] : -FLT_MAX;
                 m1[k] = lane + 32 < ns[k] ? pm[base + size_t(lane + 32) * H] : -FLT_MAX;
                 l0[k] = lane < ns[k] ? pl[base + size_t(lane) * H] : 0.0f;
@@ -352,7 +382,7 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__re
             }
 #pragma unroll
             for (int k = 0; k < kWB; ++k) {
-                const int bi = warp + 4 * k;
+                const int bi = warp + 8 * k;
                 if (bi >= NB) break;
                 const float M = warp_max(fmaxf(m0[k], m1[k]));
                 const float e0 = lane < ns[k] ? expf(m0[k] - M) : 0.0f;
@@ -367,29 +397,49 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__re
             }
         }
         __syncthreads();
-        // merged o_lat rows: thread = (sequence, row quad); up to 16 partial loads in flight
-        for (int idx = tid; idx < NB * nq; idx += blockDim.x) {
-            const int bi = idx / nq, q4 = idx - bi * nq;
-            const int ns = bi < nb ? ns_s[bi] : 0;
+        // merged o_lat rows: item = (sequence, row quad, part); the kParts lanes of
+        // an item take every kParts-th split and are added by shuffles.  Loads are
+        // branch-free (clamped split index, zero weight) so they stay in flight.
+        const int items = NB * nq * kParts;
+        for (int base = 0; base < items; base += 256) {
+            const int it = base + tid;
+            const int part = it % kParts, rest = it / kParts;
+            const int bi = rest / nq, q4 = rest - bi * nq;
+            const int ns = (it < items && bi < nb) ? ns_s[bi] : 0;
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            const float *src = po + (size_t(b0 + bi) * n_split * H + h) * r + j0 + 4 * q4;
-            for (int s0 = 0; s0 < ns; s0 += 16) {
-                float4 v[16];
+            if (ns > 0) {
+                const float *src = po + (size_t(b0 + bi) * n_split * H + h) * r + j0 + 4 * q4;
+                for (int s0 = part; s0 < ns; s0 += 16 * kParts) {
+                    float4 v[16];
+                    float wk[16];
 #pragma unroll
-                for (int k = 0; k < 16; ++k)
-                    v[k] = s0 + k < ns ? *reinterpret_cast<const float4 *>(src + size_t(s0 + k) * H * r)
-                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+                    for (int k = 0; k < 16; ++k) {
+                        const int sk = s0 + k * kParts;
+                        const int sc = sk < ns ? sk : ns - 1;
+                        v[k] = *reinterpret_cast<const float4 *>(src + size_t(sc) * H * r);
+                        wk[k] = sk < ns ? w_s[bi][sc] : 0.0f;
+                    }
 #pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    const float wk = s0 + k < ns ? w_s[bi][s0 + k] : 0.0f;
-                    acc.x = fmaf(wk, v[k].x, acc.x);
-                    acc.y = fmaf(wk, v[k].y, acc.y);
-                    acc.z = fmaf(wk, v[k].z, acc.z);
-                    acc.w = fmaf(wk, v[k].w, acc.w);
+                    for (int k = 0; k < 16; ++k) {
+                        acc.x = fmaf(wk[k], v[k].x, acc.x);
+                        acc.y = fmaf(wk[k], v[k].y, acc.y);
+                        acc.z = fmaf(wk[k], v[k].z, acc.z);
+                        acc.w = fmaf(wk[k], v[k].w, acc.w);
+                    }
                 }
             }
-            const float il = bi < nb ? inv_s[bi] : 0.0f;
-            *reinterpret_cast<float4 *>(ol_s + bi * rs + 4 * q4) = make_float4(acc.x * il, acc.y * il, acc.z * il, acc.w * il);
+#pragma unroll
+            for (int o = 1; o < kParts; o <<= 1) {
+                acc.x += __shfl_xor_sync(0xffffffffu, acc.x, o);
+                acc.y += __shfl_xor_sync(0xffffffffu, acc.y, o);
+                acc.z += __shfl_xor_sync(0xffffffffu, acc.z, o);
+                acc.w += __shfl_xor_sync(0xffffffffu, acc.w, o);
+            }
+            if (it < items && part == 0) {
+                const float il = bi < nb ? inv_s[bi] : 0.0f;
+                *reinterpret_cast<float4 *>(ol_s + bi * rs + 4 * q4) =
+                    make_float4(acc.x * il, acc.y * il, acc.z * il, acc.w * il);
+            }
         }
         __syncthreads();
         if (!ready) {
@@ -410,11 +460,13 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__re
             }
         }
 #pragma unroll
-        for (int bi = 0; bi < NB; ++bi)
-            if (bi < nb) p_s[(sub * NB + bi) * dh + col] = acc[bi];
+        for (int bi = 0; bi < NB; ++bi) p_s[(sub * NB + bi) * dh + col] = acc[bi];
         __syncthreads();
-        if (nsub == 2)
-            for (int o = tid; o < nb * dh; o += blockDim.x) p_s[o] += p_s[NB * dh + o];
+        for (int o = tid; o < nb * dh; o += blockDim.x) {      // row subsets in order
+            float v = p_s[o];
+            for (int k = 1; k < nsub; ++k) v += p_s[size_t(k) * NB * dh + o];
+            p_s[o] = v;
+        }
         cl_sync();                                   // every rank's products are complete
         for (int o = tid; o < nb * per_rank; o += blockDim.x) {
             const int bi = o / per_rank, cc = int(rank) * per_rank + (o - bi * per_rank);
@@ -448,11 +500,11 @@ int pass_nb(int B) {
 template <int NB>
 cudaError_t qproj_nb(const CUtensorMap &map, const CacheView &c, const int32_t *seq_len, int d, float *q,
                      unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
-    const int rs = c.r / kCl, ncol = qproj_cols(c.r);
-    const size_t smem = size_t(rs) * ncol * 2 + size_t(NB) * rs * 4 + size_t(NB) * ncol * 4;
+    const int rs = c.r / kCl, ncol = qproj_cols(c.r), G = 256 / (ncol / 4);
+    const size_t smem = size_t(rs) * ncol * 2 + size_t(NB) * rs * 4 + size_t(G) * NB * ncol * 4;
     cudaError_t e = ensure_smem(qproj_kernel<NB>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(qproj_kernel<NB>, dim3(kCl, d / ncol), dim3(ncol / 2), smem, s, map, c, seq_len, c.B, d, q,
+    return launch_pdl(qproj_kernel<NB>, dim3(kCl, d / ncol), dim3(256), smem, s, map, c, seq_len, c.B, d, ncol, q,
                       qmax, n_qmax, err);
 }
 
@@ -472,10 +524,10 @@ cudaError_t combine_nb(const CUtensorMap &map, const int32_t *seq_len, int B, in
                        int chunk, int n_split, const float *pm, const float *pl, const float *po, float *O, int *err,
                        cudaStream_t s) {
     const int rs = r / kCl;
-    const size_t smem = size_t(rs) * dh * 2 + size_t(NB) * rs * 4 + size_t(2) * NB * dh * 4;
+    const size_t smem = size_t(rs) * dh * 2 + size_t(NB) * rs * 4 + size_t(256 / dh) * NB * dh * 4;
     cudaError_t e = ensure_smem(combine_uv_kernel<NB>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(combine_uv_kernel<NB>, dim3(kCl, H), dim3(128), smem, s, map, seq_len, B, Tmax, H, dh, r, chunk,
+    return launch_pdl(combine_uv_kernel<NB>, dim3(kCl, H), dim3(256), smem, s, map, seq_len, B, Tmax, H, dh, r, chunk,
                       n_split, pm, pl, po, O, err);
 }
 

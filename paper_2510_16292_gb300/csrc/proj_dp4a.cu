@@ -48,6 +48,7 @@ proj_dp4a_kernel(const int8_t *__restrict__ xq, int64_t T, int d, const int8_t *
 // ---------------------------------------------------------------------------
 constexpr int kPsWarps = 8;
 constexpr int kPsMaxD = 6144;          // d <= 6144: 24 x 16-byte vectors per lane
+constexpr int kPsWarpTok = 4;          // from this many tokens on, one warp per token
 
 __global__ void __launch_bounds__(kPsWarps * 32)
 proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, const int8_t *__restrict__ w,
@@ -78,37 +79,91 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
         mbar_arrive_expect_tx(&bar, uint32_t(rows) * d);
         bulk_g2s(w_s, w + size_t(j0) * d, uint32_t(rows) * d, &bar);
     }
-    // a1: per-token int8 quantization; the whole CTA works on one token at a time
-    for (int t = 0; t < T; ++t) {
-        float f[kPsMaxD / 2048][8];
-        float m = 0.0f;
+    // a1: per-token int8 quantization.  Few tokens: the whole CTA works on one
+    // token at a time; more tokens: one warp per token (see below).
+    if (T < kPsWarpTok) {
+        for (int t = 0; t < T; ++t) {
+            float f[kPsMaxD / 2048][8];
+            float m = 0.0f;
 #pragma unroll
-        for (int k = 0; k < kPsMaxD / 2048; ++k) {
-            const int col = (k * 256 + threadIdx.x) * 8;
-            if (col < d) {
-                unpack8_bf16(*reinterpret_cast<const uint4 *>(X + size_t(t) * d + col), f[k]);
+            for (int k = 0; k < kPsMaxD / 2048; ++k) {
+                const int col = (k * 256 + threadIdx.x) * 8;
+                if (col < d) {
+                    unpack8_bf16(*reinterpret_cast<const uint4 *>(X + size_t(t) * d + col), f[k]);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(f[k][e]));
+                    for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(f[k][e]));
+                }
+            }
+            m = block_max<kPsWarps * 32>(m, red);
+            const float s = quant_scale(m, act_clip, 127.0f);
+#pragma unroll
+            for (int k = 0; k < kPsMaxD / 2048; ++k) {
+                const int col = (k * 256 + threadIdx.x) * 8;
+                if (col < d) {
+                    uint32_t lo = 0, hi = 0;
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        lo |= uint32_t(quant_code(f[k][e], s, 127) & 0xff) << (8 * e);
+                        hi |= uint32_t(quant_code(f[k][e + 4], s, 127) & 0xff) << (8 * e);
+                    }
+                    *reinterpret_cast<uint2 *>(xq_s + size_t(t) * d + col) = make_uint2(lo, hi);
+                    if (xq_out && blockIdx.x == 0)
+                        *reinterpret_cast<uint2 *>(xq_out + size_t(t) * d + col) = make_uint2(lo, hi);
+                }
+            }
+            if (threadIdx.x == 0) {
+                xs_s[t] = s;
+                if (xs_out && blockIdx.x == 0) xs_out[t] = s;
             }
         }
-        m = block_max<kPsWarps * 32>(m, red);
-        const float s = quant_scale(m, act_clip, 127.0f);
+    }
+    // one warp per token: a pass for the maximum, then a pass (from L1) for
+    // the codes; 8 vectors in flight per lane
+    for (int t = warp; t < T && T >= kPsWarpTok; t += kPsWarps) {
+        const uint16_t *xrow = X + size_t(t) * d;
+        float m = 0.0f;
+        for (int k0 = 0; k0 < kPsMaxD / 256; k0 += 8) {
+            uint4 xv[8];
 #pragma unroll
-        for (int k = 0; k < kPsMaxD / 2048; ++k) {
-            const int col = (k * 256 + threadIdx.x) * 8;
-            if (col < d) {
+            for (int k = 0; k < 8; ++k) {
+                const int col = ((k0 + k) * 32 + lane) * 8;
+                xv[k] = col < d ? *reinterpret_cast<const uint4 *>(xrow + col) : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                float f[8];
+                unpack8_bf16(xv[k], f);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(f[e]));
+            }
+        }
+        m = warp_max(m);
+        const float s = quant_scale(m, act_clip, 127.0f);
+        for (int k0 = 0; k0 < kPsMaxD / 256; k0 += 8) {
+            uint4 xv[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int col = ((k0 + k) * 32 + lane) * 8;
+                xv[k] = col < d ? *reinterpret_cast<const uint4 *>(xrow + col) : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int col = ((k0 + k) * 32 + lane) * 8;
+                if (col >= d) break;
+                float f[8];
+                unpack8_bf16(xv[k], f);
                 uint32_t lo = 0, hi = 0;
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    lo |= uint32_t(quant_code(f[k][e], s, 127) & 0xff) << (8 * e);
-                    hi |= uint32_t(quant_code(f[k][e + 4], s, 127) & 0xff) << (8 * e);
+                    lo |= uint32_t(quant_code(f[e], s, 127) & 0xff) << (8 * e);
+                    hi |= uint32_t(quant_code(f[e + 4], s, 127) & 0xff) << (8 * e);
                 }
                 *reinterpret_cast<uint2 *>(xq_s + size_t(t) * d + col) = make_uint2(lo, hi);
                 if (xq_out && blockIdx.x == 0)
                     *reinterpret_cast<uint2 *>(xq_out + size_t(t) * d + col) = make_uint2(lo, hi);
             }
         }
-        if (threadIdx.x == 0) {
+        if (lane == 0) {
             xs_s[t] = s;
             if (xs_out && blockIdx.x == 0) xs_out[t] = s;
         }
@@ -139,10 +194,14 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     __syncthreads();
     if (!last) return;
     __threadfence();
-    float *red8 = red;
-    static_assert(kRqThreads == kPsWarps * 32, "requant_row_cta expects one full CTA");
-    for (int t = 0; t < T; ++t)
-        requant_row_cta(c_hat, t, r, lat_bits, lat_clip, lat_codes, lat_scales, dst, dst_seq, dst_pos, err, red8);
+    if (T < kPsWarpTok) {
+        static_assert(kRqThreads == kPsWarps * 32, "requant_row_cta expects one full CTA");
+        for (int t = 0; t < T; ++t)
+            requant_row_cta(c_hat, t, r, lat_bits, lat_clip, lat_codes, lat_scales, dst, dst_seq, dst_pos, err, red);
+    } else {
+        for (int t = warp; t < T; t += kPsWarps)     // one warp per latent row
+            requant_row_warp(c_hat, t, r, lat_bits, lat_clip, lat_codes, lat_scales, dst, dst_seq, dst_pos, err);
+    }
     if (threadIdx.x == 0) *counter = 0;
 }
 
