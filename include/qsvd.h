@@ -228,6 +228,21 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
                                cudaStream_t stream);
 
 /*
+ * Where qsvd_latent_project requantizes the latent on the tensor-core path
+ * (a library setting, not part of the paper's method; process-wide, not
+ * thread-safe):
+ *   0  automatic (default): in the GEMM epilogue for int4 latents, and for
+ *      int8 latents when r / 256 <= 6 (the per-token maximum is exchanged
+ *      within a cluster of r / 256 CTAs);
+ *   1  always a separate requantization kernel over an fp32 latent in the
+ *      workspace;
+ *   2  in the epilogue whenever possible (int8 needs r / 256 <= 8).
+ * Codes and scales are identical either way.  Returns the previous setting,
+ * or QSVD_EINVAL for another value.
+ */
+int qsvd_set_project_epilogue(int32_t mode);
+
+/*
  * Choice of attention kernels for qsvd_latent_decode_attn (a library setting,
  * not part of the paper's method; process-wide, not thread-safe):
  *   0  automatic (default): the tensor-core kernel when the shape allows it

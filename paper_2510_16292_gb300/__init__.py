@@ -32,7 +32,8 @@ QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
 EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
            "qsvd_decode_step", "qsvd_decode_step_workspace_bytes", "qsvd_latent_project_static",
-           "qsvd_set_decode_attn_path", "qsvd_check", "qsvd_last_error", "qsvd_version")
+           "qsvd_set_decode_attn_path", "qsvd_set_project_epilogue", "qsvd_check", "qsvd_last_error",
+           "qsvd_version")
 
 
 class QsvdError(RuntimeError):
@@ -247,6 +248,16 @@ def qsvd_version() -> int:
 
 
 _lib.qsvd_set_decode_attn_path.argtypes = [_i32]
+_lib.qsvd_set_project_epilogue.argtypes = [_i32]
+
+
+def qsvd_set_project_epilogue(mode: int) -> int:
+    """0 automatic, 1 separate requantization kernel, 2 requantize in the
+    tensor-core GEMM epilogue where possible.  Returns the previous setting."""
+    st = _lib.qsvd_set_project_epilogue(mode)
+    if st < 0:
+        _check(st)
+    return st
 
 
 def qsvd_set_decode_attn_path(path: int) -> int:

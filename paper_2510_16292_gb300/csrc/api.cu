@@ -165,6 +165,13 @@ const char *qsvd_last_error(void) { return g_msg; }
 
 int qsvd_version(void) { return 100; }
 
+int qsvd_set_project_epilogue(int32_t mode) {
+    if (mode < 0 || mode > 2) return fail(QSVD_EINVAL, "set_project_epilogue: mode must be 0, 1 or 2");
+    const int prev = project_epilogue();
+    set_project_epilogue(mode);
+    return prev;
+}
+
 int qsvd_set_decode_attn_path(int32_t path) {
     if (path < 0 || path > 2) return fail(QSVD_EINVAL, "set_decode_attn_path: path must be 0, 1 or 2");
     const int prev = attn_path();
@@ -292,6 +299,13 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
         if (!aligned16(W->codes_bf16)) return fail(QSVD_EINVAL, "latent_project: codes_bf16 must be 16-byte aligned");
         e = launch_xquant(X, T, d, act_clip, xq_out, xq_bf16, xs, stream);
         if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
+        if (gemm_tc_fused_supported(T, r, lat_bits)) {
+            // a2, a3 and a4 in one kernel: the latent never leaves the registers
+            e = launch_gemm_tc_fused(xq_bf16, T, d, W->codes_bf16, W->scale, xs, r, lat_bits, lat_clip, lat_codes,
+                                     lat_scales, dst ? &dv : nullptr, dst_seq, dst_pos, nullptr, acc_out, err,
+                                     stream);
+            return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "tensor-core projection launch");
+        }
         e = launch_gemm_tc(xq_bf16, T, d, W->codes_bf16, W->scale, xs, r, c_hat, acc_out, err, stream);
         if (e != cudaSuccess) return cuda_fail(e, "tensor-core projection launch");
     } else {

@@ -123,6 +123,25 @@ __device__ __forceinline__ bool try_wait_acq_cluster(uint64_t *bar, uint32_t par
                  : "memory");
     return ok != 0;
 }
+// try_wait with a suspend-time hint: the thread sleeps (issuing nothing) until
+// the phase completes or about kSuspendNs pass.
+constexpr uint32_t kSuspendNs = 100000;
+__device__ __forceinline__ bool try_wait_sleep(uint64_t *bar, uint32_t parity, bool cluster) {
+    uint32_t ok;
+    if (cluster)
+        asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
+                     "selp.u32 %0, 1, 0, p;\n\t}"
+                     : "=r"(ok)
+                     : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
+                     : "memory");
+    else
+        asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+                     "selp.u32 %0, 1, 0, p;\n\t}"
+                     : "=r"(ok)
+                     : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
+                     : "memory");
+    return ok != 0;
+}
 __device__ __forceinline__ unsigned long long now_ns() {
     unsigned long long t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -134,8 +153,7 @@ __device__ __noinline__ bool wait_bar(uint64_t *bar, uint32_t parity, int *err, 
     if (cluster ? try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = now_ns();
     for (;;) {
-        for (int i = 0; i < 64; ++i)
-            if (cluster ? try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
+        if (try_wait_sleep(bar, parity, cluster)) return true;
         if (now_ns() - t0 > kWaitNs) {
             flag_error(err, kErrTimeout);
             return false;
@@ -513,36 +531,45 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             if (!wwait(&t1_full[s], (i / kRing) & 1, p.err)) { abort_flag = 1; break; }
             const uint8_t *slot = sm + kOffT1 + s * kSlotBytes;
             bool ok = true;
-            for (int hh = 0; hh < 2; ++hh, ++half) {
-                const int ab = half % kABufs;
-                if (half >= kABufs && !wwait(&a_empty[ab], ((half / kABufs) - 1) & 1, p.err)) { ok = false; break; }
-                uint32_t v[32];
-                if (BITS == 8) {
+            // both 64-channel halves of the chunk: convert, store to tensor memory, one wait
+            const int ab0 = half % kABufs, ab1 = (half + 1) % kABufs;
+            if (half >= kABufs && !wwait(&a_empty[ab0], ((half / kABufs) - 1) & 1, p.err)) ok = false;
+            if (ok && half + 1 >= kABufs && !wwait(&a_empty[ab1], (((half + 1) / kABufs) - 1) & 1, p.err)) ok = false;
+            if (ok) {
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {           // 4 x 16 codes = 64 channels
-                        const uint4 w = *reinterpret_cast<const uint4 *>(slot + sw128(t, hh * 4 + q));
-                        i8x4_to_h2x2(w.x, v[q * 8 + 0], v[q * 8 + 1]);
-                        i8x4_to_h2x2(w.y, v[q * 8 + 2], v[q * 8 + 3]);
-                        i8x4_to_h2x2(w.z, v[q * 8 + 4], v[q * 8 + 5]);
-                        i8x4_to_h2x2(w.w, v[q * 8 + 6], v[q * 8 + 7]);
-                    }
-                } else {
-                    const __half2 s2 = __half2half2(__ushort_as_half(sc_cur));
+                for (int hh = 0; hh < 2; ++hh) {
+                    uint32_t v[32];
+                    if (BITS == 8) {
 #pragma unroll
-                    for (int q = 0; q < 2; ++q) {           // 2 x 32 codes = 64 channels
-                        const uint4 w = *reinterpret_cast<const uint4 *>(slot + sw64(t, hh * 2 + q));
-                        i4x8_to_h2x4(w.x, s2, &v[q * 16 + 0]);
-                        i4x8_to_h2x4(w.y, s2, &v[q * 16 + 4]);
-                        i4x8_to_h2x4(w.z, s2, &v[q * 16 + 8]);
-                        i4x8_to_h2x4(w.w, s2, &v[q * 16 + 12]);
+                        for (int q = 0; q < 4; ++q) {           // 4 x 16 codes = 64 channels
+                            const uint4 w = *reinterpret_cast<const uint4 *>(slot + sw128(t, hh * 4 + q));
+                            i8x4_to_h2x2(w.x, v[q * 8 + 0], v[q * 8 + 1]);
+                            i8x4_to_h2x2(w.y, v[q * 8 + 2], v[q * 8 + 3]);
+                            i8x4_to_h2x2(w.z, v[q * 8 + 4], v[q * 8 + 5]);
+                            i8x4_to_h2x2(w.w, v[q * 8 + 6], v[q * 8 + 7]);
+                        }
+                    } else {
+                        const __half2 s2 = __half2half2(__ushort_as_half(sc_cur));
+#pragma unroll
+                        for (int q = 0; q < 2; ++q) {           // 2 x 32 codes = 64 channels
+                            const uint4 w = *reinterpret_cast<const uint4 *>(slot + sw64(t, hh * 2 + q));
+                            i4x8_to_h2x4(w.x, s2, &v[q * 16 + 0]);
+                            i4x8_to_h2x4(w.y, s2, &v[q * 16 + 4]);
+                            i4x8_to_h2x4(w.z, s2, &v[q * 16 + 8]);
+                            i4x8_to_h2x4(w.w, s2, &v[q * 16 + 12]);
+                        }
                     }
+                    tmem_st32(trow + kColA + (hh ? ab1 : ab0) * 32, v);
                 }
-                tmem_st32(trow + kColA + ab * 32, v);
                 tmem_wait_st();
                 fence_before();
                 __syncwarp();
-                if (lane == 0) arrive_local(&a_full[ab]);
+                if (lane == 0) {
+                    arrive_local(&a_full[ab0]);
+                    arrive_local(&a_full[ab1]);
+                }
             }
+            half += 2;
             __syncwarp();
             if (lane == 0) arrive_local(&t1_empty[s]);
             if (!ok) { abort_flag = 1; break; }

@@ -121,6 +121,23 @@ __device__ __forceinline__ int quant_code(float v, float s, int qmax) {
     return c < -qmax ? -qmax : (c > qmax ? qmax : c);
 }
 
+// The same code from a precomputed inv_s = __frcp_rn(s).  x = fp32(v * inv_s)
+// is within 2^-16 + 2^-17 < 2^-15 of fp32(v / s) for |v / s| <= 127.5, so the
+// two round to the same integer unless fp32(v / s) lies within 2^-15 of a
+// half-integer; inside a margin of 2^-14 around half-integers the correctly
+// rounded quotient is computed instead (also whenever inv_s == 0, which the
+// caller passes for scales too small for a finite reciprocal).  Results equal
+// quant_code's: above |v / s| = 127.5 both clamp.
+__device__ __forceinline__ float quant_inv_scale(float s) { return s > 1e-30f ? __frcp_rn(s) : 0.0f; }
+__device__ __forceinline__ int quant_code_fast(float v, float s, float inv_s, int qmax) {
+    if (s == 0.0f) return 0;
+    float x = v * inv_s;
+    const float f = x - floorf(x);
+    if (inv_s == 0.0f || fabsf(f - 0.5f) < 6.103515625e-05f) x = __fdiv_rn(v, s);   // margin 2^-14
+    int c = __float2int_rn(x);
+    return c < -qmax ? -qmax : (c > qmax ? qmax : c);
+}
+
 // int4 group scale: fp32 scale rounded to fp16 (nearest even), saturated.
 __device__ __forceinline__ __half int4_group_scale(float absmax, float clip) {
     return __float2half_rn(fminf(quant_scale(absmax, clip, 7.0f), 65504.0f));

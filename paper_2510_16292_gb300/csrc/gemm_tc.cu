@@ -20,7 +20,14 @@
 //               columns 128*((w-2)/4) .. +127, of each chunk's accumulator
 //               into int32 registers, then c_hat = (fp32(acc) s_x[t]) s_w[j]
 // Two BN-column accumulators alternate between chunks so that the MMA of
-// chunk c+1 overlaps the drain of chunk c.  A wide tile (BN=256) halves the
+// chunk c+1 overlaps the drain of chunk c.
+//
+// With LAT = 8 or 4 the per-token requantization of the latent (the rest of
+// a3) and its store (a4) run in the same epilogue; c_hat never leaves the
+// registers.  int4: a thread holds one token x one 128-channel group, so the
+// group scale is local.  int8: the absmax of a token spans the r / BN CTAs of
+// its row block, which form one cluster along N and swap their per-row maxima
+// through distributed shared memory before quantizing.  A wide tile (BN=256) halves the
 // number of MMA instructions per byte and cuts L2 traffic per MAC by a
 // quarter; narrow tiles are kept for small T, where they give more CTAs.
 #include <cuda.h>
@@ -96,11 +103,25 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
 // ---------------------------------------------------------------------------
-template <int BN>
+// Destinations of the fused requantization (LAT != 0).
+struct LatOut {
+    float clip;
+    void *codes, *scales;              // token-major, or null
+    CacheView dst;                     // dst.codes null: no cache store
+    const int32_t *seq, *pos;
+};
+
+__device__ __forceinline__ uint32_t g_cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+template <int BN, int LAT>
 __global__ void __launch_bounds__(GemmCfg<BN>::kThreads, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_w, int64_t T, int d,
                int r, const float *__restrict__ xs, const float *__restrict__ ws, float *__restrict__ c_hat,
-               int32_t *__restrict__ acc_out, int *err) {
+               int32_t *__restrict__ acc_out, const LatOut lo, int *err) {
     using C = GemmCfg<BN>;
     constexpr int kStages = C::kStages, kStageB = C::kStageB;
     extern __shared__ uint8_t smem_raw[];
@@ -110,6 +131,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
     __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages];
     __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2];
     __shared__ uint32_t tmem_base;
+    __shared__ float red_m[BN / 128][kBM];                 // per-row max of each 128-column half
+    __shared__ float xmax[8][kBM];                         // per-row max of every CTA of the cluster (int8)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m0 = blockIdx.y * kBM, n0 = blockIdx.x * BN;      // N fastest: a wave shares X tiles
     const int n_k = d / kBK;
@@ -141,6 +164,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
     const uint32_t tmem = tmem_base;
     pdl_wait();
 
+    int32_t acc[128];                                     // epilogue: the tile row's int32 sums, then c_hat bits
+    bool epi_ok = false;
     if (warp == 0) {
         // ---------------- TMA producer ----------------
         if (lane == 0) {
@@ -185,7 +210,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
         const int quad = warp & 3;                        // TMEM lane quadrant of this warp
         const int col0 = ((warp - 2) >> 2) * 128;         // this warp's 128 columns of the tile
         const int row = quad * 32 + lane;                 // row of the tile (token)
-        int32_t acc[128];
 #pragma unroll
         for (int j = 0; j < 128; ++j) acc[j] = 0;
         bool ok = true;
@@ -207,25 +231,122 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
             __syncwarp();
             if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&acc_empty[buf])) : "memory");
         }
+        epi_ok = ok;
         const int64_t t = m0 + row;
-        if (ok && t < T) {
-            const float sx = xs[t];
-            const int nc = n0 + col0;
+        const bool live = ok && t < T;
+        const int nc = n0 + col0;
+        if (live && acc_out) {
+            int32_t *ao = acc_out + t * r + nc;
+#pragma unroll
+            for (int j = 0; j < 128; j += 4)
+                *reinterpret_cast<int4 *>(ao + j) = make_int4(acc[j], acc[j + 1], acc[j + 2], acc[j + 3]);
+        }
+        // c_hat = (fp32(acc) s_x[t]) s_w[j], kept in the same registers (as float bits)
+        const float sx = live ? xs[t] : 0.0f;
+        float m = 0.0f;
+#pragma unroll
+        for (int j = 0; j < 128; ++j) {
+            const float v = __fmul_rn(__fmul_rn(__int2float_rn(acc[j]), sx), live ? ws[nc + j] : 0.0f);
+            acc[j] = __float_as_int(v);
+            m = fmaxf(m, fabsf(v));
+        }
+        if (live && c_hat) {
             float *out = c_hat + t * r + nc;
 #pragma unroll
-            for (int j = 0; j < 128; j += 4) {
-                float4 v;
-                v.x = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 0]), sx), ws[nc + j + 0]);
-                v.y = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 1]), sx), ws[nc + j + 1]);
-                v.z = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 2]), sx), ws[nc + j + 2]);
-                v.w = __fmul_rn(__fmul_rn(__int2float_rn(acc[j + 3]), sx), ws[nc + j + 3]);
-                *reinterpret_cast<float4 *>(out + j) = v;
-            }
-            if (acc_out) {
-                int32_t *ao = acc_out + t * r + nc;
+            for (int j = 0; j < 128; j += 4)
+                *reinterpret_cast<float4 *>(out + j) = make_float4(__int_as_float(acc[j]), __int_as_float(acc[j + 1]),
+                                                                   __int_as_float(acc[j + 2]), __int_as_float(acc[j + 3]));
+        }
+        if (LAT == 8) {
+            red_m[col0 / 128][row] = m;
+            asm volatile("bar.sync 1, %0;" ::"r"(C::kEpiWarps * 32) : "memory");
+            if (col0 == 0) {
+                float mc = red_m[0][row];
 #pragma unroll
-                for (int j = 0; j < 128; j += 4)
-                    *reinterpret_cast<int4 *>(ao + j) = make_int4(acc[j], acc[j + 1], acc[j + 2], acc[j + 3]);
+                for (int k = 1; k < BN / 128; ++k) mc = fmaxf(mc, red_m[k][row]);
+                // this CTA's row maximum into slot [rank][row] of every CTA of the cluster
+                const uint32_t cs = gridDim.x, rank = g_cluster_rank();
+                const uint32_t local = smem_addr(&xmax[rank][row]);
+                for (uint32_t p = 0; p < cs; ++p) {
+                    uint32_t remote;
+                    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(p));
+                    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote), "f"(mc) : "memory");
+                }
+            }
+        }
+    }
+    if (LAT == 8) {
+        // every thread of every CTA of the cluster (the maxima are exchanged)
+        asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+    }
+    if (LAT != 0 && warp >= 2) {
+        const int quad = warp & 3, col0 = ((warp - 2) >> 2) * 128, row = quad * 32 + lane;
+        const int64_t t = m0 + row;
+        const int nc = n0 + col0;
+        const bool live = epi_ok && t < T;
+        if (live) {
+            // destinations of row t (cache slot bounds-checked)
+            uint8_t *cache_codes = nullptr;
+            void *cache_scale = nullptr;
+            if (lo.dst.codes) {
+                const int b = lo.seq[t], p = lo.pos[t];
+                if (b < 0 || b >= lo.dst.B || p < 0 || p >= lo.dst.Tmax) {
+                    if (col0 == 0 && blockIdx.x == 0) flag_error(err, kErrRange);
+                } else {
+                    const size_t slot = size_t(b) * lo.dst.Tmax + p;
+                    cache_codes = static_cast<uint8_t *>(lo.dst.codes) + slot * (LAT == 8 ? r : r / 2);
+                    cache_scale = LAT == 8 ? static_cast<void *>(static_cast<float *>(lo.dst.scales) + slot)
+                                           : static_cast<void *>(static_cast<__half *>(lo.dst.scales) + slot * (r / 128));
+                }
+            }
+            uint8_t *tok_codes = lo.codes ? static_cast<uint8_t *>(lo.codes) + t * (LAT == 8 ? r : r / 2) : nullptr;
+            if (LAT == 8) {
+                float mt = 0.0f;
+                for (uint32_t p = 0; p < gridDim.x; ++p) mt = fmaxf(mt, xmax[p][row]);
+                const float s = quant_scale(mt, lo.clip, 127.0f);
+                const float is = quant_inv_scale(s);
+#pragma unroll
+                for (int j = 0; j < 128; j += 16) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        w[q] = uint32_t(quant_code_fast(__int_as_float(acc[j + 4 * q + 0]), s, is, 127) & 0xff) |
+                               (uint32_t(quant_code_fast(__int_as_float(acc[j + 4 * q + 1]), s, is, 127) & 0xff) << 8) |
+                               (uint32_t(quant_code_fast(__int_as_float(acc[j + 4 * q + 2]), s, is, 127) & 0xff) << 16) |
+                               (uint32_t(quant_code_fast(__int_as_float(acc[j + 4 * q + 3]), s, is, 127) & 0xff) << 24);
+                    const uint4 v4 = make_uint4(w[0], w[1], w[2], w[3]);
+                    if (tok_codes) *reinterpret_cast<uint4 *>(tok_codes + nc + j) = v4;
+                    if (cache_codes) *reinterpret_cast<uint4 *>(cache_codes + nc + j) = v4;
+                }
+                if (nc == 0) {                            // the CTA holding channels 0..127 writes the scale
+                    if (lo.scales) static_cast<float *>(lo.scales)[t] = s;
+                    if (cache_scale) *static_cast<float *>(cache_scale) = s;
+                }
+            } else {
+                float mg = 0.0f;                          // the thread's 128 channels are one group
+#pragma unroll
+                for (int j = 0; j < 128; ++j) mg = fmaxf(mg, fabsf(__int_as_float(acc[j])));
+                const __half hs = int4_group_scale(mg, lo.clip);
+                const float s = __half2float(hs);
+                const float is = quant_inv_scale(s);
+#pragma unroll
+                for (int j = 0; j < 128; j += 32) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint32_t x = 0;
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            x |= uint32_t(quant_code_fast(__int_as_float(acc[j + 8 * q + e]), s, is, 7) & 0xf) << (4 * e);
+                        w[q] = x;
+                    }
+                    const uint4 v4 = make_uint4(w[0], w[1], w[2], w[3]);
+                    if (tok_codes) *reinterpret_cast<uint4 *>(tok_codes + (nc + j) / 2) = v4;
+                    if (cache_codes) *reinterpret_cast<uint4 *>(cache_codes + (nc + j) / 2) = v4;
+                }
+                const int g = nc / 128;
+                if (lo.scales) static_cast<__half *>(lo.scales)[t * (r / 128) + g] = hs;
+                if (cache_scale) static_cast<__half *>(cache_scale)[g] = hs;
             }
         }
     }
@@ -270,17 +391,43 @@ static bool make_map(CUtensorMap *map, const void *base, int64_t rows, int cols,
 
 bool gemm_tc_supported(int d, int r) { return d % kBK == 0 && r % 128 == 0 && encode_fn() != nullptr; }
 
-template <int BN>
+// Tile width and whether the per-token requantization can run in the epilogue:
+// int4 always; int8 when the r / BN CTAs of a row block fit one portable
+// cluster (<= 8).
+static int pick_bn(int64_t T, int r, int lat_bits, bool *fuse) {
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t wide_tiles = ((T + kBM - 1) / kBM) * (r / 256);
+    int bn = (r % 256 == 0 && wide_tiles >= 2 * sms) ? 256 : 128;
+    if (lat_bits == 8 && r / bn > 8 && r % 256 == 0) bn = 256;
+    *fuse = lat_bits == 4 || (lat_bits == 8 && r / bn <= 8);
+    return bn;
+}
+
+template <int BN, int LAT>
 static cudaError_t launch_bn(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
-                             const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s) {
+                             const float *xs, int r, float *c_hat, int32_t *acc_out, const LatOut &lo, int *err,
+                             cudaStream_t s) {
     using C = GemmCfg<BN>;
     CUtensorMap mx, mw;
     if (!make_map(&mx, xq_bf16, T, d, kBM) || !make_map(&mw, w_bf16, r, d, BN)) return cudaErrorInvalidValue;
-    cudaError_t e = ensure_smem(gemm_tc_kernel<BN>, C::kSmem);
+    cudaError_t e = ensure_smem(gemm_tc_kernel<BN, LAT>, C::kSmem);
     if (e != cudaSuccess) return e;
-    dim3 grid(unsigned(r / BN), unsigned((T + kBM - 1) / kBM));
-    e = launch_pdl(gemm_tc_kernel<BN>, grid, dim3(C::kThreads), C::kSmem, s, mx, mw, T, d, r, xs, ws, c_hat, acc_out,
-                   err);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(r / BN), unsigned((T + kBM - 1) / kBM));
+    cfg.blockDim = dim3(C::kThreads);
+    cfg.dynamicSmemBytes = C::kSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;        // int8 epilogue: one cluster per row block
+    attr[1].val.clusterDim.x = LAT == 8 ? unsigned(r / BN) : 1u;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = LAT == 8 ? 2 : 1;
+    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN, LAT>, mx, mw, T, d, r, xs, ws, c_hat, acc_out, lo, err);
     prof_mark(s, "gemm_tc");
     return e;
 }
@@ -288,12 +435,42 @@ static cudaError_t launch_bn(const uint16_t *xq_bf16, int64_t T, int d, const ui
 cudaError_t launch_gemm_tc(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
                            const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s) {
     if (T == 0) return cudaSuccess;
-    int dev = 0, sms = 148;
-    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int64_t wide_tiles = ((T + kBM - 1) / kBM) * (r / 256);
-    if (r % 256 == 0 && wide_tiles >= 2 * sms)
-        return launch_bn<256>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, err, s);
-    return launch_bn<128>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, err, s);
+    bool fuse = false;
+    const int bn = pick_bn(T, r, 0, &fuse);
+    const LatOut lo{};
+    return bn == 256 ? launch_bn<256, 0>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s)
+                     : launch_bn<128, 0>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s);
+}
+
+namespace {
+int g_epilogue_mode = 0;     // 0 automatic, 1 separate requantization kernel, 2 fused where possible
+}
+void set_project_epilogue(int mode) { g_epilogue_mode = mode; }
+int project_epilogue() { return g_epilogue_mode; }
+
+bool gemm_tc_fused_supported(int64_t T, int r, int lat_bits) {
+    bool fuse = false;
+    const int bn = pick_bn(T, r, lat_bits, &fuse);
+    if (!fuse || g_epilogue_mode == 1) return false;
+    if (g_epilogue_mode == 2) return true;
+    // automatic: int8 clusters wider than 6 CTAs leave SMs of each GPC idle
+    return lat_bits == 4 || r / bn <= 6;
+}
+
+cudaError_t launch_gemm_tc_fused(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
+                                 const float *xs, int r, int lat_bits, float lat_clip, void *lat_codes,
+                                 void *lat_scales, const CacheView *dst, const int32_t *dst_seq,
+                                 const int32_t *dst_pos, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    bool fuse = false;
+    const int bn = pick_bn(T, r, lat_bits, &fuse);
+    if (!fuse) return cudaErrorInvalidValue;
+    LatOut lo{lat_clip, lat_codes, lat_scales, dst ? *dst : CacheView{}, dst_seq, dst_pos};
+    if (lat_bits == 8)
+        return bn == 256 ? launch_bn<256, 8>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s)
+                         : launch_bn<128, 8>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s);
+    return bn == 256 ? launch_bn<256, 4>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s)
+                     : launch_bn<128, 4>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s);
 }
 
 }  // namespace qsvd

@@ -99,6 +99,17 @@ bool gemm_tc_supported(int d, int r);
 cudaError_t launch_gemm_tc(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
                            const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s);
 
+// The same GEMM with the per-token requantization and store of the latent
+// (a3 second half + a4) in its epilogue; c_hat and acc_out are optional
+// debug outputs (null: not written).
+bool gemm_tc_fused_supported(int64_t T, int r, int lat_bits);
+void set_project_epilogue(int mode);     // 0 automatic, 1 separate requantization, 2 fused where possible
+int project_epilogue();
+cudaError_t launch_gemm_tc_fused(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
+                                 const float *xs, int r, int lat_bits, float lat_clip, void *lat_codes,
+                                 void *lat_scales, const CacheView *dst, const int32_t *dst_seq,
+                                 const int32_t *dst_pos, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s);
+
 // Per-token requantization of c_hat [T, r] into the latent format (a3 second
 // half), written token-major and/or into the cache (a4).
 cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float clip,
