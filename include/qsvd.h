@@ -245,13 +245,16 @@ int qsvd_set_project_epilogue(int32_t mode);
 /*
  * Choice of attention kernels for qsvd_latent_decode_attn (a library setting,
  * not part of the paper's method; process-wide, not thread-safe):
- *   0  automatic (default): the tensor-core kernel when the shape allows it
- *      and B * max_seq_len >= 4096, else the CUDA-core kernels;
+ *   0  automatic (default): the warp-level tensor-core kernel when
+ *      B * max_seq_len <= 16384 or the tcgen05 kernel cannot take the shape,
+ *      else the tcgen05 kernel (the warp-level kernel needs
+ *      max_seq_len <= 4096; beyond that, the CUDA-core kernels);
  *   1  always the CUDA-core kernels;
- *   2  the tensor-core kernel whenever the shape allows it.
- * The tensor-core kernel needs r % 256 == 0, r <= 1536, H <= 32 and
- * (r / 256) * ceil16(H) <= 192; other shapes always use the CUDA-core
- * kernels.  Both give the same results up to floating-point rounding.
+ *   2  the tcgen05 kernel whenever the shape allows it;
+ *   3  the warp-level tensor-core kernel whenever max_seq_len <= 4096.
+ * The tcgen05 kernel needs r % 256 == 0, r <= 1536, H <= 32 and
+ * (r / 256) * ceil16(H) <= 192; other shapes use the CUDA-core kernels.  All
+ * give the same results up to floating-point rounding.
  * Returns the previous setting, or QSVD_EINVAL for another value.
  */
 int qsvd_set_decode_attn_path(int32_t path);

@@ -149,7 +149,11 @@ bool encode_map_2d(CUtensorMap *map, CUtensorMapDataType type, const void *base,
 
 void prof_mark(cudaStream_t s, const char *label) {
     if (!t_prof_events || int(t_prof_labels.size()) >= t_prof_capacity) return;
-    if (cudaEventRecord(t_prof_events[t_prof_labels.size()], s) == cudaSuccess)
+    // inside a stream capture the record becomes an event-record node of the graph
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    (void)cudaStreamIsCapturing(s, &cs);
+    const unsigned flags = cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault;
+    if (cudaEventRecordWithFlags(t_prof_events[t_prof_labels.size()], s, flags) == cudaSuccess)
         t_prof_labels.push_back(label);
     else
         (void)cudaGetLastError();     // a bad event handle must not surface as a launch error
@@ -173,7 +177,7 @@ int qsvd_set_project_epilogue(int32_t mode) {
 }
 
 int qsvd_set_decode_attn_path(int32_t path) {
-    if (path < 0 || path > 2) return fail(QSVD_EINVAL, "set_decode_attn_path: path must be 0, 1 or 2");
+    if (path < 0 || path > 3) return fail(QSVD_EINVAL, "set_decode_attn_path: path must be 0, 1, 2 or 3");
     const int prev = attn_path();
     set_attn_path(path);
     return prev;

@@ -837,7 +837,7 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
-int g_attn_path = 0;     // 0 automatic, 1 CUDA cores, 2 tensor cores
+int g_attn_path = 0;     // 0 automatic, 1 CUDA cores, 2 tcgen05, 3 warp-level MMA
 
 }  // namespace
 
@@ -852,9 +852,9 @@ bool attn_tc_shape_ok(int r, int bits, int H) {
 }
 
 bool attn_tc_use(const CacheView &c, int H, int max_seq_len) {
-    if (g_attn_path == 1 || !attn_tc_shape_ok(c.r, c.bits, H) || !encode_fn()) return false;
+    if (g_attn_path == 1 || g_attn_path == 3 || !attn_tc_shape_ok(c.r, c.bits, H) || !encode_fn()) return false;
     if (g_attn_path == 2) return true;
-    return int64_t(c.B) * max_seq_len >= 4096;      // short caches stay on the CUDA-core kernels
+    return int64_t(c.B) * max_seq_len >= 4096;
 }
 
 int attn_tc_splits(int B, int max_seq_len, int *tiles_per_split) {

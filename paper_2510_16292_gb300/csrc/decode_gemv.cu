@@ -53,6 +53,9 @@ __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int x,
         ::"r"(smem_addr(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
         : "memory");
 }
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
 __device__ __forceinline__ void tma_prefetch(const CUtensorMap *map, int x, int y) {
     asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];"
                  ::"l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y)
@@ -76,8 +79,9 @@ __host__ __device__ __forceinline__ int box_rows(int rs) { return rs / ((rs + 25
 // ---------------------------------------------------------------------------
 template <int NB>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
-qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32_t *__restrict__ seq_len, int B,
-             int d, int ncol, float *__restrict__ q, unsigned *__restrict__ qmax, int n_qmax, int *err) {
+qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restrict__ Uq, CacheView c,
+             const int32_t *__restrict__ seq_len, int B, int d, int ncol, float *__restrict__ q,
+             unsigned *__restrict__ qmax, int n_qmax, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ int L_s[NB];
@@ -97,10 +101,13 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32
     }
     __syncthreads();
     pdl_wait();
-    if (tid == 0) {
-        mbar_arrive_expect_tx(&bar, uint32_t(rs) * ncol * 2);
-        for (int k = 0; k < rs / br; ++k) tma_2d(u_s + size_t(k) * br * ncol, &map_u, c0, j0 + k * br, &bar);
+    // the U_q tile: 16-byte asynchronous copies by every thread (many small
+    // rows: cheaper than bulk or tensor copies of 512-byte rows)
+    for (int i = tid; i < rs * (ncol / 8); i += blockDim.x) {
+        const int row = i / (ncol / 8), k = i - row * (ncol / 8);
+        cp_async16(u_s + size_t(row) * ncol + 8 * k, Uq + size_t(j0 + row) * d + c0 + 8 * k);
     }
+    asm volatile("cp.async.commit_group;" ::: "memory");
     if (rank == 0 && blockIdx.y == 0)
         for (int i = tid; i < n_qmax; i += blockDim.x) qmax[i] = 0u;
     bool ready = false;
@@ -164,11 +171,11 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, CacheView c, const int32
             }
         }
         for (int i = nb * rs + tid; i < NB * rs; i += blockDim.x) c_s[i] = 0.0f;
-        __syncthreads();
         if (!ready) {
-            mbar_wait(&bar, 0, err);
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
             ready = true;
         }
+        __syncthreads();
         // 4 columns x NB sequences over rows [g rpg, (g+1) rpg)
         float acc[NB][4];
 #pragma unroll
@@ -325,7 +332,8 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
 // ---------------------------------------------------------------------------
 template <int NB>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
-combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__restrict__ seq_len, int B, int Tmax,
+combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__restrict__ Uv,
+                  const int32_t *__restrict__ seq_len, int B, int Tmax,
                   int H, int dh, int r, int chunk, int n_split, const float *__restrict__ pm,
                   const float *__restrict__ pl, const float *__restrict__ po, float *__restrict__ O, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -349,10 +357,11 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__re
     }
     __syncthreads();
     pdl_wait();
-    if (tid == 0) {
-        mbar_arrive_expect_tx(&bar, uint32_t(rs) * dh * 2);
-        for (int k = 0; k < rs / br; ++k) tma_2d(u_s + size_t(k) * br * dh, &map_v, h * dh, j0 + k * br, &bar);
+    for (int i = tid; i < rs * (dh / 8); i += blockDim.x) {     // the U_v tile, 16-byte asynchronous copies
+        const int row = i / (dh / 8), k = i - row * (dh / 8);
+        cp_async16(u_s + size_t(row) * dh + 8 * k, Uv + size_t(j0 + row) * d + size_t(h) * dh + 8 * k);
     }
+    asm volatile("cp.async.commit_group;" ::: "memory");
     bool ready = false;
     const int nq = rs / 4;                           // row quads (r % 32 == 0)
     const int sub = tid / dh, col = tid - sub * dh;
@@ -441,11 +450,11 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const int32_t *__re
                     make_float4(acc.x * il, acc.y * il, acc.z * il, acc.w * il);
             }
         }
-        __syncthreads();
         if (!ready) {
-            mbar_wait(&bar, 0, err);
+            asm volatile("cp.async.wait_group 0;" ::: "memory");
             ready = true;
         }
+        __syncthreads();
         // this rank's rows times U_v: thread = (row subset `sub`, output column `col`)
         float acc[NB];
 #pragma unroll
@@ -498,13 +507,13 @@ int pass_nb(int B) {
 }
 
 template <int NB>
-cudaError_t qproj_nb(const CUtensorMap &map, const CacheView &c, const int32_t *seq_len, int d, float *q,
+cudaError_t qproj_nb(const CUtensorMap &map, const uint16_t *Uq, const CacheView &c, const int32_t *seq_len, int d, float *q,
                      unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
     const int rs = c.r / kCl, ncol = qproj_cols(c.r), G = 256 / (ncol / 4);
     const size_t smem = size_t(rs) * ncol * 2 + size_t(NB) * rs * 4 + size_t(G) * NB * ncol * 4;
     cudaError_t e = ensure_smem(qproj_kernel<NB>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(qproj_kernel<NB>, dim3(kCl, d / ncol), dim3(256), smem, s, map, c, seq_len, c.B, d, ncol, q,
+    return launch_pdl(qproj_kernel<NB>, dim3(kCl, d / ncol), dim3(256), smem, s, map, Uq, c, seq_len, c.B, d, ncol, q,
                       qmax, n_qmax, err);
 }
 
@@ -520,15 +529,15 @@ cudaError_t qabsorb_nb(const float *q, const uint16_t *Uk, int B, int r, int d, 
 }
 
 template <int NB>
-cudaError_t combine_nb(const CUtensorMap &map, const int32_t *seq_len, int B, int Tmax, int H, int dh, int r,
+cudaError_t combine_nb(const CUtensorMap &map, const uint16_t *Uv, const int32_t *seq_len, int B, int Tmax, int H, int dh, int r,
                        int chunk, int n_split, const float *pm, const float *pl, const float *po, float *O, int *err,
                        cudaStream_t s) {
     const int rs = r / kCl;
     const size_t smem = size_t(rs) * dh * 2 + size_t(NB) * rs * 4 + size_t(256 / dh) * NB * dh * 4;
     cudaError_t e = ensure_smem(combine_uv_kernel<NB>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(combine_uv_kernel<NB>, dim3(kCl, H), dim3(256), smem, s, map, seq_len, B, Tmax, H, dh, r, chunk,
-                      n_split, pm, pl, po, O, err);
+    return launch_pdl(combine_uv_kernel<NB>, dim3(kCl, H), dim3(256), smem, s, map, Uv, seq_len, B, Tmax, H, dh, r,
+                      chunk, n_split, pm, pl, po, O, err);
 }
 
 }  // namespace
@@ -542,11 +551,11 @@ cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const uint1
         return cudaErrorInvalidValue;
     cudaError_t e;
     switch (pass_nb(c.B)) {
-        case 1: e = qproj_nb<1>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-        case 2: e = qproj_nb<2>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-        case 4: e = qproj_nb<4>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-        case 8: e = qproj_nb<8>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-        default: e = qproj_nb<16>(map, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        case 1: e = qproj_nb<1>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        case 2: e = qproj_nb<2>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        case 4: e = qproj_nb<4>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        case 8: e = qproj_nb<8>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
+        default: e = qproj_nb<16>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
     }
     prof_mark(s, "qproj");
     return e;
@@ -576,11 +585,11 @@ cudaError_t launch_combine_uv(const int32_t *seq_len, int B, int Tmax, int H, in
         return cudaErrorInvalidValue;
     cudaError_t e;
     switch (pass_nb(B)) {
-        case 1: e = combine_nb<1>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 2: e = combine_nb<2>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 4: e = combine_nb<4>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 8: e = combine_nb<8>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        default: e = combine_nb<16>(map, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 1: e = combine_nb<1>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 2: e = combine_nb<2>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 4: e = combine_nb<4>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 8: e = combine_nb<8>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        default: e = combine_nb<16>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
     }
     prof_mark(s, "combine_uv");
     return e;

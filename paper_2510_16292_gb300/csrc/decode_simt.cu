@@ -36,13 +36,12 @@ struct DecodeWs {
 };
 
 // Partials per sequence the workspace holds: enough for either attention
-// kernel (the tensor-core kernel uses at most one per 128-token tile, <= 64).
+// kernel (chunks of at least 16 tokens, at most kMaxSplits of them), and
+// non-decreasing in max_seq_len so that a workspace sized for a bound also
+// serves every shorter call.
 static int split_capacity(int max_seq_len) {
-    const int chunk = chunk_tokens(max_seq_len);
-    const int ns = (max_seq_len + chunk - 1) / chunk;
-    int tiles = (max_seq_len + 127) / 128;
-    if (tiles > kMaxSplits) tiles = kMaxSplits;
-    return ns > tiles ? ns : tiles;
+    const int ns = (max_seq_len + 15) / 16;
+    return ns < kMaxSplits ? ns : kMaxSplits;
 }
 
 static size_t carve(int B, int max_seq_len, int r, int H, int dh, char *base, DecodeWs *w) {
@@ -312,7 +311,15 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
 
     int chunk = chunk_tokens(a.max_seq_len);
     int ns = (a.max_seq_len + chunk - 1) / chunk;
-    if (attn_tc_use(c, H, a.max_seq_len)) {
+    if (attn_mma_use(c, H, B, a.max_seq_len) && attn_mma_fits(a.max_seq_len)) {
+        // a6/a7 on the warp-level tensor-core MMA: one partial per range of ts tokens
+        int ts = 16;
+        ns = attn_mma_splits(B, H, a.max_seq_len, &ts);
+        chunk = ts;
+        e = launch_attn_mma(c, a.seq_len, w.qt, w.qmax, H, a.softmax_scale, ts, ns, w.pm, w.pl, w.po, err, s);
+        if (e != cudaSuccess) return e;
+        prof_mark(s, "attn_mma");
+    } else if (attn_tc_use(c, H, a.max_seq_len)) {
         // a6/a7 on the tensor cores: splits of whole 128-token tiles
         int per = 1;
         ns = attn_tc_splits(B, a.max_seq_len, &per);

@@ -24,7 +24,7 @@ bool encode_map_2d(CUtensorMap *map, CUtensorMapDataType type, const void *base,
 cudaError_t ensure_smem_ptr(const void *kernel, size_t bytes);
 template <typename K>
 cudaError_t ensure_smem(K kernel, size_t bytes) {
-    return bytes <= 48 * 1024 ? cudaSuccess : ensure_smem_ptr(reinterpret_cast<const void *>(kernel), bytes);
+    return ensure_smem_ptr(reinterpret_cast<const void *>(kernel), bytes);     // static + dynamic may pass 48 KiB
 }
 
 // Launch with programmatic stream serialization: the kernel may start while
@@ -146,11 +146,18 @@ cudaError_t launch_combine_uv(const int32_t *seq_len, int B, int Tmax, int H, in
 // Tensor-core latent attention (a6/a7): choice of kernel, split of each
 // sequence into partials (tiles of 128 tokens), and the launcher, which writes
 // the same (m, l, o_lat) partials as the CUDA-core kernel.
-void set_attn_path(int path);      // 0 automatic, 1 CUDA cores, 2 tensor cores where the shape allows
+void set_attn_path(int path);      // 0 automatic, 1 CUDA cores, 2 tcgen05 where the shape allows, 3 warp MMA
 int attn_path();
 bool attn_tc_shape_ok(int r, int bits, int H);
 bool attn_tc_use(const CacheView &c, int H, int max_seq_len);
 int attn_tc_splits(int B, int max_seq_len, int *tiles_per_split);
+// Warp-level tensor-core attention for small batch x length (attn_mma.cu).
+bool attn_mma_use(const CacheView &c, int H, int B, int max_seq_len);
+bool attn_mma_fits(int max_seq_len);
+int attn_mma_splits(int B, int H, int max_seq_len, int *ts);
+cudaError_t launch_attn_mma(const CacheView &c, const int32_t *seq_len, const float *qt, const unsigned *qmax, int H,
+                            float softmax_scale, int ts, int n_split, float *pm, float *pl, float *po, int *err,
+                            cudaStream_t s);
 cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const float *qt, const unsigned *qmax, int H,
                            float softmax_scale,
                            int tiles_per_split, int n_split, float *pm, float *pl, float *po, int *err,

@@ -111,6 +111,21 @@ def test_attn_tc_cache_larger_than_lengths():
     _run(32, 128, 1536, 8, [200, 513], tmax=900, seed=4)
 
 
+@pytest.mark.parametrize("bits", [8, 4])
+def test_attn_mma_ragged(bits):
+    """The warp-level MMA kernel (path 3): lengths 1, 15, 17, 700 at r = 1536,
+    H = 32 (16-token splits), against the oracle and the other kernels."""
+    outs, ref = _run(32, 128, 1536, bits, [1, 15, 17, 700], paths=(3, 2, 1), seed=12)
+
+
+@pytest.mark.parametrize("H,dh,r,bits,lens", [(40, 128, 2048, 8, [3000, 77]), (4, 64, 96, 8, [80, 33]),
+                                               (20, 64, 768, 4, [2049, 64])])
+def test_attn_mma_shapes(H, dh, r, bits, lens):
+    """H = 40 (five head groups of 8) at the 13B rank with 64-token splits,
+    the tiny layer (r = 96, padded heads), and a 32-token split with int4."""
+    _run(H, dh, r, bits, lens, paths=(3,), seed=13)
+
+
 def test_attn_tc_path_selection():
     """The automatic choice uses the tensor cores for a large batch x length
     and the setting is restored; an unsupported shape falls back silently."""
@@ -119,6 +134,6 @@ def test_attn_tc_path_selection():
     assert lib.qsvd_set_decode_attn_path(2) == 0
     assert lib.qsvd_set_decode_attn_path(0) == 2
     with pytest.raises(lib.QsvdError):
-        lib.qsvd_set_decode_attn_path(3)
+        lib.qsvd_set_decode_attn_path(4)
     # r = 2048 exceeds the tensor-core kernel's limit: path 2 still answers correctly
     _run(40, 128, 2048, 8, [300, 40], paths=(2,), seed=6)

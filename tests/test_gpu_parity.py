@@ -290,3 +290,43 @@ def test_project_13b_shape_tc():
         got = _project_outputs(W, X, wl.shape.r, bits)
         ref = latent.latent_project(synthetic.bf16_from_bits(X), w["Wq"], w["s_w"], lat_bits=bits)
         _assert_project_exact(got, ref, bits)
+
+
+# ---------------------------------------------------------------------------
+# requantization in the GEMM epilogue vs the separate kernel
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("mode", [1, 2])
+@pytest.mark.parametrize("shape_name,T", [("llava7b", 300), ("llava13b", 300)])
+def test_project_epilogue_modes(mode, shape_name, T):
+    """Both requantization placements (separate kernel: mode 1; GEMM
+    epilogue, int8 through a cluster of r/256 CTAs: mode 2) give the oracle's
+    codes and scales, into the token-major outputs and into the cache."""
+    lib = q()
+    base = synthetic.WORKLOADS[shape_name]
+    wl = synthetic.Workload("epi", base.shape, B=1, n_image=T, n_text=0, decode_steps=0, lat_bits=8)
+    inp = synthetic.gen_layer(wl, seed=11)
+    w = pipeline.prepare_weights(inp)
+    W = lib.qsvd_quantize_weight(torch.from_numpy(w["W_d"].astype(np.float32)).to(dev()))
+    X = inp.X_prefill[0]
+    r = wl.shape.r
+    prev = lib.qsvd_set_project_epilogue(mode)
+    try:
+        for bits in (8, 4):
+            got = _project_outputs(W, X, r, bits)
+            ref = latent.latent_project(synthetic.bf16_from_bits(X), w["Wq"], w["s_w"], lat_bits=bits)
+            _assert_project_exact(got, ref, bits)
+            # the cache store of the same call (rows scattered over two sequences)
+            cache = lib.LatentCache.empty(2, T, r, bits, dev())
+            seq = np.arange(T) % 2
+            pos = np.arange(T) // 2
+            lib.qsvd_latent_project(W, bf16(X), 1.0, bits, 1.0, dst=cache, dst_seq=i32(seq), dst_pos=i32(pos))
+            lib.qsvd_check()
+            codes = cache.codes.cpu().numpy()[seq, pos]
+            scales = cache.scales.cpu().numpy()[seq, pos]
+            if bits == 8:
+                np.testing.assert_array_equal(codes.astype(np.int64), ref["codes"])
+            else:
+                np.testing.assert_array_equal(codes, quant.pack_int4(ref["codes"]))
+            np.testing.assert_array_equal(scales.astype(np.float64), ref["scale"])
+    finally:
+        lib.qsvd_set_project_epilogue(prev)
