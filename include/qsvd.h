@@ -25,9 +25,13 @@
  *     reused by later calls on the same stream, but two calls that may run
  *     concurrently on the GPU need separate workspaces.
  *   - Kernels are launched with programmatic dependent launch: a call may
- *     begin prefetching its (read-only) weights into L2 while the previous
- *     kernel in the stream is still running; every read of data produced by
- *     earlier stream work happens after that work has completed.
+ *     begin copying its (read-only) weights W_d, U_q, U_k, U_v into shared
+ *     memory and L2 while the previous kernel in the stream is still running;
+ *     every read of other data produced by earlier stream work happens after
+ *     that work has completed.  So the weights must not be written by a
+ *     kernel that permits dependent launches early and runs just before on
+ *     the same stream (ordinary kernels and copies, and
+ *     qsvd_quantize_weight, are fine).
  *   - Calls are asynchronous on `stream` and never synchronize it, except
  *     qsvd_check.  A return of QSVD_OK means the work was enqueued.
  *   - bf16 buffers are passed as uint16_t bit patterns.

@@ -105,12 +105,18 @@ attn_mma_kernel(const am::Params p) {
     __half *ps = gsc + (BITS == 4 ? size_t(TS) * (r / 128) : 0);                       // [kHG][TS + 8] P
     const int pstride = TS + 8;
     pdl_trigger();
-    pdl_wait();
-    const int L = p.seq_len[b];
+    const int L = p.seq_len[b];                                    // an input: no kernel writes it
     const int t_begin = split * TS;
     if (L < 1 || L > c.Tmax || t_begin >= L) return;               // invalid lengths are flagged by qproj_kernel
     const int n = min(TS, L - t_begin);
     const size_t slot0 = size_t(b) * c.Tmax + t_begin;
+    if (threadIdx.x == 0) {
+        // L2 prefetch of the split's cache rows while the producer grid finishes
+        // (L2 is the point of coherence, so a row written meanwhile is never
+        // seen stale: the shared-memory copies below come after the wait)
+        prefetch_l2_bulk(static_cast<const uint8_t *>(c.codes) + slot0 * row_bytes, uint32_t(n) * row_bytes);
+    }
+    pdl_wait();
 
     // ---- 1. cache rows (zero beyond n), scales, query block.  The q~ loads are
     // issued first and the cache rows copied asynchronously meanwhile; the

@@ -12,20 +12,26 @@
 // tensor-memory footprint of the o_lat accumulator and the bytes each SM
 // reads.
 //
-// Per tile the CTA streams its channels twice (the second stream hits L2):
-//   pass 1  warp 0 loads 128-token x 128-channel chunks with TMA; warpgroup 1
-//           (one thread per token) converts 64 channels at a time to fp16 and
-//           stores them into tensor memory; warp 1 issues
+// Both products take their A operand from tensor memory, so no fp16 copy of
+// the cache is ever written to or read from shared memory.  Per tile the CTA
+// streams its channels twice (the second stream hits L2):
+//   pass 1  warp 0 loads 128-token x 128-channel chunks with TMA; warpgroups
+//           1-2 (thread = token, one 64-channel half each) convert them to
+//           fp16 and store them into tensor memory token-major; warp 1 issues
 //              S[t, h] += C[t, ch] Q[ch, h]      (M = 128 tokens, N = heads,
-//           A from tensor memory, B = the fp16 query block in shared memory).
-//   softmax warpgroup 3 reads S, swaps partials with the peer, applies the
-//           token scale and 1/sqrt(dh), runs the online softmax (o_lat is
-//           rescaled lazily, only when the running maximum of a head grows by
-//           more than kRescale2) and writes P (fp16, [heads x tokens]).
-//   pass 2  warp 3 loads the same chunks again; warpgroup 2 converts them to
-//           an fp16 tile in shared memory; warp 2 issues
-//              O^T[ch, h] += C^T[ch, t] P[t, h]  (M = 128 channels, K = tokens,
-//           A = the tile read channel-major, B = P).
+//           B = the fp16 query block in shared memory).
+//   softmax warpgroups 5-6 (thread = token, 16 heads each) read S, swap
+//           partials with the peer, apply the token scale and 1/sqrt(dh), run
+//           the online softmax (o_lat is rescaled lazily, only when the
+//           running maximum of a head grows by more than kRescale2) and write
+//           P (fp16, [heads x tokens]).
+//   pass 2  warp 3 loads the same chunks again (and, for int4, the tile's
+//           group scales); warpgroups 3-4 convert them to fp16, transpose
+//           8 x 8 blocks in registers (movmatrix) and store them channel-major
+//           into tensor memory; warp 2 issues
+//              O^T[ch, h] += C^T[ch, t] P[t, h]  (M = 128 channels, K = tokens).
+//           The transposed blocks put the 16 tokens of an MMA step in the
+//           order 0,1,8,9,2,3,10,11,...; P is written in the same order.
 // int8 codes are exact in fp16; the per-token scale multiplies the scores and
 // is folded into P.  int4 codes are converted to code * group-scale in fp16.
 // The query block is scaled per head by a power of two so that its largest
@@ -47,32 +53,37 @@ namespace atc {
 
 constexpr int kTile = 128;        // tokens per tile
 constexpr int kChunk = 128;       // channels per TMA chunk
-constexpr int kThreads = 512;     // 16 warps
-constexpr int kRing = 2;          // TMA slots per pass
+constexpr int kThreads = 896;     // 28 warps
+constexpr int kRing1 = 4;         // pass-1 TMA slots
+constexpr int kRing2 = 3;         // pass-2 TMA slots
 constexpr int kMaxN = 32;         // heads (padded to a multiple of 16)
+constexpr int kHalfN = 16;        // heads per softmax warpgroup
 constexpr int kMaxRc = 768;       // channels per CTA
+constexpr int kMaxGroups = 12;    // int4 scale groups per token (r <= 1536)
 constexpr float kRescale2 = 11.5f;  // lazy rescale threshold (log2 units, about 8 in natural-log units)
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per wait
 
 // dynamic shared memory (byte offsets from a 1024-aligned base)
 constexpr int kQtBytes = kMaxN * kMaxRc * 2;       // query block, fp16, 128-byte swizzled, K-major
 constexpr int kSlotBytes = kTile * kChunk;         // one int8 chunk (int4 uses half)
-constexpr int kPvaBytes = kTile * kChunk * 2;      // fp16 tile of one chunk
 constexpr int kPBytes = kMaxN * kTile * 2;         // P, fp16, 128-byte swizzled, K-major
 constexpr int kXchBytes = kTile * kMaxN * 4;       // the peer's partial scores
+constexpr int kScBytes = kTile * kMaxGroups * 2;   // int4 group scales of one tile, [token][group]
 constexpr int kOffQt = 0;
 constexpr int kOffT1 = kOffQt + kQtBytes;
-constexpr int kOffT2 = kOffT1 + kRing * kSlotBytes;
-constexpr int kOffPva = kOffT2 + kRing * kSlotBytes;
-constexpr int kOffP = kOffPva + 2 * kPvaBytes;
+constexpr int kOffT2 = kOffT1 + kRing1 * kSlotBytes;
+constexpr int kOffP = kOffT2 + kRing2 * kSlotBytes;
 constexpr int kOffXch = kOffP + 2 * kPBytes;
-constexpr int kSmemBytes = kOffXch + kXchBytes + 1024;
+constexpr int kOffSc = kOffXch + kXchBytes;
+constexpr int kOffLt = kOffSc + 2 * kScBytes;      // softmax running sums, [heads][tokens] fp32
+constexpr int kSmemBytes = kOffLt + kMaxN * kTile * 4 + 1024;
 
 // tensor memory columns
 constexpr uint32_t kColO = 0;      // o_lat^T: (r_c / 128) x Np       (<= 192)
 constexpr uint32_t kColS = 192;    // scores: 2 buffers x 32
 constexpr int kABufs = 4;          // scores A operand buffers (64 channels each)
 constexpr uint32_t kColA = 256;    // scores A operand: kABufs x 32 columns
+constexpr uint32_t kColV = 384;    // PV A operand: 2 buffers x 64 columns (128 tokens, fp16 pairs)
 constexpr uint32_t kTmemCols = 512;
 
 struct Params {
@@ -111,6 +122,11 @@ __device__ __forceinline__ void st_async_v4(uint32_t addr, float a, float b, flo
 __device__ __forceinline__ void arrive_peer(uint32_t bar_cluster_addr) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster_addr) : "memory");
 }
+// Relaxed remote arrival: used where the caller's earlier accesses to the
+// peer-written buffer are reads whose values it has already consumed.
+__device__ __forceinline__ void arrive_peer_relaxed(uint32_t bar_cluster_addr) {
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster_addr) : "memory");
+}
 __device__ __forceinline__ void arrive_local(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
@@ -123,38 +139,36 @@ __device__ __forceinline__ bool try_wait_acq_cluster(uint64_t *bar, uint32_t par
                  : "memory");
     return ok != 0;
 }
-// try_wait with a suspend-time hint: the thread sleeps (issuing nothing) until
-// the phase completes or about kSuspendNs pass.
-constexpr uint32_t kSuspendNs = 100000;
-__device__ __forceinline__ bool try_wait_sleep(uint64_t *bar, uint32_t parity, bool cluster) {
+// Cluster-scope test without the acquire (no L1 invalidation per try); the
+// caller fences once after the phase completed.
+__device__ __forceinline__ bool try_wait_relaxed_cluster(uint64_t *bar, uint32_t parity) {
     uint32_t ok;
-    if (cluster)
-        asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
-                     "selp.u32 %0, 1, 0, p;\n\t}"
-                     : "=r"(ok)
-                     : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
-                     : "memory");
-    else
-        asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-                     "selp.u32 %0, 1, 0, p;\n\t}"
-                     : "=r"(ok)
-                     : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
-                     : "memory");
+    asm volatile("{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.relaxed.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+                 "selp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(ok)
+                 : "r"(smem_addr(bar)), "r"(parity)
+                 : "memory");
     return ok != 0;
 }
+__device__ __forceinline__ void fence_acquire_cluster() { asm volatile("fence.acq_rel.cluster;" ::: "memory"); }
 __device__ __forceinline__ unsigned long long now_ns() {
     unsigned long long t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
     return t;
 }
-// Wait for phase `parity` of `bar`, for at most kWaitNs.  `cluster`: acquire
-// at cluster scope (the phase is completed by the peer CTA).
+// Wait for phase `parity` of `bar`, for at most kWaitNs.  Each try_wait
+// suspends the thread in hardware until the phase completes or a short
+// system-defined time passes, so the loop issues little; the clock is read
+// every 64 tries.  `cluster`: the phase is completed by the peer CTA (relaxed
+// tries, one cluster-scope acquire fence at the end).
 __device__ __noinline__ bool wait_bar(uint64_t *bar, uint32_t parity, int *err, bool cluster) {
-    if (cluster ? try_wait_acq_cluster(bar, parity) : mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = now_ns();
-    for (;;) {
-        if (try_wait_sleep(bar, parity, cluster)) return true;
-        if (now_ns() - t0 > kWaitNs) {
+    for (uint32_t i = 1;; ++i) {
+        if (cluster ? try_wait_relaxed_cluster(bar, parity) : mbar_try_wait(bar, parity)) {
+            if (cluster) fence_acquire_cluster();
+            return true;
+        }
+        if ((i & 63u) == 0 && now_ns() - t0 > kWaitNs) {
             flag_error(err, kErrTimeout);
             return false;
         }
@@ -170,16 +184,18 @@ __device__ __forceinline__ bool wwait(uint64_t *bar, uint32_t parity, int *err) 
 __device__ __forceinline__ bool wwait_cluster(uint64_t *bar, uint32_t parity, int *err) {
     return __all_sync(0xffffffffu, try_wait_acq_cluster(bar, parity) || wait_bar(bar, parity, err, true));
 }
-// Named barrier 1 over the 128 softmax threads, returning the OR of `v` over them.
-__device__ __forceinline__ bool group_any(bool v) {
+// Named barrier `id` over the 128 threads of one softmax warpgroup, returning
+// the OR of `v` over them.
+__device__ __forceinline__ bool group_any(bool v, int id) {
     uint32_t r;
-    asm volatile("{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.or.pred q, 1, 128, p;\n\t"
+    asm volatile("{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.or.pred q, %2, 128, p;\n\t"
                  "selp.u32 %0, 1, 0, q;\n\t}"
                  : "=r"(r)
-                 : "r"(uint32_t(v))
+                 : "r"(uint32_t(v)), "r"(id)
                  : "memory");
     return r != 0;
 }
+__device__ __forceinline__ void group_sync(int id) { asm volatile("bar.sync %0, 128;" ::"r"(id) : "memory"); }
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
     asm volatile(
         "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
@@ -255,6 +271,15 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16
         ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
         "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]));
 }
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7])
+                 : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};"
+                 ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]));
+}
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
@@ -284,6 +309,51 @@ __device__ __forceinline__ void i4x8_to_h2x4(uint32_t w, __half2 s2, uint32_t *o
     }
 }
 
+// Byte k of w (two int4 codes, the even channel in the low nibble) -> the fp16
+// pair (code_even * s, code_odd * s), products rounded to nearest.  The nibbles
+// (xor 8) are placed in the mantissas of 1024 and 1024 * 16, which the fused
+// multiply-add maps back to the codes exactly.
+__device__ __forceinline__ uint32_t i4pair_h2(uint32_t w, int k, __half2 s2) {
+    const uint32_t y = __byte_perm(w, 0u, uint32_t(k) | (4u << 4) | (uint32_t(k) << 8) | (4u << 12));
+    const uint32_t z = (y & 0x00F0000Fu) ^ 0x64806408u;            // 1024 + (lo ^ 8), 1024 + 16 (hi ^ 8)
+    const __half2 mul = __halves2half2(__ushort_as_half(0x3C00), __ushort_as_half(0x2C00));   // 1, 1/16
+    const __half2 add = __halves2half2(__ushort_as_half(0xE408), __ushort_as_half(0xD480));   // -1032, -72
+    const __half2 c = __hfma2(*reinterpret_cast<const __half2 *>(&z), mul, add);
+    const __half2 h = __hmul2(c, s2);
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+// Bytes k, k+1 of u = w ^ 0x80808080 (two int8 codes) -> their fp16 pair, exact.
+__device__ __forceinline__ uint32_t i8pair_h2(uint32_t u, int k) {
+    const uint32_t a = __byte_perm(u, 0x64646464u, uint32_t(k) | (4u << 4) | (uint32_t(k + 1) << 8) | (4u << 12));
+    const __half2 h = __hsub2(*reinterpret_cast<const __half2 *>(&a), __half2half2(__ushort_as_half(0x6480)));
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+// Transpose of an 8 x 8 fp16 matrix held one pair per thread (thread t: row
+// t/4, columns 2(t%4), 2(t%4)+1).
+__device__ __forceinline__ uint32_t movm_t(uint32_t a) {
+    uint32_t d;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+    return d;
+}
+// 16 lanes x 16 columns: thread t writes lanes t/4 (+8) at columns 2(t%4)
+// (+1), and the same 8 columns further on for v[4..7].
+__device__ __forceinline__ void tmem_st16x256_x2(uint32_t taddr, const uint32_t (&v)[8]) {
+    asm volatile("tcgen05.st.sync.aligned.16x256b.x2.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};"
+                 ::"r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]));
+}
+// 4-byte asynchronous copy; src_bytes = 0 writes zeros without reading.
+__device__ __forceinline__ void cp_async4(void *dst, const void *src, uint32_t src_bytes) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(smem_addr(dst)), "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+// Arrival on `bar` once this thread's earlier asynchronous copies have landed.
+__device__ __forceinline__ void cp_async_arrive(uint64_t *bar) {
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+// Position of token u (0..15) of an MMA step in the K order of the transposed
+// PV operand: u = 8h + 2m + e sits at 4m + 2h + e.
+__device__ __forceinline__ int kpos16(int u) { return ((u & 6) << 1) | ((u & 8) >> 2) | (u & 1); }
+
 // Byte offset of 16-byte chunk q of row `row` in a 128-byte-swizzled tile
 // (rows of 128 bytes, tile base 1024-aligned).
 __device__ __forceinline__ uint32_t sw128(uint32_t row, uint32_t q) { return row * 128u + ((q ^ (row & 7u)) << 4); }
@@ -305,12 +375,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     using namespace atc;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) uint64_t t1_full[kRing], t1_empty[kRing], t2_full[kRing], t2_empty[kRing];
+    __shared__ __align__(8) uint64_t t1_full[kRing1], t1_empty[kRing1], t2_full[kRing2], t2_empty[kRing2];
     __shared__ __align__(8) uint64_t a_full[kABufs], a_empty[kABufs], s_full[2], s_empty[2];
-    __shared__ __align__(8) uint64_t pva_full[2], pva_empty[2], p_full[2], p_empty[2];
-    __shared__ __align__(8) uint64_t xch_full, xch_empty, mma_done[2];
+    __shared__ __align__(8) uint64_t pva_full[2], pva_empty[2], p_full[2], p_empty[2], sc_full[2], sc_empty[2];
+    __shared__ __align__(8) uint64_t xch_full[2], xch_empty[2], mma_done[2];
     __shared__ uint32_t tmem_base;
-    __shared__ float red_max[4][kMaxN];
+    __shared__ float red_max[2][4][kHalfN];
     __shared__ float m_ref[kMaxN], alpha[kMaxN], q_exp[kMaxN], qfac[kMaxN];
     __shared__ volatile int abort_flag;
 
@@ -324,27 +394,31 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     constexpr uint32_t kLoadBytes = BITS == 8 ? kTile * kChunk : kTile * kChunk / 2;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < kRing; ++i) {
+        for (int i = 0; i < kRing1; ++i) {
             mbar_init(&t1_full[i], 1);
-            mbar_init(&t1_empty[i], 4);
+            mbar_init(&t1_empty[i], 8);
+        }
+        for (int i = 0; i < kRing2; ++i) {
             mbar_init(&t2_full[i], 1);
-            mbar_init(&t2_empty[i], 4);
+            mbar_init(&t2_empty[i], 8);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&s_full[i], 1);
-            mbar_init(&s_empty[i], 4);
-            mbar_init(&pva_full[i], 4);
+            mbar_init(&s_empty[i], 8);
+            mbar_init(&pva_full[i], 8);
             mbar_init(&pva_empty[i], 1);
-            mbar_init(&p_full[i], 4);
+            mbar_init(&p_full[i], 8);
             mbar_init(&p_empty[i], 1);
+            mbar_init(&sc_full[i], 32);     // one cp.async-tracked arrival per lane of warp 3
+            mbar_init(&sc_empty[i], 8);
             mbar_init(&mma_done[i], 1);
+            mbar_init(&xch_full[i], 1);     // one local expect-tx arrival + the peer's st.async bytes
+            mbar_init(&xch_empty[i], 128);  // every thread of the peer's warpgroup, after reading
         }
         for (int i = 0; i < kABufs; ++i) {
             mbar_init(&a_full[i], 4);
             mbar_init(&a_empty[i], 1);
         }
-        mbar_init(&xch_full, 1);     // one local expect-tx arrival + the peer's st.async bytes
-        mbar_init(&xch_empty, 128);  // every softmax thread of the peer, after reading
         mbar_init_fence();
         abort_flag = 0;
     }
@@ -368,6 +442,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
     const size_t row0 = size_t(b) * c.Tmax;          // cache slot of token 0 of the sequence
     const int total = n_tiles * n_chunks;             // chunk loads per pass
+    const int ngrp = r / 128;                         // int4 scale groups per token
 
     // ---- query block: per-head power-of-two scale from the max over all r
     // channels (both CTAs of the pair get the same scale), then the fp16
@@ -389,7 +464,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
         __syncthreads();
         if (warp >= 4) {
             // 8 channels per item; all loads of a thread are issued before its first conversion
-            constexpr int kPer = 8;
+            constexpr int kPer = 4;
             const int items = Np * (rc / 8);
             for (int i0 = threadIdx.x - 128; i0 < items; i0 += kPer * (kThreads - 128)) {
                 float4 va[kPer], vb[kPer];
@@ -424,34 +499,68 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     }
     __syncthreads();
 
-    if (warp == 0 || warp == 3) {
-        // ---------------- TMA producers: warp 0 pass 1, warp 3 pass 2 ----------------
+    if (warp == 0) {
+        // ---------------- TMA producer, pass 1 ----------------
         if (lane == 0 && total > 0) {
-            uint64_t *full = warp == 0 ? t1_full : t2_full;
-            uint64_t *empty = warp == 0 ? t1_empty : t2_empty;
-            uint8_t *ring = sm + (warp == 0 ? kOffT1 : kOffT2);
             int issued = 0;
-            // pass 1 keeps the chunks of the next two tiles streaming into L2
+            // keep the chunks of the next two tiles streaming into L2
             const int ahead = 2 * n_chunks;
             auto prefetch = [&](int j) {
                 tma_prefetch_2d(&map_c, (ch0 + (j % n_chunks) * kChunk) * BITS / 8,
                                 int(row0) + t_begin + (j / n_chunks) * kTile);
             };
-            if (warp == 0)
-                for (int j = 0; j < ahead && j < total; ++j) prefetch(j);
+            for (int j = 0; j < ahead && j < total; ++j) prefetch(j);
             for (int i = 0; i < total && !abort_flag; ++i) {
-                const int s = i % kRing, tile = i / n_chunks, ck = i % n_chunks;
-                if (warp == 0 && i + ahead < total) prefetch(i + ahead);
-                if (i >= kRing && !wait(&empty[s], ((i / kRing) - 1) & 1, p.err)) { abort_flag = 1; break; }
-                mbar_arrive_expect_tx(&full[s], kLoadBytes);
-                tma_load_2d(ring + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
-                            int(row0) + t_begin + tile * kTile, &full[s]);
+                const int s = i % kRing1, tile = i / n_chunks, ck = i % n_chunks;
+                if (i + ahead < total) prefetch(i + ahead);
+                if (i >= kRing1 && !wait(&t1_empty[s], ((i / kRing1) - 1) & 1, p.err)) { abort_flag = 1; break; }
+                mbar_arrive_expect_tx(&t1_full[s], kLoadBytes);
+                tma_load_2d(sm + kOffT1 + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
+                            int(row0) + t_begin + tile * kTile, &t1_full[s]);
                 ++issued;
             }
             // every issued copy has landed before the CTA may finish
-            for (int i = issued - kRing > 0 ? issued - kRing : 0; i < issued; ++i)
-                wait(&full[i % kRing], (i / kRing) & 1, p.err);
+            for (int i = issued - kRing1 > 0 ? issued - kRing1 : 0; i < issued; ++i)
+                wait(&t1_full[i % kRing1], (i / kRing1) & 1, p.err);
         }
+    } else if (warp == 3) {
+        // ---------------- TMA producer, pass 2 (+ int4 group scales) ----------------
+        int issued = 0;
+        for (int i = 0; i < total; ++i) {
+            if (__any_sync(0xffffffffu, abort_flag != 0)) break;
+            const int s = i % kRing2, tile = i / n_chunks, ck = i % n_chunks;
+            if (BITS == 4 && ck == 0) {
+                // the tile's scale rows [token][ngrp] into ring slot tile & 1 (4-byte copies;
+                // tokens past the end get zeros, so dead rows contribute 0, never NaN)
+                const int sl = tile & 1;
+                if (tile >= 2 && !wwait(&sc_empty[sl], ((tile >> 1) - 1) & 1, p.err)) { abort_flag = 1; break; }
+                uint8_t *dst = sm + kOffSc + sl * kScBytes;
+                const int nw = ngrp / 2;
+                for (int w = lane; w < kTile * nw; w += 32) {
+                    const int tt = w / nw, k = w - tt * nw;
+                    const int tok = t_begin + tile * kTile + tt;
+                    const bool live = tok < t_end;
+                    const uint32_t *src = static_cast<const uint32_t *>(c.scales) + (row0 + (live ? tok : t_begin)) * nw + k;
+                    cp_async4(dst + size_t(w) * 4, src, live ? 4u : 0u);
+                }
+                cp_async_arrive(&sc_full[sl]);
+            }
+            bool ok = true;
+            if (lane == 0) {
+                if (i >= kRing2 && !wait(&t2_empty[s], ((i / kRing2) - 1) & 1, p.err)) ok = false;
+                if (ok) {
+                    mbar_arrive_expect_tx(&t2_full[s], kLoadBytes);
+                    tma_load_2d(sm + kOffT2 + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
+                                int(row0) + t_begin + tile * kTile, &t2_full[s]);
+                }
+            }
+            if (!__shfl_sync(0xffffffffu, ok, 0)) { abort_flag = 1; break; }
+            ++issued;
+        }
+        if (lane == 0)
+            for (int i = issued - kRing2 > 0 ? issued - kRing2 : 0; i < issued; ++i)
+                wait(&t2_full[i % kRing2], (i / kRing2) & 1, p.err);
+        asm volatile("cp.async.wait_all;" ::: "memory");
     } else if (warp == 1) {
         // ---------------- scores MMA ----------------
         if (lane == 0 && n_tiles > 0) {
@@ -480,9 +589,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             wait(&mma_done[0], 0, p.err);
         }
     } else if (warp == 2) {
-        // ---------------- PV MMA: O^T += C^T P ----------------
+        // ---------------- PV MMA: O^T += C^T P, A from tensor memory ----------------
         if (lane == 0 && n_tiles > 0) {
-            const uint32_t idesc = idesc_f16(Np, 1);
+            const uint32_t idesc = idesc_f16(Np, 0);
             int chunk = 0;
             for (int tile = 0; tile < n_tiles && !abort_flag; ++tile) {
                 const int pb = tile & 1;
@@ -494,14 +603,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                     const int vb = chunk & 1;
                     if (!wait(&pva_full[vb], (chunk >> 1) & 1, p.err)) { ok = false; break; }
                     fence_after();
-                    const uint32_t abase = smem_addr(sm + kOffPva + vb * kPvaBytes);
 #pragma unroll
                     for (int k = 0; k < kTile / 16; ++k) {
-                        // A: channel-major fp16 tile; 64-channel halves 16 KiB apart, 8-token groups 1 KiB apart
-                        const uint64_t a = sdesc(abase + k * 16 * 128, kTile * 128, 1024);
                         // B: P^T rows = heads; 64-token blocks Np * 128 bytes apart
                         const uint64_t bb = sdesc(pbase + (k >> 2) * (Np * 128) + (k & 3) * 32, 16, 1024);
-                        mma_ss(tmem + kColO + ck * Np, a, bb, idesc, (tile > 0 || k > 0) ? 1u : 0u);
+                        mma_ts(tmem + kColO + ck * Np, tmem + kColV + vb * 64 + k * 8, bb, idesc,
+                               (tile > 0 || k > 0) ? 1u : 0u);
                     }
                     commit(&pva_empty[vb]);
                 }
@@ -511,143 +618,185 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             commit(&mma_done[1]);
             wait(&mma_done[1], 0, p.err);
         }
-    } else if (warp < 8) {
-        // ---------------- warpgroup 1: pass-1 converter, one thread per token ----------------
-        const int quad = warp & 3, t = quad * 32 + lane;
+    } else if (warp < 12) {
+        // ---------------- warpgroups 1-2: pass-1 converter, thread = token ----------------
+        // warp (quad, hh): tokens 32 quad + lane, channels [64 hh, 64 hh + 64) of each chunk
+        const int quad = warp & 3, hh = (warp - 4) >> 2, t = quad * 32 + lane;
         const uint32_t trow = tmem + (uint32_t(quad * 32) << 16);
-        int half = 0;
-        uint16_t sc_next = 0;
-        if (BITS == 4 && total > 0) {
-            const int tok = t_begin + t;
-            sc_next = load_group_scale(c, row0 + tok, ch0 / 128, tok < t_end);
-        }
-        for (int i = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0); ++i) {
-            const int s = i % kRing;
-            const uint16_t sc_cur = sc_next;
-            if (BITS == 4 && i + 1 < total) {      // next chunk's group scale, loaded ahead
-                const int tok = t_begin + ((i + 1) / n_chunks) * kTile + t;
-                sc_next = load_group_scale(c, row0 + tok, (ch0 / 128) + (i + 1) % n_chunks, tok < t_end);
-            }
-            if (!wwait(&t1_full[s], (i / kRing) & 1, p.err)) { abort_flag = 1; break; }
-            const uint8_t *slot = sm + kOffT1 + s * kSlotBytes;
-            bool ok = true;
-            // both 64-channel halves of the chunk: convert, store to tensor memory, one wait
-            const int ab0 = half % kABufs, ab1 = (half + 1) % kABufs;
-            if (half >= kABufs && !wwait(&a_empty[ab0], ((half / kABufs) - 1) & 1, p.err)) ok = false;
-            if (ok && half + 1 >= kABufs && !wwait(&a_empty[ab1], (((half + 1) / kABufs) - 1) & 1, p.err)) ok = false;
-            if (ok) {
+        uint16_t scc[kMaxRc / 128], scn[kMaxRc / 128];     // this token's group scales, current / next tile
+        auto load_sc = [&](int tile, uint16_t (&o)[kMaxRc / 128]) {
+            const int tok = t_begin + tile * kTile + t;
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    uint32_t v[32];
+            for (int k = 0; k < kMaxRc / 128; ++k)
+                o[k] = (k < n_chunks) ? load_group_scale(c, row0 + tok, ch0 / 128 + k, tok < t_end) : uint16_t(0);
+        };
+        if (BITS == 4 && n_tiles > 0) load_sc(0, scn);
+        for (int i = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0); ++i) {
+            const int s = i % kRing1, ck = i % n_chunks, tile = i / n_chunks;
+            if (BITS == 4 && ck == 0) {
+#pragma unroll
+                for (int k = 0; k < kMaxRc / 128; ++k) scc[k] = scn[k];
+                if (tile + 1 < n_tiles) load_sc(tile + 1, scn);      // a tile ahead
+            }
+            if (!wwait(&t1_full[s], (i / kRing1) & 1, p.err)) { abort_flag = 1; break; }
+            const uint8_t *slot = sm + kOffT1 + s * kSlotBytes;
+            const int half = 2 * i + hh, ab = half % kABufs;
+            bool ok = half < kABufs || wwait(&a_empty[ab], ((half / kABufs) - 1) & 1, p.err);
+            if (ok) {
+                uint16_t scv = scc[0];
+#pragma unroll
+                for (int k = 1; k < kMaxRc / 128; ++k)
+                    if (k == ck) scv = scc[k];
+                const __half2 s2 = __half2half2(__ushort_as_half(scv));
+                // the half-chunk's codes (64 channels), every load issued first
+                constexpr int kU = BITS == 8 ? 4 : 2;       // 16-byte units
+                uint4 wl[kU];
+#pragma unroll
+                for (int u = 0; u < kU; ++u)
+                    wl[u] = *reinterpret_cast<const uint4 *>(slot + (BITS == 8 ? sw128(t, hh * 4 + u) : sw64(t, hh * 2 + u)));
+#pragma unroll
+                for (int q = 0; q < 2; ++q) {               // 32 channels per store
+                    uint32_t v[16];
                     if (BITS == 8) {
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) {           // 4 x 16 codes = 64 channels
-                            const uint4 w = *reinterpret_cast<const uint4 *>(slot + sw128(t, hh * 4 + q));
-                            i8x4_to_h2x2(w.x, v[q * 8 + 0], v[q * 8 + 1]);
-                            i8x4_to_h2x2(w.y, v[q * 8 + 2], v[q * 8 + 3]);
-                            i8x4_to_h2x2(w.z, v[q * 8 + 4], v[q * 8 + 5]);
-                            i8x4_to_h2x2(w.w, v[q * 8 + 6], v[q * 8 + 7]);
+                        for (int u = 0; u < 2; ++u) {       // 2 x 16 codes
+                            const uint4 w = wl[q * 2 + u];
+                            i8x4_to_h2x2(w.x, v[u * 8 + 0], v[u * 8 + 1]);
+                            i8x4_to_h2x2(w.y, v[u * 8 + 2], v[u * 8 + 3]);
+                            i8x4_to_h2x2(w.z, v[u * 8 + 4], v[u * 8 + 5]);
+                            i8x4_to_h2x2(w.w, v[u * 8 + 6], v[u * 8 + 7]);
                         }
                     } else {
-                        const __half2 s2 = __half2half2(__ushort_as_half(sc_cur));
+                        const uint32_t ww[4] = {wl[q].x, wl[q].y, wl[q].z, wl[q].w};   // 32 codes
 #pragma unroll
-                        for (int q = 0; q < 2; ++q) {           // 2 x 32 codes = 64 channels
-                            const uint4 w = *reinterpret_cast<const uint4 *>(slot + sw64(t, hh * 2 + q));
-                            i4x8_to_h2x4(w.x, s2, &v[q * 16 + 0]);
-                            i4x8_to_h2x4(w.y, s2, &v[q * 16 + 4]);
-                            i4x8_to_h2x4(w.z, s2, &v[q * 16 + 8]);
-                            i4x8_to_h2x4(w.w, s2, &v[q * 16 + 12]);
-                        }
+                        for (int j = 0; j < 4; ++j)
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) v[j * 4 + k] = i4pair_h2(ww[j], k, s2);
                     }
-                    tmem_st32(trow + kColA + (hh ? ab1 : ab0) * 32, v);
+                    tmem_st16(trow + kColA + ab * 32 + q * 16, v);
                 }
                 tmem_wait_st();
                 fence_before();
                 __syncwarp();
-                if (lane == 0) {
-                    arrive_local(&a_full[ab0]);
-                    arrive_local(&a_full[ab1]);
-                }
+                if (lane == 0) arrive_local(&a_full[ab]);
             }
-            half += 2;
             __syncwarp();
             if (lane == 0) arrive_local(&t1_empty[s]);
             if (!ok) { abort_flag = 1; break; }
         }
-    } else if (warp < 12) {
-        // ---------------- warpgroup 2: pass-2 converter (fp16 tile in shared memory) ----------------
-        // thread: 16-channel group g of the chunk, tokens tb + 16 k (k = 0..7)
-        const int tid = threadIdx.x - 256, g = tid & 7, tb = tid >> 3;
-        uint16_t scn[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-        auto load_scales = [&](int i) {
-            const int tile = i / n_chunks, grp = ch0 / 128 + i % n_chunks;
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const int tok = t_begin + tile * kTile + tb + 16 * k;
-                scn[k] = load_group_scale(c, row0 + tok, grp, tok < t_end);
-            }
-        };
-        if (BITS == 4 && total > 0) load_scales(0);
+    } else if (warp < 20) {
+        // ---------------- warpgroups 3-4: pass-2 converter, channel-major into tensor memory ----------------
+        // warp (q, th): channels [32 q, 32 q + 32) of each chunk (its tensor-memory lanes),
+        // tokens [64 th, 64 th + 64).  Thread t supplies, per 8 x 8 block (tokens x channels),
+        // the pair of channels 2(t%4), 2(t%4)+1 of token t/4; movmatrix turns it into the pair
+        // of tokens 2(t%4), 2(t%4)+1 of channel t/4, one 32-bit tensor-memory word.
+        const int q = warp & 3, th = (warp - 12) >> 2, cq = lane & 3, g8 = lane >> 2;
+        // The tokens this thread supplies are 64 th + 32 h32 + 8 j + g8: their row
+        // swizzle depends on g8 only, so every shared-memory address below is a
+        // per-thread base plus a compile-time offset.
+        const uint32_t rbase = uint32_t(64 * th + g8);
+        const uint32_t off4 = rbase * 64u + ((uint32_t(q) ^ ((uint32_t(g8) >> 1) & 3u)) << 4);        // int4 rows
+        const uint32_t off8a = rbase * 128u + ((uint32_t(2 * q) ^ uint32_t(g8)) << 4);                 // int8 rows,
+        const uint32_t off8b = rbase * 128u + ((uint32_t(2 * q + 1) ^ uint32_t(g8)) << 4);             // two units
+        const int k8 = (cq & 1) * 2;
         for (int i = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0); ++i) {
-            const int s = i % kRing, vb = i & 1;
-            uint16_t scl[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) scl[k] = scn[k];
-            if (BITS == 4 && i + 1 < total) load_scales(i + 1);
-            if (!wwait(&t2_full[s], (i / kRing) & 1, p.err)) { abort_flag = 1; break; }
+            const int s = i % kRing2, vb = i & 1, tile = i / n_chunks, ck = i % n_chunks;
+            if (!wwait(&t2_full[s], (i / kRing2) & 1, p.err)) { abort_flag = 1; break; }
             if (i >= 2 && !wwait(&pva_empty[vb], ((i >> 1) - 1) & 1, p.err)) { abort_flag = 1; break; }
+            if (BITS == 4 && ck == 0 && !wwait(&sc_full[tile & 1], (tile >> 1) & 1, p.err)) { abort_flag = 1; break; }
             const uint8_t *src = sm + kOffT2 + s * kSlotBytes;
-            uint8_t *dst = sm + kOffPva + vb * kPvaBytes + (g >> 2) * (kTile * 128);
-            const int q0 = (g & 3) * 2;
+            // this thread's group scales: token rbase + 8 j' (j' = 4 h32 + j), group grp
+            const __half *scs = reinterpret_cast<const __half *>(sm + kOffSc + (tile & 1) * kScBytes) +
+                                rbase * ngrp + (ch0 / 128 + ck);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const int t = tb + 16 * k;
-                uint32_t o[8];
-                if (BITS == 8) {
-                    const uint4 w = *reinterpret_cast<const uint4 *>(src + sw128(t, g));
-                    i8x4_to_h2x2(w.x, o[0], o[1]);
-                    i8x4_to_h2x2(w.y, o[2], o[3]);
-                    i8x4_to_h2x2(w.z, o[4], o[5]);
-                    i8x4_to_h2x2(w.w, o[6], o[7]);
-                } else {
-                    const __half2 s2 = __half2half2(__ushort_as_half(scl[k]));
-                    const uint2 w = *reinterpret_cast<const uint2 *>(src + sw64(t, g >> 1) + (g & 1) * 8);
-                    i4x8_to_h2x4(w.x, s2, &o[0]);
-                    i4x8_to_h2x4(w.y, s2, &o[4]);
+            for (int h32 = 0; h32 < 2; ++h32) {             // 32 tokens: two 16x256b stores of 16 columns
+                // rows of the 4 tokens this thread supplies (16-token step g, 8-token block tb), loads first
+                constexpr int kU = BITS == 8 ? 2 : 1;       // 16-byte units of the warp's 32 channels
+                uint4 wl[4][kU];
+                __half2 s2[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {               // j = 2 g + tb
+                    const uint32_t dr = uint32_t(32 * h32 + 8 * j);         // token offset from rbase
+                    if (BITS == 8) {
+                        wl[j][0] = *reinterpret_cast<const uint4 *>(src + off8a + dr * 128u);
+                        wl[j][kU - 1] = *reinterpret_cast<const uint4 *>(src + off8b + dr * 128u);
+                    } else {
+                        wl[j][0] = *reinterpret_cast<const uint4 *>(src + off4 + dr * 64u);
+                        s2[j] = __half2half2(scs[dr * ngrp]);
+                    }
                 }
-                // [64-channel half][token][64 channels], 128-byte rows, swizzled
-                *reinterpret_cast<uint4 *>(dst + sw128(t, q0)) = make_uint4(o[0], o[1], o[2], o[3]);
-                *reinterpret_cast<uint4 *>(dst + sw128(t, q0 + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
+                uint32_t o0[8], o1[8];                       // channel blocks 0-1 and 2-3 of the warp
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int g = j >> 1, tb = j & 1;
+                    uint32_t x[4];
+                    if (BITS == 8) {
+                        // channel block cb = bytes 8cb..8cb+7; pair 2cq, 2cq+1 sits in word 2cb + (cq >> 1)
+                        const uint32_t wv[8] = {wl[j][0].x, wl[j][0].y, wl[j][0].z, wl[j][0].w,
+                                                wl[j][kU - 1].x, wl[j][kU - 1].y, wl[j][kU - 1].z, wl[j][kU - 1].w};
+#pragma unroll
+                        for (int cb = 0; cb < 4; ++cb) {
+                            const uint32_t wsel = (cq >> 1) ? wv[2 * cb + 1] : wv[2 * cb];
+                            x[cb] = i8pair_h2(wsel ^ 0x80808080u, k8);
+                        }
+                    } else {
+                        // pair 2cq, 2cq+1 of channel block cb is byte cq of word cb
+                        x[0] = i4pair_h2(wl[j][0].x, cq, s2[j]);
+                        x[1] = i4pair_h2(wl[j][0].y, cq, s2[j]);
+                        x[2] = i4pair_h2(wl[j][0].z, cq, s2[j]);
+                        x[3] = i4pair_h2(wl[j][0].w, cq, s2[j]);
+                    }
+                    // 16x256b registers of step g: (blk 2lh, tb 0), (2lh, tb 1), (2lh+1, tb 0), (2lh+1, tb 1)
+                    o0[4 * g + tb] = movm_t(x[0]);
+                    o0[4 * g + 2 + tb] = movm_t(x[1]);
+                    o1[4 * g + tb] = movm_t(x[2]);
+                    o1[4 * g + 2 + tb] = movm_t(x[3]);
+                }
+                const uint32_t col = kColV + vb * 64 + 32 * th + 16 * h32;
+                tmem_st16x256_x2(tmem + (uint32_t(32 * q) << 16) + col, o0);
+                tmem_st16x256_x2(tmem + (uint32_t(32 * q + 16) << 16) + col, o1);
             }
-            fence_async_smem();
+            tmem_wait_st();
+            fence_before();
             __syncwarp();
             if (lane == 0) {
                 arrive_local(&pva_full[vb]);
                 arrive_local(&t2_empty[s]);
+                if (BITS == 4 && ck == n_chunks - 1) arrive_local(&sc_empty[tile & 1]);
             }
         }
     } else {
-        // ---------------- warpgroup 3: exchange, online softmax, P ----------------
-        // Logits are kept in log2 units.  Each thread (one token) accumulates
-        // its own sums of p per head over the tiles; the sums over tokens are
-        // formed once, at the end.  The reference maximum m_ref of a head only
-        // moves when a logit exceeds it by more than kRescale2 (one vote per
-        // tile); then the tile maximum is reduced through shared memory, and
-        // o_lat and the sums are rescaled.  A failed wait marks the warp
-        // `bad`; the group leaves the tile loop together at its next named
-        // barrier (bar.red.or), so no warp is left at a barrier the others skip.
-        const int quad = warp & 3, t = quad * 32 + lane, wq = warp - 12;
+        // ---------------- warpgroups 5-6: exchange, online softmax, P ----------------
+        // Warpgroup hg takes heads [16 hg, 16 hg + 16); thread = token.  Logits
+        // are kept in log2 units.  Each thread accumulates its own sums of p per
+        // head over the tiles; the sums over tokens are formed once, at the end.
+        // The reference maximum m_ref of a head only moves when a logit exceeds
+        // it by more than kRescale2 (one vote per tile); then the tile maximum is
+        // reduced through shared memory, and o_lat and the sums are rescaled.  A
+        // failed wait marks the warp `bad`; the warpgroup leaves the tile loop
+        // together at its next named barrier (bar.red.or), so no warp is left at
+        // a barrier the others skip.
+        const int quad = warp & 3, hg = (warp - 20) >> 2, t = quad * 32 + lane, wq = quad;
+        const int hb = hg * kHalfN, bar_id = 1 + hg;
+        const bool grp_live = hb < Np;                      // Np = 16: the second warpgroup has no heads
         const uint32_t trow = tmem + (uint32_t(quad * 32) << 16);
         const uint32_t xch_remote = map_peer(smem_addr(sm + kOffXch), peer);
-        const uint32_t xfull_remote = map_peer(smem_addr(&xch_full), peer);
-        const uint32_t xempty_remote = map_peer(smem_addr(&xch_empty), peer);
-        float *xr = reinterpret_cast<float *>(sm + kOffXch);   // peer partials, then transposed reductions
+        const uint32_t xfull_remote = map_peer(smem_addr(&xch_full[hg]), peer);
+        const uint32_t xempty_remote = map_peer(smem_addr(&xch_empty[hg]), peer);
+        // exchange buffer: the peer's partials as [head / 4][token][4] (conflict-free float4
+        // rows); warpgroup hg's half (heads 16 hg ..) is reused as [token][16] for its
+        // tile-maximum transposition once its partials are consumed
+        float *xr = reinterpret_cast<float *>(sm + kOffXch);
         const float *tscale = static_cast<const float *>(c.scales);
         float tsc_next = 0.0f;
         if (BITS == 8 && n_tiles > 0) tsc_next = t_begin + t < t_end ? tscale[row0 + t_begin + t] : 0.0f;
-        float lt[kMaxN];
+        // P^T position of this token: 64-token block, then the K order of the PV operand
+        const int pcol = (t & 48) | kpos16(t & 15);
+
+        // running sums of p per (head, token), kept in shared memory: [head][token]
+        float *lt = reinterpret_cast<float *>(sm + kOffLt) + hb * kTile + t;
 #pragma unroll
-        for (int h = 0; h < kMaxN; ++h) lt[h] = 0.0f;
+        for (int h = 0; h < kHalfN; ++h) lt[h * kTile] = 0.0f;
         bool failed = false;
         for (int tile = 0; tile < n_tiles; ++tile) {
             const int sb = tile & 1;
@@ -658,114 +807,126 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 tsc_next = tok + kTile < t_end ? tscale[row0 + tok + kTile] : 0.0f;
             bool bad = __any_sync(0xffffffffu, abort_flag != 0);
             if (!bad) bad = !wwait(&s_full[sb], (tile >> 1) & 1, p.err);
-            float s[kMaxN];
+            float s[kHalfN];
             if (!bad) {
                 fence_after();
-                uint32_t v[32];
-                tmem_ld32(trow + kColS + sb * 32, v);
+                uint32_t v[16];
+                tmem_ld16(trow + kColS + sb * 32 + hb, v);
                 tmem_wait_ld();
 #pragma unroll
-                for (int h = 0; h < kMaxN; ++h) s[h] = __uint_as_float(v[h]);
+                for (int h = 0; h < kHalfN; ++h) s[h] = __uint_as_float(v[h]);
                 fence_before();
                 __syncwarp();
                 if (lane == 0) arrive_local(&s_empty[sb]);
             } else {
 #pragma unroll
-                for (int h = 0; h < kMaxN; ++h) s[h] = 0.0f;
+                for (int h = 0; h < kHalfN; ++h) s[h] = 0.0f;
             }
             // swap partial scores with the peer: asynchronous stores that
-            // count their bytes on the peer's xch_full, whose phase also needs
-            // the peer's own expect-tx arrival
-            if (t == 0 && !bad) mbar_arrive_expect_tx(&xch_full, kTile * kMaxN * 4);
-            if (!bad && tile > 0) bad = !wwait_cluster(&xch_empty, (tile - 1) & 1, p.err);
+            // count their bytes on the peer's xch_full[hg], whose phase also
+            // needs the peer's own expect-tx arrival
+            if (t == 0 && !bad) mbar_arrive_expect_tx(&xch_full[hg], kTile * kHalfN * 4);
+            if (!bad && tile > 0) bad = !wwait_cluster(&xch_empty[hg], (tile - 1) & 1, p.err);
             if (!bad) {
 #pragma unroll
-                for (int h = 0; h < kMaxN; h += 4)
-                    st_async_v4(xch_remote + (t * kMaxN + h) * 4, s[h], s[h + 1], s[h + 2], s[h + 3], xfull_remote);
-                bad = !wwait_cluster(&xch_full, tile & 1, p.err);
+                for (int h = 0; h < kHalfN; h += 4)
+                    st_async_v4(xch_remote + (((hb + h) >> 2) * kTile + t) * 16, s[h], s[h + 1], s[h + 2], s[h + 3], xfull_remote);
+                bad = !wwait_cluster(&xch_full[hg], tile & 1, p.err);
             }
             bool exceed = false;
             if (!bad) {
 #pragma unroll
-                for (int h = 0; h < kMaxN; h += 4) {
-                    const float4 o = *reinterpret_cast<const float4 *>(xr + t * kMaxN + h);
+                for (int h = 0; h < kHalfN; h += 4) {
+                    const float4 o = *reinterpret_cast<const float4 *>(xr + (((hb + h) >> 2) * kTile + t) * 4);
                     // rank 0 computes own + peer, rank 1 peer + own: the same sums on both CTAs
                     if (rank == 0) { s[h] += o.x; s[h + 1] += o.y; s[h + 2] += o.z; s[h + 3] += o.w; }
                     else { s[h] = o.x + s[h]; s[h + 1] = o.y + s[h + 1]; s[h + 2] = o.z + s[h + 2]; s[h + 3] = o.w + s[h + 3]; }
                 }
                 // logits in log2 units; dead tokens and padding heads get -inf
 #pragma unroll
-                for (int h = 0; h < kMaxN; ++h) {
-                    const float lg = s[h] * qfac[h] * (BITS == 8 ? tsc : 1.0f);
-                    s[h] = (live && h < H) ? lg : -INFINITY;
-                    exceed |= s[h] > m_ref[h] + kRescale2;
+                for (int h = 0; h < kHalfN; ++h) {
+                    const float lg = s[h] * qfac[hb + h] * (BITS == 8 ? tsc : 1.0f);
+                    s[h] = (live && hb + h < H) ? lg : -INFINITY;
+                    exceed |= s[h] > m_ref[hb + h] + kRescale2;
                 }
             }
-            if (group_any(bad)) { failed = true; break; }
-            if (group_any(exceed)) {
+            if (group_any(bad, bar_id)) { failed = true; break; }
+            if (group_any(exceed, bar_id)) {
                 // tile maximum per head: the logits, transposed through the exchange buffer
 #pragma unroll
-                for (int h = 0; h < kMaxN; ++h) xr[t * kMaxN + (h ^ lane)] = s[h];
-                asm volatile("bar.sync 1, 128;" ::: "memory");
+                for (int h = 0; h < kHalfN; ++h) xr[hg * (kTile * kHalfN) + t * kHalfN + (h ^ (lane & 15))] = s[h];
+                group_sync(bar_id);
                 {
+                    // lane: head lane & 15 over tokens (lane >> 4) + 2j of the warp's 32
+                    const int hl = lane & 15;
                     float m = -INFINITY;
-#pragma unroll 8
-                    for (int k = 0; k < 32; ++k) m = fmaxf(m, xr[(wq * 32 + k) * kMaxN + (lane ^ k)]);
-                    red_max[wq][lane] = m;
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const int k = (lane >> 4) + 2 * j;
+                        m = fmaxf(m, xr[hg * (kTile * kHalfN) + (wq * 32 + k) * kHalfN + (hl ^ (k & 15))]);
+                    }
+                    m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 16));
+                    if (lane < 16) red_max[hg][wq][lane] = m;
                 }
-                asm volatile("bar.sync 1, 128;" ::: "memory");
-                if (t < kMaxN) {
+                group_sync(bar_id);
+                if (t < kHalfN) {
+                    const int h = hb + t;
                     float a = 1.0f;
-                    if (t < H) {
-                        const float tm = fmaxf(fmaxf(red_max[0][t], red_max[1][t]), fmaxf(red_max[2][t], red_max[3][t]));
-                        const float mr = m_ref[t];
+                    if (h < H) {
+                        const float tm = fmaxf(fmaxf(red_max[hg][0][t], red_max[hg][1][t]),
+                                               fmaxf(red_max[hg][2][t], red_max[hg][3][t]));
+                        const float mr = m_ref[h];
                         if (tm > mr + kRescale2) {
                             a = mr == -INFINITY ? 0.0f : exp2f(mr - tm);
-                            m_ref[t] = tm;
+                            m_ref[h] = tm;
                         }
                     }
-                    alpha[t] = a;
+                    alpha[h] = a;
                 }
-                asm volatile("bar.sync 1, 128;" ::: "memory");
+                group_sync(bar_id);
 #pragma unroll
-                for (int h = 0; h < kMaxN; ++h) lt[h] *= alpha[h];
-                if (tile > 0) {
+                for (int h = 0; h < kHalfN; ++h) lt[h * kTile] *= alpha[hb + h];
+                if (tile > 0 && grp_live) {
                     // the PV MMAs of the previous tile must be complete before o_lat is scaled
                     bad = !wwait(&p_empty[(tile - 1) & 1], ((tile - 1) >> 1) & 1, p.err);
                     if (!bad) {
                         fence_after();
-                        for (int ck = 0; ck < n_chunks; ++ck) {
-                            for (int h0 = 0; h0 < Np; h0 += 16) {
-                                uint32_t v[16];
-                                tmem_ld16(trow + kColO + ck * Np + h0, v);
-                                tmem_wait_ld();
+                        for (int c8 = 0; c8 < 2 * n_chunks; ++c8) {     // 8 heads at a time
+                            const uint32_t col = trow + kColO + (c8 >> 1) * Np + hb + (c8 & 1) * 8;
+                            uint32_t v[8];
+                            tmem_ld8(col, v);
+                            tmem_wait_ld();
 #pragma unroll
-                                for (int e = 0; e < 16; ++e)
-                                    v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha[h0 + e]);
-                                tmem_st16(trow + kColO + ck * Np + h0, v);
-                            }
+                            for (int e = 0; e < 8; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha[hb + (c8 & 1) * 8 + e]);
+                            tmem_st8(col, v);
                         }
                         tmem_wait_st();
                         fence_before();
                     }
                 }
             }
-            arrive_peer(xempty_remote);     // this thread is done with the exchange buffer (release)
+            arrive_peer_relaxed(xempty_remote);   // this thread's reads of the exchange buffer have completed
             if (!bad && tile >= 2) bad = !wwait(&p_empty[sb], ((tile >> 1) - 1) & 1, p.err);
             // P^T [heads][tokens], 64-token blocks of Np rows x 128 bytes, swizzled
             uint8_t *pbuf = sm + kOffP + sb * kPBytes + (t >> 6) * (Np * 128);
-            const int col = t & 63;
+            // three passes (loads, then read-modify-writes, then stores only) so that
+            // no shared-memory load waits behind a store it might alias
 #pragma unroll
-            for (int h = 0; h < kMaxN; ++h) {
-                const float pe = h < H ? exp2f(s[h] - m_ref[h]) : 0.0f;
-                lt[h] += pe;
-                if (!bad && h < Np) {
-                    const __half hv = __float2half_rn(BITS == 8 ? pe * tsc : pe);
-                    *reinterpret_cast<__half *>(pbuf + h * 128 + ((((col >> 3) ^ (h & 7))) << 4) + (col & 7) * 2) = hv;
+            for (int h = 0; h < kHalfN; ++h) s[h] = hb + h < H ? exp2f(s[h] - m_ref[hb + h]) : 0.0f;
+#pragma unroll
+            for (int h = 0; h < kHalfN; ++h) lt[h * kTile] += s[h];
+            if (!bad) {
+#pragma unroll
+                for (int h = 0; h < kHalfN; ++h) {
+                    const int hh = hb + h;
+                    if (hh < Np) {
+                        const __half hv = __float2half_rn(BITS == 8 ? s[h] * tsc : s[h]);
+                        *reinterpret_cast<__half *>(pbuf + hh * 128 + ((((pcol >> 3) ^ (hh & 7))) << 4) + (pcol & 7) * 2) = hv;
+                    }
                 }
             }
             fence_async_smem();
-            if (group_any(bad)) { failed = true; break; }
+            if (group_any(bad, bar_id)) { failed = true; break; }
             __syncwarp();
             if (lane == 0) arrive_local(&p_full[sb]);
         }
@@ -775,33 +936,34 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             const int lt_last = n_tiles - 1;
             const bool ok = wwait(&p_empty[lt_last & 1], (lt_last >> 1) & 1, p.err);
             // sums over the tokens, transposed through the exchange buffer (the peer sends no more)
-#pragma unroll
-            for (int h = 0; h < kMaxN; ++h) xr[t * kMaxN + (h ^ lane)] = lt[h];
-            asm volatile("bar.sync 1, 128;" ::: "memory");
+            group_sync(bar_id);
             {
+                // lane: head lane & 15 over tokens (lane >> 4) + 2j of the warp's 32
+                const float *lrow = reinterpret_cast<const float *>(sm + kOffLt) + (hb + (lane & 15)) * kTile + wq * 32;
                 float sum = 0.0f;
-#pragma unroll 8
-                for (int k = 0; k < 32; ++k) sum += xr[(wq * 32 + k) * kMaxN + (lane ^ k)];
-                red_max[wq][lane] = sum;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) sum += lrow[(lane >> 4) + 2 * j];
+                sum += __shfl_xor_sync(0xffffffffu, sum, 16);
+                if (lane < 16) red_max[hg][wq][lane] = sum;
             }
-            asm volatile("bar.sync 1, 128;" ::: "memory");
-            if (!group_any(!ok)) {
-                fence_after();
-                const size_t pb = (size_t(b) * p.n_split + split) * H;
-                for (int ck = 0; ck < n_chunks; ++ck) {
-                    const int ch = ch0 + ck * kChunk + t;
-                    for (int h0 = 0; h0 < Np; h0 += 16) {
+            group_sync(bar_id);
+            if (!group_any(!ok, bar_id)) {
+                if (grp_live) {
+                    fence_after();
+                    const size_t pb = (size_t(b) * p.n_split + split) * H;
+                    for (int ck = 0; ck < n_chunks; ++ck) {
+                        const int ch = ch0 + ck * kChunk + t;
                         uint32_t v[16];
-                        tmem_ld16(trow + kColO + ck * Np + h0, v);
+                        tmem_ld16(trow + kColO + ck * Np + hb, v);
                         tmem_wait_ld();
 #pragma unroll
                         for (int e = 0; e < 16; ++e)
-                            if (h0 + e < H) p.po[(pb + h0 + e) * r + ch] = __uint_as_float(v[e]);
+                            if (hb + e < H) p.po[(pb + hb + e) * r + ch] = __uint_as_float(v[e]);
                     }
-                }
-                if (rank == 0 && t < H) {
-                    p.pm[pb + t] = m_ref[t] * 0.6931471805599453f;       // natural-log units
-                    p.pl[pb + t] = (red_max[0][t] + red_max[1][t]) + (red_max[2][t] + red_max[3][t]);
+                    if (rank == 0 && t < kHalfN && hb + t < H) {
+                        p.pm[pb + hb + t] = m_ref[hb + t] * 0.6931471805599453f;       // natural-log units
+                        p.pl[pb + hb + t] = (red_max[hg][0][t] + red_max[hg][1][t]) + (red_max[hg][2][t] + red_max[hg][3][t]);
+                    }
                 }
             } else {
                 abort_flag = 1;
@@ -862,11 +1024,21 @@ int attn_tc_splits(int B, int max_seq_len, int *tiles_per_split) {
     if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int tiles = (max_seq_len + atc::kTile - 1) / atc::kTile;
     const int64_t pairs = sms / 2;                   // CTA pairs resident at once
-    int per = int((int64_t(B) * tiles + 2 * pairs - 1) / (2 * pairs));   // about two waves
-    if (per < 1) per = 1;
-    while ((tiles + per - 1) / per > 64) ++per;      // at most 64 partials per sequence
-    *tiles_per_split = per;
-    return (tiles + per - 1) / per;
+    // tiles per split: the fewest tile steps of the busiest pair, counting about
+    // one tile step of pipeline fill per wave; at most 64 partials per sequence
+    int best = tiles, best_cost = INT32_MAX;
+    for (int per = 1; per <= tiles; ++per) {
+        const int splits = (tiles + per - 1) / per;
+        if (splits > 64) continue;
+        const int64_t waves = (int64_t(B) * splits + pairs - 1) / pairs;
+        const int64_t cost = waves * (per + 1);
+        if (cost < best_cost) {
+            best_cost = int(cost);
+            best = per;
+        }
+    }
+    *tiles_per_split = best;
+    return (tiles + best - 1) / best;
 }
 
 cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const float *qt, const unsigned *qmax, int H,

@@ -100,14 +100,16 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
         mbar_init_fence();
     }
     __syncthreads();
-    pdl_wait();
     // the U_q tile: 16-byte asynchronous copies by every thread (many small
-    // rows: cheaper than bulk or tensor copies of 512-byte rows)
+    // rows: cheaper than bulk or tensor copies of 512-byte rows).  The weights
+    // are no kernel's output, so the copies start before the wait on the
+    // producer grid and overlap its tail.
     for (int i = tid; i < rs * (ncol / 8); i += blockDim.x) {
         const int row = i / (ncol / 8), k = i - row * (ncol / 8);
         cp_async16(u_s + size_t(row) * ncol + 8 * k, Uq + size_t(j0 + row) * d + c0 + 8 * k);
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
+    pdl_wait();
     if (rank == 0 && blockIdx.y == 0)
         for (int i = tid; i < n_qmax; i += blockDim.x) qmax[i] = 0u;
     bool ready = false;
@@ -258,13 +260,13 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
         mbar_init_fence();
     }
     __syncthreads();
-    pdl_wait();
-    if (warp == 0) {
+    if (warp == 0) {            // U_k rows: no kernel's output, copied before the wait on the producer grid
         if (lane == 0) mbar_arrive_expect_tx(&bar, uint32_t(rows) * w * 2);
         __syncwarp();
         for (int i = lane; i < rows; i += 32)
             bulk_g2s(u_s + size_t(i) * ustride, Uk + size_t(j0 + i) * d + size_t(h0) * dh, uint32_t(w) * 2, &bar);
     }
+    pdl_wait();
     bool ready = false;
     const int h = h0 + warp;
     for (int b0 = 0; b0 < B; b0 += NB) {
@@ -356,12 +358,12 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__r
         mbar_init_fence();
     }
     __syncthreads();
-    pdl_wait();
     for (int i = tid; i < rs * (dh / 8); i += blockDim.x) {     // the U_v tile, 16-byte asynchronous copies
-        const int row = i / (dh / 8), k = i - row * (dh / 8);
+        const int row = i / (dh / 8), k = i - row * (dh / 8);   // (before the wait: no kernel writes U_v)
         cp_async16(u_s + size_t(row) * dh + 8 * k, Uv + size_t(j0 + row) * d + size_t(h) * dh + 8 * k);
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
+    pdl_wait();
     bool ready = false;
     const int nq = rs / 4;                           // row quads (r % 32 == 0)
     const int sub = tid / dh, col = tid - sub * dh;

@@ -74,11 +74,11 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
         mbar_init_fence();
     }
     __syncthreads();
-    pdl_wait();
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 0) {     // W_d codes: no kernel's output, copied before the wait on the producer grid
         mbar_arrive_expect_tx(&bar, uint32_t(rows) * d);
         bulk_g2s(w_s, w + size_t(j0) * d, uint32_t(rows) * d, &bar);
     }
+    pdl_wait();
     // a1: per-token int8 quantization.  Few tokens: the whole CTA works on one
     // token at a time; more tokens: one warp per token (see below).
     if (T < kPsWarpTok) {

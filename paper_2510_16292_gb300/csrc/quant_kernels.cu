@@ -99,6 +99,11 @@ weight_quant_kernel(const float *__restrict__ W, int d, int r, float clip, int8_
         codes[size_t(j) * d + k] = int8_t(c);
         if (codes_bf16) codes_bf16[size_t(j) * d + k] = int_to_bf16_bits(c);
     }
+    // The projection kernels copy W_d's codes before they wait on their
+    // producer grid: a dependent launch may begin only once the codes are
+    // visible device-wide.
+    __threadfence();
+    pdl_trigger();
 }
 
 cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int8_t *codes,
