@@ -505,19 +505,22 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             int issued = 0;
             // keep the chunks of the next two tiles streaming into L2
             const int ahead = 2 * n_chunks;
-            auto prefetch = [&](int j) {
-                tma_prefetch_2d(&map_c, (ch0 + (j % n_chunks) * kChunk) * BITS / 8,
-                                int(row0) + t_begin + (j / n_chunks) * kTile);
+            int pj = 0, pck = 0, ptile = 0;                 // next chunk to prefetch
+            auto prefetch = [&]() {
+                tma_prefetch_2d(&map_c, (ch0 + pck * kChunk) * BITS / 8, int(row0) + t_begin + ptile * kTile);
+                ++pj;
+                if (++pck == n_chunks) { pck = 0; ++ptile; }
             };
-            for (int j = 0; j < ahead && j < total; ++j) prefetch(j);
-            for (int i = 0; i < total && !abort_flag; ++i) {
-                const int s = i % kRing1, tile = i / n_chunks, ck = i % n_chunks;
-                if (i + ahead < total) prefetch(i + ahead);
+            while (pj < ahead && pj < total) prefetch();
+            for (int i = 0, tile = 0, ck = 0; i < total && !abort_flag; ++i) {
+                const int s = i % kRing1;
+                if (pj < total) prefetch();
                 if (i >= kRing1 && !wait(&t1_empty[s], ((i / kRing1) - 1) & 1, p.err)) { abort_flag = 1; break; }
                 mbar_arrive_expect_tx(&t1_full[s], kLoadBytes);
                 tma_load_2d(sm + kOffT1 + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
                             int(row0) + t_begin + tile * kTile, &t1_full[s]);
                 ++issued;
+                if (++ck == n_chunks) { ck = 0; ++tile; }
             }
             // every issued copy has landed before the CTA may finish
             for (int i = issued - kRing1 > 0 ? issued - kRing1 : 0; i < issued; ++i)
@@ -526,9 +529,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     } else if (warp == 3) {
         // ---------------- TMA producer, pass 2 (+ int4 group scales) ----------------
         int issued = 0;
-        for (int i = 0; i < total; ++i) {
+        for (int i = 0, tile = 0, ck = 0; i < total; ++i, ck = (ck + 1 == n_chunks) ? 0 : ck + 1, tile += (ck == 0)) {
             if (__any_sync(0xffffffffu, abort_flag != 0)) break;
-            const int s = i % kRing2, tile = i / n_chunks, ck = i % n_chunks;
+            const int s = i % kRing2;
             if (BITS == 4 && ck == 0) {
                 // the tile's scale rows [token][ngrp] into ring slot tile & 1 (4-byte copies;
                 // tokens past the end get zeros, so dead rows contribute 0, never NaN)
@@ -536,12 +539,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 if (tile >= 2 && !wwait(&sc_empty[sl], ((tile >> 1) - 1) & 1, p.err)) { abort_flag = 1; break; }
                 uint8_t *dst = sm + kOffSc + sl * kScBytes;
                 const int nw = ngrp / 2;
-                for (int w = lane; w < kTile * nw; w += 32) {
-                    const int tt = w / nw, k = w - tt * nw;
+                for (int tt = lane; tt < kTile; tt += 32) {
                     const int tok = t_begin + tile * kTile + tt;
                     const bool live = tok < t_end;
-                    const uint32_t *src = static_cast<const uint32_t *>(c.scales) + (row0 + (live ? tok : t_begin)) * nw + k;
-                    cp_async4(dst + size_t(w) * 4, src, live ? 4u : 0u);
+                    const uint32_t *src = static_cast<const uint32_t *>(c.scales) + (row0 + (live ? tok : t_begin)) * nw;
+                    for (int k = 0; k < nw; ++k) cp_async4(dst + size_t(tt * nw + k) * 4, src + k, live ? 4u : 0u);
                 }
                 cp_async_arrive(&sc_full[sl]);
             }
@@ -631,8 +633,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 o[k] = (k < n_chunks) ? load_group_scale(c, row0 + tok, ch0 / 128 + k, tok < t_end) : uint16_t(0);
         };
         if (BITS == 4 && n_tiles > 0) load_sc(0, scn);
-        for (int i = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0); ++i) {
-            const int s = i % kRing1, ck = i % n_chunks, tile = i / n_chunks;
+        for (int i = 0, tile = 0, ck = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0);
+             ++i, ck = (ck + 1 == n_chunks) ? 0 : ck + 1, tile += (ck == 0)) {
+            const int s = i % kRing1;
             if (BITS == 4 && ck == 0) {
 #pragma unroll
                 for (int k = 0; k < kMaxRc / 128; ++k) scc[k] = scn[k];
@@ -699,8 +702,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
         const uint32_t off8a = rbase * 128u + ((uint32_t(2 * q) ^ uint32_t(g8)) << 4);                 // int8 rows,
         const uint32_t off8b = rbase * 128u + ((uint32_t(2 * q + 1) ^ uint32_t(g8)) << 4);             // two units
         const int k8 = (cq & 1) * 2;
-        for (int i = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0); ++i) {
-            const int s = i % kRing2, vb = i & 1, tile = i / n_chunks, ck = i % n_chunks;
+        for (int i = 0, tile = 0, ck = 0; i < total && !__any_sync(0xffffffffu, abort_flag != 0);
+             ++i, ck = (ck + 1 == n_chunks) ? 0 : ck + 1, tile += (ck == 0)) {
+            const int s = i % kRing2, vb = i & 1;
             if (!wwait(&t2_full[s], (i / kRing2) & 1, p.err)) { abort_flag = 1; break; }
             if (i >= 2 && !wwait(&pva_empty[vb], ((i >> 1) - 1) & 1, p.err)) { abort_flag = 1; break; }
             if (BITS == 4 && ck == 0 && !wwait(&sc_full[tile & 1], (tile >> 1) & 1, p.err)) { abort_flag = 1; break; }
@@ -708,7 +712,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             // this thread's group scales: token rbase + 8 j' (j' = 4 h32 + j), group grp
             const __half *scs = reinterpret_cast<const __half *>(sm + kOffSc + (tile & 1) * kScBytes) +
                                 rbase * ngrp + (ch0 / 128 + ck);
-#pragma unroll
+#pragma unroll 1
             for (int h32 = 0; h32 < 2; ++h32) {             // 32 tokens: two 16x256b stores of 16 columns
                 // rows of the 4 tokens this thread supplies (16-token step g, 8-token block tb), loads first
                 constexpr int kU = BITS == 8 ? 2 : 1;       // 16-byte units of the warp's 32 channels
