@@ -160,8 +160,8 @@ class NativeBench:
         self.fused = False          # the PDL-chained calls are faster than the fused step today
         self.wsf = torch.zeros(max(1, q.qsvd_decode_step_workspace_bytes(B, wl.tmax, s.d, s.r, s.H, s.dh)),
                                dtype=torch.uint8, device=dev)
-        self.flushbuf = torch.ones(FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
-        self.flush_out = torch.zeros((), dtype=torch.int64, device=dev)
+        self.flushbuf = torch.ones(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+        self.flush_out = torch.zeros((), dtype=torch.float32, device=dev)
         self.stream = torch.cuda.current_stream()
         self._marshal()
 
@@ -229,9 +229,11 @@ class NativeBench:
             self._call(self.lib.qsvd_latent_decode_attn, self.dec_attn[t])
 
     def flush(self):
-        """Evict L2 by reading a 256 MiB buffer (leaves L2 clean, unlike a write)."""
+        """Evict L2 by reading a 256 MiB buffer: an fp32 sum in place, so no
+        temporary is written and L2 is left clean (dirty lines would slow the
+        next reads with write-backs)."""
         torch = self.torch
-        torch.sum(self.flushbuf, dim=(0,), dtype=torch.int64, out=self.flush_out)
+        torch.sum(self.flushbuf, dim=(0,), out=self.flush_out)
 
     def run_step(self, evs, stream=None):
         """evs: list of (start, end) event pairs, one per sub-step (prefill, decode 0..S-1)."""
@@ -303,13 +305,16 @@ class NativeBench:
             return T * d * 2 + T * d + 4 * T
         if label == "proj_dp4a":
             return r * d + T * d + 4 * r + 4 * T + 4 * T * r
+        if label == "proj_small":
+            # W_d codes and scales, X (bf16) in; the requantized latent rows out
+            return r * d + 4 * r + 2 * T * d + T * (tok + stok)
         if label == "requant":
             return 4 * T * r + T * (tok + stok) + 8 * T
         if label == "qproj":
             return r * d * 2 + B * (tok + stok) + 4 * B * d
         if label == "qabsorb":
             return r * d * 2 + 4 * B * d + 4 * B * H * r
-        if label in ("attn_chunk", "attn_tc"):
+        if label in ("attn_chunk", "attn_tc", "attn_mma"):
             return B * L * (tok + stok) + 4 * B * H * r
         if label == "combine_uv":
             return r * d * 2 + 4 * B * d
@@ -385,8 +390,8 @@ def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
     lc = torch.empty((T, r), dtype=torch.int8, device=dev)
     ls = torch.empty((T,), dtype=torch.float32, device=dev)
     ws = torch.zeros(q.qsvd_project_workspace_bytes(T, d, r), dtype=torch.uint8, device=dev)
-    flush = torch.ones((256 << 20) // 4, dtype=torch.int32, device=dev)
-    sink = torch.zeros((), dtype=torch.int64, device=dev)
+    flush = torch.ones((256 << 20) // 4, dtype=torch.float32, device=dev)
+    sink = torch.zeros((), dtype=torch.float32, device=dev)
     n = 16
     events = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
     for e in events:
@@ -398,7 +403,7 @@ def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
     lib.qsvd_profile_label.restype = ctypes.c_char_p
     gemm, call = [], []
     for it in range(iters + 1):
-        torch.sum(flush, dim=(0,), dtype=torch.int64, out=sink)
+        torch.sum(flush, dim=(0,), out=sink)
         lib.qsvd_profile_events(handles, n)
         q.qsvd_latent_project(W, X, lat_codes=lc, lat_scales=ls, workspace=ws)
         torch.cuda.synchronize()

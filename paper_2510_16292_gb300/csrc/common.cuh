@@ -227,15 +227,15 @@ __device__ __forceinline__ void requant_row_cta(const float *__restrict__ c_hat,
         for (int k = 0; k < kRqMaxQuads; ++k)
             m = fmaxf(m, fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w))));
         m = block_max<kRqThreads>(m, red);
-        const float s = quant_scale(m, clip, 127.0f);
+        const float s = quant_scale(m, clip, 127.0f), inv = quant_inv_scale(s);
 #pragma unroll
         for (int k = 0; k < kRqMaxQuads; ++k) {
             const int qi = threadIdx.x + k * kRqThreads;
             if (qi >= nq) break;
-            const uint32_t w = uint32_t(quant_code(v[k].x, s, 127) & 0xff) |
-                               (uint32_t(quant_code(v[k].y, s, 127) & 0xff) << 8) |
-                               (uint32_t(quant_code(v[k].z, s, 127) & 0xff) << 16) |
-                               (uint32_t(quant_code(v[k].w, s, 127) & 0xff) << 24);
+            const uint32_t w = uint32_t(quant_code_fast(v[k].x, s, inv, 127) & 0xff) |
+                               (uint32_t(quant_code_fast(v[k].y, s, inv, 127) & 0xff) << 8) |
+                               (uint32_t(quant_code_fast(v[k].z, s, inv, 127) & 0xff) << 16) |
+                               (uint32_t(quant_code_fast(v[k].w, s, inv, 127) & 0xff) << 24);
             if (tok_codes) reinterpret_cast<uint32_t *>(tok_codes)[qi] = w;
             if (cache_codes) reinterpret_cast<uint32_t *>(cache_codes)[qi] = w;
         }
@@ -252,9 +252,9 @@ __device__ __forceinline__ void requant_row_cta(const float *__restrict__ c_hat,
             float m = fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w)));
             m = warp_max(m);
             const __half hs = int4_group_scale(m, clip);
-            const float s = __half2float(hs);
-            const int c0 = quant_code(v[k].x, s, 7), c1 = quant_code(v[k].y, s, 7);
-            const int c2 = quant_code(v[k].z, s, 7), c3 = quant_code(v[k].w, s, 7);
+            const float s = __half2float(hs), inv = quant_inv_scale(s);
+            const int c0 = quant_code_fast(v[k].x, s, inv, 7), c1 = quant_code_fast(v[k].y, s, inv, 7);
+            const int c2 = quant_code_fast(v[k].z, s, inv, 7), c3 = quant_code_fast(v[k].w, s, inv, 7);
             const uint16_t w = uint16_t((c0 & 0xf) | ((c1 & 0xf) << 4) | ((c2 & 0xf) << 8) | ((c3 & 0xf) << 12));
             if (tok_codes) reinterpret_cast<uint16_t *>(tok_codes)[qi] = w;
             if (cache_codes) reinterpret_cast<uint16_t *>(cache_codes)[qi] = w;
@@ -306,13 +306,14 @@ __device__ __forceinline__ void requant_row_warp(const float *__restrict__ c_hat
             m = fmaxf(m, fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w))));
         }
         m = warp_max(m);
-        const float s = quant_scale(m, clip, 127.0f);
+        const float s = quant_scale(m, clip, 127.0f), inv = quant_inv_scale(s);
 #pragma unroll 4
         for (int qi = lane; qi < nq; qi += 32) {
             const float4 v = row[qi];
-            const uint32_t w = uint32_t(quant_code(v.x, s, 127) & 0xff) | (uint32_t(quant_code(v.y, s, 127) & 0xff) << 8) |
-                               (uint32_t(quant_code(v.z, s, 127) & 0xff) << 16) |
-                               (uint32_t(quant_code(v.w, s, 127) & 0xff) << 24);
+            const uint32_t w = uint32_t(quant_code_fast(v.x, s, inv, 127) & 0xff) |
+                               (uint32_t(quant_code_fast(v.y, s, inv, 127) & 0xff) << 8) |
+                               (uint32_t(quant_code_fast(v.z, s, inv, 127) & 0xff) << 16) |
+                               (uint32_t(quant_code_fast(v.w, s, inv, 127) & 0xff) << 24);
             if (tok_codes) reinterpret_cast<uint32_t *>(tok_codes)[qi] = w;
             if (cache_codes) reinterpret_cast<uint32_t *>(cache_codes)[qi] = w;
         }
@@ -329,9 +330,9 @@ __device__ __forceinline__ void requant_row_warp(const float *__restrict__ c_hat
             float m = fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w)));
             m = warp_max(m);
             const __half hs = int4_group_scale(m, clip);
-            const float s = __half2float(hs);
-            const int c0 = quant_code(v.x, s, 7), c1 = quant_code(v.y, s, 7);
-            const int c2 = quant_code(v.z, s, 7), c3 = quant_code(v.w, s, 7);
+            const float s = __half2float(hs), inv = quant_inv_scale(s);
+            const int c0 = quant_code_fast(v.x, s, inv, 7), c1 = quant_code_fast(v.y, s, inv, 7);
+            const int c2 = quant_code_fast(v.z, s, inv, 7), c3 = quant_code_fast(v.w, s, inv, 7);
             const uint16_t w = uint16_t((c0 & 0xf) | ((c1 & 0xf) << 4) | ((c2 & 0xf) << 8) | ((c3 & 0xf) << 12));
             if (tok_codes) reinterpret_cast<uint16_t *>(tok_codes)[qi] = w;
             if (cache_codes) reinterpret_cast<uint16_t *>(cache_codes)[qi] = w;

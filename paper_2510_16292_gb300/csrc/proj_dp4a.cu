@@ -95,7 +95,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                 }
             }
             m = block_max<kPsWarps * 32>(m, red);
-            const float s = quant_scale(m, act_clip, 127.0f);
+            const float s = quant_scale(m, act_clip, 127.0f), inv = quant_inv_scale(s);
 #pragma unroll
             for (int k = 0; k < kPsMaxD / 2048; ++k) {
                 const int col = (k * 256 + threadIdx.x) * 8;
@@ -103,8 +103,8 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                     uint32_t lo = 0, hi = 0;
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        lo |= uint32_t(quant_code(f[k][e], s, 127) & 0xff) << (8 * e);
-                        hi |= uint32_t(quant_code(f[k][e + 4], s, 127) & 0xff) << (8 * e);
+                        lo |= uint32_t(quant_code_fast(f[k][e], s, inv, 127) & 0xff) << (8 * e);
+                        hi |= uint32_t(quant_code_fast(f[k][e + 4], s, inv, 127) & 0xff) << (8 * e);
                     }
                     *reinterpret_cast<uint2 *>(xq_s + size_t(t) * d + col) = make_uint2(lo, hi);
                     if (xq_out && blockIdx.x == 0)
@@ -138,7 +138,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
             }
         }
         m = warp_max(m);
-        const float s = quant_scale(m, act_clip, 127.0f);
+        const float s = quant_scale(m, act_clip, 127.0f), inv = quant_inv_scale(s);
         for (int k0 = 0; k0 < kPsMaxD / 256; k0 += 8) {
             uint4 xv[8];
 #pragma unroll
@@ -155,8 +155,8 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                 uint32_t lo = 0, hi = 0;
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    lo |= uint32_t(quant_code(f[e], s, 127) & 0xff) << (8 * e);
-                    hi |= uint32_t(quant_code(f[e + 4], s, 127) & 0xff) << (8 * e);
+                    lo |= uint32_t(quant_code_fast(f[e], s, inv, 127) & 0xff) << (8 * e);
+                    hi |= uint32_t(quant_code_fast(f[e + 4], s, inv, 127) & 0xff) << (8 * e);
                 }
                 *reinterpret_cast<uint2 *>(xq_s + size_t(t) * d + col) = make_uint2(lo, hi);
                 if (xq_out && blockIdx.x == 0)

@@ -38,14 +38,14 @@ xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int8_t *__restr
         }
     }
     m = block_max<kXqThreads>(m, red);
-    const float s = quant_scale(m, clip, 127.0f);
+    const float s = quant_scale(m, clip, 127.0f), inv = quant_inv_scale(s);
     for (int i = threadIdx.x * 8; i < d; i += kXqThreads * 8) {
         uint32_t packed[2] = {0u, 0u};
         uint32_t bfw[4];
 #pragma unroll
         for (int e = 0; e < 8; e += 2) {
-            const int c0 = quant_code(row[i + e], s, 127);
-            const int c1 = quant_code(row[i + e + 1], s, 127);
+            const int c0 = quant_code_fast(row[i + e], s, inv, 127);
+            const int c1 = quant_code_fast(row[i + e + 1], s, inv, 127);
             packed[e >> 2] |= (uint32_t(c0 & 0xff) << ((e & 3) * 8)) |
                               (uint32_t(c1 & 0xff) << (((e & 3) + 1) * 8));
             bfw[e >> 1] = uint32_t(int_to_bf16_bits(c0)) | (uint32_t(int_to_bf16_bits(c1)) << 16);
