@@ -298,6 +298,59 @@ __device__ __forceinline__ void requant_row_warp(const float *__restrict__ c_hat
         }
     }
     uint8_t *tok_codes = lat_codes ? static_cast<uint8_t *>(lat_codes) + t * (bits == 8 ? r : r / 2) : nullptr;
+    constexpr int kRegQ = 16;                        // rows of r <= 2048 stay in registers (one round of loads)
+    if (nq <= 32 * kRegQ) {
+        float4 v[kRegQ];
+#pragma unroll
+        for (int k = 0; k < kRegQ; ++k) {
+            const int qi = k * 32 + lane;
+            v[k] = qi < nq ? row[qi] : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        if (bits == 8) {
+            float m = 0.0f;
+#pragma unroll
+            for (int k = 0; k < kRegQ; ++k)
+                m = fmaxf(m, fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w))));
+            m = warp_max(m);
+            const float s = quant_scale(m, clip, 127.0f), inv = quant_inv_scale(s);
+#pragma unroll
+            for (int k = 0; k < kRegQ; ++k) {
+                const int qi = k * 32 + lane;
+                if (qi >= nq) break;
+                const uint32_t w = uint32_t(quant_code_fast(v[k].x, s, inv, 127) & 0xff) |
+                                   (uint32_t(quant_code_fast(v[k].y, s, inv, 127) & 0xff) << 8) |
+                                   (uint32_t(quant_code_fast(v[k].z, s, inv, 127) & 0xff) << 16) |
+                                   (uint32_t(quant_code_fast(v[k].w, s, inv, 127) & 0xff) << 24);
+                if (tok_codes) reinterpret_cast<uint32_t *>(tok_codes)[qi] = w;
+                if (cache_codes) reinterpret_cast<uint32_t *>(cache_codes)[qi] = w;
+            }
+            if (lane == 0) {
+                if (lat_scales) static_cast<float *>(lat_scales)[t] = s;
+                if (cache_scale) *static_cast<float *>(cache_scale) = s;
+            }
+        } else {
+            // group g = quads 32 g .. 32 g + 31: quad k of every lane
+#pragma unroll
+            for (int k = 0; k < kRegQ; ++k) {
+                if (k * 32 >= nq) break;
+                float m = fmaxf(fmaxf(fabsf(v[k].x), fabsf(v[k].y)), fmaxf(fabsf(v[k].z), fabsf(v[k].w)));
+                m = warp_max(m);
+                const __half hs = int4_group_scale(m, clip);
+                const float s = __half2float(hs), inv = quant_inv_scale(s);
+                const int c0 = quant_code_fast(v[k].x, s, inv, 7), c1 = quant_code_fast(v[k].y, s, inv, 7);
+                const int c2 = quant_code_fast(v[k].z, s, inv, 7), c3 = quant_code_fast(v[k].w, s, inv, 7);
+                const uint16_t w = uint16_t((c0 & 0xf) | ((c1 & 0xf) << 4) | ((c2 & 0xf) << 8) | ((c3 & 0xf) << 12));
+                const int qi = k * 32 + lane;
+                if (tok_codes) reinterpret_cast<uint16_t *>(tok_codes)[qi] = w;
+                if (cache_codes) reinterpret_cast<uint16_t *>(cache_codes)[qi] = w;
+                if (lane == 0) {
+                    if (lat_scales) static_cast<__half *>(lat_scales)[t * (r / 128) + k] = hs;
+                    if (cache_scale) static_cast<__half *>(cache_scale)[k] = hs;
+                }
+            }
+        }
+        return;
+    }
     if (bits == 8) {
         float m = 0.0f;
 #pragma unroll 4

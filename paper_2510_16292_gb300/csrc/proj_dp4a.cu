@@ -6,6 +6,8 @@
 // decode path (T <= kPsMaxTok tokens): it quantizes X itself, streams its 8
 // rows of W_d codes into shared memory with one bulk copy, and the last CTA
 // to finish requantizes the latent rows and stores them (a1-a4 in one launch).
+#include <algorithm>
+
 #include "common.cuh"
 #include "launch.h"
 
@@ -50,7 +52,7 @@ constexpr int kPsWarps = 8;
 constexpr int kPsMaxD = 6144;          // d <= 6144: 24 x 16-byte vectors per lane
 constexpr int kPsWarpTok = 4;          // from this many tokens on, one warp per token
 
-__global__ void __launch_bounds__(kPsWarps * 32)
+__global__ void __launch_bounds__(kPsWarps * 32, 2)
 proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, const int8_t *__restrict__ w,
                   const float *__restrict__ ws, int r, int lat_bits, float lat_clip, float *__restrict__ c_hat,
                   int *__restrict__ counter, int8_t *__restrict__ xq_out, float *__restrict__ xs_out,
@@ -65,8 +67,9 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int j0 = blockIdx.x * kPsWarps;
     const int rows = min(kPsWarps, r - j0);
-    int8_t *w_s = reinterpret_cast<int8_t *>(smem);                  // [kPsWarps][d]
-    int8_t *xq_s = reinterpret_cast<int8_t *>(smem) + kPsWarps * d;  // [T][d]
+    const int dp = d + 16;                                           // padded row: conflict-free fragments
+    int8_t *w_s = reinterpret_cast<int8_t *>(smem);                  // [kPsWarps][dp]
+    int8_t *xq_s = reinterpret_cast<int8_t *>(smem) + kPsWarps * dp; // [T][dp]
     pdl_trigger();
     prefetch_share_l2(w, size_t(r) * d, blockIdx.x, gridDim.x);
     if (threadIdx.x == 0) {
@@ -76,7 +79,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     __syncthreads();
     if (threadIdx.x == 0) {     // W_d codes: no kernel's output, copied before the wait on the producer grid
         mbar_arrive_expect_tx(&bar, uint32_t(rows) * d);
-        bulk_g2s(w_s, w + size_t(j0) * d, uint32_t(rows) * d, &bar);
+        for (int i = 0; i < rows; ++i) bulk_g2s(w_s + size_t(i) * dp, w + size_t(j0 + i) * d, uint32_t(d), &bar);
     }
     pdl_wait();
     // a1: per-token int8 quantization.  Few tokens: the whole CTA works on one
@@ -106,7 +109,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                         lo |= uint32_t(quant_code_fast(f[k][e], s, inv, 127) & 0xff) << (8 * e);
                         hi |= uint32_t(quant_code_fast(f[k][e + 4], s, inv, 127) & 0xff) << (8 * e);
                     }
-                    *reinterpret_cast<uint2 *>(xq_s + size_t(t) * d + col) = make_uint2(lo, hi);
+                    *reinterpret_cast<uint2 *>(xq_s + size_t(t) * dp + col) = make_uint2(lo, hi);
                     if (xq_out && blockIdx.x == 0)
                         *reinterpret_cast<uint2 *>(xq_out + size_t(t) * d + col) = make_uint2(lo, hi);
                 }
@@ -117,20 +120,21 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
             }
         }
     }
-    // one warp per token: a pass for the maximum, then a pass (from L1) for
-    // the codes; 8 vectors in flight per lane
+    // one warp per token: the maximum over 12 vectors per lane in flight, then
+    // the codes from a second read of the row (L1 hits)
     for (int t = warp; t < T && T >= kPsWarpTok; t += kPsWarps) {
         const uint16_t *xrow = X + size_t(t) * d;
+        constexpr int kV = 12;
         float m = 0.0f;
-        for (int k0 = 0; k0 < kPsMaxD / 256; k0 += 8) {
-            uint4 xv[8];
+        for (int k0 = 0; k0 < kPsMaxD / 256; k0 += kV) {
+            uint4 xv[kV];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < kV; ++k) {
                 const int col = ((k0 + k) * 32 + lane) * 8;
                 xv[k] = col < d ? *reinterpret_cast<const uint4 *>(xrow + col) : make_uint4(0u, 0u, 0u, 0u);
             }
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < kV; ++k) {
                 float f[8];
                 unpack8_bf16(xv[k], f);
 #pragma unroll
@@ -139,15 +143,15 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
         }
         m = warp_max(m);
         const float s = quant_scale(m, act_clip, 127.0f), inv = quant_inv_scale(s);
-        for (int k0 = 0; k0 < kPsMaxD / 256; k0 += 8) {
-            uint4 xv[8];
+        for (int k0 = 0; k0 < kPsMaxD / 256; k0 += kV) {
+            uint4 xv[kV];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < kV; ++k) {
                 const int col = ((k0 + k) * 32 + lane) * 8;
                 xv[k] = col < d ? *reinterpret_cast<const uint4 *>(xrow + col) : make_uint4(0u, 0u, 0u, 0u);
             }
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < kV; ++k) {
                 const int col = ((k0 + k) * 32 + lane) * 8;
                 if (col >= d) break;
                 float f[8];
@@ -158,7 +162,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                     lo |= uint32_t(quant_code_fast(f[e], s, inv, 127) & 0xff) << (8 * e);
                     hi |= uint32_t(quant_code_fast(f[e + 4], s, inv, 127) & 0xff) << (8 * e);
                 }
-                *reinterpret_cast<uint2 *>(xq_s + size_t(t) * d + col) = make_uint2(lo, hi);
+                *reinterpret_cast<uint2 *>(xq_s + size_t(t) * dp + col) = make_uint2(lo, hi);
                 if (xq_out && blockIdx.x == 0)
                     *reinterpret_cast<uint2 *>(xq_out + size_t(t) * d + col) = make_uint2(lo, hi);
             }
@@ -171,12 +175,61 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     __syncthreads();
     mbar_wait(&bar, 0, err);
     // a2 + first half of a3: exact int32 dot products, then the fp32 dequantization
-    if (warp < rows) {
+    if (T >= kPsWarpTok) {
+        // Tensor cores: the CTA's 16-token x 8-channel tile (m16n8k16, codes
+        // exact in fp16), K split over the 8 warps.  A warp's partial sums stay
+        // below d/8 * 127^2 < 2^24, so they are exact integers in fp32.
+        const int g8 = lane >> 2, cq = lane & 3;
+        const int kspan = d / kPsWarps, kb = warp * kspan;
+        const bool live0 = g8 < T, live1 = g8 + 8 < T;
+        const int8_t *xa0 = xq_s + size_t(live0 ? g8 : 0) * dp, *xa1 = xq_s + size_t(live1 ? g8 + 8 : 0) * dp;
+        const int8_t *wb = w_s + size_t(g8 < rows ? g8 : 0) * dp;
+        auto pair = [](const int8_t *p) {           // two int8 codes -> fp16 pair, exact
+            const uint32_t u = uint32_t(*reinterpret_cast<const uint16_t *>(p)) ^ 0x8080u;
+            const uint32_t a = __byte_perm(u, 0x64646464u, 0x5150);
+            const __half2 h = __hsub2(*reinterpret_cast<const __half2 *>(&a), __half2half2(__ushort_as_half(0x6480)));
+            return *reinterpret_cast<const uint32_t *>(&h);
+        };
+        float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int k0 = kb; k0 < kb + kspan; k0 += 32) {
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {           // two independent accumulator chains
+                const int k = k0 + 16 * u + 2 * cq;
+                const uint32_t a0 = live0 ? pair(xa0 + k) : 0u, a1 = live1 ? pair(xa1 + k) : 0u;
+                const uint32_t a2 = live0 ? pair(xa0 + k + 8) : 0u, a3 = live1 ? pair(xa1 + k + 8) : 0u;
+                const uint32_t b0 = pair(wb + k), b1 = pair(wb + k + 8);
+                float *cc = u ? c1 : c0;
+                asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                             "{%0,%1,%2,%3};"
+                             : "+f"(cc[0]), "+f"(cc[1]), "+f"(cc[2]), "+f"(cc[3])
+                             : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+            }
+        }
+        // rows g8 / g8 + 8, channels 2cq / 2cq + 1; the warps' partials added as int32
+        int *red_i = reinterpret_cast<int *>(xq_s);   // codes no longer needed: reuse [8 warps][16][8]
+        __syncthreads();
+        red_i[(warp * 16 + g8) * 8 + 2 * cq] = __float2int_rn(c0[0] + c1[0]);
+        red_i[(warp * 16 + g8) * 8 + 2 * cq + 1] = __float2int_rn(c0[1] + c1[1]);
+        red_i[(warp * 16 + g8 + 8) * 8 + 2 * cq] = __float2int_rn(c0[2] + c1[2]);
+        red_i[(warp * 16 + g8 + 8) * 8 + 2 * cq + 1] = __float2int_rn(c0[3] + c1[3]);
+        __syncthreads();
+        if (threadIdx.x < 128) {
+            const int t = threadIdx.x >> 3, jj = threadIdx.x & 7;
+            if (t < T && jj < rows) {
+                int acc = 0;
+#pragma unroll
+                for (int w = 0; w < kPsWarps; ++w) acc += red_i[(w * 16 + t) * 8 + jj];
+                const int j = j0 + jj;
+                c_hat[size_t(t) * r + j] = __fmul_rn(__fmul_rn(__int2float_rn(acc), xs_s[t]), ws[j]);
+                if (acc_out) acc_out[size_t(t) * r + j] = acc;
+            }
+        }
+    } else if (warp < rows) {
         const int j = j0 + warp;
-        const int *wrow = reinterpret_cast<const int *>(w_s + size_t(warp) * d);
+        const int *wrow = reinterpret_cast<const int *>(w_s + size_t(warp) * dp);
         const float sw = ws[j];
         for (int t = 0; t < T; ++t) {
-            const int *xrow = reinterpret_cast<const int *>(xq_s + size_t(t) * d);
+            const int *xrow = reinterpret_cast<const int *>(xq_s + size_t(t) * dp);
             int acc = 0;
 #pragma unroll 8
             for (int i = lane; i < d / 4; i += 32) acc = __dp4a(wrow[i], xrow[i], acc);
@@ -212,7 +265,8 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
                               cudaStream_t s) {
     CacheView dv{};
     if (dst) dv = *dst;
-    const size_t smem = size_t(kPsWarps) * d + size_t(T) * d;
+    // padded rows; the tensor-core path reuses the code rows for an [8][16][8] int32 reduction
+    const size_t smem = size_t(kPsWarps) * (d + 16) + std::max(size_t(T) * (d + 16), size_t(kPsWarps) * 16 * 8 * 4);
     cudaError_t e = ensure_smem(proj_small_kernel, smem);
     if (e != cudaSuccess) return e;
     e = launch_pdl(proj_small_kernel, dim3((r + kPsWarps - 1) / kPsWarps), dim3(kPsWarps * 32), smem, s, X, T, d,

@@ -84,8 +84,10 @@ def test_project_tiny_bit_exact(tiny):
 
 
 @pytest.mark.parametrize("bits", [8, 4])
-@pytest.mark.parametrize("T", [1, 37, 640])
+@pytest.mark.parametrize("T", [1, 3, 4, 9, 16, 37, 640])
 def test_project_7b_bit_exact(l7b, bits, T):
+    """T <= 3: the decode projection quantizes with the whole CTA; 4 <= T <= 16:
+    a warp per token and the tensor-core dot products; larger T: the GEMM."""
     wl, inp, w = l7b
     W = q().qsvd_quantize_weight(torch.from_numpy(w["W_d"].astype(np.float32)).to(dev()))
     X = inp.X_prefill[0][:T]
@@ -277,6 +279,24 @@ def test_project_tc_worst_case_exact(d, r, T):
     ref = latent.latent_project(synthetic.bf16_from_bits(Xb), Wc, s_w, lat_bits=8)
     assert np.abs(ref["acc"]).max() > 2 ** 24
     _assert_project_exact(got, ref, 8)
+
+
+@pytest.mark.parametrize("T", [5, 16])
+def test_project_small_13b_and_tiny_shapes(T):
+    """The decode projection at d = 5120, r = 2048 (K split 640 per warp) and at
+    the tiny layer's d = 256 (32 per warp), against the oracle, bit-exact."""
+    for name in ("llava13b", "tiny"):
+        wl = synthetic.WORKLOADS[name]
+        s = wl.shape
+        rng = np.random.default_rng(11)
+        w = (rng.standard_normal((s.d, s.r)) / np.sqrt(s.d)).astype(np.float32)
+        X = synthetic.bf16_bits(rng.standard_normal((T, s.d)) * np.where(rng.random(s.d) < 0.01, 20.0, 1.0))
+        wq, s_w = quant.quantize_columns(w.astype(np.float64), 8)
+        W = q().qsvd_quantize_weight(torch.from_numpy(w).to(dev()))
+        for bits in ((8, 4) if s.r % 128 == 0 else (8,)):      # int4 needs whole 128-channel groups
+            got = _project_outputs(W, X, s.r, bits)
+            ref = latent.latent_project(synthetic.bf16_from_bits(X), wq, s_w, lat_bits=bits)
+            _assert_project_exact(got, ref, bits)
 
 
 def test_project_13b_shape_tc():
