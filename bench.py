@@ -43,6 +43,7 @@ import synthetic  # noqa: E402
 METRIC = "decode tokens/s + latent-cache HBM GB/s; prefill int8 TOPS (LLaVA-7B shape)"
 WORKLOAD = "llava7b"
 FLUSH_BYTES = 256 << 20
+L2_BYTES = 129 << 20          # GB300 L2 (the rotation's sizing)
 
 
 def parse():
@@ -56,6 +57,9 @@ def parse():
     p.add_argument("--no-prefill13", action="store_true")
     p.add_argument("--workload", default=WORKLOAD, choices=sorted(synthetic.WORKLOADS))
     p.add_argument("--decode-steps", type=int, default=0, help="override the workload's decode steps")
+    p.add_argument("--l2", default="rotate", choices=["rotate", "flush"],
+                   help="cold-L2 method: rotate through copies of the layer larger than L2 together, or flush "
+                        "L2 before every sub-step")
     return p.parse_args()
 
 
@@ -125,16 +129,12 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # native arm
 # ---------------------------------------------------------------------------
-class NativeBench:
-    def __init__(self, wl, rank):
-        import torch
-        import paper_2510_16292_gb300 as q
-        self.torch, self.q, self.wl = torch, q, wl
+class NativeLayer:
+    """One independently seeded copy of the layer: weights, latent cache, inputs."""
+
+    def __init__(self, nb, inp, X_from=None):
+        torch, q, wl, dev = nb.torch, nb.q, nb.wl, nb.dev
         s = wl.shape
-        self.dev = torch.device("cuda", torch.cuda.current_device())
-        inp = synthetic.gen_layer(wl, seed=rank)
-        self.inp = inp
-        dev = self.dev
 
         def bf16(bits):
             a = np.ascontiguousarray(bits).view(np.int16)
@@ -142,25 +142,59 @@ class NativeBench:
 
         self.W = q.qsvd_quantize_weight(torch.from_numpy(inp.W_d.astype(np.float32)).to(dev))
         self.U = [bf16(u) for u in (inp.U_q, inp.U_k, inp.U_v)]
+        if X_from is None:
+            self.Xp = bf16(inp.X_prefill.reshape(wl.B * wl.prefill, s.d))
+            self.Xd = bf16(inp.X_decode)                   # [S, B, d]
+        else:                                              # inputs shared with another copy
+            self.Xp, self.Xd = X_from.Xp, X_from.Xd
+        self.cache = q.LatentCache.empty(wl.B, wl.tmax, s.r, wl.lat_bits, dev)
+        self.O = torch.empty((wl.B, s.d), dtype=torch.float32, device=dev)
+
+
+class NativeBench:
+    """The layer step on the GPU.  L2 method `rotate` (default): K independently
+    seeded copies of the layer whose weights and caches together exceed twice
+    the L2, and every decode token runs through all K in turn, as in a stack of
+    layers: each layer's data comes from HBM while the kernels' code stays
+    cached, as it does in serving.  `flush`: one copy, L2 evicted by a 256 MiB
+    read before every sub-step (code cold as well)."""
+
+    def __init__(self, wl, rank, l2="rotate"):
+        import torch
+        import paper_2510_16292_gb300 as q
+        self.torch, self.q, self.wl = torch, q, wl
+        s = wl.shape
+        self.dev = torch.device("cuda", torch.cuda.current_device())
+        dev = self.dev
         B, P, S = wl.B, wl.prefill, wl.decode_steps
         self.B, self.P, self.S = B, P, S
-        self.Xp = bf16(inp.X_prefill.reshape(B * P, s.d))
-        self.Xd = bf16(inp.X_decode)                       # [S, B, d]
-        self.cache = q.LatentCache.empty(B, wl.tmax, s.r, wl.lat_bits, dev)
+        self.l2 = l2
+        tok = (s.r + 4) if wl.lat_bits == 8 else (s.r // 2 + 2 * (s.r // 128))
+        layer_bytes = 3 * s.r * s.d * 2 + s.r * s.d + B * wl.tmax * tok      # what a decode step reads
+        self.K = 1 if l2 == "flush" else max(2, min(16, -(-2 * L2_BYTES // layer_bytes)))
+        self.layer_bytes = layer_bytes
+        self.layers = []
+        for k in range(self.K):
+            share = k > 0 and B * P * s.d * 2 > L2_BYTES // 2      # large inputs cannot stay cached anyway
+            inp = synthetic.gen_layer(wl, seed=rank * 64, layer=k, prefill_rows=0 if share else None,
+                                      decode_steps=0 if share else None)
+            self.layers.append(NativeLayer(self, inp, X_from=self.layers[0] if share else None))
+        L0 = self.layers[0]
+        self.W, self.U, self.cache, self.Xp, self.Xd, self.O = L0.W, L0.U, L0.cache, L0.Xp, L0.Xd, L0.O
         i32 = lambda a: torch.as_tensor(np.asarray(a, dtype=np.int32), device=dev)  # noqa: E731
         self.pseq = i32(np.repeat(np.arange(B), P))
         self.ppos = i32(np.tile(np.arange(P), B))
         self.dseq = i32(np.arange(B))
         self.dpos = [i32(np.full(B, P + t)) for t in range(S)]
         self.dlen = [i32(np.full(B, P + t + 1)) for t in range(S)]
-        self.O = torch.empty((B, s.d), dtype=torch.float32, device=dev)
+        # one workspace of each kind: the calls run one after another on one stream
         self.wsp = torch.zeros(q.qsvd_project_workspace_bytes(B * P, s.d, s.r), dtype=torch.uint8, device=dev)
         self.wsd = torch.zeros(q.qsvd_decode_workspace_bytes(B, wl.tmax, s.r, s.H, s.dh), dtype=torch.uint8,
                                device=dev)
         self.fused = False          # the PDL-chained calls are faster than the fused step today
         self.wsf = torch.zeros(max(1, q.qsvd_decode_step_workspace_bytes(B, wl.tmax, s.d, s.r, s.H, s.dh)),
                                dtype=torch.uint8, device=dev)
-        self.flushbuf = torch.ones(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+        self.flushbuf = torch.ones(FLUSH_BYTES // 4 if l2 == "flush" else 1, dtype=torch.float32, device=dev)
         self.flush_out = torch.zeros((), dtype=torch.float32, device=dev)
         self.stream = torch.cuda.current_stream()
         self._marshal()
@@ -171,28 +205,29 @@ class NativeBench:
         q, wl, s = self.q, self.wl, self.wl.shape
         lib = q._lib
         self.lib = lib
-        self.cW = self.W._c()
-        self.cC = self.cache._c()
         st = (stream or self.stream).cuda_stream
-        self.pre_args = (ctypes.byref(self.cW), self.Xp.data_ptr(), self.B * self.P, 1.0, wl.lat_bits, 1.0,
-                         None, None, ctypes.byref(self.cC), self.pseq.data_ptr(), self.ppos.data_ptr(),
-                         None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st)
-        self.dec_proj = []
-        self.dec_attn = []
-        self.dec_fused = []
-        for t in range(self.S):
-            self.dec_proj.append((ctypes.byref(self.cW), self.Xd[t].data_ptr(), self.B, 1.0, wl.lat_bits, 1.0,
-                                  None, None, ctypes.byref(self.cC), self.dseq.data_ptr(), self.dpos[t].data_ptr(),
+        self.pre_args, self.dec_proj, self.dec_attn, self.dec_fused = [], [], [], []
+        for L in self.layers:
+            L.cW, L.cC = L.W._c(), L.cache._c()
+            self.pre_args.append((ctypes.byref(L.cW), L.Xp.data_ptr(), self.B * self.P, 1.0, wl.lat_bits, 1.0,
+                                  None, None, ctypes.byref(L.cC), self.pseq.data_ptr(), self.ppos.data_ptr(),
                                   None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st))
-            self.dec_attn.append((ctypes.byref(self.cC), self.dlen[t].data_ptr(), self.P + t + 1,
-                                  self.U[0].data_ptr(), self.U[1].data_ptr(), self.U[2].data_ptr(), s.H, s.dh,
-                                  1.0 / math.sqrt(s.dh), self.O.data_ptr(), self.wsd.data_ptr(),
-                                  self.wsd.numel(), st))
-            self.dec_fused.append((ctypes.byref(self.cW), self.Xd[t].data_ptr(), ctypes.byref(self.cC),
-                                   self.dlen[t].data_ptr(), self.P + t + 1, self.U[0].data_ptr(),
-                                   self.U[1].data_ptr(), self.U[2].data_ptr(), s.H, s.dh, 1.0, 1.0,
-                                   1.0 / math.sqrt(s.dh), self.O.data_ptr(), self.wsf.data_ptr(),
-                                   self.wsf.numel(), st))
+            proj, attn, fused = [], [], []
+            for t in range(self.S):
+                proj.append((ctypes.byref(L.cW), L.Xd[t].data_ptr(), self.B, 1.0, wl.lat_bits, 1.0,
+                             None, None, ctypes.byref(L.cC), self.dseq.data_ptr(), self.dpos[t].data_ptr(),
+                             None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st))
+                attn.append((ctypes.byref(L.cC), self.dlen[t].data_ptr(), self.P + t + 1,
+                             L.U[0].data_ptr(), L.U[1].data_ptr(), L.U[2].data_ptr(), s.H, s.dh,
+                             1.0 / math.sqrt(s.dh), L.O.data_ptr(), self.wsd.data_ptr(), self.wsd.numel(), st))
+                fused.append((ctypes.byref(L.cW), L.Xd[t].data_ptr(), ctypes.byref(L.cC),
+                              self.dlen[t].data_ptr(), self.P + t + 1, L.U[0].data_ptr(),
+                              L.U[1].data_ptr(), L.U[2].data_ptr(), s.H, s.dh, 1.0, 1.0,
+                              1.0 / math.sqrt(s.dh), L.O.data_ptr(), self.wsf.data_ptr(),
+                              self.wsf.numel(), st))
+            self.dec_proj.append(proj)
+            self.dec_attn.append(attn)
+            self.dec_fused.append(fused)
 
     def build_graph(self):
         """Capture one whole step (flushes, sub-step events and every C-ABI
@@ -219,21 +254,24 @@ class NativeBench:
             raise RuntimeError(f"qsvd status {stt}: {self.lib.qsvd_last_error().decode()}")
 
     def prefill(self):
-        self._call(self.lib.qsvd_latent_project, self.pre_args)
+        for k in range(self.K):
+            self._call(self.lib.qsvd_latent_project, self.pre_args[k])
 
     def decode(self, t):
-        if self.fused:
-            self._call(self.lib.qsvd_decode_step, self.dec_fused[t])
-        else:
-            self._call(self.lib.qsvd_latent_project, self.dec_proj[t])
-            self._call(self.lib.qsvd_latent_decode_attn, self.dec_attn[t])
+        """Decode token t through every copy of the layer."""
+        for k in range(self.K):
+            if self.fused:
+                self._call(self.lib.qsvd_decode_step, self.dec_fused[k][t])
+            else:
+                self._call(self.lib.qsvd_latent_project, self.dec_proj[k][t])
+                self._call(self.lib.qsvd_latent_decode_attn, self.dec_attn[k][t])
 
     def flush(self):
-        """Evict L2 by reading a 256 MiB buffer: an fp32 sum in place, so no
-        temporary is written and L2 is left clean (dirty lines would slow the
-        next reads with write-backs)."""
-        torch = self.torch
-        torch.sum(self.flushbuf, dim=(0,), out=self.flush_out)
+        """`flush` method: evict L2 by reading a 256 MiB buffer (an fp32 sum in
+        place, so no temporary is written and L2 is left clean; dirty lines
+        would slow the next reads with write-backs).  `rotate`: nothing."""
+        if self.l2 == "flush":
+            self.torch.sum(self.flushbuf, dim=(0,), out=self.flush_out)
 
     def run_step(self, evs, stream=None):
         """evs: list of (start, end) event pairs, one per sub-step (prefill, decode 0..S-1)."""
@@ -259,7 +297,7 @@ class NativeBench:
     # ---- kernel-level profile (CUDA events the library records between its kernels) ----
     def profile(self, steps=1):
         torch = self.torch
-        n = steps * (self.S * 12 + 8)
+        n = steps * self.K * (self.S * 12 + 8)
         events = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
         for e in events:            # torch creates the CUDA event lazily, on first record
             e.record(self.stream)
@@ -333,12 +371,15 @@ class NativeBench:
 
     # ---- end to end through the public binding with host buffers ----
     def e2e(self, steps, warmup):
-        torch, q, s = self.torch, self.q, self.wl.shape
-        hx_p = torch.empty(self.Xp.shape, dtype=torch.bfloat16, pin_memory=True)
-        hx_p.copy_(self.Xp.cpu())
-        hx_d = torch.empty(self.Xd.shape, dtype=torch.bfloat16, pin_memory=True)
-        hx_d.copy_(self.Xd.cpu())
-        hO = torch.empty((self.S, self.B, s.d), dtype=torch.float32, pin_memory=True)
+        """Per layer copy: host X -> device, projection and decode attention
+        through the Python binding, O -> host; decode tokens/s of one layer."""
+        torch, q, s, K = self.torch, self.q, self.wl.shape, self.K
+        hx_p = [torch.empty(L.Xp.shape, dtype=torch.bfloat16, pin_memory=True) for L in self.layers]
+        hx_d = [torch.empty(L.Xd.shape, dtype=torch.bfloat16, pin_memory=True) for L in self.layers]
+        for L, hp, hd in zip(self.layers, hx_p, hx_d):
+            hp.copy_(L.Xp.cpu())
+            hd.copy_(L.Xd.cpu())
+        hO = torch.empty((K, self.S, self.B, s.d), dtype=torch.float32, pin_memory=True)
         dXp = torch.empty_like(self.Xp)
         dXd = torch.empty((self.B, s.d), dtype=torch.bfloat16, device=self.dev)
         E = torch.cuda.Event
@@ -347,27 +388,30 @@ class NativeBench:
             evs = [(E(enable_timing=True), E(enable_timing=True)) for _ in range(self.S + 1)]
             self.flush()
             evs[0][0].record()
-            dXp.copy_(hx_p, non_blocking=True)
-            q.qsvd_latent_project(self.W, dXp, 1.0, self.wl.lat_bits, 1.0, dst=self.cache, dst_seq=self.pseq,
-                                  dst_pos=self.ppos, workspace=self.wsp)
+            for k, L in enumerate(self.layers):
+                dXp.copy_(hx_p[k], non_blocking=True)
+                q.qsvd_latent_project(L.W, dXp, 1.0, self.wl.lat_bits, 1.0, dst=L.cache, dst_seq=self.pseq,
+                                      dst_pos=self.ppos, workspace=self.wsp)
             evs[0][1].record()
             for t in range(self.S):
                 self.flush()
                 evs[t + 1][0].record()
-                dXd.copy_(hx_d[t], non_blocking=True)
-                q.qsvd_latent_project(self.W, dXd, 1.0, self.wl.lat_bits, 1.0, dst=self.cache,
-                                      dst_seq=self.dseq, dst_pos=self.dpos[t], workspace=self.wsp)
-                q.qsvd_latent_decode_attn(self.cache, self.dlen[t], self.P + t + 1, *self.U, s.H, s.dh, self.O,
-                                          workspace=self.wsd)
-                hO[t].copy_(self.O, non_blocking=True)
+                for k, L in enumerate(self.layers):
+                    dXd.copy_(hx_d[k][t], non_blocking=True)
+                    q.qsvd_latent_project(L.W, dXd, 1.0, self.wl.lat_bits, 1.0, dst=L.cache,
+                                          dst_seq=self.dseq, dst_pos=self.dpos[t], workspace=self.wsp)
+                    q.qsvd_latent_decode_attn(L.cache, self.dlen[t], self.P + t + 1, *L.U, s.H, s.dh, L.O,
+                                              workspace=self.wsd)
+                    hO[k, t].copy_(L.O, non_blocking=True)
                 evs[t + 1][1].record()
             torch.cuda.synchronize()
             if it >= warmup:
                 tot.append(sum(a.elapsed_time(b) for a, b in evs[1:]) * 1e-3)
         dec_s = statistics.mean(tot)
-        h2d = self.B * self.P * s.d * 2 + self.S * self.B * s.d * 2
-        d2h = self.S * self.B * s.d * 4
-        return self.B * self.S / dec_s, h2d, d2h
+        # per step (one token through the K copies)
+        h2d = K * (self.B * self.P * s.d * 2 + self.S * self.B * s.d * 2)
+        d2h = K * self.S * self.B * s.d * 4
+        return self.B * self.S * K / dec_s, h2d, d2h
 
 
 def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
@@ -431,7 +475,8 @@ def run_native(args, rank, world, local_rank):
     wl = synthetic.WORKLOADS[args.workload]
     if args.decode_steps:
         wl = dataclasses.replace(wl, decode_steps=args.decode_steps)
-    nb = NativeBench(wl, rank)
+    nb = NativeBench(wl, rank, l2=args.l2)
+    K = nb.K
     S = wl.decode_steps
     hbm, _, peak_kind = peaks()
 
@@ -451,7 +496,7 @@ def run_native(args, rank, world, local_rank):
         torch.cuda.synchronize()                   # events are re-recorded by the next replay
         pre.append(evs[0][0].elapsed_time(evs[0][1]) * 1e-3)
         d_t = [evs[t + 1][0].elapsed_time(evs[t + 1][1]) * 1e-3 for t in range(S)]
-        per_dec.append(d_t)
+        per_dec.append([x / K for x in d_t])          # per copy of the layer
         dec.append(sum(d_t))
     if world > 1:
         torch.distributed.barrier()
@@ -462,14 +507,14 @@ def run_native(args, rank, world, local_rank):
         tt = torch.tensor([dec_total, pre_total], dtype=torch.float64, device=nb.dev)
         torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
         dec_total, pre_total = float(tt[0]), float(tt[1])
-    dec_tokens = world * wl.B * S * args.steps
+    dec_tokens = world * wl.B * S * K * args.steps      # tokens through one copy of the layer, all copies
     value = dec_tokens / dec_total
     s = wl.shape
     prefill_ops = 2 * wl.B * wl.prefill * s.d * s.r
-    prefill_tops = world * prefill_ops * args.steps / pre_total / 1e12
+    prefill_tops = world * K * prefill_ops * args.steps / pre_total / 1e12
     tok_bytes = (s.r + 4) if wl.lat_bits == 8 else (s.r // 2 + 2 * (s.r // 128))
-    cache_bytes = sum(wl.B * (wl.prefill + t + 1) * tok_bytes for t in range(S))
-    roof_s = sum(nb.step_roofline_bytes(t) for t in range(S)) / (hbm * 1e9)
+    cache_bytes = K * sum(wl.B * (wl.prefill + t + 1) * tok_bytes for t in range(S))
+    roof_s = K * sum(nb.step_roofline_bytes(t) for t in range(S)) / (hbm * 1e9)
     step_frac = roof_s / statistics.mean(dec)
 
     # kernel-level profile (separate pass of the same step) -> dominant kernel + roofline
@@ -510,8 +555,12 @@ def run_native(args, rank, world, local_rank):
         "data": "synthetic",
         "config": {"workload": workload_desc(wl), "global_batch": world * wl.B,
                    "seq_len": wl.tmax, "parallelism": f"replicas x{world} (one independent layer per GPU)",
-                   "l2": "flushed (256 MiB read) before the prefill and before every decode step; "
-                         "flushes outside the timed intervals",
+                   "l2": (f"inputs larger than L2: {K} independently seeded copies of the layer "
+                          f"({K} x {nb.layer_bytes / 2**20:.0f} MiB of weights and latent cache); every decode "
+                          f"token runs through all copies in turn and value counts tokens through one copy"
+                          if args.l2 == "rotate" else
+                          "flushed (256 MiB read) before the prefill and before every decode step; "
+                          "flushes outside the timed intervals"),
                    "launch": "one CUDA graph per step (captured C-ABI calls, PDL-chained kernels)"},
         "secondary": {
             "decode_ms_per_step": round(dec_total / args.steps * 1e3, 4),
@@ -520,7 +569,7 @@ def run_native(args, rank, world, local_rank):
             "prefill_tops": round(prefill_tops, 3),
             "latent_cache_gbs": round(cache_bytes * args.steps * world / dec_total / 1e9, 2),
             "decode_step_roofline_frac": round(step_frac, 4),
-            "decode_step_roofline_us": round(roof_s / S * 1e6, 3),
+            "decode_step_roofline_us": round(roof_s / (S * K) * 1e6, 3),
             "wall_s_timed_region": round(t_wall, 3),
             "kernels": kernels,
             "prefill_13b": pre13,

@@ -50,7 +50,7 @@ proj_dp4a_kernel(const int8_t *__restrict__ xq, int64_t T, int d, const int8_t *
 // ---------------------------------------------------------------------------
 constexpr int kPsWarps = 8;
 constexpr int kPsMaxD = 6144;          // d <= 6144: 24 x 16-byte vectors per lane
-constexpr int kPsWarpTok = 4;          // from this many tokens on, one warp per token
+constexpr int kPsWarpTok = 4;          // from this many tokens on: tensor-core dot products, a warp per latent row
 
 __global__ void __launch_bounds__(kPsWarps * 32, 2)
 proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, const int8_t *__restrict__ w,
@@ -63,6 +63,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     __shared__ __align__(8) uint64_t bar;
     __shared__ float xs_s[kPsMaxTok];
     __shared__ float red[kPsWarps];
+    __shared__ float red4[kPsWarps][4];
     __shared__ int last;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int j0 = blockIdx.x * kPsWarps;
@@ -82,94 +83,67 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
         for (int i = 0; i < rows; ++i) bulk_g2s(w_s + size_t(i) * dp, w + size_t(j0 + i) * d, uint32_t(d), &bar);
     }
     pdl_wait();
-    // a1: per-token int8 quantization.  Few tokens: the whole CTA works on one
-    // token at a time; more tokens: one warp per token (see below).
-    if (T < kPsWarpTok) {
-        for (int t = 0; t < T; ++t) {
-            float f[kPsMaxD / 2048][8];
-            float m = 0.0f;
+    // a1: per-token int8 quantization by the whole CTA, up to kQg tokens at a
+    // time: one round of loads, the per-token maxima reduced together
+    constexpr int kQg = 4, kVt = kPsMaxD / 2048;    // tokens per round, 16-byte vectors per thread per token
+    for (int t0 = 0; t0 < T; t0 += kQg) {
+        const int ng = min(kQg, T - t0);
+        uint4 xv[kQg][kVt];
+        float m[kQg];
 #pragma unroll
-            for (int k = 0; k < kPsMaxD / 2048; ++k) {
+        for (int g = 0; g < kQg; ++g) {
+            m[g] = 0.0f;
+#pragma unroll
+            for (int k = 0; k < kVt; ++k) {
                 const int col = (k * 256 + threadIdx.x) * 8;
-                if (col < d) {
-                    unpack8_bf16(*reinterpret_cast<const uint4 *>(X + size_t(t) * d + col), f[k]);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(f[k][e]));
-                }
-            }
-            m = block_max<kPsWarps * 32>(m, red);
-            const float s = quant_scale(m, act_clip, 127.0f), inv = quant_inv_scale(s);
-#pragma unroll
-            for (int k = 0; k < kPsMaxD / 2048; ++k) {
-                const int col = (k * 256 + threadIdx.x) * 8;
-                if (col < d) {
-                    uint32_t lo = 0, hi = 0;
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        lo |= uint32_t(quant_code_fast(f[k][e], s, inv, 127) & 0xff) << (8 * e);
-                        hi |= uint32_t(quant_code_fast(f[k][e + 4], s, inv, 127) & 0xff) << (8 * e);
-                    }
-                    *reinterpret_cast<uint2 *>(xq_s + size_t(t) * dp + col) = make_uint2(lo, hi);
-                    if (xq_out && blockIdx.x == 0)
-                        *reinterpret_cast<uint2 *>(xq_out + size_t(t) * d + col) = make_uint2(lo, hi);
-                }
-            }
-            if (threadIdx.x == 0) {
-                xs_s[t] = s;
-                if (xs_out && blockIdx.x == 0) xs_out[t] = s;
+                xv[g][k] = (g < ng && col < d) ? *reinterpret_cast<const uint4 *>(X + size_t(t0 + g) * d + col)
+                                               : make_uint4(0u, 0u, 0u, 0u);
             }
         }
-    }
-    // one warp per token: the maximum over 12 vectors per lane in flight, then
-    // the codes from a second read of the row (L1 hits)
-    for (int t = warp; t < T && T >= kPsWarpTok; t += kPsWarps) {
-        const uint16_t *xrow = X + size_t(t) * d;
-        constexpr int kV = 12;
-        float m = 0.0f;
-        for (int k0 = 0; k0 < kPsMaxD / 256; k0 += kV) {
-            uint4 xv[kV];
 #pragma unroll
-            for (int k = 0; k < kV; ++k) {
-                const int col = ((k0 + k) * 32 + lane) * 8;
-                xv[k] = col < d ? *reinterpret_cast<const uint4 *>(xrow + col) : make_uint4(0u, 0u, 0u, 0u);
-            }
+        for (int g = 0; g < kQg; ++g) {
 #pragma unroll
-            for (int k = 0; k < kV; ++k) {
+            for (int k = 0; k < kVt; ++k) {
                 float f[8];
-                unpack8_bf16(xv[k], f);
+                unpack8_bf16(xv[g][k], f);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(f[e]));
+                for (int e = 0; e < 8; ++e) m[g] = fmaxf(m[g], fabsf(f[e]));
             }
+            m[g] = warp_max(m[g]);
         }
-        m = warp_max(m);
-        const float s = quant_scale(m, act_clip, 127.0f), inv = quant_inv_scale(s);
-        for (int k0 = 0; k0 < kPsMaxD / 256; k0 += kV) {
-            uint4 xv[kV];
+        if (lane == 0)
 #pragma unroll
-            for (int k = 0; k < kV; ++k) {
-                const int col = ((k0 + k) * 32 + lane) * 8;
-                xv[k] = col < d ? *reinterpret_cast<const uint4 *>(xrow + col) : make_uint4(0u, 0u, 0u, 0u);
-            }
+            for (int g = 0; g < kQg; ++g) red4[warp][g] = m[g];
+        __syncthreads();
+        if (threadIdx.x < ng) {
+            float mm = red4[0][threadIdx.x];
 #pragma unroll
-            for (int k = 0; k < kV; ++k) {
-                const int col = ((k0 + k) * 32 + lane) * 8;
+            for (int w = 1; w < kPsWarps; ++w) mm = fmaxf(mm, red4[w][threadIdx.x]);
+            const float s = quant_scale(mm, act_clip, 127.0f);
+            xs_s[t0 + threadIdx.x] = s;
+            if (xs_out && blockIdx.x == 0) xs_out[t0 + threadIdx.x] = s;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int g = 0; g < kQg; ++g) {
+            if (g >= ng) break;
+            const float s = xs_s[t0 + g], inv = quant_inv_scale(s);
+#pragma unroll
+            for (int k = 0; k < kVt; ++k) {
+                const int col = (k * 256 + threadIdx.x) * 8;
                 if (col >= d) break;
                 float f[8];
-                unpack8_bf16(xv[k], f);
+                unpack8_bf16(xv[g][k], f);
                 uint32_t lo = 0, hi = 0;
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     lo |= uint32_t(quant_code_fast(f[e], s, inv, 127) & 0xff) << (8 * e);
                     hi |= uint32_t(quant_code_fast(f[e + 4], s, inv, 127) & 0xff) << (8 * e);
                 }
-                *reinterpret_cast<uint2 *>(xq_s + size_t(t) * dp + col) = make_uint2(lo, hi);
+                *reinterpret_cast<uint2 *>(xq_s + size_t(t0 + g) * dp + col) = make_uint2(lo, hi);
                 if (xq_out && blockIdx.x == 0)
-                    *reinterpret_cast<uint2 *>(xq_out + size_t(t) * d + col) = make_uint2(lo, hi);
+                    *reinterpret_cast<uint2 *>(xq_out + size_t(t0 + g) * d + col) = make_uint2(lo, hi);
             }
-        }
-        if (lane == 0) {
-            xs_s[t] = s;
-            if (xs_out && blockIdx.x == 0) xs_out[t] = s;
         }
     }
     __syncthreads();
