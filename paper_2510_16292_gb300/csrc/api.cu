@@ -294,9 +294,21 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
     prof_mark(stream, "begin");
     cudaError_t e;
     if (T <= kPsMaxTok && d <= 6144 && d % 256 == 0) {
-        e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
-                              xq_out, xs_out, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq, dst_pos,
-                              err, stream);
+        if (T < kPsSplitTok) {
+            e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
+                                  xq_out, xs_out, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
+                                  dst_pos, err, stream);
+            return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "projection launch");
+        }
+        // each row quantized once, the dot products on the tensor cores, the rows requantized in parallel
+        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream);
+        if (e == cudaSuccess)
+            e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
+                                  nullptr, nullptr, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
+                                  dst_pos, err, stream, xq, xs, false);
+        if (e == cudaSuccess)
+            e = launch_requant(c_hat, T, r, lat_bits, lat_clip, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
+                               dst_pos, err, stream);
         return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "projection launch");
     }
     if (W->codes_bf16 && gemm_tc_supported(d, r)) {

@@ -91,7 +91,12 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
                               const float *ws, int r, int lat_bits, float lat_clip, float *c_hat, int *counter,
                               int8_t *xq_out, float *xs_out, int32_t *acc_out, void *lat_codes, void *lat_scales,
                               const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
-                              cudaStream_t s);
+                              cudaStream_t s, const int8_t *xq_in = nullptr, const float *xs_in = nullptr,
+                              bool tail = true);
+// From this many tokens on, the decode projection runs as three kernels:
+// xquant (one CTA per token), proj_small on the given codes, requant (one CTA
+// per row); below it, proj_small quantizes and requantizes by itself.
+constexpr int kPsSplitTok = 4;
 
 // Exact int8 GEMM on the tensor cores (bf16 images of the codes, fp32 TMEM
 // accumulators drained to int32 every 1024 of K) + the fp32 dequantization.

@@ -58,9 +58,9 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                   int *__restrict__ counter, int8_t *__restrict__ xq_out, float *__restrict__ xs_out,
                   int32_t *__restrict__ acc_out, void *__restrict__ lat_codes, void *__restrict__ lat_scales,
                   CacheView dst, const int32_t *__restrict__ dst_seq, const int32_t *__restrict__ dst_pos,
-                  int *err) {
+                  int *err, const int8_t *__restrict__ xq_in, const float *__restrict__ xs_in, int tail) {
     extern __shared__ __align__(16) uint8_t smem[];
-    __shared__ __align__(8) uint64_t bar;
+    __shared__ __align__(8) uint64_t bar, bar_x;
     __shared__ float xs_s[kPsMaxTok];
     __shared__ float red[kPsWarps];
     __shared__ float red4[kPsWarps][4];
@@ -75,6 +75,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     prefetch_share_l2(w, size_t(r) * d, blockIdx.x, gridDim.x);
     if (threadIdx.x == 0) {
         mbar_init(&bar, 1);
+        mbar_init(&bar_x, 1);
         mbar_init_fence();
     }
     __syncthreads();
@@ -83,10 +84,19 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
         for (int i = 0; i < rows; ++i) bulk_g2s(w_s + size_t(i) * dp, w + size_t(j0 + i) * d, uint32_t(d), &bar);
     }
     pdl_wait();
-    // a1: per-token int8 quantization by the whole CTA, up to kQg tokens at a
-    // time: one round of loads, the per-token maxima reduced together
+    // a1: per-token int8 quantization.  Codes quantized by the previous kernel
+    // (xq_in): bulk copies into the padded rows.  Otherwise the whole CTA
+    // quantizes, up to kQg tokens at a time: one round of loads, the per-token
+    // maxima reduced together.
     constexpr int kQg = 4, kVt = kPsMaxD / 2048;    // tokens per round, 16-byte vectors per thread per token
-    for (int t0 = 0; t0 < T; t0 += kQg) {
+    if (xq_in) {
+        if (threadIdx.x == 0) {
+            mbar_arrive_expect_tx(&bar_x, uint32_t(T) * d);
+            for (int t = 0; t < T; ++t) bulk_g2s(xq_s + size_t(t) * dp, xq_in + size_t(t) * d, uint32_t(d), &bar_x);
+        }
+        if (threadIdx.x < T) xs_s[threadIdx.x] = xs_in[threadIdx.x];
+    }
+    for (int t0 = 0; t0 < T && !xq_in; t0 += kQg) {
         const int ng = min(kQg, T - t0);
         uint4 xv[kQg][kVt];
         float m[kQg];
@@ -148,6 +158,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     }
     __syncthreads();
     mbar_wait(&bar, 0, err);
+    if (xq_in) mbar_wait(&bar_x, 0, err);
     // a2 + first half of a3: exact int32 dot products, then the fp32 dequantization
     if (T >= kPsWarpTok) {
         // Tensor cores: the CTA's 16-token x 8-channel tile (m16n8k16, codes
@@ -214,6 +225,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
             }
         }
     }
+    if (!tail) return;                   // the rows are requantized by the next kernel
     // second half of a3 + a4: the last CTA requantizes every row of c_hat
     __threadfence();
     __syncthreads();
@@ -236,7 +248,7 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
                               const float *ws, int r, int lat_bits, float lat_clip, float *c_hat, int *counter,
                               int8_t *xq_out, float *xs_out, int32_t *acc_out, void *lat_codes, void *lat_scales,
                               const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
-                              cudaStream_t s) {
+                              cudaStream_t s, const int8_t *xq_in, const float *xs_in, bool tail) {
     CacheView dv{};
     if (dst) dv = *dst;
     // padded rows; the tensor-core path reuses the code rows for an [8][16][8] int32 reduction
@@ -245,7 +257,7 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
     if (e != cudaSuccess) return e;
     e = launch_pdl(proj_small_kernel, dim3((r + kPsWarps - 1) / kPsWarps), dim3(kPsWarps * 32), smem, s, X, T, d,
                    act_clip, wcodes, ws, r, lat_bits, lat_clip, c_hat, counter, xq_out, xs_out, acc_out, lat_codes,
-                   lat_scales, dv, dst_seq, dst_pos, err);
+                   lat_scales, dv, dst_seq, dst_pos, err, xq_in, xs_in, int(tail));
     prof_mark(s, "proj_small");
     return e;
 }
