@@ -304,9 +304,13 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
     const int B = c.B, r = c.r, H = a.H, dh = a.dh, d = H * dh;
     DecodeWs w;
     carve(B, a.max_seq_len, r, H, dh, static_cast<char *>(ws), &w);
-    cudaError_t e = launch_qproj(c, a.seq_len, a.U_q, d, w.q, w.qmax, B * H, err, s);
+    // the up-projection products on the tensor cores from 8 sequences on
+    const bool mma = decode_mma_supported(B, r, d, dh);
+    cudaError_t e = mma ? launch_qproj_mma(c, a.seq_len, a.U_q, d, w.q, w.qmax, B * H, err, s)
+                        : launch_qproj(c, a.seq_len, a.U_q, d, w.q, w.qmax, B * H, err, s);
     if (e != cudaSuccess) return e;
-    e = launch_qabsorb(w.q, a.U_k, B, r, d, H, dh, w.qt, w.qmax, err, s);
+    e = mma ? launch_qabsorb_mma(w.q, a.U_k, B, r, d, H, dh, w.qt, w.qmax, s)
+            : launch_qabsorb(w.q, a.U_k, B, r, d, H, dh, w.qt, w.qmax, err, s);
     if (e != cudaSuccess) return e;
 
     int chunk = chunk_tokens(a.max_seq_len);
@@ -349,6 +353,7 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
         if (e != cudaSuccess) return e;
         prof_mark(s, "attn_chunk");
     }
+    if (mma) return launch_combine_mma(a.seq_len, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v, a.O, s);
     return launch_combine_uv(a.seq_len, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v, a.O, err, s);
 }
 

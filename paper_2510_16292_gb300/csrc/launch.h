@@ -140,6 +140,15 @@ struct DecodeArgs {
 size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
 
 // a5 and a7/a8 for all B sequences of a step (decode_gemv.cu).
+// decode_mma.cu: tensor-core forms of the three products, for 8 or more sequences
+bool decode_mma_supported(int B, int r, int d, int dh);
+cudaError_t launch_qproj_mma(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
+                             unsigned *qmax, int n_qmax, int *err, cudaStream_t s);
+cudaError_t launch_qabsorb_mma(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
+                               unsigned *qmax, cudaStream_t s);
+cudaError_t launch_combine_mma(const int32_t *seq_len, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
+                               const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
+                               cudaStream_t s);
 cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
                          unsigned *qmax, int n_qmax, int *err, cudaStream_t s);
 cudaError_t launch_qabsorb(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,

@@ -193,6 +193,27 @@ def test_decode_batch_ragged_lengths(bits):
         assert_rows_close(o, np.stack([outs[b] for b in range(3)]), f"step {step}")
 
 
+@pytest.mark.parametrize("B,bits", [(9, 8), (17, 4)])
+def test_decode_large_batch_tensor_core_products(B, bits):
+    """From 8 sequences on, the up-projection products run on the tensor cores
+    (16 sequences per pass: B = 17 takes two passes); ragged lengths."""
+    base = synthetic.WORKLOADS["llava7b"]
+    wl = synthetic.Workload("batch", base.shape, B=B, n_image=0, n_text=160, decode_steps=2, lat_bits=bits)
+    inp = synthetic.gen_layer(wl, seed=21)
+    w = pipeline.prepare_weights(inp)
+    s = wl.shape
+    ref = pipeline.OracleLayer(s, w, B, wl.tmax, bits)
+    gpu = GpuLayer(s, w, B, wl.tmax, bits)
+    lens = [1 + (37 * b) % 160 for b in range(B)]
+    for b, n in enumerate(lens):
+        ref.prefill(b, inp.X_prefill[b][:n])
+        gpu.prefill(b, inp.X_prefill[b][:n])
+    for step in range(2):
+        _, outs = ref.decode_step(inp.X_decode[step])
+        o = gpu.decode_step(inp.X_decode[step]).cpu().numpy()
+        assert_rows_close(o, np.stack([outs[b] for b in range(B)]), f"step {step}")
+
+
 def test_decode_13b_heads_and_rank():
     """H = 40 (five head groups of 8), r = 2048, d = 5120."""
     base = synthetic.WORKLOADS["llava13b"]
