@@ -57,6 +57,9 @@ def parse():
     p.add_argument("--no-prefill13", action="store_true")
     p.add_argument("--workload", default=WORKLOAD, choices=sorted(synthetic.WORKLOADS))
     p.add_argument("--decode-steps", type=int, default=0, help="override the workload's decode steps")
+    p.add_argument("--sweep", choices=["quick", "full"], default=None,
+                   help="sweep the 7B-shaped layer over rank, cached length, batch and cache precision (one JSON "
+                        "line per point) instead of the benchmark")
     p.add_argument("--l2", default="rotate", choices=["rotate", "flush"],
                    help="cold-L2 method: rotate through copies of the layer larger than L2 together, or flush "
                         "L2 before every sub-step")
@@ -648,8 +651,109 @@ def run_reference(args, rank, world):
     print(json.dumps(out), flush=True)
 
 
+# ---------------------------------------------------------------------------
+# sweep over the 7B-shaped layer (rank x cached length x batch x cache precision)
+# ---------------------------------------------------------------------------
+SWEEP_FULL = dict(r=(1024, 1536, 2048, 3072), L=(1024, 4096, 16384, 32768), B=(1, 8, 32, 64), bits=(8, 4))
+SWEEP_QUICK = dict(r=(1536, 3072), L=(1024, 32768), B=(1, 64), bits=(8, 4))
+
+
+def run_sweep(args):
+    """One JSON line per point: decode tokens/s of one layer and the fraction
+    of the step's HBM roofline (bytes a decode step must read: the latent
+    cache, the three up-projections and W_d).  The cache of each point is
+    filled with seeded codes and scales as if prefilled (the sweep measures
+    decode); weights are seeded Gaussians of the recipe's scales.  Cold L2:
+    the points' layers rotate as in the main benchmark when one layer's
+    decode bytes are below twice the L2."""
+    import torch
+    import paper_2510_16292_gb300 as q
+    dev = torch.device("cuda", torch.cuda.current_device())
+    hbm, _, peak_kind = peaks()
+    grid = SWEEP_FULL if args.sweep == "full" else SWEEP_QUICK
+    d, H, dh = 4096, 32, 128
+    g = torch.Generator(device=dev)
+    g.manual_seed(2510)
+    for r in grid["r"]:
+        for bits in grid["bits"]:
+            for B in grid["B"]:
+                for L in grid["L"]:
+                    tok = (r + 4) if bits == 8 else (r // 2 + 2 * (r // 128))
+                    layer_bytes = 3 * r * d * 2 + r * d + B * L * tok
+                    K = 1 if layer_bytes >= 2 * L2_BYTES else max(2, -(-2 * L2_BYTES // layer_bytes))
+                    layers = []
+                    for _ in range(K):
+                        Wd = torch.randn((d, r), generator=g, device=dev) / math.sqrt(d)
+                        W = q.qsvd_quantize_weight(Wd)
+                        del Wd
+                        U = [(torch.randn((r, d), generator=g, device=dev) / math.sqrt(r)).to(torch.bfloat16)
+                             for _ in range(3)]
+                        cache = q.LatentCache.empty(B, L + 1, r, bits, dev)
+                        if bits == 8:
+                            cache.codes.copy_(torch.randint(-127, 128, cache.codes.shape, generator=g, device=dev,
+                                                            dtype=torch.int8))
+                            cache.scales.copy_(torch.rand(cache.scales.shape, generator=g, device=dev) * 0.02 + 0.01)
+                        else:
+                            cache.codes.copy_(torch.randint(0, 256, cache.codes.shape, generator=g, device=dev,
+                                                            dtype=torch.uint8))
+                            cache.scales.copy_((torch.rand(cache.scales.shape, generator=g, device=dev) * 0.2
+                                                + 0.1).half())
+                        X = torch.randn((B, d), generator=g, device=dev).to(torch.bfloat16)
+                        O = torch.empty((B, d), dtype=torch.float32, device=dev)
+                        layers.append((W, U, cache, X, O))
+                    seq = torch.arange(B, dtype=torch.int32, device=dev)
+                    pos = torch.full((B,), L, dtype=torch.int32, device=dev)
+                    lens = torch.full((B,), L + 1, dtype=torch.int32, device=dev)
+                    wsp = torch.zeros(q.qsvd_project_workspace_bytes(B, d, r), dtype=torch.uint8, device=dev)
+                    wsd = torch.zeros(q.qsvd_decode_workspace_bytes(B, L + 1, r, H, dh), dtype=torch.uint8,
+                                      device=dev)
+                    st = torch.cuda.Stream()
+                    st.wait_stream(torch.cuda.current_stream())      # inputs and workspaces were filled there
+                    steps = 4
+                    E = lambda: torch.cuda.Event(enable_timing=True, external=True)  # noqa: E731
+                    evs = [(E(), E()) for _ in range(steps)]
+
+                    def one(k):
+                        W, U, cache, X, O = layers[k]
+                        q.qsvd_latent_project(W, X, 1.0, bits, 1.0, dst=cache, dst_seq=seq, dst_pos=pos,
+                                              workspace=wsp, stream=st)
+                        q.qsvd_latent_decode_attn(cache, lens, L + 1, *U, H, dh, O, workspace=wsd, stream=st)
+
+                    with torch.cuda.stream(st):
+                        for k in range(K):
+                            one(k)
+                    torch.cuda.synchronize()
+                    gr = torch.cuda.CUDAGraph()
+                    with torch.cuda.graph(gr, stream=st):
+                        for a, b in evs:
+                            a.record(st)
+                            for k in range(K):
+                                one(k)
+                            b.record(st)
+                    for _ in range(3):
+                        gr.replay()
+                    torch.cuda.synchronize()
+                    ts = []
+                    for _ in range(3):
+                        gr.replay()
+                        torch.cuda.synchronize()
+                        ts += [a.elapsed_time(b) * 1e-3 / K for a, b in evs]
+                    q.qsvd_check()
+                    t = statistics.median(ts)
+                    roof = layer_bytes / (hbm * 1e9)
+                    print(json.dumps({"sweep": {"r": r, "L": L, "B": B, "bits": bits, "layer_copies": K},
+                                      "decode_tokens_s": round(B / t, 1), "us_per_layer_step": round(t * 1e6, 2),
+                                      "step_roofline_us": round(roof * 1e6, 2), "roofline_frac": round(roof / t, 4),
+                                      "peak_gbs": hbm, "peak_kind": peak_kind}), flush=True)
+                    del layers, wsd, wsp, gr
+                    torch.cuda.empty_cache()
+
+
 def main():
     args = parse()
+    if args.sweep:
+        run_sweep(args)
+        return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

@@ -251,11 +251,11 @@ int qsvd_set_project_epilogue(int32_t mode);
  * not part of the paper's method; process-wide, not thread-safe):
  *   0  automatic (default): the warp-level tensor-core kernel when
  *      B * max_seq_len <= 16384 or the tcgen05 kernel cannot take the shape,
- *      else the tcgen05 kernel (the warp-level kernel needs
- *      max_seq_len <= 4096; beyond that, the CUDA-core kernels);
+ *      else the tcgen05 kernel (the warp-level kernel needs r <= 3072;
+ *      beyond that, the CUDA-core kernels);
  *   1  always the CUDA-core kernels;
  *   2  the tcgen05 kernel whenever the shape allows it;
- *   3  the warp-level tensor-core kernel whenever max_seq_len <= 4096.
+ *   3  the warp-level tensor-core kernel whenever r <= 3072.
  * The tcgen05 kernel needs r % 256 == 0, r <= 1536, H <= 32 and
  * (r / 256) * ceil16(H) <= 192; other shapes use the CUDA-core kernels.  All
  * give the same results up to floating-point rounding.

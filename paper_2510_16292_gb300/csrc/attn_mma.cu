@@ -1,21 +1,24 @@
-// Decode attention over the latent cache for small batch x length (Eq. 5
-// with W^u_k absorbed into the query; W^u_v is applied by combine_uv_kernel),
-// on the warp-level tensor-core MMA (mma.sync m16n8k16, fp16 in, fp32
-// accumulate).  A CTA takes one sequence, one range of TS tokens (16, 32 or
-// 64) and 8 heads; it is not pipelined: at this size a short dependency chain
-// matters more than throughput.
+// Decode attention over the latent cache for small batch x length, and for
+// shapes the tcgen05 kernel does not take (Eq. 5 with W^u_k absorbed into the
+// query; W^u_v is applied by the combine kernel), on the warp-level
+// tensor-core MMA (mma.sync m16n8k16, fp16 in, fp32 accumulate).  A CTA takes
+// one sequence, 8 heads and a range of n_sub sub-tiles of TS tokens (16, 32
+// or 64), walked one after another with a running softmax:
 //
+//   0. the fp16 query block Q~ [8 heads][r] (each head scaled by a power of
+//      two so that its largest entry is just below 2^14) is built from q~.
+//   per sub-tile:
 //   1. the TS cache rows (int8 / packed int4, padded rows) and the scales go
-//      to shared memory with 16-byte asynchronous copies; the fp16 query
-//      block Q~ [8 heads][r] (each head scaled by a power of two so that its
-//      largest entry is just below 2^14) is built from q~.
+//      to shared memory with 16-byte asynchronous copies.
 //   2. scores S[t, h] = sum_ch C[t, ch] Q~[h, ch]: each warp takes a range of
 //      16-channel steps, the warps' partial S are added in shared memory.
 //      int8: the token scale multiplies the row; int4: code * group-scale is
 //      accumulated group by group.
-//   3. per head: max over the CTA's tokens, p = 2^(logit - m), l = sum p.
-//   4. O^T[ch, h] = sum_t C[t, ch] P[t, h] over the CTA's tokens (M = 16
-//      channels per MMA, K = tokens), the token / group scale folded into P.
+//   3. per head: the running maximum m and sum l are updated (o_lat is scaled
+//      by 2^(m_old - m_new)), p = 2^(logit - m).
+//   4. O^T[ch, h] += sum_t C[t, ch] P[t, h] (M = 16 channels per MMA, K =
+//      tokens), the token / group scale folded into P; the accumulators of a
+//      warp's channel blocks stay in registers across the sub-tiles.
 //   5. the CTA's (m, l, o_lat) are written as one softmax partial.
 //
 // Within one MMA the 16 reduction indices are used in the order
@@ -43,7 +46,7 @@ struct Params {
     const int32_t *seq_len;
     const float *qt;              // [B, H, r]
     const unsigned *qmax;         // [B, H] bits of max |q~|
-    int H, TS, n_split;
+    int H, TS, n_sub, n_split;     // sub-tile tokens, sub-tiles per split, splits per sequence
     float softmax_scale;
     float *pm, *pl, *po;          // [B, n_split, H] / [B, n_split, H, r]
     int *err;
@@ -83,7 +86,7 @@ __device__ __forceinline__ uint32_t i4x4_to_i8x4(uint32_t x) {
 
 }  // namespace am
 
-template <int BITS>
+template <int BITS, int MB>
 __global__ void __launch_bounds__(am::kThreads)
 attn_mma_kernel(const am::Params p) {
     using namespace am;
@@ -92,6 +95,7 @@ attn_mma_kernel(const am::Params p) {
     __shared__ float tsc_s[kMaxTS];                 // int8 token scales
     __shared__ float qfac_s[kHG];
     __shared__ float m_s[kHG];
+    __shared__ float alpha_s[kHG];                  // o_lat rescale of the current sub-tile
     const CacheView &c = p.c;
     const int r = c.r, TS = p.TS, H = p.H;
     const int split = blockIdx.x, b = blockIdx.y, h0 = blockIdx.z * kHG;
@@ -106,21 +110,22 @@ attn_mma_kernel(const am::Params p) {
     const int pstride = TS + 8;
     pdl_trigger();
     const int L = p.seq_len[b];                                    // an input: no kernel writes it
-    const int t_begin = split * TS;
-    if (L < 1 || L > c.Tmax || t_begin >= L) return;               // invalid lengths are flagged by qproj_kernel
-    const int n = min(TS, L - t_begin);
-    const size_t slot0 = size_t(b) * c.Tmax + t_begin;
+    const int t_split = split * TS * p.n_sub;
+    if (L < 1 || L > c.Tmax || t_split >= L) return;               // invalid lengths are flagged by qproj_kernel
+    const int n_sub = min(p.n_sub, (L - t_split + TS - 1) / TS);   // sub-tiles of this CTA
     if (threadIdx.x == 0) {
         // L2 prefetch of the split's cache rows while the producer grid finishes
         // (L2 is the point of coherence, so a row written meanwhile is never
-        // seen stale: the shared-memory copies below come after the wait)
-        prefetch_l2_bulk(static_cast<const uint8_t *>(c.codes) + slot0 * row_bytes, uint32_t(n) * row_bytes);
+        // seen stale: the shared-memory copies come after the wait)
+        for (int sb = 0; sb < n_sub; ++sb) {
+            const int t0 = t_split + sb * TS;
+            prefetch_l2_bulk(static_cast<const uint8_t *>(c.codes) + (size_t(b) * c.Tmax + t0) * row_bytes,
+                             uint32_t(min(TS, L - t0)) * row_bytes);
+        }
     }
     pdl_wait();
 
-    // ---- 1. cache rows (zero beyond n), scales, query block.  The q~ loads are
-    // issued first and the cache rows copied asynchronously meanwhile; the
-    // per-head scale is applied once both the loads and qmax are in.
+    // ---- 0. query block: q~ loads first, the per-head scale applied once qmax is in
     {
         constexpr int kQL = 16;                                    // float4 per thread per pass (r <= 2048: one pass)
         const int nq4 = kHG * (r / 4);
@@ -132,22 +137,6 @@ attn_mma_kernel(const am::Params p) {
             v[u] = (i < nq4 && h0 + hl < H) ? reinterpret_cast<const float4 *>(p.qt + (size_t(b) * H + h0 + hl) * r)[q4]
                                            : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        const int cpr = row_bytes / 16;                            // 16-byte chunks per row
-        for (int i = threadIdx.x; i < TS * cpr; i += kThreads) {
-            const int t = i / cpr, k = i - t * cpr;
-            uint8_t *dst = tile + size_t(t) * rstride + k * 16;
-            if (t < n) cp_async16(dst, static_cast<const uint8_t *>(c.codes) + (slot0 + t) * row_bytes + k * 16);
-            else *reinterpret_cast<uint4 *>(dst) = make_uint4(0u, 0u, 0u, 0u);
-        }
-        if (BITS == 8) {
-            if (threadIdx.x < TS)
-                tsc_s[threadIdx.x] = threadIdx.x < n ? static_cast<const float *>(c.scales)[slot0 + threadIdx.x] : 0.0f;
-        } else {
-            for (int i = threadIdx.x; i < TS * (r / 128); i += kThreads) {
-                const int t = i / (r / 128);
-                gsc[i] = t < n ? static_cast<const __half *>(c.scales)[slot0 * (r / 128) + i] : __float2half(0.0f);
-            }
-        }
         if (threadIdx.x < kHG) {
             const int h = h0 + threadIdx.x;
             int e = 0;
@@ -157,7 +146,7 @@ attn_mma_kernel(const am::Params p) {
             }
             // scores -> logits in log2 units: undo the query scale, times softmax_scale * log2(e)
             qfac_s[threadIdx.x] = exp2f(float(e - 14)) * p.softmax_scale * 1.4426950408889634f;
-            m_s[threadIdx.x] = exp2f(float(14 - e));               // the query scale (temporary)
+            m_s[threadIdx.x] = exp2f(float(14 - e));               // the query scale
         }
         __syncthreads();
         auto store_q = [&](int i, const float4 &x) {
@@ -179,184 +168,224 @@ attn_mma_kernel(const am::Params p) {
                                          : make_float4(0.f, 0.f, 0.f, 0.f);
             store_q(i, x);
         }
-        cp_async_wait_all();
-        __syncthreads();
     }
 
-    // ---- 2. scores: warp w takes 16-channel steps w, w+8, ...; MT m-blocks of 16 tokens
     const int MT = TS / 16, nks = r / 16;
-    {
-        float acc[kMaxTS / 16][4];
+    // running softmax state of head `warp` (warps < kHG), the same in every lane
+    float m_run = -INFINITY, l_run = 0.0f;
+    // o_lat^T accumulators: channel block mb = warp + 8 j, fragment (channels g, g+8; heads 2cq, 2cq+1)
+    float o[MB][4];
 #pragma unroll
-        for (int m = 0; m < kMaxTS / 16; ++m) acc[m][0] = acc[m][1] = acc[m][2] = acc[m][3] = 0.0f;
-        float gacc[kMaxTS / 16][4];                    // int4: current group's sums
+    for (int j = 0; j < MB; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.0f;
+
+    for (int sb = 0; sb < n_sub; ++sb) {
+        const int t_begin = t_split + sb * TS;
+        const int n = min(TS, L - t_begin);
+        const size_t slot0 = size_t(b) * c.Tmax + t_begin;
+        __syncthreads();                                           // the previous sub-tile's readers are done
+        // ---- 1. cache rows (zero beyond n) and scales
+        {
+            const int cpr = row_bytes / 16;                        // 16-byte chunks per row
+            for (int i = threadIdx.x; i < TS * cpr; i += kThreads) {
+                const int t = i / cpr, k = i - t * cpr;
+                uint8_t *dst = tile + size_t(t) * rstride + k * 16;
+                if (t < n) cp_async16(dst, static_cast<const uint8_t *>(c.codes) + (slot0 + t) * row_bytes + k * 16);
+                else *reinterpret_cast<uint4 *>(dst) = make_uint4(0u, 0u, 0u, 0u);
+            }
+            if (BITS == 8) {
+                if (threadIdx.x < TS)
+                    tsc_s[threadIdx.x] = threadIdx.x < n ? static_cast<const float *>(c.scales)[slot0 + threadIdx.x] : 0.0f;
+            } else {
+                for (int i = threadIdx.x; i < TS * (r / 128); i += kThreads) {
+                    const int t = i / (r / 128);
+                    gsc[i] = t < n ? static_cast<const __half *>(c.scales)[slot0 * (r / 128) + i] : __float2half(0.0f);
+                }
+            }
+            cp_async_wait_all();
+            __syncthreads();
+        }
+
+        // ---- 2. scores: warp w takes 16-channel steps w, w+8, ...; MT m-blocks of 16 tokens
+        {
+            float acc[kMaxTS / 16][4];
 #pragma unroll
-        for (int m = 0; m < kMaxTS / 16; ++m) gacc[m][0] = gacc[m][1] = gacc[m][2] = gacc[m][3] = 0.0f;
-        int cur_grp = -1;
-        for (int ks = warp; ks < nks; ks += 8) {
-            const int k0 = ks * 16;
-            // B: Q~[head g][channels k0 + 4 cq .. + 3]
-            const uint2 bw = *reinterpret_cast<const uint2 *>(qs + size_t(g) * qstride + k0 + 4 * cq);
-            if (BITS == 4) {
-                const int grp = k0 / 128;
-                if (grp != cur_grp) {
-                    if (cur_grp >= 0) {
+            for (int m = 0; m < kMaxTS / 16; ++m) acc[m][0] = acc[m][1] = acc[m][2] = acc[m][3] = 0.0f;
+            float gacc[kMaxTS / 16][4];                    // int4: current group's sums; int8: second chain
 #pragma unroll
-                        for (int m = 0; m < kMaxTS / 16; ++m) {
-                            if (m >= MT) break;
-                            const float s0 = __half2float(gsc[(m * 16 + g) * (r / 128) + cur_grp]);
-                            const float s1 = __half2float(gsc[(m * 16 + g + 8) * (r / 128) + cur_grp]);
-                            acc[m][0] = fmaf(s0, gacc[m][0], acc[m][0]); acc[m][1] = fmaf(s0, gacc[m][1], acc[m][1]);
-                            acc[m][2] = fmaf(s1, gacc[m][2], acc[m][2]); acc[m][3] = fmaf(s1, gacc[m][3], acc[m][3]);
-                            gacc[m][0] = gacc[m][1] = gacc[m][2] = gacc[m][3] = 0.0f;
+            for (int m = 0; m < kMaxTS / 16; ++m) gacc[m][0] = gacc[m][1] = gacc[m][2] = gacc[m][3] = 0.0f;
+            int cur_grp = -1;
+            for (int ks = warp; ks < nks; ks += 8) {
+                const int k0 = ks * 16;
+                // B: Q~[head g][channels k0 + 4 cq .. + 3]
+                const uint2 bw = *reinterpret_cast<const uint2 *>(qs + size_t(g) * qstride + k0 + 4 * cq);
+                if (BITS == 4) {
+                    const int grp = k0 / 128;
+                    if (grp != cur_grp) {
+                        if (cur_grp >= 0) {
+#pragma unroll
+                            for (int m = 0; m < kMaxTS / 16; ++m) {
+                                if (m >= MT) break;
+                                const float s0 = __half2float(gsc[(m * 16 + g) * (r / 128) + cur_grp]);
+                                const float s1 = __half2float(gsc[(m * 16 + g + 8) * (r / 128) + cur_grp]);
+                                acc[m][0] = fmaf(s0, gacc[m][0], acc[m][0]); acc[m][1] = fmaf(s0, gacc[m][1], acc[m][1]);
+                                acc[m][2] = fmaf(s1, gacc[m][2], acc[m][2]); acc[m][3] = fmaf(s1, gacc[m][3], acc[m][3]);
+                                gacc[m][0] = gacc[m][1] = gacc[m][2] = gacc[m][3] = 0.0f;
+                            }
                         }
+                        cur_grp = grp;
                     }
-                    cur_grp = grp;
                 }
-            }
 #pragma unroll
-            for (int m = 0; m < kMaxTS / 16; ++m) {
-                if (m >= MT) break;
-                uint32_t a0, a1, a2, a3;
-                if (BITS == 8) {
-                    const uint32_t w0 = *reinterpret_cast<const uint32_t *>(tile + size_t(m * 16 + g) * rstride + k0 + 4 * cq);
-                    const uint32_t w1 = *reinterpret_cast<const uint32_t *>(tile + size_t(m * 16 + g + 8) * rstride + k0 + 4 * cq);
-                    i8x4_h2(w0, a0, a2);
-                    i8x4_h2(w1, a1, a3);
-                    mma16816((ks >> 3) & 1 ? gacc[m] : acc[m], a0, a1, a2, a3, bw.x, bw.y);   // two chains
-                } else {
-                    const uint32_t x0 = *reinterpret_cast<const uint16_t *>(tile + size_t(m * 16 + g) * rstride + (k0 + 4 * cq) / 2);
-                    const uint32_t x1 = *reinterpret_cast<const uint16_t *>(tile + size_t(m * 16 + g + 8) * rstride + (k0 + 4 * cq) / 2);
-                    i8x4_h2(i4x4_to_i8x4(x0), a0, a2);
-                    i8x4_h2(i4x4_to_i8x4(x1), a1, a3);
-                    mma16816(gacc[m], a0, a1, a2, a3, bw.x, bw.y);
-                }
-            }
-        }
-        if (BITS == 8) {                           // add the second chain
-#pragma unroll
-            for (int m = 0; m < kMaxTS / 16; ++m) {
-                acc[m][0] += gacc[m][0]; acc[m][1] += gacc[m][1]; acc[m][2] += gacc[m][2]; acc[m][3] += gacc[m][3];
-            }
-        }
-        if (BITS == 4 && cur_grp >= 0) {
-#pragma unroll
-            for (int m = 0; m < kMaxTS / 16; ++m) {
-                if (m >= MT) break;
-                const float s0 = __half2float(gsc[(m * 16 + g) * (r / 128) + cur_grp]);
-                const float s1 = __half2float(gsc[(m * 16 + g + 8) * (r / 128) + cur_grp]);
-                acc[m][0] = fmaf(s0, gacc[m][0], acc[m][0]); acc[m][1] = fmaf(s0, gacc[m][1], acc[m][1]);
-                acc[m][2] = fmaf(s1, gacc[m][2], acc[m][2]); acc[m][3] = fmaf(s1, gacc[m][3], acc[m][3]);
-            }
-        }
-#pragma unroll
-        for (int m = 0; m < kMaxTS / 16; ++m) {
-            if (m >= MT) break;
-            sred[warp][m * 16 + g][2 * cq] = acc[m][0];
-            sred[warp][m * 16 + g][2 * cq + 1] = acc[m][1];
-            sred[warp][m * 16 + g + 8][2 * cq] = acc[m][2];
-            sred[warp][m * 16 + g + 8][2 * cq + 1] = acc[m][3];
-        }
-    }
-    __syncthreads();
-
-    // ---- 3. softmax per head over the CTA's tokens: thread (head hl, token t) pairs, a warp per head
-    if (warp < kHG) {
-        const int hl = warp, h = h0 + hl;
-        float lg[kMaxTS / 32];
-        float mx = -INFINITY;
-#pragma unroll
-        for (int u = 0; u < kMaxTS / 32; ++u) {
-            const int t = lane + 32 * u;
-            float v = -INFINITY;
-            if (t < n && h < H) {
-                float sacc = 0.0f;
-#pragma unroll
-                for (int w = 0; w < 8; ++w) sacc += sred[w][t][hl];
-                v = sacc * qfac_s[hl] * (BITS == 8 ? tsc_s[t] : 1.0f);
-            }
-            lg[u] = v;
-            mx = fmaxf(mx, v);
-        }
-        mx = warp_max(mx);
-        float l = 0.0f;
-#pragma unroll
-        for (int u = 0; u < kMaxTS / 32; ++u) {
-            const int t = lane + 32 * u;
-            const float pe = (t < n && h < H) ? exp2f(lg[u] - mx) : 0.0f;
-            l += pe;
-            if (t < TS) ps[size_t(hl) * pstride + t] = __float2half_rn(BITS == 8 ? pe * tsc_s[t] : pe);
-        }
-        l = warp_sum(l);
-        if (lane == 0 && h < H) {
-            const size_t pb = (size_t(b) * p.n_split + split) * H + h;
-            p.pm[pb] = mx * 0.6931471805599453f;        // natural-log units
-            p.pl[pb] = l;
-        }
-    }
-    __syncthreads();
-
-    // ---- 4. O^T[ch, h] = sum_t C[t, ch] P[t, h]: warp w takes 16-channel blocks
-    // w, w+8, ...; four of them at a time (independent accumulators)
-    for (int mb0 = warp; mb0 < nks; mb0 += 32) {
-        float d[4][4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) d[u][0] = d[u][1] = d[u][2] = d[u][3] = 0.0f;
-        for (int kt = 0; kt < MT; ++kt) {
-            const int t0 = kt * 16 + 4 * cq;
-            // B: P[head g][tokens t0 .. t0 + 3]
-            const uint2 pw = *reinterpret_cast<const uint2 *>(ps + size_t(g) * pstride + t0);
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int mb = mb0 + 8 * u;
-                if (mb >= nks) break;
-                const int ch0 = mb * 16;
-                // A: channels ch0 + g, ch0 + g + 8; tokens t0 .. t0 + 3
-                uint32_t wlo = 0, whi = 0;
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const uint8_t *rowp = tile + size_t(t0 + e) * rstride;
-                    uint32_t blo, bhi;
+                for (int m = 0; m < kMaxTS / 16; ++m) {
+                    if (m >= MT) break;
+                    uint32_t a0, a1, a2, a3;
                     if (BITS == 8) {
-                        blo = rowp[ch0 + g];
-                        bhi = rowp[ch0 + g + 8];
+                        const uint32_t w0 = *reinterpret_cast<const uint32_t *>(tile + size_t(m * 16 + g) * rstride + k0 + 4 * cq);
+                        const uint32_t w1 = *reinterpret_cast<const uint32_t *>(tile + size_t(m * 16 + g + 8) * rstride + k0 + 4 * cq);
+                        i8x4_h2(w0, a0, a2);
+                        i8x4_h2(w1, a1, a3);
+                        mma16816((ks >> 3) & 1 ? gacc[m] : acc[m], a0, a1, a2, a3, bw.x, bw.y);   // two chains
                     } else {
-                        const uint32_t x0 = rowp[(ch0 + g) >> 1], x1 = rowp[(ch0 + g + 8) >> 1];
-                        const int sh = ((ch0 + g) & 1) * 4;
-                        blo = uint32_t((((int(x0 >> sh) & 0xf) ^ 8) - 8) & 0xff);
-                        bhi = uint32_t((((int(x1 >> sh) & 0xf) ^ 8) - 8) & 0xff);
+                        const uint32_t x0 = *reinterpret_cast<const uint16_t *>(tile + size_t(m * 16 + g) * rstride + (k0 + 4 * cq) / 2);
+                        const uint32_t x1 = *reinterpret_cast<const uint16_t *>(tile + size_t(m * 16 + g + 8) * rstride + (k0 + 4 * cq) / 2);
+                        i8x4_h2(i4x4_to_i8x4(x0), a0, a2);
+                        i8x4_h2(i4x4_to_i8x4(x1), a1, a3);
+                        mma16816(gacc[m], a0, a1, a2, a3, bw.x, bw.y);
                     }
-                    wlo |= blo << (8 * e);
-                    whi |= bhi << (8 * e);
                 }
-                uint32_t a0, a1, a2, a3;
-                i8x4_h2(wlo, a0, a2);
-                i8x4_h2(whi, a1, a3);
-                uint2 bw = pw;
-                if (BITS == 4) {                    // int4: times the token's group scale
-                    const int grp = ch0 / 128;
-                    const __half2 s01 = __halves2half2(gsc[(t0 + 0) * (r / 128) + grp], gsc[(t0 + 1) * (r / 128) + grp]);
-                    const __half2 s23 = __halves2half2(gsc[(t0 + 2) * (r / 128) + grp], gsc[(t0 + 3) * (r / 128) + grp]);
-                    const __half2 p01 = __hmul2(*reinterpret_cast<const __half2 *>(&pw.x), s01);
-                    const __half2 p23 = __hmul2(*reinterpret_cast<const __half2 *>(&pw.y), s23);
-                    bw.x = *reinterpret_cast<const uint32_t *>(&p01);
-                    bw.y = *reinterpret_cast<const uint32_t *>(&p23);
+            }
+            if (BITS == 8) {                           // add the second chain
+#pragma unroll
+                for (int m = 0; m < kMaxTS / 16; ++m) {
+                    acc[m][0] += gacc[m][0]; acc[m][1] += gacc[m][1]; acc[m][2] += gacc[m][2]; acc[m][3] += gacc[m][3];
                 }
-                mma16816(d[u], a0, a1, a2, a3, bw.x, bw.y);
+            }
+            if (BITS == 4 && cur_grp >= 0) {
+#pragma unroll
+                for (int m = 0; m < kMaxTS / 16; ++m) {
+                    if (m >= MT) break;
+                    const float s0 = __half2float(gsc[(m * 16 + g) * (r / 128) + cur_grp]);
+                    const float s1 = __half2float(gsc[(m * 16 + g + 8) * (r / 128) + cur_grp]);
+                    acc[m][0] = fmaf(s0, gacc[m][0], acc[m][0]); acc[m][1] = fmaf(s0, gacc[m][1], acc[m][1]);
+                    acc[m][2] = fmaf(s1, gacc[m][2], acc[m][2]); acc[m][3] = fmaf(s1, gacc[m][3], acc[m][3]);
+                }
+            }
+#pragma unroll
+            for (int m = 0; m < kMaxTS / 16; ++m) {
+                if (m >= MT) break;
+                sred[warp][m * 16 + g][2 * cq] = acc[m][0];
+                sred[warp][m * 16 + g][2 * cq + 1] = acc[m][1];
+                sred[warp][m * 16 + g + 8][2 * cq] = acc[m][2];
+                sred[warp][m * 16 + g + 8][2 * cq + 1] = acc[m][3];
             }
         }
-        // D: channels ch0 + g (+8), heads 2 cq, 2 cq + 1
-        const size_t pb = (size_t(b) * p.n_split + split) * H + h0;
+        __syncthreads();
+
+        // ---- 3. running softmax per head: a warp per head, thread per token
+        if (warp < kHG) {
+            const int hl = warp, h = h0 + hl;
+            float lg[kMaxTS / 32];
+            float mx = -INFINITY;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int mb = mb0 + 8 * u;
-            if (mb >= nks) break;
+            for (int u = 0; u < kMaxTS / 32; ++u) {
+                const int t = lane + 32 * u;
+                float v = -INFINITY;
+                if (t < n && h < H) {
+                    float sacc = 0.0f;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int hl = 2 * cq + (e & 1), ch = mb * 16 + g + (e >> 1) * 8;
-                if (h0 + hl < H) p.po[(pb + hl) * r + ch] = d[u][e];
+                    for (int w = 0; w < 8; ++w) sacc += sred[w][t][hl];
+                    v = sacc * qfac_s[hl] * (BITS == 8 ? tsc_s[t] : 1.0f);
+                }
+                lg[u] = v;
+                mx = fmaxf(mx, v);
+            }
+            mx = warp_max(mx);
+            const float m_new = fmaxf(m_run, mx);
+            const float alpha = (h < H && m_run != -INFINITY) ? exp2f(m_run - m_new) : (h < H ? 0.0f : 1.0f);
+            float l = 0.0f;
+#pragma unroll
+            for (int u = 0; u < kMaxTS / 32; ++u) {
+                const int t = lane + 32 * u;
+                const float pe = (t < n && h < H) ? exp2f(lg[u] - m_new) : 0.0f;
+                l += pe;
+                if (t < TS) ps[size_t(hl) * pstride + t] = __float2half_rn(BITS == 8 ? pe * tsc_s[t] : pe);
+            }
+            l = warp_sum(l);
+            l_run = l_run * alpha + l;
+            m_run = h < H ? m_new : m_run;
+            if (lane == 0) alpha_s[hl] = alpha;
+        }
+        __syncthreads();
+
+        // ---- 4. O^T[ch, h] += sum_t C[t, ch] P[t, h]: warp w, channel blocks w + 8 j
+        {
+            const float al0 = alpha_s[2 * cq], al1 = alpha_s[2 * cq + 1];
+#pragma unroll
+            for (int j = 0; j < MB; ++j) {
+                o[j][0] *= al0; o[j][1] *= al1; o[j][2] *= al0; o[j][3] *= al1;
+            }
+            for (int kt = 0; kt < MT; ++kt) {
+                const int t0 = kt * 16 + 4 * cq;
+                // B: P[head g][tokens t0 .. t0 + 3]
+                const uint2 pw = *reinterpret_cast<const uint2 *>(ps + size_t(g) * pstride + t0);
+                const uint8_t *row0 = tile + size_t(t0) * rstride;
+#pragma unroll
+                for (int j = 0; j < MB; ++j) {
+                    const int mb = warp + 8 * j;
+                    if (mb >= nks) break;
+                    const int ch0 = mb * 16;
+                    // A: channels ch0 + g, ch0 + g + 8; tokens t0 .. t0 + 3
+                    uint32_t wlo = 0, whi = 0;
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const uint8_t *rowp = row0 + size_t(e) * rstride;
+                        uint32_t blo, bhi;
+                        if (BITS == 8) {
+                            blo = rowp[ch0 + g];
+                            bhi = rowp[ch0 + g + 8];
+                        } else {
+                            const uint32_t x0 = rowp[(ch0 + g) >> 1], x1 = rowp[(ch0 + g + 8) >> 1];
+                            const int sh = ((ch0 + g) & 1) * 4;
+                            blo = uint32_t((((int(x0 >> sh) & 0xf) ^ 8) - 8) & 0xff);
+                            bhi = uint32_t((((int(x1 >> sh) & 0xf) ^ 8) - 8) & 0xff);
+                        }
+                        wlo |= blo << (8 * e);
+                        whi |= bhi << (8 * e);
+                    }
+                    uint32_t a0, a1, a2, a3;
+                    i8x4_h2(wlo, a0, a2);
+                    i8x4_h2(whi, a1, a3);
+                    uint2 bw = pw;
+                    if (BITS == 4) {                    // int4: times the token's group scale
+                        const int grp = ch0 / 128;
+                        const __half2 s01 = __halves2half2(gsc[(t0 + 0) * (r / 128) + grp], gsc[(t0 + 1) * (r / 128) + grp]);
+                        const __half2 s23 = __halves2half2(gsc[(t0 + 2) * (r / 128) + grp], gsc[(t0 + 3) * (r / 128) + grp]);
+                        const __half2 p01 = __hmul2(*reinterpret_cast<const __half2 *>(&pw.x), s01);
+                        const __half2 p23 = __hmul2(*reinterpret_cast<const __half2 *>(&pw.y), s23);
+                        bw.x = *reinterpret_cast<const uint32_t *>(&p01);
+                        bw.y = *reinterpret_cast<const uint32_t *>(&p23);
+                    }
+                    mma16816(o[j], a0, a1, a2, a3, bw.x, bw.y);
+                }
             }
         }
+    }
+
+    // ---- 5. the CTA's partial: o_lat^T fragments (channels g, g+8; heads 2cq, 2cq+1), m and l per head
+    const size_t pb = (size_t(b) * p.n_split + split) * H + h0;
+#pragma unroll
+    for (int j = 0; j < MB; ++j) {
+        const int mb = warp + 8 * j;
+        if (mb >= nks) break;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int hl = 2 * cq + (e & 1), ch = mb * 16 + g + (e >> 1) * 8;
+            if (h0 + hl < H) p.po[(pb + hl) * r + ch] = o[j][e];
+        }
+    }
+    if (warp < kHG && lane == 0 && h0 + warp < H) {
+        p.pm[pb + warp] = m_run * 0.6931471805599453f;        // natural-log units
+        p.pl[pb + warp] = l_run;
     }
 }
 
@@ -371,39 +400,70 @@ bool attn_mma_use(const CacheView &c, int H, int B, int max_seq_len) {
     return int64_t(B) * max_seq_len <= 16384 || !attn_tc_shape_ok(c.r, c.bits, H);
 }
 
-// Tokens per CTA: the smallest of 16, 32, 64 whose grid fits one wave of the
-// GPU (fewer, larger CTAs load the query block and write an o_lat partial
-// fewer times), and at most 64 partials per sequence.
-int attn_mma_splits(int B, int H, int max_seq_len, int *ts) {
+namespace {
+// Dynamic shared memory of one CTA: a sub-tile of cache rows, the query
+// block, int4 group scales and P.
+size_t attn_mma_smem(int r, int bits, int ts) {
+    const int row_bytes = bits == 8 ? r : r / 2;
+    return size_t(ts) * (row_bytes + am::kRowPad) + size_t(am::kHG) * (r + am::kQPad) * 2 +
+           (bits == 4 ? size_t(ts) * (r / 128) * 2 : 0) + size_t(am::kHG) * (ts + 8) * 2;
+}
+// Largest sub-tile whose rows fit next to the static arrays.
+int attn_mma_max_ts(int r, int bits) {
+    constexpr size_t kBudget = 200 * 1024;
+    int t = am::kMaxTS;
+    while (t > 16 && attn_mma_smem(r, bits, t) > kBudget) t /= 2;
+    return attn_mma_smem(r, bits, t) <= kBudget ? t : 0;
+}
+constexpr int kMaxRankMma = 3072;     // 24 channel blocks per warp at most
+}  // namespace
+
+// Sub-tile: the smallest of 16, 32, 64 (within shared memory) whose grid fits
+// one wave of the GPU; sub-tiles per split: at least enough for 64 partials
+// per sequence, and more while two waves of CTAs remain (fewer partials to
+// merge, fewer query-block loads).
+int attn_mma_splits(const CacheView &c, int B, int H, int max_seq_len, int *ts, int *n_sub) {
     int dev = 0, sms = 148;
     if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t hg = (H + am::kHG - 1) / am::kHG;
+    const int tmax = attn_mma_max_ts(c.r, c.bits);
     int t = 16;
-    while (t < am::kMaxTS && ((max_seq_len + t - 1) / t > 64 || int64_t(B) * ((max_seq_len + t - 1) / t) * hg > sms))
-        t *= 2;
+    while (t < tmax && int64_t(B) * ((max_seq_len + t - 1) / t) * hg > sms) t *= 2;
+    const int tiles = (max_seq_len + t - 1) / t;
+    int ns = (tiles + 63) / 64;
+    while (2 * ns <= tiles && int64_t(B) * hg * ((tiles + 2 * ns - 1) / (2 * ns)) >= 2 * int64_t(sms)) ns *= 2;
     *ts = t;
-    return (max_seq_len + t - 1) / t;
+    *n_sub = ns;
+    return (tiles + ns - 1) / ns;
 }
 
-bool attn_mma_fits(int max_seq_len) { return (max_seq_len + am::kMaxTS - 1) / am::kMaxTS <= 64; }
+bool attn_mma_fits(const CacheView &c, int max_seq_len) {
+    (void)max_seq_len;                // any length: a CTA walks as many sub-tiles as needed
+    return c.r <= kMaxRankMma && attn_mma_max_ts(c.r, c.bits) > 0;
+}
+
+namespace {
+template <int BITS>
+cudaError_t launch_mma_bits(const am::Params &prm, dim3 grid, size_t smem, cudaStream_t s) {
+    const int need = (prm.c.r + 127) / 128;           // channel blocks per warp
+    auto go = [&](auto kern) {
+        cudaError_t e = ensure_smem(kern, smem);
+        return e == cudaSuccess ? launch_pdl(kern, grid, dim3(am::kThreads), smem, s, prm) : e;
+    };
+    if (need <= 4) return go(attn_mma_kernel<BITS, 4>);
+    if (need <= 12) return go(attn_mma_kernel<BITS, 12>);
+    if (need <= 16) return go(attn_mma_kernel<BITS, 16>);
+    return go(attn_mma_kernel<BITS, 24>);
+}
+}  // namespace
 
 cudaError_t launch_attn_mma(const CacheView &c, const int32_t *seq_len, const float *qt, const unsigned *qmax, int H,
-                            float softmax_scale, int ts, int n_split, float *pm, float *pl, float *po, int *err,
-                            cudaStream_t s) {
-    const int row_bytes = c.bits == 8 ? c.r : c.r / 2;
-    const size_t smem = size_t(ts) * (row_bytes + am::kRowPad) + size_t(am::kHG) * (c.r + am::kQPad) * 2 +
-                        (c.bits == 4 ? size_t(ts) * (c.r / 128) * 2 : 0) + size_t(am::kHG) * (ts + 8) * 2;
-    const am::Params prm{c, seq_len, qt, qmax, H, ts, n_split, softmax_scale, pm, pl, po, err};
+                            float softmax_scale, int ts, int n_sub, int n_split, float *pm, float *pl, float *po,
+                            int *err, cudaStream_t s) {
+    const size_t smem = attn_mma_smem(c.r, c.bits, ts);
+    const am::Params prm{c, seq_len, qt, qmax, H, ts, n_sub, n_split, softmax_scale, pm, pl, po, err};
     const dim3 grid(n_split, c.B, (H + am::kHG - 1) / am::kHG);
-    cudaError_t e;
-    if (c.bits == 8) {
-        e = ensure_smem(attn_mma_kernel<8>, smem);
-        if (e == cudaSuccess) e = launch_pdl(attn_mma_kernel<8>, grid, dim3(am::kThreads), smem, s, prm);
-    } else {
-        e = ensure_smem(attn_mma_kernel<4>, smem);
-        if (e == cudaSuccess) e = launch_pdl(attn_mma_kernel<4>, grid, dim3(am::kThreads), smem, s, prm);
-    }
-    return e;
+    return c.bits == 8 ? launch_mma_bits<8>(prm, grid, smem, s) : launch_mma_bits<4>(prm, grid, smem, s);
 }
 
 }  // namespace qsvd

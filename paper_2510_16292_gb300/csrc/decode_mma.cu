@@ -377,17 +377,17 @@ combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ 
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
             if (ns > 0) {
                 const float *src = po + (size_t(b0 + bi) * n_split * H + h) * r + j0 + 4 * q4;
-                for (int s0 = 0; s0 < ns; s0 += 16) {
-                    float4 v[16];
-                    float wk[16];
+                for (int s0 = 0; s0 < ns; s0 += 8) {
+                    float4 v[8];
+                    float wk[8];
 #pragma unroll
-                    for (int k = 0; k < 16; ++k) {
+                    for (int k = 0; k < 8; ++k) {
                         const int sk = s0 + k, sc = sk < ns ? sk : ns - 1;
                         v[k] = *reinterpret_cast<const float4 *>(src + size_t(sc) * H * r);
                         wk[k] = sk < ns ? w_s[bi][sc] : 0.0f;
                     }
 #pragma unroll
-                    for (int k = 0; k < 16; ++k) {
+                    for (int k = 0; k < 8; ++k) {
                         acc.x = fmaf(wk[k], v[k].x, acc.x);
                         acc.y = fmaf(wk[k], v[k].y, acc.y);
                         acc.z = fmaf(wk[k], v[k].z, acc.z);

@@ -315,12 +315,12 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
 
     int chunk = chunk_tokens(a.max_seq_len);
     int ns = (a.max_seq_len + chunk - 1) / chunk;
-    if (attn_mma_use(c, H, B, a.max_seq_len) && attn_mma_fits(a.max_seq_len)) {
+    if (attn_mma_use(c, H, B, a.max_seq_len) && attn_mma_fits(c, a.max_seq_len)) {
         // a6/a7 on the warp-level tensor-core MMA: one partial per range of ts tokens
-        int ts = 16;
-        ns = attn_mma_splits(B, H, a.max_seq_len, &ts);
-        chunk = ts;
-        e = launch_attn_mma(c, a.seq_len, w.qt, w.qmax, H, a.softmax_scale, ts, ns, w.pm, w.pl, w.po, err, s);
+        int ts = 16, n_sub = 1;
+        ns = attn_mma_splits(c, B, H, a.max_seq_len, &ts, &n_sub);
+        chunk = ts * n_sub;
+        e = launch_attn_mma(c, a.seq_len, w.qt, w.qmax, H, a.softmax_scale, ts, n_sub, ns, w.pm, w.pl, w.po, err, s);
         if (e != cudaSuccess) return e;
         prof_mark(s, "attn_mma");
     } else if (attn_tc_use(c, H, a.max_seq_len)) {

@@ -167,11 +167,11 @@ bool attn_tc_use(const CacheView &c, int H, int max_seq_len);
 int attn_tc_splits(int B, int max_seq_len, int *tiles_per_split);
 // Warp-level tensor-core attention for small batch x length (attn_mma.cu).
 bool attn_mma_use(const CacheView &c, int H, int B, int max_seq_len);
-bool attn_mma_fits(int max_seq_len);
-int attn_mma_splits(int B, int H, int max_seq_len, int *ts);
+bool attn_mma_fits(const CacheView &c, int max_seq_len);
+int attn_mma_splits(const CacheView &c, int B, int H, int max_seq_len, int *ts, int *n_sub);
 cudaError_t launch_attn_mma(const CacheView &c, const int32_t *seq_len, const float *qt, const unsigned *qmax, int H,
-                            float softmax_scale, int ts, int n_split, float *pm, float *pl, float *po, int *err,
-                            cudaStream_t s);
+                            float softmax_scale, int ts, int n_sub, int n_split, float *pm, float *pl, float *po,
+                            int *err, cudaStream_t s);
 cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const float *qt, const unsigned *qmax, int H,
                            float softmax_scale,
                            int tiles_per_split, int n_split, float *pm, float *pl, float *po, int *err,

@@ -119,10 +119,14 @@ def test_attn_mma_ragged(bits):
 
 
 @pytest.mark.parametrize("H,dh,r,bits,lens", [(40, 128, 2048, 8, [3000, 77]), (4, 64, 96, 8, [80, 33]),
-                                               (20, 64, 768, 4, [2049, 64])])
+                                               (20, 64, 768, 4, [2049, 64]), (32, 128, 3072, 8, [1500, 33]),
+                                               (40, 128, 2048, 8, [9000, 300]), (32, 128, 3072, 4, [5000, 17])])
 def test_attn_mma_shapes(H, dh, r, bits, lens):
     """H = 40 (five head groups of 8) at the 13B rank with 64-token splits,
-    the tiny layer (r = 96, padded heads), and a 32-token split with int4."""
+    the tiny layer (r = 96, padded heads), a 32-token split with int4,
+    r = 3072, where the sub-tile is capped at 32 tokens by shared memory, and
+    lengths beyond 64 sub-tiles (each CTA walks several sub-tiles with a
+    running softmax) at r = 2048 and r = 3072 (int4)."""
     _run(H, dh, r, bits, lens, paths=(3,), seed=13)
 
 
