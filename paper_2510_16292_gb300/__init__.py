@@ -77,14 +77,24 @@ def library_path() -> str:
     return _LIB_PATH
 
 
-def _ptr(t: Optional[torch.Tensor]):
+def _ptr(t: Optional[torch.Tensor], dtype=None, name: str = "tensor"):
+    """Device pointer of a contiguous CUDA tensor; `dtype` (one dtype or a
+    tuple) is the element type the C ABI reads through that pointer."""
     if t is None:
         return None
     if not t.is_cuda:
-        raise ValueError("device tensor expected")
+        raise ValueError(f"{name}: device tensor expected")
     if not t.is_contiguous():
-        raise ValueError("contiguous tensor expected")
+        raise ValueError(f"{name}: contiguous tensor expected")
+    if dtype is not None:
+        ok = t.dtype in dtype if isinstance(dtype, tuple) else t.dtype == dtype
+        if not ok:
+            raise TypeError(f"{name}: dtype {t.dtype} where {dtype} is expected")
     return t.data_ptr()
+
+
+_I32, _BF16, _F32 = torch.int32, torch.bfloat16, torch.float32
+_CODES, _SCALES = (torch.int8, torch.uint8), (torch.float32, torch.float16)
 
 
 def _stream(stream=None):
@@ -113,7 +123,8 @@ class DownWeight:
         return self.codes.shape[0]
 
     def _c(self):
-        return _DownWeight(_ptr(self.codes), _ptr(self.codes_bf16), _ptr(self.scale), self.d, self.r)
+        return _DownWeight(_ptr(self.codes, torch.int8, "W.codes"), _ptr(self.codes_bf16, _BF16, "W.codes_bf16"),
+                           _ptr(self.scale, _F32, "W.scale"), self.d, self.r)
 
 
 @dataclasses.dataclass
@@ -138,7 +149,9 @@ class LatentCache:
         return LatentCache(codes, scales, bits, B, Tmax, r)
 
     def _c(self):
-        return _Cache(_ptr(self.codes), _ptr(self.scales), self.bits, self.B, self.Tmax, self.r)
+        return _Cache(_ptr(self.codes, torch.int8 if self.bits == 8 else torch.uint8, "cache.codes"),
+                      _ptr(self.scales, _F32 if self.bits == 8 else torch.float16, "cache.scales"),
+                      self.bits, self.B, self.Tmax, self.r)
 
     def nbytes_per_token(self) -> int:
         return self.r if self.bits == 8 else self.r // 2 + 2 * (self.r // 128)
@@ -151,7 +164,7 @@ def qsvd_quantize_weight(W_d: torch.Tensor, clip: float = 1.0, stream=None) -> D
     codes = torch.empty((r, d), dtype=torch.int8, device=dev)
     codes_bf16 = torch.empty((r, d), dtype=torch.bfloat16, device=dev)
     scale = torch.empty((r,), dtype=torch.float32, device=dev)
-    _check(_lib.qsvd_quantize_weight(_ptr(W_d), d, r, clip, _ptr(codes), _ptr(codes_bf16), _ptr(scale),
+    _check(_lib.qsvd_quantize_weight(_ptr(W_d, _F32, "W_d"), d, r, clip, _ptr(codes), _ptr(codes_bf16), _ptr(scale),
                                      _stream(stream)))
     return DownWeight(codes, codes_bf16, scale)
 
@@ -174,18 +187,21 @@ def qsvd_latent_project(W: DownWeight, X: torch.Tensor, act_clip: float = 1.0, l
                                 device=X.device)
     cw = W._c()
     cc = dst._c() if dst is not None else None
-    _check(_lib.qsvd_latent_project(ctypes.byref(cw), _ptr(X), T, act_clip, lat_bits, lat_clip,
-                                    _ptr(lat_codes), _ptr(lat_scales),
+    _check(_lib.qsvd_latent_project(ctypes.byref(cw), _ptr(X, _BF16, "X"), T, act_clip, lat_bits, lat_clip,
+                                    _ptr(lat_codes, _CODES, "lat_codes"), _ptr(lat_scales, _SCALES, "lat_scales"),
                                     ctypes.byref(cc) if cc is not None else None,
-                                    _ptr(dst_seq), _ptr(dst_pos), _ptr(xq_out), _ptr(xs_out), _ptr(acc_out),
+                                    _ptr(dst_seq, _I32, "dst_seq"), _ptr(dst_pos, _I32, "dst_pos"),
+                                    _ptr(xq_out, torch.int8, "xq_out"), _ptr(xs_out, _F32, "xs_out"),
+                                    _ptr(acc_out, _I32, "acc_out"),
                                     _ptr(workspace), workspace.numel(), _stream(stream)))
 
 
 def qsvd_cache_append(cache: LatentCache, seq: torch.Tensor, pos: torch.Tensor, lat_codes: torch.Tensor,
                       lat_scales: torch.Tensor, stream=None) -> None:
     cc = cache._c()
-    _check(_lib.qsvd_cache_append(ctypes.byref(cc), _ptr(seq), _ptr(pos), seq.numel(), _ptr(lat_codes),
-                                  _ptr(lat_scales), _stream(stream)))
+    _check(_lib.qsvd_cache_append(ctypes.byref(cc), _ptr(seq, _I32, "seq"), _ptr(pos, _I32, "pos"), seq.numel(),
+                                  _ptr(lat_codes, _CODES, "lat_codes"), _ptr(lat_scales, _SCALES, "lat_scales"),
+                                  _stream(stream)))
 
 
 def qsvd_latent_decode_attn(cache: LatentCache, seq_len: torch.Tensor, max_seq_len: int, U_q, U_k, U_v,
@@ -197,8 +213,9 @@ def qsvd_latent_decode_attn(cache: LatentCache, seq_len: torch.Tensor, max_seq_l
         workspace = torch.zeros(qsvd_decode_workspace_bytes(cache.B, max_seq_len, cache.r, H, dh),
                                 dtype=torch.uint8, device=O.device)
     cc = cache._c()
-    _check(_lib.qsvd_latent_decode_attn(ctypes.byref(cc), _ptr(seq_len), max_seq_len, _ptr(U_q), _ptr(U_k),
-                                        _ptr(U_v), H, dh, softmax_scale, _ptr(O), _ptr(workspace),
+    _check(_lib.qsvd_latent_decode_attn(ctypes.byref(cc), _ptr(seq_len, _I32, "seq_len"), max_seq_len,
+                                        _ptr(U_q, _BF16, "U_q"), _ptr(U_k, _BF16, "U_k"), _ptr(U_v, _BF16, "U_v"),
+                                        H, dh, softmax_scale, _ptr(O, _F32, "O"), _ptr(workspace),
                                         workspace.numel(), _stream(stream)))
 
 
@@ -218,9 +235,10 @@ def qsvd_decode_step(W: DownWeight, X: torch.Tensor, cache: LatentCache, seq_len
         workspace = torch.zeros(qsvd_decode_step_workspace_bytes(cache.B, max_seq_len, W.d, W.r, H, dh),
                                 dtype=torch.uint8, device=O.device)
     cw, cc = W._c(), cache._c()
-    _check(_lib.qsvd_decode_step(ctypes.byref(cw), _ptr(X), ctypes.byref(cc), _ptr(seq_len), max_seq_len,
-                                 _ptr(U_q), _ptr(U_k), _ptr(U_v), H, dh, act_clip, lat_clip, softmax_scale,
-                                 _ptr(O), _ptr(workspace), workspace.numel(), _stream(stream)))
+    _check(_lib.qsvd_decode_step(ctypes.byref(cw), _ptr(X, _BF16, "X"), ctypes.byref(cc),
+                                 _ptr(seq_len, _I32, "seq_len"), max_seq_len, _ptr(U_q, _BF16, "U_q"),
+                                 _ptr(U_k, _BF16, "U_k"), _ptr(U_v, _BF16, "U_v"), H, dh, act_clip, lat_clip,
+                                 softmax_scale, _ptr(O, _F32, "O"), _ptr(workspace), workspace.numel(), _stream(stream)))
 
 
 def qsvd_latent_project_static(W: DownWeight, X: torch.Tensor, act_clip: float = 1.0, lat_bits: int = 8,
@@ -230,10 +248,12 @@ def qsvd_latent_project_static(W: DownWeight, X: torch.Tensor, act_clip: float =
     scratch instead of a workspace; nothing is allocated on the device."""
     cw = W._c()
     cc = dst._c() if dst is not None else None
-    _check(_lib.qsvd_latent_project_static(ctypes.byref(cw), _ptr(X), X.shape[0], act_clip, lat_bits, lat_clip,
-                                           _ptr(lat_codes), _ptr(lat_scales),
-                                           ctypes.byref(cc) if cc is not None else None, _ptr(dst_seq),
-                                           _ptr(dst_pos), _stream(stream)))
+    _check(_lib.qsvd_latent_project_static(ctypes.byref(cw), _ptr(X, _BF16, "X"), X.shape[0], act_clip, lat_bits,
+                                           lat_clip, _ptr(lat_codes, _CODES, "lat_codes"),
+                                           _ptr(lat_scales, _SCALES, "lat_scales"),
+                                           ctypes.byref(cc) if cc is not None else None,
+                                           _ptr(dst_seq, _I32, "dst_seq"), _ptr(dst_pos, _I32, "dst_pos"),
+                                           _stream(stream)))
 
 
 def qsvd_check(stream=None) -> int:
@@ -261,8 +281,9 @@ def qsvd_set_project_epilogue(mode: int) -> int:
 
 
 def qsvd_set_decode_attn_path(path: int) -> int:
-    """0 automatic, 1 CUDA-core kernels, 2 tensor-core kernel where the shape
-    allows it.  Returns the previous setting."""
+    """0 automatic, 1 CUDA-core kernels, 2 tcgen05 kernel where the shape
+    allows it, 3 warp-level tensor-core kernel (r <= 3072).  Returns the
+    previous setting."""
     st = _lib.qsvd_set_decode_attn_path(path)
     if st < 0:
         _check(st)

@@ -21,10 +21,12 @@
 //      warp's channel blocks stay in registers across the sub-tiles.
 //   5. the CTA's (m, l, o_lat) are written as one softmax partial.
 //
-// Within one MMA the 16 reduction indices are used in the order
-// {0,1,4,5,8,9,12,13, 2,3,6,7,10,11,14,15} on both operands (the sum does not
-// depend on the order), so that each operand fragment comes from one 32- or
-// 64-bit shared-memory load.
+// Within one score MMA the 16 channels (the reduction index) are used in the
+// order {0,1,4,5,8,9,12,13, 2,3,6,7,10,11,14,15} on both operands (the sum
+// does not depend on the order), so that a thread's operand fragment is one
+// 32-bit (int8) or 16-bit (int4) shared-memory load.  Step 4 reloads the same
+// fragments and transposes them in registers (movmatrix): its M rows are the
+// channels in that order, which the final store undoes.
 #include <cfloat>
 #include <cuda_fp16.h>
 
@@ -35,7 +37,8 @@ namespace qsvd {
 
 namespace am {
 
-constexpr int kThreads = 256;     // 8 warps
+constexpr int kWarps = 16;
+constexpr int kThreads = 32 * kWarps;
 constexpr int kHG = 8;            // heads per CTA (one n-block)
 constexpr int kMaxTS = 64;        // tokens per CTA
 constexpr int kRowPad = 16;       // bytes of padding per cache row in shared memory
@@ -76,12 +79,37 @@ __device__ __forceinline__ void i8x4_h2(uint32_t w, uint32_t &lo, uint32_t &hi) 
     lo = *reinterpret_cast<const uint32_t *>(&ha);
     hi = *reinterpret_cast<const uint32_t *>(&hb);
 }
-// Four int4 codes (element i in bits 4i..4i+3) -> four int8 codes.
-__device__ __forceinline__ uint32_t i4x4_to_i8x4(uint32_t x) {
-    uint32_t w = 0;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) w |= (uint32_t(((int((x >> (4 * e)) & 0xf) ^ 8) - 8) & 0xff)) << (8 * e);
-    return w;
+// Byte k of w (two int4 codes, the even channel in the low nibble) -> their
+// fp16 pair, exact: the nibbles xor 8 go into the mantissas of 1024 and of
+// 1024 * 16, and one fused multiply-add maps both back to the codes.
+__device__ __forceinline__ uint32_t i4pair_h2(uint32_t w, int k) {
+    const uint32_t y = __byte_perm(w, 0u, uint32_t(k) | (4u << 4) | (uint32_t(k) << 8) | (4u << 12));
+    const uint32_t z = (y & 0x00F0000Fu) ^ 0x64806408u;              // 1024 + (lo ^ 8), 1024 + 16 (hi ^ 8)
+    const __half2 mul = __halves2half2(__ushort_as_half(0x3C00), __ushort_as_half(0x2C00));   // 1, 1/16
+    const __half2 add = __halves2half2(__ushort_as_half(0xE408), __ushort_as_half(0xD480));   // -1032, -72
+    const __half2 c = __hfma2(*reinterpret_cast<const __half2 *>(&z), mul, add);
+    return *reinterpret_cast<const uint32_t *>(&c);
+}
+// Transpose of an 8 x 8 fp16 block held one pair per thread (thread t: row
+// t/4, columns 2(t%4), 2(t%4)+1).
+__device__ __forceinline__ uint32_t movm_t(uint32_t a) {
+    uint32_t d;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+    return d;
+}
+// Score-operand fragment of cache row `row`, channel step k0: the fp16 pairs
+// of channels (4cq, 4cq+1) and (4cq+2, 4cq+3), i.e. reduction indices
+// (2cq, 2cq+1) and (2cq+8, 2cq+9) in the order above.
+template <int BITS>
+__device__ __forceinline__ void load_frag(const uint8_t *tile, int rstride, int row, int k0, int cq, uint32_t &lo,
+                                          uint32_t &hi) {
+    if (BITS == 8) {
+        i8x4_h2(*reinterpret_cast<const uint32_t *>(tile + size_t(row) * rstride + k0 + 4 * cq), lo, hi);
+    } else {
+        const uint32_t w = *reinterpret_cast<const uint16_t *>(tile + size_t(row) * rstride + (k0 + 4 * cq) / 2);
+        lo = i4pair_h2(w, 0);
+        hi = i4pair_h2(w, 1);
+    }
 }
 
 }  // namespace am
@@ -91,7 +119,7 @@ __global__ void __launch_bounds__(am::kThreads)
 attn_mma_kernel(const am::Params p) {
     using namespace am;
     extern __shared__ __align__(16) uint8_t smem[];
-    __shared__ float sred[8][kMaxTS][kHG];          // per-warp partial scores
+    __shared__ float sred[kWarps][kMaxTS][kHG];     // per-warp partial scores
     __shared__ float tsc_s[kMaxTS];                 // int8 token scales
     __shared__ float qfac_s[kHG];
     __shared__ float m_s[kHG];
@@ -125,9 +153,33 @@ attn_mma_kernel(const am::Params p) {
     }
     pdl_wait();
 
+    // sub-tile `sb`: cache rows (zero beyond the length) by 16-byte asynchronous copies, and the scales
+    auto load_tile = [&](int sb) {
+        const int t_begin = t_split + sb * TS;
+        const int n = min(TS, L - t_begin);
+        const size_t slot0 = size_t(b) * c.Tmax + t_begin;
+        const int cpr = row_bytes / 16;                            // 16-byte chunks per row
+        for (int i = threadIdx.x; i < TS * cpr; i += kThreads) {
+            const int t = i / cpr, k = i - t * cpr;
+            uint8_t *dst = tile + size_t(t) * rstride + k * 16;
+            if (t < n) cp_async16(dst, static_cast<const uint8_t *>(c.codes) + (slot0 + t) * row_bytes + k * 16);
+            else *reinterpret_cast<uint4 *>(dst) = make_uint4(0u, 0u, 0u, 0u);
+        }
+        if (BITS == 8) {
+            if (threadIdx.x < TS)
+                tsc_s[threadIdx.x] = threadIdx.x < n ? static_cast<const float *>(c.scales)[slot0 + threadIdx.x] : 0.0f;
+        } else {
+            for (int i = threadIdx.x; i < TS * (r / 128); i += kThreads) {
+                const int t = i / (r / 128);
+                gsc[i] = t < n ? static_cast<const __half *>(c.scales)[slot0 * (r / 128) + i] : __float2half(0.0f);
+            }
+        }
+    };
+    load_tile(0);                                                  // overlaps the query block below
+
     // ---- 0. query block: q~ loads first, the per-head scale applied once qmax is in
     {
-        constexpr int kQL = 16;                                    // float4 per thread per pass (r <= 2048: one pass)
+        constexpr int kQL = 8;                                     // float4 per thread per pass (r <= 2048: one pass)
         const int nq4 = kHG * (r / 4);
         float4 v[kQL];
 #pragma unroll
@@ -173,7 +225,7 @@ attn_mma_kernel(const am::Params p) {
     const int MT = TS / 16, nks = r / 16;
     // running softmax state of head `warp` (warps < kHG), the same in every lane
     float m_run = -INFINITY, l_run = 0.0f;
-    // o_lat^T accumulators: channel block mb = warp + 8 j, fragment (channels g, g+8; heads 2cq, 2cq+1)
+    // o_lat^T accumulators: channel step mb = warp + kWarps j, fragment (reduction indices g, g+8; heads 2cq, 2cq+1)
     float o[MB][4];
 #pragma unroll
     for (int j = 0; j < MB; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.0f;
@@ -181,31 +233,15 @@ attn_mma_kernel(const am::Params p) {
     for (int sb = 0; sb < n_sub; ++sb) {
         const int t_begin = t_split + sb * TS;
         const int n = min(TS, L - t_begin);
-        const size_t slot0 = size_t(b) * c.Tmax + t_begin;
-        __syncthreads();                                           // the previous sub-tile's readers are done
-        // ---- 1. cache rows (zero beyond n) and scales
-        {
-            const int cpr = row_bytes / 16;                        // 16-byte chunks per row
-            for (int i = threadIdx.x; i < TS * cpr; i += kThreads) {
-                const int t = i / cpr, k = i - t * cpr;
-                uint8_t *dst = tile + size_t(t) * rstride + k * 16;
-                if (t < n) cp_async16(dst, static_cast<const uint8_t *>(c.codes) + (slot0 + t) * row_bytes + k * 16);
-                else *reinterpret_cast<uint4 *>(dst) = make_uint4(0u, 0u, 0u, 0u);
-            }
-            if (BITS == 8) {
-                if (threadIdx.x < TS)
-                    tsc_s[threadIdx.x] = threadIdx.x < n ? static_cast<const float *>(c.scales)[slot0 + threadIdx.x] : 0.0f;
-            } else {
-                for (int i = threadIdx.x; i < TS * (r / 128); i += kThreads) {
-                    const int t = i / (r / 128);
-                    gsc[i] = t < n ? static_cast<const __half *>(c.scales)[slot0 * (r / 128) + i] : __float2half(0.0f);
-                }
-            }
-            cp_async_wait_all();
-            __syncthreads();
+        // ---- 1. cache rows and scales (sub-tile 0 was issued before the query block)
+        if (sb > 0) {
+            __syncthreads();                                       // the previous sub-tile's readers are done
+            load_tile(sb);
         }
+        cp_async_wait_all();
+        __syncthreads();
 
-        // ---- 2. scores: warp w takes 16-channel steps w, w+8, ...; MT m-blocks of 16 tokens
+        // ---- 2. scores: warp w takes 16-channel steps w, w+kWarps, ...; MT m-blocks of 16 tokens
         {
             float acc[kMaxTS / 16][4];
 #pragma unroll
@@ -214,7 +250,7 @@ attn_mma_kernel(const am::Params p) {
 #pragma unroll
             for (int m = 0; m < kMaxTS / 16; ++m) gacc[m][0] = gacc[m][1] = gacc[m][2] = gacc[m][3] = 0.0f;
             int cur_grp = -1;
-            for (int ks = warp; ks < nks; ks += 8) {
+            for (int ks = warp; ks < nks; ks += kWarps) {
                 const int k0 = ks * 16;
                 // B: Q~[head g][channels k0 + 4 cq .. + 3]
                 const uint2 bw = *reinterpret_cast<const uint2 *>(qs + size_t(g) * qstride + k0 + 4 * cq);
@@ -239,19 +275,12 @@ attn_mma_kernel(const am::Params p) {
                 for (int m = 0; m < kMaxTS / 16; ++m) {
                     if (m >= MT) break;
                     uint32_t a0, a1, a2, a3;
-                    if (BITS == 8) {
-                        const uint32_t w0 = *reinterpret_cast<const uint32_t *>(tile + size_t(m * 16 + g) * rstride + k0 + 4 * cq);
-                        const uint32_t w1 = *reinterpret_cast<const uint32_t *>(tile + size_t(m * 16 + g + 8) * rstride + k0 + 4 * cq);
-                        i8x4_h2(w0, a0, a2);
-                        i8x4_h2(w1, a1, a3);
-                        mma16816((ks >> 3) & 1 ? gacc[m] : acc[m], a0, a1, a2, a3, bw.x, bw.y);   // two chains
-                    } else {
-                        const uint32_t x0 = *reinterpret_cast<const uint16_t *>(tile + size_t(m * 16 + g) * rstride + (k0 + 4 * cq) / 2);
-                        const uint32_t x1 = *reinterpret_cast<const uint16_t *>(tile + size_t(m * 16 + g + 8) * rstride + (k0 + 4 * cq) / 2);
-                        i8x4_h2(i4x4_to_i8x4(x0), a0, a2);
-                        i8x4_h2(i4x4_to_i8x4(x1), a1, a3);
+                    load_frag<BITS>(tile, rstride, m * 16 + g, k0, cq, a0, a2);
+                    load_frag<BITS>(tile, rstride, m * 16 + g + 8, k0, cq, a1, a3);
+                    if (BITS == 8)
+                        mma16816((ks / kWarps) & 1 ? gacc[m] : acc[m], a0, a1, a2, a3, bw.x, bw.y);   // two chains
+                    else
                         mma16816(gacc[m], a0, a1, a2, a3, bw.x, bw.y);
-                    }
                 }
             }
             if (BITS == 8) {                           // add the second chain
@@ -293,7 +322,7 @@ attn_mma_kernel(const am::Params p) {
                 if (t < n && h < H) {
                     float sacc = 0.0f;
 #pragma unroll
-                    for (int w = 0; w < 8; ++w) sacc += sred[w][t][hl];
+                    for (int w = 0; w < kWarps; ++w) sacc += sred[w][t][hl];
                     v = sacc * qfac_s[hl] * (BITS == 8 ? tsc_s[t] : 1.0f);
                 }
                 lg[u] = v;
@@ -317,7 +346,7 @@ attn_mma_kernel(const am::Params p) {
         }
         __syncthreads();
 
-        // ---- 4. O^T[ch, h] += sum_t C[t, ch] P[t, h]: warp w, channel blocks w + 8 j
+        // ---- 4. O^T[ch, h] += sum_t C[t, ch] P[t, h]: warp w, channel blocks w + kWarps j
         {
             const float al0 = alpha_s[2 * cq], al1 = alpha_s[2 * cq + 1];
 #pragma unroll
@@ -325,63 +354,50 @@ attn_mma_kernel(const am::Params p) {
                 o[j][0] *= al0; o[j][1] *= al1; o[j][2] *= al0; o[j][3] *= al1;
             }
             for (int kt = 0; kt < MT; ++kt) {
-                const int t0 = kt * 16 + 4 * cq;
-                // B: P[head g][tokens t0 .. t0 + 3]
-                const uint2 pw = *reinterpret_cast<const uint2 *>(ps + size_t(g) * pstride + t0);
-                const uint8_t *row0 = tile + size_t(t0) * rstride;
+                const int tb = kt * 16;
+                // B: P[head g][tokens tb + 2cq, +1] and [tb + 8 + 2cq, +1]
+                const uint32_t pw0 = *reinterpret_cast<const uint32_t *>(ps + size_t(g) * pstride + tb + 2 * cq);
+                const uint32_t pw1 = *reinterpret_cast<const uint32_t *>(ps + size_t(g) * pstride + tb + 8 + 2 * cq);
 #pragma unroll
                 for (int j = 0; j < MB; ++j) {
-                    const int mb = warp + 8 * j;
+                    const int mb = warp + kWarps * j;
                     if (mb >= nks) break;
-                    const int ch0 = mb * 16;
-                    // A: channels ch0 + g, ch0 + g + 8; tokens t0 .. t0 + 3
-                    uint32_t wlo = 0, whi = 0;
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const uint8_t *rowp = row0 + size_t(e) * rstride;
-                        uint32_t blo, bhi;
-                        if (BITS == 8) {
-                            blo = rowp[ch0 + g];
-                            bhi = rowp[ch0 + g + 8];
-                        } else {
-                            const uint32_t x0 = rowp[(ch0 + g) >> 1], x1 = rowp[(ch0 + g + 8) >> 1];
-                            const int sh = ((ch0 + g) & 1) * 4;
-                            blo = uint32_t((((int(x0 >> sh) & 0xf) ^ 8) - 8) & 0xff);
-                            bhi = uint32_t((((int(x1 >> sh) & 0xf) ^ 8) - 8) & 0xff);
-                        }
-                        wlo |= blo << (8 * e);
-                        whi |= bhi << (8 * e);
-                    }
-                    uint32_t a0, a1, a2, a3;
-                    i8x4_h2(wlo, a0, a2);
-                    i8x4_h2(whi, a1, a3);
-                    uint2 bw = pw;
+                    // A: the score fragments of tokens tb.. tb + 15, channel step mb, transposed
+                    uint32_t x0, x1, x2, x3;
+                    load_frag<BITS>(tile, rstride, tb + g, mb * 16, cq, x0, x2);
+                    load_frag<BITS>(tile, rstride, tb + g + 8, mb * 16, cq, x1, x3);
+                    uint32_t b0 = pw0, b1 = pw1;
                     if (BITS == 4) {                    // int4: times the token's group scale
-                        const int grp = ch0 / 128;
-                        const __half2 s01 = __halves2half2(gsc[(t0 + 0) * (r / 128) + grp], gsc[(t0 + 1) * (r / 128) + grp]);
-                        const __half2 s23 = __halves2half2(gsc[(t0 + 2) * (r / 128) + grp], gsc[(t0 + 3) * (r / 128) + grp]);
-                        const __half2 p01 = __hmul2(*reinterpret_cast<const __half2 *>(&pw.x), s01);
-                        const __half2 p23 = __hmul2(*reinterpret_cast<const __half2 *>(&pw.y), s23);
-                        bw.x = *reinterpret_cast<const uint32_t *>(&p01);
-                        bw.y = *reinterpret_cast<const uint32_t *>(&p23);
+                        const int grp = mb / 8, ng = r / 128;
+                        const __half2 s0 = __halves2half2(gsc[(tb + 2 * cq) * ng + grp], gsc[(tb + 2 * cq + 1) * ng + grp]);
+                        const __half2 s1 = __halves2half2(gsc[(tb + 8 + 2 * cq) * ng + grp], gsc[(tb + 9 + 2 * cq) * ng + grp]);
+                        const __half2 p0 = __hmul2(*reinterpret_cast<const __half2 *>(&pw0), s0);
+                        const __half2 p1 = __hmul2(*reinterpret_cast<const __half2 *>(&pw1), s1);
+                        b0 = *reinterpret_cast<const uint32_t *>(&p0);
+                        b1 = *reinterpret_cast<const uint32_t *>(&p1);
                     }
-                    mma16816(o[j], a0, a1, a2, a3, bw.x, bw.y);
+                    mma16816(o[j], movm_t(x0), movm_t(x2), movm_t(x1), movm_t(x3), b0, b1);
                 }
             }
         }
     }
 
-    // ---- 5. the CTA's partial: o_lat^T fragments (channels g, g+8; heads 2cq, 2cq+1), m and l per head
+    // ---- 5. the CTA's partial: o_lat^T fragments (reduction indices g, g+8 of the
+    //         channel step, i.e. channels 4(g/2) + g%2 and that + 2; heads 2cq, 2cq+1),
+    //         m and l per head.
+    //         Lanes g = 2a and 2a + 1 hold channels 4a, 4a + 2 and 4a + 1, 4a + 3 of
+    //         heads 2cq, 2cq + 1: one exchange gives each a float4 of 4 consecutive
+    //         channels of one head (even lane: head 2cq, odd lane: head 2cq + 1).
     const size_t pb = (size_t(b) * p.n_split + split) * H + h0;
+    const int odd = g & 1, hl = 2 * cq + odd, c4 = 4 * (g >> 1);
 #pragma unroll
     for (int j = 0; j < MB; ++j) {
-        const int mb = warp + 8 * j;
+        const int mb = warp + kWarps * j;
         if (mb >= nks) break;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const int hl = 2 * cq + (e & 1), ch = mb * 16 + g + (e >> 1) * 8;
-            if (h0 + hl < H) p.po[(pb + hl) * r + ch] = o[j][e];
-        }
+        const float v0 = __shfl_xor_sync(0xffffffffu, odd ? o[j][0] : o[j][1], 4);
+        const float v1 = __shfl_xor_sync(0xffffffffu, odd ? o[j][2] : o[j][3], 4);
+        const float4 w = odd ? make_float4(v0, o[j][1], v1, o[j][3]) : make_float4(o[j][0], v0, o[j][2], v1);
+        if (h0 + hl < H) *reinterpret_cast<float4 *>(p.po + (pb + hl) * r + mb * 16 + c4) = w;
     }
     if (warp < kHG && lane == 0 && h0 + warp < H) {
         p.pm[pb + warp] = m_run * 0.6931471805599453f;        // natural-log units
@@ -408,14 +424,15 @@ size_t attn_mma_smem(int r, int bits, int ts) {
     return size_t(ts) * (row_bytes + am::kRowPad) + size_t(am::kHG) * (r + am::kQPad) * 2 +
            (bits == 4 ? size_t(ts) * (r / 128) * 2 : 0) + size_t(am::kHG) * (ts + 8) * 2;
 }
-// Largest sub-tile whose rows fit next to the static arrays.
+// Largest sub-tile whose rows fit next to the static arrays (about 33 KB of
+// the 227 KB a CTA may hold).
 int attn_mma_max_ts(int r, int bits) {
-    constexpr size_t kBudget = 200 * 1024;
+    constexpr size_t kBudget = 192 * 1024;
     int t = am::kMaxTS;
     while (t > 16 && attn_mma_smem(r, bits, t) > kBudget) t /= 2;
     return attn_mma_smem(r, bits, t) <= kBudget ? t : 0;
 }
-constexpr int kMaxRankMma = 3072;     // 24 channel blocks per warp at most
+constexpr int kMaxRankMma = 3072;     // r / 16 / kWarps channel blocks per warp at most
 }  // namespace
 
 // Sub-tile: the smallest of 16, 32, 64 (within shared memory) whose grid fits
@@ -445,15 +462,18 @@ bool attn_mma_fits(const CacheView &c, int max_seq_len) {
 namespace {
 template <int BITS>
 cudaError_t launch_mma_bits(const am::Params &prm, dim3 grid, size_t smem, cudaStream_t s) {
-    const int need = (prm.c.r + 127) / 128;           // channel blocks per warp
+    const int need = (prm.c.r / 16 + am::kWarps - 1) / am::kWarps;   // channel blocks per warp
     auto go = [&](auto kern) {
         cudaError_t e = ensure_smem(kern, smem);
         return e == cudaSuccess ? launch_pdl(kern, grid, dim3(am::kThreads), smem, s, prm) : e;
     };
+    constexpr int kMaxMB = kMaxRankMma / 16 / am::kWarps;       // r <= kMaxRankMma
+    static_assert(kMaxMB >= 12, "channel blocks per warp");
     if (need <= 4) return go(attn_mma_kernel<BITS, 4>);
+    if (need <= 8) return go(attn_mma_kernel<BITS, 8>);
     if (need <= 12) return go(attn_mma_kernel<BITS, 12>);
-    if (need <= 16) return go(attn_mma_kernel<BITS, 16>);
-    return go(attn_mma_kernel<BITS, 24>);
+    if (need <= 16) return go(attn_mma_kernel<BITS, (kMaxMB > 16 ? 16 : kMaxMB)>);
+    return go(attn_mma_kernel<BITS, kMaxMB>);
 }
 }  // namespace
 

@@ -370,6 +370,7 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__r
     const int per_rank = dh / kCl;
     constexpr int kWB = (NB + 7) / 8;                // sequences per warp in the weight phase
     constexpr int kParts = NB >= 4 ? 1 : 4 / NB;     // lanes sharing one (sequence, row quad)
+    constexpr int kBatch = 16;                       // partial rows in flight per lane
     for (int b0 = 0; b0 < B; b0 += NB) {
         const int nb = min(NB, B - b0);
         __syncthreads();
@@ -420,18 +421,18 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__r
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
             if (ns > 0) {
                 const float *src = po + (size_t(b0 + bi) * n_split * H + h) * r + j0 + 4 * q4;
-                for (int s0 = part; s0 < ns; s0 += 16 * kParts) {
-                    float4 v[16];
-                    float wk[16];
+                for (int s0 = part; s0 < ns; s0 += kBatch * kParts) {
+                    float4 v[kBatch];
+                    float wk[kBatch];
 #pragma unroll
-                    for (int k = 0; k < 16; ++k) {
+                    for (int k = 0; k < kBatch; ++k) {
                         const int sk = s0 + k * kParts;
                         const int sc = sk < ns ? sk : ns - 1;
                         v[k] = *reinterpret_cast<const float4 *>(src + size_t(sc) * H * r);
                         wk[k] = sk < ns ? w_s[bi][sc] : 0.0f;
                     }
 #pragma unroll
-                    for (int k = 0; k < 16; ++k) {
+                    for (int k = 0; k < kBatch; ++k) {
                         acc.x = fmaf(wk[k], v[k].x, acc.x);
                         acc.y = fmaf(wk[k], v[k].y, acc.y);
                         acc.z = fmaf(wk[k], v[k].z, acc.z);
