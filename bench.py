@@ -578,7 +578,8 @@ def run_native(args, rank, world, local_rank):
             "prefill_13b": pre13,
         },
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
-                     "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": None,
+                     "unit": "GB/s", "frac": round(achieved / hbm, 4),
+                     "traffic": captured_traffic(dom, args.workload), "traffic_unit": "bytes per launch",
                      "peak_kind": peak_kind},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk,
@@ -588,6 +589,30 @@ def run_native(args, rank, world, local_rank):
     if world == 1 and not args.no_cpu_baseline and args.workload == WORKLOAD:
         out["cpu_baseline"] = cpu_baseline(wl, budget_s=15.0)
     print(json.dumps(out), flush=True)
+
+
+def captured_traffic(label, workload):
+    """DRAM bytes per launch of kernel `label` on `workload` from the committed
+    ncu launch-list record (profiles/dram_traffic.json), or None when there is
+    no record or the kernel's sources changed since the capture."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "dram_traffic.json")) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    for e in rec.get("entries", []):
+        if e.get("label") != label or e.get("workload") != workload:
+            continue
+        h = hashlib.sha256()
+        try:
+            for src in e["sources"]:
+                with open(os.path.join(ROOT, src), "rb") as f:
+                    h.update(f.read())
+        except OSError:
+            return None
+        return e["bytes_per_launch"] if h.hexdigest() == e["sha256"] else None
+    return None
 
 
 # ---------------------------------------------------------------------------
