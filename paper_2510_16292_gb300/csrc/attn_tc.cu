@@ -434,9 +434,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     cluster_sync();                  // the peer's barriers exist before any remote arrive
     const uint32_t tmem = tmem_base;
     pdl_trigger();
-    pdl_wait();
 
-    const int L = p.seq_len[b];
+    const int L = p.seq_len[b];                       // an input: no kernel of the chain writes it
     const bool valid = L >= 1 && L <= c.Tmax;
     const int t_begin = split * p.tiles_per_split * kTile;
     const int t_end = valid ? min(L, t_begin + p.tiles_per_split * kTile) : t_begin;
@@ -444,31 +443,30 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     const size_t row0 = size_t(b) * c.Tmax;          // cache slot of token 0 of the sequence
     const int total = n_tiles * n_chunks;             // chunk loads per pass
     const int ngrp = r / 128;                         // int4 scale groups per token
+    // the first two tiles' chunks into L2 while the producer grid finishes (L2
+    // is the point of coherence, so a row the projection writes meanwhile is
+    // never seen stale: the shared-memory copies come after the wait)
+    constexpr int kPrefetchTiles = 2;
+    if (warp == 0 && lane == 0)
+        for (int i = 0; i < min(total, kPrefetchTiles * n_chunks); ++i)
+            tma_prefetch_2d(&map_c, (ch0 + (i % n_chunks) * kChunk) * BITS / 8, int(row0) + t_begin + (i / n_chunks) * kTile);
+    pdl_wait();
 
     // ---- query block: per-head power-of-two scale from the max over all r
     // channels (both CTAs of the pair get the same scale), then the fp16
     // block Q^T [heads][channels of this CTA], 128-byte swizzled, 64 channels
-    // per 128-byte row, blocks of Np rows.
-    if (n_tiles > 0) {
-        if (threadIdx.x < kMaxN) {
-            const int h = threadIdx.x;
-            int e = 0;
-            if (h < H) {
-                const float m = __uint_as_float(p.qmax[size_t(b) * H + h]);   // max_j |q~[b, h, j]|
-                if (m > 0.0f) frexpf(m, &e);                                   // m < 2^e
-            }
-            q_exp[h] = float(14 - e);                                          // |q~| * 2^(14-e) < 2^14
-            // scores -> logits in log2 units: undo the query scale, times softmax_scale * log2(e)
-            qfac[h] = exp2f(float(e - 14)) * p.softmax_scale * 1.4426950408889634f;
-            m_ref[h] = -INFINITY;
-        }
-        __syncthreads();
-        if (warp >= 4) {
-            // 8 channels per item; all loads of a thread are issued before its first conversion
-            constexpr int kPer = 4;
-            const int items = Np * (rc / 8);
-            for (int i0 = threadIdx.x - 128; i0 < items; i0 += kPer * (kThreads - 128)) {
-                float4 va[kPer], vb[kPer];
+    // per 128-byte row, blocks of Np rows.  Built by warps 4-27 and awaited by
+    // them and the MMA warps at named barrier 3; the TMA producers (warps 0 and
+    // 3) start streaming cache chunks at once.  The q~ loads are issued before
+    // the per-head scales are known.
+    constexpr int kQbThreads = kThreads - 64;          // every warp but 0 and 3
+    if (warp != 0 && warp != 3) {
+        if (n_tiles > 0) {
+            constexpr int kPer = 4;                     // items per thread: Np (rc / 8) <= 32 * 96 = kPer * 768
+            const int items = Np * (rc / 8);            // 8 channels per item
+            const int i0 = threadIdx.x - 128;
+            float4 va[kPer], vb[kPer];
+            if (warp >= 4) {
 #pragma unroll
                 for (int k = 0; k < kPer; ++k) {
                     const int i = i0 + k * (kThreads - 128);
@@ -480,6 +478,21 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                         vb[k] = src[1];
                     }
                 }
+            }
+            if (warp == 4) {
+                const int h = lane;
+                int e = 0;
+                if (h < H) {
+                    const float m = __uint_as_float(p.qmax[size_t(b) * H + h]);   // max_j |q~[b, h, j]|
+                    if (m > 0.0f) frexpf(m, &e);                                   // m < 2^e
+                }
+                q_exp[h] = float(14 - e);                                          // |q~| * 2^(14-e) < 2^14
+                // scores -> logits in log2 units: undo the query scale, times softmax_scale * log2(e)
+                qfac[h] = exp2f(float(e - 14)) * p.softmax_scale * 1.4426950408889634f;
+                m_ref[h] = -INFINITY;
+            }
+            asm volatile("bar.sync 3, %0;" ::"n"(kQbThreads) : "memory");
+            if (warp >= 4) {
 #pragma unroll
                 for (int k = 0; k < kPer; ++k) {
                     const int i = i0 + k * (kThreads - 128);
@@ -494,19 +507,21 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                         make_uint4(*reinterpret_cast<const uint32_t *>(&v0), *reinterpret_cast<const uint32_t *>(&v1),
                                    *reinterpret_cast<const uint32_t *>(&v2), *reinterpret_cast<const uint32_t *>(&v3));
                 }
+                fence_async_smem();
             }
-            fence_async_smem();
         }
+        asm volatile("bar.sync 3, %0;" ::"n"(kQbThreads) : "memory");
     }
-    __syncthreads();
 
     if (warp == 0) {
         // ---------------- TMA producer, pass 1 ----------------
         if (lane == 0 && total > 0) {
             int issued = 0;
-            // keep the chunks of the next two tiles streaming into L2
+            // keep the chunks of the next two tiles streaming into L2 (the first
+            // kPrefetchTiles were prefetched before the wait)
             const int ahead = 2 * n_chunks;
-            int pj = 0, pck = 0, ptile = 0;                 // next chunk to prefetch
+            int pj = min(total, kPrefetchTiles * n_chunks);  // next chunk to prefetch
+            int pck = pj % n_chunks, ptile = pj / n_chunks;
             auto prefetch = [&]() {
                 tma_prefetch_2d(&map_c, (ch0 + pck * kChunk) * BITS / 8, int(row0) + t_begin + ptile * kTile);
                 ++pj;
