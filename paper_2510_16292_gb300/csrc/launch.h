@@ -84,9 +84,12 @@ cudaError_t launch_proj_dp4a(const int8_t *xq, int64_t T, int d, const int8_t *w
                              const float *ws, const float *xs, int r, float *c_hat,
                              int32_t *acc_out, cudaStream_t s);
 
-// Decode-size projection (T <= kPsMaxTok): a1, a2, a3 and a4 in one launch.
-// `counter` must be zero before the first call; the kernel leaves it at zero.
+// Decode-size projection: for T < kPsSplitTok a1, a2, a3 and a4 in one launch
+// (`counter` must be zero before the first call; the kernel leaves it at zero);
+// up to kPsMaxSplitTok tokens on codes from xquant (xq_in, xs_in, tail = false),
+// kPsMaxTok tokens per CTA row.
 constexpr int kPsMaxTok = 16;
+constexpr int kPsMaxSplitTok = 64;
 cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, const int8_t *wcodes,
                               const float *ws, int r, int lat_bits, float lat_clip, float *c_hat, int *counter,
                               int8_t *xq_out, float *xs_out, int32_t *acc_out, void *lat_codes, void *lat_scales,

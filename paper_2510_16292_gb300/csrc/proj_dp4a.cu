@@ -3,9 +3,11 @@
 //   acc[t, j]   = sum_k xq[t, k] * w[j, k]          (exact: |acc| < 2^31)
 //   c_hat[t, j] = fp32(fp32(fp32(acc) * s_x[t]) * s_w[j])
 // proj_dp4a_kernel is the general CUDA-core path; proj_small_kernel is the
-// decode path (T <= kPsMaxTok tokens): it quantizes X itself, streams its 8
-// rows of W_d codes into shared memory with one bulk copy, and the last CTA
-// to finish requantizes the latent rows and stores them (a1-a4 in one launch).
+// decode path: for T < 4 tokens it quantizes X itself, streams its 8 rows of
+// W_d codes into shared memory with bulk copies, and the last CTA to finish
+// requantizes the latent rows and stores them (a1-a4 in one launch); for up to
+// kPsMaxSplitTok tokens it takes codes quantized by xquant_kernel, one
+// 16-token block per grid row, and leaves the requantization to requant_kernel.
 #include <algorithm>
 
 #include "common.cuh"
@@ -45,8 +47,9 @@ proj_dp4a_kernel(const int8_t *__restrict__ xq, int64_t T, int d, const int8_t *
 }
 
 // ---------------------------------------------------------------------------
-// Decode path.  CTA = 8 output channels (one warp each); every CTA quantizes
-// the T <= kPsMaxTok token rows itself (redundantly, they are tiny).
+// Decode path.  CTA = 8 output channels (one warp each) x one block of up to
+// kPsMaxTok tokens (grid row y: tokens [16 y, 16 y + 16)); without xq_in every
+// CTA quantizes its token rows itself (redundantly, they are tiny).
 // ---------------------------------------------------------------------------
 constexpr int kPsWarps = 8;
 constexpr int kPsMaxD = 6144;          // d <= 6144: 24 x 16-byte vectors per lane
@@ -61,6 +64,17 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                   int *err, const int8_t *__restrict__ xq_in, const float *__restrict__ xs_in, int tail) {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar, bar_x;
+    {   // this CTA's token block
+        const int tb = blockIdx.y * kPsMaxTok;
+        T = min(T - tb, kPsMaxTok);
+        X += size_t(tb) * d;
+        c_hat += size_t(tb) * r;
+        if (xq_in) xq_in += size_t(tb) * d;
+        if (xs_in) xs_in += tb;
+        if (xq_out) xq_out += size_t(tb) * d;
+        if (xs_out) xs_out += tb;
+        if (acc_out) acc_out += size_t(tb) * r;
+    }
     __shared__ float xs_s[kPsMaxTok];
     __shared__ float red[kPsWarps];
     __shared__ float red4[kPsWarps][4];
@@ -72,7 +86,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     int8_t *w_s = reinterpret_cast<int8_t *>(smem);                  // [kPsWarps][dp]
     int8_t *xq_s = reinterpret_cast<int8_t *>(smem) + kPsWarps * dp; // [T][dp]
     pdl_trigger();
-    prefetch_share_l2(w, size_t(r) * d, blockIdx.x, gridDim.x);
+    if (blockIdx.y == 0) prefetch_share_l2(w, size_t(r) * d, blockIdx.x, gridDim.x);
     if (threadIdx.x == 0) {
         mbar_init(&bar, 1);
         mbar_init(&bar_x, 1);
@@ -225,7 +239,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
             }
         }
     }
-    if (!tail) return;                   // the rows are requantized by the next kernel
+    if (!tail || gridDim.y > 1) return;  // the rows are requantized by the next kernel
     // second half of a3 + a4: the last CTA requantizes every row of c_hat
     __threadfence();
     __syncthreads();
@@ -252,10 +266,12 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
     CacheView dv{};
     if (dst) dv = *dst;
     // padded rows; the tensor-core path reuses the code rows for an [8][16][8] int32 reduction
-    const size_t smem = size_t(kPsWarps) * (d + 16) + std::max(size_t(T) * (d + 16), size_t(kPsWarps) * 16 * 8 * 4);
+    const int tb = std::min(T, kPsMaxTok);                       // tokens per CTA
+    const size_t smem = size_t(kPsWarps) * (d + 16) + std::max(size_t(tb) * (d + 16), size_t(kPsWarps) * 16 * 8 * 4);
     cudaError_t e = ensure_smem(proj_small_kernel, smem);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(proj_small_kernel, dim3((r + kPsWarps - 1) / kPsWarps), dim3(kPsWarps * 32), smem, s, X, T, d,
+    e = launch_pdl(proj_small_kernel, dim3((r + kPsWarps - 1) / kPsWarps, (T + kPsMaxTok - 1) / kPsMaxTok),
+                   dim3(kPsWarps * 32), smem, s, X, T, d,
                    act_clip, wcodes, ws, r, lat_bits, lat_clip, c_hat, counter, xq_out, xs_out, acc_out, lat_codes,
                    lat_scales, dv, dst_seq, dst_pos, err, xq_in, xs_in, int(tail));
     prof_mark(s, "proj_small");

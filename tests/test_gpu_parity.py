@@ -84,10 +84,11 @@ def test_project_tiny_bit_exact(tiny):
 
 
 @pytest.mark.parametrize("bits", [8, 4])
-@pytest.mark.parametrize("T", [1, 3, 4, 9, 16, 37, 640])
+@pytest.mark.parametrize("T", [1, 3, 4, 9, 16, 37, 64, 65, 640])
 def test_project_7b_bit_exact(l7b, bits, T):
-    """T <= 3: the decode projection quantizes with the whole CTA; 4 <= T <= 16:
-    a warp per token and the tensor-core dot products; larger T: the GEMM."""
+    """T <= 3: the decode projection quantizes with the whole CTA; 4 <= T <= 64:
+    xquant, the tensor-core dot products in 16-token blocks (a ragged last
+    block at 37), requant; larger T: the GEMM."""
     wl, inp, w = l7b
     W = q().qsvd_quantize_weight(torch.from_numpy(w["W_d"].astype(np.float32)).to(dev()))
     X = inp.X_prefill[0][:T]
