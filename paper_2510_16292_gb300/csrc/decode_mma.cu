@@ -14,7 +14,8 @@
 //
 // Like the CUDA-core kernels they replace at these batch sizes, each copies
 // its weight tile before waiting on the producer grid, and the cluster
-// partials are added in rank order (deterministic sums).
+// partials are added in rank order (deterministic sums).  Grid z runs the
+// 16-sequence passes side by side (each pass re-reads its weight tile from L2).
 #include <cfloat>
 #include <cuda_bf16.h>
 
@@ -80,7 +81,7 @@ __device__ __forceinline__ bool mlen_ok(int L, int Tmax) { return L >= 1 && L <=
 }  // namespace
 
 // ---------------------------------------------------------------------------
-// a5, q = c U_q.  Grid (kClQ, d / 64), cluster (kClQ, 1, 1), 128 threads.
+// a5, q = c U_q.  Grid (kClQ, d / 64, B / 16), cluster (kClQ, 1, 1), 128 threads.
 // CTA k of a cluster takes latent rows [k rs, (k+1) rs) (rs = r / kClQ, whole
 // 128-channel groups) and the cluster's 64 columns; warp w computes columns
 // 16w .. 16w+15 for 16 sequences per pass; rank k adds the kClQ partials of
@@ -108,10 +109,10 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
-    if (rank == 0 && blockIdx.y == 0)
+    if (rank == 0 && blockIdx.y == 0 && blockIdx.z == 0)
         for (int i = tid; i < n_qmax; i += 128) qmax[i] = 0u;
     bool ready = false;
-    for (int b0 = 0; b0 < B; b0 += 16) {
+    for (int b0 = 16 * int(blockIdx.z); b0 < B; b0 += 16 * int(gridDim.z)) {   // grid z: 16-sequence passes
         const int nb = min(16, B - b0);
         __syncthreads();
         if (tid < 16) {
@@ -224,7 +225,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
 }
 
 // ---------------------------------------------------------------------------
-// a5, q~ = U_k q.  Grid (r / 128, H), 128 threads: CTA (x, h) computes q~[b, h, j]
+// a5, q~ = U_k q.  Grid (r / 128, H, B / 16), 128 threads: CTA (x, h) computes q~[b, h, j]
 // for j in [128 x, 128 x + 128), warp w the 32 columns 32w .. 32w+31.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(128)
@@ -246,7 +247,7 @@ qabsorb_mma_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk,
     asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
     bool ready = false;
-    for (int b0 = 0; b0 < B; b0 += 16) {
+    for (int b0 = 16 * int(blockIdx.z); b0 < B; b0 += 16 * int(gridDim.z)) {   // grid z: 16-sequence passes
         const int nb = min(16, B - b0);
         __syncthreads();
         for (int i = tid; i < 16 * (dh / 4); i += 128) {     // A: q[b, h-block] as bf16 part + residual
@@ -311,7 +312,7 @@ qabsorb_mma_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk,
 }
 
 // ---------------------------------------------------------------------------
-// a7/a8.  Grid (kClV, H), cluster (kClV, 1, 1), 128 threads.  CTA k of head h's
+// a7/a8.  Grid (kClV, H, B / 16), cluster (kClV, 1, 1), 128 threads.  CTA k of head h's
 // cluster merges, for 16 sequences per pass, the softmax partials of latent
 // rows [k rs, (k+1) rs) (weights exp(m_s - M) / l), multiplies them by those
 // rows of U_v[:, h-block] (warp w: output columns 32w .. 32w+31), and rank k
@@ -343,7 +344,7 @@ combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ 
     pdl_wait();
     bool ready = false;
     const int per_rank = dh / kClV;
-    for (int b0 = 0; b0 < B; b0 += 16) {
+    for (int b0 = 16 * int(blockIdx.z); b0 < B; b0 += 16 * int(gridDim.z)) {   // grid z: 16-sequence passes
         const int nb = min(16, B - b0);
         __syncthreads();
         // merge weights: warp w takes sequences w, w+4, w+8, w+12
@@ -456,7 +457,7 @@ cudaError_t launch_qproj_mma(const CacheView &c, const int32_t *seq_len, const u
     const size_t smem = size_t(rs) * 72 * 2 + size_t(16) * (rs + 8) * 2 + size_t(16) * (rs / 128) * 4 + 16 * 64 * 4;
     cudaError_t e = ensure_smem(qproj_mma_kernel, smem);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(qproj_mma_kernel, dim3(kClQ, d / 64), dim3(128), smem, s, Uq, c, seq_len, c.B, d, q, qmax, n_qmax,
+    e = launch_pdl(qproj_mma_kernel, dim3(kClQ, d / 64, (c.B + 15) / 16), dim3(128), smem, s, Uq, c, seq_len, c.B, d, q, qmax, n_qmax,
                    err);
     prof_mark(s, "qproj");
     return e;
@@ -467,7 +468,7 @@ cudaError_t launch_qabsorb_mma(const float *q, const uint16_t *Uk, int B, int r,
     const size_t smem = size_t(128 + 32) * (dh + 8) * 2;
     cudaError_t e = ensure_smem(qabsorb_mma_kernel, smem);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(qabsorb_mma_kernel, dim3(r / 128, H), dim3(128), smem, s, q, Uk, B, r, d, H, dh, qt, qmax);
+    e = launch_pdl(qabsorb_mma_kernel, dim3(r / 128, H, (B + 15) / 16), dim3(128), smem, s, q, Uk, B, r, d, H, dh, qt, qmax);
     prof_mark(s, "qabsorb");
     return e;
 }
@@ -479,7 +480,7 @@ cudaError_t launch_combine_mma(const int32_t *seq_len, int B, int Tmax, int H, i
     const size_t smem = size_t(rs) * (dh + 8) * 2 + size_t(32) * (rs + 8) * 2 + size_t(16) * dh * 4;
     cudaError_t e = ensure_smem(combine_mma_kernel, smem);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(combine_mma_kernel, dim3(kClV, H), dim3(128), smem, s, Uv, seq_len, B, Tmax, H, dh, r, chunk,
+    e = launch_pdl(combine_mma_kernel, dim3(kClV, H, (B + 15) / 16), dim3(128), smem, s, Uv, seq_len, B, Tmax, H, dh, r, chunk,
                    n_split, pm, pl, po, O);
     prof_mark(s, "combine_uv");
     return e;
