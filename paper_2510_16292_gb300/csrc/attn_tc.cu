@@ -3,14 +3,14 @@
 // the softmax-weighted latent sum sum_t p_t c_t; W^u_v is applied afterwards
 // by combine_uv_kernel).
 //
-// Work unit: a cluster of two CTAs takes a contiguous range of 128-token tiles
-// of one sequence.  CTA k of the pair owns the latent channels
-// [k r/2, (k+1) r/2).  Per tile it computes partial scores over its channels,
-// the pair swaps them through distributed shared memory and both add them in
-// the same order, so both run the identical online softmax; each then
-// accumulates o_lat for its own channels.  Splitting the channels halves the
-// tensor-memory footprint of the o_lat accumulator and the bytes each SM
-// reads.
+// Work unit: a cluster of CL CTAs (CL = 2 for r <= 1536, 4 up to r = 3072)
+// takes a contiguous range of 128-token tiles of one sequence.  CTA k owns the
+// latent channels [k r/CL, (k+1) r/CL) (at most 768).  Per tile it computes
+// partial scores over its channels, sends them to every peer through
+// distributed shared memory and adds all CL partials in rank order, so every
+// CTA runs the identical online softmax; each then accumulates o_lat for its
+// own channels.  Splitting the channels bounds the tensor-memory footprint of
+// the o_lat accumulator and the bytes each SM reads.
 //
 // Both products take their A operand from tensor memory, so no fp16 copy of
 // the cache is ever written to or read from shared memory.  Per tile the CTA
@@ -21,7 +21,7 @@
 //              S[t, h] += C[t, ch] Q[ch, h]      (M = 128 tokens, N = heads,
 //           B = the fp16 query block in shared memory).
 //   softmax warpgroups 5-6 (thread = token, 16 heads each) read S, swap
-//           partials with the peer, apply the token scale and 1/sqrt(dh), run
+//           partials with the peers, apply the token scale and 1/sqrt(dh), run
 //           the online softmax (o_lat is rescaled lazily, only when the
 //           running maximum of a head grows by more than kRescale2) and write
 //           P (fp16, [heads x tokens]).
@@ -55,29 +55,37 @@ namespace atc {
 constexpr int kTile = 128;        // tokens per tile
 constexpr int kChunk = 128;       // channels per TMA chunk
 constexpr int kThreads = 896;     // 28 warps
-constexpr int kRing1 = 4;         // pass-1 TMA slots
-constexpr int kRing2 = 3;         // pass-2 TMA slots
 constexpr int kMaxN = 32;         // heads (padded to a multiple of 16)
 constexpr int kHalfN = 16;        // heads per softmax warpgroup
 constexpr int kMaxRc = 768;       // channels per CTA
-constexpr int kMaxGroups = 12;    // int4 scale groups per token (r <= 1536)
+constexpr int kMaxGroups = 24;    // int4 scale groups per token (r <= 3072)
 constexpr float kRescale2 = 11.5f;  // lazy rescale threshold (log2 units, about 8 in natural-log units)
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per wait
 
-// dynamic shared memory (byte offsets from a 1024-aligned base)
+// dynamic shared memory (byte offsets from a 1024-aligned base) of a cluster
+// of CL CTAs: the exchange buffer holds the CL - 1 peers' partial scores, and
+// a cluster of 4 pays for it with shallower TMA rings
 constexpr int kQtBytes = kMaxN * kMaxRc * 2;       // query block, fp16, 128-byte swizzled, K-major
 constexpr int kSlotBytes = kTile * kChunk;         // one int8 chunk (int4 uses half)
 constexpr int kPBytes = kMaxN * kTile * 2;         // P, fp16, 128-byte swizzled, K-major
-constexpr int kXchBytes = kTile * kMaxN * 4;       // the peer's partial scores
+constexpr int kXchSlot = kTile * kMaxN * 4;        // one peer's partial scores
 constexpr int kScBytes = kTile * kMaxGroups * 2;   // int4 group scales of one tile, [token][group]
-constexpr int kOffQt = 0;
-constexpr int kOffT1 = kOffQt + kQtBytes;
-constexpr int kOffT2 = kOffT1 + kRing1 * kSlotBytes;
-constexpr int kOffP = kOffT2 + kRing2 * kSlotBytes;
-constexpr int kOffXch = kOffP + 2 * kPBytes;
-constexpr int kOffSc = kOffXch + kXchBytes;
-constexpr int kOffLt = kOffSc + 2 * kScBytes;      // softmax running sums, [heads][tokens] fp32
-constexpr int kSmemBytes = kOffLt + kMaxN * kTile * 4 + 1024;
+template <int CL>
+struct Lay {
+    static constexpr int kRing1 = CL == 2 ? 4 : 3;    // pass-1 TMA slots
+    static constexpr int kRing2 = CL == 2 ? 3 : 2;    // pass-2 TMA slots
+    static constexpr int kOffQt = 0;
+    static constexpr int kOffT1 = kOffQt + kQtBytes;
+    static constexpr int kOffT2 = kOffT1 + kRing1 * kSlotBytes;
+    static constexpr int kOffP = kOffT2 + kRing2 * kSlotBytes;
+    static constexpr int kOffXch = kOffP + 2 * kPBytes;
+    static constexpr int kOffSc = kOffXch + (CL - 1) * kXchSlot;
+    static constexpr int kOffLt = kOffSc + 2 * kScBytes;   // softmax running sums, [heads][tokens] fp32
+    static constexpr int kSmemBytes = kOffLt + kMaxN * kTile * 4 + 1024;
+};
+static_assert(Lay<2>::kSmemBytes <= 227 * 1024 - 2048 && Lay<4>::kSmemBytes <= 227 * 1024 - 2048, "shared memory");
+// Cluster size for rank r: each CTA owns r / CL <= kMaxRc latent channels.
+__host__ __device__ constexpr int cluster_for(int r) { return r <= 2 * kMaxRc ? 2 : 4; }
 
 // tensor memory columns
 constexpr uint32_t kColO = 0;      // o_lat^T: (r_c / 128) x Np       (<= 192)
@@ -370,10 +378,12 @@ __device__ __forceinline__ uint16_t load_group_scale(const CacheView &c, size_t 
 }  // namespace atc
 
 // ---------------------------------------------------------------------------
-template <int BITS>
+template <int BITS, int CL>
 __global__ void __launch_bounds__(atc::kThreads, 1)
 attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     using namespace atc;
+    using Ly = Lay<CL>;
+    constexpr int kRing1 = Ly::kRing1, kRing2 = Ly::kRing2;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t t1_full[kRing1], t1_empty[kRing1], t2_full[kRing2], t2_empty[kRing2];
@@ -387,9 +397,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
 
     const CacheView &c = p.c;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t rank = cluster_rank(), peer = rank ^ 1u;
-    const int split = blockIdx.x >> 1, b = blockIdx.y;
-    const int r = c.r, rc = r / 2, ch0 = int(rank) * rc;
+    const uint32_t rank = cluster_rank();
+    const int split = blockIdx.x / CL, b = blockIdx.y;
+    const int r = c.r, rc = r / CL, ch0 = int(rank) * rc;
     const int n_chunks = rc / kChunk;
     const int Np = p.Np, H = p.H;
     constexpr uint32_t kLoadBytes = BITS == 8 ? kTile * kChunk : kTile * kChunk / 2;
@@ -413,8 +423,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             mbar_init(&sc_full[i], 32);     // one cp.async-tracked arrival per lane of warp 3
             mbar_init(&sc_empty[i], 8);
             mbar_init(&mma_done[i], 1);
-            mbar_init(&xch_full[i], 1);     // one local expect-tx arrival + the peer's st.async bytes
-            mbar_init(&xch_empty[i], 128);  // every thread of the peer's warpgroup, after reading
+            mbar_init(&xch_full[i], 1);     // one local expect-tx arrival + the peers' st.async bytes
+            mbar_init(&xch_empty[i], 128 * (CL - 1));   // every thread of each peer's warpgroup, after reading
         }
         for (int i = 0; i < kABufs; ++i) {
             mbar_init(&a_full[i], 4);
@@ -431,7 +441,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     fence_before();
     __syncthreads();
     fence_after();
-    cluster_sync();                  // the peer's barriers exist before any remote arrive
+    cluster_sync();                  // the peers' barriers exist before any remote arrive
     const uint32_t tmem = tmem_base;
     pdl_trigger();
 
@@ -503,7 +513,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                     const float4 a = va[k], bq = vb[k];
                     const __half2 v0 = __floats2half2_rn(a.x * sc, a.y * sc), v1 = __floats2half2_rn(a.z * sc, a.w * sc);
                     const __half2 v2 = __floats2half2_rn(bq.x * sc, bq.y * sc), v3 = __floats2half2_rn(bq.z * sc, bq.w * sc);
-                    *reinterpret_cast<uint4 *>(sm + kOffQt + kc * (Np * 128) + sw128(h, q)) =
+                    *reinterpret_cast<uint4 *>(sm + Ly::kOffQt + kc * (Np * 128) + sw128(h, q)) =
                         make_uint4(*reinterpret_cast<const uint32_t *>(&v0), *reinterpret_cast<const uint32_t *>(&v1),
                                    *reinterpret_cast<const uint32_t *>(&v2), *reinterpret_cast<const uint32_t *>(&v3));
                 }
@@ -533,7 +543,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 if (pj < total) prefetch();
                 if (i >= kRing1 && !wait(&t1_empty[s], ((i / kRing1) - 1) & 1, p.err)) { abort_flag = 1; break; }
                 mbar_arrive_expect_tx(&t1_full[s], kLoadBytes);
-                tma_load_2d(sm + kOffT1 + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
+                tma_load_2d(sm + Ly::kOffT1 + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
                             int(row0) + t_begin + tile * kTile, &t1_full[s]);
                 ++issued;
                 if (++ck == n_chunks) { ck = 0; ++tile; }
@@ -553,7 +563,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 // tokens past the end get zeros, so dead rows contribute 0, never NaN)
                 const int sl = tile & 1;
                 if (tile >= 2 && !wwait(&sc_empty[sl], ((tile >> 1) - 1) & 1, p.err)) { abort_flag = 1; break; }
-                uint8_t *dst = sm + kOffSc + sl * kScBytes;
+                uint8_t *dst = sm + Ly::kOffSc + sl * kScBytes;
                 const int nw = ngrp / 2;
                 for (int tt = lane; tt < kTile; tt += 32) {
                     const int tok = t_begin + tile * kTile + tt;
@@ -568,7 +578,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 if (i >= kRing2 && !wait(&t2_empty[s], ((i / kRing2) - 1) & 1, p.err)) ok = false;
                 if (ok) {
                     mbar_arrive_expect_tx(&t2_full[s], kLoadBytes);
-                    tma_load_2d(sm + kOffT2 + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
+                    tma_load_2d(sm + Ly::kOffT2 + s * kSlotBytes, &map_c, (ch0 + ck * kChunk) * BITS / 8,
                                 int(row0) + t_begin + tile * kTile, &t2_full[s]);
                 }
             }
@@ -593,7 +603,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                     const int ab = half % kABufs;
                     if (!wait(&a_full[ab], (half / kABufs) & 1, p.err)) { ok = false; break; }
                     fence_after();
-                    const uint32_t qblk = smem_addr(sm + kOffQt + hh * (Np * 128));
+                    const uint32_t qblk = smem_addr(sm + Ly::kOffQt + hh * (Np * 128));
 #pragma unroll
                     for (int k = 0; k < 4; ++k)
                         mma_ts(tmem + kColS + sb * 32, tmem + kColA + ab * 32 + k * 8, sdesc(qblk + k * 32, 16, 1024),
@@ -615,7 +625,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 const int pb = tile & 1;
                 if (!wait(&p_full[pb], (tile >> 1) & 1, p.err)) { abort_flag = 1; break; }
                 fence_after();
-                const uint32_t pbase = smem_addr(sm + kOffP + pb * kPBytes);
+                const uint32_t pbase = smem_addr(sm + Ly::kOffP + pb * kPBytes);
                 bool ok = true;
                 for (int ck = 0; ck < n_chunks; ++ck, ++chunk) {
                     const int vb = chunk & 1;
@@ -658,7 +668,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 if (tile + 1 < n_tiles) load_sc(tile + 1, scn);      // a tile ahead
             }
             if (!wwait(&t1_full[s], (i / kRing1) & 1, p.err)) { abort_flag = 1; break; }
-            const uint8_t *slot = sm + kOffT1 + s * kSlotBytes;
+            const uint8_t *slot = sm + Ly::kOffT1 + s * kSlotBytes;
             const int half = 2 * i + hh, ab = half % kABufs;
             bool ok = half < kABufs || wwait(&a_empty[ab], ((half / kABufs) - 1) & 1, p.err);
             if (ok) {
@@ -724,9 +734,9 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             if (!wwait(&t2_full[s], (i / kRing2) & 1, p.err)) { abort_flag = 1; break; }
             if (i >= 2 && !wwait(&pva_empty[vb], ((i >> 1) - 1) & 1, p.err)) { abort_flag = 1; break; }
             if (BITS == 4 && ck == 0 && !wwait(&sc_full[tile & 1], (tile >> 1) & 1, p.err)) { abort_flag = 1; break; }
-            const uint8_t *src = sm + kOffT2 + s * kSlotBytes;
+            const uint8_t *src = sm + Ly::kOffT2 + s * kSlotBytes;
             // this thread's group scales: token rbase + 8 j' (j' = 4 h32 + j), group grp
-            const __half *scs = reinterpret_cast<const __half *>(sm + kOffSc + (tile & 1) * kScBytes) +
+            const __half *scs = reinterpret_cast<const __half *>(sm + Ly::kOffSc + (tile & 1) * kScBytes) +
                                 rbase * ngrp + (ch0 / 128 + ck);
 #pragma unroll 1
             for (int h32 = 0; h32 < 2; ++h32) {             // 32 tokens: two 16x256b stores of 16 columns
@@ -800,13 +810,14 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
         const int hb = hg * kHalfN, bar_id = 1 + hg;
         const bool grp_live = hb < Np;                      // Np = 16: the second warpgroup has no heads
         const uint32_t trow = tmem + (uint32_t(quad * 32) << 16);
-        const uint32_t xch_remote = map_peer(smem_addr(sm + kOffXch), peer);
-        const uint32_t xfull_remote = map_peer(smem_addr(&xch_full[hg]), peer);
-        const uint32_t xempty_remote = map_peer(smem_addr(&xch_empty[hg]), peer);
-        // exchange buffer: the peer's partials as [head / 4][token][4] (conflict-free float4
-        // rows); warpgroup hg's half (heads 16 hg ..) is reused as [token][16] for its
-        // tile-maximum transposition once its partials are consumed
-        float *xr = reinterpret_cast<float *>(sm + kOffXch);
+        // exchange buffer: slot j holds the partials of peer rank + 1 + j (mod CL) as
+        // [head / 4][token][4] (conflict-free float4 rows); in slot 0, warpgroup hg's half
+        // (heads 16 hg ..) is reused as [token][16] for its tile-maximum transposition
+        // once its partials are consumed.  This CTA writes into slot CL - 2 - j of peer
+        // rank + 1 + j.
+        // (peer addresses are formed at each use: one mapa each, no live registers)
+        auto peer_of = [&](int j) { return (rank + 1u + uint32_t(j)) % uint32_t(CL); };
+        float *xr = reinterpret_cast<float *>(sm + Ly::kOffXch);
         const float *tscale = static_cast<const float *>(c.scales);
         float tsc_next = 0.0f;
         if (BITS == 8 && n_tiles > 0) tsc_next = t_begin + t < t_end ? tscale[row0 + t_begin + t] : 0.0f;
@@ -814,7 +825,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
         const int pcol = (t & 48) | kpos16(t & 15);
 
         // running sums of p per (head, token), kept in shared memory: [head][token]
-        float *lt = reinterpret_cast<float *>(sm + kOffLt) + hb * kTile + t;
+        float *lt = reinterpret_cast<float *>(sm + Ly::kOffLt) + hb * kTile + t;
 #pragma unroll
         for (int h = 0; h < kHalfN; ++h) lt[h * kTile] = 0.0f;
         bool failed = false;
@@ -842,25 +853,41 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
 #pragma unroll
                 for (int h = 0; h < kHalfN; ++h) s[h] = 0.0f;
             }
-            // swap partial scores with the peer: asynchronous stores that
+            // send the partial scores to every peer: asynchronous stores that
             // count their bytes on the peer's xch_full[hg], whose phase also
             // needs the peer's own expect-tx arrival
-            if (t == 0 && !bad) mbar_arrive_expect_tx(&xch_full[hg], kTile * kHalfN * 4);
+            if (t == 0 && !bad) mbar_arrive_expect_tx(&xch_full[hg], (CL - 1) * kTile * kHalfN * 4);
             if (!bad && tile > 0) bad = !wwait_cluster(&xch_empty[hg], (tile - 1) & 1, p.err);
             if (!bad) {
 #pragma unroll
-                for (int h = 0; h < kHalfN; h += 4)
-                    st_async_v4(xch_remote + (((hb + h) >> 2) * kTile + t) * 16, s[h], s[h + 1], s[h + 2], s[h + 3], xfull_remote);
+                for (int j = 0; j < CL - 1; ++j) {
+                    const uint32_t dst = map_peer(smem_addr(sm + Ly::kOffXch + (CL - 2 - j) * kXchSlot), peer_of(j));
+                    const uint32_t bar = map_peer(smem_addr(&xch_full[hg]), peer_of(j));
+#pragma unroll
+                    for (int h = 0; h < kHalfN; h += 4)
+                        st_async_v4(dst + (((hb + h) >> 2) * kTile + t) * 16, s[h], s[h + 1], s[h + 2], s[h + 3], bar);
+                }
                 bad = !wwait_cluster(&xch_full[hg], tile & 1, p.err);
             }
             bool exceed = false;
             if (!bad) {
+                // the partials of ranks 0, 1, .., CL - 1 added in rank order: the same sums on every CTA
 #pragma unroll
                 for (int h = 0; h < kHalfN; h += 4) {
-                    const float4 o = *reinterpret_cast<const float4 *>(xr + (((hb + h) >> 2) * kTile + t) * 4);
-                    // rank 0 computes own + peer, rank 1 peer + own: the same sums on both CTAs
-                    if (rank == 0) { s[h] += o.x; s[h + 1] += o.y; s[h + 2] += o.z; s[h + 3] += o.w; }
-                    else { s[h] = o.x + s[h]; s[h + 1] = o.y + s[h + 1]; s[h + 2] = o.z + s[h + 2]; s[h + 3] = o.w + s[h + 3]; }
+                    float4 tot = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                    for (int q = 0; q < CL; ++q) {
+                        float4 o;
+                        if (q == int(rank)) {
+                            o = make_float4(s[h], s[h + 1], s[h + 2], s[h + 3]);
+                        } else {
+                            const int slot = (q - int(rank) - 1 + CL) % CL;
+                            o = *reinterpret_cast<const float4 *>(xr + slot * (kXchSlot / 4) + (((hb + h) >> 2) * kTile + t) * 4);
+                        }
+                        if (q == 0) tot = o;
+                        else { tot.x += o.x; tot.y += o.y; tot.z += o.z; tot.w += o.w; }
+                    }
+                    s[h] = tot.x; s[h + 1] = tot.y; s[h + 2] = tot.z; s[h + 3] = tot.w;
                 }
                 // logits in log2 units; dead tokens and padding heads get -inf
 #pragma unroll
@@ -925,10 +952,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                     }
                 }
             }
-            arrive_peer_relaxed(xempty_remote);   // this thread's reads of the exchange buffer have completed
+#pragma unroll
+            for (int j = 0; j < CL - 1; ++j)      // this thread's reads of the exchange buffer have completed
+                arrive_peer_relaxed(map_peer(smem_addr(&xch_empty[hg]), peer_of(j)));
             if (!bad && tile >= 2) bad = !wwait(&p_empty[sb], ((tile >> 1) - 1) & 1, p.err);
             // P^T [heads][tokens], 64-token blocks of Np rows x 128 bytes, swizzled
-            uint8_t *pbuf = sm + kOffP + sb * kPBytes + (t >> 6) * (Np * 128);
+            uint8_t *pbuf = sm + Ly::kOffP + sb * kPBytes + (t >> 6) * (Np * 128);
             // three passes (loads, then read-modify-writes, then stores only) so that
             // no shared-memory load waits behind a store it might alias
 #pragma unroll
@@ -959,7 +988,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             group_sync(bar_id);
             {
                 // lane: head lane & 15 over tokens (lane >> 4) + 2j of the warp's 32
-                const float *lrow = reinterpret_cast<const float *>(sm + kOffLt) + (hb + (lane & 15)) * kTile + wq * 32;
+                const float *lrow = reinterpret_cast<const float *>(sm + Ly::kOffLt) + (hb + (lane & 15)) * kTile + wq * 32;
                 float sum = 0.0f;
 #pragma unroll
                 for (int j = 0; j < 16; ++j) sum += lrow[(lane >> 4) + 2 * j];
@@ -1027,10 +1056,10 @@ void set_attn_path(int path) { g_attn_path = path; }
 int attn_path() { return g_attn_path; }
 
 bool attn_tc_shape_ok(int r, int bits, int H) {
-    const int Np = (H + 15) / 16 * 16;
+    const int Np = (H + 15) / 16 * 16, cl = atc::cluster_for(r);
     if (bits != 8 && bits != 4) return false;
-    if (r % 256 || r / 2 > atc::kMaxRc || Np > atc::kMaxN) return false;
-    return (r / 2 / atc::kChunk) * Np <= int(atc::kColS - atc::kColO);
+    if (r % (cl * atc::kChunk) || r / cl > atc::kMaxRc || r / 128 > atc::kMaxGroups || Np > atc::kMaxN) return false;
+    return (r / cl / atc::kChunk) * Np <= int(atc::kColS - atc::kColO);
 }
 
 bool attn_tc_use(const CacheView &c, int H, int max_seq_len) {
@@ -1039,12 +1068,12 @@ bool attn_tc_use(const CacheView &c, int H, int max_seq_len) {
     return int64_t(c.B) * max_seq_len >= 4096;
 }
 
-int attn_tc_splits(int B, int max_seq_len, int *tiles_per_split) {
+int attn_tc_splits(int B, int r, int max_seq_len, int *tiles_per_split) {
     int dev = 0, sms = 148;
     if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int tiles = (max_seq_len + atc::kTile - 1) / atc::kTile;
-    const int64_t pairs = sms / 2;                   // CTA pairs resident at once
-    // tiles per split: the fewest tile steps of the busiest pair, counting the
+    const int64_t pairs = sms / atc::cluster_for(r); // clusters resident at once (one CTA per SM)
+    // tiles per split: the fewest tile steps of the busiest cluster, counting the
     // fixed cost of a wave (set-up, pipeline fill and drain, partial stores) as
     // 3.5 tile steps, measured on GB300 (~7 us per tile step, ~26 us per wave at
     // B = 16, L = 4096); at most 64 partials per sequence
@@ -1084,29 +1113,27 @@ cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const flo
         return cudaErrorInvalidValue;
     const atc::Params prm{c, seq_len, qt, qmax, H, (H + 15) / 16 * 16, softmax_scale, tiles_per_split, n_split,
                           pm, pl, po, err};
+    const int cl = atc::cluster_for(c.r);
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2 * n_split, c.B);
+    cfg.gridDim = dim3(cl * n_split, c.B);
     cfg.blockDim = dim3(atc::kThreads);
-    cfg.dynamicSmemBytes = atc::kSmemBytes;
+    cfg.dynamicSmemBytes = cl == 2 ? atc::Lay<2>::kSmemBytes : atc::Lay<4>::kSmemBytes;
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.x = cl;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    cudaError_t e;
-    if (c.bits == 8) {
-        e = ensure_smem(attn_tc_kernel<8>, atc::kSmemBytes);
-        if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, attn_tc_kernel<8>, map, prm);
-    } else {
-        e = ensure_smem(attn_tc_kernel<4>, atc::kSmemBytes);
-        if (e == cudaSuccess) e = cudaLaunchKernelEx(&cfg, attn_tc_kernel<4>, map, prm);
-    }
-    return e;
+    auto go = [&](auto kern) {
+        cudaError_t e = ensure_smem(kern, cfg.dynamicSmemBytes);
+        return e == cudaSuccess ? cudaLaunchKernelEx(&cfg, kern, map, prm) : e;
+    };
+    if (c.bits == 8) return cl == 2 ? go(attn_tc_kernel<8, 2>) : go(attn_tc_kernel<8, 4>);
+    return cl == 2 ? go(attn_tc_kernel<4, 2>) : go(attn_tc_kernel<4, 4>);
 }
 
 }  // namespace qsvd

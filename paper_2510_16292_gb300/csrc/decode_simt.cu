@@ -326,7 +326,7 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
     } else if (attn_tc_use(c, H, a.max_seq_len)) {
         // a6/a7 on the tensor cores: splits of whole 128-token tiles
         int per = 1;
-        ns = attn_tc_splits(B, a.max_seq_len, &per);
+        ns = attn_tc_splits(B, c.r, a.max_seq_len, &per);
         chunk = per * 128;
         e = launch_attn_tc(c, a.seq_len, w.qt, w.qmax, H, a.softmax_scale, per, ns, w.pm, w.pl, w.po, err, s);
         if (e != cudaSuccess) return e;

@@ -167,7 +167,7 @@ void set_attn_path(int path);      // 0 automatic, 1 CUDA cores, 2 tcgen05 where
 int attn_path();
 bool attn_tc_shape_ok(int r, int bits, int H);
 bool attn_tc_use(const CacheView &c, int H, int max_seq_len);
-int attn_tc_splits(int B, int max_seq_len, int *tiles_per_split);
+int attn_tc_splits(int B, int r, int max_seq_len, int *tiles_per_split);
 // Warp-level tensor-core attention for small batch x length (attn_mma.cu).
 bool attn_mma_use(const CacheView &c, int H, int B, int max_seq_len);
 bool attn_mma_fits(const CacheView &c, int max_seq_len);

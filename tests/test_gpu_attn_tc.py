@@ -105,6 +105,22 @@ def test_attn_tc_head_and_rank_shapes(H, dh, r, bits):
     _run(H, dh, r, bits, [300, 64, 1000], seed=2)
 
 
+@pytest.mark.parametrize("H,dh,r,bits,lens", [(32, 128, 2048, 8, [300, 129, 1000]), (32, 128, 3072, 4, [700, 1]),
+                                               (16, 128, 2560, 8, [257, 900]), (32, 128, 2048, 4, [128, 640])])
+def test_attn_tc_cluster_of_four(H, dh, r, bits, lens):
+    """r > 1536: four CTAs per cluster (r/4 channels each, 4-6 chunks), every
+    CTA sends its partial scores to three peers and adds all four in rank
+    order; r = 2560 gives five chunks per CTA and N = 16."""
+    _run(H, dh, r, bits, lens, paths=(2,), seed=21)
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_attn_tc_cluster_of_four_long_sequence(bits):
+    """r = 3072: one 6000-token sequence over several tiles per cluster with
+    late high scores (o_lat rescaling in all four CTAs)."""
+    _run(32, 128, 3072, bits, [6000], paths=(2,), hot=(0.1, 0.55, 0.97), seed=22)
+
+
 def test_attn_tc_cache_larger_than_lengths():
     """Tmax above every length: the rows after each sequence's end belong to
     no token and must not contribute."""
