@@ -57,9 +57,11 @@ def parse():
     p.add_argument("--no-prefill13", action="store_true")
     p.add_argument("--workload", default=WORKLOAD, choices=sorted(synthetic.WORKLOADS))
     p.add_argument("--decode-steps", type=int, default=0, help="override the workload's decode steps")
-    p.add_argument("--sweep", choices=["quick", "full"], default=None,
+    p.add_argument("--sweep", choices=["quick", "full", "point"], default=None,
                    help="sweep the 7B-shaped layer over rank, cached length, batch and cache precision (one JSON "
-                        "line per point) instead of the benchmark")
+                        "line per point) instead of the benchmark; 'point' runs the one point of --sweep-point")
+    p.add_argument("--sweep-point", default="1536,4096,16,4", metavar="R,L,B,BITS",
+                   help="rank, cached length, batch, cache bits of --sweep point")
     p.add_argument("--l2", default="rotate", choices=["rotate", "flush"],
                    help="cold-L2 method: rotate through copies of the layer larger than L2 together, or flush "
                         "L2 before every sub-step")
@@ -695,7 +697,11 @@ def run_sweep(args):
     import paper_2510_16292_gb300 as q
     dev = torch.device("cuda", torch.cuda.current_device())
     hbm, _, peak_kind = peaks()
-    grid = SWEEP_FULL if args.sweep == "full" else SWEEP_QUICK
+    if args.sweep == "point":
+        r_, L_, B_, bits_ = (int(v) for v in args.sweep_point.split(","))
+        grid = dict(r=(r_,), L=(L_,), B=(B_,), bits=(bits_,))
+    else:
+        grid = SWEEP_FULL if args.sweep == "full" else SWEEP_QUICK
     d, H, dh = 4096, 32, 128
     g = torch.Generator(device=dev)
     g.manual_seed(2510)
