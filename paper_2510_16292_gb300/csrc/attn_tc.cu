@@ -17,7 +17,9 @@
 // streams its channels twice (the second stream hits L2):
 //   pass 1  warp 0 loads 128-token x 128-channel chunks with TMA; warpgroups
 //           1-2 (thread = token, one 64-channel half each) convert them to
-//           fp16 and store them into tensor memory token-major; warp 1 issues
+//           fp16 and store them into tensor memory token-major (int4: a word
+//           of 8 codes at a time, channels in the order 0,4,1,5,2,6,3,7 of
+//           each 8, the query block in the same order); warp 1 issues
 //              S[t, h] += C[t, ch] Q[ch, h]      (M = 128 tokens, N = heads,
 //           B = the fp16 query block in shared memory).
 //   softmax warpgroups 5-6 (thread = token, 16 heads each) read S, swap
@@ -318,6 +320,26 @@ __device__ __forceinline__ void i4x8_to_h2x4(uint32_t w, __half2 s2, uint32_t *o
     }
 }
 
+// Eight int4 codes (element i in bits 4i..4i+3, two's complement) times an
+// fp16 group scale -> four fp16 pairs in the order (0,4), (1,5), (2,6), (3,7)
+// (products rounded to nearest).  The nibbles xor 8 are placed in the
+// mantissas of 1024 and 1024 * 16; one add or fused multiply-add maps them
+// back to the codes exactly.
+__device__ __forceinline__ void i4x8_h2x4_perm(uint32_t w, __half2 s2, uint32_t (&o)[4]) {
+    const uint32_t y = w >> 8;
+    const uint32_t z[4] = {(w & 0x000F000Fu) ^ 0x64086408u, (w & 0x00F000F0u) ^ 0x64806480u,
+                           (y & 0x000F000Fu) ^ 0x64086408u, (y & 0x00F000F0u) ^ 0x64806480u};
+    const __half2 b_lo = __half2half2(__ushort_as_half(0xE408));     // -1032
+    const __half2 m_hi = __half2half2(__ushort_as_half(0x2C00));     // 1/16
+    const __half2 b_hi = __half2half2(__ushort_as_half(0xD480));     // -72
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const __half2 zk = *reinterpret_cast<const __half2 *>(&z[k]);
+        const __half2 c = (k & 1) ? __hfma2(zk, m_hi, b_hi) : __hadd2(zk, b_lo);
+        const __half2 h = __hmul2(c, s2);
+        o[k] = *reinterpret_cast<const uint32_t *>(&h);
+    }
+}
 // Byte k of w (two int4 codes, the even channel in the low nibble) -> the fp16
 // pair (code_even * s, code_odd * s), products rounded to nearest.  The nibbles
 // (xor 8) are placed in the mantissas of 1024 and 1024 * 16, which the fused
@@ -511,8 +533,11 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                     const int kc = q8 >> 3, q = q8 & 7;
                     const float sc = exp2f(q_exp[h]);
                     const float4 a = va[k], bq = vb[k];
-                    const __half2 v0 = __floats2half2_rn(a.x * sc, a.y * sc), v1 = __floats2half2_rn(a.z * sc, a.w * sc);
-                    const __half2 v2 = __floats2half2_rn(bq.x * sc, bq.y * sc), v3 = __floats2half2_rn(bq.z * sc, bq.w * sc);
+                    // int4: the order of the pass-1 operand, 0,4,1,5,2,6,3,7 within each 8 channels
+                    const __half2 v0 = BITS == 4 ? __floats2half2_rn(a.x * sc, bq.x * sc) : __floats2half2_rn(a.x * sc, a.y * sc);
+                    const __half2 v1 = BITS == 4 ? __floats2half2_rn(a.y * sc, bq.y * sc) : __floats2half2_rn(a.z * sc, a.w * sc);
+                    const __half2 v2 = BITS == 4 ? __floats2half2_rn(a.z * sc, bq.z * sc) : __floats2half2_rn(bq.x * sc, bq.y * sc);
+                    const __half2 v3 = BITS == 4 ? __floats2half2_rn(a.w * sc, bq.w * sc) : __floats2half2_rn(bq.z * sc, bq.w * sc);
                     *reinterpret_cast<uint4 *>(sm + Ly::kOffQt + kc * (Np * 128) + sw128(h, q)) =
                         make_uint4(*reinterpret_cast<const uint32_t *>(&v0), *reinterpret_cast<const uint32_t *>(&v1),
                                    *reinterpret_cast<const uint32_t *>(&v2), *reinterpret_cast<const uint32_t *>(&v3));
@@ -698,9 +723,12 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                     } else {
                         const uint32_t ww[4] = {wl[q].x, wl[q].y, wl[q].z, wl[q].w};   // 32 codes
 #pragma unroll
-                        for (int j = 0; j < 4; ++j)
+                        for (int j = 0; j < 4; ++j) {    // channels 8j..8j+7 in the order 0,4,1,5,2,6,3,7
+                            uint32_t o4[4];
+                            i4x8_h2x4_perm(ww[j], s2, o4);
 #pragma unroll
-                            for (int k = 0; k < 4; ++k) v[j * 4 + k] = i4pair_h2(ww[j], k, s2);
+                            for (int k = 0; k < 4; ++k) v[j * 4 + k] = o4[k];
+                        }
                     }
                     tmem_st16(trow + kColA + ab * 32 + q * 16, v);
                 }
