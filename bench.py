@@ -474,6 +474,27 @@ def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
             "peak_kind": kind}
 
 
+def cross_rank(values, op="max"):
+    """Per-rank totals reduced over the ranks of the default process group
+    (max: the job takes as long as its slowest rank; min: the slowest rank's
+    throughput).  Without a process group, or with one rank, the values are
+    returned unchanged."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in values]
+    dev = torch.device("cuda", torch.cuda.current_device()) if dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX if op == "max" else dist.ReduceOp.MIN)
+    return [float(v) for v in t.cpu()]
+
+
+def job_throughput(units_per_rank, world, slowest_seconds):
+    """Whole-job throughput: the units every rank processed over the slowest
+    rank's time (weak scaling: each rank runs its own replica)."""
+    return units_per_rank * world / slowest_seconds
+
+
 def run_native(args, rank, world, local_rank):
     import torch
     torch.cuda.set_device(local_rank)
@@ -507,13 +528,8 @@ def run_native(args, rank, world, local_rank):
         torch.distributed.barrier()
     t_wall = time.perf_counter() - t_wall
     clk = clocks.stop()
-    dec_total, pre_total = sum(dec), sum(pre)
-    if world > 1:
-        tt = torch.tensor([dec_total, pre_total], dtype=torch.float64, device=nb.dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        dec_total, pre_total = float(tt[0]), float(tt[1])
-    dec_tokens = world * wl.B * S * K * args.steps      # tokens through one copy of the layer, all copies
-    value = dec_tokens / dec_total
+    dec_total, pre_total = cross_rank([sum(dec), sum(pre)], "max")
+    value = job_throughput(wl.B * S * K * args.steps, world, dec_total)
     s = wl.shape
     prefill_ops = 2 * wl.B * wl.prefill * s.d * s.r
     prefill_tops = world * K * prefill_ops * args.steps / pre_total / 1e12
@@ -542,10 +558,7 @@ def run_native(args, rank, world, local_rank):
     e2e = None
     if not args.no_e2e:
         e2e_val, h2d, d2h = nb.e2e(steps=min(args.steps, 3), warmup=1)
-        if world > 1:
-            tt = torch.tensor([e2e_val], dtype=torch.float64, device=nb.dev)
-            torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MIN)
-            e2e_val = float(tt[0]) * world
+        e2e_val = cross_rank([e2e_val], "min")[0] * world     # the slowest rank's rate, every rank
         e2e = {"value": round(e2e_val, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h}
 

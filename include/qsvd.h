@@ -269,6 +269,17 @@ int qsvd_set_decode_attn_path(int32_t path);
  */
 int qsvd_check(cudaStream_t stream);
 
+/*
+ * Failure-detection self-test (no counterpart in the paper).  Enqueues on
+ * `stream` one thread that waits on an mbarrier no one arrives on for at
+ * most timeout_ms milliseconds (1..1000), then sets the timeout bit of the
+ * device error word and returns: the path every bounded device wait of the
+ * library takes when it expires.  The next qsvd_check returns QSVD_ETIMEOUT
+ * and clears the word; the CUDA context stays usable.  Returns QSVD_EINVAL
+ * for a timeout outside 1..1000.
+ */
+int qsvd_selftest_wait_timeout(int32_t timeout_ms, cudaStream_t stream);
+
 /* Message of the last failure on the calling thread ("" if none). */
 const char *qsvd_last_error(void);
 

@@ -33,7 +33,7 @@ EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspac
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
            "qsvd_decode_step", "qsvd_decode_step_workspace_bytes", "qsvd_latent_project_static",
            "qsvd_set_decode_attn_path", "qsvd_set_project_epilogue", "qsvd_check", "qsvd_last_error",
-           "qsvd_version")
+           "qsvd_selftest_wait_timeout", "qsvd_version")
 
 
 class QsvdError(RuntimeError):
@@ -261,6 +261,15 @@ def qsvd_check(stream=None) -> int:
     st = _lib.qsvd_check(_stream(stream))
     _check(st)
     return st
+
+
+_lib.qsvd_selftest_wait_timeout.argtypes = [_i32, _vp]
+
+
+def qsvd_selftest_wait_timeout(timeout_ms: int = 5, stream=None) -> None:
+    """Enqueue a bounded device wait that expires after `timeout_ms`; the next
+    qsvd_check raises QsvdError with status QSVD_ETIMEOUT."""
+    _check(_lib.qsvd_selftest_wait_timeout(timeout_ms, _stream(stream)))
 
 
 def qsvd_version() -> int:

@@ -222,6 +222,16 @@ int qsvd_check(cudaStream_t stream) {
     return QSVD_OK;
 }
 
+int qsvd_selftest_wait_timeout(int32_t timeout_ms, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (timeout_ms < 1 || timeout_ms > 1000) return fail(QSVD_EINVAL, "selftest_wait_timeout: timeout_ms outside 1..1000");
+    prof_mark(stream, "begin");
+    cudaError_t e = launch_selftest_wait(static_cast<unsigned long long>(timeout_ms) * 1000000ull, err, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "selftest launch");
+}
+
 int qsvd_quantize_weight(const float *W_d, int32_t d, int32_t r, float clip, int8_t *codes,
                          uint16_t *codes_bf16, float *scale, cudaStream_t stream) {
     int *err = nullptr;

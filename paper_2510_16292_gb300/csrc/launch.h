@@ -199,4 +199,7 @@ cudaError_t launch_decode_fused(const FusedArgs &a, void *ws, size_t ws_bytes, i
 cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *err,
                           cudaStream_t s);
 
+// Failure-detection self-test: a bounded wait on a barrier nothing completes.
+cudaError_t launch_selftest_wait(unsigned long long limit_ns, int *err, cudaStream_t s);
+
 }  // namespace qsvd

@@ -174,4 +174,32 @@ cudaError_t launch_append(const CacheView &c, const int32_t *seq, const int32_t 
     return e;
 }
 
+// ---------------------------------------------------------------------------
+// Failure-detection self-test: one thread waits on an mbarrier that nothing
+// arrives on until `limit_ns` of globaltimer have passed, then sets the
+// timeout bit of the device error word and returns, as every bounded wait of
+// the library does when it expires.
+// ---------------------------------------------------------------------------
+__global__ void selftest_wait_kernel(unsigned long long limit_ns, int *err) {
+    __shared__ __align__(8) uint64_t bar;
+    mbar_init(&bar, 1);
+    mbar_init_fence();
+    unsigned long long t0, t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+    for (;;) {
+        if (mbar_try_wait(&bar, 0)) return;                 // never: no arrival is ever made
+        asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+        if (t - t0 > limit_ns) {
+            flag_error(err, kErrTimeout);
+            return;
+        }
+    }
+}
+
+cudaError_t launch_selftest_wait(unsigned long long limit_ns, int *err, cudaStream_t s) {
+    selftest_wait_kernel<<<1, 1, 0, s>>>(limit_ns, err);
+    prof_mark(s, "selftest_wait");
+    return cudaGetLastError();
+}
+
 }  // namespace qsvd

@@ -279,6 +279,26 @@ def test_error_paths(tiny):
     assert e.value.status == lib.QSVD_ERANGE
 
 
+def test_bounded_wait_expiry_is_reported():
+    """Failure detection without a fault: a bounded device wait on a barrier
+    nothing completes expires after 5 ms, sets the timeout bit, and qsvd_check
+    reports QSVD_ETIMEOUT once; the context keeps running kernels after it."""
+    lib = q()
+    lib.qsvd_check()
+    lib.qsvd_selftest_wait_timeout(5)
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_check()
+    assert e.value.status == lib.QSVD_ETIMEOUT
+    assert lib.qsvd_check() == lib.QSVD_OK          # the word was cleared
+    for bad in (0, 1001):
+        with pytest.raises(lib.QsvdError) as e:
+            lib.qsvd_selftest_wait_timeout(bad)
+        assert e.value.status == lib.QSVD_EINVAL
+    W = lib.qsvd_quantize_weight(torch.ones((64, 16), dtype=torch.float32, device=dev()))
+    assert lib.qsvd_check() == lib.QSVD_OK
+    assert int(W.codes.abs().max()) == 127
+
+
 # ---------------------------------------------------------------------------
 # tensor-core projection: exactness at the extremes of the int8 range
 # ---------------------------------------------------------------------------
