@@ -121,6 +121,56 @@ def test_attn_tc_cluster_of_four_long_sequence(bits):
     _run(32, 128, 3072, bits, [6000], paths=(2,), hot=(0.1, 0.55, 0.97), seed=22)
 
 
+@pytest.mark.parametrize("bits", [4, 8])
+def test_decode7b_full_size_sampled(bits):
+    """The decode-heavy 7B shape at full size, in the launch configuration the
+    benchmark times (automatic path: the tcgen05 kernel, one wave of CTA pairs
+    over 9-tile splits): B = 16 sequences of 4097 cached tokens, r = 1536,
+    H = 32.  Sequences 0, 9 and 15 hold oracle-quantized latent rows with late
+    high-score tokens and are checked against the oracle; the other 13 hold
+    seeded random codes and scales (they share the launch, not the check)."""
+    lib = q()
+    B, L, r, H, dh = 16, 4097, 1536, 32, 128
+    checked = (0, 9, 15)
+    U_q, U_k, U_v = _up_weights(H, dh, r, seed=31)
+    rng = np.random.default_rng(32)
+    cache = lib.LatentCache.empty(B, L, r, bits, dev())
+    g = torch.Generator(device=dev()).manual_seed(33)
+    if bits == 8:
+        cache.codes.copy_(torch.randint(-127, 128, cache.codes.shape, generator=g, device=dev(), dtype=torch.int8))
+        cache.scales.copy_(torch.rand(cache.scales.shape, generator=g, device=dev()) * 0.01 + 0.005)
+    else:
+        cache.codes.copy_(torch.randint(0, 256, cache.codes.shape, generator=g, device=dev(), dtype=torch.uint8))
+        cache.scales.copy_((torch.rand(cache.scales.shape, generator=g, device=dev()) * 0.2 + 0.05).half())
+    refs = []
+    for b in checked:
+        x = synthetic.latent_rows(L, r, rng)
+        for f in (0.05, 0.5, 0.93):
+            x[int(f * (L - 1))] = x[L - 1]
+        if bits == 8:
+            codes, sc = quant.quantize_rows(x, 8)
+            C = quant.dequantize_rows(codes, sc)
+            cache.codes[b] = torch.from_numpy(codes.astype(np.int8)).to(dev())
+            cache.scales[b] = torch.from_numpy(sc.astype(np.float32)).to(dev())
+        else:
+            codes, s16 = quant.quantize_int4_groups(x)
+            C = quant.dequantize_int4_groups(codes, s16)
+            cache.codes[b] = torch.from_numpy(quant.pack_int4(codes)).to(dev())
+            cache.scales[b] = torch.from_numpy(s16.astype(np.float16)).to(dev())
+        refs.append(attention.decode_attention_absorbed(
+            C, synthetic.bf16_from_bits(U_q), synthetic.bf16_from_bits(U_k), synthetic.bf16_from_bits(U_v), H, dh))
+    O = torch.full((B, H * dh), float("nan"), dtype=torch.float32, device=dev())
+    prev = lib.qsvd_set_decode_attn_path(0)
+    try:
+        lib.qsvd_latent_decode_attn(cache, i32([L] * B), L, bf16(U_q), bf16(U_k), bf16(U_v), H, dh, O)
+        lib.qsvd_check()
+    finally:
+        lib.qsvd_set_decode_attn_path(prev)
+    got = O.cpu().numpy()
+    assert np.isfinite(got).all()
+    assert_rows_close(got[list(checked)], np.stack(refs), "decode7b full size")
+
+
 def test_attn_tc_cache_larger_than_lengths():
     """Tmax above every length: the rows after each sequence's end belong to
     no token and must not contribute."""
