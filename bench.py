@@ -55,7 +55,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-prefill13", action="store_true")
-    p.add_argument("--workload", default=WORKLOAD, choices=sorted(synthetic.WORKLOADS))
+    # the tiny layer's W_d and U come from the oracle's joint SVD: it is a parity case (tests/), not a benchmark
+    p.add_argument("--workload", default=WORKLOAD, choices=sorted(k for k in synthetic.WORKLOADS if k != "tiny"))
     p.add_argument("--decode-steps", type=int, default=0, help="override the workload's decode steps")
     p.add_argument("--sweep", choices=["quick", "full", "point"], default=None,
                    help="sweep the 7B-shaped layer over rank, cached length, batch and cache precision (one JSON "

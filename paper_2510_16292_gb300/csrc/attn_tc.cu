@@ -42,6 +42,7 @@
 // Every wait is bounded in time (on expiry the error word gets kErrTimeout and
 // the CTA abandons its tiles); a CTA always drains its own copies and MMAs,
 // meets its peer at the final cluster barrier, and frees its tensor memory.
+#include <algorithm>
 #include <cfloat>
 #include <cstdint>
 #include <cuda.h>
@@ -102,7 +103,8 @@ struct Params {
     const int32_t *seq_len;
     const float *qt;        // [B, H, r] fp32
     const unsigned *qmax;   // [B, H] bit patterns of max_j |qt[b, h, j]| (non-negative floats)
-    int H, Np;              // heads, heads padded to a multiple of 16
+    int H, Hs, Np;          // heads in all (array stride); heads of this launch (<= 32), padded to 16
+                            // (qt, qmax, pm, pl, po point at the launch's first head)
     float softmax_scale;
     int tiles_per_split, n_split;
     float *pm, *pl, *po;    // [B, n_split, H] and [B, n_split, H, r]
@@ -423,7 +425,8 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     const int split = blockIdx.x / CL, b = blockIdx.y;
     const int r = c.r, rc = r / CL, ch0 = int(rank) * rc;
     const int n_chunks = rc / kChunk;
-    const int Np = p.Np, H = p.H;
+    // H: this launch's heads; the arrays' head stride is p.H
+    const int Np = p.Np, H = p.Hs;
     constexpr uint32_t kLoadBytes = BITS == 8 ? kTile * kChunk : kTile * kChunk / 2;
 
     if (threadIdx.x == 0) {
@@ -505,7 +508,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                     const int h = i / (rc / 8), q8 = i % (rc / 8);
                     va[k] = vb[k] = make_float4(0.f, 0.f, 0.f, 0.f);
                     if (i < items && h < H) {
-                        const float4 *src = reinterpret_cast<const float4 *>(p.qt + (size_t(b) * H + h) * r + ch0 + q8 * 8);
+                        const float4 *src = reinterpret_cast<const float4 *>(p.qt + (size_t(b) * p.H + h) * r + ch0 + q8 * 8);
                         va[k] = src[0];
                         vb[k] = src[1];
                     }
@@ -515,7 +518,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
                 const int h = lane;
                 int e = 0;
                 if (h < H) {
-                    const float m = __uint_as_float(p.qmax[size_t(b) * H + h]);   // max_j |q~[b, h, j]|
+                    const float m = __uint_as_float(p.qmax[size_t(b) * p.H + h]);   // max_j |q~[b, h, j]|
                     if (m > 0.0f) frexpf(m, &e);                                   // m < 2^e
                 }
                 q_exp[h] = float(14 - e);                                          // |q~| * 2^(14-e) < 2^14
@@ -1027,7 +1030,7 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
             if (!group_any(!ok, bar_id)) {
                 if (grp_live) {
                     fence_after();
-                    const size_t pb = (size_t(b) * p.n_split + split) * H;
+                    const size_t pb = (size_t(b) * p.n_split + split) * p.H;
                     for (int ck = 0; ck < n_chunks; ++ck) {
                         const int ch = ch0 + ck * kChunk + t;
                         uint32_t v[16];
@@ -1083,10 +1086,11 @@ int g_attn_path = 0;     // 0 automatic, 1 CUDA cores, 2 tcgen05, 3 warp-level M
 void set_attn_path(int path) { g_attn_path = path; }
 int attn_path() { return g_attn_path; }
 
+// Heads go in launches of at most kMaxN (32); each reads the whole cache.
 bool attn_tc_shape_ok(int r, int bits, int H) {
-    const int Np = (H + 15) / 16 * 16, cl = atc::cluster_for(r);
+    const int Np = (std::min(H, atc::kMaxN) + 15) / 16 * 16, cl = atc::cluster_for(r);
     if (bits != 8 && bits != 4) return false;
-    if (r % (cl * atc::kChunk) || r / cl > atc::kMaxRc || r / 128 > atc::kMaxGroups || Np > atc::kMaxN) return false;
+    if (H < 1 || r % (cl * atc::kChunk) || r / cl > atc::kMaxRc || r / 128 > atc::kMaxGroups) return false;
     return (r / cl / atc::kChunk) * Np <= int(atc::kColS - atc::kColO);
 }
 
@@ -1139,8 +1143,7 @@ cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const flo
            c.bits == 8 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return cudaErrorInvalidValue;
-    const atc::Params prm{c, seq_len, qt, qmax, H, (H + 15) / 16 * 16, softmax_scale, tiles_per_split, n_split,
-                          pm, pl, po, err};
+    atc::Params prm{c, seq_len, qt, qmax, H, 0, 0, softmax_scale, tiles_per_split, n_split, pm, pl, po, err};
     const int cl = atc::cluster_for(c.r);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(cl * n_split, c.B);
@@ -1158,7 +1161,18 @@ cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const flo
     cfg.numAttrs = 2;
     auto go = [&](auto kern) {
         cudaError_t e = ensure_smem(kern, cfg.dynamicSmemBytes);
-        return e == cudaSuccess ? cudaLaunchKernelEx(&cfg, kern, map, prm) : e;
+        // one launch per group of at most 32 heads (H = 40: heads 0-31, then 32-39)
+        for (int h0 = 0; h0 < H && e == cudaSuccess; h0 += atc::kMaxN) {
+            prm.qt = qt + size_t(h0) * c.r;
+            prm.qmax = qmax + h0;
+            prm.pm = pm + h0;
+            prm.pl = pl + h0;
+            prm.po = po + size_t(h0) * c.r;
+            prm.Hs = std::min(atc::kMaxN, H - h0);
+            prm.Np = (prm.Hs + 15) / 16 * 16;
+            e = cudaLaunchKernelEx(&cfg, kern, map, prm);
+        }
+        return e;
     };
     if (c.bits == 8) return cl == 2 ? go(attn_tc_kernel<8, 2>) : go(attn_tc_kernel<8, 4>);
     return cl == 2 ? go(attn_tc_kernel<4, 2>) : go(attn_tc_kernel<4, 4>);

@@ -171,6 +171,15 @@ def test_decode7b_full_size_sampled(bits):
     assert_rows_close(got[list(checked)], np.stack(refs), "decode7b full size")
 
 
+@pytest.mark.parametrize("H,dh,r,bits,lens", [(40, 128, 2048, 8, [3000, 77]), (40, 128, 2048, 4, [1200, 300]),
+                                               (48, 64, 1024, 8, [500, 129])])
+def test_attn_tc_more_than_32_heads(H, dh, r, bits, lens):
+    """H > 32: one launch per group of at most 32 heads over the same splits
+    (the 13B shape, H = 40: heads 0-31 then 32-39 with N = 16; H = 48 with
+    pairs of CTAs: 32 + 16 heads), each launch's partials at its heads."""
+    _run(H, dh, r, bits, lens, paths=(2,), seed=23)
+
+
 def test_attn_tc_cache_larger_than_lengths():
     """Tmax above every length: the rows after each sequence's end belong to
     no token and must not contribute."""
@@ -205,5 +214,5 @@ def test_attn_tc_path_selection():
     assert lib.qsvd_set_decode_attn_path(0) == 2
     with pytest.raises(lib.QsvdError):
         lib.qsvd_set_decode_attn_path(4)
-    # r = 2048 exceeds the tensor-core kernel's limit: path 2 still answers correctly
-    _run(40, 128, 2048, 8, [300, 40], paths=(2,), seed=6)
+    # r = 2304 does not split into four CTAs of whole 128-channel chunks: path 2 still answers correctly
+    _run(8, 128, 2304, 8, [300, 40], paths=(2,), seed=6)
