@@ -55,6 +55,9 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-prefill13", action="store_true")
+    p.add_argument("--no-prefill-attn", action="store_true")
+    p.add_argument("--prefill-sweep", default=None, metavar="ROWS,...",
+                   help="only time causal prefill attention for these rows-per-group settings (0 = automatic)")
     # the tiny layer's W_d and U come from the oracle's joint SVD: it is a parity case (tests/), not a benchmark
     p.add_argument("--workload", default=WORKLOAD, choices=sorted(k for k in synthetic.WORKLOADS if k != "tiny"))
     p.add_argument("--decode-steps", type=int, default=0, help="override the workload's decode steps")
@@ -475,6 +478,105 @@ def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
             "peak_kind": kind}
 
 
+PREFILL_SHAPES = {
+    # the 7B-shaped prompt (576 image-like + 64 text-like tokens), int8 cache
+    "llava7b": dict(d=4096, H=32, dh=128, r=1536, B=1, T=640, bits=8),
+    # the 13B-shaped batch (8 prompts of 5 x 576 + 128 tokens), int8 cache
+    "llava13b": dict(d=5120, H=40, dh=128, r=2048, B=8, T=3008, bits=8),
+}
+
+
+def prefill_attn_probe(name, iters=3, group_rows=0):
+    """Causal prefill attention: every token of B prompts of T tokens attends
+    to its own prefix (qsvd_latent_prefill_attn over all B*T rows in one
+    call), cold L2 before each call.  The cache codes, scales and U are seeded
+    torch random values (the time does not depend on them; the parity tests
+    check the numbers).  Reports the call's time, tokens/s, and the tensor
+    throughput of the attention kernel (scores and the weighted latent sum,
+    4 H r flops per attended token) from a separate pass with library
+    events between the kernels."""
+    import torch
+    import paper_2510_16292_gb300 as q
+    c = PREFILL_SHAPES[name]
+    d, H, dh, r, B, T, bits = (c[k] for k in ("d", "H", "dh", "r", "B", "T", "bits"))
+    dev = torch.device("cuda", torch.cuda.current_device())
+    g = torch.Generator(device=dev)
+    g.manual_seed(4321)
+    cache = q.LatentCache.empty(B, T, r, bits, dev)
+    if bits == 8:
+        cache.codes.copy_(torch.randint(-127, 128, cache.codes.shape, generator=g, device=dev, dtype=torch.int8))
+        cache.scales.copy_(torch.rand(cache.scales.shape, generator=g, device=dev) * 0.02 + 0.005)
+    else:
+        cache.codes.copy_(torch.randint(0, 256, cache.codes.shape, generator=g, device=dev, dtype=torch.uint8))
+        cache.scales.copy_((torch.rand(cache.scales.shape, generator=g, device=dev) * 0.2 + 0.05).half())
+    U = [(torch.randn((r, H * dh), generator=g, device=dev) / math.sqrt(r)).to(torch.bfloat16) for _ in range(3)]
+    n = B * T
+    q_seq = torch.arange(B, device=dev, dtype=torch.int32).repeat_interleave(T)
+    q_len = torch.arange(1, T + 1, device=dev, dtype=torch.int32).repeat(B)
+    O = torch.empty((n, H * dh), dtype=torch.float32, device=dev)
+    prev = q.qsvd_set_prefill_group_rows(group_rows)
+    try:
+        ws = torch.zeros(q.qsvd_prefill_workspace_bytes(n, T, r, H, dh), dtype=torch.uint8, device=dev)
+        flush = torch.ones((256 << 20) // 4, dtype=torch.float32, device=dev)
+        sink = torch.zeros((), dtype=torch.float32, device=dev)
+        call = lambda: q.qsvd_latent_prefill_attn(cache, q_seq, q_len, T, *U, H, dh, O, workspace=ws)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        times = []
+        for it in range(iters + 1):
+            torch.sum(flush, dim=(0,), out=sink)
+            e0.record()
+            call()
+            e1.record()
+            torch.cuda.synchronize()
+            if it:
+                times.append(e0.elapsed_time(e1) * 1e-3)
+        # per-kernel split: events recorded by the library after each launch
+        cap = 8 + 6 * (n // 16 + 1)
+        events = [torch.cuda.Event(enable_timing=True) for _ in range(cap)]
+        for e in events:
+            e.record()
+        torch.cuda.synchronize()
+        handles = (ctypes.c_void_p * cap)(*[ctypes.c_void_p(e.cuda_event) for e in events])
+        lib = q._lib
+        lib.qsvd_profile_count.restype = ctypes.c_int32
+        lib.qsvd_profile_label.restype = ctypes.c_char_p
+        torch.sum(flush, dim=(0,), out=sink)
+        lib.qsvd_profile_events(handles, cap)
+        call()
+        torch.cuda.synchronize()
+        cnt = lib.qsvd_profile_count()
+        labels = [lib.qsvd_profile_label(i).decode() for i in range(cnt)]
+        lib.qsvd_profile_events(None, 0)
+        q.qsvd_check()
+    finally:
+        q.qsvd_set_prefill_group_rows(prev)
+    by = {}
+    for i in range(1, cnt):
+        e = by.setdefault(labels[i], [0, 0.0])
+        e[0] += 1
+        e[1] += events[i - 1].elapsed_time(events[i]) * 1e-3
+    tot = sum(v[1] for v in by.values())
+    att = next((k for k in ("attn_tc", "attn_mma", "attn_chunk") if k in by), None)
+    sum_len = B * T * (T + 1) // 2
+    attn_flops = 4.0 * H * r * sum_len
+    exec_flops = attn_flops + 6.0 * n * r * d
+    _, bf16_peak, kind = peaks()
+    t = min(times)
+    out = {"shape": f"{B} x {T} tokens, d={d} H={H} r={r} int{bits}", "rows": n,
+           "call_us": round(t * 1e6, 1), "tokens_per_s": round(n / t, 1),
+           "executed_tflops": round(exec_flops / t / 1e12, 2),
+           "kernels": {k: {"launches": v[0], "us": round(v[1] * 1e6, 1), "share": round(v[1] / tot, 4)}
+                       for k, v in sorted(by.items())}}
+    if att:
+        a_t = by[att][1]
+        out["attn_kernel"] = att
+        out["attn_tflops"] = round(attn_flops / a_t / 1e12, 2)
+        out["attn_frac_of_bf16_peak"] = round(attn_flops / a_t / 1e12 / bf16_peak, 4)
+        out["peak_kind"] = kind
+    del cache, U, O, ws, flush
+    return out
+
+
 def cross_rank(values, op="max"):
     """Per-rank totals reduced over the ranks of the default process group
     (max: the job takes as long as its slowest rank; min: the slowest rank's
@@ -564,6 +666,7 @@ def run_native(args, rank, world, local_rank):
                "d2h_bytes_per_step": d2h}
 
     pre13 = prefill_gemm_probe() if not args.no_prefill13 else None
+    pre_attn = None if args.no_prefill_attn else {k: prefill_attn_probe(k) for k in PREFILL_SHAPES}
     if rank != 0:
         return
     out = {
@@ -592,6 +695,7 @@ def run_native(args, rank, world, local_rank):
             "wall_s_timed_region": round(t_wall, 3),
             "kernels": kernels,
             "prefill_13b": pre13,
+            "prefill_attn": pre_attn,
         },
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4),
@@ -798,6 +902,12 @@ def main():
     args = parse()
     if args.sweep:
         run_sweep(args)
+        return
+    if args.prefill_sweep is not None:
+        for rows in (int(x) for x in args.prefill_sweep.split(",")):
+            for name in PREFILL_SHAPES:
+                print(json.dumps({"prefill_attn": name, "group_rows": rows,
+                                  **prefill_attn_probe(name, iters=args.steps, group_rows=rows)}), flush=True)
         return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))

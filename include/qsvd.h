@@ -14,6 +14,7 @@
  *   qsvd_latent_project      C = Q(X) Q(W_d), requantized per token (Eq. 11-12)
  *   qsvd_cache_append        store latent rows in the latent cache (Fig. 2(f))
  *   qsvd_latent_decode_attn  one decode step of attention over that cache (Eq. 5)
+ *   qsvd_latent_prefill_attn causal attention of prompt tokens over that cache
  *
  * Conventions shared by every entry point:
  *   - Row-vector convention Y = X W, as in the paper.  E = d = H * dh.
@@ -182,6 +183,34 @@ int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int
 size_t qsvd_decode_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t r, int32_t H, int32_t dh);
 
 /*
+ * Causal attention of prompt tokens over the latent cache (prefill; Fig. 2(f)
+ * and Eq. 5 with the causal mask of a decoder).  Row i of the call is one
+ * query: the token at position q_len[i]-1 of cache sequence q_seq[i], which
+ * attends to positions 0 .. q_len[i]-1 of that sequence, exactly as
+ * qsvd_latent_decode_attn does for a sequence of length q_len[i].  A prompt
+ * of T tokens appended at positions t0 .. t0+T-1 of sequence b (by
+ * qsvd_latent_project with dst = cache) is prefilled with q_seq[i] = b and
+ * q_len[i] = t0 + i + 1; rows of several sequences may be mixed freely.
+ *   q_seq, q_len  device int32 [n]; 0 <= q_seq[i] < cache->B and
+ *                 1 <= q_len[i] <= max_len <= Tmax.  A row outside these
+ *                 ranges is skipped, its output row is zero, and QSVD_ERANGE
+ *                 is flagged for qsvd_check;
+ *   max_len       host-side bound on q_len used to size the launches;
+ *   U_q, U_k, U_v bf16 [r, H*dh] row-major;  O fp32 [n, H*dh] out.
+ * The rows are processed in consecutive groups that reuse one workspace of
+ * qsvd_prefill_workspace_bytes(n, max_len, r, H, dh) bytes; the cache is only
+ * read.  n may be 0 (nothing is enqueued).  Requirements as for
+ * qsvd_latent_decode_attn.
+ */
+int qsvd_latent_prefill_attn(const qsvd_cache *cache, const int32_t *q_seq, const int32_t *q_len,
+                             int64_t n, int32_t max_len,
+                             const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v,
+                             int32_t H, int32_t dh, float softmax_scale, float *O,
+                             void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+size_t qsvd_prefill_workspace_bytes(int64_t n, int32_t max_len, int32_t r, int32_t H, int32_t dh);
+
+/*
  * One whole decode step for a small batch, in a single launch: for each of
  * the B = cache->B sequences, the new token X[b] (bf16 [B, d]) is quantized
  * and projected (Eq. 12), its latent is requantized and stored at position
@@ -256,12 +285,25 @@ int qsvd_set_project_epilogue(int32_t mode);
  *   1  always the CUDA-core kernels;
  *   2  the tcgen05 kernel whenever the shape allows it;
  *   3  the warp-level tensor-core kernel whenever r <= 3072.
- * The tcgen05 kernel needs r % 256 == 0, r <= 1536, H <= 32 and
- * (r / 256) * ceil16(H) <= 192; other shapes use the CUDA-core kernels.  All
- * give the same results up to floating-point rounding.
+ * The tcgen05 kernel needs r <= 3072 with r % 256 == 0 up to r = 1536
+ * (clusters of two CTAs) and r % 512 == 0 above (clusters of four); it takes
+ * the heads in launches of up to 32.  Other shapes use the warp-level kernel
+ * (r <= 3072) or the CUDA-core kernels.  All give the same results up to
+ * floating-point rounding.  qsvd_latent_prefill_attn follows the same
+ * setting.
  * Returns the previous setting, or QSVD_EINVAL for another value.
  */
 int qsvd_set_decode_attn_path(int32_t path);
+
+/*
+ * Rows per group of qsvd_latent_prefill_attn (a library setting, not part of
+ * the paper's method; process-wide, not thread-safe): 0 (default) picks the
+ * largest power of two up to 1024 whose workspace stays within 2 GiB; a
+ * value in [1, 65535] fixes the group size (the workspace size query follows
+ * it).  Results do not depend on it.  Returns the previous setting, or
+ * QSVD_EINVAL for a value outside [0, 65535].
+ */
+int qsvd_set_prefill_group_rows(int32_t rows);
 
 /*
  * Synchronizes `stream`, then reads and clears the device error word.

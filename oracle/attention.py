@@ -13,6 +13,10 @@ included) attended.  ``decode_attention`` materialises K and V -- the plain
 definition.  ``decode_attention_absorbed`` regroups the same products
 (q~_h = W^u_k,h q_h, scores C q~_h, o_h = (p^T C) W^u_v,h) and exists only so
 the tests can check the two agree.
+
+``prefill_attention`` is the prompt's side of the same layer: every prompt
+token queries the cache of its own sequence under a decoder's causal mask
+(Fig. 2(f): the prompt's latents are cached, then attended).
 """
 from __future__ import annotations
 
@@ -88,3 +92,31 @@ def decode_attention_loops(C, U_q, U_k, U_v, H: int, dh: int, softmax_scale=None
         for e in cols:
             out[e] = sum(w[t] / z * V[t][e] for t in range(L))
     return np.array(out)
+
+
+def prefill_attention(C, U_q, U_k, U_v, H: int, dh: int, softmax_scale=None, t0: int = 0):
+    """Causal attention of the prompt tokens at positions t0 .. L-1 of one
+    sequence, L = len(C) (C: fp64 [L, r] dequantized latent rows of
+    positions 0 .. L-1).  The decoder's masked self-attention in matrix form:
+    Q = C[t0:] U_q, K = C U_k, V = C U_v and per head h
+
+        S_h = Q_h K_h^T * softmax_scale,  S_h[i, t] = -inf for t > t0 + i,
+        O_h = softmax_rows(S_h) V_h.
+
+    Returns fp64 [L - t0, H*dh]; row i is the output of position t0 + i."""
+    C = np.asarray(C, dtype=np.float64)
+    L = C.shape[0]
+    if softmax_scale is None:
+        softmax_scale = 1.0 / math.sqrt(dh)
+    T = L - t0
+    Q = C[t0:] @ U_q
+    K = C @ U_k
+    V = C @ U_v
+    masked = np.arange(L)[None, :] > (t0 + np.arange(T))[:, None]    # keys after the query
+    O = np.empty((T, H * dh))
+    for h in range(H):
+        sl = slice(h * dh, (h + 1) * dh)
+        S = (Q[:, sl] @ K[:, sl].T) * softmax_scale
+        S[masked] = -np.inf
+        O[:, sl] = softmax(S) @ V[:, sl]
+    return O

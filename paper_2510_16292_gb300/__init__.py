@@ -7,7 +7,8 @@ kernels; there is no host fallback.  Importing this package fails loudly if
 the library has not been built (``python paper_2510_16292_gb300/build.py``).
 
 Names follow the C ABI: ``qsvd_quantize_weight``, ``qsvd_latent_project``,
-``qsvd_cache_append``, ``qsvd_latent_decode_attn``, ``qsvd_check``, plus the
+``qsvd_cache_append``, ``qsvd_latent_decode_attn``, ``qsvd_latent_prefill_attn``,
+``qsvd_check``, plus the
 workspace-size queries.  ``DownWeight`` and ``LatentCache`` hold the torch
 tensors behind the two C structs.
 """
@@ -31,8 +32,9 @@ QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
 EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
+           "qsvd_latent_prefill_attn", "qsvd_prefill_workspace_bytes",
            "qsvd_decode_step", "qsvd_decode_step_workspace_bytes", "qsvd_latent_project_static",
-           "qsvd_set_decode_attn_path", "qsvd_set_project_epilogue", "qsvd_check", "qsvd_last_error",
+           "qsvd_set_decode_attn_path", "qsvd_set_project_epilogue", "qsvd_set_prefill_group_rows", "qsvd_check", "qsvd_last_error",
            "qsvd_selftest_wait_timeout", "qsvd_version")
 
 
@@ -63,6 +65,10 @@ _lib.qsvd_latent_decode_attn.argtypes = [ctypes.POINTER(_Cache), _vp, _i32, _vp,
                                          _vp, _vp, _sz, _vp]
 _lib.qsvd_decode_workspace_bytes.argtypes = [_i32, _i32, _i32, _i32, _i32]
 _lib.qsvd_decode_workspace_bytes.restype = _sz
+_lib.qsvd_latent_prefill_attn.argtypes = [ctypes.POINTER(_Cache), _vp, _vp, _i64, _i32, _vp, _vp, _vp, _i32, _i32,
+                                          _f32, _vp, _vp, _sz, _vp]
+_lib.qsvd_prefill_workspace_bytes.argtypes = [_i64, _i32, _i32, _i32, _i32]
+_lib.qsvd_prefill_workspace_bytes.restype = _sz
 _lib.qsvd_decode_step.argtypes = [ctypes.POINTER(_DownWeight), _vp, ctypes.POINTER(_Cache), _vp, _i32, _vp, _vp,
                                   _vp, _i32, _i32, _f32, _f32, _f32, _vp, _vp, _sz, _vp]
 _lib.qsvd_decode_step_workspace_bytes.argtypes = [_i32, _i32, _i32, _i32, _i32, _i32]
@@ -219,6 +225,30 @@ def qsvd_latent_decode_attn(cache: LatentCache, seq_len: torch.Tensor, max_seq_l
                                         workspace.numel(), _stream(stream)))
 
 
+def qsvd_prefill_workspace_bytes(n: int, max_len: int, r: int, H: int, dh: int) -> int:
+    return int(_lib.qsvd_prefill_workspace_bytes(n, max_len, r, H, dh))
+
+
+def qsvd_latent_prefill_attn(cache: LatentCache, q_seq: torch.Tensor, q_len: torch.Tensor, max_len: int,
+                             U_q, U_k, U_v, H: int, dh: int, O: torch.Tensor,
+                             softmax_scale: Optional[float] = None, workspace=None, stream=None) -> None:
+    """Row i: the token at position q_len[i]-1 of sequence q_seq[i] attends to
+    positions 0 .. q_len[i]-1 of that sequence (causal prefill)."""
+    if softmax_scale is None:
+        softmax_scale = 1.0 / math.sqrt(dh)
+    n = q_seq.numel()
+    if q_len.numel() != n:
+        raise ValueError("q_seq and q_len differ in length")
+    if workspace is None:
+        workspace = torch.zeros(max(1, qsvd_prefill_workspace_bytes(n, max_len, cache.r, H, dh)),
+                                dtype=torch.uint8, device=O.device)
+    cc = cache._c()
+    _check(_lib.qsvd_latent_prefill_attn(ctypes.byref(cc), _ptr(q_seq, _I32, "q_seq"), _ptr(q_len, _I32, "q_len"),
+                                         n, max_len, _ptr(U_q, _BF16, "U_q"), _ptr(U_k, _BF16, "U_k"),
+                                         _ptr(U_v, _BF16, "U_v"), H, dh, softmax_scale, _ptr(O, _F32, "O"),
+                                         _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
 def qsvd_decode_step_workspace_bytes(B: int, max_seq_len: int, d: int, r: int, H: int, dh: int) -> int:
     return int(_lib.qsvd_decode_step_workspace_bytes(B, max_seq_len, d, r, H, dh))
 
@@ -277,6 +307,7 @@ def qsvd_version() -> int:
 
 
 _lib.qsvd_set_decode_attn_path.argtypes = [_i32]
+_lib.qsvd_set_prefill_group_rows.argtypes = [_i32]
 _lib.qsvd_set_project_epilogue.argtypes = [_i32]
 
 
@@ -284,6 +315,15 @@ def qsvd_set_project_epilogue(mode: int) -> int:
     """0 automatic, 1 separate requantization kernel, 2 requantize in the
     tensor-core GEMM epilogue where possible.  Returns the previous setting."""
     st = _lib.qsvd_set_project_epilogue(mode)
+    if st < 0:
+        _check(st)
+    return st
+
+
+def qsvd_set_prefill_group_rows(rows: int) -> int:
+    """Rows per group of qsvd_latent_prefill_attn; 0 automatic.  Returns the
+    previous setting."""
+    st = _lib.qsvd_set_prefill_group_rows(rows)
     if st < 0:
         _check(st)
     return st

@@ -1,5 +1,6 @@
 // C ABI of the QSVD latent-attention path (declared in include/qsvd.h):
 // argument validation, workspace carving and kernel launch order.
+#include <algorithm>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -78,7 +79,9 @@ int check_cache(const qsvd_cache *c) {
     return QSVD_OK;
 }
 
-CacheView view(const qsvd_cache *c) { return CacheView{c->codes, c->scales, c->bits, c->B, c->Tmax, c->r}; }
+CacheView view(const qsvd_cache *c) {
+    return CacheView{c->codes, c->scales, c->bits, c->B, c->Tmax, c->r, nullptr, c->B};
+}
 
 // Profiling state of the calling thread (see qsvd_profile_events).
 thread_local cudaEvent_t *t_prof_events = nullptr;
@@ -390,6 +393,68 @@ int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int
     prof_mark(stream, "begin");
     cudaError_t e = launch_decode(a, workspace, workspace_bytes, err, stream);
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "decode_attn launch");
+}
+
+// Rows of one prefill group: the largest power of two up to kPrefillMaxRows
+// whose decode workspace (queries and softmax partials, fp32) stays within
+// kPrefillWsTarget bytes.  Larger groups measured faster all the way to 1024
+// rows (fewer launches, fuller waves).
+static int g_prefill_rows = 0;   // qsvd_set_prefill_group_rows; 0: automatic
+
+static int prefill_group_rows(int64_t n, int max_len, int r, int H, int dh) {
+    if (g_prefill_rows > 0) return int(std::min<int64_t>(g_prefill_rows, n));
+    int rows = kPrefillMaxRows;
+    while (rows > 16 && decode_workspace_bytes(rows, max_len, r, H, dh) > kPrefillWsTarget) rows /= 2;
+    return int(std::min<int64_t>(rows, n));
+}
+
+int qsvd_set_prefill_group_rows(int32_t rows) {
+    if (rows < 0 || rows > 65535) return fail(QSVD_EINVAL, "set_prefill_group_rows: rows outside [0, 65535]");
+    const int prev = g_prefill_rows;
+    g_prefill_rows = rows;
+    return prev;
+}
+
+size_t qsvd_prefill_workspace_bytes(int64_t n, int32_t max_len, int32_t r, int32_t H, int32_t dh) {
+    if (n <= 0 || max_len <= 0 || r <= 0 || H <= 0 || dh <= 0) return 0;
+    return decode_workspace_bytes(prefill_group_rows(n, max_len, r, H, dh), max_len, r, H, dh);
+}
+
+int qsvd_latent_prefill_attn(const qsvd_cache *cache, const int32_t *q_seq, const int32_t *q_len, int64_t n,
+                             int32_t max_len, const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v,
+                             int32_t H, int32_t dh, float softmax_scale, float *O, void *workspace,
+                             size_t workspace_bytes, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if ((st = check_cache(cache))) return st;
+    if (n < 0) return fail(QSVD_EINVAL, "prefill_attn: n < 0");
+    if (n == 0) return QSVD_OK;
+    if (!q_seq || !q_len || !U_q || !U_k || !U_v || !O) return fail(QSVD_EINVAL, "prefill_attn: null pointer");
+    if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "prefill_attn: dh must be 64 or 128");
+    if (H <= 0) return fail(QSVD_EINVAL, "prefill_attn: H must be positive");
+    if (cache->r > 3072 || cache->r % 32) return fail(QSVD_EUNSUPPORTED, "prefill_attn: need r %% 32 == 0 and r <= 3072");
+    if ((H * dh) % 256 || H * dh > 6144) return fail(QSVD_EUNSUPPORTED, "prefill_attn: need H*dh %% 256 == 0 and H*dh <= 6144");
+    if (max_len < 1 || max_len > cache->Tmax) return fail(QSVD_EINVAL, "prefill_attn: max_len outside [1, Tmax]");
+    const void *ptrs[] = {q_seq, q_len, U_q, U_k, U_v, O, workspace};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(QSVD_EINVAL, "prefill_attn: pointers must be 16-byte aligned");
+    const int rows = prefill_group_rows(n, max_len, cache->r, H, dh);
+    const size_t need = decode_workspace_bytes(rows, max_len, cache->r, H, dh);
+    if (!workspace || workspace_bytes < need) return fail(QSVD_ENOSPC, "prefill_attn: workspace needs %zu bytes", need);
+    const size_t d = size_t(H) * dh;
+    prof_mark(stream, "begin");
+    for (int64_t i0 = 0; i0 < n; i0 += rows) {
+        // a group of rows is a decode step over a view whose row b is cache
+        // sequence q_seq[i0 + b] at length q_len[i0 + b]
+        CacheView v = view(cache);
+        v.B = int(std::min<int64_t>(rows, n - i0));
+        v.seq_map = q_seq + i0;
+        DecodeArgs a{v, q_len + i0, max_len, U_q, U_k, U_v, H, dh, softmax_scale, O + size_t(i0) * d};
+        const cudaError_t e = launch_decode(a, workspace, workspace_bytes, err, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "prefill_attn launch");
+    }
+    return QSVD_OK;
 }
 
 size_t qsvd_decode_step_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t d, int32_t r, int32_t H,

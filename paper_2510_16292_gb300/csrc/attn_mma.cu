@@ -137,7 +137,10 @@ attn_mma_kernel(const am::Params p) {
     __half *ps = gsc + (BITS == 4 ? size_t(TS) * (r / 128) : 0);                       // [kHG][TS + 8] P
     const int pstride = TS + 8;
     pdl_trigger();
-    const int L = p.seq_len[b];                                    // an input: no kernel writes it
+    // lengths and sequence map: call inputs, complete before this grid starts
+    // (the query kernels let their dependents start only after their own wait)
+    const int sq = view_seq(c, b);
+    const int L = sq < 0 ? 0 : p.seq_len[b];
     const int t_split = split * TS * p.n_sub;
     if (L < 1 || L > c.Tmax || t_split >= L) return;               // invalid lengths are flagged by qproj_kernel
     const int n_sub = min(p.n_sub, (L - t_split + TS - 1) / TS);   // sub-tiles of this CTA
@@ -147,7 +150,7 @@ attn_mma_kernel(const am::Params p) {
         // seen stale: the shared-memory copies come after the wait)
         for (int sb = 0; sb < n_sub; ++sb) {
             const int t0 = t_split + sb * TS;
-            prefetch_l2_bulk(static_cast<const uint8_t *>(c.codes) + (size_t(b) * c.Tmax + t0) * row_bytes,
+            prefetch_l2_bulk(static_cast<const uint8_t *>(c.codes) + (size_t(sq) * c.Tmax + t0) * row_bytes,
                              uint32_t(min(TS, L - t0)) * row_bytes);
         }
     }
@@ -157,7 +160,7 @@ attn_mma_kernel(const am::Params p) {
     auto load_tile = [&](int sb) {
         const int t_begin = t_split + sb * TS;
         const int n = min(TS, L - t_begin);
-        const size_t slot0 = size_t(b) * c.Tmax + t_begin;
+        const size_t slot0 = size_t(sq) * c.Tmax + t_begin;
         const int cpr = row_bytes / 16;                            // 16-byte chunks per row
         for (int i = threadIdx.x; i < TS * cpr; i += kThreads) {
             const int t = i / cpr, k = i - t * cpr;

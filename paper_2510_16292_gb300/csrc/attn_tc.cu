@@ -470,12 +470,15 @@ attn_tc_kernel(const __grid_constant__ CUtensorMap map_c, const atc::Params p) {
     const uint32_t tmem = tmem_base;
     pdl_trigger();
 
-    const int L = p.seq_len[b];                       // an input: no kernel of the chain writes it
+    // lengths and sequence map: call inputs, complete before this grid starts
+    // (the query kernels let their dependents start only after their own wait)
+    const int sq = view_seq(c, b);
+    const int L = sq < 0 ? 0 : p.seq_len[b];
     const bool valid = L >= 1 && L <= c.Tmax;
     const int t_begin = split * p.tiles_per_split * kTile;
     const int t_end = valid ? min(L, t_begin + p.tiles_per_split * kTile) : t_begin;
     const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
-    const size_t row0 = size_t(b) * c.Tmax;          // cache slot of token 0 of the sequence
+    const size_t row0 = size_t(valid ? sq : 0) * c.Tmax;   // cache slot of token 0 of the sequence
     const int total = n_tiles * n_chunks;             // chunk loads per pass
     const int ngrp = r / 128;                         // int4 scale groups per token
     // the first two tiles' chunks into L2 while the producer grid finishes (L2
@@ -1135,7 +1138,7 @@ cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const flo
     // x one chunk (128 bytes of int8, 128-byte swizzle; 64 bytes of int4, 64-byte swizzle)
     const int row_bytes = c.bits == 8 ? c.r : c.r / 2;
     CUtensorMap map;
-    const cuuint64_t dims[2] = {cuuint64_t(row_bytes), cuuint64_t(int64_t(c.B) * c.Tmax)};
+    const cuuint64_t dims[2] = {cuuint64_t(row_bytes), cuuint64_t(int64_t(c.nseq) * c.Tmax)};
     const cuuint64_t strides[1] = {cuuint64_t(row_bytes)};
     const cuuint32_t box[2] = {c.bits == 8 ? 128u : 64u, 128u};
     const cuuint32_t estr[2] = {1, 1};

@@ -84,7 +84,7 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
              unsigned *__restrict__ qmax, int n_qmax, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar;
-    __shared__ int L_s[NB];
+    __shared__ int L_s[NB], Q_s[NB];   // length and cache sequence of each row
     const int r = c.r, rs = r / kCl, br = box_rows(rs);
     const int ncq = ncol / 4, G = 256 / ncq, rpg = rs / G;
     const uint32_t rank = cl_rank();
@@ -93,7 +93,6 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
     float *c_s = reinterpret_cast<float *>(smem + size_t(rs) * ncol * 2);        // [NB][rs]
     float *part = c_s + NB * rs;                                                 // [G][NB][ncol]
     const int tid = threadIdx.x;
-    pdl_trigger();
     if (tid == 0) {
         for (int k = 0; k < rs / br; ++k) tma_prefetch(&map_u, c0, j0 + k * br);
         mbar_init(&bar, 1);
@@ -110,6 +109,8 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
+    pdl_trigger();   // after the wait: the attention kernel two launches on reads the
+                     // lengths before its own wait, and they are complete by then
     if (rank == 0 && blockIdx.y == 0)
         for (int i = tid; i < n_qmax; i += blockDim.x) qmax[i] = 0u;
     bool ready = false;
@@ -121,11 +122,13 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
         __syncthreads();
         if (tid < NB) {
             int L = tid < nb ? seq_len[b0 + tid] : 0;
-            if (tid < nb && !len_ok(L, c.Tmax)) {
+            const int sq = tid < nb ? view_seq(c, b0 + tid) : 0;
+            if (tid < nb && (sq < 0 || !len_ok(L, c.Tmax))) {
                 if (rank == 0 && blockIdx.y == 0) flag_error(err, kErrRange);
                 L = 0;
             }
             L_s[tid] = L;
+            Q_s[tid] = sq;
         }
         __syncthreads();
         // dequantized latent rows c_{L-1}: code words and scales, every load issued first
@@ -141,7 +144,7 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
                 const int bi = w / wpr, x = w - bi * wpr;
                 const int L = L_s[bi];
                 if (L > 0) {
-                    const size_t slot = size_t(b0 + bi) * c.Tmax + (L - 1);
+                    const size_t slot = size_t(Q_s[bi]) * c.Tmax + (L - 1);
                     if (c.bits == 8) {
                         wv[k] = reinterpret_cast<const uint32_t *>(static_cast<const int8_t *>(c.codes) + slot * r + j0)[x];
                         sv[k] = static_cast<const float *>(c.scales)[slot];
@@ -251,7 +254,6 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
     const int rows = min(kQaRows, r - j0);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int w = hg * dh;
-    pdl_trigger();
     if (threadIdx.x < 32)
         for (int i = lane; i < rows; i += 32)
             prefetch_l2_bulk(Uk + size_t(j0 + i) * d + size_t(h0) * dh, uint32_t(w) * 2);
@@ -267,6 +269,8 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
             bulk_g2s(u_s + size_t(i) * ustride, Uk + size_t(j0 + i) * d + size_t(h0) * dh, uint32_t(w) * 2, &bar);
     }
     pdl_wait();
+    pdl_trigger();   // after the wait: the attention kernel two launches on reads the
+                     // lengths before its own wait, and they are complete by then
     bool ready = false;
     const int h = h0 + warp;
     for (int b0 = 0; b0 < B; b0 += NB) {
@@ -335,7 +339,7 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
 template <int NB>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
 combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__restrict__ Uv,
-                  const int32_t *__restrict__ seq_len, int B, int Tmax,
+                  const int32_t *__restrict__ seq_len, const int32_t *__restrict__ seq_map, int nseq, int B, int Tmax,
                   int H, int dh, int r, int chunk, int n_split, const float *__restrict__ pm,
                   const float *__restrict__ pl, const float *__restrict__ po, float *__restrict__ O, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -381,7 +385,7 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__r
 #pragma unroll
             for (int k = 0; k < kWB; ++k) {
                 const int bi = warp + 8 * k;
-                const int L = bi < nb ? seq_len[b0 + bi] : 0;
+                const int L = bi < nb ? row_len(seq_len, seq_map, nseq, b0 + bi) : 0;
                 ns[k] = len_ok(L, Tmax) ? (L + chunk - 1) / chunk : 0;
             }
 #pragma unroll
@@ -532,14 +536,15 @@ cudaError_t qabsorb_nb(const float *q, const uint16_t *Uk, int B, int r, int d, 
 }
 
 template <int NB>
-cudaError_t combine_nb(const CUtensorMap &map, const uint16_t *Uv, const int32_t *seq_len, int B, int Tmax, int H, int dh, int r,
+cudaError_t combine_nb(const CUtensorMap &map, const uint16_t *Uv, const int32_t *seq_len, const int32_t *seq_map,
+                       int nseq, int B, int Tmax, int H, int dh, int r,
                        int chunk, int n_split, const float *pm, const float *pl, const float *po, float *O, int *err,
                        cudaStream_t s) {
     const int rs = r / kCl;
     const size_t smem = size_t(rs) * dh * 2 + size_t(NB) * rs * 4 + size_t(256 / dh) * NB * dh * 4;
     cudaError_t e = ensure_smem(combine_uv_kernel<NB>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(combine_uv_kernel<NB>, dim3(kCl, H), dim3(256), smem, s, map, Uv, seq_len, B, Tmax, H, dh, r,
+    return launch_pdl(combine_uv_kernel<NB>, dim3(kCl, H), dim3(256), smem, s, map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r,
                       chunk, n_split, pm, pl, po, O, err);
 }
 
@@ -578,7 +583,7 @@ cudaError_t launch_qabsorb(const float *q, const uint16_t *Uk, int B, int r, int
     return e;
 }
 
-cudaError_t launch_combine_uv(const int32_t *seq_len, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
+cudaError_t launch_combine_uv(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
                               const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
                               int *err, cudaStream_t s) {
     const int rs = r / kCl, d = H * dh;
@@ -588,11 +593,11 @@ cudaError_t launch_combine_uv(const int32_t *seq_len, int B, int Tmax, int H, in
         return cudaErrorInvalidValue;
     cudaError_t e;
     switch (pass_nb(B)) {
-        case 1: e = combine_nb<1>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 2: e = combine_nb<2>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 4: e = combine_nb<4>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 8: e = combine_nb<8>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        default: e = combine_nb<16>(map, Uv, seq_len, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 1: e = combine_nb<1>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 2: e = combine_nb<2>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 4: e = combine_nb<4>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        case 8: e = combine_nb<8>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
+        default: e = combine_nb<16>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
     }
     prof_mark(s, "combine_uv");
     return e;

@@ -91,7 +91,7 @@ __global__ void __cluster_dims__(kClQ, 1, 1) __launch_bounds__(128)
 qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__restrict__ seq_len, int B, int d,
                  float *__restrict__ q, unsigned *__restrict__ qmax, int n_qmax, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ int L_s[16];
+    __shared__ int L_s[16], Q_s[16];   // length and cache sequence of each row
     const int r = c.r, rs = r / kClQ, ngl = rs / 128;
     const uint32_t rank = mrank();
     const int c0 = blockIdx.y * 64, j0 = int(rank) * rs;
@@ -102,13 +102,14 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
     uint16_t *a_s = u_s + size_t(rs) * kUS;                                  // [16][kAS]
     float *sc_s = reinterpret_cast<float *>(a_s + 16 * kAS);                 // [16][ngl]
     float *part = sc_s + 16 * ngl;                                           // [16][64]
-    pdl_trigger();
     for (int i = tid; i < rs * 8; i += 128) {        // U_q tile: no kernel's output, copied before the wait
         const int row = i >> 3, k = i & 7;
         mcp16(u_s + size_t(row) * kUS + 8 * k, Uq + size_t(j0 + row) * d + c0 + 8 * k);
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
+    pdl_trigger();   // after the wait: the attention kernel two launches on reads the
+                     // lengths before its own wait, and they are complete by then
     if (rank == 0 && blockIdx.y == 0 && blockIdx.z == 0)
         for (int i = tid; i < n_qmax; i += 128) qmax[i] = 0u;
     bool ready = false;
@@ -117,11 +118,13 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
         __syncthreads();
         if (tid < 16) {
             int L = tid < nb ? seq_len[b0 + tid] : 0;
-            if (tid < nb && !mlen_ok(L, c.Tmax)) {
+            const int sq = tid < nb ? view_seq(c, b0 + tid) : 0;
+            if (tid < nb && (sq < 0 || !mlen_ok(L, c.Tmax))) {
                 if (rank == 0 && blockIdx.y == 0) flag_error(err, kErrRange);
                 L = 0;
             }
             L_s[tid] = L;
+            Q_s[tid] = sq;
         }
         __syncthreads();
         // A: the codes of row c_{L-1} in bf16 (exact); rows without a token are zero
@@ -132,7 +135,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
                 uint4 w = make_uint4(0u, 0u, 0u, 0u);
                 if (L > 0)
                     w = *reinterpret_cast<const uint4 *>(static_cast<const int8_t *>(c.codes) +
-                                                         (size_t(b0 + row) * c.Tmax + L - 1) * r + j0 + 16 * ch);
+                                                         (size_t(Q_s[row]) * c.Tmax + L - 1) * r + j0 + 16 * ch);
                 const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
                 uint32_t o[8];
 #pragma unroll
@@ -147,7 +150,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
             for (int i = tid; i < 16 * ngl; i += 128) {
                 const int row = i / ngl;
                 const int L = L_s[row];
-                sc_s[i] = L > 0 ? static_cast<const float *>(c.scales)[size_t(b0 + row) * c.Tmax + L - 1] : 0.0f;
+                sc_s[i] = L > 0 ? static_cast<const float *>(c.scales)[size_t(Q_s[row]) * c.Tmax + L - 1] : 0.0f;
             }
         } else {
             for (int i = tid; i < 16 * (rs / 32); i += 128) {
@@ -156,7 +159,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
                 uint4 w = make_uint4(0u, 0u, 0u, 0u);
                 if (L > 0)
                     w = *reinterpret_cast<const uint4 *>(static_cast<const uint8_t *>(c.codes) +
-                                                         (size_t(b0 + row) * c.Tmax + L - 1) * (r / 2) + j0 / 2 +
+                                                         (size_t(Q_s[row]) * c.Tmax + L - 1) * (r / 2) + j0 / 2 +
                                                          16 * ch);
                 const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
                 uint4 *dst = reinterpret_cast<uint4 *>(a_s + size_t(row) * kAS + 32 * ch);
@@ -173,7 +176,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
             for (int i = tid; i < 16 * ngl; i += 128) {
                 const int row = i / ngl, g = i - row * ngl;
                 const int L = L_s[row];
-                sc_s[i] = L > 0 ? __half2float(static_cast<const __half *>(c.scales)[(size_t(b0 + row) * c.Tmax + L - 1) *
+                sc_s[i] = L > 0 ? __half2float(static_cast<const __half *>(c.scales)[(size_t(Q_s[row]) * c.Tmax + L - 1) *
                                                                                      (r / 128) + j0 / 128 + g])
                                 : 0.0f;
             }
@@ -239,13 +242,14 @@ qabsorb_mma_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk,
     uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                      // [128 j][kS]
     uint16_t *ah_s = u_s + 128 * kS;                                         // [16][kS]
     uint16_t *al_s = ah_s + 16 * kS;                                         // [16][kS]
-    pdl_trigger();
     for (int i = tid; i < 128 * (dh / 8); i += 128) {    // U_k rows: no kernel's output, copied before the wait
         const int row = i / (dh / 8), k = i - row * (dh / 8);
         mcp16(u_s + size_t(row) * kS + 8 * k, Uk + size_t(j0 + row) * d + size_t(h) * dh + 8 * k);
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
+    pdl_trigger();   // after the wait: the attention kernel two launches on reads the
+                     // lengths before its own wait, and they are complete by then
     bool ready = false;
     for (int b0 = 16 * int(blockIdx.z); b0 < B; b0 += 16 * int(gridDim.z)) {   // grid z: 16-sequence passes
         const int nb = min(16, B - b0);
@@ -319,7 +323,8 @@ qabsorb_mma_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk,
 // adds the kClV products of columns k dh/kClV .. in rank order.
 // ---------------------------------------------------------------------------
 __global__ void __cluster_dims__(kClV, 1, 1) __launch_bounds__(128)
-combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ seq_len, int B, int Tmax, int H,
+combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ seq_len,
+                   const int32_t *__restrict__ seq_map, int nseq, int B, int Tmax, int H,
                    int dh, int r, int chunk, int n_split, const float *__restrict__ pm, const float *__restrict__ pl,
                    const float *__restrict__ po, float *__restrict__ O) {
     extern __shared__ __align__(128) uint8_t smem[];
@@ -351,7 +356,7 @@ combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ 
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             const int bi = warp + 4 * k;
-            const int L = bi < nb ? seq_len[b0 + bi] : 0;
+            const int L = bi < nb ? row_len(seq_len, seq_map, nseq, b0 + bi) : 0;
             const int ns = mlen_ok(L, Tmax) ? (L + chunk - 1) / chunk : 0;
             const size_t base = size_t(b0 + bi) * n_split * H + h;
             const float m0 = lane < ns ? pm[base + size_t(lane) * H] : -FLT_MAX;
@@ -473,14 +478,14 @@ cudaError_t launch_qabsorb_mma(const float *q, const uint16_t *Uk, int B, int r,
     return e;
 }
 
-cudaError_t launch_combine_mma(const int32_t *seq_len, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
+cudaError_t launch_combine_mma(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
                                const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
                                cudaStream_t s) {
     const int rs = r / kClV;
     const size_t smem = size_t(rs) * (dh + 8) * 2 + size_t(32) * (rs + 8) * 2 + size_t(16) * dh * 4;
     cudaError_t e = ensure_smem(combine_mma_kernel, smem);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(combine_mma_kernel, dim3(kClV, H, (B + 15) / 16), dim3(128), smem, s, Uv, seq_len, B, Tmax, H, dh, r, chunk,
+    e = launch_pdl(combine_mma_kernel, dim3(kClV, H, (B + 15) / 16), dim3(128), smem, s, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk,
                    n_split, pm, pl, po, O);
     prof_mark(s, "combine_uv");
     return e;

@@ -107,9 +107,10 @@ attn_chunk_kernel(CacheView c, const int32_t *__restrict__ seq_len, const float 
     uint8_t *tile = reinterpret_cast<uint8_t *>(ts + 2 * sub);      // [2][sub][row_bytes] codes
     const int slot_bytes = row_bytes;
     pdl_trigger();
-    if (blockIdx.z == 0 && threadIdx.x == 0 && t_begin < c.Tmax) {
+    const int sq = view_seq(c, b);   // a call input, complete before this grid starts (see qproj)
+    if (blockIdx.z == 0 && threadIdx.x == 0 && t_begin < c.Tmax && sq >= 0) {
         const int rows = min(chunk, c.Tmax - t_begin);
-        const char *base = static_cast<const char *>(c.codes) + (size_t(b) * c.Tmax + t_begin) * row_bytes;
+        const char *base = static_cast<const char *>(c.codes) + (size_t(sq) * c.Tmax + t_begin) * row_bytes;
         for (size_t o = 0; o < size_t(rows) * row_bytes; o += 65536)
             prefetch_l2_bulk(base + o, uint32_t(min(size_t(65536), size_t(rows) * row_bytes - o)));
     }
@@ -120,7 +121,7 @@ attn_chunk_kernel(CacheView c, const int32_t *__restrict__ seq_len, const float 
     }
     __syncthreads();
     pdl_wait();
-    const int L = seq_len[b];
+    const int L = sq < 0 ? 0 : seq_len[b];
     if (!valid_len(L, c.Tmax) || t_begin >= L) return;        // invalid lengths are flagged by qproj_kernel
     const int n = min(L, t_begin + chunk) - t_begin;
     const int n_sub = (n + sub - 1) / sub;
@@ -128,7 +129,7 @@ attn_chunk_kernel(CacheView c, const int32_t *__restrict__ seq_len, const float 
     auto issue = [&](int st, int buf) {                       // thread 0 only
         const int t0 = t_begin + st * sub;
         const int rows = min(sub, t_begin + n - t0);
-        const size_t slot0 = size_t(b) * c.Tmax + t0;
+        const size_t slot0 = size_t(sq) * c.Tmax + t0;
         uint8_t *dst = tile + size_t(buf) * sub * slot_bytes;
         const uint32_t code_bytes = uint32_t(rows) * row_bytes;
         mbar_arrive_expect_tx(&bar[buf], code_bytes);
@@ -159,10 +160,10 @@ attn_chunk_kernel(CacheView c, const int32_t *__restrict__ seq_len, const float 
         const int rows = min(sub, n - st * sub);
         const uint8_t *tl_codes = tile + size_t(buf) * sub * slot_bytes;
         const __half *tl_gs = static_cast<const __half *>(c.scales) +
-                              (size_t(b) * c.Tmax + t_begin + st * sub) * (r / 128);   // int4 group scales
+                              (size_t(sq) * c.Tmax + t_begin + st * sub) * (r / 128);   // int4 group scales
         float *tsc = ts + buf * sub;
         if (BITS == 8 && threadIdx.x < rows)
-            tsc[threadIdx.x] = static_cast<const float *>(c.scales)[size_t(b) * c.Tmax + t_begin + st * sub + threadIdx.x];
+            tsc[threadIdx.x] = static_cast<const float *>(c.scales)[size_t(sq) * c.Tmax + t_begin + st * sub + threadIdx.x];
         mbar_wait(&bar[buf], uint32_t((st >> 1) & 1), err);
         __syncthreads();
         // scores of this sub-tile: one warp per token
@@ -353,8 +354,8 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
         if (e != cudaSuccess) return e;
         prof_mark(s, "attn_chunk");
     }
-    if (mma) return launch_combine_mma(a.seq_len, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v, a.O, s);
-    return launch_combine_uv(a.seq_len, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v, a.O, err, s);
+    if (mma) return launch_combine_mma(a.seq_len, c.seq_map, c.nseq, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v, a.O, s);
+    return launch_combine_uv(a.seq_len, c.seq_map, c.nseq, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v, a.O, err, s);
 }
 
 }  // namespace qsvd

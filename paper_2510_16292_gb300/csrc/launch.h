@@ -54,7 +54,11 @@ enum : int { kErrRange = 1, kErrTimeout = 2 };
 int *error_word_for_current_device();
 int set_last_error(int code, const char *msg);
 
-// Plain description of a latent cache (mirrors qsvd_cache).
+// Plain description of a latent cache (mirrors qsvd_cache), seen as B rows
+// of queries.  Without a sequence map, row b is sequence b of the cache
+// (decode: one query per sequence).  With one, row b reads cache sequence
+// seq_map[b] of the nseq the cache holds, so several rows can query the same
+// sequence at different lengths (causal prefill).
 struct CacheView {
     void *codes;
     void *scales;
@@ -62,7 +66,29 @@ struct CacheView {
     int B;
     int Tmax;
     int r;
+    const int32_t *seq_map;   // [B] device, nullable; an input no kernel writes
+    int nseq;                 // sequences held by the cache
 };
+
+#ifdef __CUDACC__
+// Cache sequence behind query row b, or -1 when the map points outside the
+// cache (the row is then treated like one with an invalid length).
+__device__ __forceinline__ int view_seq(const CacheView &c, int b) {
+    if (!c.seq_map) return b;
+    const int q = c.seq_map[b];
+    return q >= 0 && q < c.nseq ? q : -1;
+}
+
+// Length of query row b for the merge kernels: 0 (no partials) when its map
+// entry points outside the cache.
+__device__ __forceinline__ int row_len(const int32_t *seq_len, const int32_t *seq_map, int nseq, int b) {
+    if (seq_map) {
+        const int q = seq_map[b];
+        if (q < 0 || q >= nseq) return 0;
+    }
+    return seq_len[b];
+}
+#endif
 
 // Profiling marker: when the calling thread has enabled profiling
 // (qsvd_profile_events), records the next caller-provided event on `s` and
@@ -142,6 +168,12 @@ struct DecodeArgs {
 };
 size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
 
+// Causal prefill over the cache (qsvd_latent_prefill_attn) runs the decode
+// chain on groups of query rows: at most kPrefillMaxRows rows per group, fewer
+// while a group's workspace would exceed kPrefillWsTarget bytes.
+constexpr int kPrefillMaxRows = 1024;
+constexpr size_t kPrefillWsTarget = size_t(2) << 30;
+
 // a5 and a7/a8 for all B sequences of a step (decode_gemv.cu).
 // decode_mma.cu: tensor-core forms of the three products, for 8 or more sequences
 bool decode_mma_supported(int B, int r, int d, int dh);
@@ -149,14 +181,14 @@ cudaError_t launch_qproj_mma(const CacheView &c, const int32_t *seq_len, const u
                              unsigned *qmax, int n_qmax, int *err, cudaStream_t s);
 cudaError_t launch_qabsorb_mma(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
                                unsigned *qmax, cudaStream_t s);
-cudaError_t launch_combine_mma(const int32_t *seq_len, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
+cudaError_t launch_combine_mma(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
                                const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
                                cudaStream_t s);
 cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
                          unsigned *qmax, int n_qmax, int *err, cudaStream_t s);
 cudaError_t launch_qabsorb(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
                            unsigned *qmax, int *err, cudaStream_t s);
-cudaError_t launch_combine_uv(const int32_t *seq_len, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
+cudaError_t launch_combine_uv(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
                               const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
                               int *err, cudaStream_t s);
 

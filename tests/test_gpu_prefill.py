@@ -1,0 +1,172 @@
+"""Causal prefill attention over the latent cache (qsvd_latent_prefill_attn)
+against the oracle's masked matrix form (oracle.attention.prefill_attention).
+
+Each test projects prompts into the cache on both sides (codes bit-exact),
+then lets every prompt token attend to its own prefix.  Per output row the
+bar is the decode tolerance: max |error| <= 2e-3 * ||row||_2."""
+import numpy as np
+import pytest
+import torch
+
+import synthetic
+from gpu_util import GpuLayer, assert_rows_close, dev, i32, q
+from oracle import attention, pipeline
+
+pytestmark = pytest.mark.gpu
+
+
+def _layers(name, B, n_text, bits, seed, n_image=0, tmax=None):
+    base = synthetic.WORKLOADS[name]
+    wl = synthetic.Workload("prefill", base.shape, B=B, n_image=n_image, n_text=n_text, decode_steps=0,
+                            lat_bits=bits)
+    inp = synthetic.gen_layer(wl, seed=seed)
+    w = pipeline.prepare_weights(inp)
+    tmax = wl.tmax if tmax is None else tmax
+    ref = pipeline.OracleLayer(wl.shape, w, B, tmax, bits, track=[])
+    gpu = GpuLayer(wl.shape, w, B, tmax, bits)
+    return wl, inp, ref, gpu
+
+
+def _gpu_prefill(gpu, q_seq, q_len, max_len=None):
+    s = gpu.s
+    O = torch.full((len(q_seq), s.d), float("nan"), dtype=torch.float32, device=dev())
+    max_len = int(max(q_len)) if max_len is None else max_len
+    gpu.lib.qsvd_latent_prefill_attn(gpu.cache, i32(q_seq), i32(q_len), max_len, gpu.U_q, gpu.U_k, gpu.U_v,
+                                     s.H, s.dh, O)
+    return O
+
+
+def _oracle_rows(ref, b, t0, L):
+    """Oracle outputs of positions t0 .. L-1 of sequence b."""
+    return attention.prefill_attention(ref.cache.rows(b, L), ref.U_q, ref.U_k, ref.U_v, ref.s.H, ref.s.dh,
+                                       t0=t0)
+
+
+def _assert_cache_equal(ref, gpu, b, L):
+    got = gpu.cache.codes[b, :L].cpu().numpy().view(np.uint8)
+    np.testing.assert_array_equal(got, ref.cache.packed_codes()[b, :L].view(np.uint8))
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_prefill_one_prompt(bits):
+    """A 300-token prompt (two full 128-token tiles and a ragged one): every
+    position attends to positions 0 .. itself."""
+    wl, inp, ref, gpu = _layers("llava7b", 1, 300, bits, seed=41)
+    ref.prefill(0, inp.X_prefill[0])
+    gpu.prefill(0, inp.X_prefill[0])
+    _assert_cache_equal(ref, gpu, 0, 300)
+    O = _gpu_prefill(gpu, np.zeros(300), np.arange(1, 301))
+    q().qsvd_check()
+    assert_rows_close(O.cpu().numpy(), _oracle_rows(ref, 0, 0, 300), f"prefill int{bits}")
+
+
+def test_prefill_llava_prompt_all_rows():
+    """The 7B-shaped prompt of 576 image-like and 64 text-like tokens, int8:
+    640 rows in five groups of 128 that reuse one workspace."""
+    wl, inp, ref, gpu = _layers("llava7b", 1, 64, 8, seed=42, n_image=576)
+    ref.prefill(0, inp.X_prefill[0])
+    gpu.prefill(0, inp.X_prefill[0])
+    n = wl.prefill
+    prev = q().qsvd_set_prefill_group_rows(128)
+    try:
+        assert q().qsvd_prefill_workspace_bytes(n, n, wl.shape.r, wl.shape.H, wl.shape.dh) == \
+            q().qsvd_decode_workspace_bytes(128, n, wl.shape.r, wl.shape.H, wl.shape.dh)
+        O = _gpu_prefill(gpu, np.zeros(n), np.arange(1, n + 1))
+        q().qsvd_check()
+    finally:
+        q().qsvd_set_prefill_group_rows(prev)
+    assert_rows_close(O.cpu().numpy(), _oracle_rows(ref, 0, 0, n), "prefill 640")
+
+
+def test_prefill_continuation_and_mixed_rows():
+    """Sequence 0 holds 100 earlier tokens and appends 150 more; sequence 1
+    holds a 200-token prompt.  One call takes the 150 + 200 rows in a shuffled
+    order (int4 cache)."""
+    wl, inp, ref, gpu = _layers("llava7b", 2, 250, 4, seed=43)
+    for side in (ref, gpu):
+        side.prefill(0, inp.X_prefill[0][:100])
+        side.prefill(0, inp.X_prefill[0][100:250])
+        side.prefill(1, inp.X_prefill[1][:200])
+    rows = [(0, 100 + i + 1) for i in range(150)] + [(1, i + 1) for i in range(200)]
+    order = np.random.default_rng(7).permutation(len(rows))
+    q_seq = np.array([rows[k][0] for k in order])
+    q_len = np.array([rows[k][1] for k in order])
+    O = _gpu_prefill(gpu, q_seq, q_len).cpu().numpy()
+    q().qsvd_check()
+    ref0 = _oracle_rows(ref, 0, 100, 250)
+    ref1 = _oracle_rows(ref, 1, 0, 200)
+    want = np.stack([ref0[L - 101] if b == 0 else ref1[L - 1] for b, L in zip(q_seq, q_len)])
+    assert_rows_close(O, want, "mixed rows")
+
+
+def test_prefill_13b_more_than_32_heads():
+    """d = 5120, H = 40 (two head groups on the tcgen05 path), r = 2048."""
+    wl, inp, ref, gpu = _layers("llava13b", 1, 200, 8, seed=44)
+    ref.prefill(0, inp.X_prefill[0])
+    gpu.prefill(0, inp.X_prefill[0])
+    O = _gpu_prefill(gpu, np.zeros(200), np.arange(1, 201))
+    q().qsvd_check()
+    assert_rows_close(O.cpu().numpy(), _oracle_rows(ref, 0, 0, 200), "prefill 13B")
+
+
+def test_prefill_13b_long_prompt_sampled():
+    """One 13B-shaped prompt of 3008 tokens (5 x 576 image-like + 128 text),
+    every row computed on the GPU; sampled rows (tile edges, the middle, the
+    last) checked against the oracle's decode over the prefix."""
+    wl, inp, ref, gpu = _layers("llava13b", 1, 128, 8, seed=45, n_image=2880)
+    ref.prefill(0, inp.X_prefill[0])
+    gpu.prefill(0, inp.X_prefill[0])
+    n = wl.prefill
+    O = _gpu_prefill(gpu, np.zeros(n), np.arange(1, n + 1)).cpu().numpy()
+    q().qsvd_check()
+    assert np.isfinite(O).all()
+    C = ref.cache.rows(0, n)
+    s = wl.shape
+    for t in (0, 1, 127, 128, 1500, n - 1):
+        want = attention.decode_attention(C[:t + 1], ref.U_q, ref.U_k, ref.U_v, s.H, s.dh)
+        assert_rows_close(O[t:t + 1], want[None], f"row {t}")
+
+
+def test_prefill_invalid_rows_are_zero_and_flagged():
+    """Rows whose sequence lies outside the cache or whose length is outside
+    [1, Tmax] are skipped: zero output, QSVD_ERANGE from qsvd_check; the
+    other rows of the call are unaffected."""
+    wl, inp, ref, gpu = _layers("llava7b", 2, 40, 8, seed=46)
+    for side in (ref, gpu):
+        side.prefill(0, inp.X_prefill[0])
+        side.prefill(1, inp.X_prefill[1])
+    lib = q()
+    tmax = gpu.cache.Tmax
+    q_seq = np.array([0, -1, 1, 2, 0, 1, 0])
+    q_len = np.array([5, 5, 40, 3, 0, tmax + 1, 40])
+    O = _gpu_prefill(gpu, q_seq, q_len, max_len=tmax).cpu().numpy()
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_check()
+    assert e.value.status == lib.QSVD_ERANGE
+    lib.qsvd_check()                       # the flag was cleared
+    for i in (1, 3, 4, 5):
+        np.testing.assert_array_equal(O[i], 0.0)
+    want = np.stack([_oracle_rows(ref, 0, 4, 5)[0], _oracle_rows(ref, 1, 39, 40)[0],
+                     _oracle_rows(ref, 0, 39, 40)[0]])
+    assert_rows_close(O[[0, 2, 6]], want, "valid rows")
+
+
+def test_prefill_host_argument_errors():
+    wl, inp, ref, gpu = _layers("llava7b", 1, 16, 8, seed=47)
+    lib, s = q(), wl.shape
+    O = torch.empty((4, s.d), dtype=torch.float32, device=dev())
+    with pytest.raises(ValueError):
+        lib.qsvd_latent_prefill_attn(gpu.cache, i32([0, 0, 0, 0]), i32([1, 2, 3]), 3, gpu.U_q, gpu.U_k, gpu.U_v,
+                                     s.H, s.dh, O)
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_latent_prefill_attn(gpu.cache, i32([0] * 4), i32([1, 2, 3, 4]), gpu.cache.Tmax + 1, gpu.U_q,
+                                     gpu.U_k, gpu.U_v, s.H, s.dh, O)
+    assert e.value.status == lib.QSVD_EINVAL
+    small = torch.zeros(256, dtype=torch.uint8, device=dev())
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_latent_prefill_attn(gpu.cache, i32([0] * 4), i32([1, 2, 3, 4]), 4, gpu.U_q, gpu.U_k, gpu.U_v,
+                                     s.H, s.dh, O, workspace=small)
+    assert e.value.status == lib.QSVD_ENOSPC
+    empty = torch.empty((0,), dtype=torch.int32, device=dev())
+    lib.qsvd_latent_prefill_attn(gpu.cache, empty, empty, 1, gpu.U_q, gpu.U_k, gpu.U_v, s.H, s.dh, O)
+    lib.qsvd_check()

@@ -61,3 +61,45 @@ def test_dominant_token_and_head_blocks():
     o = attention.decode_attention(C, Uq, Uk, Uv, H, dh, softmax_scale=1.0)
     np.testing.assert_allclose(o[:2], Uv[1, :2], atol=1e-12)
     np.testing.assert_allclose(o[2:], (C @ Uv)[:, 2:].mean(0), atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# causal prefill (every prompt token attends to the cached prefix, itself included)
+# ---------------------------------------------------------------------------
+def test_prefill_rows_equal_decode_on_each_prefix():
+    """Row i of the masked matrix form is the decode step of the sequence cut
+    after position t0 + i (decode is pinned above by brute force)."""
+    for seed, (L, t0, r, H, dh) in enumerate([(9, 0, 12, 3, 4), (33, 20, 40, 2, 8), (5, 4, 6, 2, 3)]):
+        C, (Uq, Uk, Uv) = _case(L, r, H, dh, seed + 10)
+        O = attention.prefill_attention(C, Uq, Uk, Uv, H, dh, t0=t0)
+        assert O.shape == (L - t0, H * dh)
+        for i in range(L - t0):
+            ref = attention.decode_attention(C[:t0 + i + 1], Uq, Uk, Uv, H, dh)
+            np.testing.assert_allclose(O[i], ref, atol=1e-12 * max(1.0, np.abs(ref).max()))
+
+
+def test_prefill_equals_brute_force_loops():
+    C, (Uq, Uk, Uv) = _case(L=6, r=5, H=2, dh=3, seed=31)
+    O = attention.prefill_attention(C, Uq, Uk, Uv, 2, 3, t0=1)
+    for i in range(5):
+        np.testing.assert_allclose(O[i], attention.decode_attention_loops(C[:i + 2], Uq, Uk, Uv, 2, 3),
+                                   atol=1e-12)
+
+
+def test_prefill_is_causal():
+    """Changing the latents after position t0 + i leaves row i unchanged and
+    changes the later rows."""
+    C, (Uq, Uk, Uv) = _case(L=12, r=10, H=2, dh=4, seed=32)
+    O = attention.prefill_attention(C, Uq, Uk, Uv, 2, 4)
+    C2 = C.copy()
+    C2[7:] += 5.0
+    O2 = attention.prefill_attention(C2, Uq, Uk, Uv, 2, 4)
+    np.testing.assert_array_equal(O[:7], O2[:7])
+    assert np.abs(O[7:] - O2[7:]).min(axis=1).max() > 1e-3
+
+
+def test_prefill_first_token_is_its_value_row():
+    """Position 0 sees only itself: o = c_0 U_v whatever the query."""
+    C, (Uq, Uk, Uv) = _case(L=4, r=8, H=2, dh=4, seed=33)
+    O = attention.prefill_attention(C, Uq, Uk, Uv, 2, 4)
+    np.testing.assert_allclose(O[0], C[0] @ Uv, atol=1e-13)
