@@ -56,6 +56,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-prefill13", action="store_true")
     p.add_argument("--no-prefill-attn", action="store_true")
+    p.add_argument("--prefill-probe", action="store_true",
+                   help="only time causal prefill attention (both paths, both shapes) and print it")
     p.add_argument("--prefill-sweep", default=None, metavar="ROWS,...",
                    help="only time causal prefill attention for these rows-per-group settings (0 = automatic)")
     # the tiny layer's W_d and U come from the oracle's joint SVD: it is a parity case (tests/), not a benchmark
@@ -486,15 +488,19 @@ PREFILL_SHAPES = {
 }
 
 
-def prefill_attn_probe(name, iters=3, group_rows=0):
+def prefill_attn_probe(name, iters=3, group_rows=0, path="blocks"):
     """Causal prefill attention: every token of B prompts of T tokens attends
-    to its own prefix (qsvd_latent_prefill_attn over all B*T rows in one
-    call), cold L2 before each call.  The cache codes, scales and U are seeded
-    torch random values (the time does not depend on them; the parity tests
-    check the numbers).  Reports the call's time, tokens/s, and the tensor
-    throughput of the attention kernel (scores and the weighted latent sum,
-    4 H r flops per attended token) from a separate pass with library
-    events between the kernels."""
+    to its own prefix, cold L2 before each call.  path "blocks": one
+    qsvd_latent_prefill call over the B prompt blocks (K and V materialised;
+    the fp16 [U_q U_k U_v]^T is prepared once, outside the timed region);
+    path "rows": one qsvd_latent_prefill_attn call over all B*T query rows
+    (the decode kernels' absorbed form).  The cache codes, scales and U are
+    seeded torch random values (the time does not depend on them; the parity
+    tests check the numbers).  Reports the call's time, tokens/s, and per
+    kernel its time share and tensor throughput (algorithmic flops: the
+    Q/K/V product 2*L*r*3d per block, causal attention 4*H*dh per visible
+    (query, key) pair; the absorbed form 4*H*r per pair) from a separate pass
+    with library events between the kernels."""
     import torch
     import paper_2510_16292_gb300 as q
     c = PREFILL_SHAPES[name]
@@ -516,10 +522,16 @@ def prefill_attn_probe(name, iters=3, group_rows=0):
     O = torch.empty((n, H * dh), dtype=torch.float32, device=dev)
     prev = q.qsvd_set_prefill_group_rows(group_rows)
     try:
-        ws = torch.zeros(q.qsvd_prefill_workspace_bytes(n, T, r, H, dh), dtype=torch.uint8, device=dev)
         flush = torch.ones((256 << 20) // 4, dtype=torch.float32, device=dev)
         sink = torch.zeros((), dtype=torch.float32, device=dev)
-        call = lambda: q.qsvd_latent_prefill_attn(cache, q_seq, q_len, T, *U, H, dh, O, workspace=ws)
+        if path == "blocks":
+            blocks = [(b, 0, T) for b in range(B)]
+            Ut = q.qsvd_prefill_weights(*U)
+            ws = torch.zeros(q.qsvd_latent_prefill_workspace_bytes(blocks, r, H, dh), dtype=torch.uint8, device=dev)
+            call = lambda: q.qsvd_latent_prefill(cache, blocks, Ut, H, dh, O, workspace=ws)  # noqa: E731
+        else:
+            ws = torch.zeros(q.qsvd_prefill_workspace_bytes(n, T, r, H, dh), dtype=torch.uint8, device=dev)
+            call = lambda: q.qsvd_latent_prefill_attn(cache, q_seq, q_len, T, *U, H, dh, O, workspace=ws)  # noqa: E731
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         times = []
         for it in range(iters + 1):
@@ -556,23 +568,24 @@ def prefill_attn_probe(name, iters=3, group_rows=0):
         e[0] += 1
         e[1] += events[i - 1].elapsed_time(events[i]) * 1e-3
     tot = sum(v[1] for v in by.values())
-    att = next((k for k in ("attn_tc", "attn_mma", "attn_chunk") if k in by), None)
-    sum_len = B * T * (T + 1) // 2
-    attn_flops = 4.0 * H * r * sum_len
-    exec_flops = attn_flops + 6.0 * n * r * d
+    pairs = B * T * (T + 1) // 2                       # visible (query, key) pairs
+    if path == "blocks":
+        flops = {"qkv_gemm": 2.0 * n * r * 3 * d, "fa": 4.0 * H * dh * pairs}
+    else:
+        att = next((k for k in ("attn_tc", "attn_mma", "attn_chunk") if k in by), "attn_tc")
+        flops = {att: 4.0 * H * r * pairs, "qproj": 2.0 * n * r * d, "qabsorb": 2.0 * n * r * d,
+                 "combine_uv": 2.0 * n * r * d}
     _, bf16_peak, kind = peaks()
     t = min(times)
-    out = {"shape": f"{B} x {T} tokens, d={d} H={H} r={r} int{bits}", "rows": n,
+    kern = {}
+    for k, v in sorted(by.items()):
+        kern[k] = {"launches": v[0], "us": round(v[1] * 1e6, 1), "share": round(v[1] / tot, 4)}
+        if k in flops:
+            kern[k]["tflops"] = round(flops[k] / v[1] / 1e12, 1)
+            kern[k]["frac_of_bf16_peak"] = round(flops[k] / v[1] / 1e12 / bf16_peak, 4)
+    out = {"path": path, "shape": f"{B} x {T} tokens, d={d} H={H} r={r} int{bits}", "rows": n,
            "call_us": round(t * 1e6, 1), "tokens_per_s": round(n / t, 1),
-           "executed_tflops": round(exec_flops / t / 1e12, 2),
-           "kernels": {k: {"launches": v[0], "us": round(v[1] * 1e6, 1), "share": round(v[1] / tot, 4)}
-                       for k, v in sorted(by.items())}}
-    if att:
-        a_t = by[att][1]
-        out["attn_kernel"] = att
-        out["attn_tflops"] = round(attn_flops / a_t / 1e12, 2)
-        out["attn_frac_of_bf16_peak"] = round(attn_flops / a_t / 1e12 / bf16_peak, 4)
-        out["peak_kind"] = kind
+           "call_tflops": round(sum(flops.values()) / t / 1e12, 1), "kernels": kern, "peak_kind": kind}
     del cache, U, O, ws, flush
     return out
 
@@ -666,7 +679,8 @@ def run_native(args, rank, world, local_rank):
                "d2h_bytes_per_step": d2h}
 
     pre13 = prefill_gemm_probe() if not args.no_prefill13 else None
-    pre_attn = None if args.no_prefill_attn else {k: prefill_attn_probe(k) for k in PREFILL_SHAPES}
+    pre_attn = None if args.no_prefill_attn else {
+        k: {p: prefill_attn_probe(k, path=p) for p in ("blocks", "rows")} for k in PREFILL_SHAPES}
     if rank != 0:
         return
     out = {
@@ -903,11 +917,18 @@ def main():
     if args.sweep:
         run_sweep(args)
         return
+    if args.prefill_probe:
+        for name in PREFILL_SHAPES:
+            for path in ("blocks", "rows"):
+                print(json.dumps({"prefill_attn": name, **prefill_attn_probe(name, iters=args.steps, path=path)}),
+                      flush=True)
+        return
     if args.prefill_sweep is not None:
         for rows in (int(x) for x in args.prefill_sweep.split(",")):
             for name in PREFILL_SHAPES:
                 print(json.dumps({"prefill_attn": name, "group_rows": rows,
-                                  **prefill_attn_probe(name, iters=args.steps, group_rows=rows)}), flush=True)
+                                  **prefill_attn_probe(name, iters=args.steps, group_rows=rows, path="rows")}),
+                      flush=True)
         return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))

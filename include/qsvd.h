@@ -15,6 +15,7 @@
  *   qsvd_cache_append        store latent rows in the latent cache (Fig. 2(f))
  *   qsvd_latent_decode_attn  one decode step of attention over that cache (Eq. 5)
  *   qsvd_latent_prefill_attn causal attention of prompt tokens over that cache
+ *   qsvd_latent_prefill      the same for whole prompt blocks, K and V materialised
  *
  * Conventions shared by every entry point:
  *   - Row-vector convention Y = X W, as in the paper.  E = d = H * dh.
@@ -209,6 +210,42 @@ int qsvd_latent_prefill_attn(const qsvd_cache *cache, const int32_t *q_seq, cons
                              void *workspace, size_t workspace_bytes, cudaStream_t stream);
 
 size_t qsvd_prefill_workspace_bytes(int64_t n, int32_t max_len, int32_t r, int32_t H, int32_t dh);
+
+/*
+ * Causal prefill of whole prompt blocks in the materialised form (Eq. 5 as
+ * written): the latent rows of a block are multiplied by U_q, U_k and U_v on
+ * the tensor cores (fp16 operands, fp32 accumulation, fp16 Q, K, V), then
+ * every query attends causally to its prefix at head size dh.  At prefill
+ * this needs r / dh times fewer products than qsvd_latent_prefill_attn, which
+ * keeps the decode kernels' absorbed form; both compute the same attention.
+ *
+ * Block k: positions t0 .. t0+T-1 of cache sequence seq, already stored in
+ * the cache together with positions 0 .. t0-1 (a continued prompt reads
+ * them as keys), attend to positions 0 .. their own.  Its T output rows
+ * follow the rows of blocks 0 .. k-1 in O (fp32 [sum T, H*dh]).  The blocks
+ * array is host memory and is read before the call returns.
+ *   Ut  fp16 [3*H*dh, r]: [U_q U_k U_v]^T from qsvd_prefill_weights (once per
+ *       layer; U_* bf16 [r, H*dh]).
+ *   workspace  qsvd_latent_prefill_workspace_bytes(blocks, n_blocks, r, H, dh)
+ *       bytes: fp16 copies of the blocks' latent rows and of Q, K, V.
+ * Requirements: dh == 128, H*dh % 256 == 0, r % 64 == 0; a block outside the
+ * cache (seq outside [0, B), t0 < 0, T < 1, t0 + T > Tmax) returns
+ * QSVD_EINVAL before anything is enqueued.  fp16 Q, K, V hold magnitudes up
+ * to 65504.
+ */
+typedef struct {
+    int32_t seq, t0, T;
+} qsvd_prefill_block;
+
+int qsvd_prefill_weights(const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v, int32_t r, int32_t d,
+                         uint16_t *Ut, cudaStream_t stream);
+
+int qsvd_latent_prefill(const qsvd_cache *cache, const qsvd_prefill_block *blocks, int32_t n_blocks,
+                        const uint16_t *Ut, int32_t H, int32_t dh, float softmax_scale, float *O,
+                        void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+size_t qsvd_latent_prefill_workspace_bytes(const qsvd_prefill_block *blocks, int32_t n_blocks, int32_t r,
+                                           int32_t H, int32_t dh);
 
 /*
  * One whole decode step for a small batch, in a single launch: for each of

@@ -32,7 +32,8 @@ QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
 EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
-           "qsvd_latent_prefill_attn", "qsvd_prefill_workspace_bytes",
+           "qsvd_latent_prefill_attn", "qsvd_prefill_workspace_bytes", "qsvd_prefill_weights",
+           "qsvd_latent_prefill", "qsvd_latent_prefill_workspace_bytes",
            "qsvd_decode_step", "qsvd_decode_step_workspace_bytes", "qsvd_latent_project_static",
            "qsvd_set_decode_attn_path", "qsvd_set_project_epilogue", "qsvd_set_prefill_group_rows", "qsvd_check", "qsvd_last_error",
            "qsvd_selftest_wait_timeout", "qsvd_version")
@@ -54,6 +55,10 @@ class _Cache(ctypes.Structure):
                 ("B", ctypes.c_int32), ("Tmax", ctypes.c_int32), ("r", ctypes.c_int32)]
 
 
+class _PrefillBlock(ctypes.Structure):
+    _fields_ = [("seq", ctypes.c_int32), ("t0", ctypes.c_int32), ("T", ctypes.c_int32)]
+
+
 _vp, _i32, _i64, _f32, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
 _lib.qsvd_quantize_weight.argtypes = [_vp, _i32, _i32, _f32, _vp, _vp, _vp, _vp]
 _lib.qsvd_latent_project.argtypes = [ctypes.POINTER(_DownWeight), _vp, _i64, _f32, _i32, _f32, _vp, _vp,
@@ -69,6 +74,11 @@ _lib.qsvd_latent_prefill_attn.argtypes = [ctypes.POINTER(_Cache), _vp, _vp, _i64
                                           _f32, _vp, _vp, _sz, _vp]
 _lib.qsvd_prefill_workspace_bytes.argtypes = [_i64, _i32, _i32, _i32, _i32]
 _lib.qsvd_prefill_workspace_bytes.restype = _sz
+_lib.qsvd_prefill_weights.argtypes = [_vp, _vp, _vp, _i32, _i32, _vp, _vp]
+_lib.qsvd_latent_prefill.argtypes = [ctypes.POINTER(_Cache), ctypes.POINTER(_PrefillBlock), _i32, _vp, _i32, _i32,
+                                     _f32, _vp, _vp, _sz, _vp]
+_lib.qsvd_latent_prefill_workspace_bytes.argtypes = [ctypes.POINTER(_PrefillBlock), _i32, _i32, _i32, _i32]
+_lib.qsvd_latent_prefill_workspace_bytes.restype = _sz
 _lib.qsvd_decode_step.argtypes = [ctypes.POINTER(_DownWeight), _vp, ctypes.POINTER(_Cache), _vp, _i32, _vp, _vp,
                                   _vp, _i32, _i32, _f32, _f32, _f32, _vp, _vp, _sz, _vp]
 _lib.qsvd_decode_step_workspace_bytes.argtypes = [_i32, _i32, _i32, _i32, _i32, _i32]
@@ -247,6 +257,42 @@ def qsvd_latent_prefill_attn(cache: LatentCache, q_seq: torch.Tensor, q_len: tor
                                          n, max_len, _ptr(U_q, _BF16, "U_q"), _ptr(U_k, _BF16, "U_k"),
                                          _ptr(U_v, _BF16, "U_v"), H, dh, softmax_scale, _ptr(O, _F32, "O"),
                                          _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def _blocks(blocks):
+    arr = (_PrefillBlock * max(1, len(blocks)))()
+    for i, (b, t0, T) in enumerate(blocks):
+        arr[i] = _PrefillBlock(int(b), int(t0), int(T))
+    return arr
+
+
+def qsvd_prefill_weights(U_q, U_k, U_v, stream=None) -> torch.Tensor:
+    """fp16 [3d, r] = [U_q U_k U_v]^T, the weight operand of qsvd_latent_prefill."""
+    r, d = U_q.shape
+    Ut = torch.empty((3 * d, r), dtype=torch.float16, device=U_q.device)
+    _check(_lib.qsvd_prefill_weights(_ptr(U_q, _BF16, "U_q"), _ptr(U_k, _BF16, "U_k"), _ptr(U_v, _BF16, "U_v"),
+                                     r, d, _ptr(Ut), _stream(stream)))
+    return Ut
+
+
+def qsvd_latent_prefill_workspace_bytes(blocks, r: int, H: int, dh: int) -> int:
+    return int(_lib.qsvd_latent_prefill_workspace_bytes(_blocks(blocks), len(blocks), r, H, dh))
+
+
+def qsvd_latent_prefill(cache: LatentCache, blocks, Ut: torch.Tensor, H: int, dh: int, O: torch.Tensor,
+                        softmax_scale: Optional[float] = None, workspace=None, stream=None) -> None:
+    """blocks: (seq, t0, T) triples; block k's T queries (positions t0 ..
+    t0+T-1 of sequence seq) attend causally to the cache; their outputs follow
+    the earlier blocks' rows in O [sum T, H*dh]."""
+    if softmax_scale is None:
+        softmax_scale = 1.0 / math.sqrt(dh)
+    if workspace is None:
+        workspace = torch.zeros(max(1, qsvd_latent_prefill_workspace_bytes(blocks, cache.r, H, dh)),
+                                dtype=torch.uint8, device=O.device)
+    cc = cache._c()
+    _check(_lib.qsvd_latent_prefill(ctypes.byref(cc), _blocks(blocks), len(blocks), _ptr(Ut, torch.float16, "Ut"), H,
+                                    dh, softmax_scale, _ptr(O, _F32, "O"), _ptr(workspace), workspace.numel(),
+                                    _stream(stream)))
 
 
 def qsvd_decode_step_workspace_bytes(B: int, max_seq_len: int, d: int, r: int, H: int, dh: int) -> int:

@@ -457,6 +457,101 @@ int qsvd_latent_prefill_attn(const qsvd_cache *cache, const int32_t *q_seq, cons
     return QSVD_OK;
 }
 
+}  // extern "C"
+
+// Splits the (validated) host block list into launches of at most
+// kPrefillMaxBlocks blocks and calls f(PrefillBlocks) for each; returns the
+// first non-zero status of f.
+template <typename F>
+static int prefill_chunks(const qsvd_prefill_block *blocks, int32_t n_blocks, F &&f) {
+    int64_t out = 0;
+    for (int32_t i0 = 0; i0 < n_blocks; i0 += kPrefillMaxBlocks) {
+        PrefillBlocks bl{};
+        bl.n = std::min<int32_t>(kPrefillMaxBlocks, n_blocks - i0);
+        int row = 0, tiles = 0;
+        for (int k = 0; k < bl.n; ++k) {
+            const qsvd_prefill_block &b = blocks[i0 + k];     // validated by the caller
+            if (out > INT32_MAX - b.T) return fail(QSVD_EINVAL, "latent_prefill: more than 2^31 output rows");
+            bl.seq[k] = b.seq;
+            bl.t0[k] = b.t0;
+            bl.L[k] = b.t0 + b.T;
+            bl.row_off[k] = row;
+            bl.out_off[k] = int(out);
+            bl.qtile_off[k] = tiles;
+            row += (bl.L[k] + 127) / 128 * 128;
+            tiles += (b.T + 127) / 128;
+            out += b.T;
+        }
+        bl.qtile_off[bl.n] = tiles;
+        const int st = f(bl);
+        if (st) return st;
+    }
+    return QSVD_OK;
+}
+
+extern "C" {
+
+int qsvd_prefill_weights(const uint16_t *U_q, const uint16_t *U_k, const uint16_t *U_v, int32_t r, int32_t d,
+                         uint16_t *Ut, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!U_q || !U_k || !U_v || !Ut) return fail(QSVD_EINVAL, "prefill_weights: null pointer");
+    if (r <= 0 || d <= 0 || r % 64 || d % 256) return fail(QSVD_EUNSUPPORTED, "prefill_weights: need r %% 64 == 0 and d %% 256 == 0");
+    const void *ptrs[] = {U_q, U_k, U_v, Ut};
+    for (const void *p : ptrs)
+        if (!aligned16(p)) return fail(QSVD_EINVAL, "prefill_weights: pointers must be 16-byte aligned");
+    prof_mark(stream, "begin");
+    const cudaError_t e = launch_prefill_weights(U_q, U_k, U_v, r, d, Ut, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "prefill_weights launch");
+}
+
+size_t qsvd_latent_prefill_workspace_bytes(const qsvd_prefill_block *blocks, int32_t n_blocks, int32_t r,
+                                           int32_t H, int32_t dh) {
+    if (!blocks || n_blocks <= 0 || r <= 0 || H <= 0 || dh <= 0) return 0;
+    size_t R = 0;
+    for (int32_t i0 = 0; i0 < n_blocks; i0 += kPrefillMaxBlocks) {
+        size_t Rc = 0;
+        for (int32_t k = i0; k < std::min<int32_t>(n_blocks, i0 + kPrefillMaxBlocks); ++k)
+            Rc += size_t((int64_t(std::max(blocks[k].t0, 0)) + std::max(blocks[k].T, 0) + 127) / 128 * 128);
+        R = std::max(R, Rc);
+    }
+    return prefill_mat_workspace_bytes(R, r, H * dh);
+}
+
+int qsvd_latent_prefill(const qsvd_cache *cache, const qsvd_prefill_block *blocks, int32_t n_blocks,
+                        const uint16_t *Ut, int32_t H, int32_t dh, float softmax_scale, float *O, void *workspace,
+                        size_t workspace_bytes, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if ((st = check_cache(cache))) return st;
+    if (n_blocks < 0) return fail(QSVD_EINVAL, "latent_prefill: n_blocks < 0");
+    if (n_blocks == 0) return QSVD_OK;
+    if (!blocks || !Ut || !O) return fail(QSVD_EINVAL, "latent_prefill: null pointer");
+    if (dh != 128) return fail(QSVD_EUNSUPPORTED, "latent_prefill: dh must be 128 (qsvd_latent_prefill_attn takes dh = 64)");
+    if (H <= 0 || (H * dh) % 256) return fail(QSVD_EUNSUPPORTED, "latent_prefill: need H * dh %% 256 == 0");
+    if (cache->r % 64) return fail(QSVD_EUNSUPPORTED, "latent_prefill: need r %% 64 == 0");
+    const void *ptrs[] = {Ut, O, workspace};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(QSVD_EINVAL, "latent_prefill: pointers must be 16-byte aligned");
+    for (int32_t k = 0; k < n_blocks; ++k) {
+        const qsvd_prefill_block &b = blocks[k];
+        if (b.seq < 0 || b.seq >= cache->B || b.t0 < 0 || b.T < 1 || int64_t(b.t0) + b.T > cache->Tmax)
+            return fail(QSVD_EINVAL, "latent_prefill: block %d (seq %d, t0 %d, T %d) outside the cache", int(k),
+                        int(b.seq), int(b.t0), int(b.T));
+    }
+    const size_t need = qsvd_latent_prefill_workspace_bytes(blocks, n_blocks, cache->r, H, dh);
+    if (!workspace || workspace_bytes < need)
+        return fail(QSVD_ENOSPC, "latent_prefill: workspace needs %zu bytes", need);
+    const CacheView c = view(cache);
+    prof_mark(stream, "begin");
+    return prefill_chunks(blocks, n_blocks, [&](const PrefillBlocks &bl) -> int {
+        const cudaError_t e = launch_prefill_mat(c, bl, Ut, H, softmax_scale, O, workspace, err, stream);
+        return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "latent_prefill launch");
+    });
+}
+
 size_t qsvd_decode_step_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t d, int32_t r, int32_t H,
                                         int32_t dh) {
     if (B <= 0 || max_seq_len <= 0 || d <= 0 || r <= 0 || H <= 0 || dh <= 0) return 0;

@@ -171,6 +171,25 @@ size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
 // Causal prefill over the cache (qsvd_latent_prefill_attn) runs the decode
 // chain on groups of query rows: at most kPrefillMaxRows rows per group, fewer
 // while a group's workspace would exceed kPrefillWsTarget bytes.
+// Materialised causal prefill (prefill_tc.cu): at most kPrefillMaxBlocks
+// prompt blocks per launch.  Block k covers positions t0[k] .. L[k]-1 of cache
+// sequence seq[k] as queries and 0 .. L[k]-1 as keys; its latent rows start
+// at row row_off[k] (a multiple of 128) of the workspace matrices, its
+// outputs at row out_off[k] of O, and its query tiles at qtile_off[k].
+constexpr int kPrefillMaxBlocks = 64;
+struct PrefillBlocks {
+    int n;
+    int seq[kPrefillMaxBlocks], t0[kPrefillMaxBlocks], L[kPrefillMaxBlocks];
+    int row_off[kPrefillMaxBlocks], out_off[kPrefillMaxBlocks];
+    int qtile_off[kPrefillMaxBlocks + 1];
+};
+size_t prefill_mat_rows(const PrefillBlocks &bl);
+size_t prefill_mat_workspace_bytes(size_t R, int r, int d);
+cudaError_t launch_prefill_weights(const uint16_t *Uq, const uint16_t *Uk, const uint16_t *Uv, int r, int d,
+                                   uint16_t *Ut, cudaStream_t s);
+cudaError_t launch_prefill_mat(const CacheView &c, const PrefillBlocks &bl, const uint16_t *Ut, int H,
+                               float softmax_scale, float *O, void *ws, int *err, cudaStream_t s);
+
 constexpr int kPrefillMaxRows = 1024;
 constexpr size_t kPrefillWsTarget = size_t(2) << 30;
 

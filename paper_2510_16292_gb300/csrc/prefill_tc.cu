@@ -1,0 +1,553 @@
+// Causal prefill attention over the latent cache in the materialised form
+// (Eq. 5 as written: K = C U_k, V = C U_v, Q = C U_q, then the decoder's
+// causal softmax attention), on the 5th-generation tensor cores.
+//
+// At prefill every prompt token queries its prefix, so the work is a dense
+// contraction: regrouping U_k into the query (the absorbed form the decode
+// kernels use) would multiply the score and weighted-sum products by r / dh
+// (12 to 16 at the LLaVA shapes).  Here the latent rows of a block are
+// multiplied once by [U_q U_k U_v] and the attention runs at head size dh.
+//
+//   ut_kernel        offline: fp16 [3d, r] = [U_q U_k U_v]^T (bf16 in), so
+//                    that both GEMM operands are K-major
+//   lat_prep_kernel  the latent rows of every block as an fp16 GEMM operand:
+//                    int8 codes (exact in fp16) with the token scale kept
+//                    for the epilogue, or int4 code x group scale rounded to
+//                    fp16 (scale 1); rows padded to 128 per block with zeros
+//   qkv_gemm_kernel  [R, r] x [r, 3d] on tcgen05 (M = 128 rows, N = 256
+//                    columns, K staged 64 at a time through a TMA ring), fp32
+//                    accumulator in tensor memory; the epilogue applies the
+//                    token scale and writes Q and K row-major, V transposed
+//                    ([d, R], so that a key tile of V is K-major for the
+//                    attention's second product), all fp16
+//   fa_kernel        one CTA per (128-query tile, head): S = Q K^T into
+//                    tensor memory (two buffers), causal mask and online
+//                    softmax in registers (thread = query row), P (fp16)
+//                    into tensor memory, O += P V with A from tensor memory;
+//                    O is rescaled only when a row's running maximum grows
+//                    by more than 2^8 (otherwise the stale maximum keeps
+//                    every p below 2^8); K and V stream through 3-deep rings.
+//
+// Every wait is bounded (kErrTimeout on expiry); each CTA frees its tensor
+// memory before it exits.
+#include <algorithm>
+#include <cfloat>
+#include <cmath>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_fp16.h>
+
+#include "common.cuh"
+#include "launch.h"
+#include "tcgen05.cuh"
+
+namespace qsvd {
+
+namespace pf {
+
+constexpr int kRowTile = 128;           // rows per GEMM tile, queries and keys per attention tile
+constexpr int kDh = 128;                // head size of the attention kernel
+
+// ---- Q/K/V GEMM
+constexpr int kGemmN = 256, kGemmK = 64;
+constexpr int kGemmStageA = kRowTile * kGemmK * 2;       // 16 KiB
+constexpr int kGemmStageB = kGemmN * kGemmK * 2;         // 32 KiB
+constexpr int kGemmStages = 4;
+constexpr int kGemmEpiWarps = 8;                         // 2 x 4 lane quadrants x 128 columns
+constexpr int kGemmThreads = 64 + 32 * kGemmEpiWarps;
+constexpr size_t kGemmSmem = size_t(kGemmStages) * (kGemmStageA + kGemmStageB) + 1024;
+
+// ---- attention
+constexpr int kFaThreads = 192;                          // TMA, MMA, 4 softmax warps
+constexpr int kTileBytes = kRowTile * kDh * 2;           // 32 KiB: 128 rows x 128 fp16 (two 64-column boxes)
+constexpr int kBox = kRowTile * 128;                     // 16 KiB: one box (128 rows x 128 bytes)
+constexpr int kRing = 3;
+constexpr size_t kFaSmem = size_t(1 + 2 * kRing) * kTileBytes + 1024;
+constexpr uint32_t kColO = 0, kColS = 128, kColP = 384, kFaTmemCols = 512;
+constexpr float kRescale2 = 8.0f;                        // lazy rescale threshold (log2 units)
+
+}  // namespace pf
+
+// ---------------------------------------------------------------------------
+// [U_q U_k U_v]^T in fp16: Ut[n, k] = U_{n / d}[k, n % d]
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256)
+ut_kernel(const uint16_t *__restrict__ Uq, const uint16_t *__restrict__ Uk, const uint16_t *__restrict__ Uv, int r,
+          int d, __half *__restrict__ Ut) {
+    __shared__ float tile[32][33];
+    const int n0 = blockIdx.x * 32, k0 = blockIdx.y * 32;
+    const int part = n0 / d, c0 = n0 - part * d;
+    const uint16_t *U = part == 0 ? Uq : (part == 1 ? Uk : Uv);
+    for (int i = threadIdx.y; i < 32; i += 8)
+        tile[i][threadIdx.x] = bf16_to_f32(U[size_t(k0 + i) * d + c0 + threadIdx.x]);
+    __syncthreads();
+    for (int i = threadIdx.y; i < 32; i += 8)
+        Ut[size_t(n0 + i) * r + k0 + threadIdx.x] = __float2half_rn(tile[threadIdx.x][i]);
+}
+
+// ---------------------------------------------------------------------------
+// latent rows of the blocks -> fp16 operand A [R, r] and row scale rs [R]
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256)
+lat_prep_kernel(CacheView c, PrefillBlocks bl, int R, __half *__restrict__ A, float *__restrict__ rs) {
+    pdl_wait();
+    pdl_trigger();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int row = blockIdx.x * 8 + warp;
+    if (row >= R) return;
+    int k = 0;
+    while (k + 1 < bl.n && bl.row_off[k + 1] <= row) ++k;
+    const int p = row - bl.row_off[k];
+    const bool live = p < bl.L[k];
+    const int r = c.r;
+    __half *dst = A + size_t(row) * r;
+    const size_t slot = size_t(bl.seq[k]) * c.Tmax + p;
+    if (c.bits == 8) {
+        if (lane == 0) rs[row] = live ? static_cast<const float *>(c.scales)[slot] : 0.0f;
+        const int8_t *src = static_cast<const int8_t *>(c.codes) + slot * r;
+        for (int j = 8 * lane; j < r; j += 256) {
+            uint4 o = make_uint4(0u, 0u, 0u, 0u);
+            if (live) {
+                const uint2 w = *reinterpret_cast<const uint2 *>(src + j);
+                const uint32_t ws[2] = {w.x, w.y};
+                uint32_t h[4];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const __half2 a = __halves2half2(__int2half_rn(int8_t(ws[e] & 0xff)),
+                                                     __int2half_rn(int8_t((ws[e] >> 8) & 0xff)));
+                    const __half2 b = __halves2half2(__int2half_rn(int8_t((ws[e] >> 16) & 0xff)),
+                                                     __int2half_rn(int8_t(ws[e] >> 24)));
+                    h[2 * e] = *reinterpret_cast<const uint32_t *>(&a);
+                    h[2 * e + 1] = *reinterpret_cast<const uint32_t *>(&b);
+                }
+                o = make_uint4(h[0], h[1], h[2], h[3]);
+            }
+            *reinterpret_cast<uint4 *>(dst + j) = o;
+        }
+    } else {
+        if (lane == 0) rs[row] = live ? 1.0f : 0.0f;
+        const uint8_t *src = static_cast<const uint8_t *>(c.codes) + slot * (r / 2);
+        const __half *gs = static_cast<const __half *>(c.scales) + slot * (r / 128);
+        for (int j = 8 * lane; j < r; j += 256) {
+            uint4 o = make_uint4(0u, 0u, 0u, 0u);
+            if (live) {
+                const uint32_t w = *reinterpret_cast<const uint32_t *>(src + j / 2);   // 8 codes, element i in bits 4i..
+                const float s = __half2float(gs[j / 128]);
+                uint32_t h[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int lo = int((w >> (8 * e)) & 0xf), hi = int((w >> (8 * e + 4)) & 0xf);
+                    const __half2 v = __halves2half2(__float2half_rn(float((lo ^ 8) - 8) * s),
+                                                     __float2half_rn(float((hi ^ 8) - 8) * s));
+                    h[e] = *reinterpret_cast<const uint32_t *>(&v);
+                }
+                o = make_uint4(h[0], h[1], h[2], h[3]);
+            }
+            *reinterpret_cast<uint4 *>(dst + j) = o;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Q | K | V^T = (A [R, r] x Ut^T [r, 3d]) * rs[row], fp16 out
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(pf::kGemmThreads, 1)
+qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b, int R, int r,
+                int d, const float *__restrict__ rs, __half *__restrict__ Qm, __half *__restrict__ Km,
+                __half *__restrict__ Vt, int *err) {
+    using namespace pf;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + size_t(kGemmStages) * kGemmStageA;
+    __shared__ __align__(8) uint64_t full_bar[kGemmStages], empty_bar[kGemmStages], acc_full;
+    __shared__ uint32_t tmem_base;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.y * kRowTile, n0 = blockIdx.x * kGemmN;
+    const int n_k = r / kGemmK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kGemmStages; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        mbar_init(&acc_full, 1);
+        mbar_init_fence();
+        tc::prefetch_map(&map_a);
+        tc::prefetch_map(&map_b);
+    }
+    if (warp == 1) tc::tmem_alloc(&tmem_base, kGemmN);
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tmem = tmem_base;
+    pdl_wait();
+    pdl_trigger();
+
+    if (warp == 0) {
+        if (lane == 0) {
+            for (int i = 0; i < n_k; ++i) {
+                const int s = i % kGemmStages;
+                if (i >= kGemmStages && !tc::wait(&empty_bar[s], ((i / kGemmStages) - 1) & 1, err)) break;
+                mbar_arrive_expect_tx(&full_bar[s], kGemmStageA + kGemmStageB);
+                tc::tma_load_2d(sA + size_t(s) * kGemmStageA, &map_a, i * kGemmK, m0, &full_bar[s]);
+                tc::tma_load_2d(sB + size_t(s) * kGemmStageB, &map_b, i * kGemmK, n0, &full_bar[s]);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_f16f32(kGemmN);
+            bool ok = true;
+            for (int i = 0; i < n_k && ok; ++i) {
+                const int s = i % kGemmStages;
+                ok = tc::wait(&full_bar[s], (i / kGemmStages) & 1, err);
+                if (!ok) break;
+                tc::fence_after();
+                const uint32_t a0 = smem_addr(sA + size_t(s) * kGemmStageA);
+                const uint32_t b0 = smem_addr(sB + size_t(s) * kGemmStageB);
+#pragma unroll
+                for (int ks = 0; ks < kGemmK / 16; ++ks)
+                    tc::mma_ss(tmem, tc::desc_sw128(a0 + ks * 32), tc::desc_sw128(b0 + ks * 32), idesc,
+                               (i > 0 || ks > 0) ? 1u : 0u);
+                tc::commit(&empty_bar[s]);
+            }
+            if (ok) tc::commit(&acc_full);
+        }
+    } else {
+        const int quad = warp & 3, col0 = ((warp - 2) >> 2) * 128;
+        const int row = m0 + quad * 32 + lane;
+        const bool ok = tc::wwait(&acc_full, 0, err);
+        tc::fence_after();
+        if (ok) {
+            const float sc = rs[row];
+            const int part = n0 / d, cbase = n0 - part * d + col0;
+            const uint32_t taddr = tmem + (uint32_t(quad * 32) << 16) + uint32_t(col0);
+#pragma unroll 1
+            for (int j0 = 0; j0 < 128; j0 += 32) {
+                uint32_t v[32];
+                tc::tmem_ld32(taddr + j0, v);
+                tc::tmem_wait_ld();
+                uint32_t h[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const __half2 x = __floats2half2_rn(__uint_as_float(v[2 * j]) * sc, __uint_as_float(v[2 * j + 1]) * sc);
+                    h[j] = *reinterpret_cast<const uint32_t *>(&x);
+                }
+                if (part < 2) {
+                    uint4 *dst = reinterpret_cast<uint4 *>((part == 0 ? Qm : Km) + size_t(row) * d + cbase + j0);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) dst[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+                } else {
+                    // V^T: lanes hold consecutive rows, so each column's 32 stores are contiguous
+                    uint16_t *dst = reinterpret_cast<uint16_t *>(Vt) + size_t(cbase + j0) * R + row;
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        dst[size_t(2 * j) * R] = uint16_t(h[j] & 0xffffu);
+                        dst[size_t(2 * j + 1) * R] = uint16_t(h[j] >> 16);
+                    }
+                }
+            }
+        }
+    }
+    tc::fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::fence_after();
+        tc::tmem_free(tmem, kGemmN);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// causal attention, one CTA per (128-query tile, head)
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(pf::kFaThreads, 1)
+fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
+          const __grid_constant__ CUtensorMap map_vt, PrefillBlocks bl, int d, float c_log2, float *__restrict__ O,
+          int *err) {
+    using namespace pf;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sQ = smem;
+    uint8_t *sK = smem + kTileBytes;                         // [kRing] tiles
+    uint8_t *sV = sK + size_t(kRing) * kTileBytes;           // [kRing] tiles (V^T: dh rows x 128 keys)
+    __shared__ __align__(8) uint64_t q_full, k_full[pf::kRing], k_empty[pf::kRing], v_full[pf::kRing],
+        v_empty[pf::kRing], s_full[2], s_empty[2], p_full, o_done;
+    __shared__ uint32_t tmem_base;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    // work unit: query tiles in reverse order (the longest causal rows first)
+    const int tile = int(gridDim.x) - 1 - int(blockIdx.x), h = blockIdx.y;
+    int k = 0;
+    while (k + 1 < bl.n && bl.qtile_off[k + 1] <= tile) ++k;
+    const int qs = bl.t0[k] + (tile - bl.qtile_off[k]) * kRowTile;     // position of the tile's first query
+    const int L = bl.L[k], row0 = bl.row_off[k];
+    const int n = min(qs + kRowTile - 1, L - 1) / kRowTile + 1;         // key tiles up to the last query
+
+    if (threadIdx.x == 0) {
+        mbar_init(&q_full, 1);
+        for (int s = 0; s < kRing; ++s) {
+            mbar_init(&k_full[s], 1);
+            mbar_init(&k_empty[s], 1);
+            mbar_init(&v_full[s], 1);
+            mbar_init(&v_empty[s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&s_full[s], 1);
+            mbar_init(&s_empty[s], 4);
+        }
+        mbar_init(&p_full, 4);
+        mbar_init(&o_done, 1);
+        mbar_init_fence();
+        tc::prefetch_map(&map_q);
+        tc::prefetch_map(&map_k);
+        tc::prefetch_map(&map_vt);
+    }
+    if (warp == 1) tc::tmem_alloc(&tmem_base, kFaTmemCols);
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tmem = tmem_base;
+    pdl_wait();
+    pdl_trigger();
+    const int x0 = h * kDh;                                  // head's first column in Q and K, row in V^T
+
+    if (warp == 0) {
+        // ---------------- TMA producer ----------------
+        if (lane == 0) {
+            mbar_arrive_expect_tx(&q_full, kTileBytes);
+            tc::tma_load_2d(sQ, &map_q, x0, row0 + qs, &q_full);
+            tc::tma_load_2d(sQ + kBox, &map_q, x0 + 64, row0 + qs, &q_full);
+            for (int j = 0; j < n; ++j) {
+                const int s = j % kRing;
+                const uint32_t par = ((j / kRing) - 1) & 1;
+                if (j >= kRing && !tc::wait(&k_empty[s], par, err)) break;
+                mbar_arrive_expect_tx(&k_full[s], kTileBytes);
+                uint8_t *kd = sK + size_t(s) * kTileBytes;
+                tc::tma_load_2d(kd, &map_k, x0, row0 + j * kRowTile, &k_full[s]);
+                tc::tma_load_2d(kd + kBox, &map_k, x0 + 64, row0 + j * kRowTile, &k_full[s]);
+                if (j >= kRing && !tc::wait(&v_empty[s], par, err)) break;
+                mbar_arrive_expect_tx(&v_full[s], kTileBytes);
+                uint8_t *vd = sV + size_t(s) * kTileBytes;
+                tc::tma_load_2d(vd, &map_vt, row0 + j * kRowTile, x0, &v_full[s]);
+                tc::tma_load_2d(vd + kBox, &map_vt, row0 + j * kRowTile + 64, x0, &v_full[s]);
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer ----------------
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_f16f32(kRowTile);
+            const uint32_t q0 = smem_addr(sQ);
+            bool ok = tc::wait(&q_full, 0, err);
+            auto issue_s = [&](int j) -> bool {
+                const int ks = j % kRing, sb = j & 1;
+                if (!tc::wait(&k_full[ks], (j / kRing) & 1, err)) return false;
+                if (j >= 2 && !tc::wait(&s_empty[sb], ((j >> 1) - 1) & 1, err)) return false;
+                tc::fence_after();
+                const uint32_t k0 = smem_addr(sK + size_t(ks) * kTileBytes);
+#pragma unroll
+                for (int kk = 0; kk < kDh / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
+                    tc::mma_ss(tmem + kColS + sb * 128, tc::desc_sw128(q0 + off), tc::desc_sw128(k0 + off), idesc,
+                               kk > 0 ? 1u : 0u);
+                }
+                tc::commit(&s_full[sb]);
+                tc::commit(&k_empty[ks]);
+                return true;
+            };
+            if (ok) ok = issue_s(0);
+            if (ok && n > 1) ok = issue_s(1);
+            for (int j = 0; j < n && ok; ++j) {
+                const int vs = j % kRing;
+                ok = tc::wait(&p_full, j & 1, err) && tc::wait(&v_full[vs], (j / kRing) & 1, err);
+                if (!ok) break;
+                tc::fence_after();
+                const uint32_t v0 = smem_addr(sV + size_t(vs) * kTileBytes);
+#pragma unroll
+                for (int kk = 0; kk < kRowTile / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
+                    tc::mma_ts(tmem + kColO, tmem + kColP + kk * 8, tc::desc_sw128(v0 + off), idesc,
+                               (j > 0 || kk > 0) ? 1u : 0u);
+                }
+                tc::commit(&o_done);
+                tc::commit(&v_empty[vs]);
+                if (j + 2 < n) ok = issue_s(j + 2);
+            }
+        }
+    } else {
+        // ---------------- softmax warps 2..5: thread = query row ----------------
+        const int quad = warp & 3;
+        const int qrow = quad * 32 + lane;
+        const int p = qs + qrow;                                      // query position
+        const uint32_t trow = tmem + (uint32_t(quad * 32) << 16);
+        float m = -INFINITY, l = 0.0f;
+        bool ok = true;
+        for (int j = 0; j < n && ok; ++j) {
+            const int sb = j & 1;
+            ok = tc::wwait(&s_full[sb], (j >> 1) & 1, err);
+            if (!ok) break;
+            tc::fence_after();
+            float x[128];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                uint32_t v[32];
+                tc::tmem_ld32(trow + kColS + sb * 128 + q * 32, v);
+                tc::tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) x[q * 32 + i] = __uint_as_float(v[i]);
+            }
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) tc::arrive(&s_empty[sb]);
+            const int kmax = p - j * kRowTile;                        // keys 0 .. kmax of the tile are visible
+            float mt = -INFINITY;
+#pragma unroll
+            for (int i = 0; i < 128; ++i) {
+                x[i] = i <= kmax ? x[i] * c_log2 : -INFINITY;
+                mt = fmaxf(mt, x[i]);
+            }
+            const float m_new = fmaxf(m, mt);
+            if (j > 0) {
+                ok = tc::wwait(&o_done, (j - 1) & 1, err);
+                if (!ok) break;
+                tc::fence_after();
+                const bool need = m_new > m + kRescale2;
+                if (__any_sync(0xffffffffu, need)) {
+                    const float alpha = need ? exp2f(m - m_new) : 1.0f;
+#pragma unroll 1
+                    for (int q = 0; q < 4; ++q) {
+                        uint32_t v[32];
+                        tc::tmem_ld32(trow + kColO + q * 32, v);
+                        tc::tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+                        tc::tmem_st32(trow + kColO + q * 32, v);
+                    }
+                    tc::tmem_wait_st();
+                    if (need) {
+                        l *= alpha;
+                        m = m_new;
+                    }
+                }
+            } else {
+                m = m_new;
+            }
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                uint32_t pk[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float a = exp2f(x[64 * half + 2 * i] - m), b = exp2f(x[64 * half + 2 * i + 1] - m);
+                    l += a + b;
+                    const __half2 hp = __floats2half2_rn(a, b);
+                    pk[i] = *reinterpret_cast<const uint32_t *>(&hp);
+                }
+                tc::tmem_st32(trow + kColP + half * 32, pk);
+            }
+            tc::tmem_wait_st();
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) tc::arrive(&p_full);
+        }
+        if (ok) ok = tc::wwait(&o_done, (n - 1) & 1, err);
+        tc::fence_after();
+        if (ok) {
+            const float inv = 1.0f / l;
+            const bool live = p < L;
+            float *out = O + (size_t(bl.out_off[k]) + (p - bl.t0[k])) * d + x0;
+#pragma unroll 1
+            for (int q = 0; q < 4; ++q) {
+                uint32_t v[32];
+                tc::tmem_ld32(trow + kColO + q * 32, v);
+                tc::tmem_wait_ld();
+                if (live) {
+#pragma unroll
+                    for (int i = 0; i < 32; i += 4)
+                        *reinterpret_cast<float4 *>(out + q * 32 + i) =
+                            make_float4(__uint_as_float(v[i]) * inv, __uint_as_float(v[i + 1]) * inv,
+                                        __uint_as_float(v[i + 2]) * inv, __uint_as_float(v[i + 3]) * inv);
+                }
+            }
+        }
+    }
+    tc::fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::fence_after();
+        tc::tmem_free(tmem, kFaTmemCols);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+namespace {
+size_t align256(size_t b) { return (b + 255) & ~size_t(255); }
+}  // namespace
+
+size_t prefill_mat_rows(const PrefillBlocks &bl) {
+    size_t R = 0;
+    for (int k = 0; k < bl.n; ++k) R += size_t((bl.L[k] + pf::kRowTile - 1) / pf::kRowTile) * pf::kRowTile;
+    return R;
+}
+
+size_t prefill_mat_workspace_bytes(size_t R, int r, int d) {
+    return align256(R * r * 2) + align256(R * 4) + 3 * align256(R * d * 2);
+}
+
+cudaError_t launch_prefill_weights(const uint16_t *Uq, const uint16_t *Uk, const uint16_t *Uv, int r, int d,
+                                   uint16_t *Ut, cudaStream_t s) {
+    ut_kernel<<<dim3(3 * d / 32, r / 32), dim3(32, 8), 0, s>>>(Uq, Uk, Uv, r, d, reinterpret_cast<__half *>(Ut));
+    const cudaError_t e = cudaGetLastError();
+    prof_mark(s, "ut");
+    return e;
+}
+
+cudaError_t launch_prefill_mat(const CacheView &c, const PrefillBlocks &bl, const uint16_t *Ut, int H,
+                               float softmax_scale, float *O, void *ws, int *err, cudaStream_t s) {
+    using namespace pf;
+    const int r = c.r, d = H * kDh;
+    const int R = int(prefill_mat_rows(bl));
+    char *p = static_cast<char *>(ws);
+    __half *A = reinterpret_cast<__half *>(p);
+    p += align256(size_t(R) * r * 2);
+    float *rs = reinterpret_cast<float *>(p);
+    p += align256(size_t(R) * 4);
+    __half *Qm = reinterpret_cast<__half *>(p);
+    p += align256(size_t(R) * d * 2);
+    __half *Km = reinterpret_cast<__half *>(p);
+    p += align256(size_t(R) * d * 2);
+    __half *Vt = reinterpret_cast<__half *>(p);
+
+    cudaError_t e = launch_pdl(lat_prep_kernel, dim3((R + 7) / 8), dim3(256), 0, s, c, bl, R, A, rs);
+    if (e != cudaSuccess) return e;
+    prof_mark(s, "lat_prep");
+
+    CUtensorMap ma, mb;
+    if (!encode_map_2d(&ma, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, A, uint64_t(r), uint64_t(R), uint64_t(r) * 2, 64,
+                       kRowTile, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_map_2d(&mb, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Ut, uint64_t(r), uint64_t(3 * d), uint64_t(r) * 2, 64,
+                       kGemmN, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    if ((e = ensure_smem(qkv_gemm_kernel, kGemmSmem)) != cudaSuccess) return e;
+    e = launch_pdl(qkv_gemm_kernel, dim3(3 * d / kGemmN, R / kRowTile), dim3(kGemmThreads), kGemmSmem, s, ma, mb, R,
+                   r, d, static_cast<const float *>(rs), Qm, Km, Vt, err);
+    if (e != cudaSuccess) return e;
+    prof_mark(s, "qkv_gemm");
+
+    CUtensorMap mq, mk, mv;
+    if (!encode_map_2d(&mq, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Qm, uint64_t(d), uint64_t(R), uint64_t(d) * 2, 64,
+                       kRowTile, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_map_2d(&mk, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Km, uint64_t(d), uint64_t(R), uint64_t(d) * 2, 64,
+                       kRowTile, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_map_2d(&mv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, Vt, uint64_t(R), uint64_t(d), uint64_t(R) * 2, 64,
+                       kRowTile, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    if ((e = ensure_smem(fa_kernel, kFaSmem)) != cudaSuccess) return e;
+    const float c_log2 = softmax_scale * 1.4426950408889634f;
+    e = launch_pdl(fa_kernel, dim3(bl.qtile_off[bl.n], H), dim3(kFaThreads), kFaSmem, s, mq, mk, mv, bl, d, c_log2, O,
+                   err);
+    prof_mark(s, "fa");
+    return e;
+}
+
+}  // namespace qsvd

@@ -170,3 +170,117 @@ def test_prefill_host_argument_errors():
     empty = torch.empty((0,), dtype=torch.int32, device=dev())
     lib.qsvd_latent_prefill_attn(gpu.cache, empty, empty, 1, gpu.U_q, gpu.U_k, gpu.U_v, s.H, s.dh, O)
     lib.qsvd_check()
+
+
+# ---------------------------------------------------------------------------
+# whole prompt blocks, K and V materialised (qsvd_latent_prefill)
+# ---------------------------------------------------------------------------
+def _gpu_blocks(gpu, blocks, Ut=None):
+    s = gpu.s
+    Ut = gpu.lib.qsvd_prefill_weights(gpu.U_q, gpu.U_k, gpu.U_v) if Ut is None else Ut
+    n = sum(T for _, _, T in blocks)
+    O = torch.full((n, s.d), float("nan"), dtype=torch.float32, device=dev())
+    gpu.lib.qsvd_latent_prefill(gpu.cache, blocks, Ut, s.H, s.dh, O)
+    q().qsvd_check()
+    return O.cpu().numpy()
+
+
+def test_prefill_weights_transpose():
+    """Ut = [U_q U_k U_v]^T in fp16 (bf16 values are exact in fp16 at these
+    magnitudes)."""
+    wl, inp, ref, gpu = _layers("llava7b", 1, 4, 8, seed=50)
+    Ut = gpu.lib.qsvd_prefill_weights(gpu.U_q, gpu.U_k, gpu.U_v).float().cpu().numpy()
+    want = np.concatenate([ref.U_q, ref.U_k, ref.U_v], axis=1).T
+    np.testing.assert_array_equal(Ut, want.astype(np.float16).astype(np.float32))
+
+
+@pytest.mark.parametrize("bits", [8, 4])
+def test_latent_prefill_one_prompt(bits):
+    wl, inp, ref, gpu = _layers("llava7b", 1, 300, bits, seed=51)
+    ref.prefill(0, inp.X_prefill[0])
+    gpu.prefill(0, inp.X_prefill[0])
+    O = _gpu_blocks(gpu, [(0, 0, 300)])
+    assert_rows_close(O, _oracle_rows(ref, 0, 0, 300), f"blocks int{bits}")
+
+
+def test_latent_prefill_llava_prompt():
+    wl, inp, ref, gpu = _layers("llava7b", 1, 64, 8, seed=52, n_image=576)
+    ref.prefill(0, inp.X_prefill[0])
+    gpu.prefill(0, inp.X_prefill[0])
+    n = wl.prefill
+    assert_rows_close(_gpu_blocks(gpu, [(0, 0, n)]), _oracle_rows(ref, 0, 0, n), "blocks 640")
+
+
+def test_latent_prefill_mixed_blocks():
+    """Blocks of two sequences in one call: a continued prompt (t0 = 100), a
+    short block inside another one's range, a block shorter than a tile, and
+    t0 values that are not multiples of 128 (int4 cache)."""
+    wl, inp, ref, gpu = _layers("llava7b", 2, 260, 4, seed=53)
+    for side in (ref, gpu):
+        side.prefill(0, inp.X_prefill[0][:260])
+        side.prefill(1, inp.X_prefill[1][:200])
+    blocks = [(1, 0, 200), (0, 100, 160), (0, 37, 20), (1, 190, 10), (0, 0, 1)]
+    O = _gpu_blocks(gpu, blocks)
+    want = np.concatenate([_oracle_rows(ref, b, t0, t0 + T) for b, t0, T in blocks])
+    assert_rows_close(O, want, "mixed blocks")
+
+
+def test_latent_prefill_13b_heads():
+    wl, inp, ref, gpu = _layers("llava13b", 1, 300, 8, seed=54)
+    ref.prefill(0, inp.X_prefill[0])
+    gpu.prefill(0, inp.X_prefill[0])
+    assert_rows_close(_gpu_blocks(gpu, [(0, 0, 300)]), _oracle_rows(ref, 0, 0, 300), "blocks 13B")
+
+
+def test_latent_prefill_13b_batch_sampled():
+    """The 13B-shaped batch at full size (8 prompts of 5 x 576 + 128 tokens,
+    one call), sampled rows of two prompts checked against the oracle."""
+    wl, inp, ref, gpu = _layers("llava13b", 8, 128, 8, seed=55, n_image=2880)
+    n = wl.prefill
+    for b in range(8):
+        gpu.prefill(b, inp.X_prefill[b])
+    for b in (0, 7):
+        ref.prefill(b, inp.X_prefill[b])
+    O = _gpu_blocks(gpu, [(b, 0, n) for b in range(8)])
+    assert np.isfinite(O).all()
+    s = wl.shape
+    for b in (0, 7):
+        _assert_cache_equal(ref, gpu, b, n)
+        C = ref.cache.rows(b, n)
+        K, V = C @ ref.U_k, C @ ref.U_v
+        for t in (0, 127, 128, 1500, n - 1):
+            want = attention.decode_attention(C[:t + 1], ref.U_q, ref.U_k, ref.U_v, s.H, s.dh,
+                                              K=K[:t + 1], V=V[:t + 1])
+            assert_rows_close(O[b * n + t:b * n + t + 1], want[None], f"seq {b} row {t}")
+
+
+def test_latent_prefill_more_than_64_blocks():
+    """70 blocks take two launches that reuse one workspace."""
+    wl, inp, ref, gpu = _layers("llava7b", 2, 140, 8, seed=56)
+    for side in (ref, gpu):
+        side.prefill(0, inp.X_prefill[0])
+        side.prefill(1, inp.X_prefill[1])
+    blocks = [(i % 2, 2 * i, 1 + i % 3) for i in range(70)]
+    O = _gpu_blocks(gpu, blocks)
+    want = np.concatenate([_oracle_rows(ref, b, t0, t0 + T) for b, t0, T in blocks])
+    assert_rows_close(O, want, "70 blocks")
+
+
+def test_latent_prefill_argument_errors():
+    wl, inp, ref, gpu = _layers("llava7b", 1, 16, 8, seed=57)
+    lib, s = q(), wl.shape
+    Ut = lib.qsvd_prefill_weights(gpu.U_q, gpu.U_k, gpu.U_v)
+    O = torch.empty((16, s.d), dtype=torch.float32, device=dev())
+    for bad in ([(1, 0, 4)], [(0, -1, 4)], [(0, 0, 0)], [(0, 10, 7)], [(0, 0, 4), (-1, 0, 4)]):
+        with pytest.raises(lib.QsvdError) as e:
+            lib.qsvd_latent_prefill(gpu.cache, bad, Ut, s.H, s.dh, O)
+        assert e.value.status == lib.QSVD_EINVAL
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_latent_prefill(gpu.cache, [(0, 0, 4)], Ut, s.H, s.dh, O,
+                                workspace=torch.zeros(256, dtype=torch.uint8, device=dev()))
+    assert e.value.status == lib.QSVD_ENOSPC
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_latent_prefill(gpu.cache, [(0, 0, 4)], Ut, 2 * s.H, 64, O)
+    assert e.value.status == lib.QSVD_EUNSUPPORTED
+    lib.qsvd_latent_prefill(gpu.cache, [], Ut, s.H, s.dh, O)
+    lib.qsvd_check()
