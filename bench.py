@@ -57,7 +57,9 @@ def parse():
     p.add_argument("--no-prefill13", action="store_true")
     p.add_argument("--no-prefill-attn", action="store_true")
     p.add_argument("--prefill-probe", action="store_true",
-                   help="only time causal prefill attention (both paths, both shapes) and print it")
+                   help="only time causal prefill attention and print one line per shape and path")
+    p.add_argument("--prefill-shapes", default=",".join(PREFILL_REPORTED), help="shapes of --prefill-probe")
+    p.add_argument("--prefill-paths", default="blocks,rows", help="paths of --prefill-probe")
     p.add_argument("--prefill-sweep", default=None, metavar="ROWS,...",
                    help="only time causal prefill attention for these rows-per-group settings (0 = automatic)")
     # the tiny layer's W_d and U come from the oracle's joint SVD: it is a parity case (tests/), not a benchmark
@@ -485,7 +487,10 @@ PREFILL_SHAPES = {
     "llava7b": dict(d=4096, H=32, dh=128, r=1536, B=1, T=640, bits=8),
     # the 13B-shaped batch (8 prompts of 5 x 576 + 128 tokens), int8 cache
     "llava13b": dict(d=5120, H=40, dh=128, r=2048, B=8, T=3008, bits=8),
+    # one prompt of the 13B batch (the size for kernel captures)
+    "llava13b_1seq": dict(d=5120, H=40, dh=128, r=2048, B=1, T=3008, bits=8),
 }
+PREFILL_REPORTED = ("llava7b", "llava13b")
 
 
 def prefill_attn_probe(name, iters=3, group_rows=0, path="blocks"):
@@ -680,7 +685,7 @@ def run_native(args, rank, world, local_rank):
 
     pre13 = prefill_gemm_probe() if not args.no_prefill13 else None
     pre_attn = None if args.no_prefill_attn else {
-        k: {p: prefill_attn_probe(k, path=p) for p in ("blocks", "rows")} for k in PREFILL_SHAPES}
+        k: {p: prefill_attn_probe(k, path=p) for p in ("blocks", "rows")} for k in PREFILL_REPORTED}
     if rank != 0:
         return
     out = {
@@ -918,14 +923,14 @@ def main():
         run_sweep(args)
         return
     if args.prefill_probe:
-        for name in PREFILL_SHAPES:
-            for path in ("blocks", "rows"):
+        for name in args.prefill_shapes.split(","):
+            for path in args.prefill_paths.split(","):
                 print(json.dumps({"prefill_attn": name, **prefill_attn_probe(name, iters=args.steps, path=path)}),
                       flush=True)
         return
     if args.prefill_sweep is not None:
         for rows in (int(x) for x in args.prefill_sweep.split(",")):
-            for name in PREFILL_SHAPES:
+            for name in PREFILL_REPORTED:
                 print(json.dumps({"prefill_attn": name, "group_rows": rows,
                                   **prefill_attn_probe(name, iters=args.steps, group_rows=rows, path="rows")}),
                       flush=True)

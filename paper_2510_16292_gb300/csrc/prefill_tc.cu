@@ -26,7 +26,8 @@
 //                    into tensor memory, O += P V with A from tensor memory;
 //                    O is rescaled only when a row's running maximum grows
 //                    by more than 2^8 (otherwise the stale maximum keeps
-//                    every p below 2^8); K and V stream through 3-deep rings.
+//                    every p below 2^8); K and V stream through rings of
+//                    3 and 2 tiles.
 //
 // Every wait is bounded (kErrTimeout on expiry); each CTA frees its tensor
 // memory before it exits.
@@ -58,15 +59,36 @@ constexpr int kGemmThreads = 64 + 32 * kGemmEpiWarps;
 constexpr size_t kGemmSmem = size_t(kGemmStages) * (kGemmStageA + kGemmStageB) + 1024;
 
 // ---- attention
-constexpr int kFaThreads = 192;                          // TMA, MMA, 4 softmax warps
+constexpr int kFaThreads = 352;                          // TMA (Q, K), MMA, 8 softmax warps, TMA (V)
 constexpr int kTileBytes = kRowTile * kDh * 2;           // 32 KiB: 128 rows x 128 fp16 (two 64-column boxes)
 constexpr int kBox = kRowTile * 128;                     // 16 KiB: one box (128 rows x 128 bytes)
-constexpr int kRing = 3;
-constexpr size_t kFaSmem = size_t(1 + 2 * kRing) * kTileBytes + 1024;
-constexpr uint32_t kColO = 0, kColS = 128, kColP = 384, kFaTmemCols = 512;
+constexpr int kRingK = 3, kRingV = 2;                    // K tiles are needed two products before V tiles
+constexpr size_t kFaSmem = size_t(1 + kRingK + kRingV) * kTileBytes + 1024;
+constexpr uint32_t kColO = 0, kColS = 128, kColP = 384, kFaTmemCols = 512;   // S, P: two buffers each
 constexpr float kRescale2 = 8.0f;                        // lazy rescale threshold (log2 units)
 
 }  // namespace pf
+
+// AND of `v` over the 64 threads of named barrier `id` (the two softmax
+// warps of one tensor-memory lane quadrant); also orders their shared-memory
+// accesses like bar.sync.
+__device__ __forceinline__ bool pair_all(bool v, int id) {
+    uint32_t r;
+    asm volatile("{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, %2, 64, p;\n\t"
+                 "selp.u32 %0, 1, 0, q;\n\t}"
+                 : "=r"(r)
+                 : "r"(uint32_t(v)), "r"(id)
+                 : "memory");
+    return r != 0;
+}
+
+// 2^x with the MUFU approximation (relative error about 2^-22; x = -inf and
+// x below the fp32 range give +0).
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
 
 // ---------------------------------------------------------------------------
 // [U_q U_k U_v]^T in fp16: Ut[n, k] = U_{n / d}[k, n % d]
@@ -92,60 +114,52 @@ __global__ void __launch_bounds__(256)
 lat_prep_kernel(CacheView c, PrefillBlocks bl, int R, __half *__restrict__ A, float *__restrict__ rs) {
     pdl_wait();
     pdl_trigger();
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int row = blockIdx.x * 8 + warp;
-    if (row >= R) return;
+    const int r = c.r, per_row = r / 8;                       // threads per row: 8 channels each
+    const int t = int(blockIdx.x) * blockDim.x + threadIdx.x;      // R * r / 8 < 2^31 (checked by the host)
+    if (t >= R * per_row) return;
+    const int row = t / per_row, j = (t - row * per_row) * 8;
     int k = 0;
     while (k + 1 < bl.n && bl.row_off[k + 1] <= row) ++k;
     const int p = row - bl.row_off[k];
     const bool live = p < bl.L[k];
-    const int r = c.r;
-    __half *dst = A + size_t(row) * r;
     const size_t slot = size_t(bl.seq[k]) * c.Tmax + p;
+    uint4 o = make_uint4(0u, 0u, 0u, 0u);
     if (c.bits == 8) {
-        if (lane == 0) rs[row] = live ? static_cast<const float *>(c.scales)[slot] : 0.0f;
-        const int8_t *src = static_cast<const int8_t *>(c.codes) + slot * r;
-        for (int j = 8 * lane; j < r; j += 256) {
-            uint4 o = make_uint4(0u, 0u, 0u, 0u);
-            if (live) {
-                const uint2 w = *reinterpret_cast<const uint2 *>(src + j);
-                const uint32_t ws[2] = {w.x, w.y};
-                uint32_t h[4];
+        if (j == 0) rs[row] = live ? static_cast<const float *>(c.scales)[slot] : 0.0f;
+        if (live) {
+            const uint2 w = *reinterpret_cast<const uint2 *>(static_cast<const int8_t *>(c.codes) + slot * r + j);
+            const uint32_t ws[2] = {w.x, w.y};
+            uint32_t h[4];
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const __half2 a = __halves2half2(__int2half_rn(int8_t(ws[e] & 0xff)),
-                                                     __int2half_rn(int8_t((ws[e] >> 8) & 0xff)));
-                    const __half2 b = __halves2half2(__int2half_rn(int8_t((ws[e] >> 16) & 0xff)),
-                                                     __int2half_rn(int8_t(ws[e] >> 24)));
-                    h[2 * e] = *reinterpret_cast<const uint32_t *>(&a);
-                    h[2 * e + 1] = *reinterpret_cast<const uint32_t *>(&b);
-                }
-                o = make_uint4(h[0], h[1], h[2], h[3]);
+            for (int e = 0; e < 2; ++e) {
+                const __half2 a = __halves2half2(__int2half_rn(int8_t(ws[e] & 0xff)),
+                                                 __int2half_rn(int8_t((ws[e] >> 8) & 0xff)));
+                const __half2 b = __halves2half2(__int2half_rn(int8_t((ws[e] >> 16) & 0xff)),
+                                                 __int2half_rn(int8_t(ws[e] >> 24)));
+                h[2 * e] = *reinterpret_cast<const uint32_t *>(&a);
+                h[2 * e + 1] = *reinterpret_cast<const uint32_t *>(&b);
             }
-            *reinterpret_cast<uint4 *>(dst + j) = o;
+            o = make_uint4(h[0], h[1], h[2], h[3]);
         }
     } else {
-        if (lane == 0) rs[row] = live ? 1.0f : 0.0f;
-        const uint8_t *src = static_cast<const uint8_t *>(c.codes) + slot * (r / 2);
-        const __half *gs = static_cast<const __half *>(c.scales) + slot * (r / 128);
-        for (int j = 8 * lane; j < r; j += 256) {
-            uint4 o = make_uint4(0u, 0u, 0u, 0u);
-            if (live) {
-                const uint32_t w = *reinterpret_cast<const uint32_t *>(src + j / 2);   // 8 codes, element i in bits 4i..
-                const float s = __half2float(gs[j / 128]);
-                uint32_t h[4];
+        if (j == 0) rs[row] = live ? 1.0f : 0.0f;
+        if (live) {
+            // 8 codes, element i in bits 4i .. 4i+3, times the group's fp16 scale
+            const uint32_t w = *reinterpret_cast<const uint32_t *>(static_cast<const uint8_t *>(c.codes) +
+                                                                   slot * (r / 2) + j / 2);
+            const float s = __half2float(static_cast<const __half *>(c.scales)[slot * (r / 128) + j / 128]);
+            uint32_t h[4];
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int lo = int((w >> (8 * e)) & 0xf), hi = int((w >> (8 * e + 4)) & 0xf);
-                    const __half2 v = __halves2half2(__float2half_rn(float((lo ^ 8) - 8) * s),
-                                                     __float2half_rn(float((hi ^ 8) - 8) * s));
-                    h[e] = *reinterpret_cast<const uint32_t *>(&v);
-                }
-                o = make_uint4(h[0], h[1], h[2], h[3]);
+            for (int e = 0; e < 4; ++e) {
+                const int lo = int((w >> (8 * e)) & 0xf), hi = int((w >> (8 * e + 4)) & 0xf);
+                const __half2 v = __halves2half2(__float2half_rn(float((lo ^ 8) - 8) * s),
+                                                 __float2half_rn(float((hi ^ 8) - 8) * s));
+                h[e] = *reinterpret_cast<const uint32_t *>(&v);
             }
-            *reinterpret_cast<uint4 *>(dst + j) = o;
+            o = make_uint4(h[0], h[1], h[2], h[3]);
         }
     }
+    *reinterpret_cast<uint4 *>(A + size_t(row) * r + j) = o;
 }
 
 // ---------------------------------------------------------------------------
@@ -268,11 +282,13 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sQ = smem;
-    uint8_t *sK = smem + kTileBytes;                         // [kRing] tiles
-    uint8_t *sV = sK + size_t(kRing) * kTileBytes;           // [kRing] tiles (V^T: dh rows x 128 keys)
-    __shared__ __align__(8) uint64_t q_full, k_full[pf::kRing], k_empty[pf::kRing], v_full[pf::kRing],
-        v_empty[pf::kRing], s_full[2], s_empty[2], p_full, o_done;
+    uint8_t *sK = smem + kTileBytes;                         // [kRingK] tiles
+    uint8_t *sV = sK + size_t(kRingK) * kTileBytes;          // [kRingV] tiles (V^T: dh rows x 128 keys)
+    __shared__ __align__(8) uint64_t q_full, k_full[pf::kRingK], k_empty[pf::kRingK], v_full[pf::kRingV],
+        v_empty[pf::kRingV], s_full[2], s_empty[2], p_full[2], o_done[2];
     __shared__ uint32_t tmem_base;
+    __shared__ float red[2][2][pf::kRowTile];              // partial row maxima [tile parity][half][row]
+    __shared__ float lsum[2][pf::kRowTile];                // partial row sums [half][row]
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     // work unit: query tiles in reverse order (the longest causal rows first)
@@ -285,18 +301,20 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
 
     if (threadIdx.x == 0) {
         mbar_init(&q_full, 1);
-        for (int s = 0; s < kRing; ++s) {
+        for (int s = 0; s < kRingK; ++s) {
             mbar_init(&k_full[s], 1);
             mbar_init(&k_empty[s], 1);
+        }
+        for (int s = 0; s < kRingV; ++s) {
             mbar_init(&v_full[s], 1);
             mbar_init(&v_empty[s], 1);
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&s_full[s], 1);
-            mbar_init(&s_empty[s], 4);
+            mbar_init(&s_empty[s], 8);
+            mbar_init(&p_full[s], 8);     // P buffer s written (one arrival per softmax warp)
+            mbar_init(&o_done[s], 1);     // the O += P V that read P buffer s has completed
         }
-        mbar_init(&p_full, 4);
-        mbar_init(&o_done, 1);
         mbar_init_fence();
         tc::prefetch_map(&map_q);
         tc::prefetch_map(&map_k);
@@ -312,24 +330,31 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
     const int x0 = h * kDh;                                  // head's first column in Q and K, row in V^T
 
     if (warp == 0) {
-        // ---------------- TMA producer ----------------
+        // ---------------- TMA producer of Q and K ----------------
         if (lane == 0) {
             mbar_arrive_expect_tx(&q_full, kTileBytes);
             tc::tma_load_2d(sQ, &map_q, x0, row0 + qs, &q_full);
             tc::tma_load_2d(sQ + kBox, &map_q, x0 + 64, row0 + qs, &q_full);
             for (int j = 0; j < n; ++j) {
-                const int s = j % kRing;
-                const uint32_t par = ((j / kRing) - 1) & 1;
-                if (j >= kRing && !tc::wait(&k_empty[s], par, err)) break;
-                mbar_arrive_expect_tx(&k_full[s], kTileBytes);
-                uint8_t *kd = sK + size_t(s) * kTileBytes;
-                tc::tma_load_2d(kd, &map_k, x0, row0 + j * kRowTile, &k_full[s]);
-                tc::tma_load_2d(kd + kBox, &map_k, x0 + 64, row0 + j * kRowTile, &k_full[s]);
-                if (j >= kRing && !tc::wait(&v_empty[s], par, err)) break;
-                mbar_arrive_expect_tx(&v_full[s], kTileBytes);
-                uint8_t *vd = sV + size_t(s) * kTileBytes;
-                tc::tma_load_2d(vd, &map_vt, row0 + j * kRowTile, x0, &v_full[s]);
-                tc::tma_load_2d(vd + kBox, &map_vt, row0 + j * kRowTile + 64, x0, &v_full[s]);
+                const int ks = j % kRingK;
+                if (j >= kRingK && !tc::wait(&k_empty[ks], ((j / kRingK) - 1) & 1, err)) break;
+                mbar_arrive_expect_tx(&k_full[ks], kTileBytes);
+                uint8_t *kd = sK + size_t(ks) * kTileBytes;
+                tc::tma_load_2d(kd, &map_k, x0, row0 + j * kRowTile, &k_full[ks]);
+                tc::tma_load_2d(kd + kBox, &map_k, x0 + 64, row0 + j * kRowTile, &k_full[ks]);
+            }
+        }
+    } else if (warp == kFaThreads / 32 - 1) {
+        // ---------------- TMA producer of V (its own warp: a V stage frees only
+        // when O += P V has run, which must not hold back the K stream) ----------------
+        if (lane == 0) {
+            for (int j = 0; j < n; ++j) {
+                const int vs = j % kRingV;
+                if (j >= kRingV && !tc::wait(&v_empty[vs], ((j / kRingV) - 1) & 1, err)) break;
+                mbar_arrive_expect_tx(&v_full[vs], kTileBytes);
+                uint8_t *vd = sV + size_t(vs) * kTileBytes;
+                tc::tma_load_2d(vd, &map_vt, row0 + j * kRowTile, x0, &v_full[vs]);
+                tc::tma_load_2d(vd + kBox, &map_vt, row0 + j * kRowTile + 64, x0, &v_full[vs]);
             }
         }
     } else if (warp == 1) {
@@ -339,8 +364,8 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
             const uint32_t q0 = smem_addr(sQ);
             bool ok = tc::wait(&q_full, 0, err);
             auto issue_s = [&](int j) -> bool {
-                const int ks = j % kRing, sb = j & 1;
-                if (!tc::wait(&k_full[ks], (j / kRing) & 1, err)) return false;
+                const int ks = j % kRingK, sb = j & 1;
+                if (!tc::wait(&k_full[ks], (j / kRingK) & 1, err)) return false;
                 if (j >= 2 && !tc::wait(&s_empty[sb], ((j >> 1) - 1) & 1, err)) return false;
                 tc::fence_after();
                 const uint32_t k0 = smem_addr(sK + size_t(ks) * kTileBytes);
@@ -357,107 +382,143 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
             if (ok) ok = issue_s(0);
             if (ok && n > 1) ok = issue_s(1);
             for (int j = 0; j < n && ok; ++j) {
-                const int vs = j % kRing;
-                ok = tc::wait(&p_full, j & 1, err) && tc::wait(&v_full[vs], (j / kRing) & 1, err);
+                // S_{j+2} goes to the tensor pipe as soon as the softmax has read S_j
+                // (early in its work on tile j), ahead of O += P_j V, so the scores
+                // of a tile are ready long before the softmax reaches it
+                if (j + 2 < n && !(ok = issue_s(j + 2))) break;
+                const int vs = j % kRingV, pb = j & 1;
+                ok = tc::wait(&p_full[pb], (j >> 1) & 1, err) && tc::wait(&v_full[vs], (j / kRingV) & 1, err);
                 if (!ok) break;
                 tc::fence_after();
                 const uint32_t v0 = smem_addr(sV + size_t(vs) * kTileBytes);
 #pragma unroll
                 for (int kk = 0; kk < kRowTile / 16; ++kk) {
                     const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
-                    tc::mma_ts(tmem + kColO, tmem + kColP + kk * 8, tc::desc_sw128(v0 + off), idesc,
+                    tc::mma_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8, tc::desc_sw128(v0 + off), idesc,
                                (j > 0 || kk > 0) ? 1u : 0u);
                 }
-                tc::commit(&o_done);
+                tc::commit(&o_done[pb]);
                 tc::commit(&v_empty[vs]);
-                if (j + 2 < n) ok = issue_s(j + 2);
             }
         }
     } else {
-        // ---------------- softmax warps 2..5: thread = query row ----------------
-        const int quad = warp & 3;
+        // ---------------- softmax warps 2..9: thread = query row ----------------
+        // Two warps per tensor-memory lane quadrant; warp half h (0 or 1) takes
+        // keys 64h .. 64h+63 of every tile (and O columns 64h .. 64h+63).  The
+        // partners swap their partial row maxima through shared memory (slot
+        // by tile parity) under a 64-thread named barrier, so both hold the
+        // same running maximum m of s * c_log2 (c_log2 > 0); p = 2^(s c_log2 -
+        // m).  P alternates between two tensor-memory buffers, so tile j is
+        // written while O += P_{j-1} V still runs; only a rescale of O waits
+        // for that product.  The partial row sums meet at the end.
+        const int quad = warp & 3, half = (warp - 2) >> 2;
         const int qrow = quad * 32 + lane;
         const int p = qs + qrow;                                      // query position
         const uint32_t trow = tmem + (uint32_t(quad * 32) << 16);
-        float m = -INFINITY, l = 0.0f;
+        const int bar_id = 1 + quad;                                  // named barrier of the quadrant's pair
+        float m = -INFINITY, ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
         bool ok = true;
-        for (int j = 0; j < n && ok; ++j) {
-            const int sb = j & 1;
-            ok = tc::wwait(&s_full[sb], (j >> 1) & 1, err);
-            if (!ok) break;
-            tc::fence_after();
-            float x[128];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                uint32_t v[32];
-                tc::tmem_ld32(trow + kColS + sb * 128 + q * 32, v);
-                tc::tmem_wait_ld();
-#pragma unroll
-                for (int i = 0; i < 32; ++i) x[q * 32 + i] = __uint_as_float(v[i]);
-            }
-            tc::fence_before();
-            __syncwarp();
-            if (lane == 0) tc::arrive(&s_empty[sb]);
-            const int kmax = p - j * kRowTile;                        // keys 0 .. kmax of the tile are visible
+        // Both warps of a pair run the same iterations: the outcome of every
+        // bounded wait is AND-reduced over the pair at the exchange barrier, and
+        // a failure ends the loop for both there, so neither is ever left alone
+        // at a named barrier.
+        for (int j = 0; j < n; ++j) {
+            const int sb = j & 1, pb = j & 1;
+            const bool got = ok && tc::wwait(&s_full[sb], (j >> 1) & 1, err);
+            uint32_t v[2][32];
             float mt = -INFINITY;
-#pragma unroll
-            for (int i = 0; i < 128; ++i) {
-                x[i] = i <= kmax ? x[i] * c_log2 : -INFINITY;
-                mt = fmaxf(mt, x[i]);
-            }
-            const float m_new = fmaxf(m, mt);
-            if (j > 0) {
-                ok = tc::wwait(&o_done, (j - 1) & 1, err);
-                if (!ok) break;
+            if (got) {
                 tc::fence_after();
+#pragma unroll
+                for (int q = 0; q < 2; ++q) tc::tmem_ld32(trow + kColS + sb * 128 + half * 64 + q * 32, v[q]);
+                tc::tmem_wait_ld();
+                tc::fence_before();
+                __syncwarp();
+                if (lane == 0) tc::arrive(&s_empty[sb]);
+                const int kmax = p - j * kRowTile - half * 64;        // keys 0 .. kmax of this half are visible
+                if (kmax < 63) {
+#pragma unroll
+                    for (int i = 0; i < 64; ++i)
+                        if (i > kmax) v[i >> 5][i & 31] = __float_as_uint(-INFINITY);
+                }
+                float mx[4];                                          // chain e: keys i = e (mod 4), then a tree
+#pragma unroll
+                for (int e = 0; e < 4; ++e) mx[e] = __uint_as_float(v[0][e]);
+#pragma unroll
+                for (int i = 4; i < 64; ++i) mx[i & 3] = fmaxf(mx[i & 3], __uint_as_float(v[i >> 5][i & 31]));
+                mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+            }
+            red[j & 1][half][qrow] = mt;
+            ok = pair_all(got, bar_id);
+            if (!ok) break;
+            mt = fmaxf(mt, red[j & 1][half ^ 1][qrow]);
+            const float m_new = fmaxf(m, mt * c_log2);
+            if (j > 0) {
                 const bool need = m_new > m + kRescale2;
                 if (__any_sync(0xffffffffu, need)) {
-                    const float alpha = need ? exp2f(m - m_new) : 1.0f;
+                    // O must hold every product up to tile j-1 before it is scaled
+                    ok = tc::wwait(&o_done[pb ^ 1], ((j - 1) >> 1) & 1, err);
+                    if (ok) {
+                        tc::fence_after();
+                        const float alpha = need ? ex2_approx(m - m_new) : 1.0f;
 #pragma unroll 1
-                    for (int q = 0; q < 4; ++q) {
-                        uint32_t v[32];
-                        tc::tmem_ld32(trow + kColO + q * 32, v);
-                        tc::tmem_wait_ld();
+                        for (int q = 0; q < 2; ++q) {
+                            uint32_t o[32];
+                            tc::tmem_ld32(trow + kColO + half * 64 + q * 32, o);
+                            tc::tmem_wait_ld();
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
-                        tc::tmem_st32(trow + kColO + q * 32, v);
-                    }
-                    tc::tmem_wait_st();
-                    if (need) {
-                        l *= alpha;
-                        m = m_new;
+                            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                            tc::tmem_st32(trow + kColO + half * 64 + q * 32, o);
+                        }
+                        tc::tmem_wait_st();
+                        if (need) {
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) ls[e] *= alpha;
+                            m = m_new;
+                        }
                     }
                 }
             } else {
                 m = m_new;
             }
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
+            if (ok && j >= 2) {                                       // P buffer pb was read by O += P_{j-2} V
+                ok = tc::wwait(&o_done[pb], ((j - 2) >> 1) & 1, err);
+                if (ok) tc::fence_after();
+            }
+            if (ok) {
                 uint32_t pk[32];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const float a = exp2f(x[64 * half + 2 * i] - m), b = exp2f(x[64 * half + 2 * i + 1] - m);
-                    l += a + b;
+                for (int i = 0; i < 32; ++i) {                        // column i of this half: keys 64 half + 2i, +1
+                    const float a = ex2_approx(fmaf(__uint_as_float(v[(2 * i) >> 5][(2 * i) & 31]), c_log2, -m));
+                    const float b =
+                        ex2_approx(fmaf(__uint_as_float(v[(2 * i + 1) >> 5][(2 * i + 1) & 31]), c_log2, -m));
+                    ls[(2 * i) & 3] += a;
+                    ls[(2 * i + 1) & 3] += b;
                     const __half2 hp = __floats2half2_rn(a, b);
                     pk[i] = *reinterpret_cast<const uint32_t *>(&hp);
                 }
-                tc::tmem_st32(trow + kColP + half * 32, pk);
+                tc::tmem_st32(trow + kColP + pb * 64 + half * 32, pk);
+                tc::tmem_wait_st();
+                tc::fence_before();
+                __syncwarp();
+                if (lane == 0) tc::arrive(&p_full[pb]);
             }
-            tc::tmem_wait_st();
-            tc::fence_before();
-            __syncwarp();
-            if (lane == 0) tc::arrive(&p_full);
         }
-        if (ok) ok = tc::wwait(&o_done, (n - 1) & 1, err);
+        // both halves' sums of the row (the pair leaves the loop together)
+        float l = (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        lsum[half][qrow] = l;
+        ok = pair_all(ok, bar_id);
+        l += lsum[half ^ 1][qrow];
+        if (ok) ok = tc::wwait(&o_done[(n - 1) & 1], ((n - 1) >> 1) & 1, err);
         tc::fence_after();
         if (ok) {
             const float inv = 1.0f / l;
             const bool live = p < L;
-            float *out = O + (size_t(bl.out_off[k]) + (p - bl.t0[k])) * d + x0;
+            float *out = O + (size_t(bl.out_off[k]) + (p - bl.t0[k])) * d + x0 + half * 64;
 #pragma unroll 1
-            for (int q = 0; q < 4; ++q) {
+            for (int q = 0; q < 2; ++q) {
                 uint32_t v[32];
-                tc::tmem_ld32(trow + kColO + q * 32, v);
+                tc::tmem_ld32(trow + kColO + half * 64 + q * 32, v);
                 tc::tmem_wait_ld();
                 if (live) {
 #pragma unroll
@@ -518,7 +579,9 @@ cudaError_t launch_prefill_mat(const CacheView &c, const PrefillBlocks &bl, cons
     p += align256(size_t(R) * d * 2);
     __half *Vt = reinterpret_cast<__half *>(p);
 
-    cudaError_t e = launch_pdl(lat_prep_kernel, dim3((R + 7) / 8), dim3(256), 0, s, c, bl, R, A, rs);
+    const int64_t prep_threads = int64_t(R) * (r / 8);
+    cudaError_t e = launch_pdl(lat_prep_kernel, dim3(unsigned((prep_threads + 255) / 256)), dim3(256), 0, s, c, bl, R,
+                               A, rs);
     if (e != cudaSuccess) return e;
     prof_mark(s, "lat_prep");
 
