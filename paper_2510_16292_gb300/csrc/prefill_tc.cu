@@ -15,8 +15,10 @@
 //                    for the epilogue, or int4 code x group scale rounded to
 //                    fp16 (scale 1); rows padded to 128 per block with zeros
 //   qkv_gemm_kernel  [R, r] x [r, 3d] on tcgen05 (M = 128 rows, N = 256
-//                    columns, K staged 64 at a time through a TMA ring), fp32
-//                    accumulator in tensor memory; the epilogue applies the
+//                    columns, K staged 64 at a time through a TMA ring), one
+//                    persistent CTA per SM with two fp32 accumulators in
+//                    tensor memory (the epilogue of a tile overlaps the main
+//                    loop of the next); the epilogue applies the
 //                    token scale and writes Q and K row-major, V transposed
 //                    ([d, R], so that a key tile of V is K-major for the
 //                    attention's second product), all fp16
@@ -169,28 +171,35 @@ __global__ void __launch_bounds__(pf::kGemmThreads, 1)
 qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b, int R, int r,
                 int d, const float *__restrict__ rs, __half *__restrict__ Qm, __half *__restrict__ Km,
                 __half *__restrict__ Vt, int *err) {
+    // Persistent: CTA c takes tiles c, c + gridDim.x, ... (N fastest, so the
+    // CTAs in flight share A rows and all of Ut stays in L2).  Two tensor-memory
+    // accumulators alternate between a CTA's tiles, so the epilogue of one tile
+    // overlaps the main loop of the next.
     using namespace pf;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sA = smem;
     uint8_t *sB = smem + size_t(kGemmStages) * kGemmStageA;
-    __shared__ __align__(8) uint64_t full_bar[kGemmStages], empty_bar[kGemmStages], acc_full;
+    __shared__ __align__(8) uint64_t full_bar[kGemmStages], empty_bar[kGemmStages], acc_full[2], acc_empty[2];
     __shared__ uint32_t tmem_base;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.y * kRowTile, n0 = blockIdx.x * kGemmN;
     const int n_k = r / kGemmK;
+    const int tiles_n = 3 * d / kGemmN, n_tiles = (R / kRowTile) * tiles_n;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kGemmStages; ++s) {
             mbar_init(&full_bar[s], 1);
             mbar_init(&empty_bar[s], 1);
         }
-        mbar_init(&acc_full, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], kGemmEpiWarps);
+        }
         mbar_init_fence();
         tc::prefetch_map(&map_a);
         tc::prefetch_map(&map_b);
     }
-    if (warp == 1) tc::tmem_alloc(&tmem_base, kGemmN);
+    if (warp == 1) tc::tmem_alloc(&tmem_base, 2 * kGemmN);
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
@@ -200,42 +209,57 @@ qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant
 
     if (warp == 0) {
         if (lane == 0) {
-            for (int i = 0; i < n_k; ++i) {
-                const int s = i % kGemmStages;
-                if (i >= kGemmStages && !tc::wait(&empty_bar[s], ((i / kGemmStages) - 1) & 1, err)) break;
-                mbar_arrive_expect_tx(&full_bar[s], kGemmStageA + kGemmStageB);
-                tc::tma_load_2d(sA + size_t(s) * kGemmStageA, &map_a, i * kGemmK, m0, &full_bar[s]);
-                tc::tma_load_2d(sB + size_t(s) * kGemmStageB, &map_b, i * kGemmK, n0, &full_bar[s]);
+            int it = 0;                                       // k-stages issued by this CTA so far
+            bool ok = true;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                const int m0 = (t / tiles_n) * kRowTile, n0 = (t % tiles_n) * kGemmN;
+                for (int i = 0; i < n_k; ++i, ++it) {
+                    const int s = it % kGemmStages;
+                    if (it >= kGemmStages && !(ok = tc::wait(&empty_bar[s], ((it / kGemmStages) - 1) & 1, err)))
+                        break;
+                    mbar_arrive_expect_tx(&full_bar[s], kGemmStageA + kGemmStageB);
+                    tc::tma_load_2d(sA + size_t(s) * kGemmStageA, &map_a, i * kGemmK, m0, &full_bar[s]);
+                    tc::tma_load_2d(sB + size_t(s) * kGemmStageB, &map_b, i * kGemmK, n0, &full_bar[s]);
+                }
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_f16f32(kGemmN);
             bool ok = true;
-            for (int i = 0; i < n_k && ok; ++i) {
-                const int s = i % kGemmStages;
-                ok = tc::wait(&full_bar[s], (i / kGemmStages) & 1, err);
-                if (!ok) break;
+            int it = 0, ti = 0;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ti) {
+                const int buf = ti & 1;
+                if (ti >= 2 && !(ok = tc::wait(&acc_empty[buf], ((ti >> 1) - 1) & 1, err))) break;
                 tc::fence_after();
-                const uint32_t a0 = smem_addr(sA + size_t(s) * kGemmStageA);
-                const uint32_t b0 = smem_addr(sB + size_t(s) * kGemmStageB);
+                const uint32_t acc = tmem + uint32_t(buf * kGemmN);
+                for (int i = 0; i < n_k; ++i, ++it) {
+                    const int s = it % kGemmStages;
+                    if (!(ok = tc::wait(&full_bar[s], (it / kGemmStages) & 1, err))) break;
+                    tc::fence_after();
+                    const uint32_t a0 = smem_addr(sA + size_t(s) * kGemmStageA);
+                    const uint32_t b0 = smem_addr(sB + size_t(s) * kGemmStageB);
 #pragma unroll
-                for (int ks = 0; ks < kGemmK / 16; ++ks)
-                    tc::mma_ss(tmem, tc::desc_sw128(a0 + ks * 32), tc::desc_sw128(b0 + ks * 32), idesc,
-                               (i > 0 || ks > 0) ? 1u : 0u);
-                tc::commit(&empty_bar[s]);
+                    for (int ks = 0; ks < kGemmK / 16; ++ks)
+                        tc::mma_ss(acc, tc::desc_sw128(a0 + ks * 32), tc::desc_sw128(b0 + ks * 32), idesc,
+                                   (i > 0 || ks > 0) ? 1u : 0u);
+                    tc::commit(&empty_bar[s]);
+                }
+                if (ok) tc::commit(&acc_full[buf]);
             }
-            if (ok) tc::commit(&acc_full);
         }
     } else {
         const int quad = warp & 3, col0 = ((warp - 2) >> 2) * 128;
-        const int row = m0 + quad * 32 + lane;
-        const bool ok = tc::wwait(&acc_full, 0, err);
-        tc::fence_after();
-        if (ok) {
+        int ti = 0;
+        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++ti) {
+            const int buf = ti & 1;
+            const int m0 = (t / tiles_n) * kRowTile, n0 = (t % tiles_n) * kGemmN;
+            const int row = m0 + quad * 32 + lane;
+            if (!tc::wwait(&acc_full[buf], (ti >> 1) & 1, err)) break;
+            tc::fence_after();
             const float sc = rs[row];
             const int part = n0 / d, cbase = n0 - part * d + col0;
-            const uint32_t taddr = tmem + (uint32_t(quad * 32) << 16) + uint32_t(col0);
+            const uint32_t taddr = tmem + (uint32_t(quad * 32) << 16) + uint32_t(buf * kGemmN + col0);
 #pragma unroll 1
             for (int j0 = 0; j0 < 128; j0 += 32) {
                 uint32_t v[32];
@@ -261,13 +285,17 @@ qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant
                     }
                 }
             }
+            // this warp's columns of the accumulator are drained
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) tc::arrive(&acc_empty[buf]);
         }
     }
     tc::fence_before();
     __syncthreads();
     if (warp == 1) {
         tc::fence_after();
-        tc::tmem_free(tmem, kGemmN);
+        tc::tmem_free(tmem, 2 * kGemmN);
     }
 }
 
@@ -592,8 +620,11 @@ cudaError_t launch_prefill_mat(const CacheView &c, const PrefillBlocks &bl, cons
                        kGemmN, CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
     if ((e = ensure_smem(qkv_gemm_kernel, kGemmSmem)) != cudaSuccess) return e;
-    e = launch_pdl(qkv_gemm_kernel, dim3(3 * d / kGemmN, R / kRowTile), dim3(kGemmThreads), kGemmSmem, s, ma, mb, R,
-                   r, d, static_cast<const float *>(rs), Qm, Km, Vt, err);
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int gemm_tiles = (3 * d / kGemmN) * (R / kRowTile);
+    e = launch_pdl(qkv_gemm_kernel, dim3(std::min(gemm_tiles, sms)), dim3(kGemmThreads), kGemmSmem, s, ma, mb, R, r, d,
+                   static_cast<const float *>(rs), Qm, Km, Vt, err);
     if (e != cudaSuccess) return e;
     prof_mark(s, "qkv_gemm");
 
