@@ -61,7 +61,7 @@ constexpr int kGemmThreads = 64 + 32 * kGemmEpiWarps;
 constexpr size_t kGemmSmem = size_t(kGemmStages) * (kGemmStageA + kGemmStageB) + 1024;
 
 // ---- attention
-constexpr int kFaThreads = 352;                          // TMA (Q, K), MMA, 8 softmax warps, TMA (V)
+constexpr int kFaThreads = 384;                          // TMA (Q, K), S MMAs, 8 softmax, TMA (V), PV MMAs
 constexpr int kTileBytes = kRowTile * kDh * 2;           // 32 KiB: 128 rows x 128 fp16 (two 64-column boxes)
 constexpr int kBox = kRowTile * 128;                     // 16 KiB: one box (128 rows x 128 bytes)
 constexpr int kRingK = 3, kRingV = 2;                    // K tiles are needed two products before V tiles
@@ -372,7 +372,7 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
                 tc::tma_load_2d(kd + kBox, &map_k, x0 + 64, row0 + j * kRowTile, &k_full[ks]);
             }
         }
-    } else if (warp == kFaThreads / 32 - 1) {
+    } else if (warp == kFaThreads / 32 - 2) {
         // ---------------- TMA producer of V (its own warp: a V stage frees only
         // when O += P V has run, which must not hold back the K stream) ----------------
         if (lane == 0) {
@@ -386,15 +386,20 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
             }
         }
     } else if (warp == 1) {
-        // ---------------- MMA issuer ----------------
+        // ---------------- S = Q K^T issuer ----------------
+        // The scores and O += P V are issued from two threads: one thread
+        // spends ~100 cycles per tcgen05.mma, more than a 128 x 128 x 16
+        // product takes, so a single issuer would bound the tensor pipe.  The
+        // two touch disjoint tensor memory (S buffers vs P buffers and O), and
+        // each commit tracks its own thread's products.
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_f16f32(kRowTile);
             const uint32_t q0 = smem_addr(sQ);
             bool ok = tc::wait(&q_full, 0, err);
-            auto issue_s = [&](int j) -> bool {
+            for (int j = 0; j < n && ok; ++j) {
                 const int ks = j % kRingK, sb = j & 1;
-                if (!tc::wait(&k_full[ks], (j / kRingK) & 1, err)) return false;
-                if (j >= 2 && !tc::wait(&s_empty[sb], ((j >> 1) - 1) & 1, err)) return false;
+                if (!(ok = tc::wait(&k_full[ks], (j / kRingK) & 1, err))) break;
+                if (j >= 2 && !(ok = tc::wait(&s_empty[sb], ((j >> 1) - 1) & 1, err))) break;
                 tc::fence_after();
                 const uint32_t k0 = smem_addr(sK + size_t(ks) * kTileBytes);
 #pragma unroll
@@ -405,15 +410,14 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
                 }
                 tc::commit(&s_full[sb]);
                 tc::commit(&k_empty[ks]);
-                return true;
-            };
-            if (ok) ok = issue_s(0);
-            if (ok && n > 1) ok = issue_s(1);
+            }
+        }
+    } else if (warp == kFaThreads / 32 - 1) {
+        // ---------------- O += P V issuer ----------------
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_f16f32(kRowTile);
+            bool ok = true;
             for (int j = 0; j < n && ok; ++j) {
-                // S_{j+2} goes to the tensor pipe as soon as the softmax has read S_j
-                // (early in its work on tile j), ahead of O += P_j V, so the scores
-                // of a tile are ready long before the softmax reaches it
-                if (j + 2 < n && !(ok = issue_s(j + 2))) break;
                 const int vs = j % kRingV, pb = j & 1;
                 ok = tc::wait(&p_full[pb], (j >> 1) & 1, err) && tc::wait(&v_full[vs], (j / kRingV) & 1, err);
                 if (!ok) break;
