@@ -13,7 +13,9 @@ events on the launching stream around each sub-step.
 
 value = decode tokens/s (all ranks' tokens / max-over-ranks decode time).
 Secondary figures: prefill TOPS (2*T*d*r over the projection call), latent
-cache GB/s, and the decode step's fraction of its HBM roofline.
+cache GB/s, the decode step's fraction of its HBM roofline, and the causal
+prefill attention of the 7B prompt and the 13B batch (tokens/s and per-kernel
+fractions of the bf16 tensor peak, both entry points).
 
 --impl reference times the CPU oracle (the plain fp64 definition) on a
 bounded sample of the same workload on the host cores.

@@ -1,6 +1,7 @@
 // C ABI of the QSVD latent-attention path (declared in include/qsvd.h):
 // argument validation, workspace carving and kernel launch order.
 #include <algorithm>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -532,6 +533,8 @@ int qsvd_latent_prefill(const qsvd_cache *cache, const qsvd_prefill_block *block
     if (dh != 128) return fail(QSVD_EUNSUPPORTED, "latent_prefill: dh must be 128 (qsvd_latent_prefill_attn takes dh = 64)");
     if (H <= 0 || (H * dh) % 256) return fail(QSVD_EUNSUPPORTED, "latent_prefill: need H * dh %% 256 == 0");
     if (cache->r % 64) return fail(QSVD_EUNSUPPORTED, "latent_prefill: need r %% 64 == 0");
+    if (!(softmax_scale > 0.0f) || !std::isfinite(softmax_scale))
+        return fail(QSVD_EINVAL, "latent_prefill: softmax_scale must be positive and finite");
     const void *ptrs[] = {Ut, O, workspace};
     for (const void *p : ptrs)
         if (p && !aligned16(p)) return fail(QSVD_EINVAL, "latent_prefill: pointers must be 16-byte aligned");

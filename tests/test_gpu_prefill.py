@@ -282,5 +282,9 @@ def test_latent_prefill_argument_errors():
     with pytest.raises(lib.QsvdError) as e:
         lib.qsvd_latent_prefill(gpu.cache, [(0, 0, 4)], Ut, 2 * s.H, 64, O)
     assert e.value.status == lib.QSVD_EUNSUPPORTED
+    for bad_scale in (0.0, -0.1, float("inf")):
+        with pytest.raises(lib.QsvdError) as e:
+            lib.qsvd_latent_prefill(gpu.cache, [(0, 0, 4)], Ut, s.H, s.dh, O, softmax_scale=bad_scale)
+        assert e.value.status == lib.QSVD_EINVAL
     lib.qsvd_latent_prefill(gpu.cache, [], Ut, s.H, s.dh, O)
     lib.qsvd_check()
