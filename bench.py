@@ -58,6 +58,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-prefill13", action="store_true")
     p.add_argument("--no-prefill-attn", action="store_true")
+    p.add_argument("--rot", action="store_true",
+                   help="rotate X by H1 on the fly (Eq. 12; weights quantized as H1 W_d) in every projection")
     p.add_argument("--prefill-probe", action="store_true",
                    help="only time causal prefill attention and print one line per shape and path")
     p.add_argument("--prefill-shapes", default=",".join(PREFILL_REPORTED), help="shapes of --prefill-probe")
@@ -155,7 +157,8 @@ class NativeLayer:
             a = np.ascontiguousarray(bits).view(np.int16)
             return torch.from_numpy(a).view(torch.bfloat16).to(dev)
 
-        self.W = q.qsvd_quantize_weight(torch.from_numpy(inp.W_d.astype(np.float32)).to(dev))
+        rot = (s.d & -s.d) if nb.rot else 0             # H1 on the fly: the largest power-of-two block
+        self.W = q.qsvd_quantize_weight(torch.from_numpy(inp.W_d.astype(np.float32)).to(dev), rot=rot)
         self.U = [bf16(u) for u in (inp.U_q, inp.U_k, inp.U_v)]
         if X_from is None:
             self.Xp = bf16(inp.X_prefill.reshape(wl.B * wl.prefill, s.d))
@@ -174,10 +177,10 @@ class NativeBench:
     cached, as it does in serving.  `flush`: one copy, L2 evicted by a 256 MiB
     read before every sub-step (code cold as well)."""
 
-    def __init__(self, wl, rank, l2="rotate"):
+    def __init__(self, wl, rank, l2="rotate", rot=False):
         import torch
         import paper_2510_16292_gb300 as q
-        self.torch, self.q, self.wl = torch, q, wl
+        self.torch, self.q, self.wl, self.rot = torch, q, wl, rot
         s = wl.shape
         self.dev = torch.device("cuda", torch.cuda.current_device())
         dev = self.dev
@@ -624,7 +627,7 @@ def run_native(args, rank, world, local_rank):
     wl = synthetic.WORKLOADS[args.workload]
     if args.decode_steps:
         wl = dataclasses.replace(wl, decode_steps=args.decode_steps)
-    nb = NativeBench(wl, rank, l2=args.l2)
+    nb = NativeBench(wl, rank, l2=args.l2, rot=args.rot)
     K = nb.K
     S = wl.decode_steps
     hbm, _, peak_kind = peaks()
@@ -696,7 +699,8 @@ def run_native(args, rank, world, local_rank):
         "ms_per_step": round((dec_total + pre_total) / args.steps * 1e3, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int8/fp32",
         "data": "synthetic",
-        "config": {"workload": workload_desc(wl), "global_batch": world * wl.B,
+        "config": {"workload": workload_desc(wl) + (" + online H1 rotation of X (Eq. 12)" if args.rot else ""),
+                   "global_batch": world * wl.B,
                    "seq_len": wl.tmax, "parallelism": f"replicas x{world} (one independent layer per GPU)",
                    "l2": (f"inputs larger than L2: {K} independently seeded copies of the layer "
                           f"({K} x {nb.layer_bytes / 2**20:.0f} MiB of weights and latent cache); every decode "

@@ -11,6 +11,7 @@
  *
  * This library implements, on the caller's CUDA stream:
  *   qsvd_quantize_weight     offline per-channel int8 RTN of W_d (Sec. 4 setup)
+ *   qsvd_quantize_weight_rotated  the same of H1 W_d (Eq. 12's online rotation)
  *   qsvd_latent_project      C = Q(X) Q(W_d), requantized per token (Eq. 11-12)
  *   qsvd_cache_append        store latent rows in the latent cache (Fig. 2(f))
  *   qsvd_latent_decode_attn  one decode step of attention over that cache (Eq. 5)
@@ -89,6 +90,9 @@ typedef struct qsvd_down_weight {
     const float    *scale;       /* [r]    */
     int32_t d;
     int32_t r;
+    int32_t rot;                 /* 0: the codes quantize W_d and X is quantized as it is (H1 = I or folded
+                                    offline); b > 0: they quantize H1 W_d (qsvd_quantize_weight_rotated) and
+                                    qsvd_latent_project rotates every row of X by H1 before quantizing it */
 } qsvd_down_weight;
 
 /*
@@ -146,6 +150,25 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
                         void *workspace, size_t workspace_bytes, cudaStream_t stream);
 
 size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r);
+
+/*
+ * The rotation H1 of Eq. 11-12 applied on the fly (for models where it is not
+ * folded into the previous layer): C = Q(X H1^T) Q(H1 W_d).  H1 is the
+ * block-diagonal normalized Walsh-Hadamard matrix I_{d/rot} (x) H_rot /
+ * sqrt(rot) (Sylvester H_rot, rot a power of two >= 2 dividing d; the
+ * largest such rot spreads outliers furthest), symmetric and orthogonal, so
+ * (X H1)(H1 W_d) = X W_d.  Both the weight quantizer below and
+ * qsvd_latent_project compute it as the fast Walsh-Hadamard transform in fp32
+ * (stages h = 1, 2, ..., rot/2 in that order, pair (i, i+h) with (i & h) == 0
+ * -> (v_i + v_{i+h}, v_i - v_{i+h}), then every entry times fp32(1/sqrt(rot))),
+ * so the codes are reproducible bit for bit.
+ * qsvd_quantize_weight_rotated: as qsvd_quantize_weight, of H1 W_d; the
+ * caller sets rot in the qsvd_down_weight it builds from the outputs.
+ * Needs d <= 6144.  qsvd_decode_step and qsvd_latent_project_static refuse
+ * rotated weights (QSVD_EUNSUPPORTED).
+ */
+int qsvd_quantize_weight_rotated(const float *W_d, int32_t d, int32_t r, float clip, int32_t rot, int8_t *codes,
+                                 uint16_t *codes_bf16, float *scale, cudaStream_t stream);
 
 /*
  * Latent cache append (the store of Fig. 2(f)): row i of the token-major

@@ -1,9 +1,9 @@
 """The quantized joint down-projection and the latent cache (Sec. 3.1, 3.3).
 
-Eq. 12: C_qkv ~= Q(X H1^T) Q(H1 W^d_qkv H2^T).  The rotations H1, H2 are
-folded offline into the weights (Sec. 2.3 background: X' = XH with the
-matching H^T applied to W), so on this path H1 = H2 = I and
-C_qkv ~= Q(X) Q(W_d):
+Eq. 12: C_qkv ~= Q(X H1^T) Q(H1 W^d_qkv H2^T).  H2 folds offline into the
+weights (Sec. 2.3 background: X' = XH with the matching H^T applied to W).
+H1 is either folded too (H1 = I here: C_qkv ~= Q(X) Q(W_d)) or applied to X
+on the fly (``rot``, oracle.rotate) with W_d replaced by H1 W_d:
 
   1. X [T, d] -> int8 codes Xq and an fp32 scale s_x per token;
   2. acc[t, j] = sum_k Xq[t, k] * Wq[k, j]      (exact integer arithmetic);
@@ -17,7 +17,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from . import quant
+from . import quant, rotate
 
 
 def int_matmul(A, B):
@@ -61,9 +61,13 @@ def requantize_latent(c_hat, lat_bits: int, lat_clip: float = 1.0):
     raise ValueError("lat_bits must be 8 or 4")
 
 
-def latent_project(X, Wq, s_w, act_clip=1.0, lat_bits=8, lat_clip=1.0):
+def latent_project(X, Wq, s_w, act_clip=1.0, lat_bits=8, lat_clip=1.0, rot: int = 0):
     """Steps 1-4 for a block of tokens.  Returns a dict with every
-    intermediate the GPU path can expose: xq, s_x, acc, c_hat, codes, scale."""
+    intermediate the GPU path can expose: xq, s_x, acc, c_hat, codes, scale.
+    rot = b > 0: the rows are rotated by H1 (block b, oracle.rotate) before
+    step 1, as Eq. 12 quantizes X H1^T; Wq must then be the codes of H1 W^d."""
+    if rot:
+        X = rotate.rotate_rows(np.asarray(X, dtype=np.float32), rot)
     xq, s_x = quantize_activations(X, act_clip)
     acc = down_project(xq, Wq)
     c_hat = dequantize_acc(acc, s_x, s_w)

@@ -21,14 +21,16 @@ import numpy as np
 
 from synthetic import LayerInputs, bf16_bits, bf16_from_bits
 
-from . import attention, latent, quant, svd
+from . import attention, latent, quant, rotate, svd
 
 TINY_BETA = 0.5
 
 
-def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1.0):
+def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1.0, rot: int = 0):
     """Returns dict(W_d fp32 values [d, r], Wq int64 [d, r], s_w [r],
-    U_q/U_k/U_v bf16 bits [r, d])."""
+    U_q/U_k/U_v bf16 bits [r, d], rot).  rot = b > 0: Wq, s_w quantize
+    H1 W_d (oracle.rotate, block b) instead of W_d (W_d itself is returned
+    unrotated: it is what the caller hands to the GPU's rotating quantizer)."""
     s = inp.workload.shape
     if inp.W_qkv is not None:
         d = s.d
@@ -38,9 +40,9 @@ def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1
         U_q, U_k, U_v = bf16_bits(Uq), bf16_bits(Uk), bf16_bits(Uv)
     else:
         W_d, U_q, U_k, U_v = inp.W_d, inp.U_q, inp.U_k, inp.U_v
-    Wq, s_w = quant.quantize_columns(W_d, 8, w_clip)
+    Wq, s_w = quant.quantize_columns(rotate.rotate_weight(W_d, rot) if rot else W_d, 8, w_clip)
     c = np.ascontiguousarray
-    return dict(W_d=c(W_d), Wq=c(Wq), s_w=c(s_w), U_q=c(U_q), U_k=c(U_k), U_v=c(U_v))
+    return dict(W_d=c(W_d), Wq=c(Wq), s_w=c(s_w), U_q=c(U_q), U_k=c(U_k), U_v=c(U_v), rot=rot)
 
 
 class OracleLayer:
@@ -66,7 +68,7 @@ class OracleLayer:
         """Eq. 12 for a block of tokens given as bf16 bits [T, d]."""
         X = bf16_from_bits(X_bits)
         return latent.latent_project(X, self.w["Wq"], self.w["s_w"],
-                                     self.act_clip, self.bits, self.lat_clip)
+                                     self.act_clip, self.bits, self.lat_clip, self.w.get("rot", 0))
 
     def _append(self, seq, pos, codes, scale):
         self.cache.append(seq, pos, codes, scale)

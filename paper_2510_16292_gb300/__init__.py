@@ -30,7 +30,7 @@ _lib = ctypes.CDLL(_LIB_PATH)
 
 QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
-EXPORTS = ("qsvd_quantize_weight", "qsvd_latent_project", "qsvd_project_workspace_bytes",
+EXPORTS = ("qsvd_quantize_weight", "qsvd_quantize_weight_rotated", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
            "qsvd_latent_prefill_attn", "qsvd_prefill_workspace_bytes", "qsvd_prefill_weights",
            "qsvd_latent_prefill", "qsvd_latent_prefill_workspace_bytes",
@@ -47,7 +47,7 @@ class QsvdError(RuntimeError):
 
 class _DownWeight(ctypes.Structure):
     _fields_ = [("codes", ctypes.c_void_p), ("codes_bf16", ctypes.c_void_p), ("scale", ctypes.c_void_p),
-                ("d", ctypes.c_int32), ("r", ctypes.c_int32)]
+                ("d", ctypes.c_int32), ("r", ctypes.c_int32), ("rot", ctypes.c_int32)]
 
 
 class _Cache(ctypes.Structure):
@@ -61,6 +61,7 @@ class _PrefillBlock(ctypes.Structure):
 
 _vp, _i32, _i64, _f32, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
 _lib.qsvd_quantize_weight.argtypes = [_vp, _i32, _i32, _f32, _vp, _vp, _vp, _vp]
+_lib.qsvd_quantize_weight_rotated.argtypes = [_vp, _i32, _i32, _f32, _i32, _vp, _vp, _vp, _vp]
 _lib.qsvd_latent_project.argtypes = [ctypes.POINTER(_DownWeight), _vp, _i64, _f32, _i32, _f32, _vp, _vp,
                                      ctypes.POINTER(_Cache), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
 _lib.qsvd_project_workspace_bytes.argtypes = [_i64, _i32, _i32]
@@ -125,10 +126,13 @@ def _check(status: int):
 
 @dataclasses.dataclass
 class DownWeight:
-    """Quantized W_d: codes int8 [r, d], codes_bf16 bf16 [r, d], scale fp32 [r]."""
+    """Quantized W_d: codes int8 [r, d], codes_bf16 bf16 [r, d], scale fp32 [r];
+    rot > 0: the codes quantize H1 W_d (block Hadamard of rot channels) and
+    the projection rotates X by H1 on the fly."""
     codes: torch.Tensor
     codes_bf16: torch.Tensor
     scale: torch.Tensor
+    rot: int = 0
 
     @property
     def d(self):
@@ -140,7 +144,7 @@ class DownWeight:
 
     def _c(self):
         return _DownWeight(_ptr(self.codes, torch.int8, "W.codes"), _ptr(self.codes_bf16, _BF16, "W.codes_bf16"),
-                           _ptr(self.scale, _F32, "W.scale"), self.d, self.r)
+                           _ptr(self.scale, _F32, "W.scale"), self.d, self.r, self.rot)
 
 
 @dataclasses.dataclass
@@ -173,16 +177,21 @@ class LatentCache:
         return self.r if self.bits == 8 else self.r // 2 + 2 * (self.r // 128)
 
 
-def qsvd_quantize_weight(W_d: torch.Tensor, clip: float = 1.0, stream=None) -> DownWeight:
-    """W_d fp32 [d, r] -> DownWeight (per-output-channel int8 RTN)."""
+def qsvd_quantize_weight(W_d: torch.Tensor, clip: float = 1.0, stream=None, rot: int = 0) -> DownWeight:
+    """W_d fp32 [d, r] -> DownWeight (per-output-channel int8 RTN); rot > 0:
+    of H1 W_d (qsvd_quantize_weight_rotated), and the projection then rotates X."""
     d, r = W_d.shape
     dev = W_d.device
     codes = torch.empty((r, d), dtype=torch.int8, device=dev)
     codes_bf16 = torch.empty((r, d), dtype=torch.bfloat16, device=dev)
     scale = torch.empty((r,), dtype=torch.float32, device=dev)
-    _check(_lib.qsvd_quantize_weight(_ptr(W_d, _F32, "W_d"), d, r, clip, _ptr(codes), _ptr(codes_bf16), _ptr(scale),
-                                     _stream(stream)))
-    return DownWeight(codes, codes_bf16, scale)
+    if rot:
+        _check(_lib.qsvd_quantize_weight_rotated(_ptr(W_d, _F32, "W_d"), d, r, clip, rot, _ptr(codes),
+                                                 _ptr(codes_bf16), _ptr(scale), _stream(stream)))
+    else:
+        _check(_lib.qsvd_quantize_weight(_ptr(W_d, _F32, "W_d"), d, r, clip, _ptr(codes), _ptr(codes_bf16),
+                                         _ptr(scale), _stream(stream)))
+    return DownWeight(codes, codes_bf16, scale, rot)
 
 
 def qsvd_project_workspace_bytes(T: int, d: int, r: int) -> int:

@@ -249,6 +249,21 @@ int qsvd_quantize_weight(const float *W_d, int32_t d, int32_t r, float clip, int
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "quantize_weight launch");
 }
 
+int qsvd_quantize_weight_rotated(const float *W_d, int32_t d, int32_t r, float clip, int32_t rot, int8_t *codes,
+                                 uint16_t *codes_bf16, float *scale, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!W_d || !codes || !scale) return fail(QSVD_EINVAL, "quantize_weight_rotated: null pointer");
+    if (d <= 0 || r <= 0) return fail(QSVD_EINVAL, "quantize_weight_rotated: d and r must be positive");
+    if (!(clip > 0.0f && clip <= 1.0f)) return fail(QSVD_EINVAL, "quantize_weight_rotated: clip must lie in (0, 1]");
+    if (rot < 2 || (rot & (rot - 1)) || d % rot) return fail(QSVD_EINVAL, "quantize_weight_rotated: rot must be a power of two >= 2 dividing d");
+    if (d > 6144) return fail(QSVD_EUNSUPPORTED, "quantize_weight_rotated: d > 6144");
+    prof_mark(stream, "begin");
+    cudaError_t e = launch_quantize_weight(W_d, d, r, clip, codes, codes_bf16, scale, stream, rot);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "quantize_weight_rotated launch");
+}
+
 size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r) {
     if (T < 0 || d <= 0 || r <= 0) return 0;
     return 256 +                                // completion counter (zero at rest)
@@ -271,6 +286,9 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
     const int d = W->d, r = W->r;
     if (d <= 0 || r <= 0 || d % 64 || r % 16) return fail(QSVD_EINVAL, "latent_project: need d %% 64 == 0 and r %% 16 == 0");
     if (r > 4096) return fail(QSVD_EUNSUPPORTED, "latent_project: r > 4096");
+    const int rot = W->rot;
+    if (rot && (rot < 2 || (rot & (rot - 1)) || d % rot))
+        return fail(QSVD_EINVAL, "latent_project: W->rot must be 0 or a power of two >= 2 dividing d");
     if (lat_bits != 8 && lat_bits != 4) return fail(QSVD_EINVAL, "latent_project: lat_bits must be 8 or 4");
     if (lat_bits == 4 && r % 128) return fail(QSVD_EUNSUPPORTED, "latent_project: int4 needs r %% 128 == 0");
     if (!(act_clip > 0.0f && act_clip <= 1.0f) || !(lat_clip > 0.0f && lat_clip <= 1.0f))
@@ -308,14 +326,14 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
     prof_mark(stream, "begin");
     cudaError_t e;
     if (T <= kPsMaxSplitTok && d <= 6144 && d % 256 == 0) {
-        if (T < kPsSplitTok) {
+        if (T < kPsSplitTok && !rot) {                  // the quantizer fused into the projection (no H1)
             e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
                                   xq_out, xs_out, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
                                   dst_pos, err, stream);
             return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "projection launch");
         }
         // each row quantized once, the dot products on the tensor cores, the rows requantized in parallel
-        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream);
+        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream, rot);
         if (e == cudaSuccess)
             e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
                                   nullptr, nullptr, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
@@ -327,7 +345,7 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
     }
     if (W->codes_bf16 && gemm_tc_supported(d, r)) {
         if (!aligned16(W->codes_bf16)) return fail(QSVD_EINVAL, "latent_project: codes_bf16 must be 16-byte aligned");
-        e = launch_xquant(X, T, d, act_clip, xq_out, xq_bf16, xs, stream);
+        e = launch_xquant(X, T, d, act_clip, xq_out, xq_bf16, xs, stream, rot);
         if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
         if (gemm_tc_fused_supported(T, r, lat_bits)) {
             // a2, a3 and a4 in one kernel: the latent never leaves the registers
@@ -339,7 +357,7 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
         e = launch_gemm_tc(xq_bf16, T, d, W->codes_bf16, W->scale, xs, r, c_hat, acc_out, err, stream);
         if (e != cudaSuccess) return cuda_fail(e, "tensor-core projection launch");
     } else {
-        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream);
+        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream, rot);
         if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
         e = launch_proj_dp4a(xq, T, d, W->codes, W->scale, xs, r, c_hat, acc_out, stream);
         if (e != cudaSuccess) return cuda_fail(e, "projection launch");
@@ -571,6 +589,7 @@ int qsvd_decode_step(const qsvd_down_weight *W, const uint16_t *X, const qsvd_ca
     if ((st = check_cache(cache))) return st;
     if (!W || !W->codes || !W->scale || !X || !seq_len || !U_q || !U_k || !U_v || !O)
         return fail(QSVD_EINVAL, "decode_step: null pointer");
+    if (W->rot) return fail(QSVD_EUNSUPPORTED, "decode_step: rotated weights (W->rot) need qsvd_latent_project");
     const int d = W->d, r = W->r;
     if (r != cache->r) return fail(QSVD_EINVAL, "decode_step: weight rank differs from the cache's");
     if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "decode_step: dh must be 64 or 128");

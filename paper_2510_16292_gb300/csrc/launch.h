@@ -96,13 +96,15 @@ __device__ __forceinline__ int row_len(const int32_t *seq_len, const int32_t *se
 // after each kernel launch, and each entry point once before its first one.
 void prof_mark(cudaStream_t s, const char *label);
 
-// Per-token int8 quantization of X [T, d] bf16 (a1).
+// Per-token int8 quantization of X [T, d] bf16 (a1); rot > 0: of X H1^T,
+// H1 the block Hadamard rotation with blocks of rot channels (quant_kernels.cu).
 cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip,
-                          int8_t *xq, uint16_t *xq_bf16, float *xs, cudaStream_t s);
+                          int8_t *xq, uint16_t *xq_bf16, float *xs, cudaStream_t s, int rot = 0);
 
-// Per-output-channel int8 RTN of W_d [d, r] fp32 -> codes [r, d] (+ bf16 image).
+// Per-output-channel int8 RTN of W_d [d, r] fp32 -> codes [r, d] (+ bf16 image);
+// rot > 0: of H1 W_d.
 cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int8_t *codes,
-                                   uint16_t *codes_bf16, float *scale, cudaStream_t s);
+                                   uint16_t *codes_bf16, float *scale, cudaStream_t s, int rot = 0);
 
 // Exact int8 GEMM on the CUDA cores (dp4a) with the dequant epilogue (a2, a3 first half):
 // c_hat[t, j] = (fp32(acc) * xs[t]) * ws[j].

@@ -60,6 +60,7 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
         g_scratch_ptr[dev] = p;
     }
     if (!W || !W->codes || !W->scale || !X) return sfail(QSVD_EINVAL, "latent_project_static: null pointer");
+    if (W->rot) return sfail(QSVD_EUNSUPPORTED, "latent_project_static: rotated weights (W->rot) need qsvd_latent_project");
     const void *ptrs[] = {X, W->codes, lat_codes, lat_scales};
     for (const void *p : ptrs)
         if (p && (reinterpret_cast<uintptr_t>(p) & 15u))

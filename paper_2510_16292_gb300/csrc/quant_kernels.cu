@@ -1,12 +1,22 @@
 // Quantization, requantization and cache-append kernels.
 //
-//   xquant_kernel       a1: per-token symmetric int8 RTN of X (Sec. 4 setup;
-//                       Q(X H1^T) of Eq. 12 with H1 = I).
+//   xquant_kernel       a1: per-token symmetric int8 RTN of X (Sec. 4 setup),
+//                       Q(X H1^T) of Eq. 12: H1 = I, or the block Hadamard
+//                       rotation applied to the row first (rot = block size).
 //   weight_quant_kernel offline per-output-channel int8 RTN of W_d.
+//   weight_quant_rot_kernel  the same for H1 W_d (the rotation down each
+//                       column first).
+// H1 = I_{d/b} (x) H_b / sqrt(b) (H_b Sylvester, b a power of two dividing d)
+// by the fast Walsh-Hadamard transform in fp32: stages h = 1, 2, ..., b/2 in
+// that order, pair (i, i+h) with (i & h) == 0 -> (v_i + v_{i+h}, v_i - v_{i+h}),
+// then every entry times fp32(1/sqrt(b)).  The stage order fixes every
+// rounding, so the result does not depend on how threads share the pairs.
 //   requant_kernel      a3/a4: Eq. 11's Q(C_qkv), per token (int8) or per
 //                       128-channel group (int4), written token-major and/or
 //                       straight into the latent cache.
 //   append_kernel       a4: latent rows -> cache slots.
+#include <cmath>
+
 #include "common.cuh"
 #include "launch.h"
 
@@ -18,8 +28,26 @@ namespace qsvd {
 // ---------------------------------------------------------------------------
 constexpr int kXqThreads = 256;
 
+// Fast Walsh-Hadamard transform of every length-b block of v[0 .. n) in
+// shared memory (all threads of the CTA; b a power of two dividing n), then
+// v *= scale.  Ends with the CTA synchronized.
+__device__ __forceinline__ void fwht_smem(float *v, int n, int b, float scale) {
+    __syncthreads();
+    for (int h = 1; h < b; h <<= 1) {
+        for (int p = threadIdx.x; p < n / 2; p += blockDim.x) {
+            const int i = (p / h) * 2 * h + (p % h);          // (i & h) == 0; i + h stays in i's block
+            const float a = v[i], c = v[i + h];
+            v[i] = __fadd_rn(a, c);
+            v[i + h] = __fsub_rn(a, c);
+        }
+        __syncthreads();
+    }
+    for (int i = threadIdx.x; i < n; i += blockDim.x) v[i] = __fmul_rn(v[i], scale);
+    __syncthreads();
+}
+
 __global__ void __launch_bounds__(kXqThreads)
-xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int8_t *__restrict__ xq,
+xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int rot, float rot_scale, int8_t *__restrict__ xq,
               uint16_t *__restrict__ xq_bf16, float *__restrict__ xs) {
     extern __shared__ float row[];
     __shared__ float red[kXqThreads / 32];
@@ -36,6 +64,11 @@ xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int8_t *__restr
             row[i + e] = f[e];
             m = fmaxf(m, fabsf(f[e]));
         }
+    }
+    if (rot) {                                           // x H1^T, then the absmax of the rotated row
+        fwht_smem(row, d, rot, rot_scale);
+        m = 0.0f;
+        for (int i = threadIdx.x; i < d; i += kXqThreads) m = fmaxf(m, fabsf(row[i]));
     }
     m = block_max<kXqThreads>(m, red);
     const float s = quant_scale(m, clip, 127.0f), inv = quant_inv_scale(s);
@@ -58,15 +91,16 @@ xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int8_t *__restr
 }
 
 cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip, int8_t *xq,
-                          uint16_t *xq_bf16, float *xs, cudaStream_t s) {
+                          uint16_t *xq_bf16, float *xs, cudaStream_t s, int rot) {
     if (T == 0) return cudaSuccess;
     const size_t smem = size_t(d) * sizeof(float);
     if (smem > 48 * 1024) {
         cudaError_t e = ensure_smem(xquant_kernel, smem);
         if (e != cudaSuccess) return e;
     }
-    cudaError_t e = launch_pdl(xquant_kernel, dim3(unsigned(T)), dim3(kXqThreads), smem, s, X, d, clip, xq,
-                               xq_bf16, xs);
+    const float rot_scale = rot ? float(1.0 / std::sqrt(double(rot))) : 1.0f;
+    cudaError_t e = launch_pdl(xquant_kernel, dim3(unsigned(T)), dim3(kXqThreads), smem, s, X, d, clip, rot,
+                               rot_scale, xq, xq_bf16, xs);
     prof_mark(s, "xquant");
     return e;
 }
@@ -106,9 +140,62 @@ weight_quant_kernel(const float *__restrict__ W, int d, int r, float clip, int8_
     pdl_trigger();
 }
 
+// Offline, rotated: kWqrCols columns of W_d per CTA, staged column-major in
+// shared memory, transformed by H1 down each column, then quantized per
+// column like weight_quant_kernel.
+constexpr int kWqrCols = 4;
+
+__global__ void __launch_bounds__(256)
+weight_quant_rot_kernel(const float *__restrict__ W, int d, int r, float clip, int rot, float rot_scale,
+                        int8_t *__restrict__ codes, uint16_t *__restrict__ codes_bf16, float *__restrict__ scale) {
+    extern __shared__ float col[];                        // [kWqrCols][d]
+    __shared__ float red[kWqrCols][8];
+    __shared__ float sc[kWqrCols];
+    const int j0 = blockIdx.x * kWqrCols;
+    const int nc = min(kWqrCols, r - j0);
+    for (int i = threadIdx.x; i < kWqrCols * d; i += blockDim.x) {
+        const int c = i % kWqrCols, k = i / kWqrCols;
+        col[c * d + k] = c < nc ? W[size_t(k) * r + j0 + c] : 0.0f;
+    }
+    fwht_smem(col, kWqrCols * d, rot, rot_scale);         // blocks of rot never cross a column (rot divides d)
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int c = 0; c < kWqrCols; ++c) {
+        float m = 0.0f;
+        for (int k = threadIdx.x; k < d; k += blockDim.x) m = fmaxf(m, fabsf(col[c * d + k]));
+        m = warp_max(m);
+        if (lane == 0) red[c][warp] = m;
+    }
+    __syncthreads();
+    if (threadIdx.x < kWqrCols) {
+        float m = 0.0f;
+        for (int w = 0; w < 8; ++w) m = fmaxf(m, red[threadIdx.x][w]);
+        sc[threadIdx.x] = quant_scale(m, clip, 127.0f);
+    }
+    __syncthreads();
+    for (int c = 0; c < nc; ++c) {
+        const float s = sc[c];
+        if (threadIdx.x == 0) scale[j0 + c] = s;
+        for (int k = threadIdx.x; k < d; k += blockDim.x) {
+            const int q = quant_code(col[c * d + k], s, 127);
+            codes[size_t(j0 + c) * d + k] = int8_t(q);
+            if (codes_bf16) codes_bf16[size_t(j0 + c) * d + k] = int_to_bf16_bits(q);
+        }
+    }
+    __threadfence();                                      // see weight_quant_kernel
+    pdl_trigger();
+}
+
 cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int8_t *codes,
-                                   uint16_t *codes_bf16, float *scale, cudaStream_t s) {
-    weight_quant_kernel<<<dim3((r + 31) / 32), 256, 0, s>>>(W, d, r, clip, codes, codes_bf16, scale);
+                                   uint16_t *codes_bf16, float *scale, cudaStream_t s, int rot) {
+    if (rot) {
+        const size_t smem = size_t(kWqrCols) * d * sizeof(float);
+        cudaError_t e = ensure_smem(weight_quant_rot_kernel, smem);
+        if (e != cudaSuccess) return e;
+        weight_quant_rot_kernel<<<dim3((r + kWqrCols - 1) / kWqrCols), 256, smem, s>>>(
+            W, d, r, clip, rot, float(1.0 / std::sqrt(double(rot))), codes, codes_bf16, scale);
+    } else {
+        weight_quant_kernel<<<dim3((r + 31) / 32), 256, 0, s>>>(W, d, r, clip, codes, codes_bf16, scale);
+    }
     prof_mark(s, "weight_quant");
     return cudaGetLastError();
 }

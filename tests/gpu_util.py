@@ -60,7 +60,7 @@ class GpuLayer:
         self.lib, self.s, self.B, self.bits = lib, shape, B, bits
         self.act_clip, self.lat_clip = act_clip, lat_clip
         self.W = lib.qsvd_quantize_weight(
-            torch.from_numpy(np.asarray(weights["W_d"], dtype=np.float32)).to(dev()))
+            torch.from_numpy(np.asarray(weights["W_d"], dtype=np.float32)).to(dev()), rot=weights.get("rot", 0))
         self.U_q, self.U_k, self.U_v = (bf16(weights[k]) for k in ("U_q", "U_k", "U_v"))
         self.cache = lib.LatentCache.empty(B, tmax, shape.r, bits, dev())
         self.len = np.zeros(B, dtype=np.int64)
