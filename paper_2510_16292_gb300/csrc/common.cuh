@@ -146,6 +146,58 @@ __device__ __forceinline__ __half int4_group_scale(float absmax, float clip) {
 // ---------------------------------------------------------------------------
 // Reductions
 // ---------------------------------------------------------------------------
+// Block Hadamard transform of a row (the rotation H1; the stage order is the
+// one fwht_smem in quant_kernels.cu follows, so results are identical).
+// fwht8_regs: stages h = 1, 2, 4 on 8 consecutive, 8-aligned values.
+__device__ __forceinline__ void fwht8_regs(float (&f)[8]) {
+#pragma unroll
+    for (int hh = 1; hh < 8; hh <<= 1)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            if (e & hh) continue;
+            const float a = f[e], c = f[e + hh];
+            f[e] = __fadd_rn(a, c);
+            f[e + hh] = __fsub_rn(a, c);
+        }
+}
+// fwht_smem_rounds: the remaining stages, in rounds of up to four.  In a
+// round starting at stride h0, a thread takes groups of 2^k elements spaced
+// h0 apart (the group's base has zeros in the bits the round's strides
+// cover), so the round's stages pair elements within a group only and run in
+// registers; one barrier per round.  Every butterfly combines the same two
+// values in the same stage order as fwht_smem, so the results are identical.
+// `first` stages (h < first) have already been applied by the caller.
+__device__ __forceinline__ void fwht_smem_rounds(float *v, int n, int b, int first) {
+    for (int h0 = first; h0 < b; h0 <<= 4) {
+        int ks = 0;
+        while (ks < 4 && (h0 << ks) < b) ++ks;            // stages h0, 2 h0, ..., 2^(ks-1) h0
+        const int gsz = 1 << ks, ngroups = n >> ks;
+        for (int g = threadIdx.x; g < ngroups; g += blockDim.x) {
+            const int base = (g / h0) * (gsz * h0) + (g % h0);
+            float x[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+                if (e < gsz) x[e] = v[base + e * h0];
+#pragma unroll
+            for (int st = 0; st < 4; ++st) {
+                if (st >= ks) break;
+                const int hh = 1 << st;
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    if (e >= gsz || (e & hh)) continue;
+                    const float a = x[e], c = x[e + hh];
+                    x[e] = __fadd_rn(a, c);
+                    x[e + hh] = __fsub_rn(a, c);
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+                if (e < gsz) v[base + e * h0] = x[e];
+        }
+        __syncthreads();
+    }
+}
+
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));

@@ -46,44 +46,6 @@ __device__ __forceinline__ void fwht_smem(float *v, int n, int b, float scale) {
     __syncthreads();
 }
 
-// The same transform, faster: stages run in rounds of up to four.  In a
-// round starting at stride h0, a thread takes groups of 2^k elements spaced
-// h0 apart (the group's base has zeros in the bits the round's strides
-// cover), so the round's stages pair elements within a group only and run in
-// registers; one barrier per round.  Every butterfly combines the same two
-// values in the same stage order as fwht_smem, so the results are identical.
-// `first` stages (h < first) have already been applied by the caller.
-__device__ __forceinline__ void fwht_smem_rounds(float *v, int n, int b, int first) {
-    for (int h0 = first; h0 < b; h0 <<= 4) {
-        int ks = 0;
-        while (ks < 4 && (h0 << ks) < b) ++ks;            // stages h0, 2 h0, ..., 2^(ks-1) h0
-        const int gsz = 1 << ks, ngroups = n >> ks;
-        for (int g = threadIdx.x; g < ngroups; g += blockDim.x) {
-            const int base = (g / h0) * (gsz * h0) + (g % h0);
-            float x[16];
-#pragma unroll
-            for (int e = 0; e < 16; ++e)
-                if (e < gsz) x[e] = v[base + e * h0];
-#pragma unroll
-            for (int st = 0; st < 4; ++st) {
-                if (st >= ks) break;
-                const int hh = 1 << st;
-#pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    if (e >= gsz || (e & hh)) continue;
-                    const float a = x[e], c = x[e + hh];
-                    x[e] = __fadd_rn(a, c);
-                    x[e + hh] = __fsub_rn(a, c);
-                }
-            }
-#pragma unroll
-            for (int e = 0; e < 16; ++e)
-                if (e < gsz) v[base + e * h0] = x[e];
-        }
-        __syncthreads();
-    }
-}
-
 __global__ void __launch_bounds__(kXqThreads)
 xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int rot, float rot_scale, int8_t *__restrict__ xq,
               uint16_t *__restrict__ xq_bf16, float *__restrict__ xs) {
@@ -100,17 +62,7 @@ xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int rot, float 
     for (int i = threadIdx.x * 8; i < d; i += kXqThreads * 8) {
         float f[8];
         unpack8_bf16(*reinterpret_cast<const uint4 *>(x + i), f);
-        if (pre) {
-#pragma unroll
-            for (int hh = 1; hh < 8; hh <<= 1)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    if (e & hh) continue;
-                    const float a = f[e], c = f[e + hh];
-                    f[e] = __fadd_rn(a, c);
-                    f[e + hh] = __fsub_rn(a, c);
-                }
-        }
+        if (pre) fwht8_regs(f);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             row[i + e] = f[e];
