@@ -253,8 +253,9 @@ size_t qsvd_prefill_workspace_bytes(int64_t n, int32_t max_len, int32_t r, int32
  *       bytes: fp16 copies of the blocks' latent rows and of Q, K, V.
  * Requirements: dh == 128, H*dh % 256 == 0, r % 64 == 0, softmax_scale > 0
  * and finite; a block outside the cache (seq outside [0, B), t0 < 0, T < 1,
- * t0 + T > Tmax) returns QSVD_EINVAL before anything is enqueued.  fp16 Q, K, V hold magnitudes up
- * to 65504.
+ * t0 + T > Tmax) returns QSVD_EINVAL before anything is enqueued; a launch of
+ * 64 blocks whose padded rows R give R * r / 8 >= 2^31 returns
+ * QSVD_EUNSUPPORTED.  fp16 Q, K, V hold magnitudes up to 65504.
  */
 typedef struct {
     int32_t seq, t0, T;

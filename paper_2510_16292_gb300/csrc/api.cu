@@ -564,6 +564,14 @@ int qsvd_latent_prefill(const qsvd_cache *cache, const qsvd_prefill_block *block
             return fail(QSVD_EINVAL, "latent_prefill: block %d (seq %d, t0 %d, T %d) outside the cache", int(k),
                         int(b.seq), int(b.t0), int(b.T));
     }
+    for (int32_t i0 = 0; i0 < n_blocks; i0 += kPrefillMaxBlocks) {
+        // the kernels index a launch's padded rows (and R * r / 8 prep threads) with 32-bit integers
+        int64_t R = 0;
+        for (int32_t k = i0; k < std::min<int32_t>(n_blocks, i0 + kPrefillMaxBlocks); ++k)
+            R += (int64_t(blocks[k].t0) + blocks[k].T + 127) / 128 * 128;
+        if (R * (cache->r / 8) >= (int64_t(1) << 31))
+            return fail(QSVD_EUNSUPPORTED, "latent_prefill: blocks %d.. hold too many rows for one launch", int(i0));
+    }
     const size_t need = qsvd_latent_prefill_workspace_bytes(blocks, n_blocks, cache->r, H, dh);
     if (!workspace || workspace_bytes < need)
         return fail(QSVD_ENOSPC, "latent_prefill: workspace needs %zu bytes", need);
