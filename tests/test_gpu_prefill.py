@@ -288,3 +288,32 @@ def test_latent_prefill_argument_errors():
         assert e.value.status == lib.QSVD_EINVAL
     lib.qsvd_latent_prefill(gpu.cache, [], Ut, s.H, s.dh, O)
     lib.qsvd_check()
+
+
+def test_prefill_rows_tiny_dh64():
+    """The tiny layer (d = 256, H = 4, dh = 64, r = 96, weights from the joint
+    SVD): the row path, which also serves dh = 64."""
+    wl = synthetic.WORKLOADS["tiny"]
+    inp = synthetic.gen_layer(wl, seed=48)
+    w = pipeline.prepare_weights(inp)
+    ref = pipeline.OracleLayer(wl.shape, w, 1, wl.tmax, 8, track=[])
+    gpu = GpuLayer(wl.shape, w, 1, wl.tmax, 8)
+    ref.prefill(0, inp.X_prefill[0])
+    gpu.prefill(0, inp.X_prefill[0])
+    n = wl.prefill
+    O = _gpu_prefill(gpu, np.zeros(n), np.arange(1, n + 1))
+    q().qsvd_check()
+    assert_rows_close(O.cpu().numpy(), _oracle_rows(ref, 0, 0, n), "tiny rows")
+
+
+def test_latent_prefill_13b_int4_continued():
+    """Block path, int4 cache, H = 40: a prompt continued at t0 = 77 (not a
+    multiple of 128) and a second sequence's whole prompt."""
+    wl, inp, ref, gpu = _layers("llava13b", 2, 260, 4, seed=58)
+    for side in (ref, gpu):
+        side.prefill(0, inp.X_prefill[0][:260])
+        side.prefill(1, inp.X_prefill[1][:150])
+    blocks = [(0, 77, 183), (1, 0, 150)]
+    O = _gpu_blocks(gpu, blocks)
+    want = np.concatenate([_oracle_rows(ref, b, t0, t0 + T) for b, t0, T in blocks])
+    assert_rows_close(O, want, "13B int4 blocks")
