@@ -26,11 +26,15 @@ from . import attention, latent, quant, rotate, svd
 TINY_BETA = 0.5
 
 
-def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1.0, rot: int = 0):
+def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1.0, rot: int = 0,
+                    u_bits: int = 0):
     """Returns dict(W_d fp32 values [d, r], Wq int64 [d, r], s_w [r],
     U_q/U_k/U_v bf16 bits [r, d], rot).  rot = b > 0: Wq, s_w quantize
     H1 W_d (oracle.rotate, block b) instead of W_d (W_d itself is returned
-    unrotated: it is what the caller hands to the GPU's rotating quantizer)."""
+    unrotated: it is what the caller hands to the GPU's rotating quantizer).
+    u_bits = 8 or 4: Eq. 11's Q(H2 W^u) as well (H2 = I): every column of
+    U_q, U_k, U_v quantized per output channel (U*_codes, U*_scale), and the
+    attention uses the dequantized values (U*_deq)."""
     s = inp.workload.shape
     if inp.W_qkv is not None:
         d = s.d
@@ -42,7 +46,20 @@ def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1
         W_d, U_q, U_k, U_v = inp.W_d, inp.U_q, inp.U_k, inp.U_v
     Wq, s_w = quant.quantize_columns(rotate.rotate_weight(W_d, rot) if rot else W_d, 8, w_clip)
     c = np.ascontiguousarray
-    return dict(W_d=c(W_d), Wq=c(Wq), s_w=c(s_w), U_q=c(U_q), U_k=c(U_k), U_v=c(U_v), rot=rot)
+    out = dict(W_d=c(W_d), Wq=c(Wq), s_w=c(s_w), U_q=c(U_q), U_k=c(U_k), U_v=c(U_v), rot=rot, u_bits=u_bits)
+    if u_bits:
+        for k in ("U_q", "U_k", "U_v"):
+            codes, scale = quantize_up(bf16_from_bits(out[k]), u_bits)
+            out[k + "_codes"], out[k + "_scale"] = codes, scale
+            out[k + "_deq"] = codes.astype(np.float64) * scale[None, :]
+    return out
+
+
+def quantize_up(U, bits: int = 8):
+    """Eq. 11's Q(W^u) for one up-projection U [r, d] (bf16 values): symmetric
+    RTN per output channel (column), the weight quantizer of the Sec. 4 setup.
+    Returns (codes int64 [r, d], scale fp64 [d] holding fp32 values)."""
+    return quant.quantize_columns(np.asarray(U, dtype=np.float64), bits)
 
 
 class OracleLayer:
@@ -53,9 +70,12 @@ class OracleLayer:
                  track: Optional[Iterable[int]] = None):
         self.s = shape
         self.w = weights
-        self.U_q = bf16_from_bits(weights["U_q"])
-        self.U_k = bf16_from_bits(weights["U_k"])
-        self.U_v = bf16_from_bits(weights["U_v"])
+        if weights.get("u_bits"):
+            self.U_q, self.U_k, self.U_v = (weights[k + "_deq"] for k in ("U_q", "U_k", "U_v"))
+        else:
+            self.U_q = bf16_from_bits(weights["U_q"])
+            self.U_k = bf16_from_bits(weights["U_k"])
+            self.U_v = bf16_from_bits(weights["U_v"])
         self.B, self.tmax, self.bits = B, tmax, lat_bits
         self.act_clip, self.lat_clip = act_clip, lat_clip
         self.cache = latent.LatentCache(B, tmax, shape.r, lat_bits)
