@@ -58,6 +58,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-prefill13", action="store_true")
     p.add_argument("--no-prefill-attn", action="store_true")
+    p.add_argument("--importance-probe", action="store_true",
+                   help="only time the Eq. 10 importance scores of one 7B-shaped layer and print one line")
     p.add_argument("--rot", action="store_true",
                    help="rotate X by H1 on the fly (Eq. 12; weights quantized as H1 W_d) in every projection")
     p.add_argument("--prefill-probe", action="store_true",
@@ -600,6 +602,41 @@ def prefill_attn_probe(name, iters=3, group_rows=0, path="blocks"):
     return out
 
 
+def importance_probe(iters=3, N=1, m=4096, n=12288, k=4096):
+    """Offline Eq. 10 scores of every singular value of a 7B-shaped W_concat
+    (E x 3E, E = 4096) for N calibration gradients: 2 N m n k flops on the
+    fp32 CUDA cores.  Inputs: seeded torch Gaussians (the time does not
+    depend on the values).  Peak: 152 SMs x 128 fp32 lanes x 2 flops x the
+    SM clock (2070 MHz), the CUDA-core fp32 rate."""
+    import torch
+    import paper_2510_16292_gb300 as q
+    dev = torch.device("cuda", torch.cuda.current_device())
+    g = torch.Generator(device=dev)
+    g.manual_seed(99)
+    U = torch.randn((m, k), generator=g, device=dev)
+    s = torch.rand((k,), generator=g, device=dev)
+    Vt = torch.randn((k, n), generator=g, device=dev)
+    G = torch.randn((N, m, n), generator=g, device=dev)
+    ws = torch.empty(int(q._lib.qsvd_importance_workspace_bytes(N, k)), dtype=torch.uint8, device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    times = []
+    for it in range(iters + 1):
+        e0.record()
+        q.qsvd_importance_scores(U, s, Vt, G, workspace=ws)
+        e1.record()
+        torch.cuda.synchronize()
+        if it:
+            times.append(e0.elapsed_time(e1) * 1e-3)
+    q.qsvd_check()
+    t = min(times)
+    flops = 2.0 * N * m * n * k
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    peak = sms * 128 * 2 * 2.07e9 / 1e12
+    return {"importance_scores": f"N={N} m={m} n={n} k={k}", "ms": round(t * 1e3, 3),
+            "tflops": round(flops / t / 1e12, 2), "bound": "alu", "peak_tflops": round(peak, 1),
+            "frac": round(flops / t / 1e12 / peak, 4), "peak_kind": "derived: SMs x 128 fp32 lanes x 2 x 2070 MHz"}
+
+
 def cross_rank(values, op="max"):
     """Per-rank totals reduced over the ranks of the default process group
     (max: the job takes as long as its slowest rank; min: the slowest rank's
@@ -927,6 +964,9 @@ def main():
     args = parse()
     if args.sweep:
         run_sweep(args)
+        return
+    if args.importance_probe:
+        print(json.dumps(importance_probe(iters=args.steps)), flush=True)
         return
     if args.prefill_probe:
         for name in args.prefill_shapes.split(","):

@@ -12,6 +12,7 @@
  * This library implements, on the caller's CUDA stream:
  *   qsvd_quantize_weight     offline per-channel int8 RTN of W_d (Sec. 4 setup)
  *   qsvd_quantize_weight_rotated  the same of H1 W_d (Eq. 12's online rotation)
+ *   qsvd_importance_scores   offline Eq. 10 scores of singular values (Sec. 3.2)
  *   qsvd_latent_project      C = Q(X) Q(W_d), requantized per token (Eq. 11-12)
  *   qsvd_cache_append        store latent rows in the latent cache (Fig. 2(f))
  *   qsvd_latent_decode_attn  one decode step of attention over that cache (Eq. 5)
@@ -150,6 +151,23 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
                         void *workspace, size_t workspace_bytes, cudaStream_t stream);
 
 size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r);
+
+/*
+ * Offline preparation, Sec. 3.2: importance scores of a layer's singular
+ * values (Eq. 10), score_i = (1/N) sum_n (sigma_i [U^T G_n V]_{ii})^2, for
+ * the cross-layer rank budget (keep the k highest scores of all layers).
+ *   U fp32 [m, k] (left singular vectors as columns), sigma fp32 [k],
+ *   Vt fp32 [k, n] (right singular vectors as rows), G fp32 [N, m, n] (the
+ *   loss gradient for each of N calibration samples), scores fp32 [k] out.
+ *   workspace: qsvd_importance_workspace_bytes(N, k) bytes.
+ * fp32 on the CUDA cores; the per-sample sums are accumulated with atomics,
+ * so the last bits vary between runs.  N <= 65535 per call.
+ */
+int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, const float *G, int32_t N, int32_t m,
+                           int32_t n, int32_t k, float *scores, void *workspace, size_t workspace_bytes,
+                           cudaStream_t stream);
+
+size_t qsvd_importance_workspace_bytes(int32_t N, int32_t k);
 
 /*
  * The rotation H1 of Eq. 11-12 applied on the fly (for models where it is not

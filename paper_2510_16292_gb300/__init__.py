@@ -30,7 +30,8 @@ _lib = ctypes.CDLL(_LIB_PATH)
 
 QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
-EXPORTS = ("qsvd_quantize_weight", "qsvd_quantize_weight_rotated", "qsvd_latent_project", "qsvd_project_workspace_bytes",
+EXPORTS = ("qsvd_quantize_weight", "qsvd_quantize_weight_rotated", "qsvd_importance_scores",
+           "qsvd_importance_workspace_bytes", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
            "qsvd_latent_prefill_attn", "qsvd_prefill_workspace_bytes", "qsvd_prefill_weights",
            "qsvd_latent_prefill", "qsvd_latent_prefill_workspace_bytes",
@@ -62,6 +63,9 @@ class _PrefillBlock(ctypes.Structure):
 _vp, _i32, _i64, _f32, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
 _lib.qsvd_quantize_weight.argtypes = [_vp, _i32, _i32, _f32, _vp, _vp, _vp, _vp]
 _lib.qsvd_quantize_weight_rotated.argtypes = [_vp, _i32, _i32, _f32, _i32, _vp, _vp, _vp, _vp]
+_lib.qsvd_importance_scores.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
+_lib.qsvd_importance_workspace_bytes.argtypes = [_i32, _i32]
+_lib.qsvd_importance_workspace_bytes.restype = _sz
 _lib.qsvd_latent_project.argtypes = [ctypes.POINTER(_DownWeight), _vp, _i64, _f32, _i32, _f32, _vp, _vp,
                                      ctypes.POINTER(_Cache), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
 _lib.qsvd_project_workspace_bytes.argtypes = [_i64, _i32, _i32]
@@ -192,6 +196,22 @@ def qsvd_quantize_weight(W_d: torch.Tensor, clip: float = 1.0, stream=None, rot:
         _check(_lib.qsvd_quantize_weight(_ptr(W_d, _F32, "W_d"), d, r, clip, _ptr(codes), _ptr(codes_bf16),
                                          _ptr(scale), _stream(stream)))
     return DownWeight(codes, codes_bf16, scale, rot)
+
+
+def qsvd_importance_scores(U: torch.Tensor, sigma: torch.Tensor, Vt: torch.Tensor, G: torch.Tensor,
+                           workspace=None, stream=None) -> torch.Tensor:
+    """Eq. 10 scores of the singular values: U [m, k], sigma [k], Vt [k, n],
+    G [N, m, n] (one gradient per calibration sample), all fp32 on the device."""
+    m, k = U.shape
+    N, _, n = G.shape
+    scores = torch.empty((k,), dtype=torch.float32, device=U.device)
+    if workspace is None:
+        workspace = torch.empty(max(1, int(_lib.qsvd_importance_workspace_bytes(N, k))), dtype=torch.uint8,
+                                device=U.device)
+    _check(_lib.qsvd_importance_scores(_ptr(U, _F32, "U"), _ptr(sigma, _F32, "sigma"), _ptr(Vt, _F32, "Vt"),
+                                       _ptr(G, _F32, "G"), N, m, n, k, _ptr(scores), _ptr(workspace),
+                                       workspace.numel(), _stream(stream)))
+    return scores
 
 
 def qsvd_project_workspace_bytes(T: int, d: int, r: int) -> int:

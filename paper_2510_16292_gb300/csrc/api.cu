@@ -583,6 +583,28 @@ int qsvd_latent_prefill(const qsvd_cache *cache, const qsvd_prefill_block *block
     });
 }
 
+size_t qsvd_importance_workspace_bytes(int32_t N, int32_t k) {
+    if (N <= 0 || k <= 0) return 0;
+    return align256(size_t(N) * k * sizeof(float));
+}
+
+int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, const float *G, int32_t N, int32_t m,
+                           int32_t n, int32_t k, float *scores, void *workspace, size_t workspace_bytes,
+                           cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!U || !sigma || !Vt || !G || !scores) return fail(QSVD_EINVAL, "importance_scores: null pointer");
+    if (N <= 0 || m <= 0 || n <= 0 || k <= 0) return fail(QSVD_EINVAL, "importance_scores: N, m, n, k must be positive");
+    if (N > 65535) return fail(QSVD_EUNSUPPORTED, "importance_scores: more than 65535 samples per call");
+    const size_t need = qsvd_importance_workspace_bytes(N, k);
+    if (!workspace || workspace_bytes < need)
+        return fail(QSVD_ENOSPC, "importance_scores: workspace needs %zu bytes", need);
+    prof_mark(stream, "begin");
+    const cudaError_t e = launch_importance(U, sigma, Vt, G, N, m, n, k, scores, static_cast<float *>(workspace), stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "importance_scores launch");
+}
+
 size_t qsvd_decode_step_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t d, int32_t r, int32_t H,
                                         int32_t dh) {
     if (B <= 0 || max_seq_len <= 0 || d <= 0 || r <= 0 || H <= 0 || dh <= 0) return 0;

@@ -170,6 +170,10 @@ struct DecodeArgs {
 };
 size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
 
+// Eq. 10 importance scores (prep_importance.cu); t: [N, k] fp32 scratch.
+cudaError_t launch_importance(const float *U, const float *sigma, const float *Vt, const float *G, int N, int m, int n,
+                              int k, float *scores, float *t, cudaStream_t s);
+
 // Causal prefill over the cache (qsvd_latent_prefill_attn) runs the decode
 // chain on groups of query rows: at most kPrefillMaxRows rows per group, fewer
 // while a group's workspace would exceed kPrefillWsTarget bytes.
