@@ -301,6 +301,8 @@ size_t qsvd_latent_prefill_workspace_bytes(const qsvd_prefill_block *blocks, int
  * bound by launch latency rather than by its bytes.
  * The launch is cooperative (one CTA per SM, grid-wide barriers whose waits
  * are bounded: an expired wait abandons the step and flags QSVD_ETIMEOUT).
+ * Every call first clears the grid barrier's counters in the workspace (one
+ * small memset on the stream), so a call after an expired wait starts clean.
  * Requirements: B <= 8; d = H*dh, d % 256 == 0, d <= 6144; r <= 3072;
  * dh in {64, 128}.  workspace: qsvd_decode_step_workspace_bytes(...) bytes.
  */

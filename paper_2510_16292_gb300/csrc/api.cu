@@ -96,6 +96,10 @@ int *error_word_for_current_device() {
     return device_setup(&err) == QSVD_OK ? err : nullptr;
 }
 
+int setup_current_device(int **err) { return device_setup(err); }
+
+int validate_cache(const qsvd_cache *c) { return check_cache(c); }
+
 int set_last_error(int code, const char *msg) { return fail(code, "%s", msg); }
 
 cudaError_t ensure_smem_ptr(const void *kernel, size_t bytes) {

@@ -611,6 +611,10 @@ cudaError_t launch_decode_fused(const FusedArgs &f, void *ws, size_t ws_bytes, i
     const size_t smem = fuse_smem_bytes(a.B, a.d, a.c.r, a.c.bits, a.dh);
     cudaError_t e = ensure_smem(decode_step_kernel, smem);
     if (e != cudaSuccess) return e;
+    // the grid barrier's arrival count and generation start at zero on every
+    // call: a call whose barrier wait expired leaves some CTAs counted
+    e = cudaMemsetAsync(a.w_.bar, 0, 2 * sizeof(unsigned), s);
+    if (e != cudaSuccess) return e;
     int dev = 0, sms = 0, per_sm = 0;
     e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);

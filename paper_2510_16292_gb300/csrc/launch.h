@@ -9,6 +9,8 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+struct qsvd_cache;   // include/qsvd.h
+
 namespace qsvd {
 
 // 2D tiled TMA descriptor over a row-major matrix of `outer` rows x `inner`
@@ -53,6 +55,14 @@ enum : int { kErrRange = 1, kErrTimeout = 2 };
 // device is unusable), and the thread's last-error message setter.
 int *error_word_for_current_device();
 int set_last_error(int code, const char *msg);
+
+// Entry-point prologue shared by every C ABI call (api.cu): checks once per
+// device that it is an sm_103 part and gives its error word; returns a QSVD_*
+// status (the message is set on failure).
+int setup_current_device(int **err);
+// Checks a caller's cache description (pointers non-null and 16-byte aligned,
+// bits 8 or 4, positive sizes, r % 16 == 0, int4 with r % 128 == 0).
+int validate_cache(const ::qsvd_cache *c);
 
 // Plain description of a latent cache (mirrors qsvd_cache), seen as B rows
 // of queries.  Without a sequence map, row b is sequence b of the cache

@@ -12,6 +12,7 @@
 // process exits.  Nothing here calls cudaMalloc, cudaFree or any allocating
 // routine.
 #include <cstdio>
+#include <mutex>
 
 #include "launch.h"
 #include "qsvd.h"
@@ -30,8 +31,26 @@ namespace {
 
 constexpr int kMaxDev = 64;
 void *g_scratch_ptr[kMaxDev];      // device address of g_project_scratch per device (set up once)
+std::mutex g_scratch_mu;
 
 int sfail(int code, const char *msg) { return set_last_error(code, msg); }
+
+// Set-up, once per device with that device current: the host-side name of
+// the array is not a device address, so ask the runtime for the real one.
+int scratch_for_current_device(void **out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev)
+        return sfail(QSVD_ECUDA, "latent_project_static: no usable current device");
+    std::lock_guard<std::mutex> lock(g_scratch_mu);
+    if (!g_scratch_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_project_scratch) != cudaSuccess || !p)
+            return sfail(QSVD_ECUDA, "latent_project_static: cudaGetSymbolAddress of the scratch array failed");
+        g_scratch_ptr[dev] = p;
+    }
+    *out = g_scratch_ptr[dev];
+    return QSVD_OK;
+}
 
 }  // namespace
 }  // namespace qsvd
@@ -44,21 +63,11 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
                                int32_t lat_bits, float lat_clip, void *lat_codes, void *lat_scales,
                                const qsvd_cache *dst, const int32_t *dst_seq, const int32_t *dst_pos,
                                cudaStream_t stream) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev)
-        return sfail(QSVD_ECUDA, "latent_project_static: no usable current device");
-    int major = 0, minor = 0;
-    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
-    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-    if (major != 10 || minor != 3) return sfail(QSVD_EUNSUPPORTED, "latent_project_static: needs an sm_103 device");
-    // Set-up, once per device with that device current: the host-side name of
-    // the array is not a device address; ask the runtime for the real one.
-    if (!g_scratch_ptr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_project_scratch) != cudaSuccess || !p)
-            return sfail(QSVD_ECUDA, "latent_project_static: cudaGetSymbolAddress of the scratch array failed");
-        g_scratch_ptr[dev] = p;
-    }
+    int *err = nullptr;
+    int st = setup_current_device(&err);     // sm_103 check and error word, cached per device
+    if (st) return st;
+    void *scratch = nullptr;
+    if ((st = scratch_for_current_device(&scratch))) return st;
     if (!W || !W->codes || !W->scale || !X) return sfail(QSVD_EINVAL, "latent_project_static: null pointer");
     if (W->rot) return sfail(QSVD_EUNSUPPORTED, "latent_project_static: rotated weights (W->rot) need qsvd_latent_project");
     const void *ptrs[] = {X, W->codes, lat_codes, lat_scales};
@@ -82,13 +91,14 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
     if (!tok && !dst) return sfail(QSVD_EINVAL, "latent_project_static: no destination for the latent");
     CacheView dv{};
     if (dst) {
-        if (!dst->codes || !dst->scales || dst->bits != lat_bits || dst->r != r || dst->B <= 0 || dst->Tmax <= 0)
+        if ((st = validate_cache(dst))) return st;      // null, alignment (the rows are stored as words), sizes
+        if (dst->bits != lat_bits || dst->r != r)
             return sfail(QSVD_EINVAL, "latent_project_static: cache does not match the projection");
         if (T > 0 && (!dst_seq || !dst_pos)) return sfail(QSVD_EINVAL, "latent_project_static: dst_seq/dst_pos required");
         dv = CacheView{dst->codes, dst->scales, dst->bits, dst->B, dst->Tmax, dst->r};
     }
     if (T == 0) return QSVD_OK;
-    char *base = static_cast<char *>(g_scratch_ptr[dev]);
+    char *base = static_cast<char *>(scratch);
     int *counter = reinterpret_cast<int *>(base);
     float *c_hat = reinterpret_cast<float *>(base + kStaticCounterBytes);
     // The array keeps the previous call's contents; only the completion
@@ -97,7 +107,7 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
     if (e == cudaSuccess)
         e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
                               nullptr, nullptr, nullptr, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq, dst_pos,
-                              error_word_for_current_device(), stream);
+                              err, stream);
     if (e != cudaSuccess) {
         char msg[160];
         snprintf(msg, sizeof(msg), "latent_project_static: %s", cudaGetErrorString(e));
