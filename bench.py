@@ -60,6 +60,9 @@ def parse():
     p.add_argument("--no-prefill-attn", action="store_true")
     p.add_argument("--importance-probe", action="store_true",
                    help="only time the Eq. 10 importance scores of one 7B-shaped layer and print one line")
+    p.add_argument("--u-bits", type=int, default=0, choices=[0, 8, 4],
+                   help="quantize U_q, U_k, U_v per output channel to int8 or int4 (Eq. 11) and run decode "
+                        "attention on the codes (qsvd_latent_decode_attn_qu); 0: bf16 up-projections")
     p.add_argument("--rot", action="store_true",
                    help="rotate X by H1 on the fly (Eq. 12; weights quantized as H1 W_d) in every projection")
     p.add_argument("--prefill-probe", action="store_true",
@@ -162,6 +165,8 @@ class NativeLayer:
         rot = (s.d & -s.d) if nb.rot else 0             # H1 on the fly: the largest power-of-two block
         self.W = q.qsvd_quantize_weight(torch.from_numpy(inp.W_d.astype(np.float32)).to(dev), rot=rot)
         self.U = [bf16(u) for u in (inp.U_q, inp.U_k, inp.U_v)]
+        # Eq. 11's Q(W^u): the decode step reads the codes instead of the bf16 values
+        self.UQ = [q.qsvd_quantize_up(u, nb.u_bits) for u in self.U] if nb.u_bits else None
         if X_from is None:
             self.Xp = bf16(inp.X_prefill.reshape(wl.B * wl.prefill, s.d))
             self.Xd = bf16(inp.X_decode)                   # [S, B, d]
@@ -179,10 +184,10 @@ class NativeBench:
     cached, as it does in serving.  `flush`: one copy, L2 evicted by a 256 MiB
     read before every sub-step (code cold as well)."""
 
-    def __init__(self, wl, rank, l2="rotate", rot=False):
+    def __init__(self, wl, rank, l2="rotate", rot=False, u_bits=0):
         import torch
         import paper_2510_16292_gb300 as q
-        self.torch, self.q, self.wl, self.rot = torch, q, wl, rot
+        self.torch, self.q, self.wl, self.rot, self.u_bits = torch, q, wl, rot, u_bits
         s = wl.shape
         self.dev = torch.device("cuda", torch.cuda.current_device())
         dev = self.dev
@@ -190,7 +195,7 @@ class NativeBench:
         self.B, self.P, self.S = B, P, S
         self.l2 = l2
         tok = (s.r + 4) if wl.lat_bits == 8 else (s.r // 2 + 2 * (s.r // 128))
-        layer_bytes = 3 * s.r * s.d * 2 + s.r * s.d + B * wl.tmax * tok      # what a decode step reads
+        layer_bytes = 3 * self.up_bytes() + s.r * s.d + B * wl.tmax * tok      # what a decode step reads
         self.K = 1 if l2 == "flush" else max(2, min(16, -(-2 * L2_BYTES // layer_bytes)))
         self.layer_bytes = layer_bytes
         self.layers = []
@@ -219,6 +224,12 @@ class NativeBench:
         self.stream = torch.cuda.current_stream()
         self._marshal()
 
+    def up_bytes(self):
+        """Bytes of one up-projection as the decode step reads it: bf16 values,
+        or int8 / int4 codes plus one fp32 scale per output channel."""
+        s = self.wl.shape
+        return s.r * s.d * 2 if not self.u_bits else s.r * s.d * self.u_bits // 8 + 4 * s.d
+
     def _marshal(self, stream=None):
         """Pre-build the ctypes argument tuples of every C-ABI call of a step,
         bound to `stream` (default: the current stream)."""
@@ -229,6 +240,7 @@ class NativeBench:
         self.pre_args, self.dec_proj, self.dec_attn, self.dec_fused = [], [], [], []
         for L in self.layers:
             L.cW, L.cC = L.W._c(), L.cache._c()
+            L.cU = [u._c() for u in L.UQ] if L.UQ else None
             self.pre_args.append((ctypes.byref(L.cW), L.Xp.data_ptr(), self.B * self.P, 1.0, wl.lat_bits, 1.0,
                                   None, None, ctypes.byref(L.cC), self.pseq.data_ptr(), self.ppos.data_ptr(),
                                   None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st))
@@ -237,8 +249,9 @@ class NativeBench:
                 proj.append((ctypes.byref(L.cW), L.Xd[t].data_ptr(), self.B, 1.0, wl.lat_bits, 1.0,
                              None, None, ctypes.byref(L.cC), self.dseq.data_ptr(), self.dpos[t].data_ptr(),
                              None, None, None, self.wsp.data_ptr(), self.wsp.numel(), st))
-                attn.append((ctypes.byref(L.cC), self.dlen[t].data_ptr(), self.P + t + 1,
-                             L.U[0].data_ptr(), L.U[1].data_ptr(), L.U[2].data_ptr(), s.H, s.dh,
+                ups = ([ctypes.byref(u) for u in L.cU] if L.cU else
+                       [L.U[0].data_ptr(), L.U[1].data_ptr(), L.U[2].data_ptr()])
+                attn.append((ctypes.byref(L.cC), self.dlen[t].data_ptr(), self.P + t + 1, *ups, s.H, s.dh,
                              1.0 / math.sqrt(s.dh), L.O.data_ptr(), self.wsd.data_ptr(), self.wsd.numel(), st))
                 fused.append((ctypes.byref(L.cW), L.Xd[t].data_ptr(), ctypes.byref(L.cC),
                               self.dlen[t].data_ptr(), self.P + t + 1, L.U[0].data_ptr(),
@@ -284,7 +297,8 @@ class NativeBench:
                 self._call(self.lib.qsvd_decode_step, self.dec_fused[k][t])
             else:
                 self._call(self.lib.qsvd_latent_project, self.dec_proj[k][t])
-                self._call(self.lib.qsvd_latent_decode_attn, self.dec_attn[k][t])
+                self._call(self.lib.qsvd_latent_decode_attn_qu if self.u_bits else self.lib.qsvd_latent_decode_attn,
+                           self.dec_attn[k][t])
 
     def flush(self):
         """`flush` method: evict L2 by reading a 256 MiB buffer (an fp32 sum in
@@ -368,14 +382,15 @@ class NativeBench:
             return r * d + 4 * r + 2 * T * d + T * (tok + stok)
         if label == "requant":
             return 4 * T * r + T * (tok + stok) + 8 * T
+        ub = self.up_bytes()
         if label == "qproj":
-            return r * d * 2 + B * (tok + stok) + 4 * B * d
+            return ub + B * (tok + stok) + 4 * B * d
         if label == "qabsorb":
-            return r * d * 2 + 4 * B * d + 4 * B * H * r
+            return ub + 4 * B * d + 4 * B * H * r
         if label in ("attn_chunk", "attn_tc", "attn_mma"):
             return B * L * (tok + stok) + 4 * B * H * r
         if label == "combine_uv":
-            return r * d * 2 + 4 * B * d
+            return ub + 4 * B * d
         if label == "decode_step":
             return self.step_roofline_bytes(ctx[1])
         return 0
@@ -387,7 +402,7 @@ class NativeBench:
         d, r = s.d, s.r
         tok = (r + 4) if self.wl.lat_bits == 8 else (r // 2 + 2 * (r // 128))
         L = self.P + t + 1
-        return B * L * tok + B * tok + 3 * r * d * 2 + d * r + 4 * r + B * d * 2 + 4 * B * d
+        return B * L * tok + B * tok + 3 * self.up_bytes() + d * r + 4 * r + B * d * 2 + 4 * B * d
 
     # ---- end to end through the public binding with host buffers ----
     def e2e(self, steps, warmup):
@@ -420,8 +435,12 @@ class NativeBench:
                     dXd.copy_(hx_d[k][t], non_blocking=True)
                     q.qsvd_latent_project(L.W, dXd, 1.0, self.wl.lat_bits, 1.0, dst=L.cache,
                                           dst_seq=self.dseq, dst_pos=self.dpos[t], workspace=self.wsp)
-                    q.qsvd_latent_decode_attn(L.cache, self.dlen[t], self.P + t + 1, *L.U, s.H, s.dh, L.O,
-                                              workspace=self.wsd)
+                    if L.UQ:
+                        q.qsvd_latent_decode_attn_qu(L.cache, self.dlen[t], self.P + t + 1, *L.UQ, s.H, s.dh, L.O,
+                                                     workspace=self.wsd)
+                    else:
+                        q.qsvd_latent_decode_attn(L.cache, self.dlen[t], self.P + t + 1, *L.U, s.H, s.dh, L.O,
+                                                  workspace=self.wsd)
                     hO[k, t].copy_(L.O, non_blocking=True)
                 evs[t + 1][1].record()
             torch.cuda.synchronize()
@@ -435,12 +454,14 @@ class NativeBench:
         return self.B * self.S * K / dec_s, h2d, d2h
 
 
-def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
+def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3, w4a4=False):
     """Prefill projection at the LLaVA-13B batch shape (8 x (5 x 576 + 128)
     tokens, d=5120, r=2048): time of the whole qsvd_latent_project call and of
     its tensor-core GEMM kernel (library events), cold L2 before each call.
     Inputs: seeded torch Gaussians (X with the outlier-channel pattern of the
-    synthetic recipe), W_d columns scaled by j^-0.5."""
+    synthetic recipe), W_d columns scaled by j^-0.5.  w4a4: int4 codes of W_d
+    and X on the fp8 (e4m3) tensor-core path, an int4 latent, measured against
+    the fp8 peak (the measured bf16 peak times the nominal fp8 / bf16 ratio, 2)."""
     import torch
     import paper_2510_16292_gb300 as q
     dev = torch.device("cuda", torch.cuda.current_device())
@@ -451,9 +472,14 @@ def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
     X = X.to(torch.bfloat16)
     Wd = torch.randn((d, r), generator=g, device=dev) / math.sqrt(d)
     Wd *= torch.arange(1, r + 1, device=dev, dtype=torch.float32) ** -0.5
-    W = q.qsvd_quantize_weight(Wd.contiguous())
-    lc = torch.empty((T, r), dtype=torch.int8, device=dev)
-    ls = torch.empty((T,), dtype=torch.float32, device=dev)
+    W = q.qsvd_quantize_weight(Wd.contiguous(), w_bits=4 if w4a4 else 8, x_bits=4 if w4a4 else 8)
+    if w4a4:
+        lc = torch.empty((T, r // 2), dtype=torch.uint8, device=dev)
+        ls = torch.empty((T, r // 128), dtype=torch.float16, device=dev)
+    else:
+        lc = torch.empty((T, r), dtype=torch.int8, device=dev)
+        ls = torch.empty((T,), dtype=torch.float32, device=dev)
+    kname = "gemm_f8" if w4a4 else "gemm_tc"
     ws = torch.zeros(q.qsvd_project_workspace_bytes(T, d, r), dtype=torch.uint8, device=dev)
     flush = torch.ones((256 << 20) // 4, dtype=torch.float32, device=dev)
     sink = torch.zeros((), dtype=torch.float32, device=dev)
@@ -470,24 +496,30 @@ def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3):
     for it in range(iters + 1):
         torch.sum(flush, dim=(0,), out=sink)
         lib.qsvd_profile_events(handles, n)
-        q.qsvd_latent_project(W, X, lat_codes=lc, lat_scales=ls, workspace=ws)
+        q.qsvd_latent_project(W, X, lat_bits=4 if w4a4 else 8, lat_codes=lc, lat_scales=ls, workspace=ws)
         torch.cuda.synchronize()
         cnt = lib.qsvd_profile_count()
         labels = [lib.qsvd_profile_label(i).decode() for i in range(cnt)]
         lib.qsvd_profile_events(None, 0)
         if it == 0:
             continue
-        gi = labels.index("gemm_tc")
+        gi = labels.index(kname)
         gemm.append(events[gi - 1].elapsed_time(events[gi]) * 1e-3)
         call.append(events[0].elapsed_time(events[cnt - 1]) * 1e-3)
     ops = 2.0 * T * d * r
     _, bf16_peak, kind = peaks()
     g_s, c_s = min(gemm), min(call)
     del X, W, lc, ls, ws, flush
-    return {"shape": f"T={T} d={d} r={r} (8 x 3008 tokens, LLaVA-13B layer)", "gemm_us": round(g_s * 1e6, 2),
-            "gemm_tops": round(ops / g_s / 1e12, 1), "gemm_frac_of_bf16_peak": round(ops / g_s / 1e12 / bf16_peak, 4),
-            "project_call_us": round(c_s * 1e6, 2), "project_call_tops": round(ops / c_s / 1e12, 1),
-            "peak_kind": kind}
+    out = {"shape": f"T={T} d={d} r={r} (8 x 3008 tokens, LLaVA-13B layer)", "gemm_us": round(g_s * 1e6, 2),
+           "gemm_tops": round(ops / g_s / 1e12, 1), "gemm_frac_of_bf16_peak": round(ops / g_s / 1e12 / bf16_peak, 4),
+           "project_call_us": round(c_s * 1e6, 2), "project_call_tops": round(ops / c_s / 1e12, 1),
+           "peak_kind": kind}
+    if w4a4:
+        out["setting"] = "W4A4 (int4 X and W_d as e4m3, kind::f8f6f4), int4 latent"
+        out["gemm_frac_of_fp8_peak"] = round(ops / g_s / 1e12 / (2 * bf16_peak), 4)
+        out["fp8_peak_tflops"] = round(2 * bf16_peak, 1)
+        out["fp8_peak_kind"] = kind + " bf16 x nominal fp8/bf16 ratio 2"
+    return out
 
 
 PREFILL_SHAPES = {
@@ -665,7 +697,7 @@ def run_native(args, rank, world, local_rank):
     wl = synthetic.WORKLOADS[args.workload]
     if args.decode_steps:
         wl = dataclasses.replace(wl, decode_steps=args.decode_steps)
-    nb = NativeBench(wl, rank, l2=args.l2, rot=args.rot)
+    nb = NativeBench(wl, rank, l2=args.l2, rot=args.rot, u_bits=args.u_bits)
     K = nb.K
     S = wl.decode_steps
     hbm, _, peak_kind = peaks()
@@ -727,6 +759,7 @@ def run_native(args, rank, world, local_rank):
                "d2h_bytes_per_step": d2h}
 
     pre13 = prefill_gemm_probe() if not args.no_prefill13 else None
+    pre13_w4 = prefill_gemm_probe(w4a4=True) if not args.no_prefill13 else None
     pre_attn = None if args.no_prefill_attn else {
         k: {p: prefill_attn_probe(k, path=p) for p in ("blocks", "rows")} for k in PREFILL_REPORTED}
     if rank != 0:
@@ -737,7 +770,9 @@ def run_native(args, rank, world, local_rank):
         "ms_per_step": round((dec_total + pre_total) / args.steps * 1e3, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int8/fp32",
         "data": "synthetic",
-        "config": {"workload": workload_desc(wl) + (" + online H1 rotation of X (Eq. 12)" if args.rot else ""),
+        "config": {"workload": workload_desc(wl) + (" + online H1 rotation of X (Eq. 12)" if args.rot else "") +
+                   (f" + int{args.u_bits} up-projections (Eq. 11 Q(W^u), per-output-channel scales)"
+                    if args.u_bits else ""),
                    "global_batch": world * wl.B,
                    "seq_len": wl.tmax, "parallelism": f"replicas x{world} (one independent layer per GPU)",
                    "l2": (f"inputs larger than L2: {K} independently seeded copies of the layer "
@@ -758,6 +793,7 @@ def run_native(args, rank, world, local_rank):
             "wall_s_timed_region": round(t_wall, 3),
             "kernels": kernels,
             "prefill_13b": pre13,
+            "prefill_13b_w4a4": pre13_w4,
             "prefill_attn": pre_attn,
         },
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,

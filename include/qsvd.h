@@ -16,6 +16,8 @@
  *   qsvd_latent_project      C = Q(X) Q(W_d), requantized per token (Eq. 11-12)
  *   qsvd_cache_append        store latent rows in the latent cache (Fig. 2(f))
  *   qsvd_latent_decode_attn  one decode step of attention over that cache (Eq. 5)
+ *   qsvd_quantize_up         offline per-channel RTN of an up-projection (Eq. 11)
+ *   qsvd_latent_decode_attn_qu  the decode step with quantized up-projections
  *   qsvd_latent_prefill_attn causal attention of prompt tokens over that cache
  *   qsvd_latent_prefill      the same for whole prompt blocks, K and V materialised
  *
@@ -73,7 +75,7 @@ extern "C" {
 #define QSVD_EUNSUPPORTED  -2  /* device is not sm_103, or a shape the kernels do not cover */
 #define QSVD_ECUDA         -3  /* a CUDA runtime call or launch failed */
 #define QSVD_ETIMEOUT      -4  /* a bounded device-side wait expired (from qsvd_check) */
-#define QSVD_ERANGE        -5  /* a cache position or sequence index out of range */
+#define QSVD_ERANGE        -5  /* a cache position or sequence index out of range, or a value saturated at the fp16 range of the block prefill */
 #define QSVD_ENOSPC        -6  /* workspace smaller than the *_workspace_bytes figure */
 
 /*
@@ -84,6 +86,15 @@ extern "C" {
  * patterns in the same layout; it is the tensor-core operand of the prefill
  * GEMM (every int8 code is exact in bf16).  All three are produced by
  * qsvd_quantize_weight.  Requirements: d % 64 == 0, r % 16 == 0.
+ *
+ * The quantization setting (Sec. 4 setup: W8A8, W8A4, W4A4) is part of the
+ * weight: w_bits says how W_d was quantized (8: codes in [-127, 127]; 4: in
+ * [-7, 7], stored one per int8 byte; 0 reads as 8) and x_bits how
+ * qsvd_latent_project quantizes X per token (8 or 4; 0 reads as 8).  With
+ * w_bits = x_bits = 4 the prefill GEMM runs on codes_e4m3, the codes as fp8
+ * e4m3 bytes (every value in [-7, 7] is exact in e4m3), on the fp8 tensor-core
+ * path; without it, or for the mixed settings, on codes_bf16.  The latent is
+ * requantized to lat_bits as before (W4A4 pairs with an int4 latent cache).
  */
 typedef struct qsvd_down_weight {
     const int8_t   *codes;       /* [r, d] */
@@ -94,6 +105,9 @@ typedef struct qsvd_down_weight {
     int32_t rot;                 /* 0: the codes quantize W_d and X is quantized as it is (H1 = I or folded
                                     offline); b > 0: they quantize H1 W_d (qsvd_quantize_weight_rotated) and
                                     qsvd_latent_project rotates every row of X by H1 before quantizing it */
+    int32_t w_bits;              /* 8 (or 0) or 4: bits of the codes */
+    int32_t x_bits;              /* 8 (or 0) or 4: bits X is quantized to per token */
+    const uint8_t *codes_e4m3;   /* [r, d] or NULL: the codes as fp8 e4m3 (W4A4 tensor-core operand) */
 } qsvd_down_weight;
 
 /*
@@ -125,9 +139,19 @@ int qsvd_quantize_weight(const float *W_d, int32_t d, int32_t r, float clip,
                          cudaStream_t stream);
 
 /*
+ * The same for any setting: bits 8 or 4 (codes in [-7, 7] for 4), rot 0 or
+ * the H1 block size (as qsvd_quantize_weight_rotated), and optional images
+ * codes_bf16 [r, d] and codes_e4m3 [r, d] (fp8 e4m3 bytes; needs bits 4).
+ */
+int qsvd_quantize_weight_ex(const float *W_d, int32_t d, int32_t r, float clip, int32_t bits, int32_t rot,
+                            int8_t *codes, uint16_t *codes_bf16, uint8_t *codes_e4m3, float *scale,
+                            cudaStream_t stream);
+
+/*
  * Quantized joint down-projection with the latent requantization fused
  * behind it (Eq. 12 with H1 = H2 = I, then Eq. 11's Q(C_qkv)):
- *   1. X [T, d] bf16 is quantized per token to int8 (clip `act_clip`);
+ *   1. X [T, d] bf16 is quantized per token to int8 (int4 codes when
+ *      W->x_bits == 4) (clip `act_clip`);
  *   2. acc[t, j] = sum_k xq[t, k] * codes[j, k]    exact int32;
  *   3. c[t, j] = fp32(fp32(fp32(acc) * s_x[t]) * scale[j])   (no FMA);
  *   4. c[t, :] is requantized per token to `lat_bits` (8: one fp32 scale per
@@ -225,6 +249,48 @@ int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int
 size_t qsvd_decode_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t r, int32_t H, int32_t dh);
 
 /*
+ * Quantized up-projection (Eq. 11: Y' = Q(C) Q(H2 W^u) with H2 = I, the
+ * rotation folded offline), for qsvd_latent_decode_attn_qu.  One of U_q, U_k,
+ * U_v ([r, d] with d = H * dh; column c is output channel c) quantized per
+ * output channel by symmetric RTN (the weight quantizer of the Sec. 4 setup):
+ *   bits == 8: codes int8 [r, d], codes[j * d + c] the code of U[j, c];
+ *   bits == 4: codes uint8 [r, d/2], column 2i in the low nibble of byte
+ *              j * d/2 + i, two's complement;
+ *   scale fp32 [d]: U[j, c] ~ code(j, c) * scale[c].
+ */
+typedef struct qsvd_up_weight {
+    const void  *codes;
+    const float *scale;
+    int32_t bits;
+    int32_t r;
+    int32_t d;
+} qsvd_up_weight;
+
+/*
+ * Offline Q(W^u) (Eq. 11) of one up-projection: U bf16 [r, d] row-major ->
+ * codes and scale in the qsvd_up_weight layout above (the library's quantizer
+ * with q_max = 127 or 7 and clipping ratio `clip` in (0, 1], per column).
+ * Requirements: d % 32 == 0, bits 8 or 4.
+ */
+int qsvd_quantize_up(const uint16_t *U, int32_t r, int32_t d, int32_t bits, float clip, void *codes, float *scale,
+                     cudaStream_t stream);
+
+/*
+ * qsvd_latent_decode_attn with quantized up-projections (Eq. 11): the same
+ * decode step (Eq. 5, U_k absorbed into the query, U_v applied last) where
+ * every product with an up-projection reads its int8 or int4 codes and
+ * applies the per-output-channel scales (q = s_q * (c U_q codes);
+ * q~_h = U_k codes (s_k * q_h); o = s_v * (o_lat U_v codes)), so a step
+ * streams half (int8) or a quarter (int4) of the bf16 weight bytes.  The
+ * three weights may differ in bits; each must have r = cache->r and d = H*dh.
+ * Workspace and requirements as for qsvd_latent_decode_attn.
+ */
+int qsvd_latent_decode_attn_qu(const qsvd_cache *cache, const int32_t *seq_len, int32_t max_seq_len,
+                               const qsvd_up_weight *U_q, const qsvd_up_weight *U_k, const qsvd_up_weight *U_v,
+                               int32_t H, int32_t dh, float softmax_scale, float *O,
+                               void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * Causal attention of prompt tokens over the latent cache (prefill; Fig. 2(f)
  * and Eq. 5 with the causal mask of a decoder).  Row i of the call is one
  * query: the token at position q_len[i]-1 of cache sequence q_seq[i], which
@@ -273,7 +339,10 @@ size_t qsvd_prefill_workspace_bytes(int64_t n, int32_t max_len, int32_t r, int32
  * and finite; a block outside the cache (seq outside [0, B), t0 < 0, T < 1,
  * t0 + T > Tmax) returns QSVD_EINVAL before anything is enqueued; a launch of
  * 64 blocks whose padded rows R give R * r / 8 >= 2^31 returns
- * QSVD_EUNSUPPORTED.  fp16 Q, K, V hold magnitudes up to 65504.
+ * QSVD_EUNSUPPORTED.  fp16 Ut, Q, K, V (and the int4 latent operand) hold
+ * magnitudes up to 65504: a larger value is saturated to +-65504 and flags
+ * QSVD_ERANGE for qsvd_check (qsvd_prefill_weights likewise for |U| above
+ * 65504), so no inf is produced silently.
  */
 typedef struct {
     int32_t seq, t0, T;

@@ -5,7 +5,8 @@ weights (Sec. 2.3 background: X' = XH with the matching H^T applied to W).
 H1 is either folded too (H1 = I here: C_qkv ~= Q(X) Q(W_d)) or applied to X
 on the fly (``rot``, oracle.rotate) with W_d replaced by H1 W_d:
 
-  1. X [T, d] -> int8 codes Xq and an fp32 scale s_x per token;
+  1. X [T, d] -> int8 codes Xq (int4 in the W4A4 setting, with int4 codes
+     of W_d too) and an fp32 scale s_x per token;
   2. acc[t, j] = sum_k Xq[t, k] * Wq[k, j]      (exact integer arithmetic);
   3. c_hat[t, j] = fp32( fp32( fp32(acc[t,j]) * s_x[t] ) * s_w[j] );
   4. Eq. 11's Q(C_qkv): c_hat is quantized per token again -- int8 with one
@@ -32,13 +33,14 @@ def int_matmul(A, B):
     return np.rint(A.astype(np.float64) @ B.astype(np.float64)).astype(np.int64)
 
 
-def quantize_activations(X, act_clip: float = 1.0):
-    """Step 1: per-token int8 codes and fp32 scales of X (bf16 values)."""
-    return quant.quantize_rows(X, 8, act_clip)
+def quantize_activations(X, act_clip: float = 1.0, x_bits: int = 8):
+    """Step 1: per-token codes (int8, or int4 for the W4A4 setting of the
+    Sec. 4 setup) and fp32 scales of X (bf16 values)."""
+    return quant.quantize_rows(X, x_bits, act_clip)
 
 
 def down_project(Xq, Wq):
-    """Step 2: acc = Xq @ Wq with Wq [d, r] int8 codes (int64 result)."""
+    """Step 2: acc = Xq @ Wq with Wq [d, r] int8 or int4 codes (int64 result)."""
     return int_matmul(Xq, Wq)
 
 
@@ -61,14 +63,15 @@ def requantize_latent(c_hat, lat_bits: int, lat_clip: float = 1.0):
     raise ValueError("lat_bits must be 8 or 4")
 
 
-def latent_project(X, Wq, s_w, act_clip=1.0, lat_bits=8, lat_clip=1.0, rot: int = 0):
+def latent_project(X, Wq, s_w, act_clip=1.0, lat_bits=8, lat_clip=1.0, rot: int = 0, x_bits: int = 8):
     """Steps 1-4 for a block of tokens.  Returns a dict with every
     intermediate the GPU path can expose: xq, s_x, acc, c_hat, codes, scale.
     rot = b > 0: the rows are rotated by H1 (block b, oracle.rotate) before
-    step 1, as Eq. 12 quantizes X H1^T; Wq must then be the codes of H1 W^d."""
+    step 1, as Eq. 12 quantizes X H1^T; Wq must then be the codes of H1 W^d.
+    x_bits = 4 with 4-bit Wq is the W4A4 setting (Sec. 4 setup)."""
     if rot:
         X = rotate.rotate_rows(np.asarray(X, dtype=np.float32), rot)
-    xq, s_x = quantize_activations(X, act_clip)
+    xq, s_x = quantize_activations(X, act_clip, x_bits)
     acc = down_project(xq, Wq)
     c_hat = dequantize_acc(acc, s_x, s_w)
     codes, scale = requantize_latent(c_hat, lat_bits, lat_clip)

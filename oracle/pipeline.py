@@ -27,14 +27,15 @@ TINY_BETA = 0.5
 
 
 def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1.0, rot: int = 0,
-                    u_bits: int = 0):
+                    u_bits: int = 0, w_bits: int = 8):
     """Returns dict(W_d fp32 values [d, r], Wq int64 [d, r], s_w [r],
     U_q/U_k/U_v bf16 bits [r, d], rot).  rot = b > 0: Wq, s_w quantize
     H1 W_d (oracle.rotate, block b) instead of W_d (W_d itself is returned
     unrotated: it is what the caller hands to the GPU's rotating quantizer).
     u_bits = 8 or 4: Eq. 11's Q(H2 W^u) as well (H2 = I): every column of
     U_q, U_k, U_v quantized per output channel (U*_codes, U*_scale), and the
-    attention uses the dequantized values (U*_deq)."""
+    attention uses the dequantized values (U*_deq).  w_bits = 4: W_d's codes
+    are int4 (with x_bits = 4 in OracleLayer, the W4A4 setting of Sec. 4)."""
     s = inp.workload.shape
     if inp.W_qkv is not None:
         d = s.d
@@ -44,9 +45,10 @@ def prepare_weights(inp: LayerInputs, beta: float = TINY_BETA, w_clip: float = 1
         U_q, U_k, U_v = bf16_bits(Uq), bf16_bits(Uk), bf16_bits(Uv)
     else:
         W_d, U_q, U_k, U_v = inp.W_d, inp.U_q, inp.U_k, inp.U_v
-    Wq, s_w = quant.quantize_columns(rotate.rotate_weight(W_d, rot) if rot else W_d, 8, w_clip)
+    Wq, s_w = quant.quantize_columns(rotate.rotate_weight(W_d, rot) if rot else W_d, w_bits, w_clip)
     c = np.ascontiguousarray
-    out = dict(W_d=c(W_d), Wq=c(Wq), s_w=c(s_w), U_q=c(U_q), U_k=c(U_k), U_v=c(U_v), rot=rot, u_bits=u_bits)
+    out = dict(W_d=c(W_d), Wq=c(Wq), s_w=c(s_w), U_q=c(U_q), U_k=c(U_k), U_v=c(U_v), rot=rot, u_bits=u_bits,
+               w_bits=w_bits)
     if u_bits:
         for k in ("U_q", "U_k", "U_v"):
             codes, scale = quantize_up(bf16_from_bits(out[k]), u_bits)
@@ -67,7 +69,7 @@ class OracleLayer:
 
     def __init__(self, shape, weights: Dict, B: int, tmax: int, lat_bits: int,
                  act_clip: float = 1.0, lat_clip: float = 1.0,
-                 track: Optional[Iterable[int]] = None):
+                 track: Optional[Iterable[int]] = None, x_bits: int = 8):
         self.s = shape
         self.w = weights
         if weights.get("u_bits"):
@@ -77,7 +79,7 @@ class OracleLayer:
             self.U_k = bf16_from_bits(weights["U_k"])
             self.U_v = bf16_from_bits(weights["U_v"])
         self.B, self.tmax, self.bits = B, tmax, lat_bits
-        self.act_clip, self.lat_clip = act_clip, lat_clip
+        self.act_clip, self.lat_clip, self.x_bits = act_clip, lat_clip, x_bits
         self.cache = latent.LatentCache(B, tmax, shape.r, lat_bits)
         self.len = np.zeros(B, dtype=np.int64)
         self.track = set(range(B)) if track is None else set(track)
@@ -88,7 +90,7 @@ class OracleLayer:
         """Eq. 12 for a block of tokens given as bf16 bits [T, d]."""
         X = bf16_from_bits(X_bits)
         return latent.latent_project(X, self.w["Wq"], self.w["s_w"],
-                                     self.act_clip, self.bits, self.lat_clip, self.w.get("rot", 0))
+                                     self.act_clip, self.bits, self.lat_clip, self.w.get("rot", 0), self.x_bits)
 
     def _append(self, seq, pos, codes, scale):
         self.cache.append(seq, pos, codes, scale)

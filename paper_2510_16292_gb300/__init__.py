@@ -30,9 +30,10 @@ _lib = ctypes.CDLL(_LIB_PATH)
 
 QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
-EXPORTS = ("qsvd_quantize_weight", "qsvd_quantize_weight_rotated", "qsvd_importance_scores",
+EXPORTS = ("qsvd_quantize_weight", "qsvd_quantize_weight_rotated", "qsvd_quantize_weight_ex", "qsvd_importance_scores",
            "qsvd_importance_workspace_bytes", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
+           "qsvd_quantize_up", "qsvd_latent_decode_attn_qu",
            "qsvd_latent_prefill_attn", "qsvd_prefill_workspace_bytes", "qsvd_prefill_weights",
            "qsvd_latent_prefill", "qsvd_latent_prefill_workspace_bytes",
            "qsvd_decode_step", "qsvd_decode_step_workspace_bytes", "qsvd_latent_project_static",
@@ -48,12 +49,18 @@ class QsvdError(RuntimeError):
 
 class _DownWeight(ctypes.Structure):
     _fields_ = [("codes", ctypes.c_void_p), ("codes_bf16", ctypes.c_void_p), ("scale", ctypes.c_void_p),
-                ("d", ctypes.c_int32), ("r", ctypes.c_int32), ("rot", ctypes.c_int32)]
+                ("d", ctypes.c_int32), ("r", ctypes.c_int32), ("rot", ctypes.c_int32),
+                ("w_bits", ctypes.c_int32), ("x_bits", ctypes.c_int32), ("codes_e4m3", ctypes.c_void_p)]
 
 
 class _Cache(ctypes.Structure):
     _fields_ = [("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p), ("bits", ctypes.c_int32),
                 ("B", ctypes.c_int32), ("Tmax", ctypes.c_int32), ("r", ctypes.c_int32)]
+
+
+class _UpWeight(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_void_p), ("scale", ctypes.c_void_p), ("bits", ctypes.c_int32),
+                ("r", ctypes.c_int32), ("d", ctypes.c_int32)]
 
 
 class _PrefillBlock(ctypes.Structure):
@@ -63,6 +70,7 @@ class _PrefillBlock(ctypes.Structure):
 _vp, _i32, _i64, _f32, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
 _lib.qsvd_quantize_weight.argtypes = [_vp, _i32, _i32, _f32, _vp, _vp, _vp, _vp]
 _lib.qsvd_quantize_weight_rotated.argtypes = [_vp, _i32, _i32, _f32, _i32, _vp, _vp, _vp, _vp]
+_lib.qsvd_quantize_weight_ex.argtypes = [_vp, _i32, _i32, _f32, _i32, _i32, _vp, _vp, _vp, _vp, _vp]
 _lib.qsvd_importance_scores.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
 _lib.qsvd_importance_workspace_bytes.argtypes = [_i32, _i32]
 _lib.qsvd_importance_workspace_bytes.restype = _sz
@@ -73,6 +81,10 @@ _lib.qsvd_project_workspace_bytes.restype = _sz
 _lib.qsvd_cache_append.argtypes = [ctypes.POINTER(_Cache), _vp, _vp, _i64, _vp, _vp, _vp]
 _lib.qsvd_latent_decode_attn.argtypes = [ctypes.POINTER(_Cache), _vp, _i32, _vp, _vp, _vp, _i32, _i32, _f32,
                                          _vp, _vp, _sz, _vp]
+_lib.qsvd_quantize_up.argtypes = [_vp, _i32, _i32, _i32, _f32, _vp, _vp, _vp]
+_lib.qsvd_latent_decode_attn_qu.argtypes = [ctypes.POINTER(_Cache), _vp, _i32, ctypes.POINTER(_UpWeight),
+                                            ctypes.POINTER(_UpWeight), ctypes.POINTER(_UpWeight), _i32, _i32, _f32,
+                                            _vp, _vp, _sz, _vp]
 _lib.qsvd_decode_workspace_bytes.argtypes = [_i32, _i32, _i32, _i32, _i32]
 _lib.qsvd_decode_workspace_bytes.restype = _sz
 _lib.qsvd_latent_prefill_attn.argtypes = [ctypes.POINTER(_Cache), _vp, _vp, _i64, _i32, _vp, _vp, _vp, _i32, _i32,
@@ -132,11 +144,16 @@ def _check(status: int):
 class DownWeight:
     """Quantized W_d: codes int8 [r, d], codes_bf16 bf16 [r, d], scale fp32 [r];
     rot > 0: the codes quantize H1 W_d (block Hadamard of rot channels) and
-    the projection rotates X by H1 on the fly."""
+    the projection rotates X by H1 on the fly.  w_bits / x_bits: the setting
+    (8/8 W8A8, 8/4 W8A4, 4/4 W4A4); codes_e4m3 uint8 [r, d]: the fp8 image
+    of 4-bit codes, the W4A4 tensor-core operand."""
     codes: torch.Tensor
     codes_bf16: torch.Tensor
     scale: torch.Tensor
     rot: int = 0
+    w_bits: int = 8
+    x_bits: int = 8
+    codes_e4m3: Optional[torch.Tensor] = None
 
     @property
     def d(self):
@@ -148,7 +165,8 @@ class DownWeight:
 
     def _c(self):
         return _DownWeight(_ptr(self.codes, torch.int8, "W.codes"), _ptr(self.codes_bf16, _BF16, "W.codes_bf16"),
-                           _ptr(self.scale, _F32, "W.scale"), self.d, self.r, self.rot)
+                           _ptr(self.scale, _F32, "W.scale"), self.d, self.r, self.rot, self.w_bits, self.x_bits,
+                           _ptr(self.codes_e4m3, torch.uint8, "W.codes_e4m3"))
 
 
 @dataclasses.dataclass
@@ -181,14 +199,69 @@ class LatentCache:
         return self.r if self.bits == 8 else self.r // 2 + 2 * (self.r // 128)
 
 
-def qsvd_quantize_weight(W_d: torch.Tensor, clip: float = 1.0, stream=None, rot: int = 0) -> DownWeight:
-    """W_d fp32 [d, r] -> DownWeight (per-output-channel int8 RTN); rot > 0:
-    of H1 W_d (qsvd_quantize_weight_rotated), and the projection then rotates X."""
+@dataclasses.dataclass
+class UpWeight:
+    """Eq. 11's Q(W^u) of one up-projection [r, d]: codes int8 [r, d] (bits 8)
+    or packed int4 uint8 [r, d/2] (bits 4), scale fp32 [d] per output channel."""
+    codes: torch.Tensor
+    scale: torch.Tensor
+    bits: int
+
+    @property
+    def r(self):
+        return self.codes.shape[0]
+
+    @property
+    def d(self):
+        return self.scale.shape[0]
+
+    def _c(self):
+        return _UpWeight(_ptr(self.codes, (torch.int8, torch.uint8), "U.codes"), _ptr(self.scale, _F32, "U.scale"),
+                         self.bits, self.r, self.d)
+
+
+def qsvd_quantize_up(U: torch.Tensor, bits: int = 8, clip: float = 1.0, stream=None) -> UpWeight:
+    """U bf16 [r, d] -> UpWeight (per-output-channel RTN to int8 or int4)."""
+    r, d = U.shape
+    if bits == 8:
+        codes = torch.empty((r, d), dtype=torch.int8, device=U.device)
+    else:
+        codes = torch.empty((r, d // 2), dtype=torch.uint8, device=U.device)
+    scale = torch.empty((d,), dtype=torch.float32, device=U.device)
+    _check(_lib.qsvd_quantize_up(_ptr(U, _BF16, "U"), r, d, bits, clip, _ptr(codes), _ptr(scale), _stream(stream)))
+    return UpWeight(codes, scale, bits)
+
+
+def qsvd_latent_decode_attn_qu(cache: "LatentCache", seq_len: torch.Tensor, max_seq_len: int, U_q: UpWeight,
+                               U_k: UpWeight, U_v: UpWeight, H: int, dh: int, O: torch.Tensor,
+                               softmax_scale: Optional[float] = None, workspace=None, stream=None) -> None:
+    """Decode attention with quantized up-projections (Eq. 11)."""
+    if softmax_scale is None:
+        softmax_scale = 1.0 / math.sqrt(dh)
+    if workspace is None:
+        workspace = torch.zeros(qsvd_decode_workspace_bytes(cache.B, max_seq_len, cache.r, H, dh),
+                                dtype=torch.uint8, device=O.device)
+    cc, uq, uk, uv = cache._c(), U_q._c(), U_k._c(), U_v._c()
+    _check(_lib.qsvd_latent_decode_attn_qu(ctypes.byref(cc), _ptr(seq_len, _I32, "seq_len"), max_seq_len,
+                                           ctypes.byref(uq), ctypes.byref(uk), ctypes.byref(uv), H, dh, softmax_scale,
+                                           _ptr(O, _F32, "O"), _ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def qsvd_quantize_weight(W_d: torch.Tensor, clip: float = 1.0, stream=None, rot: int = 0, w_bits: int = 8,
+                         x_bits: int = 8) -> DownWeight:
+    """W_d fp32 [d, r] -> DownWeight (per-output-channel RTN, int8 or with
+    w_bits = 4 int4 codes plus their e4m3 image); rot > 0: of H1 W_d, and the
+    projection then rotates X.  x_bits: how the projection quantizes X."""
     d, r = W_d.shape
     dev = W_d.device
     codes = torch.empty((r, d), dtype=torch.int8, device=dev)
     codes_bf16 = torch.empty((r, d), dtype=torch.bfloat16, device=dev)
     scale = torch.empty((r,), dtype=torch.float32, device=dev)
+    if w_bits != 8 or x_bits != 8:
+        e4 = torch.empty((r, d), dtype=torch.uint8, device=dev) if w_bits == 4 else None
+        _check(_lib.qsvd_quantize_weight_ex(_ptr(W_d, _F32, "W_d"), d, r, clip, w_bits, rot, _ptr(codes),
+                                            _ptr(codes_bf16), _ptr(e4), _ptr(scale), _stream(stream)))
+        return DownWeight(codes, codes_bf16, scale, rot, w_bits, x_bits, e4)
     if rot:
         _check(_lib.qsvd_quantize_weight_rotated(_ptr(W_d, _F32, "W_d"), d, r, clip, rot, _ptr(codes),
                                                  _ptr(codes_bf16), _ptr(scale), _stream(stream)))

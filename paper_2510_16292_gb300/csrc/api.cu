@@ -143,6 +143,8 @@ EncodeTiledFn encode_tiled() {
 }
 }  // namespace
 
+bool tensor_maps_available() { return encode_tiled() != nullptr; }
+
 bool encode_map_2d(CUtensorMap *map, CUtensorMapDataType type, const void *base, uint64_t inner, uint64_t outer,
                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swizzle) {
     EncodeTiledFn fn = encode_tiled();
@@ -225,7 +227,7 @@ int qsvd_check(cudaStream_t stream) {
         if (e != cudaSuccess) return cuda_fail(e, "clear error word");
     }
     if (word & kErrTimeout) return fail(QSVD_ETIMEOUT, "a bounded device wait expired");
-    if (word & kErrRange) return fail(QSVD_ERANGE, "a cache position, sequence index or length was out of range");
+    if (word & kErrRange) return fail(QSVD_ERANGE, "a cache position, sequence index or length was out of range, or a value was saturated at the fp16 range");
     g_msg[0] = 0;
     return QSVD_OK;
 }
@@ -251,6 +253,26 @@ int qsvd_quantize_weight(const float *W_d, int32_t d, int32_t r, float clip, int
     prof_mark(stream, "begin");
     cudaError_t e = launch_quantize_weight(W_d, d, r, clip, codes, codes_bf16, scale, stream);
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "quantize_weight launch");
+}
+
+int qsvd_quantize_weight_ex(const float *W_d, int32_t d, int32_t r, float clip, int32_t bits, int32_t rot,
+                            int8_t *codes, uint16_t *codes_bf16, uint8_t *codes_e4m3, float *scale,
+                            cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!W_d || !codes || !scale) return fail(QSVD_EINVAL, "quantize_weight_ex: null pointer");
+    if (d <= 0 || r <= 0) return fail(QSVD_EINVAL, "quantize_weight_ex: d and r must be positive");
+    if (!(clip > 0.0f && clip <= 1.0f)) return fail(QSVD_EINVAL, "quantize_weight_ex: clip must lie in (0, 1]");
+    if (bits != 8 && bits != 4) return fail(QSVD_EINVAL, "quantize_weight_ex: bits must be 8 or 4");
+    if (codes_e4m3 && bits != 4) return fail(QSVD_EINVAL, "quantize_weight_ex: an e4m3 image needs bits 4");
+    if (rot && (rot < 2 || (rot & (rot - 1)) || d % rot))
+        return fail(QSVD_EINVAL, "quantize_weight_ex: rot must be 0 or a power of two >= 2 dividing d");
+    if (rot && d > 6144) return fail(QSVD_EUNSUPPORTED, "quantize_weight_ex: rotation needs d <= 6144");
+    prof_mark(stream, "begin");
+    cudaError_t e = launch_quantize_weight(W_d, d, r, clip, codes, codes_bf16, scale, stream, rot, bits == 8 ? 127 : 7,
+                                           codes_e4m3);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "quantize_weight_ex launch");
 }
 
 int qsvd_quantize_weight_rotated(const float *W_d, int32_t d, int32_t r, float clip, int32_t rot, int8_t *codes,
@@ -295,6 +317,9 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
         return fail(QSVD_EINVAL, "latent_project: W->rot must be 0 or a power of two >= 2 dividing d");
     if (lat_bits != 8 && lat_bits != 4) return fail(QSVD_EINVAL, "latent_project: lat_bits must be 8 or 4");
     if (lat_bits == 4 && r % 128) return fail(QSVD_EUNSUPPORTED, "latent_project: int4 needs r %% 128 == 0");
+    const int wb = W->w_bits ? W->w_bits : 8, xb = W->x_bits ? W->x_bits : 8;
+    if ((wb != 8 && wb != 4) || (xb != 8 && xb != 4)) return fail(QSVD_EINVAL, "latent_project: W->w_bits and W->x_bits must be 8 or 4");
+    const int act_qmax = xb == 8 ? 127 : 7;
     if (!(act_clip > 0.0f && act_clip <= 1.0f) || !(lat_clip > 0.0f && lat_clip <= 1.0f))
         return fail(QSVD_EINVAL, "latent_project: clip ratios must lie in (0, 1]");
     const bool tok = lat_codes != nullptr || lat_scales != nullptr;
@@ -335,23 +360,37 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
         if (T < kPsSplitTok && !rot) {
             e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
                                   xq_out, xs_out, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
-                                  dst_pos, err, stream);
+                                  dst_pos, err, stream, nullptr, nullptr, true, act_qmax);
             return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "projection launch");
         }
         // each row quantized once, the dot products on the tensor cores, the rows requantized in parallel
-        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream, rot);
+        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream, rot, act_qmax);
         if (e == cudaSuccess)
             e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
                                   nullptr, nullptr, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
-                                  dst_pos, err, stream, xq, xs, false);
+                                  dst_pos, err, stream, xq, xs, false, act_qmax);
         if (e == cudaSuccess)
             e = launch_requant(c_hat, T, r, lat_bits, lat_clip, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
                                dst_pos, err, stream);
         return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "projection launch");
     }
-    if (W->codes_bf16 && gemm_tc_supported(d, r)) {
+    if (wb == 4 && xb == 4 && W->codes_e4m3 && gemm_f8_supported(d, r)) {
+        // W4A4 on the fp8 tensor-core path: e4m3 images of the int4 codes, exact products and sums
+        if (!aligned16(W->codes_e4m3)) return fail(QSVD_EINVAL, "latent_project: codes_e4m3 must be 16-byte aligned");
+        uint8_t *xq_f8 = reinterpret_cast<uint8_t *>(xq_bf16);            // the image slot holds T * d bytes
+        e = launch_xquant(X, T, d, act_clip, xq_out, nullptr, xs, stream, rot, act_qmax, xq_f8);
+        if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
+        if (gemm_tc_fused_supported(T, r, lat_bits)) {
+            e = launch_gemm_f8(xq_f8, T, d, W->codes_e4m3, W->scale, xs, r, lat_bits, lat_clip, lat_codes, lat_scales,
+                               dst ? &dv : nullptr, dst_seq, dst_pos, nullptr, acc_out, err, stream);
+            return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "fp8 tensor-core projection launch");
+        }
+        e = launch_gemm_f8(xq_f8, T, d, W->codes_e4m3, W->scale, xs, r, 0, lat_clip, nullptr, nullptr, nullptr,
+                           nullptr, nullptr, c_hat, acc_out, err, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "fp8 tensor-core projection launch");
+    } else if (W->codes_bf16 && gemm_tc_supported(d, r)) {
         if (!aligned16(W->codes_bf16)) return fail(QSVD_EINVAL, "latent_project: codes_bf16 must be 16-byte aligned");
-        e = launch_xquant(X, T, d, act_clip, xq_out, xq_bf16, xs, stream, rot);
+        e = launch_xquant(X, T, d, act_clip, xq_out, xq_bf16, xs, stream, rot, act_qmax);
         if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
         if (gemm_tc_fused_supported(T, r, lat_bits)) {
             // a2, a3 and a4 in one kernel: the latent never leaves the registers
@@ -363,7 +402,7 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
         e = launch_gemm_tc(xq_bf16, T, d, W->codes_bf16, W->scale, xs, r, c_hat, acc_out, err, stream);
         if (e != cudaSuccess) return cuda_fail(e, "tensor-core projection launch");
     } else {
-        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream, rot);
+        e = launch_xquant(X, T, d, act_clip, xq, nullptr, xs, stream, rot, act_qmax);
         if (e != cudaSuccess) return cuda_fail(e, "xquant launch");
         e = launch_proj_dp4a(xq, T, d, W->codes, W->scale, xs, r, c_hat, acc_out, stream);
         if (e != cudaSuccess) return cuda_fail(e, "projection launch");
@@ -414,10 +453,59 @@ int qsvd_latent_decode_attn(const qsvd_cache *cache, const int32_t *seq_len, int
     const size_t need = qsvd_decode_workspace_bytes(cache->B, max_seq_len, cache->r, H, dh);
     if (!workspace || workspace_bytes < need)
         return fail(QSVD_ENOSPC, "decode_attn: workspace needs %zu bytes", need);
-    DecodeArgs a{view(cache), seq_len, max_seq_len, U_q, U_k, U_v, H, dh, softmax_scale, O};
+    DecodeArgs a{view(cache), seq_len, max_seq_len, UpW{U_q, nullptr, 16}, UpW{U_k, nullptr, 16},
+                 UpW{U_v, nullptr, 16}, H, dh, softmax_scale, O};
     prof_mark(stream, "begin");
     cudaError_t e = launch_decode(a, workspace, workspace_bytes, err, stream);
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "decode_attn launch");
+}
+
+int qsvd_quantize_up(const uint16_t *U, int32_t r, int32_t d, int32_t bits, float clip, void *codes, float *scale,
+                     cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!U || !codes || !scale) return fail(QSVD_EINVAL, "quantize_up: null pointer");
+    if (r <= 0 || d <= 0 || d % 32) return fail(QSVD_EINVAL, "quantize_up: need r > 0 and d %% 32 == 0");
+    if (bits != 8 && bits != 4) return fail(QSVD_EINVAL, "quantize_up: bits must be 8 or 4");
+    if (!(clip > 0.0f && clip <= 1.0f)) return fail(QSVD_EINVAL, "quantize_up: clip must lie in (0, 1]");
+    prof_mark(stream, "begin");
+    const cudaError_t e = launch_quantize_up(U, r, d, bits, clip, codes, scale, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "quantize_up launch");
+}
+
+int qsvd_latent_decode_attn_qu(const qsvd_cache *cache, const int32_t *seq_len, int32_t max_seq_len,
+                               const qsvd_up_weight *U_q, const qsvd_up_weight *U_k, const qsvd_up_weight *U_v,
+                               int32_t H, int32_t dh, float softmax_scale, float *O, void *workspace,
+                               size_t workspace_bytes, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if ((st = check_cache(cache))) return st;
+    if (!seq_len || !U_q || !U_k || !U_v || !O) return fail(QSVD_EINVAL, "decode_attn_qu: null pointer");
+    if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "decode_attn_qu: dh must be 64 or 128");
+    if (H <= 0) return fail(QSVD_EINVAL, "decode_attn_qu: H must be positive");
+    if (cache->r > 3072 || cache->r % 32) return fail(QSVD_EUNSUPPORTED, "decode_attn_qu: need r %% 32 == 0 and r <= 3072");
+    if ((H * dh) % 256 || H * dh > 6144) return fail(QSVD_EUNSUPPORTED, "decode_attn_qu: need H*dh %% 256 == 0 and H*dh <= 6144");
+    if (max_seq_len < 1 || max_seq_len > cache->Tmax) return fail(QSVD_EINVAL, "decode_attn_qu: max_seq_len outside [1, Tmax]");
+    const qsvd_up_weight *Us[3] = {U_q, U_k, U_v};
+    for (const qsvd_up_weight *u : Us) {
+        if (!u->codes || !u->scale) return fail(QSVD_EINVAL, "decode_attn_qu: null weight pointer");
+        if (u->bits != 8 && u->bits != 4) return fail(QSVD_EINVAL, "decode_attn_qu: weight bits must be 8 or 4");
+        if (u->r != cache->r || u->d != H * dh) return fail(QSVD_EINVAL, "decode_attn_qu: weight shape differs from [r, H*dh]");
+        if (!aligned16(u->codes) || !aligned16(u->scale)) return fail(QSVD_EINVAL, "decode_attn_qu: pointers must be 16-byte aligned");
+    }
+    if (!aligned16(O) || (workspace && !aligned16(workspace)))
+        return fail(QSVD_EINVAL, "decode_attn_qu: pointers must be 16-byte aligned");
+    const size_t need = qsvd_decode_workspace_bytes(cache->B, max_seq_len, cache->r, H, dh);
+    if (!workspace || workspace_bytes < need)
+        return fail(QSVD_ENOSPC, "decode_attn_qu: workspace needs %zu bytes", need);
+    DecodeArgs a{view(cache), seq_len, max_seq_len, UpW{U_q->codes, U_q->scale, U_q->bits},
+                 UpW{U_k->codes, U_k->scale, U_k->bits}, UpW{U_v->codes, U_v->scale, U_v->bits}, H, dh,
+                 softmax_scale, O};
+    prof_mark(stream, "begin");
+    const cudaError_t e = launch_decode(a, workspace, workspace_bytes, err, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "decode_attn_qu launch");
 }
 
 // Rows of one prefill group: the largest power of two up to kPrefillMaxRows
@@ -475,7 +563,8 @@ int qsvd_latent_prefill_attn(const qsvd_cache *cache, const int32_t *q_seq, cons
         CacheView v = view(cache);
         v.B = int(std::min<int64_t>(rows, n - i0));
         v.seq_map = q_seq + i0;
-        DecodeArgs a{v, q_len + i0, max_len, U_q, U_k, U_v, H, dh, softmax_scale, O + size_t(i0) * d};
+        DecodeArgs a{v, q_len + i0, max_len, UpW{U_q, nullptr, 16}, UpW{U_k, nullptr, 16}, UpW{U_v, nullptr, 16},
+                     H, dh, softmax_scale, O + size_t(i0) * d};
         const cudaError_t e = launch_decode(a, workspace, workspace_bytes, err, stream);
         if (e != cudaSuccess) return cuda_fail(e, "prefill_attn launch");
     }
@@ -527,7 +616,7 @@ int qsvd_prefill_weights(const uint16_t *U_q, const uint16_t *U_k, const uint16_
     for (const void *p : ptrs)
         if (!aligned16(p)) return fail(QSVD_EINVAL, "prefill_weights: pointers must be 16-byte aligned");
     prof_mark(stream, "begin");
-    const cudaError_t e = launch_prefill_weights(U_q, U_k, U_v, r, d, Ut, stream);
+    const cudaError_t e = launch_prefill_weights(U_q, U_k, U_v, r, d, Ut, err, stream);
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "prefill_weights launch");
 }
 
@@ -626,6 +715,8 @@ int qsvd_decode_step(const qsvd_down_weight *W, const uint16_t *X, const qsvd_ca
     if (!W || !W->codes || !W->scale || !X || !seq_len || !U_q || !U_k || !U_v || !O)
         return fail(QSVD_EINVAL, "decode_step: null pointer");
     if (W->rot) return fail(QSVD_EUNSUPPORTED, "decode_step: rotated weights (W->rot) need qsvd_latent_project");
+    if ((W->w_bits && W->w_bits != 8) || (W->x_bits && W->x_bits != 8))
+        return fail(QSVD_EUNSUPPORTED, "decode_step: 4-bit settings (W->w_bits, W->x_bits) need qsvd_latent_project");
     const int d = W->d, r = W->r;
     if (r != cache->r) return fail(QSVD_EINVAL, "decode_step: weight rank differs from the cache's");
     if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "decode_step: dh must be 64 or 128");

@@ -48,7 +48,7 @@ struct Params {
     CacheView c;
     const int32_t *seq_len;
     const float *qt;              // [B, H, r]
-    const unsigned *qmax;         // [B, H] bits of max |q~|
+    const unsigned *qmax;         // [B, H] bits of max |q~|, or null: formed from q~ (r <= 2048)
     int H, TS, n_sub, n_split;     // sub-tile tokens, sub-tiles per split, splits per sequence
     float softmax_scale;
     float *pm, *pl, *po;          // [B, n_split, H] / [B, n_split, H, r]
@@ -124,6 +124,7 @@ attn_mma_kernel(const am::Params p) {
     __shared__ float qfac_s[kHG];
     __shared__ float m_s[kHG];
     __shared__ float alpha_s[kHG];                  // o_lat rescale of the current sub-tile
+    __shared__ unsigned hmax_s[kHG];                // per-head max |q~| (bits) when p.qmax is null
     const CacheView &c = p.c;
     const int r = c.r, TS = p.TS, H = p.H;
     const int split = blockIdx.x, b = blockIdx.y, h0 = blockIdx.z * kHG;
@@ -192,11 +193,26 @@ attn_mma_kernel(const am::Params p) {
             v[u] = (i < nq4 && h0 + hl < H) ? reinterpret_cast<const float4 *>(p.qt + (size_t(b) * H + h0 + hl) * r)[q4]
                                            : make_float4(0.f, 0.f, 0.f, 0.f);
         }
+        if (!p.qmax) {
+            // the per-head maxima from the loaded block itself (r <= 2048: one pass
+            // holds every channel of the CTA's heads), as non-negative float bits
+            if (threadIdx.x < kHG) hmax_s[threadIdx.x] = 0u;
+            __syncthreads();
+#pragma unroll
+            for (int u = 0; u < kQL; ++u) {
+                // a warp's 32 float4 belong to one head (r / 4 is a multiple of 32)
+                const int i = threadIdx.x + u * kThreads;
+                const float4 x = v[u];
+                const float mx = warp_max(fmaxf(fmaxf(fabsf(x.x), fabsf(x.y)), fmaxf(fabsf(x.z), fabsf(x.w))));
+                if (lane == 0 && i < nq4) atomicMax(&hmax_s[i / (r / 4)], __float_as_uint(mx));
+            }
+            __syncthreads();
+        }
         if (threadIdx.x < kHG) {
             const int h = h0 + threadIdx.x;
             int e = 0;
             if (h < H) {
-                const float m = __uint_as_float(p.qmax[size_t(b) * H + h]);
+                const float m = __uint_as_float(p.qmax ? p.qmax[size_t(b) * H + h] : hmax_s[threadIdx.x]);
                 if (m > 0.0f) frexpf(m, &e);
             }
             // scores -> logits in log2 units: undo the query scale, times softmax_scale * log2(e)

@@ -5,6 +5,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
+#include <cuda_fp8.h>
 
 #include "launch.h"
 
@@ -38,6 +39,31 @@ __device__ __forceinline__ void prefetch_share_l2(const void *base, size_t bytes
         prefetch_l2_bulk(c + o, uint32_t(len));
     }
 }
+
+// The fp32 at the same shared-memory offset in CTAs 0 .. 7 of the cluster,
+// as one instruction block so that the eight remote loads are in flight
+// together (the caller adds them in rank order).
+__device__ __forceinline__ void cluster_ld8(const void *p, float (&v)[8]) {
+    const uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(p));
+    asm volatile("{\n\t.reg .b32 a<8>;\n\t"
+                 "mapa.shared::cluster.u32 a0, %8, 0;\n\tmapa.shared::cluster.u32 a1, %8, 1;\n\t"
+                 "mapa.shared::cluster.u32 a2, %8, 2;\n\tmapa.shared::cluster.u32 a3, %8, 3;\n\t"
+                 "mapa.shared::cluster.u32 a4, %8, 4;\n\tmapa.shared::cluster.u32 a5, %8, 5;\n\t"
+                 "mapa.shared::cluster.u32 a6, %8, 6;\n\tmapa.shared::cluster.u32 a7, %8, 7;\n\t"
+                 "ld.shared::cluster.f32 %0, [a0];\n\tld.shared::cluster.f32 %1, [a1];\n\t"
+                 "ld.shared::cluster.f32 %2, [a2];\n\tld.shared::cluster.f32 %3, [a3];\n\t"
+                 "ld.shared::cluster.f32 %4, [a4];\n\tld.shared::cluster.f32 %5, [a5];\n\t"
+                 "ld.shared::cluster.f32 %6, [a6];\n\tld.shared::cluster.f32 %7, [a7];\n\t}"
+                 : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]), "=f"(v[7])
+                 : "r"(a)
+                 : "memory");
+}
+// Split cluster barrier: arrive (release this CTA's earlier accesses) now,
+// wait (acquire) later, so work in between overlaps the peers' arrival.
+__device__ __forceinline__ void cluster_arrive() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
 __device__ __forceinline__ void flag_error(int *err, int bit) {
     if (err) atomicOr(err, bit);
@@ -103,6 +129,10 @@ __device__ __forceinline__ void unpack8_bf16(const uint4 &v, float (&f)[8]) {
 // bf16 bit pattern of a small integer (|c| <= 255 is exact in bf16).
 __device__ __forceinline__ uint16_t int_to_bf16_bits(int c) {
     return uint16_t(__float_as_uint(float(c)) >> 16);
+}
+// fp8 e4m3 byte of a small integer (|c| <= 16 is exact in e4m3: 3 mantissa bits).
+__device__ __forceinline__ uint8_t int_to_e4m3(int c) {
+    return uint8_t(__nv_cvt_float_to_fp8(float(c), __NV_SATFINITE, __NV_E4M3));
 }
 
 // ---------------------------------------------------------------------------

@@ -27,7 +27,7 @@ namespace qsvd {
 namespace {
 
 constexpr int kBC = 16;          // largest NB
-constexpr int kCl = 8;           // CTAs per cluster (split of the r latent rows)
+constexpr int kCl = 8;           // CTAs per cluster (split of the r latent rows; cluster_ld8 reads 8 ranks)
 constexpr int kQaRows = 32;      // U_k rows per qabsorb CTA (one per lane)
 constexpr int kMaxSplitsG = 64;  // softmax partials per sequence
 
@@ -38,14 +38,6 @@ __device__ __forceinline__ uint32_t cl_rank() {
 }
 __device__ __forceinline__ void cl_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-// Load a float from the same shared-memory offset in CTA `rank` of the cluster.
-__device__ __forceinline__ float ld_rank(const float *p, uint32_t rank) {
-    uint32_t a;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_addr(p)), "r"(rank));
-    float v;
-    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
-    return v;
 }
 __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
     asm volatile(
@@ -67,6 +59,71 @@ __device__ __forceinline__ bool len_ok(int L, int Tmax) { return L >= 1 && L <= 
 // Rows of a weight tile per TMA box (box dimensions are at most 256).
 __host__ __device__ __forceinline__ int box_rows(int rs) { return rs / ((rs + 255) / 256); }
 
+// Up-projection weights are read in one of three formats (WB = bits per
+// weight): 16 = bf16 values; 8 = int8 codes; 4 = packed int4 codes (element
+// 2i in the low nibble of byte i, two's complement).  The codes of Eq. 11's
+// Q(W^u) have one fp32 scale per output channel, applied by the kernels to
+// the products' inputs or outputs.  The conversions below are exact: an int8
+// byte b placed in the mantissa of 2^23 gives 2^23 + (b ^ 0x80) as an fp32,
+// and subtracting 2^23 + 128 leaves the code; a nibble likewise with 2^23 + 8.
+__device__ __forceinline__ float i8_byte(uint32_t u, int k) {       // u = word ^ 0x80808080
+    return __uint_as_float(__byte_perm(u, 0x4B000000u, uint32_t(k) | (4u << 4) | (5u << 8) | (7u << 12))) -
+           8388736.0f;
+}
+__device__ __forceinline__ float i4_nib(uint32_t x, int k) {        // x = word ^ 0x88888888
+    return __uint_as_float(((x >> (4 * k)) & 0xFu) | 0x4B000000u) - 8388616.0f;
+}
+// Four consecutive weights of a tile row, starting at weight 4 * q4.
+template <int WB>
+__device__ __forceinline__ void load_w4(const uint8_t *row, int q4, float (&u)[4]) {
+    if (WB == 16) {
+        const uint2 w2 = *reinterpret_cast<const uint2 *>(row + 8 * q4);
+        u[0] = bf16_lo(w2.x); u[1] = bf16_hi(w2.x); u[2] = bf16_lo(w2.y); u[3] = bf16_hi(w2.y);
+    } else if (WB == 8) {
+        const uint32_t x = *reinterpret_cast<const uint32_t *>(row + 4 * q4) ^ 0x80808080u;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) u[e] = i8_byte(x, e);
+    } else {
+        const uint32_t x = uint32_t(*reinterpret_cast<const uint16_t *>(row + 2 * q4)) ^ 0x8888u;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) u[e] = i4_nib(x, e);
+    }
+}
+// Weight `col` of a tile row.
+template <int WB>
+__device__ __forceinline__ float load_w1(const uint8_t *row, int col) {
+    if (WB == 16) return bf16_to_f32(reinterpret_cast<const uint16_t *>(row)[col]);
+    if (WB == 8) return float(int8_t(row[col]));
+    const int b = (row[col >> 1] >> (4 * (col & 1))) & 0xF;
+    return float((b ^ 8) - 8);
+}
+// The 128 / WB weights held in 16 bytes.
+template <int WB>
+__device__ __forceinline__ void unpack16B(const uint4 &v, float (&f)[128 / WB]) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    if (WB == 16) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            f[2 * k] = bf16_lo(w[k]);
+            f[2 * k + 1] = bf16_hi(w[k]);
+        }
+    } else if (WB == 8) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t x = w[k] ^ 0x80808080u;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) f[4 * k + e] = i8_byte(x, e);
+        }
+    } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t x = w[k] ^ 0x88888888u;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) f[8 * k + e] = i4_nib(x, e);
+        }
+    }
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -77,24 +134,25 @@ __host__ __device__ __forceinline__ int box_rows(int rs) { return rs / ((rs + 25
 // shared memory, then rank k adds the kCl partials of columns
 // [k ncol/kCl, (k+1) ncol/kCl) in rank order.  CTA (0, 0) also clears qmax.
 // ---------------------------------------------------------------------------
-template <int NB>
+template <int NB, int WB>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
-qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restrict__ Uq, CacheView c,
-             const int32_t *__restrict__ seq_len, int B, int d, int ncol, float *__restrict__ q,
+qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint8_t *__restrict__ Uq, const float *__restrict__ sq,
+             CacheView c, const int32_t *__restrict__ seq_len, int B, int d, int ncol, float *__restrict__ q,
              unsigned *__restrict__ qmax, int n_qmax, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ int L_s[NB], Q_s[NB];   // length and cache sequence of each row
     const int r = c.r, rs = r / kCl, br = box_rows(rs);
     const int ncq = ncol / 4, G = 256 / ncq, rpg = rs / G;
+    const int rb = ncol * WB / 8;                                                // tile row bytes
     const uint32_t rank = cl_rank();
     const int c0 = blockIdx.y * ncol, j0 = int(rank) * rs;
-    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                          // [rs][ncol] bf16
-    float *c_s = reinterpret_cast<float *>(smem + size_t(rs) * ncol * 2);        // [NB][rs]
+    uint8_t *u_s = smem;                                                         // [rs][rb] weight codes
+    float *c_s = reinterpret_cast<float *>(smem + size_t(rs) * rb);              // [NB][rs]
     float *part = c_s + NB * rs;                                                 // [G][NB][ncol]
     const int tid = threadIdx.x;
     if (tid == 0) {
-        for (int k = 0; k < rs / br; ++k) tma_prefetch(&map_u, c0, j0 + k * br);
+        for (int k = 0; k < rs / br; ++k) tma_prefetch(&map_u, WB == 16 ? c0 : c0 * WB / 8, j0 + k * br);
         mbar_init(&bar, 1);
         mbar_init_fence();
     }
@@ -103,9 +161,9 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
     // rows: cheaper than bulk or tensor copies of 512-byte rows).  The weights
     // are no kernel's output, so the copies start before the wait on the
     // producer grid and overlap its tail.
-    for (int i = tid; i < rs * (ncol / 8); i += blockDim.x) {
-        const int row = i / (ncol / 8), k = i - row * (ncol / 8);
-        cp_async16(u_s + size_t(row) * ncol + 8 * k, Uq + size_t(j0 + row) * d + c0 + 8 * k);
+    for (int i = tid; i < rs * (rb / 16); i += blockDim.x) {
+        const int row = i / (rb / 16), k = i - row * (rb / 16);
+        cp_async16(u_s + size_t(row) * rb + 16 * k, Uq + (size_t(j0 + row) * d + c0) * WB / 8 + 16 * k);
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
@@ -190,10 +248,7 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
         for (; i + 4 <= i1; i += 4) {
             float u[4][4];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const uint2 w2 = *reinterpret_cast<const uint2 *>(u_s + size_t(i + k) * ncol + 4 * cq);
-                u[k][0] = bf16_lo(w2.x); u[k][1] = bf16_hi(w2.x); u[k][2] = bf16_lo(w2.y); u[k][3] = bf16_hi(w2.y);
-            }
+            for (int k = 0; k < 4; ++k) load_w4<WB>(u_s + size_t(i + k) * rb, cq, u[k]);
 #pragma unroll
             for (int bi = 0; bi < NB; ++bi) {
                 const float4 cv = *reinterpret_cast<const float4 *>(c_s + bi * rs + i);
@@ -203,8 +258,9 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
             }
         }
         for (; i < i1; ++i) {                          // rows left over when rpg % 4 != 0
-            const uint2 w2 = *reinterpret_cast<const uint2 *>(u_s + size_t(i) * ncol + 4 * cq);
-            const float u0 = bf16_lo(w2.x), u1 = bf16_hi(w2.x), u2 = bf16_lo(w2.y), u3 = bf16_hi(w2.y);
+            float u4[4];
+            load_w4<WB>(u_s + size_t(i) * rb, cq, u4);
+            const float u0 = u4[0], u1 = u4[1], u2 = u4[2], u3 = u4[3];
 #pragma unroll
             for (int bi = 0; bi < NB; ++bi) {
                 const float cv = c_s[bi * rs + i];
@@ -227,9 +283,12 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
         cl_sync();                                   // every rank's partials are complete
         for (int o = tid; o < nb * per_rank; o += blockDim.x) {
             const int bi = o / per_rank, col = int(rank) * per_rank + (o - bi * per_rank);
+            float pk[kCl];
+            cluster_ld8(part + bi * ncol + col, pk);
             float v = 0.0f;
 #pragma unroll
-            for (int k = 0; k < kCl; ++k) v += ld_rank(part + bi * ncol + col, uint32_t(k));
+            for (int k = 0; k < kCl; ++k) v += pk[k];       // rank order
+            if (WB != 16) v *= sq[c0 + col];         // per-output-channel scale of Q(U_q)
             q[size_t(b0 + bi) * d + c0 + col] = v;
         }
         cl_sync();                                   // partials read before they are overwritten / the CTA exits
@@ -241,32 +300,34 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint16_t *__restri
 // of U_k, warp = head.  The head block of the 32 rows sits in shared memory
 // with rows padded by 16 bytes (conflict-free 16-byte reads).
 // ---------------------------------------------------------------------------
-template <int NB>
+template <int NB, int WB>
 __global__ void __launch_bounds__(256)
-qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int B, int r, int d, int H, int dh,
-               int hg, float *__restrict__ qt, unsigned *__restrict__ qmax, int *err) {
+qabsorb_kernel(const float *__restrict__ q, const uint8_t *__restrict__ Uk, const float *__restrict__ sk, int B, int r,
+               int d, int H, int dh, int hg, float *__restrict__ qt, unsigned *__restrict__ qmax, int *err) {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar;
-    const int ustride = hg * dh + 8;                                             // bf16 per padded row
-    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                          // [32][ustride]
-    float *q_s = reinterpret_cast<float *>(smem + size_t(kQaRows) * ustride * 2); // [NB][hg * dh]
+    const int w = hg * dh;
+    const int wb = w * WB / 8;                                                   // weight bytes per row
+    const int ustride = wb + 16;                                                 // bytes per padded row
+    uint8_t *u_s = smem;                                                         // [32][ustride]
+    float *q_s = reinterpret_cast<float *>(smem + size_t(kQaRows) * ustride);    // [NB][hg * dh]
     const int j0 = blockIdx.x * kQaRows, h0 = blockIdx.y * hg;
     const int rows = min(kQaRows, r - j0);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int w = hg * dh;
     if (threadIdx.x < 32)
         for (int i = lane; i < rows; i += 32)
-            prefetch_l2_bulk(Uk + size_t(j0 + i) * d + size_t(h0) * dh, uint32_t(w) * 2);
+            prefetch_l2_bulk(Uk + (size_t(j0 + i) * d + size_t(h0) * dh) * WB / 8, uint32_t(wb));
     if (threadIdx.x == 0) {
         mbar_init(&bar, 1);
         mbar_init_fence();
     }
     __syncthreads();
     if (warp == 0) {            // U_k rows: no kernel's output, copied before the wait on the producer grid
-        if (lane == 0) mbar_arrive_expect_tx(&bar, uint32_t(rows) * w * 2);
+        if (lane == 0) mbar_arrive_expect_tx(&bar, uint32_t(rows) * wb);
         __syncwarp();
         for (int i = lane; i < rows; i += 32)
-            bulk_g2s(u_s + size_t(i) * ustride, Uk + size_t(j0 + i) * d + size_t(h0) * dh, uint32_t(w) * 2, &bar);
+            bulk_g2s(u_s + size_t(i) * ustride, Uk + (size_t(j0 + i) * d + size_t(h0) * dh) * WB / 8, uint32_t(wb),
+                     &bar);
     }
     pdl_wait();
     pdl_trigger();   // after the wait: the attention kernel two launches on reads the
@@ -292,7 +353,15 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
 #pragma unroll
             for (int k = 0; k < NB; ++k) {
                 const int idx = threadIdx.x + k * blockDim.x;
-                if (idx < n4) reinterpret_cast<float4 *>(q_s)[idx] = v[k];
+                if (idx < n4) {
+                    float4 x = v[k];
+                    if (WB != 16) {     // Q(U_k)'s per-output-channel scales fold into q
+                        const int c4 = idx % (w / 4);
+                        const float4 sc = reinterpret_cast<const float4 *>(sk + size_t(h0) * dh)[c4];
+                        x.x *= sc.x; x.y *= sc.y; x.z *= sc.z; x.w *= sc.w;
+                    }
+                    reinterpret_cast<float4 *>(q_s)[idx] = x;
+                }
             }
         }
         __syncthreads();
@@ -303,18 +372,21 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
         float acc[NB];
 #pragma unroll
         for (int bi = 0; bi < NB; ++bi) acc[bi] = 0.0f;
-        const uint16_t *urow = u_s + size_t(lane) * ustride + warp * dh;
-        for (int i = 0; i < dh; i += 8) {
-            float f[8];
-            unpack8_bf16(*reinterpret_cast<const uint4 *>(urow + i), f);
+        const uint8_t *urow = u_s + size_t(lane) * ustride + size_t(warp) * dh * WB / 8;
+        constexpr int kStep = 128 / WB;                  // weights per 16-byte read
+        for (int i = 0; i < dh; i += kStep) {
+            float f[kStep];
+            unpack16B<WB>(*reinterpret_cast<const uint4 *>(urow + i * WB / 8), f);
 #pragma unroll
             for (int bi = 0; bi < NB; ++bi) {
                 if (bi >= nb) break;
-                const float4 qa = *reinterpret_cast<const float4 *>(q_s + bi * w + warp * dh + i);
-                const float4 qb = *reinterpret_cast<const float4 *>(q_s + bi * w + warp * dh + i + 4);
                 float a = acc[bi];
-                a = fmaf(f[0], qa.x, a); a = fmaf(f[1], qa.y, a); a = fmaf(f[2], qa.z, a); a = fmaf(f[3], qa.w, a);
-                a = fmaf(f[4], qb.x, a); a = fmaf(f[5], qb.y, a); a = fmaf(f[6], qb.z, a); a = fmaf(f[7], qb.w, a);
+#pragma unroll
+                for (int e = 0; e < kStep; e += 4) {
+                    const float4 qa = *reinterpret_cast<const float4 *>(q_s + bi * w + warp * dh + i + e);
+                    a = fmaf(f[e], qa.x, a); a = fmaf(f[e + 1], qa.y, a);
+                    a = fmaf(f[e + 2], qa.z, a); a = fmaf(f[e + 3], qa.w, a);
+                }
                 acc[bi] = a;
             }
         }
@@ -336,9 +408,9 @@ qabsorb_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int
 // of U_v[:, h-block], and rank k adds the kCl products for its share of the
 // dh output columns in rank order.
 // ---------------------------------------------------------------------------
-template <int NB>
+template <int NB, int WB>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
-combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__restrict__ Uv,
+combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint8_t *__restrict__ Uv, const float *__restrict__ sv,
                   const int32_t *__restrict__ seq_len, const int32_t *__restrict__ seq_map, int nseq, int B, int Tmax,
                   int H, int dh, int r, int chunk, int n_split, const float *__restrict__ pm,
                   const float *__restrict__ pl, const float *__restrict__ po, float *__restrict__ O, int *err) {
@@ -352,19 +424,20 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__r
     const int j0 = int(rank) * rs;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nsub = 256 / dh;
-    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                          // [rs][dh] bf16
-    float *ol_s = reinterpret_cast<float *>(smem + size_t(rs) * dh * 2);         // [NB][rs]
+    const int rb = dh * WB / 8;                                                  // tile row bytes
+    uint8_t *u_s = smem;                                                         // [rs][rb] weight codes
+    float *ol_s = reinterpret_cast<float *>(smem + size_t(rs) * rb);             // [NB][rs]
     float *p_s = ol_s + NB * rs;                                                 // [nsub][NB][dh]
     pdl_trigger();
     if (tid == 0) {
-        for (int k = 0; k < rs / br; ++k) tma_prefetch(&map_v, h * dh, j0 + k * br);
+        for (int k = 0; k < rs / br; ++k) tma_prefetch(&map_v, WB == 16 ? h * dh : h * rb, j0 + k * br);
         mbar_init(&bar, 1);
         mbar_init_fence();
     }
     __syncthreads();
-    for (int i = tid; i < rs * (dh / 8); i += blockDim.x) {     // the U_v tile, 16-byte asynchronous copies
-        const int row = i / (dh / 8), k = i - row * (dh / 8);   // (before the wait: no kernel writes U_v)
-        cp_async16(u_s + size_t(row) * dh + 8 * k, Uv + size_t(j0 + row) * d + size_t(h) * dh + 8 * k);
+    for (int i = tid; i < rs * (rb / 16); i += blockDim.x) {    // the U_v tile, 16-byte asynchronous copies
+        const int row = i / (rb / 16), k = i - row * (rb / 16); // (before the wait: no kernel writes U_v)
+        cp_async16(u_s + size_t(row) * rb + 16 * k, Uv + (size_t(j0 + row) * d + size_t(h) * dh) * WB / 8 + 16 * k);
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
@@ -467,8 +540,8 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__r
 #pragma unroll
         for (int bi = 0; bi < NB; ++bi) acc[bi] = 0.0f;
         for (int i = 4 * sub; i < rs; i += 4 * nsub) {
-            const float u0 = bf16_to_f32(u_s[size_t(i) * dh + col]), u1 = bf16_to_f32(u_s[size_t(i + 1) * dh + col]);
-            const float u2 = bf16_to_f32(u_s[size_t(i + 2) * dh + col]), u3 = bf16_to_f32(u_s[size_t(i + 3) * dh + col]);
+            const float u0 = load_w1<WB>(u_s + size_t(i) * rb, col), u1 = load_w1<WB>(u_s + size_t(i + 1) * rb, col);
+            const float u2 = load_w1<WB>(u_s + size_t(i + 2) * rb, col), u3 = load_w1<WB>(u_s + size_t(i + 3) * rb, col);
 #pragma unroll
             for (int bi = 0; bi < NB; ++bi) {
                 const float4 o = *reinterpret_cast<const float4 *>(ol_s + bi * rs + i);
@@ -486,9 +559,12 @@ combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint16_t *__r
         cl_sync();                                   // every rank's products are complete
         for (int o = tid; o < nb * per_rank; o += blockDim.x) {
             const int bi = o / per_rank, cc = int(rank) * per_rank + (o - bi * per_rank);
+            float pk[kCl];
+            cluster_ld8(p_s + bi * dh + cc, pk);
             float v = 0.0f;
 #pragma unroll
-            for (int k = 0; k < kCl; ++k) v += ld_rank(p_s + bi * dh + cc, uint32_t(k));
+            for (int k = 0; k < kCl; ++k) v += pk[k];       // rank order
+            if (WB != 16) v *= sv[size_t(h) * dh + cc];     // per-output-channel scale of Q(U_v)
             O[size_t(b0 + bi) * d + size_t(h) * dh + cc] = v;
         }
         cl_sync();
@@ -513,92 +589,121 @@ int pass_nb(int B) {
     return nb;
 }
 
-template <int NB>
-cudaError_t qproj_nb(const CUtensorMap &map, const uint16_t *Uq, const CacheView &c, const int32_t *seq_len, int d, float *q,
+template <int NB, int WB>
+cudaError_t qproj_nb(const CUtensorMap &map, const UpW &Uq, const CacheView &c, const int32_t *seq_len, int d, float *q,
                      unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
     const int rs = c.r / kCl, ncol = qproj_cols(c.r), G = 256 / (ncol / 4);
-    const size_t smem = size_t(rs) * ncol * 2 + size_t(NB) * rs * 4 + size_t(G) * NB * ncol * 4;
-    cudaError_t e = ensure_smem(qproj_kernel<NB>, smem);
+    const size_t smem = size_t(rs) * ncol * WB / 8 + size_t(NB) * rs * 4 + size_t(G) * NB * ncol * 4;
+    cudaError_t e = ensure_smem(qproj_kernel<NB, WB>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(qproj_kernel<NB>, dim3(kCl, d / ncol), dim3(256), smem, s, map, Uq, c, seq_len, c.B, d, ncol, q,
-                      qmax, n_qmax, err);
+    return launch_pdl(qproj_kernel<NB, WB>, dim3(kCl, d / ncol), dim3(256), smem, s, map,
+                      static_cast<const uint8_t *>(Uq.w), Uq.scale, c, seq_len, c.B, d, ncol, q, qmax, n_qmax, err);
 }
 
-template <int NB>
-cudaError_t qabsorb_nb(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
+template <int NB, int WB>
+cudaError_t qabsorb_nb(const float *q, const UpW &Uk, int B, int r, int d, int H, int dh, float *qt,
                        unsigned *qmax, int *err, cudaStream_t s) {
     const int hg = qabsorb_hg(H);
-    const size_t smem = size_t(kQaRows) * (hg * dh + 8) * 2 + size_t(NB) * hg * dh * 4;
-    cudaError_t e = ensure_smem(qabsorb_kernel<NB>, smem);
+    const size_t smem = size_t(kQaRows) * (size_t(hg) * dh * WB / 8 + 16) + size_t(NB) * hg * dh * 4;
+    cudaError_t e = ensure_smem(qabsorb_kernel<NB, WB>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(qabsorb_kernel<NB>, dim3((r + kQaRows - 1) / kQaRows, H / hg), dim3(32 * hg), smem, s, q, Uk,
-                      B, r, d, H, dh, hg, qt, qmax, err);
+    return launch_pdl(qabsorb_kernel<NB, WB>, dim3((r + kQaRows - 1) / kQaRows, H / hg), dim3(32 * hg), smem, s, q,
+                      static_cast<const uint8_t *>(Uk.w), Uk.scale, B, r, d, H, dh, hg, qt, qmax, err);
 }
 
-template <int NB>
-cudaError_t combine_nb(const CUtensorMap &map, const uint16_t *Uv, const int32_t *seq_len, const int32_t *seq_map,
+template <int NB, int WB>
+cudaError_t combine_nb(const CUtensorMap &map, const UpW &Uv, const int32_t *seq_len, const int32_t *seq_map,
                        int nseq, int B, int Tmax, int H, int dh, int r,
                        int chunk, int n_split, const float *pm, const float *pl, const float *po, float *O, int *err,
                        cudaStream_t s) {
     const int rs = r / kCl;
-    const size_t smem = size_t(rs) * dh * 2 + size_t(NB) * rs * 4 + size_t(256 / dh) * NB * dh * 4;
-    cudaError_t e = ensure_smem(combine_uv_kernel<NB>, smem);
+    const size_t smem = size_t(rs) * dh * WB / 8 + size_t(NB) * rs * 4 + size_t(256 / dh) * NB * dh * 4;
+    cudaError_t e = ensure_smem(combine_uv_kernel<NB, WB>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(combine_uv_kernel<NB>, dim3(kCl, H), dim3(256), smem, s, map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r,
-                      chunk, n_split, pm, pl, po, O, err);
+    return launch_pdl(combine_uv_kernel<NB, WB>, dim3(kCl, H), dim3(256), smem, s, map,
+                      static_cast<const uint8_t *>(Uv.w), Uv.scale, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk,
+                      n_split, pm, pl, po, O, err);
 }
+
+// Tensor map over an up-projection [r, d] for the L2 prefetch of a CTA's
+// tile: bf16 elements, or the bytes of the int8 / int4 codes.
+bool up_map(CUtensorMap *map, const UpW &U, int r, int d, int box_cols, int box_r) {
+    if (U.bits == 16)
+        return encode_map_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, U.w, uint64_t(d), uint64_t(r), uint64_t(d) * 2,
+                             uint32_t(box_cols), uint32_t(box_r), CU_TENSOR_MAP_SWIZZLE_NONE);
+    const uint64_t rowb = uint64_t(d) * U.bits / 8;
+    return encode_map_2d(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, U.w, rowb, uint64_t(r), rowb,
+                         uint32_t(box_cols * U.bits / 8), uint32_t(box_r), CU_TENSOR_MAP_SWIZZLE_NONE);
+}
+
+// Dispatch on the pass size NB (the batch rounded up to a power of two, at
+// most kBC) and the weight format.
+template <template <int, int> class F, typename... A>
+cudaError_t dispatch_nb_wb(int B, int bits, A &&...a) {
+    switch (bits) {
+        case 16:
+            switch (pass_nb(B)) {
+                case 1: return F<1, 16>::run(a...);
+                case 2: return F<2, 16>::run(a...);
+                case 4: return F<4, 16>::run(a...);
+                case 8: return F<8, 16>::run(a...);
+                default: return F<16, 16>::run(a...);
+            }
+        case 8:
+            switch (pass_nb(B)) {
+                case 1: return F<1, 8>::run(a...);
+                case 2: return F<2, 8>::run(a...);
+                case 4: return F<4, 8>::run(a...);
+                case 8: return F<8, 8>::run(a...);
+                default: return F<16, 8>::run(a...);
+            }
+        default:
+            switch (pass_nb(B)) {
+                case 1: return F<1, 4>::run(a...);
+                case 2: return F<2, 4>::run(a...);
+                case 4: return F<4, 4>::run(a...);
+                case 8: return F<8, 4>::run(a...);
+                default: return F<16, 4>::run(a...);
+            }
+    }
+}
+template <int NB, int WB> struct QprojF {
+    template <typename... A> static cudaError_t run(A &&...a) { return qproj_nb<NB, WB>(a...); }
+};
+template <int NB, int WB> struct QabsorbF {
+    template <typename... A> static cudaError_t run(A &&...a) { return qabsorb_nb<NB, WB>(a...); }
+};
+template <int NB, int WB> struct CombineF {
+    template <typename... A> static cudaError_t run(A &&...a) { return combine_nb<NB, WB>(a...); }
+};
 
 }  // namespace
 
-cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
+cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const UpW &Uq, int d, float *q,
                          unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
     const int rs = c.r / kCl, ncol = qproj_cols(c.r);
     CUtensorMap map;
-    if (!encode_map_2d(&map, CU_TENSOR_MAP_DATA_TYPE_UINT16, Uq, uint64_t(d), uint64_t(c.r), uint64_t(d) * 2,
-                       uint32_t(ncol), uint32_t(box_rows(rs)), CU_TENSOR_MAP_SWIZZLE_NONE))
-        return cudaErrorInvalidValue;
-    cudaError_t e;
-    switch (pass_nb(c.B)) {
-        case 1: e = qproj_nb<1>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-        case 2: e = qproj_nb<2>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-        case 4: e = qproj_nb<4>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-        case 8: e = qproj_nb<8>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-        default: e = qproj_nb<16>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s); break;
-    }
+    if (!up_map(&map, Uq, c.r, d, ncol, box_rows(rs))) return cudaErrorInvalidValue;
+    const cudaError_t e = dispatch_nb_wb<QprojF>(c.B, Uq.bits, map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s);
     prof_mark(s, "qproj");
     return e;
 }
 
-cudaError_t launch_qabsorb(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
+cudaError_t launch_qabsorb(const float *q, const UpW &Uk, int B, int r, int d, int H, int dh, float *qt,
                            unsigned *qmax, int *err, cudaStream_t s) {
-    cudaError_t e;
-    switch (pass_nb(B)) {
-        case 1: e = qabsorb_nb<1>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
-        case 2: e = qabsorb_nb<2>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
-        case 4: e = qabsorb_nb<4>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
-        case 8: e = qabsorb_nb<8>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
-        default: e = qabsorb_nb<16>(q, Uk, B, r, d, H, dh, qt, qmax, err, s); break;
-    }
+    const cudaError_t e = dispatch_nb_wb<QabsorbF>(B, Uk.bits, q, Uk, B, r, d, H, dh, qt, qmax, err, s);
     prof_mark(s, "qabsorb");
     return e;
 }
 
-cudaError_t launch_combine_uv(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
-                              const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
-                              int *err, cudaStream_t s) {
+cudaError_t launch_combine_uv(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh,
+                              int r, int chunk, int n_split, const float *pm, const float *pl, const float *po,
+                              const UpW &Uv, float *O, int *err, cudaStream_t s) {
     const int rs = r / kCl, d = H * dh;
     CUtensorMap map;
-    if (!encode_map_2d(&map, CU_TENSOR_MAP_DATA_TYPE_UINT16, Uv, uint64_t(d), uint64_t(r), uint64_t(d) * 2,
-                       uint32_t(dh), uint32_t(box_rows(rs)), CU_TENSOR_MAP_SWIZZLE_NONE))
-        return cudaErrorInvalidValue;
-    cudaError_t e;
-    switch (pass_nb(B)) {
-        case 1: e = combine_nb<1>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 2: e = combine_nb<2>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 4: e = combine_nb<4>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        case 8: e = combine_nb<8>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-        default: e = combine_nb<16>(map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk, n_split, pm, pl, po, O, err, s); break;
-    }
+    if (!up_map(&map, Uv, r, d, dh, box_rows(rs))) return cudaErrorInvalidValue;
+    const cudaError_t e = dispatch_nb_wb<CombineF>(B, Uv.bits, map, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r,
+                                                   chunk, n_split, pm, pl, po, O, err, s);
     prof_mark(s, "combine_uv");
     return e;
 }

@@ -306,12 +306,22 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
     DecodeWs w;
     carve(B, a.max_seq_len, r, H, dh, static_cast<char *>(ws), &w);
     // the up-projection products on the tensor cores from 8 sequences on
-    const bool mma = decode_mma_supported(B, r, d, dh);
-    cudaError_t e = mma ? launch_qproj_mma(c, a.seq_len, a.U_q, d, w.q, w.qmax, B * H, err, s)
-                        : launch_qproj(c, a.seq_len, a.U_q, d, w.q, w.qmax, B * H, err, s);
-    if (e != cudaSuccess) return e;
-    e = mma ? launch_qabsorb_mma(w.q, a.U_k, B, r, d, H, dh, w.qt, w.qmax, s)
-            : launch_qabsorb(w.q, a.U_k, B, r, d, H, dh, w.qt, w.qmax, err, s);
+    // (bf16 weights only: quantized up-projections take the CUDA-core forms at every batch size)
+    const bool bf16_up = a.U_q.bits == 16 && a.U_k.bits == 16 && a.U_v.bits == 16;
+    const bool mma = bf16_up && decode_mma_supported(B, r, d, dh);
+    cudaError_t e;
+    // the warp-level attention kernel can form the per-head maxima of q~ itself (r <= 2048)
+    const bool mma_attn = attn_mma_use(c, H, B, a.max_seq_len) && attn_mma_fits(c, a.max_seq_len);
+    const bool local_qmax = mma_attn && r <= 2048 && r % 128 == 0;
+    if (!mma && qfuse_use(c, a.U_q, a.U_k, H, dh)) {
+        e = launch_qfuse(c, a.seq_len, a.U_q, a.U_k, H, dh, w.qt, local_qmax ? nullptr : w.qmax, err, s);
+    } else {
+        e = mma ? launch_qproj_mma(c, a.seq_len, static_cast<const uint16_t *>(a.U_q.w), d, w.q, w.qmax, B * H, err, s)
+                : launch_qproj(c, a.seq_len, a.U_q, d, w.q, w.qmax, B * H, err, s);
+        if (e != cudaSuccess) return e;
+        e = mma ? launch_qabsorb_mma(w.q, static_cast<const uint16_t *>(a.U_k.w), B, r, d, H, dh, w.qt, w.qmax, s)
+                : launch_qabsorb(w.q, a.U_k, B, r, d, H, dh, w.qt, w.qmax, err, s);
+    }
     if (e != cudaSuccess) return e;
 
     int chunk = chunk_tokens(a.max_seq_len);
@@ -321,7 +331,9 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
         int ts = 16, n_sub = 1;
         ns = attn_mma_splits(c, B, H, a.max_seq_len, &ts, &n_sub);
         chunk = ts * n_sub;
-        e = launch_attn_mma(c, a.seq_len, w.qt, w.qmax, H, a.softmax_scale, ts, n_sub, ns, w.pm, w.pl, w.po, err, s);
+        const bool fused_q = !mma && qfuse_use(c, a.U_q, a.U_k, H, dh);
+        e = launch_attn_mma(c, a.seq_len, w.qt, fused_q && local_qmax ? nullptr : w.qmax, H, a.softmax_scale, ts,
+                            n_sub, ns, w.pm, w.pl, w.po, err, s);
         if (e != cudaSuccess) return e;
         prof_mark(s, "attn_mma");
     } else if (attn_tc_use(c, H, a.max_seq_len)) {
@@ -354,8 +366,11 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
         if (e != cudaSuccess) return e;
         prof_mark(s, "attn_chunk");
     }
-    if (mma) return launch_combine_mma(a.seq_len, c.seq_map, c.nseq, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v, a.O, s);
-    return launch_combine_uv(a.seq_len, c.seq_map, c.nseq, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v, a.O, err, s);
+    if (mma)
+        return launch_combine_mma(a.seq_len, c.seq_map, c.nseq, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po,
+                                  static_cast<const uint16_t *>(a.U_v.w), a.O, s);
+    return launch_combine_uv(a.seq_len, c.seq_map, c.nseq, B, c.Tmax, H, dh, r, chunk, ns, w.pm, w.pl, w.po, a.U_v,
+                             a.O, err, s);
 }
 
 }  // namespace qsvd

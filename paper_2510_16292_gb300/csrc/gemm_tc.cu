@@ -34,73 +34,34 @@
 
 #include "common.cuh"
 #include "launch.h"
+#include "tcgen05.cuh"
 
 namespace qsvd {
 
 constexpr int kBM = 128, kBK = 64;
+constexpr int kRowB = 128;                     // bytes of K per staged tile row (one 128-byte swizzle atom)
 constexpr int kChunkK = 1024;                  // <= 2^24 / 127^2 products per exact fp32 partial
-constexpr int kStageA = kBM * kBK * 2;         // 16 KiB
+constexpr int kStageA = kBM * kRowB;           // 16 KiB
 constexpr int kRingBytes = 192 * 1024;         // TMA ring (stages of A + B tiles)
 
-template <int BN> struct GemmCfg {
-    static constexpr int kStageB = BN * kBK * 2;
+// OPB: operand bits.  16: the codes as bf16 (kind::f16, K = 16 per MMA, 64 per
+// stage).  8: int4-valued codes as fp8 e4m3 (kind::f8f6f4, K = 32 per MMA,
+// 128 per stage); every |x w| <= 49, so a partial sum stays an exact fp32
+// integer for d < 2^24 / 49 and the accumulator is drained once at the end.
+template <int BN, int OPB = 16> struct GemmCfg {
+    static constexpr int kBKe = kRowB * 8 / OPB;      // K elements per stage
+    static constexpr int kStageB = BN * kRowB;
     static constexpr int kStages = kRingBytes / (kStageA + kStageB);
     static constexpr int kEpiWarps = BN / 32;
     static constexpr int kThreads = 64 + 32 * kEpiWarps;
     static constexpr size_t kSmem = size_t(kStages) * (kStageA + kStageB) + 1024;   // + alignment slack
-    // bf16 x bf16 -> f32, both K-major, M=128, N=BN
-    static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(BN >> 3) << 17) |
-                                       (uint32_t(kBM >> 4) << 24);
+    // f32 accumulator, A and B K-major, M=128, N=BN; bf16 x bf16 (kind::f16) or e4m3 x e4m3 (kind::f8f6f4)
+    static constexpr uint32_t kIdesc = (1u << 4) | (OPB == 16 ? (1u << 7) | (1u << 10) : 0u) |
+                                       (uint32_t(BN >> 3) << 17) | (uint32_t(kBM >> 4) << 24);
 };
 
-// ---------------------------------------------------------------------------
-// PTX wrappers
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y, uint64_t *bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
-        ::"r"(smem_addr(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
-        : "memory");
-}
-
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
-// 1024 bytes apart (the layout TMA's 128B swizzle writes for 64 bf16 per row).
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-    return uint64_t((saddr & 0x3FFFF) >> 4) | (uint64_t(1) << 16) | (uint64_t(1024 >> 4) << 32) |
-           (uint64_t(1) << 46) | (uint64_t(2) << 61);
-}
-
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
-    asm volatile("{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
-                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
-                 ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
-}
-// Spin on an mbarrier phase inline (no call), bounded; false on expiry.
-__device__ __forceinline__ bool spin_wait(uint64_t *bar, uint32_t parity, int *err) {
-    for (long i = 0; i < kWaitLimit; ++i)
-        if (mbar_try_wait(bar, parity)) return true;
-    return mbar_wait(bar, parity, err);     // flags the timeout, then a last bounded wait
-}
-__device__ __forceinline__ void umma_commit(uint64_t *bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
-                 ::"r"(smem_addr(bar)) : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// 32 consecutive columns of this warp's 32 lanes.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
-          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
-          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
-        : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// PTX wrappers: tcgen05.cuh (tc::); a spin on an mbarrier phase, bounded.
+__device__ __forceinline__ bool spin_wait(uint64_t *bar, uint32_t parity, int *err) { return tc::wait(bar, parity, err); }
 
 // ---------------------------------------------------------------------------
 // Destinations of the fused requantization (LAT != 0).
@@ -117,17 +78,17 @@ __device__ __forceinline__ uint32_t g_cluster_rank() {
     return r;
 }
 
-template <int BN, int LAT>
-__global__ void __launch_bounds__(GemmCfg<BN>::kThreads, 1)
+template <int BN, int LAT, int OPB>
+__global__ void __launch_bounds__(GemmCfg<BN, OPB>::kThreads, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_w, int64_t T, int d,
                int r, const float *__restrict__ xs, const float *__restrict__ ws, float *__restrict__ c_hat,
                int32_t *__restrict__ acc_out, const LatOut lo, int *err) {
-    using C = GemmCfg<BN>;
-    constexpr int kStages = C::kStages, kStageB = C::kStageB;
+    using C = GemmCfg<BN, OPB>;
+    constexpr int kStages = C::kStages, kStageB = C::kStageB, kBKe = C::kBKe;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *sA = smem;                                    // [kStages][128 x 64] bf16, SW128
-    uint8_t *sB = smem + size_t(kStages) * kStageA;        // [kStages][BN x 64] bf16, SW128
+    uint8_t *sA = smem;                                    // [kStages][128 x 128 B] SW128
+    uint8_t *sB = smem + size_t(kStages) * kStageA;        // [kStages][BN x 128 B] SW128
     __shared__ __align__(8) uint64_t full_bar[kStages], empty_bar[kStages];
     __shared__ __align__(8) uint64_t acc_full[2], acc_empty[2];
     __shared__ uint32_t tmem_base;
@@ -135,8 +96,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
     __shared__ float xmax[8][kBM];                         // per-row max of every CTA of the cluster (int8)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int m0 = blockIdx.y * kBM, n0 = blockIdx.x * BN;      // N fastest: a wave shares X tiles
-    const int n_k = d / kBK;
-    const int stages_per_chunk = kChunkK / kBK;
+    const int n_k = d / kBKe;
+    const int stages_per_chunk = OPB == 16 ? kChunkK / kBKe : n_k;
     const int n_chunks = (n_k + stages_per_chunk - 1) / stages_per_chunk;
 
     pdl_trigger();
@@ -158,9 +119,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
                      ::"r"(smem_addr(&tmem_base)), "r"(2 * BN));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
-    tc_fence_before();
+    tc::fence_before();
     __syncthreads();
-    tc_fence_after();
+    tc::fence_after();
     const uint32_t tmem = tmem_base;
     pdl_wait();
 
@@ -173,8 +134,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
                 const int s = i % kStages;
                 if (i >= kStages && !spin_wait(&empty_bar[s], ((i / kStages) - 1) & 1, err)) break;
                 mbar_arrive_expect_tx(&full_bar[s], kStageA + kStageB);
-                tma_load_2d(sA + size_t(s) * kStageA, &map_x, i * kBK, m0, &full_bar[s]);
-                tma_load_2d(sB + size_t(s) * kStageB, &map_w, i * kBK, n0, &full_bar[s]);
+                tc::tma_load_2d(sA + size_t(s) * kStageA, &map_x, i * kBKe, m0, &full_bar[s]);
+                tc::tma_load_2d(sB + size_t(s) * kStageB, &map_w, i * kBKe, n0, &full_bar[s]);
             }
         }
     } else if (warp == 1) {
@@ -185,7 +146,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
                 const int buf = c & 1;
                 if (c >= 2) {
                     ok = spin_wait(&acc_empty[buf], ((c >> 1) - 1) & 1, err);
-                    tc_fence_after();
+                    tc::fence_after();
                 }
                 const uint32_t d_tmem = tmem + uint32_t(buf * BN);
                 const int i0 = c * stages_per_chunk, i1 = min(n_k, i0 + stages_per_chunk);
@@ -193,16 +154,21 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
                     const int s = i % kStages;
                     ok = spin_wait(&full_bar[s], (i / kStages) & 1, err);
                     if (!ok) break;
-                    tc_fence_after();
+                    tc::fence_after();
                     const uint32_t a0 = smem_addr(sA + size_t(s) * kStageA);
                     const uint32_t b0 = smem_addr(sB + size_t(s) * kStageB);
 #pragma unroll
-                    for (int ks = 0; ks < kBK / 16; ++ks)
-                        umma_bf16(d_tmem, sw128_desc(a0 + ks * 32), sw128_desc(b0 + ks * 32), C::kIdesc,
-                                  (i > i0 || ks > 0) ? 1u : 0u);
-                    umma_commit(&empty_bar[s]);          // stage s may be refilled once these MMAs finish
+                    for (int ks = 0; ks < kRowB / 32; ++ks) {     // 32 bytes of K per MMA
+                        if (OPB == 16)
+                            tc::mma_ss(d_tmem, tc::desc_sw128(a0 + ks * 32), tc::desc_sw128(b0 + ks * 32), C::kIdesc,
+                                      (i > i0 || ks > 0) ? 1u : 0u);
+                        else
+                            tc::mma_ss_f8(d_tmem, tc::desc_sw128(a0 + ks * 32), tc::desc_sw128(b0 + ks * 32), C::kIdesc,
+                                    (i > i0 || ks > 0) ? 1u : 0u);
+                    }
+                    tc::commit(&empty_bar[s]);          // stage s may be refilled once these MMAs finish
                 }
-                if (ok) umma_commit(&acc_full[buf]);     // chunk c's partial sum is complete
+                if (ok) tc::commit(&acc_full[buf]);     // chunk c's partial sum is complete
             }
         }
     } else {
@@ -216,18 +182,18 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
         for (int c = 0; c < n_chunks && ok; ++c) {
             const int buf = c & 1;
             ok = spin_wait(&acc_full[buf], (c >> 1) & 1, err);
-            tc_fence_after();
+            tc::fence_after();
             if (!ok) break;
             const uint32_t taddr = tmem + (uint32_t(quad * 32) << 16) + uint32_t(buf * BN + col0);
 #pragma unroll
             for (int j0 = 0; j0 < 128; j0 += 32) {
                 uint32_t v[32];
-                tmem_ld32(taddr + j0, v);
-                tmem_ld_wait();
+                tc::tmem_ld32(taddr + j0, v);
+                tc::tmem_wait_ld();
 #pragma unroll
                 for (int j = 0; j < 32; ++j) acc[j0 + j] += __float2int_rn(__uint_as_float(v[j]));
             }
-            tc_fence_before();
+            tc::fence_before();
             __syncwarp();
             if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&acc_empty[buf])) : "memory");
         }
@@ -350,9 +316,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
             }
         }
     }
-    tc_fence_before();
+    tc::fence_before();
     __syncthreads();
-    tc_fence_after();
+    tc::fence_after();
     if (warp == 1)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * BN));
 }
@@ -360,36 +326,15 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant_
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
-typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-static EncodeTiledFn encode_fn() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &p, cudaEnableDefault, &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(p);
-    }
-    return fn;
+// Operand matrix [rows, cols] row-major (cols contiguous): bf16 (OPB 16) or
+// one byte per element (OPB 8), box [box_rows x 128 bytes], 128B swizzle.
+static bool make_map(CUtensorMap *map, const void *base, int64_t rows, int cols, int box_rows, int opb = 16) {
+    return encode_map_2d(map, opb == 16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, base,
+                         uint64_t(cols), uint64_t(rows), uint64_t(cols) * opb / 8, uint32_t(kRowB * 8 / opb),
+                         uint32_t(box_rows), CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
-// bf16 matrix [rows, cols] row-major (cols contiguous), box [box_rows x 64 cols], 128B swizzle.
-static bool make_map(CUtensorMap *map, const void *base, int64_t rows, int cols, int box_rows) {
-    EncodeTiledFn fn = encode_fn();
-    if (!fn) return false;
-    const cuuint64_t dims[2] = {cuuint64_t(cols), cuuint64_t(rows)};
-    const cuuint64_t strides[1] = {cuuint64_t(cols) * 2};
-    const cuuint32_t box[2] = {cuuint32_t(kBK), cuuint32_t(box_rows)};
-    const cuuint32_t estr[2] = {1, 1};
-    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-bool gemm_tc_supported(int d, int r) { return d % kBK == 0 && r % 128 == 0 && encode_fn() != nullptr; }
+bool gemm_tc_supported(int d, int r) { return d % kBK == 0 && r % 128 == 0 && tensor_maps_available(); }
 
 // Tile width and whether the per-token requantization can run in the epilogue:
 // int4 always; int8 when the r / BN CTAs of a row block fit one portable
@@ -404,14 +349,14 @@ static int pick_bn(int64_t T, int r, int lat_bits, bool *fuse) {
     return bn;
 }
 
-template <int BN, int LAT>
-static cudaError_t launch_bn(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
+template <int BN, int LAT, int OPB = 16>
+static cudaError_t launch_bn(const void *xq_op, int64_t T, int d, const void *w_op, const float *ws,
                              const float *xs, int r, float *c_hat, int32_t *acc_out, const LatOut &lo, int *err,
                              cudaStream_t s) {
-    using C = GemmCfg<BN>;
+    using C = GemmCfg<BN, OPB>;
     CUtensorMap mx, mw;
-    if (!make_map(&mx, xq_bf16, T, d, kBM) || !make_map(&mw, w_bf16, r, d, BN)) return cudaErrorInvalidValue;
-    cudaError_t e = ensure_smem(gemm_tc_kernel<BN, LAT>, C::kSmem);
+    if (!make_map(&mx, xq_op, T, d, kBM, OPB) || !make_map(&mw, w_op, r, d, BN, OPB)) return cudaErrorInvalidValue;
+    cudaError_t e = ensure_smem(gemm_tc_kernel<BN, LAT, OPB>, C::kSmem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(unsigned(r / BN), unsigned((T + kBM - 1) / kBM));
@@ -427,8 +372,8 @@ static cudaError_t launch_bn(const uint16_t *xq_bf16, int64_t T, int d, const ui
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = LAT == 8 ? 2 : 1;
-    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN, LAT>, mx, mw, T, d, r, xs, ws, c_hat, acc_out, lo, err);
-    prof_mark(s, "gemm_tc");
+    e = cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN, LAT, OPB>, mx, mw, T, d, r, xs, ws, c_hat, acc_out, lo, err);
+    prof_mark(s, OPB == 16 ? "gemm_tc" : "gemm_f8");
     return e;
 }
 
@@ -471,6 +416,30 @@ cudaError_t launch_gemm_tc_fused(const uint16_t *xq_bf16, int64_t T, int d, cons
                          : launch_bn<128, 8>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s);
     return bn == 256 ? launch_bn<256, 4>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s)
                      : launch_bn<128, 4>(xq_bf16, T, d, w_bf16, ws, xs, r, c_hat, acc_out, lo, err, s);
+}
+
+// W4A4: the same GEMM on fp8 e4m3 images of int4-valued codes (every value in
+// [-7, 7] is exact in e4m3), kind::f8f6f4; lat_bits 0 leaves the
+// requantization to a separate kernel (c_hat written).
+bool gemm_f8_supported(int d, int r) { return d % kRowB == 0 && r % 128 == 0 && d < (1 << 24) / 49 && tensor_maps_available(); }
+
+cudaError_t launch_gemm_f8(const uint8_t *xq_f8, int64_t T, int d, const uint8_t *w_f8, const float *ws,
+                           const float *xs, int r, int lat_bits, float lat_clip, void *lat_codes, void *lat_scales,
+                           const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, float *c_hat,
+                           int32_t *acc_out, int *err, cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    bool fuse = false;
+    const int bn = pick_bn(T, r, lat_bits, &fuse);
+    LatOut lo{lat_clip, lat_codes, lat_scales, dst ? *dst : CacheView{}, dst_seq, dst_pos};
+    if (lat_bits == 8 && fuse)
+        return bn == 256 ? launch_bn<256, 8, 8>(xq_f8, T, d, w_f8, ws, xs, r, c_hat, acc_out, lo, err, s)
+                         : launch_bn<128, 8, 8>(xq_f8, T, d, w_f8, ws, xs, r, c_hat, acc_out, lo, err, s);
+    if (lat_bits == 4)
+        return bn == 256 ? launch_bn<256, 4, 8>(xq_f8, T, d, w_f8, ws, xs, r, c_hat, acc_out, lo, err, s)
+                         : launch_bn<128, 4, 8>(xq_f8, T, d, w_f8, ws, xs, r, c_hat, acc_out, lo, err, s);
+    const LatOut none{};
+    return bn == 256 ? launch_bn<256, 0, 8>(xq_f8, T, d, w_f8, ws, xs, r, c_hat, acc_out, none, err, s)
+                     : launch_bn<128, 0, 8>(xq_f8, T, d, w_f8, ws, xs, r, c_hat, acc_out, none, err, s);
 }
 
 }  // namespace qsvd

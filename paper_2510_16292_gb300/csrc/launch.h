@@ -19,6 +19,8 @@ namespace qsvd {
 // the parameters.  Defined in api.cu.
 bool encode_map_2d(CUtensorMap *map, CUtensorMapDataType type, const void *base, uint64_t inner, uint64_t outer,
                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, CUtensorMapSwizzle swizzle);
+// Whether the driver's tensor-map encoder could be resolved (api.cu).
+bool tensor_maps_available();
 
 // Raise a kernel's dynamic shared memory limit to the maximum the first time
 // it needs more than the default (so that no attribute call happens while a
@@ -108,13 +110,22 @@ void prof_mark(cudaStream_t s, const char *label);
 
 // Per-token int8 quantization of X [T, d] bf16 (a1); rot > 0: of X H1^T,
 // H1 the block Hadamard rotation with blocks of rot channels (quant_kernels.cu).
+// qmax 127 (int8) or 7 (int4 codes, W4A4 / W8A4); xq_f8: optional fp8 e4m3 image of the codes.
 cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip,
-                          int8_t *xq, uint16_t *xq_bf16, float *xs, cudaStream_t s, int rot = 0);
+                          int8_t *xq, uint16_t *xq_bf16, float *xs, cudaStream_t s, int rot = 0, int qmax = 127,
+                          uint8_t *xq_f8 = nullptr);
 
 // Per-output-channel int8 RTN of W_d [d, r] fp32 -> codes [r, d] (+ bf16 image);
 // rot > 0: of H1 W_d.
+// qmax 127 (int8) or 7 (int4-valued codes); codes_f8: optional fp8 e4m3 image.
 cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int8_t *codes,
-                                   uint16_t *codes_bf16, float *scale, cudaStream_t s, int rot = 0);
+                                   uint16_t *codes_bf16, float *scale, cudaStream_t s, int rot = 0, int qmax = 127,
+                                   uint8_t *codes_f8 = nullptr);
+
+// Per-output-channel RTN of an up-projection U [r, d] bf16 (Eq. 11's Q(W^u)):
+// int8 codes [r, d] or packed int4 [r, d/2], fp32 scale [d]; d % 32 == 0.
+cudaError_t launch_quantize_up(const uint16_t *U, int r, int d, int bits, float clip, void *codes, float *scale,
+                               cudaStream_t s);
 
 // Exact int8 GEMM on the CUDA cores (dp4a) with the dequant epilogue (a2, a3 first half):
 // c_hat[t, j] = (fp32(acc) * xs[t]) * ws[j].
@@ -133,7 +144,7 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
                               int8_t *xq_out, float *xs_out, int32_t *acc_out, void *lat_codes, void *lat_scales,
                               const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
                               cudaStream_t s, const int8_t *xq_in = nullptr, const float *xs_in = nullptr,
-                              bool tail = true);
+                              bool tail = true, int act_qmax = 127);
 // From this many tokens on, the decode projection runs as three kernels:
 // xquant (one CTA per token), proj_small on the given codes, requant (one CTA
 // per row); below it, proj_small quantizes and requantizes by itself.
@@ -144,6 +155,14 @@ constexpr int kPsSplitTok = 4;
 bool gemm_tc_supported(int d, int r);
 cudaError_t launch_gemm_tc(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
                            const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s);
+
+// W4A4: the GEMM on fp8 e4m3 images of int4-valued codes (kind::f8f6f4),
+// with the requantization epilogue for lat_bits 8 / 4 (0: c_hat only).
+bool gemm_f8_supported(int d, int r);
+cudaError_t launch_gemm_f8(const uint8_t *xq_f8, int64_t T, int d, const uint8_t *w_f8, const float *ws,
+                           const float *xs, int r, int lat_bits, float lat_clip, void *lat_codes, void *lat_scales,
+                           const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, float *c_hat,
+                           int32_t *acc_out, int *err, cudaStream_t s);
 
 // The same GEMM with the per-token requantization and store of the latent
 // (a3 second half + a4) in its epilogue; c_hat and acc_out are optional
@@ -168,12 +187,21 @@ cudaError_t launch_append(const CacheView &c, const int32_t *seq, const int32_t 
                           const void *lat_codes, const void *lat_scales, int *err,
                           cudaStream_t s);
 
+// An up-projection [r, d] as the decode kernels read it: bf16 values (bits
+// 16, scale null), or Eq. 11's Q(W^u): int8 codes [r, d] (bits 8) or packed
+// int4 codes [r, d/2] (bits 4) with one fp32 scale per output channel [d].
+struct UpW {
+    const void *w;
+    const float *scale;
+    int bits;
+};
+
 // Decode attention (a5-a8).
 struct DecodeArgs {
     CacheView cache;
     const int32_t *seq_len;
     int max_seq_len;
-    const uint16_t *U_q, *U_k, *U_v;
+    UpW U_q, U_k, U_v;
     int H, dh;
     float softmax_scale;
     float *O;
@@ -202,7 +230,7 @@ struct PrefillBlocks {
 size_t prefill_mat_rows(const PrefillBlocks &bl);
 size_t prefill_mat_workspace_bytes(size_t R, int r, int d);
 cudaError_t launch_prefill_weights(const uint16_t *Uq, const uint16_t *Uk, const uint16_t *Uv, int r, int d,
-                                   uint16_t *Ut, cudaStream_t s);
+                                   uint16_t *Ut, int *err, cudaStream_t s);
 cudaError_t launch_prefill_mat(const CacheView &c, const PrefillBlocks &bl, const uint16_t *Ut, int H,
                                float softmax_scale, float *O, void *ws, int *err, cudaStream_t s);
 
@@ -219,13 +247,21 @@ cudaError_t launch_qabsorb_mma(const float *q, const uint16_t *Uk, int B, int r,
 cudaError_t launch_combine_mma(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
                                const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
                                cudaStream_t s);
-cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
+// The CUDA-core forms (decode_gemv.cu); they read every weight format.
+cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const UpW &Uq, int d, float *q,
                          unsigned *qmax, int n_qmax, int *err, cudaStream_t s);
-cudaError_t launch_qabsorb(const float *q, const uint16_t *Uk, int B, int r, int d, int H, int dh, float *qt,
+cudaError_t launch_qabsorb(const float *q, const UpW &Uk, int B, int r, int d, int H, int dh, float *qt,
                            unsigned *qmax, int *err, cudaStream_t s);
-cudaError_t launch_combine_uv(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh, int r, int chunk, int n_split,
-                              const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
-                              int *err, cudaStream_t s);
+cudaError_t launch_combine_uv(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh,
+                              int r, int chunk, int n_split, const float *pm, const float *pl, const float *po,
+                              const UpW &Uv, float *O, int *err, cudaStream_t s);
+
+// a5 in one launch for up to four sequences (decode_qfuse.cu): q and q~ per
+// head in a cluster, q_h exchanged in distributed shared memory; used when
+// U_q and U_k share a format and the whole grid is resident at once.
+bool qfuse_use(const CacheView &c, const UpW &Uq, const UpW &Uk, int H, int dh);
+cudaError_t launch_qfuse(const CacheView &c, const int32_t *seq_len, const UpW &Uq, const UpW &Uk, int H, int dh,
+                         float *qt, unsigned *qmax, int *err, cudaStream_t s);
 
 // Tensor-core latent attention (a6/a7): choice of kernel, split of each
 // sequence into partials (tiles of 128 tokens), and the launcher, which writes

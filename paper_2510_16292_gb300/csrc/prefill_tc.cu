@@ -10,6 +10,8 @@
 //
 //   ut_kernel        offline: fp16 [3d, r] = [U_q U_k U_v]^T (bf16 in), so
 //                    that both GEMM operands are K-major
+// Every fp16 rounding (Ut, the int4 latent operand, Q, K, V) saturates at
+// +-65504 and flags a range error instead of producing inf.
 //   lat_prep_kernel  the latent rows of every block as an fp16 GEMM operand:
 //                    int8 codes (exact in fp16) with the token scale kept
 //                    for the epilogue, or int4 code x group scale rounded to
@@ -47,6 +49,14 @@
 namespace qsvd {
 
 namespace pf {
+
+// fp16 conversion with the range guard of the materialised operands: a value
+// beyond +-65504 (fp16's largest finite) is saturated to it and `over` is set
+// (the caller flags kErrRange once), so nothing becomes inf silently.
+__device__ __forceinline__ __half2 h2_sat(float a, float b, bool &over) {
+    over |= !(fabsf(a) <= 65504.0f) || !(fabsf(b) <= 65504.0f);
+    return __floats2half2_rn(fminf(fmaxf(a, -65504.0f), 65504.0f), fminf(fmaxf(b, -65504.0f), 65504.0f));
+}
 
 constexpr int kRowTile = 128;           // rows per GEMM tile, queries and keys per attention tile
 constexpr int kDh = 128;                // head size of the attention kernel
@@ -97,7 +107,7 @@ __device__ __forceinline__ float ex2_approx(float x) {
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256)
 ut_kernel(const uint16_t *__restrict__ Uq, const uint16_t *__restrict__ Uk, const uint16_t *__restrict__ Uv, int r,
-          int d, __half *__restrict__ Ut) {
+          int d, __half *__restrict__ Ut, int *err) {
     __shared__ float tile[32][33];
     const int n0 = blockIdx.x * 32, k0 = blockIdx.y * 32;
     const int part = n0 / d, c0 = n0 - part * d;
@@ -105,15 +115,17 @@ ut_kernel(const uint16_t *__restrict__ Uq, const uint16_t *__restrict__ Uk, cons
     for (int i = threadIdx.y; i < 32; i += 8)
         tile[i][threadIdx.x] = bf16_to_f32(U[size_t(k0 + i) * d + c0 + threadIdx.x]);
     __syncthreads();
+    bool over = false;
     for (int i = threadIdx.y; i < 32; i += 8)
-        Ut[size_t(n0 + i) * r + k0 + threadIdx.x] = __float2half_rn(tile[threadIdx.x][i]);
+        Ut[size_t(n0 + i) * r + k0 + threadIdx.x] = __low2half(pf::h2_sat(tile[threadIdx.x][i], 0.0f, over));
+    if (over) flag_error(err, kErrRange);
 }
 
 // ---------------------------------------------------------------------------
 // latent rows of the blocks -> fp16 operand A [R, r] and row scale rs [R]
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256)
-lat_prep_kernel(CacheView c, PrefillBlocks bl, int R, __half *__restrict__ A, float *__restrict__ rs) {
+lat_prep_kernel(CacheView c, PrefillBlocks bl, int R, __half *__restrict__ A, float *__restrict__ rs, int *err) {
     pdl_wait();
     pdl_trigger();
     const int r = c.r, per_row = r / 8;                       // threads per row: 8 channels each
@@ -151,13 +163,14 @@ lat_prep_kernel(CacheView c, PrefillBlocks bl, int R, __half *__restrict__ A, fl
                                                                    slot * (r / 2) + j / 2);
             const float s = __half2float(static_cast<const __half *>(c.scales)[slot * (r / 128) + j / 128]);
             uint32_t h[4];
+            bool over = false;             // |code| * s reaches 7 * 65504 at most
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int lo = int((w >> (8 * e)) & 0xf), hi = int((w >> (8 * e + 4)) & 0xf);
-                const __half2 v = __halves2half2(__float2half_rn(float((lo ^ 8) - 8) * s),
-                                                 __float2half_rn(float((hi ^ 8) - 8) * s));
+                const __half2 v = pf::h2_sat(float((lo ^ 8) - 8) * s, float((hi ^ 8) - 8) * s, over);
                 h[e] = *reinterpret_cast<const uint32_t *>(&v);
             }
+            if (over) flag_error(err, kErrRange);
             o = make_uint4(h[0], h[1], h[2], h[3]);
         }
     }
@@ -266,11 +279,13 @@ qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant
                 tc::tmem_ld32(taddr + j0, v);
                 tc::tmem_wait_ld();
                 uint32_t h[16];
+                bool over = false;
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
-                    const __half2 x = __floats2half2_rn(__uint_as_float(v[2 * j]) * sc, __uint_as_float(v[2 * j + 1]) * sc);
+                    const __half2 x = h2_sat(__uint_as_float(v[2 * j]) * sc, __uint_as_float(v[2 * j + 1]) * sc, over);
                     h[j] = *reinterpret_cast<const uint32_t *>(&x);
                 }
+                if (over) flag_error(err, kErrRange);
                 if (part < 2) {
                     uint4 *dst = reinterpret_cast<uint4 *>((part == 0 ? Qm : Km) + size_t(row) * d + cbase + j0);
 #pragma unroll
@@ -588,8 +603,8 @@ size_t prefill_mat_workspace_bytes(size_t R, int r, int d) {
 }
 
 cudaError_t launch_prefill_weights(const uint16_t *Uq, const uint16_t *Uk, const uint16_t *Uv, int r, int d,
-                                   uint16_t *Ut, cudaStream_t s) {
-    ut_kernel<<<dim3(3 * d / 32, r / 32), dim3(32, 8), 0, s>>>(Uq, Uk, Uv, r, d, reinterpret_cast<__half *>(Ut));
+                                   uint16_t *Ut, int *err, cudaStream_t s) {
+    ut_kernel<<<dim3(3 * d / 32, r / 32), dim3(32, 8), 0, s>>>(Uq, Uk, Uv, r, d, reinterpret_cast<__half *>(Ut), err);
     const cudaError_t e = cudaGetLastError();
     prof_mark(s, "ut");
     return e;
@@ -613,7 +628,7 @@ cudaError_t launch_prefill_mat(const CacheView &c, const PrefillBlocks &bl, cons
 
     const int64_t prep_threads = int64_t(R) * (r / 8);
     cudaError_t e = launch_pdl(lat_prep_kernel, dim3(unsigned((prep_threads + 255) / 256)), dim3(256), 0, s, c, bl, R,
-                               A, rs);
+                               A, rs, err);
     if (e != cudaSuccess) return e;
     prof_mark(s, "lat_prep");
 

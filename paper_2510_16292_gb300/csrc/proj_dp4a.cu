@@ -61,7 +61,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                   int *__restrict__ counter, int8_t *__restrict__ xq_out, float *__restrict__ xs_out,
                   int32_t *__restrict__ acc_out, void *__restrict__ lat_codes, void *__restrict__ lat_scales,
                   CacheView dst, const int32_t *__restrict__ dst_seq, const int32_t *__restrict__ dst_pos,
-                  int *err, const int8_t *__restrict__ xq_in, const float *__restrict__ xs_in, int tail) {
+                  int *err, const int8_t *__restrict__ xq_in, const float *__restrict__ xs_in, int tail, int act_qmax) {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar, bar_x;
     {   // this CTA's token block
@@ -96,6 +96,14 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
     if (threadIdx.x == 0) {     // W_d codes: no kernel's output, copied before the wait on the producer grid
         mbar_arrive_expect_tx(&bar, uint32_t(rows) * d);
         for (int i = 0; i < rows; ++i) bulk_g2s(w_s + size_t(i) * dp, w + size_t(j0 + i) * d, uint32_t(d), &bar);
+    } else if (threadIdx.x <= T && !xq_in) {
+        // the token rows into L2 while the producer grid finishes (L2 is the point of
+        // coherence, so a row written meanwhile is never seen stale: the reads come after the wait)
+        prefetch_l2_bulk(X + size_t(threadIdx.x - 1) * d, uint32_t(d) * 2);
+    } else if (tail && blockIdx.x == 0 && dst.codes && threadIdx.x >= 32 && threadIdx.x < 32 + T) {
+        // the append indices the last CTA reads (inputs, same argument)
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(dst_seq + (threadIdx.x - 32)) : "memory");
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(dst_pos + (threadIdx.x - 32)) : "memory");
     }
     pdl_wait();
     // a1: per-token int8 quantization.  Codes quantized by the previous kernel
@@ -143,7 +151,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
             float mm = red4[0][threadIdx.x];
 #pragma unroll
             for (int w = 1; w < kPsWarps; ++w) mm = fmaxf(mm, red4[w][threadIdx.x]);
-            const float s = quant_scale(mm, act_clip, 127.0f);
+            const float s = quant_scale(mm, act_clip, float(act_qmax));
             xs_s[t0 + threadIdx.x] = s;
             if (xs_out && blockIdx.x == 0) xs_out[t0 + threadIdx.x] = s;
         }
@@ -161,8 +169,8 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                 uint32_t lo = 0, hi = 0;
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    lo |= uint32_t(quant_code_fast(f[e], s, inv, 127) & 0xff) << (8 * e);
-                    hi |= uint32_t(quant_code_fast(f[e + 4], s, inv, 127) & 0xff) << (8 * e);
+                    lo |= uint32_t(quant_code_fast(f[e], s, inv, act_qmax) & 0xff) << (8 * e);
+                    hi |= uint32_t(quant_code_fast(f[e + 4], s, inv, act_qmax) & 0xff) << (8 * e);
                 }
                 *reinterpret_cast<uint2 *>(xq_s + size_t(t0 + g) * dp + col) = make_uint2(lo, hi);
                 if (xq_out && blockIdx.x == 0)
@@ -262,7 +270,7 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
                               const float *ws, int r, int lat_bits, float lat_clip, float *c_hat, int *counter,
                               int8_t *xq_out, float *xs_out, int32_t *acc_out, void *lat_codes, void *lat_scales,
                               const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
-                              cudaStream_t s, const int8_t *xq_in, const float *xs_in, bool tail) {
+                              cudaStream_t s, const int8_t *xq_in, const float *xs_in, bool tail, int act_qmax) {
     CacheView dv{};
     if (dst) dv = *dst;
     // padded rows; the tensor-core path reuses the code rows for an [8][16][8] int32 reduction
@@ -273,7 +281,7 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
     e = launch_pdl(proj_small_kernel, dim3((r + kPsWarps - 1) / kPsWarps, (T + kPsMaxTok - 1) / kPsMaxTok),
                    dim3(kPsWarps * 32), smem, s, X, T, d,
                    act_clip, wcodes, ws, r, lat_bits, lat_clip, c_hat, counter, xq_out, xs_out, acc_out, lat_codes,
-                   lat_scales, dv, dst_seq, dst_pos, err, xq_in, xs_in, int(tail));
+                   lat_scales, dv, dst_seq, dst_pos, err, xq_in, xs_in, int(tail), act_qmax);
     prof_mark(s, "proj_small");
     return e;
 }

@@ -70,6 +70,9 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
     if ((st = scratch_for_current_device(&scratch))) return st;
     if (!W || !W->codes || !W->scale || !X) return sfail(QSVD_EINVAL, "latent_project_static: null pointer");
     if (W->rot) return sfail(QSVD_EUNSUPPORTED, "latent_project_static: rotated weights (W->rot) need qsvd_latent_project");
+    const int xb = W->x_bits ? W->x_bits : 8, wb = W->w_bits ? W->w_bits : 8;
+    if ((xb != 8 && xb != 4) || (wb != 8 && wb != 4))
+        return sfail(QSVD_EINVAL, "latent_project_static: W->w_bits and W->x_bits must be 8 or 4");
     const void *ptrs[] = {X, W->codes, lat_codes, lat_scales};
     for (const void *p : ptrs)
         if (p && (reinterpret_cast<uintptr_t>(p) & 15u))
@@ -107,7 +110,7 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
     if (e == cudaSuccess)
         e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
                               nullptr, nullptr, nullptr, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq, dst_pos,
-                              err, stream);
+                              err, stream, nullptr, nullptr, true, xb == 8 ? 127 : 7);
     if (e != cudaSuccess) {
         char msg[160];
         snprintf(msg, sizeof(msg), "latent_project_static: %s", cudaGetErrorString(e));

@@ -15,6 +15,8 @@
 //                       128-channel group (int4), written token-major and/or
 //                       straight into the latent cache.
 //   append_kernel       a4: latent rows -> cache slots.
+//   up_quant_kernel     offline per-output-channel RTN of an up-projection
+//                       (Eq. 11's Q(W^u)), int8 or int4.
 #include <cmath>
 
 #include "common.cuh"
@@ -47,8 +49,9 @@ __device__ __forceinline__ void fwht_smem(float *v, int n, int b, float scale) {
 }
 
 __global__ void __launch_bounds__(kXqThreads)
-xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int rot, float rot_scale, int8_t *__restrict__ xq,
-              uint16_t *__restrict__ xq_bf16, float *__restrict__ xs) {
+xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int rot, float rot_scale, int qmax,
+              int8_t *__restrict__ xq, uint16_t *__restrict__ xq_bf16, uint8_t *__restrict__ xq_f8,
+              float *__restrict__ xs) {
     extern __shared__ float row[];
     __shared__ float red[kXqThreads / 32];
     const int64_t t = blockIdx.x;
@@ -80,27 +83,30 @@ xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int rot, float 
         }
     }
     m = block_max<kXqThreads>(m, red);
-    const float s = quant_scale(m, clip, 127.0f), inv = quant_inv_scale(s);
+    const float s = quant_scale(m, clip, float(qmax)), inv = quant_inv_scale(s);
     for (int i = threadIdx.x * 8; i < d; i += kXqThreads * 8) {
-        uint32_t packed[2] = {0u, 0u};
+        uint32_t packed[2] = {0u, 0u}, f8w[2] = {0u, 0u};
         uint32_t bfw[4];
 #pragma unroll
         for (int e = 0; e < 8; e += 2) {
-            const int c0 = quant_code_fast(row[i + e], s, inv, 127);
-            const int c1 = quant_code_fast(row[i + e + 1], s, inv, 127);
+            const int c0 = quant_code_fast(row[i + e], s, inv, qmax);
+            const int c1 = quant_code_fast(row[i + e + 1], s, inv, qmax);
             packed[e >> 2] |= (uint32_t(c0 & 0xff) << ((e & 3) * 8)) |
                               (uint32_t(c1 & 0xff) << (((e & 3) + 1) * 8));
+            f8w[e >> 2] |= (uint32_t(int_to_e4m3(c0)) << ((e & 3) * 8)) |
+                           (uint32_t(int_to_e4m3(c1)) << (((e & 3) + 1) * 8));
             bfw[e >> 1] = uint32_t(int_to_bf16_bits(c0)) | (uint32_t(int_to_bf16_bits(c1)) << 16);
         }
         if (xq) *reinterpret_cast<uint2 *>(xq + t * d + i) = make_uint2(packed[0], packed[1]);
         if (xq_bf16)
             *reinterpret_cast<uint4 *>(xq_bf16 + t * d + i) = make_uint4(bfw[0], bfw[1], bfw[2], bfw[3]);
+        if (xq_f8) *reinterpret_cast<uint2 *>(xq_f8 + t * d + i) = make_uint2(f8w[0], f8w[1]);
     }
     if (threadIdx.x == 0 && xs) xs[t] = s;
 }
 
 cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip, int8_t *xq,
-                          uint16_t *xq_bf16, float *xs, cudaStream_t s, int rot) {
+                          uint16_t *xq_bf16, float *xs, cudaStream_t s, int rot, int qmax, uint8_t *xq_f8) {
     if (T == 0) return cudaSuccess;
     const size_t smem = size_t(d) * sizeof(float);
     if (smem > 48 * 1024) {
@@ -109,7 +115,7 @@ cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip, int8_
     }
     const float rot_scale = rot ? float(1.0 / std::sqrt(double(rot))) : 1.0f;
     cudaError_t e = launch_pdl(xquant_kernel, dim3(unsigned(T)), dim3(kXqThreads), smem, s, X, d, clip, rot,
-                               rot_scale, xq, xq_bf16, xs);
+                               rot_scale, qmax, xq, xq_bf16, xq_f8, xs);
     prof_mark(s, "xquant");
     return e;
 }
@@ -119,8 +125,8 @@ cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip, int8_
 // CTA = 32 columns x 8 row lanes; coalesced reads along a row of W_d.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256)
-weight_quant_kernel(const float *__restrict__ W, int d, int r, float clip, int8_t *__restrict__ codes,
-                    uint16_t *__restrict__ codes_bf16, float *__restrict__ scale) {
+weight_quant_kernel(const float *__restrict__ W, int d, int r, float clip, int qmax, int8_t *__restrict__ codes,
+                    uint16_t *__restrict__ codes_bf16, uint8_t *__restrict__ codes_f8, float *__restrict__ scale) {
     __shared__ float red[8][33];
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int j = blockIdx.x * 32 + tx;
@@ -131,16 +137,17 @@ weight_quant_kernel(const float *__restrict__ W, int d, int r, float clip, int8_
     __syncthreads();
     if (ty == 0) {
         for (int i = 1; i < 8; ++i) m = fmaxf(m, red[i][tx]);
-        red[0][tx] = quant_scale(m, clip, 127.0f);
+        red[0][tx] = quant_scale(m, clip, float(qmax));
     }
     __syncthreads();
     const float s = red[0][tx];
     if (j >= r) return;
     if (ty == 0) scale[j] = s;
     for (int k = ty; k < d; k += 8) {
-        const int c = quant_code(W[size_t(k) * r + j], s, 127);
+        const int c = quant_code(W[size_t(k) * r + j], s, qmax);
         codes[size_t(j) * d + k] = int8_t(c);
         if (codes_bf16) codes_bf16[size_t(j) * d + k] = int_to_bf16_bits(c);
+        if (codes_f8) codes_f8[size_t(j) * d + k] = int_to_e4m3(c);
     }
     // The projection kernels copy W_d's codes before they wait on their
     // producer grid: a dependent launch may begin only once the codes are
@@ -155,8 +162,9 @@ weight_quant_kernel(const float *__restrict__ W, int d, int r, float clip, int8_
 constexpr int kWqrCols = 4;
 
 __global__ void __launch_bounds__(256)
-weight_quant_rot_kernel(const float *__restrict__ W, int d, int r, float clip, int rot, float rot_scale,
-                        int8_t *__restrict__ codes, uint16_t *__restrict__ codes_bf16, float *__restrict__ scale) {
+weight_quant_rot_kernel(const float *__restrict__ W, int d, int r, float clip, int rot, float rot_scale, int qmax,
+                        int8_t *__restrict__ codes, uint16_t *__restrict__ codes_bf16, uint8_t *__restrict__ codes_f8,
+                        float *__restrict__ scale) {
     extern __shared__ float col[];                        // [kWqrCols][d]
     __shared__ float red[kWqrCols][8];
     __shared__ float sc[kWqrCols];
@@ -178,16 +186,17 @@ weight_quant_rot_kernel(const float *__restrict__ W, int d, int r, float clip, i
     if (threadIdx.x < kWqrCols) {
         float m = 0.0f;
         for (int w = 0; w < 8; ++w) m = fmaxf(m, red[threadIdx.x][w]);
-        sc[threadIdx.x] = quant_scale(m, clip, 127.0f);
+        sc[threadIdx.x] = quant_scale(m, clip, float(qmax));
     }
     __syncthreads();
     for (int c = 0; c < nc; ++c) {
         const float s = sc[c];
         if (threadIdx.x == 0) scale[j0 + c] = s;
         for (int k = threadIdx.x; k < d; k += blockDim.x) {
-            const int q = quant_code(col[c * d + k], s, 127);
+            const int q = quant_code(col[c * d + k], s, qmax);
             codes[size_t(j0 + c) * d + k] = int8_t(q);
             if (codes_bf16) codes_bf16[size_t(j0 + c) * d + k] = int_to_bf16_bits(q);
+            if (codes_f8) codes_f8[size_t(j0 + c) * d + k] = int_to_e4m3(q);
         }
     }
     __threadfence();                                      // see weight_quant_kernel
@@ -195,15 +204,17 @@ weight_quant_rot_kernel(const float *__restrict__ W, int d, int r, float clip, i
 }
 
 cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int8_t *codes,
-                                   uint16_t *codes_bf16, float *scale, cudaStream_t s, int rot) {
+                                   uint16_t *codes_bf16, float *scale, cudaStream_t s, int rot, int qmax,
+                                   uint8_t *codes_f8) {
     if (rot) {
         const size_t smem = size_t(kWqrCols) * d * sizeof(float);
         cudaError_t e = ensure_smem(weight_quant_rot_kernel, smem);
         if (e != cudaSuccess) return e;
         weight_quant_rot_kernel<<<dim3((r + kWqrCols - 1) / kWqrCols), 256, smem, s>>>(
-            W, d, r, clip, rot, float(1.0 / std::sqrt(double(rot))), codes, codes_bf16, scale);
+            W, d, r, clip, rot, float(1.0 / std::sqrt(double(rot))), qmax, codes, codes_bf16, codes_f8, scale);
     } else {
-        weight_quant_kernel<<<dim3((r + 31) / 32), 256, 0, s>>>(W, d, r, clip, codes, codes_bf16, scale);
+        weight_quant_kernel<<<dim3((r + 31) / 32), 256, 0, s>>>(W, d, r, clip, qmax, codes, codes_bf16, codes_f8,
+                                                                 scale);
     }
     prof_mark(s, "weight_quant");
     return cudaGetLastError();
@@ -268,6 +279,50 @@ cudaError_t launch_append(const CacheView &c, const int32_t *seq, const int32_t 
                                static_cast<const uint8_t *>(lat_codes), static_cast<const uint8_t *>(lat_scales), err);
     prof_mark(s, "append");
     return e;
+}
+
+// ---------------------------------------------------------------------------
+// Offline Q(W^u) of Eq. 11 (H2 = I), the weight quantizer of the Sec. 4
+// setup: per output channel (column c of U [r, d], bf16) symmetric RTN to
+// `bits` (8: int8 codes [r, d]; 4: packed int4 [r, d/2], column 2i in the low
+// nibble) with an fp32 scale per column.  CTA = 32 columns (lane) x 8 row
+// groups (warp).
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256)
+up_quant_kernel(const uint16_t *__restrict__ U, int r, int d, int bits, float clip, uint8_t *__restrict__ codes,
+                float *__restrict__ scale) {
+    __shared__ float red[8][33];
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int c = blockIdx.x * 32 + tx;        // d % 32 == 0: every lane has a column
+    const int qm = bits == 8 ? 127 : 7;
+    float m = 0.0f;
+    for (int j = ty; j < r; j += 8) m = fmaxf(m, fabsf(bf16_to_f32(U[size_t(j) * d + c])));
+    red[ty][tx] = m;
+    __syncthreads();
+    if (ty == 0) {
+        for (int i = 1; i < 8; ++i) m = fmaxf(m, red[i][tx]);
+        red[0][tx] = quant_scale(m, clip, float(qm));
+        scale[c] = red[0][tx];
+    }
+    __syncthreads();
+    const float s = red[0][tx];
+    for (int j = ty; j < r; j += 8) {
+        const int code = quant_code(bf16_to_f32(U[size_t(j) * d + c]), s, qm);
+        if (bits == 8) {
+            codes[size_t(j) * d + c] = uint8_t(int8_t(code));
+        } else {
+            const int hi = __shfl_down_sync(0xffffffffu, code, 1);
+            if ((tx & 1) == 0) codes[(size_t(j) * d + c) / 2] = uint8_t((code & 0xF) | ((hi & 0xF) << 4));
+        }
+    }
+}
+
+cudaError_t launch_quantize_up(const uint16_t *U, int r, int d, int bits, float clip, void *codes, float *scale,
+                               cudaStream_t s) {
+    up_quant_kernel<<<dim3(unsigned(d / 32)), dim3(256), 0, s>>>(U, r, d, bits, clip, static_cast<uint8_t *>(codes),
+                                                                scale);
+    prof_mark(s, "up_quant");
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------

@@ -55,7 +55,7 @@ def test_llava13b_full_batch_chained_decode():
     gpu.len[:] = P
     for b in tracked:
         np.testing.assert_array_equal(cache_codes_np(gpu.cache, b, P), ref.cache.codes[b, :P])
-        np.testing.assert_array_equal(cache_scales_np(gpu.cache, b, P), ref.cache.scales[b, :P])
+        np.testing.assert_array_equal(cache_scales_np(gpu.cache, b, P), ref.cache.scale[b, :P])
     prev = lib.qsvd_set_decode_attn_path(0)
     try:
         for t in range(steps):
@@ -70,7 +70,7 @@ def test_llava13b_full_batch_chained_decode():
     L = P + steps
     for b in tracked:
         np.testing.assert_array_equal(cache_codes_np(gpu.cache, b, L), ref.cache.codes[b, :L])
-        np.testing.assert_array_equal(cache_scales_np(gpu.cache, b, L), ref.cache.scales[b, :L])
+        np.testing.assert_array_equal(cache_scales_np(gpu.cache, b, L), ref.cache.scale[b, :L])
 
 
 def _up_weights(H, dh, r, seed):

@@ -317,3 +317,35 @@ def test_latent_prefill_13b_int4_continued():
     O = _gpu_blocks(gpu, blocks)
     want = np.concatenate([_oracle_rows(ref, b, t0, t0 + T) for b, t0, T in blocks])
     assert_rows_close(O, want, "13B int4 blocks")
+
+
+def test_latent_prefill_fp16_range_guard():
+    """Values beyond fp16's range saturate at +-65504 and flag QSVD_ERANGE
+    instead of turning into inf: an up-projection entry of 1e5 in
+    qsvd_prefill_weights, and Q / K / V beyond 65504 in the block GEMM (a
+    latent of magnitude ~1e3 against entries ~400); the outputs stay finite."""
+    lib = q()
+    H, dh, r, L = 32, 128, 1536, 200
+    d = H * dh
+    rng = np.random.default_rng(61)
+    U = [synthetic.bf16_bits(rng.standard_normal((r, d)) * 400.0) for _ in range(3)]
+    Ub = [torch.from_numpy(u.view(np.int16)).view(torch.bfloat16).to(dev()) for u in U]
+    big = U[0].copy()
+    big[3, 5] = synthetic.bf16_bits(np.array([1e5]))[0]
+    Ubig = torch.from_numpy(big.view(np.int16)).view(torch.bfloat16).to(dev())
+    Ut = lib.qsvd_prefill_weights(Ubig, Ub[1], Ub[2])
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_check()
+    assert e.value.status == lib.QSVD_ERANGE
+    assert float(Ut.float().abs().max()) == 65504.0 and torch.isfinite(Ut.float()).all()
+    Ut = lib.qsvd_prefill_weights(*Ub)
+    lib.qsvd_check()                                        # in range: no flag
+    cache = lib.LatentCache.empty(1, L, r, 8, dev())
+    cache.codes.copy_(torch.randint(-127, 128, cache.codes.shape, device=dev(), dtype=torch.int8))
+    cache.scales.fill_(8.0)                                 # latent entries up to ~1000
+    O = torch.empty((L, d), dtype=torch.float32, device=dev())
+    lib.qsvd_latent_prefill(cache, [(0, 0, L)], Ut, H, dh, O)
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_check()
+    assert e.value.status == lib.QSVD_ERANGE
+    assert torch.isfinite(O).all()

@@ -28,24 +28,53 @@ def test_dequantize_acc_matches_float32_arithmetic():
     np.testing.assert_array_equal(got, ref.astype(np.float64))
 
 
-def test_projection_within_quantization_error():
+@pytest.mark.parametrize("x_bits,w_bits", [(8, 8), (4, 4), (8, 4)])
+def test_projection_within_quantization_error(x_bits, w_bits):
     """The dequantized latent differs from the exact X W_d by no more than
     the rounding of X and W_d to their grids allows:
-    |X W - s_x s_w Xq Wq| <= sum_k ( s_x/2 |W_kj| + s_x |Xq_k| s_w/2 )."""
+    |X W - s_x s_w Xq Wq| <= sum_k ( s_x/2 |W_kj| + s_x |Xq_k| s_w/2 ),
+    for int8 (W8A8) and int4 (W4A4, and int4 weights with int8 X) codes."""
     rng = np.random.default_rng(2)
     T, d, r = 9, 64, 24
     X = rng.standard_normal((T, d)).astype(np.float32).astype(np.float64)
     X[:, 3] *= 20
     W = (rng.standard_normal((d, r)) / 8).astype(np.float32).astype(np.float64)
-    Wq, s_w = quant.quantize_columns(W, 8)
-    out = latent.latent_project(X, Wq, s_w, lat_bits=8)
+    Wq, s_w = quant.quantize_columns(W, w_bits)
+    out = latent.latent_project(X, Wq, s_w, lat_bits=8, x_bits=x_bits)
+    assert np.abs(out["xq"]).max() == (1 << (x_bits - 1)) - 1
+    assert np.abs(Wq).max() == (1 << (w_bits - 1)) - 1
     exact = X @ W
     bound = (out["s_x"][:, None] / 2) * np.abs(W).sum(0)[None, :] \
         + (out["s_x"][:, None] * np.abs(out["xq"]).sum(1)[:, None]) * (s_w[None, :] / 2)
     err = np.abs(exact - out["c_hat"])
     assert np.all(err <= bound * (1 + 1e-5) + 1e-6 * np.abs(exact))
-    # and the bound is not vacuous: the error is far below |C|
-    assert np.median(err / (np.abs(exact) + 1e-9)) < 0.05
+    # and the bound is not vacuous: the error is far below |C| (int4 grids are 18x coarser)
+    assert np.median(err / (np.abs(exact) + 1e-9)) < (0.05 if x_bits == w_bits == 8 else 0.6)
+
+
+def test_w4a4_projection_brute_force():
+    """W4A4 on a tiny block, every step recomputed by hand in numpy float32:
+    4-bit codes from a search over [-7, 7], the integer sums by loops, then
+    (fp32(acc) s_x) s_w; and |acc| <= 49 d, the bound that keeps every
+    partial sum exact in fp32 for d < 2^24 / 49."""
+    rng = np.random.default_rng(21)
+    T, d, r = 3, 40, 5
+    X = (rng.standard_normal((T, d)) * 2).astype(np.float32)
+    W = (rng.standard_normal((d, r)) / 6).astype(np.float32)
+    Wq, s_w = quant.quantize_columns(W.astype(np.float64), 4)
+    out = latent.latent_project(X.astype(np.float64), Wq, s_w, lat_bits=8, x_bits=4)
+    for t in range(T):
+        s = np.float32(np.max(np.abs(X[t]))) / np.float32(7)
+        assert out["s_x"][t] == float(s)
+        for k in range(d):
+            x = X[t, k] / s
+            c = min(range(-7, 8), key=lambda v: (abs(float(x) - v), v % 2))
+            assert out["xq"][t, k] == c
+        for j in range(r):
+            acc = sum(int(out["xq"][t, k]) * int(Wq[k, j]) for k in range(d))
+            assert out["acc"][t, j] == acc and abs(acc) <= 49 * d
+            c_hat = (np.float32(acc) * np.float32(out["s_x"][t])) * np.float32(s_w[j])
+            assert out["c_hat"][t, j] == float(c_hat)
 
 
 def test_latent_requant_roundtrip_int8_int4():
