@@ -650,7 +650,7 @@ def importance_probe(iters=3, N=1, m=4096, n=12288, k=4096):
     s = torch.rand((k,), generator=g, device=dev)
     Vt = torch.randn((k, n), generator=g, device=dev)
     G = torch.randn((N, m, n), generator=g, device=dev)
-    ws = torch.empty(int(q._lib.qsvd_importance_workspace_bytes(N, k)), dtype=torch.uint8, device=dev)
+    ws = torch.empty(int(q._lib.qsvd_importance_workspace_bytes(N, m, k)), dtype=torch.uint8, device=dev)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     times = []
     for it in range(iters + 1):

@@ -13,6 +13,7 @@
  *   qsvd_quantize_weight     offline per-channel int8 RTN of W_d (Sec. 4 setup)
  *   qsvd_quantize_weight_rotated  the same of H1 W_d (Eq. 12's online rotation)
  *   qsvd_importance_scores   offline Eq. 10 scores of singular values (Sec. 3.2)
+ *   qsvd_rank_budget         offline cross-layer top-k of those scores (Sec. 3.2)
  *   qsvd_latent_project      C = Q(X) Q(W_d), requantized per token (Eq. 11-12)
  *   qsvd_cache_append        store latent rows in the latent cache (Fig. 2(f))
  *   qsvd_latent_decode_attn  one decode step of attention over that cache (Eq. 5)
@@ -183,15 +184,29 @@ size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r);
  *   U fp32 [m, k] (left singular vectors as columns), sigma fp32 [k],
  *   Vt fp32 [k, n] (right singular vectors as rows), G fp32 [N, m, n] (the
  *   loss gradient for each of N calibration samples), scores fp32 [k] out.
- *   workspace: qsvd_importance_workspace_bytes(N, k) bytes.
- * fp32 on the CUDA cores; the per-sample sums are accumulated with atomics,
- * so the last bits vary between runs.  N <= 65535 per call.
+ *   workspace: qsvd_importance_workspace_bytes(N, m, k) bytes.
+ * fp32 on the CUDA cores; the sums run in a fixed order, so the result is
+ * the same bit for bit on every run.  N <= 65535 per call.
  */
 int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, const float *G, int32_t N, int32_t m,
                            int32_t n, int32_t k, float *scores, void *workspace, size_t workspace_bytes,
                            cudaStream_t stream);
 
-size_t qsvd_importance_workspace_bytes(int32_t N, int32_t k);
+size_t qsvd_importance_workspace_bytes(int32_t N, int32_t m, int32_t k);
+
+/*
+ * The cross-layer rank budget of Sec. 3.2 (the global sort after Eq. 10):
+ * of the n singular values of all layers -- scores fp32 [n], the layers'
+ * score vectors concatenated in layer order -- keep the k highest-scoring
+ * ones: keep[i] = 1 for those, 0 for the rest (uint8 [n] out).  Equal scores
+ * go to the lower position (the lower layer, then the lower index).  Scores
+ * must not be NaN.  Exactly k entries are kept (0 <= k <= n).  workspace:
+ * qsvd_rank_budget_workspace_bytes() bytes.
+ */
+int qsvd_rank_budget(const float *scores, int32_t n, int32_t k, uint8_t *keep, void *workspace,
+                     size_t workspace_bytes, cudaStream_t stream);
+
+size_t qsvd_rank_budget_workspace_bytes(void);
 
 /*
  * The rotation H1 of Eq. 11-12 applied on the fly (for models where it is not

@@ -31,7 +31,7 @@ _lib = ctypes.CDLL(_LIB_PATH)
 QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
 EXPORTS = ("qsvd_quantize_weight", "qsvd_quantize_weight_rotated", "qsvd_quantize_weight_ex", "qsvd_importance_scores",
-           "qsvd_importance_workspace_bytes", "qsvd_latent_project", "qsvd_project_workspace_bytes",
+           "qsvd_importance_workspace_bytes", "qsvd_rank_budget", "qsvd_rank_budget_workspace_bytes", "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
            "qsvd_quantize_up", "qsvd_latent_decode_attn_qu",
            "qsvd_latent_prefill_attn", "qsvd_prefill_workspace_bytes", "qsvd_prefill_weights",
@@ -72,7 +72,10 @@ _lib.qsvd_quantize_weight.argtypes = [_vp, _i32, _i32, _f32, _vp, _vp, _vp, _vp]
 _lib.qsvd_quantize_weight_rotated.argtypes = [_vp, _i32, _i32, _f32, _i32, _vp, _vp, _vp, _vp]
 _lib.qsvd_quantize_weight_ex.argtypes = [_vp, _i32, _i32, _f32, _i32, _i32, _vp, _vp, _vp, _vp, _vp]
 _lib.qsvd_importance_scores.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
-_lib.qsvd_importance_workspace_bytes.argtypes = [_i32, _i32]
+_lib.qsvd_importance_workspace_bytes.argtypes = [_i32, _i32, _i32]
+_lib.qsvd_rank_budget.argtypes = [_vp, _i32, _i32, _vp, _vp, _sz, _vp]
+_lib.qsvd_rank_budget_workspace_bytes.argtypes = []
+_lib.qsvd_rank_budget_workspace_bytes.restype = _sz
 _lib.qsvd_importance_workspace_bytes.restype = _sz
 _lib.qsvd_latent_project.argtypes = [ctypes.POINTER(_DownWeight), _vp, _i64, _f32, _i32, _f32, _vp, _vp,
                                      ctypes.POINTER(_Cache), _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
@@ -279,12 +282,24 @@ def qsvd_importance_scores(U: torch.Tensor, sigma: torch.Tensor, Vt: torch.Tenso
     N, _, n = G.shape
     scores = torch.empty((k,), dtype=torch.float32, device=U.device)
     if workspace is None:
-        workspace = torch.empty(max(1, int(_lib.qsvd_importance_workspace_bytes(N, k))), dtype=torch.uint8,
+        workspace = torch.empty(max(1, int(_lib.qsvd_importance_workspace_bytes(N, m, k))), dtype=torch.uint8,
                                 device=U.device)
     _check(_lib.qsvd_importance_scores(_ptr(U, _F32, "U"), _ptr(sigma, _F32, "sigma"), _ptr(Vt, _F32, "Vt"),
                                        _ptr(G, _F32, "G"), N, m, n, k, _ptr(scores), _ptr(workspace),
                                        workspace.numel(), _stream(stream)))
     return scores
+
+
+def qsvd_rank_budget(scores: torch.Tensor, k: int, workspace=None, stream=None) -> torch.Tensor:
+    """Cross-layer rank budget: scores fp32 [n] (every layer's scores in layer
+    order) -> keep uint8 [n], 1 for the k highest (ties: the lower position)."""
+    n = scores.numel()
+    keep = torch.empty((n,), dtype=torch.uint8, device=scores.device)
+    if workspace is None:
+        workspace = torch.empty(int(_lib.qsvd_rank_budget_workspace_bytes()), dtype=torch.uint8, device=scores.device)
+    _check(_lib.qsvd_rank_budget(_ptr(scores, _F32, "scores"), n, k, _ptr(keep), _ptr(workspace), workspace.numel(),
+                                 _stream(stream)))
+    return keep
 
 
 def qsvd_project_workspace_bytes(T: int, d: int, r: int) -> int:

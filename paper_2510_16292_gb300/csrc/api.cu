@@ -676,9 +676,26 @@ int qsvd_latent_prefill(const qsvd_cache *cache, const qsvd_prefill_block *block
     });
 }
 
-size_t qsvd_importance_workspace_bytes(int32_t N, int32_t k) {
-    if (N <= 0 || k <= 0) return 0;
-    return align256(size_t(N) * k * sizeof(float));
+size_t qsvd_importance_workspace_bytes(int32_t N, int32_t m, int32_t k) {
+    if (N <= 0 || m <= 0 || k <= 0) return 0;
+    return align256(size_t(N) * ((size_t(m) + kImpRowTile - 1) / kImpRowTile) * k * sizeof(float));
+}
+
+size_t qsvd_rank_budget_workspace_bytes(void) { return rank_workspace_bytes(); }
+
+int qsvd_rank_budget(const float *scores, int32_t n, int32_t k, uint8_t *keep, void *workspace,
+                     size_t workspace_bytes, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!scores || !keep) return fail(QSVD_EINVAL, "rank_budget: null pointer");
+    if (n <= 0 || k < 0 || k > n) return fail(QSVD_EINVAL, "rank_budget: need n > 0 and 0 <= k <= n");
+    if (!workspace || workspace_bytes < rank_workspace_bytes())
+        return fail(QSVD_ENOSPC, "rank_budget: workspace needs %zu bytes", rank_workspace_bytes());
+    if (!aligned16(workspace)) return fail(QSVD_EINVAL, "rank_budget: workspace must be 16-byte aligned");
+    prof_mark(stream, "begin");
+    const cudaError_t e = launch_rank_budget(scores, n, k, keep, workspace, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "rank_budget launch");
 }
 
 int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, const float *G, int32_t N, int32_t m,
@@ -690,7 +707,7 @@ int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, 
     if (!U || !sigma || !Vt || !G || !scores) return fail(QSVD_EINVAL, "importance_scores: null pointer");
     if (N <= 0 || m <= 0 || n <= 0 || k <= 0) return fail(QSVD_EINVAL, "importance_scores: N, m, n, k must be positive");
     if (N > 65535) return fail(QSVD_EUNSUPPORTED, "importance_scores: more than 65535 samples per call");
-    const size_t need = qsvd_importance_workspace_bytes(N, k);
+    const size_t need = qsvd_importance_workspace_bytes(N, m, k);
     if (!workspace || workspace_bytes < need)
         return fail(QSVD_ENOSPC, "importance_scores: workspace needs %zu bytes", need);
     prof_mark(stream, "begin");
