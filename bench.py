@@ -63,6 +63,9 @@ def parse():
     p.add_argument("--u-bits", type=int, default=0, choices=[0, 8, 4],
                    help="quantize U_q, U_k, U_v per output channel to int8 or int4 (Eq. 11) and run decode "
                         "attention on the codes (qsvd_latent_decode_attn_qu); 0: bf16 up-projections")
+    p.add_argument("--attn-path", type=int, default=0, choices=[0, 1, 2, 3],
+                   help="decode attention kernel choice (qsvd_set_decode_attn_path): 0 automatic, 1 CUDA cores, "
+                        "2 tcgen05, 3 warp-level MMA")
     p.add_argument("--rot", action="store_true",
                    help="rotate X by H1 on the fly (Eq. 12; weights quantized as H1 W_d) in every projection")
     p.add_argument("--prefill-probe", action="store_true",
@@ -902,6 +905,12 @@ SWEEP_FULL = dict(r=(1024, 1536, 2048, 3072), L=(1024, 4096, 16384, 32768), B=(1
 SWEEP_QUICK = dict(r=(1536, 3072), L=(1024, 32768), B=(1, 64), bits=(8, 4))
 
 
+def set_attn_path(args):
+    if args.attn_path:
+        import paper_2510_16292_gb300 as q
+        q.qsvd_set_decode_attn_path(args.attn_path)
+
+
 def run_sweep(args):
     """One JSON line per point: decode tokens/s of one layer and the fraction
     of the step's HBM roofline (bytes a decode step must read: the latent
@@ -1003,6 +1012,7 @@ def run_sweep(args):
 
 def main():
     args = parse()
+    set_attn_path(args)
     if args.sweep:
         run_sweep(args)
         return

@@ -242,32 +242,6 @@ __host__ __device__ constexpr uint32_t idesc_f16(int n, int a_mn) {
 }
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
-// Four int8 codes -> two fp16 pairs, exact: the half with bits 0x64xx is
-// 1024 + xx, so (code + 128) placed in the low byte gives 1152 + code.
-__device__ __forceinline__ void i8x4_to_h2x2(uint32_t w, uint32_t &lo, uint32_t &hi) {
-    const uint32_t u = w ^ 0x80808080u;
-    const uint32_t a = __byte_perm(u, 0x64646464u, 0x5150);
-    const uint32_t b = __byte_perm(u, 0x64646464u, 0x5352);
-    const __half2 bias = __half2half2(__ushort_as_half(0x6480));      // 1152
-    const __half2 ha = __hsub2(*reinterpret_cast<const __half2 *>(&a), bias);
-    const __half2 hb = __hsub2(*reinterpret_cast<const __half2 *>(&b), bias);
-    lo = *reinterpret_cast<const uint32_t *>(&ha);
-    hi = *reinterpret_cast<const uint32_t *>(&hb);
-}
-// Eight int4 codes (element i in bits 4i..4i+3, two's complement) times an
-// fp16 group scale -> four fp16 pairs (products rounded to nearest).
-__device__ __forceinline__ void i4x8_to_h2x4(uint32_t w, __half2 s2, uint32_t *o) {
-    const __half2 bias = __half2half2(__ushort_as_half(0x6408));      // 1032 = 1024 + 8
-    const uint32_t x = w ^ 0x88888888u;                               // code + 8 in every nibble
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const uint32_t n0 = (x >> (8 * k)) & 0xfu, n1 = (x >> (8 * k + 4)) & 0xfu;
-        const uint32_t p = (0x6400u | n0) | ((0x6400u | n1) << 16);
-        const __half2 h = __hmul2(__hsub2(*reinterpret_cast<const __half2 *>(&p), bias), s2);
-        o[k] = *reinterpret_cast<const uint32_t *>(&h);
-    }
-}
-
 // Eight int4 codes (element i in bits 4i..4i+3, two's complement) times an
 // fp16 group scale -> four fp16 pairs in the order (0,4), (1,5), (2,6), (3,7)
 // (products rounded to nearest).  The nibbles xor 8 are placed in the
