@@ -50,6 +50,23 @@ namespace qsvd {
 
 namespace pf {
 
+// Stores of the GEMM's outputs with an L2 evict-first policy: Q, K and V^T
+// (3 d x R fp16, hundreds of MB at the 13B batch) would otherwise evict Ut
+// (3 d x r fp16) from L2 between the waves of tiles that re-read it.
+__device__ __forceinline__ uint64_t evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+__device__ __forceinline__ void st_v4_ef(void *p, uint4 v, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v4.b32 [%0], {%1, %2, %3, %4}, %5;"
+                 ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "l"(pol)
+                 : "memory");
+}
+__device__ __forceinline__ void st_u16_ef(void *p, uint16_t v, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.b16 [%0], %1, %2;" ::"l"(p), "h"(v), "l"(pol) : "memory");
+}
+
 // fp16 conversion with the range guard of the materialised operands: a value
 // beyond +-65504 (fp16's largest finite) is saturated to it and `over` is set
 // (the caller flags kErrRange once), so nothing becomes inf silently.
@@ -63,6 +80,7 @@ constexpr int kDh = 128;                // head size of the attention kernel
 
 // ---- Q/K/V GEMM
 constexpr int kGemmN = 256, kGemmK = 64;
+constexpr int kGemmGroupM = 38;         // row tiles per rasterisation group of qkv_gemm
 constexpr int kGemmStageA = kRowTile * kGemmK * 2;       // 16 KiB
 constexpr int kGemmStageB = kGemmN * kGemmK * 2;         // 32 KiB
 constexpr int kGemmStages = 4;
@@ -177,6 +195,19 @@ lat_prep_kernel(CacheView c, PrefillBlocks bl, int R, __half *__restrict__ A, fl
     *reinterpret_cast<uint4 *>(A + size_t(row) * r + j) = o;
 }
 
+// Tile t -> (first row m0, first column n0).  Groups of kGemmGroupM row tiles
+// (the last group may be shorter); within a group the row tile runs fastest.
+// With 152 CTAs in flight a wave covers about four column tiles of one group:
+// ~4 MiB of Ut and the group's 19 MiB of A rows, so each A row tile is read
+// from DRAM once and Ut once per group instead of once per wave.
+__device__ __forceinline__ void gemm_tile(int t, int tiles_m, int tiles_n, int &m0, int &n0) {
+    const int per_group = pf::kGemmGroupM * tiles_n;
+    const int g = t / per_group, idx = t - g * per_group;
+    const int gm = min(pf::kGemmGroupM, tiles_m - g * pf::kGemmGroupM);
+    m0 = (g * pf::kGemmGroupM + idx % gm) * pf::kRowTile;
+    n0 = (idx / gm) * pf::kGemmN;
+}
+
 // ---------------------------------------------------------------------------
 // Q | K | V^T = (A [R, r] x Ut^T [r, 3d]) * rs[row], fp16 out
 // ---------------------------------------------------------------------------
@@ -184,10 +215,12 @@ __global__ void __launch_bounds__(pf::kGemmThreads, 1)
 qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b, int R, int r,
                 int d, const float *__restrict__ rs, __half *__restrict__ Qm, __half *__restrict__ Km,
                 __half *__restrict__ Vt, int *err) {
-    // Persistent: CTA c takes tiles c, c + gridDim.x, ... (N fastest, so the
-    // CTAs in flight share A rows and all of Ut stays in L2).  Two tensor-memory
-    // accumulators alternate between a CTA's tiles, so the epilogue of one tile
-    // overlaps the main loop of the next.
+    // Persistent: CTA c takes tiles c, c + gridDim.x, ...  Tiles are numbered
+    // in groups of kGemmGroupM row tiles, row fastest within a group (see
+    // gemm_tile), so the CTAs in flight share a few Ut column tiles and a group's
+    // A rows stay in L2 while its Ut columns stream past once.  Two
+    // tensor-memory accumulators alternate between a CTA's tiles, so the
+    // epilogue of one tile overlaps the main loop of the next.
     using namespace pf;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -197,7 +230,7 @@ qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant
     __shared__ uint32_t tmem_base;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n_k = r / kGemmK;
-    const int tiles_n = 3 * d / kGemmN, n_tiles = (R / kRowTile) * tiles_n;
+    const int tiles_m = R / kRowTile, tiles_n = 3 * d / kGemmN, n_tiles = tiles_m * tiles_n;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kGemmStages; ++s) {
@@ -225,7 +258,8 @@ qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant
             int it = 0;                                       // k-stages issued by this CTA so far
             bool ok = true;
             for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-                const int m0 = (t / tiles_n) * kRowTile, n0 = (t % tiles_n) * kGemmN;
+                int m0, n0;
+                gemm_tile(t, tiles_m, tiles_n, m0, n0);
                 for (int i = 0; i < n_k; ++i, ++it) {
                     const int s = it % kGemmStages;
                     if (it >= kGemmStages && !(ok = tc::wait(&empty_bar[s], ((it / kGemmStages) - 1) & 1, err)))
@@ -263,10 +297,12 @@ qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant
         }
     } else {
         const int quad = warp & 3, col0 = ((warp - 2) >> 2) * 128;
+        const uint64_t pol = evict_first_policy();
         int ti = 0;
         for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++ti) {
             const int buf = ti & 1;
-            const int m0 = (t / tiles_n) * kRowTile, n0 = (t % tiles_n) * kGemmN;
+            int m0, n0;
+            gemm_tile(t, tiles_m, tiles_n, m0, n0);
             const int row = m0 + quad * 32 + lane;
             if (!tc::wwait(&acc_full[buf], (ti >> 1) & 1, err)) break;
             tc::fence_after();
@@ -289,14 +325,14 @@ qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant
                 if (part < 2) {
                     uint4 *dst = reinterpret_cast<uint4 *>((part == 0 ? Qm : Km) + size_t(row) * d + cbase + j0);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) dst[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+                    for (int q = 0; q < 4; ++q) st_v4_ef(dst + q, make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]), pol);
                 } else {
                     // V^T: lanes hold consecutive rows, so each column's 32 stores are contiguous
                     uint16_t *dst = reinterpret_cast<uint16_t *>(Vt) + size_t(cbase + j0) * R + row;
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
-                        dst[size_t(2 * j) * R] = uint16_t(h[j] & 0xffffu);
-                        dst[size_t(2 * j + 1) * R] = uint16_t(h[j] >> 16);
+                        st_u16_ef(dst + size_t(2 * j) * R, uint16_t(h[j] & 0xffffu), pol);
+                        st_u16_ef(dst + size_t(2 * j + 1) * R, uint16_t(h[j] >> 16), pol);
                     }
                 }
             }
