@@ -24,14 +24,17 @@
 //                    token scale and writes Q and K row-major, V transposed
 //                    ([d, R], so that a key tile of V is K-major for the
 //                    attention's second product), all fp16
-//   fa_kernel        one CTA per (128-query tile, head): S = Q K^T into
-//                    tensor memory (two buffers), causal mask and online
-//                    softmax in registers (thread = query row), P (fp16)
-//                    into tensor memory, O += P V with A from tensor memory;
-//                    O is rescaled only when a row's running maximum grows
-//                    by more than 2^8 (otherwise the stale maximum keeps
-//                    every p below 2^8); K and V stream through rings of
-//                    3 and 2 tiles.
+//   fa_kernel        one CTA per (pair of 128-query tiles A and B of a
+//                    block, head), both tiles against each K/V tile the CTA
+//                    loads: S_x = Q_x K^T into tensor memory, causal mask and
+//                    online softmax in registers (4 warps per tile, thread =
+//                    query row), P_x (fp16) over S_x's columns, O_x += P_x V
+//                    with A from tensor memory.  While one tile's softmax
+//                    runs, the tensor pipe works on the other tile's
+//                    products.  O_x is rescaled only when a row's running
+//                    maximum grows by more than 2^8 (otherwise the stale
+//                    maximum keeps every p below 2^8); K and V stream through
+//                    rings of 2 and 3 tiles.
 //
 // Every wait is bounded (kErrTimeout on expiry); each CTA frees its tensor
 // memory before it exits.
@@ -89,28 +92,16 @@ constexpr int kGemmThreads = 64 + 32 * kGemmEpiWarps;
 constexpr size_t kGemmSmem = size_t(kGemmStages) * (kGemmStageA + kGemmStageB) + 1024;
 
 // ---- attention
-constexpr int kFaThreads = 384;                          // TMA (Q, K), S MMAs, 8 softmax, TMA (V), PV MMAs
+constexpr int kFaThreads = 384;                          // TMA (Q, K), S MMAs, TMA (V), PV MMAs, 2 x 4 softmax
 constexpr int kTileBytes = kRowTile * kDh * 2;           // 32 KiB: 128 rows x 128 fp16 (two 64-column boxes)
 constexpr int kBox = kRowTile * 128;                     // 16 KiB: one box (128 rows x 128 bytes)
-constexpr int kRingK = 3, kRingV = 2;                    // K tiles are needed two products before V tiles
-constexpr size_t kFaSmem = size_t(1 + kRingK + kRingV) * kTileBytes + 1024;
-constexpr uint32_t kColO = 0, kColS = 128, kColP = 384, kFaTmemCols = 512;   // S, P: two buffers each
+constexpr int kRingK = 2, kRingV = 3;                    // V tiles are needed a softmax later than K tiles
+constexpr size_t kFaSmem = size_t(2 + kRingK + kRingV) * kTileBytes + 1024;
+// tensor memory: O_A, O_B (columns 0..255), S_A, S_B (256..511); P_x overwrites S_x's first 64 columns
+constexpr uint32_t kColO = 0, kColS = 256, kFaTmemCols = 512;
 constexpr float kRescale2 = 8.0f;                        // lazy rescale threshold (log2 units)
 
 }  // namespace pf
-
-// AND of `v` over the 64 threads of named barrier `id` (the two softmax
-// warps of one tensor-memory lane quadrant); also orders their shared-memory
-// accesses like bar.sync.
-__device__ __forceinline__ bool pair_all(bool v, int id) {
-    uint32_t r;
-    asm volatile("{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\tbar.red.and.pred q, %2, 64, p;\n\t"
-                 "selp.u32 %0, 1, 0, q;\n\t}"
-                 : "=r"(r)
-                 : "r"(uint32_t(v)), "r"(id)
-                 : "memory");
-    return r != 0;
-}
 
 // 2^x with the MUFU approximation (relative error about 2^-22; x = -inf and
 // x below the fp32 range give +0).
@@ -351,7 +342,7 @@ qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant
 }
 
 // ---------------------------------------------------------------------------
-// causal attention, one CTA per (128-query tile, head)
+// causal attention, one CTA per (pair of 128-query tiles, head)
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(pf::kFaThreads, 1)
 fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
@@ -360,23 +351,29 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
     using namespace pf;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *sQ = smem;
-    uint8_t *sK = smem + kTileBytes;                         // [kRingK] tiles
+    uint8_t *sQ = smem;                                      // query tiles A and B
+    uint8_t *sK = smem + 2 * kTileBytes;                     // [kRingK] tiles
     uint8_t *sV = sK + size_t(kRingK) * kTileBytes;          // [kRingV] tiles (V^T: dh rows x 128 keys)
     __shared__ __align__(8) uint64_t q_full, k_full[pf::kRingK], k_empty[pf::kRingK], v_full[pf::kRingV],
-        v_empty[pf::kRingV], s_full[2], s_empty[2], p_full[2], o_done[2];
+        v_empty[pf::kRingV], s_full[2], p_full[2], o_done[2];
     __shared__ uint32_t tmem_base;
-    __shared__ float red[2][2][pf::kRowTile];              // partial row maxima [tile parity][half][row]
-    __shared__ float lsum[2][pf::kRowTile];                // partial row sums [half][row]
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    // work unit: query tiles in reverse order (the longest causal rows first)
-    const int tile = int(gridDim.x) - 1 - int(blockIdx.x), h = blockIdx.y;
-    int k = 0;
-    while (k + 1 < bl.n && bl.qtile_off[k + 1] <= tile) ++k;
-    const int qs = bl.t0[k] + (tile - bl.qtile_off[k]) * kRowTile;     // position of the tile's first query
+    // Work unit: query tiles 2u (A) and 2u + 1 (B, absent past the block's
+    // last tile) of one block, units in reverse order (the longest causal rows first).
+    int unit = int(gridDim.x) - 1 - int(blockIdx.x), k = 0;
+    while (k + 1 < bl.n) {
+        const int pairs = (bl.qtile_off[k + 1] - bl.qtile_off[k] + 1) >> 1;
+        if (unit < pairs) break;
+        unit -= pairs;
+        ++k;
+    }
     const int L = bl.L[k], row0 = bl.row_off[k];
-    const int n = min(qs + kRowTile - 1, L - 1) / kRowTile + 1;         // key tiles up to the last query
+    const int qs = bl.t0[k] + 2 * unit * kRowTile;                      // position of tile A's first query
+    const bool has_b = 2 * unit + 1 < bl.qtile_off[k + 1] - bl.qtile_off[k];
+    const int n_a = min(qs + kRowTile - 1, L - 1) / kRowTile + 1;      // key tiles of A
+    const int n_b = has_b ? min(qs + 2 * kRowTile - 1, L - 1) / kRowTile + 1 : 0;   // of B (n_a <= n_b)
+    const int n = max(n_a, n_b);
 
     if (threadIdx.x == 0) {
         mbar_init(&q_full, 1);
@@ -388,11 +385,10 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
             mbar_init(&v_full[s], 1);
             mbar_init(&v_empty[s], 1);
         }
-        for (int s = 0; s < 2; ++s) {
-            mbar_init(&s_full[s], 1);
-            mbar_init(&s_empty[s], 8);
-            mbar_init(&p_full[s], 8);     // P buffer s written (one arrival per softmax warp)
-            mbar_init(&o_done[s], 1);     // the O += P V that read P buffer s has completed
+        for (int x = 0; x < 2; ++x) {
+            mbar_init(&s_full[x], 1);     // S_x of the current key tile is in tensor memory
+            mbar_init(&p_full[x], 4);     // P_x written (one arrival per softmax warp of tile x)
+            mbar_init(&o_done[x], 1);     // O_x += P_x V has completed (S_x / P_x columns free again)
         }
         mbar_init_fence();
         tc::prefetch_map(&map_q);
@@ -406,14 +402,18 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
     const uint32_t tmem = tmem_base;
     pdl_wait();
     pdl_trigger();
-    const int x0 = h * kDh;                                  // head's first column in Q and K, row in V^T
+    const int x0 = blockIdx.y * kDh;                         // head's first column in Q and K, row in V^T
 
+    if (warp < 4) {                                          // warpgroup 0: TMA and MMA issue
     if (warp == 0) {
         // ---------------- TMA producer of Q and K ----------------
         if (lane == 0) {
-            mbar_arrive_expect_tx(&q_full, kTileBytes);
-            tc::tma_load_2d(sQ, &map_q, x0, row0 + qs, &q_full);
-            tc::tma_load_2d(sQ + kBox, &map_q, x0 + 64, row0 + qs, &q_full);
+            mbar_arrive_expect_tx(&q_full, (has_b ? 2 : 1) * kTileBytes);
+            for (int x = 0; x < (has_b ? 2 : 1); ++x) {
+                uint8_t *qd = sQ + size_t(x) * kTileBytes;
+                tc::tma_load_2d(qd, &map_q, x0, row0 + qs + x * kRowTile, &q_full);
+                tc::tma_load_2d(qd + kBox, &map_q, x0 + 64, row0 + qs + x * kRowTile, &q_full);
+            }
             for (int j = 0; j < n; ++j) {
                 const int ks = j % kRingK;
                 if (j >= kRingK && !tc::wait(&k_empty[ks], ((j / kRingK) - 1) & 1, err)) break;
@@ -423,9 +423,8 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
                 tc::tma_load_2d(kd + kBox, &map_k, x0 + 64, row0 + j * kRowTile, &k_full[ks]);
             }
         }
-    } else if (warp == kFaThreads / 32 - 2) {
-        // ---------------- TMA producer of V (its own warp: a V stage frees only
-        // when O += P V has run, which must not hold back the K stream) ----------------
+    } else if (warp == 2) {
+        // ---------------- TMA producer of V ----------------
         if (lane == 0) {
             for (int j = 0; j < n; ++j) {
                 const int vs = j % kRingV;
@@ -437,178 +436,159 @@ fa_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUt
             }
         }
     } else if (warp == 1) {
-        // ---------------- S = Q K^T issuer ----------------
-        // The scores and O += P V are issued from two threads: one thread
-        // spends ~100 cycles per tcgen05.mma, more than a 128 x 128 x 16
-        // product takes, so a single issuer would bound the tensor pipe.  The
-        // two touch disjoint tensor memory (S buffers vs P buffers and O), and
-        // each commit tracks its own thread's products.
+        // ---------------- S_x = Q_x K^T issuer ----------------
+        // S_x of key tile j overwrites P_x of tile j - 1, so it waits for
+        // O_x += P_x V of tile j - 1; the other query tile's products fill the
+        // tensor pipe meanwhile.  The scores and the O products are issued
+        // from two threads (one thread spends ~100 cycles per tcgen05.mma).
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_f16f32(kRowTile);
-            const uint32_t q0 = smem_addr(sQ);
             bool ok = tc::wait(&q_full, 0, err);
             for (int j = 0; j < n && ok; ++j) {
-                const int ks = j % kRingK, sb = j & 1;
+                const int ks = j % kRingK;
                 if (!(ok = tc::wait(&k_full[ks], (j / kRingK) & 1, err))) break;
-                if (j >= 2 && !(ok = tc::wait(&s_empty[sb], ((j >> 1) - 1) & 1, err))) break;
-                tc::fence_after();
                 const uint32_t k0 = smem_addr(sK + size_t(ks) * kTileBytes);
+                for (int x = 0; x < 2 && ok; ++x) {
+                    if (j >= (x ? n_b : n_a)) continue;
+                    if (j > 0 && !(ok = tc::wait(&o_done[x], (j - 1) & 1, err))) break;
+                    tc::fence_after();
+                    const uint32_t q0 = smem_addr(sQ + size_t(x) * kTileBytes);
 #pragma unroll
-                for (int kk = 0; kk < kDh / 16; ++kk) {
-                    const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
-                    tc::mma_ss(tmem + kColS + sb * 128, tc::desc_sw128(q0 + off), tc::desc_sw128(k0 + off), idesc,
-                               kk > 0 ? 1u : 0u);
+                    for (int kk = 0; kk < kDh / 16; ++kk) {
+                        const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
+                        tc::mma_ss(tmem + kColS + x * 128, tc::desc_sw128(q0 + off), tc::desc_sw128(k0 + off),
+                                   idesc, kk > 0 ? 1u : 0u);
+                    }
+                    tc::commit(&s_full[x]);
                 }
-                tc::commit(&s_full[sb]);
                 tc::commit(&k_empty[ks]);
             }
         }
-    } else if (warp == kFaThreads / 32 - 1) {
-        // ---------------- O += P V issuer ----------------
+    } else if (warp == 3) {
+        // ---------------- O_x += P_x V issuer ----------------
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_f16f32(kRowTile);
             bool ok = true;
             for (int j = 0; j < n && ok; ++j) {
-                const int vs = j % kRingV, pb = j & 1;
-                ok = tc::wait(&p_full[pb], (j >> 1) & 1, err) && tc::wait(&v_full[vs], (j / kRingV) & 1, err);
-                if (!ok) break;
-                tc::fence_after();
+                const int vs = j % kRingV;
+                if (!(ok = tc::wait(&v_full[vs], (j / kRingV) & 1, err))) break;
                 const uint32_t v0 = smem_addr(sV + size_t(vs) * kTileBytes);
+                for (int x = 0; x < 2 && ok; ++x) {
+                    if (j >= (x ? n_b : n_a)) continue;
+                    if (!(ok = tc::wait(&p_full[x], j & 1, err))) break;
+                    tc::fence_after();
 #pragma unroll
-                for (int kk = 0; kk < kRowTile / 16; ++kk) {
-                    const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
-                    tc::mma_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8, tc::desc_sw128(v0 + off), idesc,
-                               (j > 0 || kk > 0) ? 1u : 0u);
+                    for (int kk = 0; kk < kRowTile / 16; ++kk) {
+                        const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
+                        tc::mma_ts(tmem + kColO + x * 128, tmem + kColS + x * 128 + kk * 8,
+                                   tc::desc_sw128(v0 + off), idesc, (j > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    tc::commit(&o_done[x]);
                 }
-                tc::commit(&o_done[pb]);
                 tc::commit(&v_empty[vs]);
             }
         }
+    }
     } else {
-        // ---------------- softmax warps 2..9: thread = query row ----------------
-        // Two warps per tensor-memory lane quadrant; warp half h (0 or 1) takes
-        // keys 64h .. 64h+63 of every tile (and O columns 64h .. 64h+63).  The
-        // partners swap their partial row maxima through shared memory (slot
-        // by tile parity) under a 64-thread named barrier, so both hold the
-        // same running maximum m of s * c_log2 (c_log2 > 0); p = 2^(s c_log2 -
-        // m).  P alternates between two tensor-memory buffers, so tile j is
-        // written while O += P_{j-1} V still runs; only a rescale of O waits
-        // for that product.  The partial row sums meet at the end.
-        const int quad = warp & 3, half = (warp - 2) >> 2;
+        // ---------------- softmax warps: 4 per query tile, thread = query row ----------------
+        // Running maximum m of s * c_log2 (c_log2 > 0); p = 2^(s c_log2 - m),
+        // written as fp16 pairs over the first 64 columns of S_x (chunk c of
+        // 32 keys into columns 16c .. 16c+15, which held scores already read).
+        // O_x is rescaled only when m grows by more than kRescale2: it then
+        // holds every product up to tile j - 1, since S_x of tile j was issued
+        // after that product completed.
+        const int x = (warp - 4) >> 2, quad = warp & 3;
+        const int nX = x ? n_b : n_a;
         const int qrow = quad * 32 + lane;
-        const int p = qs + qrow;                                      // query position
+        const int p = qs + x * kRowTile + qrow;                       // query position
         const uint32_t trow = tmem + (uint32_t(quad * 32) << 16);
-        const int bar_id = 1 + quad;                                  // named barrier of the quadrant's pair
+        const uint32_t tS = trow + kColS + x * 128, tO = trow + kColO + x * 128;
         float m = -INFINITY, ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
         bool ok = true;
-        // Both warps of a pair run the same iterations: the outcome of every
-        // bounded wait is AND-reduced over the pair at the exchange barrier, and
-        // a failure ends the loop for both there, so neither is ever left alone
-        // at a named barrier.
-        for (int j = 0; j < n; ++j) {
-            const int sb = j & 1, pb = j & 1;
-            const bool got = ok && tc::wwait(&s_full[sb], (j >> 1) & 1, err);
-            uint32_t v[2][32];
-            float mt = -INFINITY;
-            if (got) {
-                tc::fence_after();
+        for (int j = 0; j < nX; ++j) {
+            if (!(ok = tc::wwait(&s_full[x], j & 1, err))) break;
+            tc::fence_after();
+            const int kmax = p - j * kRowTile;                        // keys 0 .. kmax of this tile are visible
+            uint32_t v[4][32];                                        // the row's 128 scores, one load round trip
 #pragma unroll
-                for (int q = 0; q < 2; ++q) tc::tmem_ld32(trow + kColS + sb * 128 + half * 64 + q * 32, v[q]);
-                tc::tmem_wait_ld();
-                tc::fence_before();
-                __syncwarp();
-                if (lane == 0) tc::arrive(&s_empty[sb]);
-                const int kmax = p - j * kRowTile - half * 64;        // keys 0 .. kmax of this half are visible
-                if (kmax < 63) {
+            for (int c = 0; c < 4; ++c) tc::tmem_ld32(tS + c * 32, v[c]);
+            tc::tmem_wait_ld();
+            if (kmax < 127) {
 #pragma unroll
-                    for (int i = 0; i < 64; ++i)
-                        if (i > kmax) v[i >> 5][i & 31] = __float_as_uint(-INFINITY);
-                }
-                float mx[4];                                          // chain e: keys i = e (mod 4), then a tree
-#pragma unroll
-                for (int e = 0; e < 4; ++e) mx[e] = __uint_as_float(v[0][e]);
-#pragma unroll
-                for (int i = 4; i < 64; ++i) mx[i & 3] = fmaxf(mx[i & 3], __uint_as_float(v[i >> 5][i & 31]));
-                mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+                for (int i = 0; i < 128; ++i)
+                    if (i > kmax) v[i >> 5][i & 31] = __float_as_uint(-INFINITY);
             }
-            red[j & 1][half][qrow] = mt;
-            ok = pair_all(got, bar_id);
-            if (!ok) break;
-            mt = fmaxf(mt, red[j & 1][half ^ 1][qrow]);
+            float mx[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) mx[e] = __uint_as_float(v[0][e]);
+#pragma unroll
+            for (int i = 4; i < 128; ++i) mx[i & 3] = fmaxf(mx[i & 3], __uint_as_float(v[i >> 5][i & 31]));
+            const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
             const float m_new = fmaxf(m, mt * c_log2);
+            bool rescale = false;                                     // some row of the warp rescales O_x
+            float alpha = 1.0f;
             if (j > 0) {
                 const bool need = m_new > m + kRescale2;
-                if (__any_sync(0xffffffffu, need)) {
-                    // O must hold every product up to tile j-1 before it is scaled
-                    ok = tc::wwait(&o_done[pb ^ 1], ((j - 1) >> 1) & 1, err);
-                    if (ok) {
-                        tc::fence_after();
-                        const float alpha = need ? ex2_approx(m - m_new) : 1.0f;
-#pragma unroll 1
-                        for (int q = 0; q < 2; ++q) {
-                            uint32_t o[32];
-                            tc::tmem_ld32(trow + kColO + half * 64 + q * 32, o);
-                            tc::tmem_wait_ld();
+                rescale = __any_sync(0xffffffffu, need);
+                if (need) {
+                    alpha = ex2_approx(m - m_new);
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                            tc::tmem_st32(trow + kColO + half * 64 + q * 32, o);
-                        }
-                        tc::tmem_wait_st();
-                        if (need) {
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) ls[e] *= alpha;
-                            m = m_new;
-                        }
-                    }
+                    for (int e = 0; e < 4; ++e) ls[e] *= alpha;
+                    m = m_new;
                 }
             } else {
                 m = m_new;
             }
-            if (ok && j >= 2) {                                       // P buffer pb was read by O += P_{j-2} V
-                ok = tc::wwait(&o_done[pb], ((j - 2) >> 1) & 1, err);
-                if (ok) tc::fence_after();
-            }
-            if (ok) {
-                uint32_t pk[32];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {                        // column i of this half: keys 64 half + 2i, +1
-                    const float a = ex2_approx(fmaf(__uint_as_float(v[(2 * i) >> 5][(2 * i) & 31]), c_log2, -m));
-                    const float b =
-                        ex2_approx(fmaf(__uint_as_float(v[(2 * i + 1) >> 5][(2 * i + 1) & 31]), c_log2, -m));
+            for (int c = 0; c < 4; ++c) {
+                uint32_t pk[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const float a = ex2_approx(fmaf(__uint_as_float(v[c][2 * i]), c_log2, -m));
+                    const float b = ex2_approx(fmaf(__uint_as_float(v[c][2 * i + 1]), c_log2, -m));
                     ls[(2 * i) & 3] += a;
                     ls[(2 * i + 1) & 3] += b;
                     const __half2 hp = __floats2half2_rn(a, b);
                     pk[i] = *reinterpret_cast<const uint32_t *>(&hp);
                 }
-                tc::tmem_st32(trow + kColP + pb * 64 + half * 32, pk);
-                tc::tmem_wait_st();
-                tc::fence_before();
-                __syncwarp();
-                if (lane == 0) tc::arrive(&p_full[pb]);
+                tc::tmem_st16(tS + c * 16, pk);
             }
-        }
-        // both halves' sums of the row (the pair leaves the loop together)
-        float l = (ls[0] + ls[1]) + (ls[2] + ls[3]);
-        lsum[half][qrow] = l;
-        ok = pair_all(ok, bar_id);
-        l += lsum[half ^ 1][qrow];
-        if (ok) ok = tc::wwait(&o_done[(n - 1) & 1], ((n - 1) >> 1) & 1, err);
-        tc::fence_after();
-        if (ok) {
-            const float inv = 1.0f / l;
-            const bool live = p < L;
-            float *out = O + (size_t(bl.out_off[k]) + (p - bl.t0[k])) * d + x0 + half * 64;
+            if (rescale) {                                            // before O_x += P_x V of this tile
 #pragma unroll 1
-            for (int q = 0; q < 2; ++q) {
-                uint32_t v[32];
-                tc::tmem_ld32(trow + kColO + half * 64 + q * 32, v);
-                tc::tmem_wait_ld();
-                if (live) {
+                for (int q = 0; q < 8; ++q) {
+                    uint32_t o[16];
+                    tc::tmem_ld16(tO + q * 16, o);
+                    tc::tmem_wait_ld();
 #pragma unroll
-                    for (int i = 0; i < 32; i += 4)
-                        *reinterpret_cast<float4 *>(out + q * 32 + i) =
-                            make_float4(__uint_as_float(v[i]) * inv, __uint_as_float(v[i + 1]) * inv,
-                                        __uint_as_float(v[i + 2]) * inv, __uint_as_float(v[i + 3]) * inv);
+                    for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                    tc::tmem_st16(tO + q * 16, o);
+                }
+            }
+            tc::tmem_wait_st();
+            tc::fence_before();
+            __syncwarp();
+            if (lane == 0) tc::arrive(&p_full[x]);
+        }
+        if (nX > 0) {
+            const float l = (ls[0] + ls[1]) + (ls[2] + ls[3]);
+            if (ok) ok = tc::wwait(&o_done[x], (nX - 1) & 1, err);
+            tc::fence_after();
+            if (ok) {
+                const float inv = 1.0f / l;
+                const bool live = p < L;
+                float *out = O + (size_t(bl.out_off[k]) + (p - bl.t0[k])) * d + x0;
+#pragma unroll 1
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t v[32];
+                    tc::tmem_ld32(tO + q * 32, v);
+                    tc::tmem_wait_ld();
+                    if (live) {
+#pragma unroll
+                        for (int i = 0; i < 32; i += 4)
+                            *reinterpret_cast<float4 *>(out + q * 32 + i) =
+                                make_float4(__uint_as_float(v[i]) * inv, __uint_as_float(v[i + 1]) * inv,
+                                            __uint_as_float(v[i + 2]) * inv, __uint_as_float(v[i + 3]) * inv);
+                    }
                 }
             }
         }
@@ -693,8 +673,9 @@ cudaError_t launch_prefill_mat(const CacheView &c, const PrefillBlocks &bl, cons
         return cudaErrorInvalidValue;
     if ((e = ensure_smem(fa_kernel, kFaSmem)) != cudaSuccess) return e;
     const float c_log2 = softmax_scale * 1.4426950408889634f;
-    e = launch_pdl(fa_kernel, dim3(bl.qtile_off[bl.n], H), dim3(kFaThreads), kFaSmem, s, mq, mk, mv, bl, d, c_log2, O,
-                   err);
+    int pairs = 0;                                            // query-tile pairs over all blocks
+    for (int k = 0; k < bl.n; ++k) pairs += (bl.qtile_off[k + 1] - bl.qtile_off[k] + 1) / 2;
+    e = launch_pdl(fa_kernel, dim3(pairs, H), dim3(kFaThreads), kFaSmem, s, mq, mk, mv, bl, d, c_log2, O, err);
     prof_mark(s, "fa");
     return e;
 }
