@@ -640,10 +640,11 @@ def prefill_attn_probe(name, iters=3, group_rows=0, path="blocks"):
 
 def importance_probe(iters=3, N=1, m=4096, n=12288, k=4096):
     """Offline Eq. 10 scores of every singular value of a 7B-shaped W_concat
-    (E x 3E, E = 4096) for N calibration gradients: 2 N m n k flops on the
-    fp32 CUDA cores.  Inputs: seeded torch Gaussians (the time does not
-    depend on the values).  Peak: 152 SMs x 128 fp32 lanes x 2 flops x the
-    SM clock (2070 MHz), the CUDA-core fp32 rate."""
+    (E x 3E, E = 4096) for N calibration gradients: 2 N m n k algorithmic
+    flops, done as three tf32 tensor-core products (the 3xTF32 split keeps
+    fp32 accuracy).  Inputs: seeded torch Gaussians (the time does not depend
+    on the values).  Peak: the measured dense bf16 rate x the nominal tf32 /
+    bf16 ratio (1.1 / 2.25 PFLOP/s); frac counts the three tf32 products."""
     import torch
     import paper_2510_16292_gb300 as q
     dev = torch.device("cuda", torch.cuda.current_device())
@@ -666,11 +667,12 @@ def importance_probe(iters=3, N=1, m=4096, n=12288, k=4096):
     q.qsvd_check()
     t = min(times)
     flops = 2.0 * N * m * n * k
-    sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    peak = sms * 128 * 2 * 2.07e9 / 1e12
+    _, bf16_peak, kind = peaks()
+    peak = bf16_peak * 1.1 / 2.25
     return {"importance_scores": f"N={N} m={m} n={n} k={k}", "ms": round(t * 1e3, 3),
-            "tflops": round(flops / t / 1e12, 2), "bound": "alu", "peak_tflops": round(peak, 1),
-            "frac": round(flops / t / 1e12 / peak, 4), "peak_kind": "derived: SMs x 128 fp32 lanes x 2 x 2070 MHz"}
+            "tflops": round(flops / t / 1e12, 2), "tf32_tflops": round(3 * flops / t / 1e12, 2), "bound": "tensor",
+            "peak_tflops": round(peak, 1), "frac": round(3 * flops / t / 1e12 / peak, 4),
+            "peak_kind": f"{kind} bf16 x 1.1 / 2.25 (nominal tf32 / bf16)"}
 
 
 def cross_rank(values, op="max"):

@@ -711,7 +711,7 @@ int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, 
     if (!workspace || workspace_bytes < need)
         return fail(QSVD_ENOSPC, "importance_scores: workspace needs %zu bytes", need);
     prof_mark(stream, "begin");
-    const cudaError_t e = launch_importance(U, sigma, Vt, G, N, m, n, k, scores, static_cast<float *>(workspace), stream);
+    const cudaError_t e = launch_importance(U, sigma, Vt, G, N, m, n, k, scores, static_cast<float *>(workspace), err, stream);
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "importance_scores launch");
 }
 

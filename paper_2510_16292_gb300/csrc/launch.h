@@ -211,7 +211,7 @@ size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
 // Eq. 10 importance scores (prep_importance.cu); part: [N, ceil(m / 64), k] fp32 scratch.
 constexpr int kImpRowTile = 64;
 cudaError_t launch_importance(const float *U, const float *sigma, const float *Vt, const float *G, int N, int m, int n,
-                              int k, float *scores, float *part, cudaStream_t s);
+                              int k, float *scores, float *part, int *err, cudaStream_t s);
 // Cross-layer rank budget: keep[i] = 1 for the k highest scores (ties: lower i).
 size_t rank_workspace_bytes();
 cudaError_t launch_rank_budget(const float *scores, int n, int k, uint8_t *keep, void *ws, cudaStream_t s);

@@ -4,14 +4,21 @@
 //   score_i = (1/N) sum_n ( sigma_i [U^T G_n V]_{ii} )^2,
 //   [U^T G V]_{ii} = sum_j U[j, i] sum_l G[j, l] V^T[i, l].
 //
-// diag_kernel: one CTA per (64 singular values i, 64 rows j, sample n)
-// accumulates P[j, i] = sum_l G[j, l] V^T[i, l] over 32-wide chunks of l
-// staged in shared memory (each thread a 4 x 4 block of (j, i)), then writes
-// sum_j U[j, i] P[j, i] over its 64 rows as the partial part[n, jt, i] of row
-// tile jt.  score_kernel adds the row tiles in order (the result does not
-// depend on scheduling: the same bits every run), squares and averages.  fp32
-// throughout on the CUDA cores: the gradients need fp32 range, and this runs
-// once per layer offline.
+// diag_tc_kernel (the tensor-core path): one CTA per (128 singular values i,
+// 128 rows j, sample n) forms P^T[i, j] = sum_l V^T[i, l] G[j, l] with
+// tcgen05.mma kind::tf32 in the 3xTF32 split: every fp32 operand x is
+// x_hi + x_lo with x_hi = x with its low 13 mantissa bits cleared (exact in
+// tf32) and x_lo = x - x_hi (exact in fp32), and P^T accumulates
+// hi*hi + hi*lo + lo*hi in fp32 tensor memory (the dropped lo*lo term is below
+// 2^-20 of each product), so the result keeps fp32-level accuracy.  TMA
+// brings 32-column fp32 tiles of both operands; four converter warps split
+// them into hi and lo images in shared memory; the epilogue (thread = i)
+// writes sum_j U[j, i] P^T[i, j] over the CTA's 128 rows as part[n, jt, i].
+// diag_kernel (CUDA cores, for row lengths n that TMA cannot stride: n % 4
+// != 0): one CTA per (64 i, 64 j, n) accumulating P[j, i] over 32-wide
+// chunks of l staged in shared memory (each thread a 4 x 4 block of (j, i)).
+// score_kernel adds the row tiles in order (the result does not depend on
+// scheduling: the same bits every run), squares and averages.
 //
 // The cross-layer rank budget (the global sort of Sec. 3.2) keeps the k
 // highest scores over every layer: rank_hist_kernel / rank_pick_kernel find
@@ -23,6 +30,7 @@
 
 #include "common.cuh"
 #include "launch.h"
+#include "tcgen05.cuh"
 
 namespace qsvd {
 
@@ -78,6 +86,130 @@ diag_kernel(const float *__restrict__ U, const float *__restrict__ Vt, const flo
         for (int y = 0; y < 16; ++y) s += red[y][threadIdx.x];
         const int i = i0 + threadIdx.x;
         if (i < k) part[(size_t(smp) * gridDim.y + blockIdx.y) * k + i] = s;
+    }
+}
+
+namespace imp {
+constexpr int kTile = 128;                                 // i and j per CTA
+constexpr int kKs = 32;                                    // fp32 columns of l per stage (one 128-byte row)
+constexpr int kImg = kTile * kKs * 4;                      // 16 KiB: one operand image of one stage
+constexpr int kStages = 3;
+constexpr int kThreads = 192;                              // TMA, MMA, 4 converter / epilogue warps
+constexpr size_t kSmem = size_t(kStages) * 4 * kImg + 1024; // per stage: A hi, A lo, B hi, B lo
+}  // namespace imp
+
+__global__ void __launch_bounds__(imp::kThreads, 1)
+diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_g,
+               const float *__restrict__ U, int m, int n, int k, float *__restrict__ part, int *err) {
+    using namespace imp;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t full[kStages], conv[kStages], empty[kStages], acc_full;
+    __shared__ uint32_t tmem_base;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int i0 = blockIdx.x * kTile, j0 = blockIdx.y * kTile, smp = blockIdx.z;
+    const int n_k = (n + kKs - 1) / kKs;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);        // both raw tiles landed
+            mbar_init(&conv[s], 4);        // hi / lo images written (one arrival per converter warp)
+            mbar_init(&empty[s], 1);       // the stage's products completed
+        }
+        mbar_init(&acc_full, 1);
+        mbar_init_fence();
+        tc::prefetch_map(&map_v);
+        tc::prefetch_map(&map_g);
+    }
+    if (warp == 1) tc::tmem_alloc(&tmem_base, kTile);
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tmem = tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            for (int it = 0; it < n_k; ++it) {
+                const int s = it % kStages;
+                if (it >= kStages && !tc::wait(&empty[s], ((it / kStages) - 1) & 1, err)) break;
+                uint8_t *st = smem + size_t(s) * 4 * kImg;
+                mbar_arrive_expect_tx(&full[s], 2 * kImg);
+                tc::tma_load_2d(st, &map_v, it * kKs, i0, &full[s]);                       // V^T rows i
+                tc::tma_load_2d(st + 2 * kImg, &map_g, it * kKs, smp * m + j0, &full[s]);  // G_n rows j
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc::idesc_tf32f32(kTile);
+            bool ok = true;
+            for (int it = 0; it < n_k && ok; ++it) {
+                const int s = it % kStages;
+                if (!(ok = tc::wait(&conv[s], (it / kStages) & 1, err))) break;
+                tc::fence_after();
+                const uint32_t a_hi = smem_addr(smem + size_t(s) * 4 * kImg), a_lo = a_hi + kImg;
+                const uint32_t b_hi = a_hi + 2 * kImg, b_lo = a_hi + 3 * kImg;
+#pragma unroll
+                for (int kk = 0; kk < kKs / 8; ++kk) {
+                    const uint32_t o = kk * 32;
+                    tc::mma_ss_tf32(tmem, tc::desc_sw128(a_lo + o), tc::desc_sw128(b_hi + o), idesc,
+                                    (it > 0 || kk > 0) ? 1u : 0u);
+                    tc::mma_ss_tf32(tmem, tc::desc_sw128(a_hi + o), tc::desc_sw128(b_lo + o), idesc, 1u);
+                    tc::mma_ss_tf32(tmem, tc::desc_sw128(a_hi + o), tc::desc_sw128(b_hi + o), idesc, 1u);
+                }
+                tc::commit(&empty[s]);
+            }
+            if (ok) tc::commit(&acc_full);
+        }
+    } else {
+        // converters: the raw tile becomes the hi image in place, the lo image
+        // goes to the next 16 KiB (same byte offsets, so the swizzle carries over)
+        const int ct = threadIdx.x - 64;
+        bool ok = true;
+        for (int it = 0; it < n_k; ++it) {
+            const int s = it % kStages;
+            if (!(ok = tc::wwait(&full[s], (it / kStages) & 1, err))) break;
+            uint8_t *st = smem + size_t(s) * 4 * kImg;
+#pragma unroll 4
+            for (int c = ct; c < 2 * kImg / 16; c += 128) {
+                float4 *hi = reinterpret_cast<float4 *>(st + (c < kImg / 16 ? 0 : 2 * kImg) + size_t(c % (kImg / 16)) * 16);
+                float4 v = *hi, lo;
+                const float4 h = make_float4(__uint_as_float(__float_as_uint(v.x) & 0xFFFFE000u),
+                                             __uint_as_float(__float_as_uint(v.y) & 0xFFFFE000u),
+                                             __uint_as_float(__float_as_uint(v.z) & 0xFFFFE000u),
+                                             __uint_as_float(__float_as_uint(v.w) & 0xFFFFE000u));
+                lo = make_float4(v.x - h.x, v.y - h.y, v.z - h.z, v.w - h.w);
+                *hi = h;
+                *reinterpret_cast<float4 *>(reinterpret_cast<uint8_t *>(hi) + kImg) = lo;
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // generic writes -> tensor core reads
+            __syncwarp();
+            if (lane == 0) tc::arrive(&conv[s]);
+        }
+        // epilogue: thread = singular value i (tensor-memory lane), 128 columns j
+        const int quad = warp & 3, i = i0 + quad * 32 + lane;
+        if (ok) ok = tc::wwait(&acc_full, 0, err);
+        tc::fence_after();
+        if (ok) {
+            float acc = 0.0f;
+#pragma unroll 1
+            for (int q = 0; q < kTile / 32; ++q) {
+                uint32_t v[32];
+                tc::tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + q * 32, v);
+                tc::tmem_wait_ld();
+#pragma unroll
+                for (int c = 0; c < 32; ++c) {
+                    const int j = j0 + q * 32 + c;
+                    if (j < m && i < k) acc = fmaf(U[size_t(j) * k + i], __uint_as_float(v[c]), acc);
+                }
+            }
+            if (i < k) part[(size_t(smp) * gridDim.y + blockIdx.y) * k + i] = acc;
+        }
+    }
+    tc::fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc::fence_after();
+        tc::tmem_free(tmem, kTile);
     }
 }
 
@@ -185,10 +317,27 @@ cudaError_t launch_rank_budget(const float *scores, int n, int k, uint8_t *keep,
 }
 
 cudaError_t launch_importance(const float *U, const float *sigma, const float *Vt, const float *G, int N, int m, int n,
-                              int k, float *scores, float *part, cudaStream_t s) {
-    const int jt = (m + kImpTile - 1) / kImpTile;
-    diag_kernel<<<dim3((k + kImpTile - 1) / kImpTile, jt, N), 256, 0, s>>>(U, Vt, G, m, n, k, part);
-    cudaError_t e = cudaGetLastError();
+                              int k, float *scores, float *part, int *err, cudaStream_t s) {
+    int jt;
+    cudaError_t e;
+    CUtensorMap mv, mg;
+    // TMA needs 16-byte row strides (n % 4 == 0) and 16-byte aligned bases
+    const bool tc_path = n % 4 == 0 && (reinterpret_cast<uintptr_t>(Vt) & 15) == 0 &&
+                         (reinterpret_cast<uintptr_t>(G) & 15) == 0 && tensor_maps_available() &&
+                         encode_map_2d(&mv, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Vt, uint64_t(n), uint64_t(k),
+                                       uint64_t(n) * 4, imp::kKs, imp::kTile, CU_TENSOR_MAP_SWIZZLE_128B) &&
+                         encode_map_2d(&mg, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, G, uint64_t(n), uint64_t(N) * m,
+                                       uint64_t(n) * 4, imp::kKs, imp::kTile, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (tc_path) {
+        jt = (m + imp::kTile - 1) / imp::kTile;
+        if ((e = ensure_smem(diag_tc_kernel, imp::kSmem)) != cudaSuccess) return e;
+        diag_tc_kernel<<<dim3((k + imp::kTile - 1) / imp::kTile, jt, N), imp::kThreads, imp::kSmem, s>>>(
+            mv, mg, U, m, n, k, part, err);
+    } else {
+        jt = (m + kImpTile - 1) / kImpTile;
+        diag_kernel<<<dim3((k + kImpTile - 1) / kImpTile, jt, N), 256, 0, s>>>(U, Vt, G, m, n, k, part);
+    }
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     prof_mark(s, "importance_diag");
     score_kernel<<<(k + 127) / 128, 128, 0, s>>>(part, sigma, N, k, jt, scores);

@@ -32,13 +32,28 @@ def _problem(N, m, n, k, seed):
 @pytest.mark.parametrize("N,m,n,k", [(1, 64, 32, 64), (3, 200, 150, 70), (2, 96, 300, 129),
                                      (2, 1024, 3072, 1024)])
 def test_importance_scores_match_oracle(N, m, n, k):
-    """Tiles of 64 singular values and 64 rows with ragged edges, k > n and
-    k < n, and a joint-QKV-like shape (n = 3m) with 16 row tiles."""
+    """Ragged tiles (128 singular values and 128 rows per tensor-core CTA, 64
+    on the CUDA-core path that n = 150 takes), k > n and k < n, and a
+    joint-QKV-like shape (n = 3m) with 8 row tiles."""
     U, s, Vt, G = _problem(N, m, n, k, seed=N * 1000 + m)
     got = q().qsvd_importance_scores(f32(U), f32(s), f32(Vt), f32(G)).cpu().numpy().astype(np.float64)
     q().qsvd_check()
     want = rank.importance_scores(r32(U), r32(s), r32(Vt), [r32(g) for g in G])
     np.testing.assert_allclose(got, want, rtol=1e-4, atol=1e-4 * want.max())
+
+
+def test_importance_scores_bench_shape_sampled():
+    """The 7B joint-QKV shape the bench times (m = 4096, n = 3 x 4096,
+    k = 4096, one sample) on the tensor-core path; 96 singular values
+    checked against the oracle (a score depends only on its own singular
+    triplet and G, so the oracle runs on that subset)."""
+    N, m, n, k = 1, 4096, 12288, 4096
+    U, s, Vt, G = _problem(N, m, n, k, seed=11)
+    got = q().qsvd_importance_scores(f32(U), f32(s), f32(Vt), f32(G)).cpu().numpy().astype(np.float64)
+    q().qsvd_check()
+    idx = np.unique(np.concatenate([np.arange(32), np.random.default_rng(5).choice(k, 64, replace=False)]))
+    want = rank.importance_scores(r32(U[:, idx]), r32(s[idx]), r32(Vt[idx]), [r32(g) for g in G])
+    np.testing.assert_allclose(got[idx], want, rtol=1e-4, atol=1e-4 * want.max())
 
 
 def test_importance_scores_deterministic_and_budget_boundary():
