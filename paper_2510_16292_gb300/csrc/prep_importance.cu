@@ -90,12 +90,15 @@ diag_kernel(const float *__restrict__ U, const float *__restrict__ Vt, const flo
 }
 
 namespace imp {
-constexpr int kTile = 128;                                 // i and j per CTA
+constexpr int kTile = 128;                                 // i per CTA (tensor-memory lanes)
+constexpr int kTileJ = 256;                                // j per CTA (accumulator columns)
 constexpr int kKs = 32;                                    // fp32 columns of l per stage (one 128-byte row)
-constexpr int kImg = kTile * kKs * 4;                      // 16 KiB: one operand image of one stage
-constexpr int kStages = 3;
+constexpr int kImg = kTile * kKs * 4;                      // 16 KiB: one image of the A (V^T) tile of a stage
+constexpr int kImgB = kTileJ * kKs * 4;                    // 32 KiB: one image of the B (G) tile
+constexpr int kStages = 2;
 constexpr int kThreads = 192;                              // TMA, MMA, 4 converter / epilogue warps
-constexpr size_t kSmem = size_t(kStages) * 4 * kImg + 1024; // per stage: A hi, A lo, B hi, B lo
+constexpr int kStage = 2 * kImg + 2 * kImgB;               // per stage: A hi, A lo, B hi, B lo
+constexpr size_t kSmem = size_t(kStages) * kStage + 1024;
 }  // namespace imp
 
 __global__ void __launch_bounds__(imp::kThreads, 1)
@@ -107,7 +110,7 @@ diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant_
     __shared__ __align__(8) uint64_t full[kStages], conv[kStages], empty[kStages], acc_full;
     __shared__ uint32_t tmem_base;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int i0 = blockIdx.x * kTile, j0 = blockIdx.y * kTile, smp = blockIdx.z;
+    const int i0 = blockIdx.x * kTile, j0 = blockIdx.y * kTileJ, smp = blockIdx.z;
     const int n_k = (n + kKs - 1) / kKs;
 
     if (threadIdx.x == 0) {
@@ -121,7 +124,7 @@ diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant_
         tc::prefetch_map(&map_v);
         tc::prefetch_map(&map_g);
     }
-    if (warp == 1) tc::tmem_alloc(&tmem_base, kTile);
+    if (warp == 1) tc::tmem_alloc(&tmem_base, kTileJ);
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
@@ -132,22 +135,22 @@ diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant_
             for (int it = 0; it < n_k; ++it) {
                 const int s = it % kStages;
                 if (it >= kStages && !tc::wait(&empty[s], ((it / kStages) - 1) & 1, err)) break;
-                uint8_t *st = smem + size_t(s) * 4 * kImg;
-                mbar_arrive_expect_tx(&full[s], 2 * kImg);
+                uint8_t *st = smem + size_t(s) * kStage;
+                mbar_arrive_expect_tx(&full[s], kImg + kImgB);
                 tc::tma_load_2d(st, &map_v, it * kKs, i0, &full[s]);                       // V^T rows i
                 tc::tma_load_2d(st + 2 * kImg, &map_g, it * kKs, smp * m + j0, &full[s]);  // G_n rows j
             }
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            constexpr uint32_t idesc = tc::idesc_tf32f32(kTile);
+            constexpr uint32_t idesc = tc::idesc_tf32f32(kTileJ);
             bool ok = true;
             for (int it = 0; it < n_k && ok; ++it) {
                 const int s = it % kStages;
                 if (!(ok = tc::wait(&conv[s], (it / kStages) & 1, err))) break;
                 tc::fence_after();
-                const uint32_t a_hi = smem_addr(smem + size_t(s) * 4 * kImg), a_lo = a_hi + kImg;
-                const uint32_t b_hi = a_hi + 2 * kImg, b_lo = a_hi + 3 * kImg;
+                const uint32_t a_hi = smem_addr(smem + size_t(s) * kStage), a_lo = a_hi + kImg;
+                const uint32_t b_hi = a_hi + 2 * kImg, b_lo = b_hi + kImgB;
 #pragma unroll
                 for (int kk = 0; kk < kKs / 8; ++kk) {
                     const uint32_t o = kk * 32;
@@ -168,10 +171,11 @@ diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant_
         for (int it = 0; it < n_k; ++it) {
             const int s = it % kStages;
             if (!(ok = tc::wwait(&full[s], (it / kStages) & 1, err))) break;
-            uint8_t *st = smem + size_t(s) * 4 * kImg;
+            uint8_t *st = smem + size_t(s) * kStage;
 #pragma unroll 4
-            for (int c = ct; c < 2 * kImg / 16; c += 128) {
-                float4 *hi = reinterpret_cast<float4 *>(st + (c < kImg / 16 ? 0 : 2 * kImg) + size_t(c % (kImg / 16)) * 16);
+            for (int c = ct; c < (kImg + kImgB) / 16; c += 128) {
+                const bool a = c < kImg / 16;                          // A chunks, then B chunks
+                float4 *hi = reinterpret_cast<float4 *>(st + (a ? size_t(c) * 16 : 2 * kImg + size_t(c - kImg / 16) * 16));
                 float4 v = *hi, lo;
                 const float4 h = make_float4(__uint_as_float(__float_as_uint(v.x) & 0xFFFFE000u),
                                              __uint_as_float(__float_as_uint(v.y) & 0xFFFFE000u),
@@ -179,7 +183,7 @@ diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant_
                                              __uint_as_float(__float_as_uint(v.w) & 0xFFFFE000u));
                 lo = make_float4(v.x - h.x, v.y - h.y, v.z - h.z, v.w - h.w);
                 *hi = h;
-                *reinterpret_cast<float4 *>(reinterpret_cast<uint8_t *>(hi) + kImg) = lo;
+                *reinterpret_cast<float4 *>(reinterpret_cast<uint8_t *>(hi) + (a ? kImg : kImgB)) = lo;
             }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // generic writes -> tensor core reads
             __syncwarp();
@@ -192,7 +196,7 @@ diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant_
         if (ok) {
             float acc = 0.0f;
 #pragma unroll 1
-            for (int q = 0; q < kTile / 32; ++q) {
+            for (int q = 0; q < kTileJ / 32; ++q) {
                 uint32_t v[32];
                 tc::tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + q * 32, v);
                 tc::tmem_wait_ld();
@@ -209,7 +213,7 @@ diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant_
     __syncthreads();
     if (warp == 1) {
         tc::fence_after();
-        tc::tmem_free(tmem, kTile);
+        tc::tmem_free(tmem, kTileJ);
     }
 }
 
@@ -327,9 +331,9 @@ cudaError_t launch_importance(const float *U, const float *sigma, const float *V
                          encode_map_2d(&mv, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Vt, uint64_t(n), uint64_t(k),
                                        uint64_t(n) * 4, imp::kKs, imp::kTile, CU_TENSOR_MAP_SWIZZLE_128B) &&
                          encode_map_2d(&mg, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, G, uint64_t(n), uint64_t(N) * m,
-                                       uint64_t(n) * 4, imp::kKs, imp::kTile, CU_TENSOR_MAP_SWIZZLE_128B);
+                                       uint64_t(n) * 4, imp::kKs, imp::kTileJ, CU_TENSOR_MAP_SWIZZLE_128B);
     if (tc_path) {
-        jt = (m + imp::kTile - 1) / imp::kTile;
+        jt = (m + imp::kTileJ - 1) / imp::kTileJ;
         if ((e = ensure_smem(diag_tc_kernel, imp::kSmem)) != cudaSuccess) return e;
         diag_tc_kernel<<<dim3((k + imp::kTile - 1) / imp::kTile, jt, N), imp::kThreads, imp::kSmem, s>>>(
             mv, mg, U, m, n, k, part, err);

@@ -32,9 +32,9 @@ def _problem(N, m, n, k, seed):
 @pytest.mark.parametrize("N,m,n,k", [(1, 64, 32, 64), (3, 200, 150, 70), (2, 96, 300, 129),
                                      (2, 1024, 3072, 1024)])
 def test_importance_scores_match_oracle(N, m, n, k):
-    """Ragged tiles (128 singular values and 128 rows per tensor-core CTA, 64
+    """Ragged tiles (128 singular values and 256 rows per tensor-core CTA, 64
     on the CUDA-core path that n = 150 takes), k > n and k < n, and a
-    joint-QKV-like shape (n = 3m) with 8 row tiles."""
+    joint-QKV-like shape (n = 3m) with 4 row tiles."""
     U, s, Vt, G = _problem(N, m, n, k, seed=N * 1000 + m)
     got = q().qsvd_importance_scores(f32(U), f32(s), f32(Vt), f32(G)).cpu().numpy().astype(np.float64)
     q().qsvd_check()
