@@ -5,7 +5,7 @@
 //   [U^T G V]_{ii} = sum_j U[j, i] sum_l G[j, l] V^T[i, l].
 //
 // diag_tc_kernel (the tensor-core path): one CTA per (128 singular values i,
-// 128 rows j, sample n) forms P^T[i, j] = sum_l V^T[i, l] G[j, l] with
+// 256 rows j, sample n) forms P^T[i, j] = sum_l V^T[i, l] G[j, l] with
 // tcgen05.mma kind::tf32 in the 3xTF32 split: every fp32 operand x is
 // x_hi + x_lo with x_hi = x with its low 13 mantissa bits cleared (exact in
 // tf32) and x_lo = x - x_hi (exact in fp32), and P^T accumulates
