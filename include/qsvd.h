@@ -185,8 +185,12 @@ size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r);
  *   Vt fp32 [k, n] (right singular vectors as rows), G fp32 [N, m, n] (the
  *   loss gradient for each of N calibration samples), scores fp32 [k] out.
  *   workspace: qsvd_importance_workspace_bytes(N, m, k) bytes.
- * fp32 on the CUDA cores; the sums run in a fixed order, so the result is
- * the same bit for bit on every run.  N <= 65535 per call.
+ * The products G_n V run on the tensor cores as three tf32 products per fp32
+ * product (each operand split into a tf32 part and an fp32 remainder), which
+ * keeps fp32-level accuracy; rows of G and Vt need n % 4 == 0 and 16-byte
+ * aligned bases for that path, other shapes run in fp32 on the CUDA cores.
+ * All sums run in a fixed order, so the result is the same bit for bit on
+ * every run.  N <= 65535 per call.
  */
 int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, const float *G, int32_t N, int32_t m,
                            int32_t n, int32_t k, float *scores, void *workspace, size_t workspace_bytes,
