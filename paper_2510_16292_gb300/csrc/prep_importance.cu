@@ -11,8 +11,9 @@
 // tf32) and x_lo = x - x_hi (exact in fp32), and P^T accumulates
 // hi*hi + hi*lo + lo*hi in fp32 tensor memory (the dropped lo*lo term is below
 // 2^-20 of each product), so the result keeps fp32-level accuracy.  TMA
-// brings 32-column fp32 tiles of both operands; four converter warps split
-// them into hi and lo images in shared memory; the epilogue (thread = i)
+// brings 32-column fp32 tiles of both operands; the raw tile is the hi
+// operand as it stands (a tf32 product reads the upper 19 bits of each word),
+// and four converter warps write the lo image beside it; the epilogue (thread = i)
 // writes sum_j U[j, i] P^T[i, j] over the CTA's 128 rows as part[n, jt, i].
 // diag_kernel (CUDA cores, for row lengths n that TMA cannot stride: n % 4
 // != 0): one CTA per (64 i, 64 j, n) accumulating P[j, i] over 32-wide
@@ -164,27 +165,29 @@ diag_tc_kernel(const __grid_constant__ CUtensorMap map_v, const __grid_constant_
             if (ok) tc::commit(&acc_full);
         }
     } else {
-        // converters: the raw tile becomes the hi image in place, the lo image
-        // goes to the next 16 KiB (same byte offsets, so the swizzle carries over)
+        // converters: the raw tile serves as the hi operand (the tf32 product
+        // reads only the upper 19 bits of each fp32 word, x with its low 13
+        // mantissa bits cleared); the lo image x - hi goes to the next image
+        // (same byte offsets, so the swizzle carries over)
         const int ct = threadIdx.x - 64;
         bool ok = true;
+        auto split = [](uint8_t *img, int img_bytes, int ct) {
+#pragma unroll 4
+            for (int c = ct; c < img_bytes / 16; c += 128) {
+                const float4 v = *reinterpret_cast<const float4 *>(img + size_t(c) * 16);
+                const float4 lo = make_float4(v.x - __uint_as_float(__float_as_uint(v.x) & 0xFFFFE000u),
+                                              v.y - __uint_as_float(__float_as_uint(v.y) & 0xFFFFE000u),
+                                              v.z - __uint_as_float(__float_as_uint(v.z) & 0xFFFFE000u),
+                                              v.w - __uint_as_float(__float_as_uint(v.w) & 0xFFFFE000u));
+                *reinterpret_cast<float4 *>(img + img_bytes + size_t(c) * 16) = lo;
+            }
+        };
         for (int it = 0; it < n_k; ++it) {
             const int s = it % kStages;
             if (!(ok = tc::wwait(&full[s], (it / kStages) & 1, err))) break;
             uint8_t *st = smem + size_t(s) * kStage;
-#pragma unroll 4
-            for (int c = ct; c < (kImg + kImgB) / 16; c += 128) {
-                const bool a = c < kImg / 16;                          // A chunks, then B chunks
-                float4 *hi = reinterpret_cast<float4 *>(st + (a ? size_t(c) * 16 : 2 * kImg + size_t(c - kImg / 16) * 16));
-                float4 v = *hi, lo;
-                const float4 h = make_float4(__uint_as_float(__float_as_uint(v.x) & 0xFFFFE000u),
-                                             __uint_as_float(__float_as_uint(v.y) & 0xFFFFE000u),
-                                             __uint_as_float(__float_as_uint(v.z) & 0xFFFFE000u),
-                                             __uint_as_float(__float_as_uint(v.w) & 0xFFFFE000u));
-                lo = make_float4(v.x - h.x, v.y - h.y, v.z - h.z, v.w - h.w);
-                *hi = h;
-                *reinterpret_cast<float4 *>(reinterpret_cast<uint8_t *>(hi) + (a ? kImg : kImgB)) = lo;
-            }
+            split(st, kImg, ct);
+            split(st + 2 * kImg, kImgB, ct);
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // generic writes -> tensor core reads
             __syncwarp();
             if (lane == 0) tc::arrive(&conv[s]);
