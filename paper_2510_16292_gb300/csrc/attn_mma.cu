@@ -432,7 +432,7 @@ bool attn_mma_use(const CacheView &c, int H, int B, int max_seq_len) {
     const int path = attn_path();
     if (path == 1 || path == 2) return false;
     if (path == 3) return true;
-    return int64_t(B) * max_seq_len <= 16384 || !attn_tc_shape_ok(c.r, c.bits, H);
+    return int64_t(B) * max_seq_len <= mma_tokens_max(c.r) || !attn_tc_shape_ok(c.r, c.bits, H);
 }
 
 namespace {

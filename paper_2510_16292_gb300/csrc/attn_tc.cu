@@ -998,7 +998,7 @@ bool attn_tc_shape_ok(int r, int bits, int H) {
 bool attn_tc_use(const CacheView &c, int H, int max_seq_len) {
     if (g_attn_path == 1 || g_attn_path == 3 || !attn_tc_shape_ok(c.r, c.bits, H) || !tensor_maps_available()) return false;
     if (g_attn_path == 2) return true;
-    return int64_t(c.B) * max_seq_len >= 4096;
+    return int64_t(c.B) * max_seq_len > mma_tokens_max(c.r);
 }
 
 int attn_tc_splits(int B, int r, int max_seq_len, int *tiles_per_split) {

@@ -276,6 +276,12 @@ bool attn_tc_shape_ok(int r, int bits, int H);
 bool attn_tc_use(const CacheView &c, int H, int max_seq_len);
 int attn_tc_splits(int B, int r, int max_seq_len, int *tiles_per_split);
 // Warp-level tensor-core attention for small batch x length (attn_mma.cu).
+// The automatic choice takes it while B x L (cached tokens of the step) is at
+// most mma_tokens_max(r), and the tcgen05 kernel above that: the crossover
+// measured on GB300 over B = 1..16, L = 512..4096, r = 1024..3072, int8 and
+// int4 (whole decode steps; the tcgen05 kernel is up to 2.7x faster above it,
+// the warp-level one up to 1.4x faster below it).
+constexpr int64_t mma_tokens_max(int r) { return r <= 2048 ? 2048 : 1024; }
 bool attn_mma_use(const CacheView &c, int H, int B, int max_seq_len);
 bool attn_mma_fits(const CacheView &c, int max_seq_len);
 int attn_mma_splits(const CacheView &c, int B, int H, int max_seq_len, int *ts, int *n_sub);
