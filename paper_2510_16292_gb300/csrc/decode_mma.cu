@@ -1,5 +1,5 @@
 // Tensor-core forms of the per-step up-projection products (a5, a8) for
-// batches of 8 or more sequences.  The batch rows are the M dimension of
+// batches of 5 or more sequences.  The batch rows are the M dimension of
 // mma.sync.m16n8k16 (16 rows per pass), the bf16 up-projection is the B
 // operand, read from its shared-memory tile with ldmatrix, and fp32
 // activations are split into a bf16 part and a bf16 residual (two MMAs; the
@@ -450,10 +450,13 @@ combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ 
 }
 
 // ---------------------------------------------------------------------------
-// Shapes these kernels take: 8 or more sequences, r % 512 == 0 (whole 128-channel
+// Shapes these kernels take: 5 or more sequences, r % 512 == 0 (whole 128-channel
 // groups per qproj rank), dh == 128 (four warps of 32 output columns in combine).
+// From 5 sequences on they beat the CUDA-core forms (measured on GB300: whole
+// decode steps at B = 5 and 6 are 12-17 % faster; at B = 4 the CUDA-core forms
+// win at r = 3072 and at long caches).
 bool decode_mma_supported(int B, int r, int d, int dh) {
-    return B >= 8 && r % 512 == 0 && d % 64 == 0 && dh == 128;
+    return B >= 5 && r % 512 == 0 && d % 64 == 0 && dh == 128;
 }
 
 cudaError_t launch_qproj_mma(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,

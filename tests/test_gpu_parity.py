@@ -194,10 +194,11 @@ def test_decode_batch_ragged_lengths(bits):
         assert_rows_close(o, np.stack([outs[b] for b in range(3)]), f"step {step}")
 
 
-@pytest.mark.parametrize("B,bits", [(9, 8), (17, 4)])
+@pytest.mark.parametrize("B,bits", [(5, 8), (6, 4), (9, 8), (17, 4)])
 def test_decode_large_batch_tensor_core_products(B, bits):
-    """From 8 sequences on, the up-projection products run on the tensor cores
-    (16 sequences per pass: B = 17 takes two passes); ragged lengths."""
+    """From 5 sequences on, the up-projection products run on the tensor cores
+    (16 sequences per pass: B = 5 fills 5 of them, B = 17 takes two passes);
+    ragged lengths."""
     base = synthetic.WORKLOADS["llava7b"]
     wl = synthetic.Workload("batch", base.shape, B=B, n_image=0, n_text=160, decode_steps=2, lat_bits=bits)
     inp = synthetic.gen_layer(wl, seed=21)
