@@ -448,7 +448,8 @@ int qsvd_set_project_epilogue(int32_t mode);
  * Choice of attention kernels for qsvd_latent_decode_attn (a library setting,
  * not part of the paper's method; process-wide, not thread-safe):
  *   0  automatic (default): the warp-level tensor-core kernel when
- *      B * max_seq_len <= 16384 or the tcgen05 kernel cannot take the shape,
+ *      B * max_seq_len <= 2048 (1024 for r > 2048) or the tcgen05 kernel
+ *      cannot take the shape,
  *      else the tcgen05 kernel (the warp-level kernel needs r <= 3072;
  *      beyond that, the CUDA-core kernels);
  *   1  always the CUDA-core kernels;

@@ -305,7 +305,7 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
     const int B = c.B, r = c.r, H = a.H, dh = a.dh, d = H * dh;
     DecodeWs w;
     carve(B, a.max_seq_len, r, H, dh, static_cast<char *>(ws), &w);
-    // the up-projection products on the tensor cores from 8 sequences on
+    // the up-projection products on the tensor cores from 5 sequences on
     // (bf16 weights only: quantized up-projections take the CUDA-core forms at every batch size)
     const bool bf16_up = a.U_q.bits == 16 && a.U_k.bits == 16 && a.U_v.bits == 16;
     const bool mma = bf16_up && decode_mma_supported(B, r, d, dh);
