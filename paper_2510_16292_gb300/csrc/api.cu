@@ -355,12 +355,16 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
     prof_mark(stream, "begin");
     cudaError_t e;
     if (T <= kPsMaxSplitTok && d <= 6144 && d % 256 == 0) {
-        // the quantizer fused into the projection; with H1 the rotation runs once per
-        // row in xquant instead (in every CTA of the projection it measured slower)
+        // one token: the quantizer fused into the projection, then the requantization
+        // kernel; with H1 the rotation runs once per row in xquant instead (in every
+        // CTA of the projection it measured slower)
         if (T < kPsSplitTok && !rot) {
             e = launch_proj_small(X, int(T), d, act_clip, W->codes, W->scale, r, lat_bits, lat_clip, c_hat, counter,
                                   xq_out, xs_out, acc_out, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
-                                  dst_pos, err, stream, nullptr, nullptr, true, act_qmax);
+                                  dst_pos, err, stream, nullptr, nullptr, false, act_qmax);
+            if (e == cudaSuccess)
+                e = launch_requant(c_hat, T, r, lat_bits, lat_clip, lat_codes, lat_scales, dst ? &dv : nullptr, dst_seq,
+                                   dst_pos, err, stream);
             return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "projection launch");
         }
         // each row quantized once, the dot products on the tensor cores, the rows requantized in parallel

@@ -133,10 +133,12 @@ cudaError_t launch_proj_dp4a(const int8_t *xq, int64_t T, int d, const int8_t *w
                              const float *ws, const float *xs, int r, float *c_hat,
                              int32_t *acc_out, cudaStream_t s);
 
-// Decode-size projection: for T < kPsSplitTok a1, a2, a3 and a4 in one launch
-// (`counter` must be zero before the first call; the kernel leaves it at zero);
-// up to kPsMaxSplitTok tokens on codes from xquant (xq_in, xs_in, tail = false),
-// kPsMaxTok tokens per CTA row.
+// Decode-size projection: with `tail`, a1, a2, a3 and a4 in one launch for
+// T < 4 (the last CTA requantizes; `counter` must be zero before the first
+// call, the kernel leaves it at zero); without it, the latent rows go to
+// requant_kernel.  X is quantized by the kernel itself, or taken as codes from
+// xquant (xq_in, xs_in) for up to kPsMaxSplitTok tokens; kPsMaxTok tokens per
+// CTA row.
 constexpr int kPsMaxTok = 16;
 constexpr int kPsMaxSplitTok = 64;
 cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, const int8_t *wcodes,
@@ -147,8 +149,11 @@ cudaError_t launch_proj_small(const uint16_t *X, int T, int d, float act_clip, c
                               bool tail = true, int act_qmax = 127);
 // From this many tokens on, the decode projection runs as three kernels:
 // xquant (one CTA per token), proj_small on the given codes, requant (one CTA
-// per row); below it, proj_small quantizes and requantizes by itself.
-constexpr int kPsSplitTok = 4;
+// per row); below it (one token), proj_small quantizes the row itself and
+// requant_kernel follows.  Measured on GB300 (whole decode steps): at one token
+// this is 1.3 us faster than xquant first and 1.8 us faster than the last CTA
+// of proj_small requantizing; from two tokens on, xquant first is fastest.
+constexpr int kPsSplitTok = 2;
 
 // Exact int8 GEMM on the tensor cores (bf16 images of the codes, fp32 TMEM
 // accumulators drained to int32 every 1024 of K) + the fp32 dequantization.
