@@ -29,6 +29,21 @@ namespace {
 constexpr int kClQ = 4;          // qproj: CTAs per cluster (split of the r latent rows)
 constexpr int kClV = 8;          // combine: CTAs per cluster
 constexpr int kMaxSplitsM = 64;  // softmax partials per sequence
+constexpr int kCmbRows = 64;     // combine: U_v rows per ring slot
+// Ring slots (128-row groups) of the query projection's U_q stream: three
+// while a third of an SM holds them (rs <= 384), else two; never more than the
+// groups.
+__host__ __device__ constexpr int qp_slots(int rs) {
+    const int want = rs <= 384 ? 3 : 2, groups = rs / 128;
+    return groups < want ? groups : want;
+}
+// Ring slots of the combine's U_v stream: three while they fit beside the
+// merged rows in a third of an SM's shared memory (rs <= 192), else two; never
+// more than the chunks.
+__host__ __device__ constexpr int cmb_slots(int rs) {
+    const int want = rs <= 3 * kCmbRows ? 3 : 2, chunks = rs / kCmbRows;
+    return chunks < want ? chunks : want;
+}
 
 __device__ __forceinline__ uint32_t mrank() {
     uint32_t r;
@@ -84,8 +99,11 @@ __device__ __forceinline__ bool mlen_ok(int L, int Tmax) { return L >= 1 && L <=
 // a5, q = c U_q.  Grid (kClQ, d / 64, B / 16), cluster (kClQ, 1, 1), 128 threads.
 // CTA k of a cluster takes latent rows [k rs, (k+1) rs) (rs = r / kClQ, whole
 // 128-channel groups) and the cluster's 64 columns; warp w computes columns
-// 16w .. 16w+15 for 16 sequences per pass; rank k adds the kClQ partials of
-// columns 16k .. 16k+15 in rank order.  CTA (0, 0) also clears qmax.
+// 16w .. 16w+15 for the 16 sequences of its pass (grid z); rank k adds the kClQ
+// partials of columns 16k .. 16k+15 in rank order.  CTA (0, 0) also clears
+// qmax.  The U_q rows stream through a ring of qp_slots(rs) slots of one
+// 128-row group each (the first slots are copied before the wait on the
+// producer grid), so three CTAs share an SM at every rank up to 3072.
 // ---------------------------------------------------------------------------
 __global__ void __cluster_dims__(kClQ, 1, 1) __launch_bounds__(128)
 qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__restrict__ seq_len, int B, int d,
@@ -98,24 +116,29 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     constexpr int kUS = 72;                                                  // padded U row (bf16)
     const int kAS = rs + 8;                                                  // padded A row (bf16)
-    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                      // [rs][kUS]
-    uint16_t *a_s = u_s + size_t(rs) * kUS;                                  // [16][kAS]
+    const int n_slots = qp_slots(rs);
+    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                      // [n_slots][128][kUS]
+    uint16_t *a_s = u_s + size_t(n_slots) * 128 * kUS;                       // [16][kAS]
     float *sc_s = reinterpret_cast<float *>(a_s + 16 * kAS);                 // [16][ngl]
     float *part = sc_s + 16 * ngl;                                           // [16][64]
-    for (int i = tid; i < rs * 8; i += 128) {        // U_q tile: no kernel's output, copied before the wait
-        const int row = i >> 3, k = i & 7;
-        mcp16(u_s + size_t(row) * kUS + 8 * k, Uq + size_t(j0 + row) * d + c0 + 8 * k);
+    auto load_group = [&](int g) {                   // U_q rows [j0 + 128 g, +128), the cluster's 64 columns
+        uint16_t *dst = u_s + size_t(g % n_slots) * 128 * kUS;
+        for (int i = tid; i < 128 * 8; i += 128) {
+            const int row = i >> 3, k = i & 7;
+            mcp16(dst + size_t(row) * kUS + 8 * k, Uq + size_t(j0 + g * 128 + row) * d + c0 + 8 * k);
+        }
+    };
+    for (int g = 0; g < n_slots; ++g) {              // one commit group per slot (U_q is no kernel's output)
+        load_group(g);
+        asm volatile("cp.async.commit_group;" ::: "memory");
     }
-    asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
     pdl_trigger();   // after the wait: the attention kernel two launches on reads the
                      // lengths before its own wait, and they are complete by then
     if (rank == 0 && blockIdx.y == 0 && blockIdx.z == 0)
         for (int i = tid; i < n_qmax; i += 128) qmax[i] = 0u;
-    bool ready = false;
-    for (int b0 = 16 * int(blockIdx.z); b0 < B; b0 += 16 * int(gridDim.z)) {   // grid z: 16-sequence passes
-        const int nb = min(16, B - b0);
-        __syncthreads();
+    {
+        const int b0 = 16 * int(blockIdx.z), nb = min(16, B - b0);
         if (tid < 16) {
             int L = tid < nb ? seq_len[b0 + tid] : 0;
             const int sq = tid < nb ? view_seq(c, b0 + tid) : 0;
@@ -181,21 +204,22 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
                                 : 0.0f;
             }
         }
-        if (!ready) {
-            asm volatile("cp.async.wait_group 0;" ::: "memory");
-            ready = true;
-        }
-        __syncthreads();
         // 16 rows x 16 columns per warp: per 128-channel group, fp32 sums scaled by the group's scale
         float out[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
         const int g8 = lane >> 2;
         for (int g = 0; g < ngl; ++g) {
+            // group g is commit group g; the n_slots - 1 younger groups may still be in flight
+            if (n_slots == 3) asm volatile("cp.async.wait_group 2;" ::: "memory");
+            else if (n_slots == 2) asm volatile("cp.async.wait_group 1;" ::: "memory");
+            else asm volatile("cp.async.wait_group 0;" ::: "memory");
+            __syncthreads();                         // the group (and, the first time, the codes) visible
+            const uint16_t *us = u_s + size_t(g % n_slots) * 128 * kUS;
             float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
 #pragma unroll
             for (int ks = 0; ks < 8; ++ks) {
                 const int k = g * 128 + ks * 16;
                 uint32_t bfr[4], afr[4];
-                ldsm_x4_t(bfr, u_s + size_t(k + (lane & 7) + ((lane >> 3) & 1) * 8) * kUS + 16 * warp + (lane >> 4) * 8);
+                ldsm_x4_t(bfr, us + size_t(ks * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * kUS + 16 * warp + (lane >> 4) * 8);
                 ldsm_x4(afr, a_s + size_t(lane & 15) * kAS + k + (lane >> 4) * 8);
                 mma_bf16(acc[0], afr, bfr[0], bfr[1]);
                 mma_bf16(acc[1], afr, bfr[2], bfr[3]);
@@ -208,6 +232,11 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
                 out[nt][2] = fmaf(s_hi, acc[nt][2], out[nt][2]);
                 out[nt][3] = fmaf(s_hi, acc[nt][3], out[nt][3]);
             }
+            if (g + n_slots < ngl) {
+                __syncthreads();                     // every warp is done with the slot
+                load_group(g + n_slots);
+            }
+            asm volatile("cp.async.commit_group;" ::: "memory");
         }
 #pragma unroll
         for (int nt = 0; nt < 2; ++nt) {
@@ -223,7 +252,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
             for (int k = 0; k < kClQ; ++k) v += mld_rank(part + row * 64 + col, uint32_t(k));
             q[size_t(b0 + row) * d + c0 + col] = v;
         }
-        msync();                                     // partials read before they are overwritten / the CTA exits
+        msync();                                     // partials read before the CTA exits
     }
 }
 
@@ -316,11 +345,17 @@ qabsorb_mma_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk,
 }
 
 // ---------------------------------------------------------------------------
-// a7/a8.  Grid (kClV, H, B / 16), cluster (kClV, 1, 1), 128 threads.  CTA k of head h's
-// cluster merges, for 16 sequences per pass, the softmax partials of latent
-// rows [k rs, (k+1) rs) (weights exp(m_s - M) / l), multiplies them by those
-// rows of U_v[:, h-block] (warp w: output columns 32w .. 32w+31), and rank k
-// adds the kClV products of columns k dh/kClV .. in rank order.
+// a7/a8.  Grid (kClV, H, B / 16), cluster (kClV, 1, 1), 128 threads.  CTA k of
+// head h's cluster merges, for the 16 sequences of its pass (grid z), the
+// softmax partials of latent rows [k rs, (k+1) rs) (weights exp(m_s - M) / l),
+// multiplies them by those rows of U_v[:, h-block] (warp w: output columns
+// 32w .. 32w+31), and rank k adds the kClV products of columns k dh/kClV .. in
+// rank order.  The U_v rows stream through a ring of cmb_slots(rs) slots of
+// kCmbRows rows (the first slots are copied before the wait on the producer
+// grid), so a CTA holds at most ~70 KB of shared memory at every rank up to
+// 3072: three CTAs share an SM and the grid runs as one wave.  Every load of
+// the merge is issued before its results are used (the merge weights of four
+// sequences per warp, the partials of two outputs per thread).
 // ---------------------------------------------------------------------------
 __global__ void __cluster_dims__(kClV, 1, 1) __launch_bounds__(128)
 combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ seq_len,
@@ -328,102 +363,142 @@ combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ 
                    int dh, int r, int chunk, int n_split, const float *__restrict__ pm, const float *__restrict__ pl,
                    const float *__restrict__ po, float *__restrict__ O) {
     extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ float w_s[16][kMaxSplitsM];
     __shared__ float inv_s[16];
     __shared__ int ns_s[16];
     const int rs = r / kClV, d = H * dh, h = blockIdx.y;
+    const int n_ck = rs / kCmbRows, n_slots = cmb_slots(rs);
     const uint32_t rank = mrank();
     const int j0 = int(rank) * rs;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g8 = lane >> 2;
     const int kS = dh + 8, kAS = rs + 8;
-    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                      // [rs][kS]
-    uint16_t *ah_s = u_s + size_t(rs) * kS;                                  // [16][kAS]
+    uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                      // [n_slots][kCmbRows][kS]
+    uint16_t *ah_s = u_s + size_t(n_slots) * kCmbRows * kS;                  // [16][kAS]
     uint16_t *al_s = ah_s + 16 * kAS;                                        // [16][kAS]
     float *part = reinterpret_cast<float *>(al_s + 16 * kAS);                // [16][dh]
+    float *w_s = part;           // [16][kMaxSplitsM] merge weights, dead before part is written
+    const int b0 = 16 * int(blockIdx.z), nb = min(16, B - b0);
+    auto load_chunk = [&](int ck) {                  // U_v rows [j0 + 64 ck, +64) of head h's columns
+        uint16_t *dst = u_s + size_t(ck % n_slots) * kCmbRows * kS;
+        const uint16_t *src = Uv + size_t(j0 + ck * kCmbRows) * d + size_t(h) * dh;
+        for (int i = tid; i < kCmbRows * (dh / 8); i += 128) {
+            const int row = i / (dh / 8), k = i - row * (dh / 8);
+            mcp16(dst + size_t(row) * kS + 8 * k, src + size_t(row) * d + 8 * k);
+        }
+    };
     pdl_trigger();
-    for (int i = tid; i < rs * (dh / 8); i += 128) {     // the U_v tile (before the wait: no kernel writes U_v)
-        const int row = i / (dh / 8), k = i - row * (dh / 8);
-        mcp16(u_s + size_t(row) * kS + 8 * k, Uv + size_t(j0 + row) * d + size_t(h) * dh + 8 * k);
+    for (int ck = 0; ck < n_slots; ++ck) {           // one commit group per slot (U_v is no kernel's output)
+        if (ck < n_ck) load_chunk(ck);
+        asm volatile("cp.async.commit_group;" ::: "memory");
     }
-    asm volatile("cp.async.commit_group;" ::: "memory");
     pdl_wait();
-    bool ready = false;
-    const int per_rank = dh / kClV;
-    for (int b0 = 16 * int(blockIdx.z); b0 < B; b0 += 16 * int(gridDim.z)) {   // grid z: 16-sequence passes
-        const int nb = min(16, B - b0);
-        __syncthreads();
-        // merge weights: warp w takes sequences w, w+4, w+8, w+12
+    // merge weights: warp w takes sequences w, w+4, w+8, w+12; the entries past a
+    // row's splits (allocated, possibly stale) are loaded with the others and masked
+    {
+        int Lk[4];
+        float mk[4][2], lk[4][2];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             const int bi = warp + 4 * k;
-            const int L = bi < nb ? row_len(seq_len, seq_map, nseq, b0 + bi) : 0;
-            const int ns = mlen_ok(L, Tmax) ? (L + chunk - 1) / chunk : 0;
-            const size_t base = size_t(b0 + bi) * n_split * H + h;
-            const float m0 = lane < ns ? pm[base + size_t(lane) * H] : -FLT_MAX;
-            const float m1 = lane + 32 < ns ? pm[base + size_t(lane + 32) * H] : -FLT_MAX;
-            const float l0 = lane < ns ? pl[base + size_t(lane) * H] : 0.0f;
-            const float l1 = lane + 32 < ns ? pl[base + size_t(lane + 32) * H] : 0.0f;
+            const bool row = bi < nb;
+            Lk[k] = row ? row_len(seq_len, seq_map, nseq, b0 + bi) : 0;
+            const size_t base = size_t(b0 + (row ? bi : 0)) * n_split * H + h;
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int s = lane + 32 * u;
+                const bool ok = row && s < n_split;
+                mk[k][u] = ok ? pm[base + size_t(s) * H] : -FLT_MAX;
+                lk[k][u] = ok ? pl[base + size_t(s) * H] : 0.0f;
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int bi = warp + 4 * k;
+            const int L = Lk[k];
+            const int ns = mlen_ok(L, Tmax) ? min((L + chunk - 1) / chunk, n_split) : 0;
+            const float m0 = lane < ns ? mk[k][0] : -FLT_MAX, m1 = lane + 32 < ns ? mk[k][1] : -FLT_MAX;
             const float M = warp_max(fmaxf(m0, m1));
             const float e0 = lane < ns ? expf(m0 - M) : 0.0f;
             const float e1 = lane + 32 < ns ? expf(m1 - M) : 0.0f;
-            w_s[bi][lane] = e0;
-            w_s[bi][lane + 32] = e1;
-            const float l = warp_sum(e0 * l0 + e1 * l1);
+            w_s[bi * kMaxSplitsM + lane] = e0;
+            w_s[bi * kMaxSplitsM + lane + 32] = e1;
+            const float l = warp_sum((lane < ns ? e0 * lk[k][0] : 0.0f) + (lane + 32 < ns ? e1 * lk[k][1] : 0.0f));
             if (lane == 0) {
                 inv_s[bi] = ns ? 1.0f / l : 0.0f;
                 ns_s[bi] = ns;
             }
         }
-        __syncthreads();
-        // merged o_lat rows (this rank's channels) as bf16 part + residual; branch-free partial loads
-        const int nq = rs / 4;
-        for (int it = tid; it < 16 * nq; it += 128) {
-            const int bi = it / nq, q4 = it - bi * nq;
-            const int ns = ns_s[bi];
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (ns > 0) {
-                const float *src = po + (size_t(b0 + bi) * n_split * H + h) * r + j0 + 4 * q4;
-                for (int s0 = 0; s0 < ns; s0 += 8) {
-                    float4 v[8];
-                    float wk[8];
+    }
+    __syncthreads();
+    // merged o_lat rows (this rank's channels) as bf16 part + residual, two outputs per thread
+    const int nq = rs / 4;
+    for (int it0 = tid; it0 < 16 * nq; it0 += 256) {
+        int bi[2], q4[2], ns[2];
+        float4 acc[2];
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        const int sk = s0 + k, sc = sk < ns ? sk : ns - 1;
-                        v[k] = *reinterpret_cast<const float4 *>(src + size_t(sc) * H * r);
-                        wk[k] = sk < ns ? w_s[bi][sc] : 0.0f;
-                    }
+        for (int u = 0; u < 2; ++u) {
+            const int it = it0 + 128 * u;
+            const bool live = it < 16 * nq;
+            bi[u] = live ? it / nq : 0;
+            q4[u] = live ? it - bi[u] * nq : 0;
+            ns[u] = live ? ns_s[bi[u]] : 0;
+            acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        const int nsm = max(ns[0], ns[1]);
+        for (int s0 = 0; s0 < nsm; s0 += 8) {
+            float4 v[2][8];
+            float wk[2][8];
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        acc.x = fmaf(wk[k], v[k].x, acc.x);
-                        acc.y = fmaf(wk[k], v[k].y, acc.y);
-                        acc.z = fmaf(wk[k], v[k].z, acc.z);
-                        acc.w = fmaf(wk[k], v[k].w, acc.w);
-                    }
+            for (int u = 0; u < 2; ++u) {
+                const float *src = po + (size_t(b0 + bi[u]) * n_split * H + h) * r + j0 + 4 * q4[u];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const int sk = s0 + k;
+                    const bool ok = sk < ns[u];
+                    v[u][k] = ok ? *reinterpret_cast<const float4 *>(src + size_t(sk) * H * r) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    wk[u][k] = ok ? w_s[bi[u] * kMaxSplitsM + sk] : 0.0f;
                 }
             }
-            const float il = inv_s[bi];
-            uint32_t h0, l0, h1, l1;
-            split2(acc.x * il, acc.y * il, h0, l0);
-            split2(acc.z * il, acc.w * il, h1, l1);
-            *reinterpret_cast<uint2 *>(ah_s + size_t(bi) * kAS + 4 * q4) = make_uint2(h0, h1);
-            *reinterpret_cast<uint2 *>(al_s + size_t(bi) * kAS + 4 * q4) = make_uint2(l0, l1);
-        }
-        if (!ready) {
-            asm volatile("cp.async.wait_group 0;" ::: "memory");
-            ready = true;
-        }
-        __syncthreads();
-        float acc[4][4];
 #pragma unroll
-        for (int nt = 0; nt < 4; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.0f;
-        for (int ks = 0; ks < rs / 16; ++ks) {
+            for (int u = 0; u < 2; ++u)
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    acc[u].x = fmaf(wk[u][k], v[u][k].x, acc[u].x);
+                    acc[u].y = fmaf(wk[u][k], v[u][k].y, acc[u].y);
+                    acc[u].z = fmaf(wk[u][k], v[u][k].z, acc[u].z);
+                    acc[u].w = fmaf(wk[u][k], v[u][k].w, acc[u].w);
+                }
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            if (it0 + 128 * u >= 16 * nq) break;
+            const float il = inv_s[bi[u]];
+            uint32_t h0, l0, h1, l1;
+            split2(acc[u].x * il, acc[u].y * il, h0, l0);
+            split2(acc[u].z * il, acc[u].w * il, h1, l1);
+            *reinterpret_cast<uint2 *>(ah_s + size_t(bi[u]) * kAS + 4 * q4[u]) = make_uint2(h0, h1);
+            *reinterpret_cast<uint2 *>(al_s + size_t(bi[u]) * kAS + 4 * q4[u]) = make_uint2(l0, l1);
+        }
+    }
+    float acc[4][4];
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.0f;
+    for (int ck = 0; ck < n_ck; ++ck) {
+        // chunk ck is commit group ck; the n_slots - 1 younger groups may still be in flight
+        if (n_slots == 3) asm volatile("cp.async.wait_group 2;" ::: "memory");
+        else if (n_slots == 2) asm volatile("cp.async.wait_group 1;" ::: "memory");
+        else asm volatile("cp.async.wait_group 0;" ::: "memory");
+        __syncthreads();                             // the chunk (and, the first time, the merged rows) visible
+        const uint16_t *us = u_s + size_t(ck % n_slots) * kCmbRows * kS;
+#pragma unroll
+        for (int kl = 0; kl < kCmbRows / 16; ++kl) {
+            const int ks = ck * (kCmbRows / 16) + kl;
             uint32_t ah[4], al[4];
             ldsm_x4(ah, ah_s + size_t(lane & 15) * kAS + ks * 16 + (lane >> 4) * 8);
             ldsm_x4(al, al_s + size_t(lane & 15) * kAS + ks * 16 + (lane >> 4) * 8);
 #pragma unroll
             for (int p = 0; p < 2; ++p) {
                 uint32_t bfr[4];
-                ldsm_x4_t(bfr, u_s + size_t(ks * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * kS + 32 * warp + 16 * p +
+                ldsm_x4_t(bfr, us + size_t(kl * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * kS + 32 * warp + 16 * p +
                                    (lane >> 4) * 8);
                 mma_bf16(acc[2 * p], ah, bfr[0], bfr[1]);
                 mma_bf16(acc[2 * p], al, bfr[0], bfr[1]);
@@ -431,22 +506,29 @@ combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ 
                 mma_bf16(acc[2 * p + 1], al, bfr[2], bfr[3]);
             }
         }
-#pragma unroll
-        for (int nt = 0; nt < 4; ++nt) {
-            const int col = 32 * warp + 8 * nt + 2 * (lane & 3);
-            *reinterpret_cast<float2 *>(part + g8 * dh + col) = make_float2(acc[nt][0], acc[nt][1]);
-            *reinterpret_cast<float2 *>(part + (g8 + 8) * dh + col) = make_float2(acc[nt][2], acc[nt][3]);
+        if (ck + n_slots < n_ck) {
+            __syncthreads();                         // every warp is done with the slot
+            load_chunk(ck + n_slots);
         }
-        msync();                                     // every rank's products are complete
-        for (int o = tid; o < nb * per_rank; o += 128) {
-            const int bi = o / per_rank, cc = int(rank) * per_rank + (o - bi * per_rank);
-            float v = 0.0f;
-#pragma unroll
-            for (int k = 0; k < kClV; ++k) v += mld_rank(part + bi * dh + cc, uint32_t(k));
-            O[size_t(b0 + bi) * d + size_t(h) * dh + cc] = v;
-        }
-        msync();
+        asm volatile("cp.async.commit_group;" ::: "memory");
     }
+    __syncthreads();                                 // the merge weights (in part) are dead
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+        const int col = 32 * warp + 8 * nt + 2 * (lane & 3);
+        *reinterpret_cast<float2 *>(part + g8 * dh + col) = make_float2(acc[nt][0], acc[nt][1]);
+        *reinterpret_cast<float2 *>(part + (g8 + 8) * dh + col) = make_float2(acc[nt][2], acc[nt][3]);
+    }
+    msync();                                         // every rank's products are complete
+    const int per_rank = dh / kClV;
+    for (int o = tid; o < nb * per_rank; o += 128) {
+        const int bi = o / per_rank, cc = int(rank) * per_rank + (o - bi * per_rank);
+        float v = 0.0f;
+#pragma unroll
+        for (int k = 0; k < kClV; ++k) v += mld_rank(part + bi * dh + cc, uint32_t(k));
+        O[size_t(b0 + bi) * d + size_t(h) * dh + cc] = v;
+    }
+    msync();                                         // partials read before the CTA exits
 }
 
 // ---------------------------------------------------------------------------
@@ -462,7 +544,8 @@ bool decode_mma_supported(int B, int r, int d, int dh) {
 cudaError_t launch_qproj_mma(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
                              unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
     const int rs = c.r / kClQ;
-    const size_t smem = size_t(rs) * 72 * 2 + size_t(16) * (rs + 8) * 2 + size_t(16) * (rs / 128) * 4 + 16 * 64 * 4;
+    const size_t smem = size_t(qp_slots(rs)) * 128 * 72 * 2 + size_t(16) * (rs + 8) * 2 + size_t(16) * (rs / 128) * 4 +
+                        16 * 64 * 4;
     cudaError_t e = ensure_smem(qproj_mma_kernel, smem);
     if (e != cudaSuccess) return e;
     e = launch_pdl(qproj_mma_kernel, dim3(kClQ, d / 64, (c.B + 15) / 16), dim3(128), smem, s, Uq, c, seq_len, c.B, d, q, qmax, n_qmax,
@@ -485,7 +568,8 @@ cudaError_t launch_combine_mma(const int32_t *seq_len, const int32_t *seq_map, i
                                const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
                                cudaStream_t s) {
     const int rs = r / kClV;
-    const size_t smem = size_t(rs) * (dh + 8) * 2 + size_t(32) * (rs + 8) * 2 + size_t(16) * dh * 4;
+    const size_t smem = size_t(cmb_slots(rs)) * kCmbRows * (dh + 8) * 2 + size_t(32) * (rs + 8) * 2 +
+                        size_t(16) * dh * 4;
     cudaError_t e = ensure_smem(combine_mma_kernel, smem);
     if (e != cudaSuccess) return e;
     e = launch_pdl(combine_mma_kernel, dim3(kClV, H, (B + 15) / 16), dim3(128), smem, s, Uv, seq_len, seq_map, nseq, B, Tmax, H, dh, r, chunk,
