@@ -31,10 +31,10 @@ constexpr int kClV = 8;          // combine: CTAs per cluster
 constexpr int kMaxSplitsM = 64;  // softmax partials per sequence
 constexpr int kCmbRows = 64;     // combine: U_v rows per ring slot
 // Ring slots (128-row groups) of the query projection's U_q stream: three
-// while a third of an SM holds them (rs <= 384), else two; never more than the
-// groups.
+// while a third of an SM holds them beside the codes (rs <= 512), else two;
+// never more than the groups.
 __host__ __device__ constexpr int qp_slots(int rs) {
-    const int want = rs <= 384 ? 3 : 2, groups = rs / 128;
+    const int want = rs <= 512 ? 3 : 2, groups = rs / 128;
     return groups < want ? groups : want;
 }
 // Ring slots of the combine's U_v stream: three while they fit beside the
@@ -120,7 +120,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
     uint16_t *u_s = reinterpret_cast<uint16_t *>(smem);                      // [n_slots][128][kUS]
     uint16_t *a_s = u_s + size_t(n_slots) * 128 * kUS;                       // [16][kAS]
     float *sc_s = reinterpret_cast<float *>(a_s + 16 * kAS);                 // [16][ngl]
-    float *part = sc_s + 16 * ngl;                                           // [16][64]
+    float *part = reinterpret_cast<float *>(smem);                           // [16][64], over the ring once it is dead
     auto load_group = [&](int g) {                   // U_q rows [j0 + 128 g, +128), the cluster's 64 columns
         uint16_t *dst = u_s + size_t(g % n_slots) * 128 * kUS;
         for (int i = tid; i < 128 * 8; i += 128) {
@@ -238,6 +238,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
             }
             asm volatile("cp.async.commit_group;" ::: "memory");
         }
+        __syncthreads();                             // the ring is dead: part takes its first bytes
 #pragma unroll
         for (int nt = 0; nt < 2; ++nt) {
             const int col = 16 * warp + 8 * nt + 2 * (lane & 3);
@@ -544,8 +545,7 @@ bool decode_mma_supported(int B, int r, int d, int dh) {
 cudaError_t launch_qproj_mma(const CacheView &c, const int32_t *seq_len, const uint16_t *Uq, int d, float *q,
                              unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
     const int rs = c.r / kClQ;
-    const size_t smem = size_t(qp_slots(rs)) * 128 * 72 * 2 + size_t(16) * (rs + 8) * 2 + size_t(16) * (rs / 128) * 4 +
-                        16 * 64 * 4;
+    const size_t smem = size_t(qp_slots(rs)) * 128 * 72 * 2 + size_t(16) * (rs + 8) * 2 + size_t(16) * (rs / 128) * 4;
     cudaError_t e = ensure_smem(qproj_mma_kernel, smem);
     if (e != cudaSuccess) return e;
     e = launch_pdl(qproj_mma_kernel, dim3(kClQ, d / 64, (c.B + 15) / 16), dim3(128), smem, s, Uq, c, seq_len, c.B, d, q, qmax, n_qmax,
