@@ -409,21 +409,27 @@ class NativeBench:
 
     # ---- end to end through the public binding with host buffers ----
     def e2e(self, steps, warmup):
-        """Per layer copy: host X -> device, projection and decode attention
-        through the Python binding, O -> host; decode tokens/s of one layer."""
+        """Per decode token: one host -> device copy of the token's X rows for
+        the K layer copies, the projection and the decode attention of every
+        copy through the Python binding, one device -> host copy of their O
+        rows.  Timed twice: as a CUDA graph captured from those binding calls
+        and copies (one graph per step, replayed the way a decode loop in a
+        server replays it) and eagerly (every call made from Python,
+        host-bound).  Returns decode tokens/s of one layer for both and the
+        bytes copied per step."""
         torch, q, s, K = self.torch, self.q, self.wl.shape, self.K
         hx_p = [torch.empty(L.Xp.shape, dtype=torch.bfloat16, pin_memory=True) for L in self.layers]
-        hx_d = [torch.empty(L.Xd.shape, dtype=torch.bfloat16, pin_memory=True) for L in self.layers]
-        for L, hp, hd in zip(self.layers, hx_p, hx_d):
+        for L, hp in zip(self.layers, hx_p):
             hp.copy_(L.Xp.cpu())
-            hd.copy_(L.Xd.cpu())
-        hO = torch.empty((K, self.S, self.B, s.d), dtype=torch.float32, pin_memory=True)
+        hx_d = torch.empty((self.S, K, self.B, s.d), dtype=torch.bfloat16, pin_memory=True)
+        for k, L in enumerate(self.layers):
+            hx_d[:, k].copy_(L.Xd.cpu())
+        hO = torch.empty((self.S, K, self.B, s.d), dtype=torch.float32, pin_memory=True)
         dXp = torch.empty_like(self.Xp)
-        dXd = torch.empty((self.B, s.d), dtype=torch.bfloat16, device=self.dev)
-        E = torch.cuda.Event
-        tot = []
-        for it in range(warmup + steps):
-            evs = [(E(enable_timing=True), E(enable_timing=True)) for _ in range(self.S + 1)]
+        dX = torch.empty((K, self.B, s.d), dtype=torch.bfloat16, device=self.dev)
+        dO = torch.empty((K, self.B, s.d), dtype=torch.float32, device=self.dev)
+
+        def step(evs):
             self.flush()
             evs[0][0].record()
             for k, L in enumerate(self.layers):
@@ -434,27 +440,50 @@ class NativeBench:
             for t in range(self.S):
                 self.flush()
                 evs[t + 1][0].record()
+                dX.copy_(hx_d[t], non_blocking=True)
                 for k, L in enumerate(self.layers):
-                    dXd.copy_(hx_d[k][t], non_blocking=True)
-                    q.qsvd_latent_project(L.W, dXd, 1.0, self.wl.lat_bits, 1.0, dst=L.cache,
+                    q.qsvd_latent_project(L.W, dX[k], 1.0, self.wl.lat_bits, 1.0, dst=L.cache,
                                           dst_seq=self.dseq, dst_pos=self.dpos[t], workspace=self.wsp)
                     if L.UQ:
-                        q.qsvd_latent_decode_attn_qu(L.cache, self.dlen[t], self.P + t + 1, *L.UQ, s.H, s.dh, L.O,
+                        q.qsvd_latent_decode_attn_qu(L.cache, self.dlen[t], self.P + t + 1, *L.UQ, s.H, s.dh, dO[k],
                                                      workspace=self.wsd)
                     else:
-                        q.qsvd_latent_decode_attn(L.cache, self.dlen[t], self.P + t + 1, *L.U, s.H, s.dh, L.O,
+                        q.qsvd_latent_decode_attn(L.cache, self.dlen[t], self.P + t + 1, *L.U, s.H, s.dh, dO[k],
                                                   workspace=self.wsd)
-                    hO[k, t].copy_(L.O, non_blocking=True)
+                hO[t].copy_(dO, non_blocking=True)
                 evs[t + 1][1].record()
+
+        def decode_seconds(evs):
+            return sum(a.elapsed_time(b) for a, b in evs[1:]) * 1e-3
+
+        E = torch.cuda.Event
+        eager = []
+        for it in range(warmup + steps):
+            evs = [(E(enable_timing=True), E(enable_timing=True)) for _ in range(self.S + 1)]
+            step(evs)
             torch.cuda.synchronize()
             if it >= warmup:
-                tot.append(sum(a.elapsed_time(b) for a, b in evs[1:]) * 1e-3)
-        dec_s = statistics.mean(tot)
+                eager.append(decode_seconds(evs))
+        gs = torch.cuda.Stream()
+        gs.wait_stream(torch.cuda.current_stream())
+        gevs = [(E(enable_timing=True, external=True), E(enable_timing=True, external=True))
+                for _ in range(self.S + 1)]
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=gs):
+            step(gevs)
+        torch.cuda.synchronize()
+        graphed = []
+        for it in range(warmup + steps):
+            g.replay()
+            torch.cuda.synchronize()
+            if it >= warmup:
+                graphed.append(decode_seconds(gevs))
         # bytes copied inside the timed intervals (evs[1:]: the S decode tokens
         # through the K copies); the prefill's X copies are outside them
         h2d = K * self.S * self.B * s.d * 2
         d2h = K * self.S * self.B * s.d * 4
-        return self.B * self.S * K / dec_s, h2d, d2h
+        tokens = self.B * self.S * K
+        return tokens / statistics.mean(graphed), tokens / statistics.mean(eager), h2d, d2h
 
 
 def prefill_gemm_probe(T=24064, d=5120, r=2048, iters=3, w4a4=False):
@@ -758,10 +787,12 @@ def run_native(args, rank, world, local_rank):
 
     e2e = None
     if not args.no_e2e:
-        e2e_val, h2d, d2h = nb.e2e(steps=min(args.steps, 3), warmup=3)
-        e2e_val = cross_rank([e2e_val], "min")[0] * world     # the slowest rank's rate, every rank
+        e2e_val, e2e_eager, h2d, d2h = nb.e2e(steps=min(args.steps, 3), warmup=3)
+        e2e_val, e2e_eager = (v * world for v in cross_rank([e2e_val, e2e_eager], "min"))   # slowest rank, every rank
         e2e = {"value": round(e2e_val, 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h}
+               "d2h_bytes_per_step": d2h,
+               "launch": "one CUDA graph per step captured from the binding's calls and host copies",
+               "eager_value": round(e2e_eager, 1)}
 
     pre13 = prefill_gemm_probe() if not args.no_prefill13 else None
     pre13_w4 = prefill_gemm_probe(w4a4=True) if not args.no_prefill13 else None

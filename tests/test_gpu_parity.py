@@ -216,6 +216,29 @@ def test_decode_large_batch_tensor_core_products(B, bits):
         assert_rows_close(o, np.stack([outs[b] for b in range(B)]), f"step {step}")
 
 
+@pytest.mark.parametrize("r,bits", [(512, 8), (1024, 4), (3072, 8)])
+def test_decode_batched_weight_rings(r, bits):
+    """The batched up-projection kernels stream their weight rows through a
+    shared-memory ring: r = 512 takes one slot (one 128-row group of U_q, one
+    64-row chunk of U_v per CTA), r = 1024 two slots exactly filled, r = 3072
+    six groups / chunks through two slots (the ring wraps three times).
+    d = 1024 (8 heads), B = 6, ragged lengths."""
+    wl = synthetic.Workload("rings", synthetic.LayerShape(1024, 8, 128, r), B=6, n_image=0, n_text=90,
+                            decode_steps=2, lat_bits=bits)
+    inp = synthetic.gen_layer(wl, seed=23)
+    w = pipeline.prepare_weights(inp)
+    s = wl.shape
+    ref = pipeline.OracleLayer(s, w, wl.B, wl.tmax, bits)
+    gpu = GpuLayer(s, w, wl.B, wl.tmax, bits)
+    for b, n in enumerate((1, 17, 40, 64, 77, 90)):
+        ref.prefill(b, inp.X_prefill[b][:n])
+        gpu.prefill(b, inp.X_prefill[b][:n])
+    for step in range(2):
+        _, outs = ref.decode_step(inp.X_decode[step])
+        o = gpu.decode_step(inp.X_decode[step]).cpu().numpy()
+        assert_rows_close(o, np.stack([outs[b] for b in range(wl.B)]), f"r {r} step {step}")
+
+
 def test_decode_13b_heads_and_rank():
     """H = 40 (five head groups of 8), r = 2048, d = 5120."""
     base = synthetic.WORKLOADS["llava13b"]
