@@ -17,6 +17,7 @@
 //   append_kernel       a4: latent rows -> cache slots.
 //   up_quant_kernel     offline per-output-channel RTN of an up-projection
 //                       (Eq. 11's Q(W^u)), int8 or int4.
+#include <algorithm>
 #include <cmath>
 
 #include "common.cuh"
@@ -105,9 +106,88 @@ xquant_kernel(const uint16_t *__restrict__ X, int d, float clip, int rot, float 
     if (threadIdx.x == 0 && xs) xs[t] = s;
 }
 
+// a1 without a rotation, for rows of up to kXrMaxD channels: 128 threads per
+// row, every 16-byte load of the row issued at once and the row kept in
+// registers (no staging through shared memory), so a row needs one round trip
+// to memory; at 70 registers per thread seven CTAs share an SM (xquant_kernel:
+// 61 registers x 256 threads, four rows, two or three dependent loads per
+// thread).  The codes are those of xquant_kernel (the same absmax, scale and
+// quantizer).
+constexpr int kXrThreads = 128;
+constexpr int kXrLoads = 6;                              // 16-byte loads per thread
+constexpr int kXrMaxD = kXrThreads * kXrLoads * 8;       // 6144 channels
+
+__global__ void __launch_bounds__(kXrThreads, 7)
+xquant_rows_kernel(const uint16_t *__restrict__ X, int64_t T, int d, float clip, int qmax, int8_t *__restrict__ xq,
+                   uint16_t *__restrict__ xq_bf16, uint8_t *__restrict__ xq_f8, float *__restrict__ xs) {
+    __shared__ float red[2][kXrThreads / 32];
+    pdl_trigger();
+    pdl_wait();
+    for (int64_t t = blockIdx.x, n = 0; t < T; t += gridDim.x, ++n) {   // rows of this CTA
+        const uint16_t *x = X + t * d;
+        uint4 v[kXrLoads];
+#pragma unroll
+        for (int k = 0; k < kXrLoads; ++k) {
+            const int i = (k * kXrThreads + int(threadIdx.x)) * 8;
+            v[k] = i < d ? *reinterpret_cast<const uint4 *>(x + i) : make_uint4(0u, 0u, 0u, 0u);
+        }
+        float m = 0.0f;
+#pragma unroll
+        for (int k = 0; k < kXrLoads; ++k) {
+            float f[8];
+            unpack8_bf16(v[k], f);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(f[e]));
+        }
+        m = block_max<kXrThreads>(m, red[n & 1]);      // alternate buffers: no barrier between rows
+        const float s = quant_scale(m, clip, float(qmax)), inv = quant_inv_scale(s);
+#pragma unroll
+        for (int k = 0; k < kXrLoads; ++k) {
+            const int i = (k * kXrThreads + int(threadIdx.x)) * 8;
+            if (i >= d) break;
+            float f[8];
+            unpack8_bf16(v[k], f);
+            int c[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) c[e] = quant_code_fast(f[e], s, inv, qmax);
+            if (xq_bf16) {
+                uint32_t w[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    w[e] = uint32_t(int_to_bf16_bits(c[2 * e])) | (uint32_t(int_to_bf16_bits(c[2 * e + 1])) << 16);
+                *reinterpret_cast<uint4 *>(xq_bf16 + t * d + i) = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+            if (xq) {
+                uint32_t w[2] = {0u, 0u};
+#pragma unroll
+                for (int e = 0; e < 8; ++e) w[e >> 2] |= uint32_t(c[e] & 0xff) << ((e & 3) * 8);
+                *reinterpret_cast<uint2 *>(xq + t * d + i) = make_uint2(w[0], w[1]);
+            }
+            if (xq_f8) {
+                uint32_t w[2] = {0u, 0u};
+#pragma unroll
+                for (int e = 0; e < 8; ++e) w[e >> 2] |= uint32_t(int_to_e4m3(c[e])) << ((e & 3) * 8);
+                *reinterpret_cast<uint2 *>(xq_f8 + t * d + i) = make_uint2(w[0], w[1]);
+            }
+        }
+        if (threadIdx.x == 0 && xs) xs[t] = s;
+    }
+}
+
 cudaError_t launch_xquant(const uint16_t *X, int64_t T, int d, float clip, int8_t *xq,
                           uint16_t *xq_bf16, float *xs, cudaStream_t s, int rot, int qmax, uint8_t *xq_f8) {
     if (T == 0) return cudaSuccess;
+    if (!rot && d <= kXrMaxD && d % 8 == 0) {
+        // one CTA per row up to the rows that are resident at once (seven per SM); beyond, each CTA walks
+        // rows with a stride of the grid (no CTA launches per row)
+        int dev = 0, sms = 148;
+        if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        const int64_t grid = std::min<int64_t>(T, int64_t(sms) * 7);
+        cudaError_t e = launch_pdl(xquant_rows_kernel, dim3(unsigned(grid)), dim3(kXrThreads), 0, s, X, T, d, clip,
+                                   qmax, xq, xq_bf16, xq_f8, xs);
+        prof_mark(s, "xquant");
+        return e;
+    }
     const size_t smem = size_t(d) * sizeof(float);
     if (smem > 48 * 1024) {
         cudaError_t e = ensure_smem(xquant_kernel, smem);
