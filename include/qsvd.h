@@ -166,7 +166,9 @@ int qsvd_quantize_weight_ex(const float *W_d, int32_t d, int32_t r, float clip, 
  * Optional intermediates for inspection (NULL skips the write):
  *   xq_out int8 [T, d], xs_out fp32 [T], acc_out int32 [T, r].
  * workspace: at least qsvd_project_workspace_bytes(T, d, r) bytes, 256-byte
- * aligned.  T may be 0 (nothing is enqueued).
+ * aligned (while T * r <= 80 * 128 * 128 it includes room for four int32
+ * [T, r] partial sums: a product with few tiles splits K over more CTAs).
+ * T may be 0 (nothing is enqueued).
  */
 int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
                         float act_clip, int32_t lat_bits, float lat_clip,
@@ -435,7 +437,9 @@ int qsvd_latent_project_static(const qsvd_down_weight *W, const uint16_t *X, int
  * thread-safe):
  *   0  automatic (default): in the GEMM epilogue for int4 latents, and for
  *      int8 latents when r / 256 <= 6 (the per-token maximum is exchanged
- *      within a cluster of r / 256 CTAs);
+ *      within a cluster of r / 256 CTAs) and the 256-column tiles fill at
+ *      least one wave of the GPU (ceil(T / 128) * r / 256 >= the SM count;
+ *      below that the separate kernel with twice the tiles is faster);
  *   1  always a separate requantization kernel over an fp32 latent in the
  *      workspace;
  *   2  in the epilogue whenever possible (int8 needs r / 256 <= 8).

@@ -296,7 +296,8 @@ size_t qsvd_project_workspace_bytes(int64_t T, int32_t d, int32_t r) {
            align256(size_t(T) * d) +            // int8 codes of X
            align256(size_t(T) * 4) +            // s_x
            align256(size_t(T) * r * 4) +        // dequantized latent c_hat
-           align256(size_t(T) * d * 2);         // bf16 image of the X codes (tensor-core operand)
+           align256(size_t(T) * d * 2) +        // bf16 image of the X codes (tensor-core operand)
+           (T * r <= kSplitMaxElems ? align256(size_t(kMaxSplitK) * T * r * 4) : 0);   // split-K partials
 }
 
 int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T, float act_clip,
@@ -402,6 +403,18 @@ int qsvd_latent_project(const qsvd_down_weight *W, const uint16_t *X, int64_t T,
                                      lat_scales, dst ? &dv : nullptr, dst_seq, dst_pos, nullptr, acc_out, err,
                                      stream);
             return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "tensor-core projection launch");
+        }
+        const int splits = gemm_tc_splits(T, d, r);
+        if (splits > 1) {
+            // few tiles: split K over more CTAs; the splits' sums are added, dequantized and
+            // requantized row by row
+            int32_t *part = reinterpret_cast<int32_t *>(reinterpret_cast<char *>(xq_bf16) + align256(size_t(T) * d * 2));
+            e = launch_gemm_tc(xq_bf16, T, d, W->codes_bf16, W->scale, xs, r, nullptr, nullptr, err, stream, splits,
+                               part);
+            if (e == cudaSuccess)
+                e = launch_split_requant(part, splits, T, r, xs, W->scale, acc_out, lat_bits, lat_clip, lat_codes,
+                                         lat_scales, dst ? &dv : nullptr, dst_seq, dst_pos, err, stream);
+            return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "split-K projection launch");
         }
         e = launch_gemm_tc(xq_bf16, T, d, W->codes_bf16, W->scale, xs, r, c_hat, acc_out, err, stream);
         if (e != cudaSuccess) return cuda_fail(e, "tensor-core projection launch");

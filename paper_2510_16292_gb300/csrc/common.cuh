@@ -15,6 +15,11 @@ namespace qsvd {
 // prologue now / wait until every earlier kernel in the stream has finished
 // and its writes are visible.  Both are no-ops without the launch attribute.
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+// Data written by the grid this one waits on is never read through a
+// `const T *__restrict__` pointer (the read-only path): a dependent grid runs
+// while its producer still writes, so such loads may be scheduled ahead of
+// this wait and see stale values (measured: a row requantizer reading the
+// GEMM's partial sums that way returned wrong codes on every run).
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 // Bulk prefetch of [p, p + bytes) into L2 (16-byte aligned, bytes % 16 == 0).
@@ -295,19 +300,14 @@ __device__ __forceinline__ float block_max(float v, float *red) {
 constexpr int kRqThreads = 256;
 constexpr int kRqMaxQuads = 4;     // r <= 4096
 
-__device__ __forceinline__ void requant_row_cta(const float *__restrict__ c_hat, int64_t t, int r, int bits,
-                                                float clip, void *__restrict__ lat_codes,
-                                                void *__restrict__ lat_scales, const CacheView &dst,
-                                                const int32_t *__restrict__ dst_seq,
-                                                const int32_t *__restrict__ dst_pos, int *err, float *red) {
-    const float *row = c_hat + t * r;
+// The requantization of row t from its values already in registers: thread
+// i holds channels 4 (i + k kRqThreads) .. + 3 in v[k] (zeros past r).
+__device__ __forceinline__ void requant_row_values(const float4 (&v)[kRqMaxQuads], int64_t t, int r, int bits,
+                                                   float clip, void *__restrict__ lat_codes,
+                                                   void *__restrict__ lat_scales, const CacheView &dst,
+                                                   const int32_t *__restrict__ dst_seq,
+                                                   const int32_t *__restrict__ dst_pos, int *err, float *red) {
     const int nq = r / 4;
-    float4 v[kRqMaxQuads];
-#pragma unroll
-    for (int k = 0; k < kRqMaxQuads; ++k) {
-        const int qi = threadIdx.x + k * kRqThreads;
-        v[k] = qi < nq ? reinterpret_cast<const float4 *>(row)[qi] : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
     // cache destination of this row (if any), bounds-checked
     uint8_t *cache_codes = nullptr;
     void *cache_scale = nullptr;
@@ -376,11 +376,28 @@ __device__ __forceinline__ void requant_row_cta(const float *__restrict__ c_hat,
 }
 
 
+__device__ __forceinline__ void requant_row_cta(const float *c_hat, int64_t t, int r, int bits,
+                                                float clip, void *__restrict__ lat_codes,
+                                                void *__restrict__ lat_scales, const CacheView &dst,
+                                                const int32_t *__restrict__ dst_seq,
+                                                const int32_t *__restrict__ dst_pos, int *err, float *red) {
+    const float *row = c_hat + t * r;
+    const int nq = r / 4;
+    float4 v[kRqMaxQuads];
+#pragma unroll
+    for (int k = 0; k < kRqMaxQuads; ++k) {
+        const int qi = threadIdx.x + k * kRqThreads;
+        v[k] = qi < nq ? reinterpret_cast<const float4 *>(row)[qi] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    requant_row_values(v, t, r, bits, clip, lat_codes, lat_scales, dst, dst_seq, dst_pos, err, red);
+}
+
+
 // The same per-token requantization by one warp (no block barriers): two
 // passes over the row, the second reading it back from L1/L2.  Codes and
 // scales are identical to requant_row_cta's (the maximum does not depend on
 // the order of reduction).
-__device__ __forceinline__ void requant_row_warp(const float *__restrict__ c_hat, int64_t t, int r, int bits,
+__device__ __forceinline__ void requant_row_warp(const float *c_hat, int64_t t, int r, int bits,
                                                  float clip, void *__restrict__ lat_codes,
                                                  void *__restrict__ lat_scales, const CacheView &dst,
                                                  const int32_t *__restrict__ dst_seq,

@@ -302,7 +302,7 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint8_t *__restric
 // ---------------------------------------------------------------------------
 template <int NB, int WB>
 __global__ void __launch_bounds__(256)
-qabsorb_kernel(const float *__restrict__ q, const uint8_t *__restrict__ Uk, const float *__restrict__ sk, int B, int r,
+qabsorb_kernel(const float *q, const uint8_t *__restrict__ Uk, const float *__restrict__ sk, int B, int r,
                int d, int H, int dh, int hg, float *__restrict__ qt, unsigned *__restrict__ qmax, int *err) {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar;
@@ -412,8 +412,8 @@ template <int NB, int WB>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
 combine_uv_kernel(const __grid_constant__ CUtensorMap map_v, const uint8_t *__restrict__ Uv, const float *__restrict__ sv,
                   const int32_t *__restrict__ seq_len, const int32_t *__restrict__ seq_map, int nseq, int B, int Tmax,
-                  int H, int dh, int r, int chunk, int n_split, const float *__restrict__ pm,
-                  const float *__restrict__ pl, const float *__restrict__ po, float *__restrict__ O, int *err) {
+                  int H, int dh, int r, int chunk, int n_split, const float *pm,
+                  const float *pl, const float *po, float *__restrict__ O, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ float w_s[NB][kMaxSplitsG];

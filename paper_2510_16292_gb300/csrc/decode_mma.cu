@@ -262,7 +262,7 @@ qproj_mma_kernel(const uint16_t *__restrict__ Uq, CacheView c, const int32_t *__
 // for j in [128 x, 128 x + 128), warp w the 32 columns 32w .. 32w+31.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(128)
-qabsorb_mma_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk, int B, int r, int d, int H, int dh,
+qabsorb_mma_kernel(const float *q, const uint16_t *__restrict__ Uk, int B, int r, int d, int H, int dh,
                    float *__restrict__ qt, unsigned *__restrict__ qmax) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ float mx_s[4][16];
@@ -361,8 +361,8 @@ qabsorb_mma_kernel(const float *__restrict__ q, const uint16_t *__restrict__ Uk,
 __global__ void __cluster_dims__(kClV, 1, 1) __launch_bounds__(128)
 combine_mma_kernel(const uint16_t *__restrict__ Uv, const int32_t *__restrict__ seq_len,
                    const int32_t *__restrict__ seq_map, int nseq, int B, int Tmax, int H,
-                   int dh, int r, int chunk, int n_split, const float *__restrict__ pm, const float *__restrict__ pl,
-                   const float *__restrict__ po, float *__restrict__ O) {
+                   int dh, int r, int chunk, int n_split, const float *pm, const float *pl,
+                   const float *po, float *__restrict__ O) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ float inv_s[16];
     __shared__ int ns_s[16];

@@ -89,7 +89,7 @@ __device__ __forceinline__ bool valid_len(int L, int Tmax) { return L >= 1 && L 
 // ---------------------------------------------------------------------------
 template <int BITS>
 __global__ void __launch_bounds__(kAtThreads)
-attn_chunk_kernel(CacheView c, const int32_t *__restrict__ seq_len, const float *__restrict__ qt, int H,
+attn_chunk_kernel(CacheView c, const int32_t *__restrict__ seq_len, const float *qt, int H,
                   float softmax_scale, int chunk, int sub, int n_split, float *__restrict__ pm,
                   float *__restrict__ pl, float *__restrict__ po, int *err) {
     extern __shared__ __align__(16) uint8_t smem[];

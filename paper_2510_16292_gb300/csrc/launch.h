@@ -158,8 +158,25 @@ constexpr int kPsSplitTok = 2;
 // Exact int8 GEMM on the tensor cores (bf16 images of the codes, fp32 TMEM
 // accumulators drained to int32 every 1024 of K) + the fp32 dequantization.
 bool gemm_tc_supported(int d, int r);
+// splits > 1 (with part: [splits, T, r] int32 scratch): each CTA sums its
+// slice of K; split_requant adds the slices, dequantizes and requantizes.
 cudaError_t launch_gemm_tc(const uint16_t *xq_bf16, int64_t T, int d, const uint16_t *w_bf16, const float *ws,
-                           const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s);
+                           const float *xs, int r, float *c_hat, int32_t *acc_out, int *err, cudaStream_t s,
+                           int splits = 1, int32_t *part = nullptr);
+// K splits for a separate-epilogue projection of T tokens (1: none).  Splits
+// are taken only while the tiles fill less than half the GPU, which needs
+// T * r <= kSplitMaxElems (80 tiles of 128 x 128 at most); the projection
+// workspace holds kMaxSplitK int32 partial latents up to that size.
+constexpr int kMaxSplitK = 4;
+constexpr int64_t kSplitMaxElems = int64_t(80) * 128 * 128;
+int gemm_tc_splits(int64_t T, int d, int r);
+// a2 + a3 after a split-K GEMM: per token row, the sum of the splits' int32
+// partials (written to acc_out if given), c_hat = (fp32(acc) s_x) s_w, and the
+// requantization and store of requant.
+cudaError_t launch_split_requant(const int32_t *part, int splits, int64_t T, int r, const float *xs, const float *ws,
+                                 int32_t *acc_out, int bits, float clip, void *lat_codes, void *lat_scales,
+                                 const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
+                                 cudaStream_t s);
 
 // W4A4: the GEMM on fp8 e4m3 images of int4-valued codes (kind::f8f6f4),
 // with the requantization epilogue for lat_bits 8 / 4 (0: c_hat only).

@@ -204,7 +204,7 @@ __device__ __forceinline__ void gemm_tile(int t, int tiles_m, int tiles_n, int &
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(pf::kGemmThreads, 1)
 qkv_gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b, int R, int r,
-                int d, const float *__restrict__ rs, __half *__restrict__ Qm, __half *__restrict__ Km,
+                int d, const float *rs, __half *__restrict__ Qm, __half *__restrict__ Km,
                 __half *__restrict__ Vt, int *err) {
     // Persistent: CTA c takes tiles c, c + gridDim.x, ...  Tiles are numbered
     // in groups of kGemmGroupM row tiles, row fastest within a group (see

@@ -19,8 +19,8 @@ constexpr int kPjWarps = 8;       // output channels per CTA (one per warp)
 constexpr int kPjTokens = 16;     // tokens per CTA (grid.y tiles T)
 
 __global__ void __launch_bounds__(kPjWarps * 32)
-proj_dp4a_kernel(const int8_t *__restrict__ xq, int64_t T, int d, const int8_t *__restrict__ w,
-                 const float *__restrict__ ws, const float *__restrict__ xs, int r,
+proj_dp4a_kernel(const int8_t *xq, int64_t T, int d, const int8_t *__restrict__ w,
+                 const float *__restrict__ ws, const float *xs, int r,
                  float *__restrict__ c_hat, int32_t *__restrict__ acc_out) {
     const int lane = threadIdx.x & 31;
     const int j = blockIdx.x * kPjWarps + (threadIdx.x >> 5);
@@ -61,7 +61,7 @@ proj_small_kernel(const uint16_t *__restrict__ X, int T, int d, float act_clip, 
                   int *__restrict__ counter, int8_t *__restrict__ xq_out, float *__restrict__ xs_out,
                   int32_t *__restrict__ acc_out, void *__restrict__ lat_codes, void *__restrict__ lat_scales,
                   CacheView dst, const int32_t *__restrict__ dst_seq, const int32_t *__restrict__ dst_pos,
-                  int *err, const int8_t *__restrict__ xq_in, const float *__restrict__ xs_in, int tail, int act_qmax) {
+                  int *err, const int8_t *xq_in, const float *xs_in, int tail, int act_qmax) {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar, bar_x;
     {   // this CTA's token block

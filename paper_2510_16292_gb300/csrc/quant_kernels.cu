@@ -304,7 +304,7 @@ cudaError_t launch_quantize_weight(const float *W, int d, int r, float clip, int
 // a3/a4: requantize one latent row per CTA (requant_row_cta, common.cuh).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kRqThreads)
-requant_kernel(const float *__restrict__ c_hat, int r, int bits, float clip,
+requant_kernel(const float *c_hat, int r, int bits, float clip,
                void *__restrict__ lat_codes, void *__restrict__ lat_scales, CacheView dst,
                const int32_t *__restrict__ dst_seq, const int32_t *__restrict__ dst_pos,
                int *err) {
@@ -322,6 +322,73 @@ cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float
     if (dst) d = *dst;
     cudaError_t e = launch_pdl(requant_kernel, dim3(unsigned(T)), dim3(kRqThreads), 0, s, c_hat, r, bits, clip,
                                lat_codes, lat_scales, d, dst_seq, dst_pos, err);
+    prof_mark(s, "requant");
+    return e;
+}
+
+// ---------------------------------------------------------------------------
+// a2/a3/a4 after a split-K projection GEMM: one CTA per token row adds the
+// splits' int32 partial sums in split order (exact: |acc| < 2^31), forms
+// c_hat = (fp32(acc) s_x) s_w exactly as the GEMM epilogue does, and
+// requantizes and stores the row from registers.  The partials and s_x are
+// written by the grids this one waits on, so they are not read through the
+// read-only path (no __restrict__): the loads stay behind the wait.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kRqThreads)
+split_requant_kernel(const int32_t *part, int splits, int64_t T, int r, const float *xs,
+                     const float *__restrict__ ws, int32_t *__restrict__ acc_out, int bits, float clip,
+                     void *__restrict__ lat_codes, void *__restrict__ lat_scales, CacheView dst,
+                     const int32_t *__restrict__ dst_seq, const int32_t *__restrict__ dst_pos, int *err) {
+    __shared__ float red[kRqThreads / 32];
+    pdl_trigger();
+    pdl_wait();
+    const int64_t t = blockIdx.x;
+    const int nq = r / 4;
+    const float sx = xs[t];
+    int4 p4[kRqMaxQuads][kMaxSplitK];                 // every partial of the thread's quads, loads issued first
+#pragma unroll
+    for (int k = 0; k < kRqMaxQuads; ++k) {
+        const int qi = int(threadIdx.x) + k * kRqThreads;
+#pragma unroll
+        for (int z = 0; z < kMaxSplitK; ++z)
+            p4[k][z] = qi < nq && z < splits
+                           ? reinterpret_cast<const int4 *>(part + (size_t(z) * size_t(T) + size_t(t)) * r)[qi]
+                           : make_int4(0, 0, 0, 0);
+    }
+    float4 v[kRqMaxQuads];
+#pragma unroll
+    for (int k = 0; k < kRqMaxQuads; ++k) {
+        const int qi = int(threadIdx.x) + k * kRqThreads;
+        v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (qi < nq) {
+            int4 a = p4[k][0];
+#pragma unroll
+            for (int z = 1; z < kMaxSplitK; ++z) {       // in split order; absent splits are zeros
+                a.x += p4[k][z].x;
+                a.y += p4[k][z].y;
+                a.z += p4[k][z].z;
+                a.w += p4[k][z].w;
+            }
+            if (acc_out) reinterpret_cast<int4 *>(acc_out + size_t(t) * r)[qi] = a;
+            const float4 w = reinterpret_cast<const float4 *>(ws)[qi];
+            v[k] = make_float4(__fmul_rn(__fmul_rn(__int2float_rn(a.x), sx), w.x),
+                               __fmul_rn(__fmul_rn(__int2float_rn(a.y), sx), w.y),
+                               __fmul_rn(__fmul_rn(__int2float_rn(a.z), sx), w.z),
+                               __fmul_rn(__fmul_rn(__int2float_rn(a.w), sx), w.w));
+        }
+    }
+    requant_row_values(v, t, r, bits, clip, lat_codes, lat_scales, dst, dst_seq, dst_pos, err, red);
+}
+
+cudaError_t launch_split_requant(const int32_t *part, int splits, int64_t T, int r, const float *xs, const float *ws,
+                                 int32_t *acc_out, int bits, float clip, void *lat_codes, void *lat_scales,
+                                 const CacheView *dst, const int32_t *dst_seq, const int32_t *dst_pos, int *err,
+                                 cudaStream_t s) {
+    if (T == 0) return cudaSuccess;
+    CacheView d{};
+    if (dst) d = *dst;
+    cudaError_t e = launch_pdl(split_requant_kernel, dim3(unsigned(T)), dim3(kRqThreads), 0, s, part, splits, T, r, xs,
+                               ws, acc_out, bits, clip, lat_codes, lat_scales, d, dst_seq, dst_pos, err);
     prof_mark(s, "requant");
     return e;
 }
