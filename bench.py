@@ -66,6 +66,9 @@ def parse():
     p.add_argument("--attn-path", type=int, default=0, choices=[0, 1, 2, 3],
                    help="decode attention kernel choice (qsvd_set_decode_attn_path): 0 automatic, 1 CUDA cores, "
                         "2 tcgen05, 3 warp-level MMA")
+    p.add_argument("--decode-call", choices=["step", "pair"], default="pair",
+                   help="decode API: one qsvd_decode_step call per token (step) or qsvd_latent_project + "
+                        "qsvd_latent_decode_attn (pair)")
     p.add_argument("--rot", action="store_true",
                    help="rotate X by H1 on the fly (Eq. 12; weights quantized as H1 W_d) in every projection")
     p.add_argument("--prefill-probe", action="store_true",
@@ -187,7 +190,7 @@ class NativeBench:
     cached, as it does in serving.  `flush`: one copy, L2 evicted by a 256 MiB
     read before every sub-step (code cold as well)."""
 
-    def __init__(self, wl, rank, l2="rotate", rot=False, u_bits=0):
+    def __init__(self, wl, rank, l2="rotate", rot=False, u_bits=0, decode_call="pair"):
         import torch
         import paper_2510_16292_gb300 as q
         self.torch, self.q, self.wl, self.rot, self.u_bits = torch, q, wl, rot, u_bits
@@ -219,7 +222,8 @@ class NativeBench:
         self.wsp = torch.zeros(q.qsvd_project_workspace_bytes(B * P, s.d, s.r), dtype=torch.uint8, device=dev)
         self.wsd = torch.zeros(q.qsvd_decode_workspace_bytes(B, wl.tmax, s.r, s.H, s.dh), dtype=torch.uint8,
                                device=dev)
-        self.fused = False          # the PDL-chained calls are faster than the fused step today
+        # "step": one qsvd_decode_step call per token; "pair": qsvd_latent_project + qsvd_latent_decode_attn
+        self.fused = decode_call == "step"
         self.wsf = torch.zeros(max(1, q.qsvd_decode_step_workspace_bytes(B, wl.tmax, s.d, s.r, s.H, s.dh)),
                                dtype=torch.uint8, device=dev)
         self.flushbuf = torch.ones(FLUSH_BYTES // 4 if l2 == "flush" else 1, dtype=torch.float32, device=dev)
@@ -442,6 +446,10 @@ class NativeBench:
                 evs[t + 1][0].record()
                 dX.copy_(hx_d[t], non_blocking=True)
                 for k, L in enumerate(self.layers):
+                    if self.fused:
+                        q.qsvd_decode_step(L.W, dX[k], L.cache, self.dlen[t], self.P + t + 1, *L.U, s.H, s.dh, dO[k],
+                                           workspace=self.wsf)
+                        continue
                     q.qsvd_latent_project(L.W, dX[k], 1.0, self.wl.lat_bits, 1.0, dst=L.cache,
                                           dst_seq=self.dseq, dst_pos=self.dpos[t], workspace=self.wsp)
                     if L.UQ:
@@ -731,7 +739,9 @@ def run_native(args, rank, world, local_rank):
     wl = synthetic.WORKLOADS[args.workload]
     if args.decode_steps:
         wl = dataclasses.replace(wl, decode_steps=args.decode_steps)
-    nb = NativeBench(wl, rank, l2=args.l2, rot=args.rot, u_bits=args.u_bits)
+    if args.decode_call == "step" and (args.rot or args.u_bits):
+        raise SystemExit("--decode-call step takes bf16 up-projections and unrotated weights")
+    nb = NativeBench(wl, rank, l2=args.l2, rot=args.rot, u_bits=args.u_bits, decode_call=args.decode_call)
     K = nb.K
     S = wl.decode_steps
     hbm, _, peak_kind = peaks()
@@ -817,7 +827,9 @@ def run_native(args, rank, world, local_rank):
                           if args.l2 == "rotate" else
                           "flushed (256 MiB read) before the prefill and before every decode step; "
                           "flushes outside the timed intervals"),
-                   "launch": "one CUDA graph per step (captured C-ABI calls, PDL-chained kernels)"},
+                   "launch": "one CUDA graph per step (captured C-ABI calls, PDL-chained kernels)",
+                   "decode_call": ("qsvd_decode_step" if args.decode_call == "step" else
+                                   "qsvd_latent_project + qsvd_latent_decode_attn")},
         "secondary": {
             "decode_ms_per_step": round(dec_total / args.steps * 1e3, 4),
             "prefill_ms_per_step": round(pre_total / args.steps * 1e3, 4),

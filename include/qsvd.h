@@ -380,21 +380,23 @@ size_t qsvd_latent_prefill_workspace_bytes(const qsvd_prefill_block *blocks, int
                                            int32_t H, int32_t dh);
 
 /*
- * One whole decode step for a small batch, in a single launch: for each of
- * the B = cache->B sequences, the new token X[b] (bf16 [B, d]) is quantized
- * and projected (Eq. 12), its latent is requantized and stored at position
- * seq_len[b] - 1 of sequence b (Eq. 11, Fig. 2(f)), and attention over
- * positions 0 .. seq_len[b]-1 is computed as in qsvd_latent_decode_attn
- * (Eq. 5).  The result equals qsvd_latent_project(dst = cache,
- * dst_seq = b, dst_pos = seq_len[b] - 1) followed by qsvd_latent_decode_attn,
- * with the same arithmetic; it exists because a small-batch decode step is
- * bound by launch latency rather than by its bytes.
- * The launch is cooperative (one CTA per SM, grid-wide barriers whose waits
- * are bounded: an expired wait abandons the step and flags QSVD_ETIMEOUT).
- * Every call first clears the grid barrier's counters in the workspace (one
- * small memset on the stream), so a call after an expired wait starts clean.
- * Requirements: B <= 8; d = H*dh, d % 256 == 0, d <= 6144; r <= 3072;
- * dh in {64, 128}.  workspace: qsvd_decode_step_workspace_bytes(...) bytes.
+ * One whole decode step in one call: for each of the B = cache->B sequences,
+ * the new token X[b] (bf16 [B, d]) is quantized and projected (Eq. 12), its
+ * latent is requantized and stored at position seq_len[b] - 1 of sequence b
+ * (Eq. 11, Fig. 2(f)), and attention over positions 0 .. seq_len[b]-1 is
+ * computed as in qsvd_latent_decode_attn (Eq. 5).  The result equals
+ * qsvd_latent_project(dst = cache, dst_seq = b, dst_pos = seq_len[b] - 1)
+ * followed by qsvd_latent_decode_attn, codes and scales bit for bit.  It
+ * exists because a small-batch decode step is bound by the latency of its
+ * chain of dependent launches rather than by its bytes: knowing both halves,
+ * the call lets the query kernel requantize and store the new latents itself
+ * (B <= 4), one launch and one dependent round trip fewer than the two calls.
+ * An invalid slot (seq_len[b] outside [1, Tmax]) is skipped and flags
+ * QSVD_ERANGE for qsvd_check.
+ * Requirements: B <= 64; d = H*dh, d % 256 == 0, d <= 6144; r % 32 == 0,
+ * r <= 3072; dh in {64, 128}; 8-bit X and W_d codes without a rotation.
+ * workspace: qsvd_decode_step_workspace_bytes(...) bytes, zero-filled before
+ * its first use.
  */
 int qsvd_decode_step(const qsvd_down_weight *W, const uint16_t *X, const qsvd_cache *cache,
                      const int32_t *seq_len, int32_t max_seq_len,

@@ -732,10 +732,16 @@ int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, 
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "importance_scores launch");
 }
 
+// Workspace of a decode step: the projection's part (completion counter, X
+// codes and scales, the new latents c_hat) followed by the attention's.
+static size_t step_proj_bytes(int B, int d, int r) {
+    return 256 + align256(size_t(B) * d) + align256(size_t(B) * 4) + align256(size_t(B) * r * 4);
+}
+
 size_t qsvd_decode_step_workspace_bytes(int32_t B, int32_t max_seq_len, int32_t d, int32_t r, int32_t H,
                                         int32_t dh) {
     if (B <= 0 || max_seq_len <= 0 || d <= 0 || r <= 0 || H <= 0 || dh <= 0) return 0;
-    return fused_workspace_bytes(B, max_seq_len, d, r, H, dh);
+    return step_proj_bytes(B, d, r) + decode_workspace_bytes(B, max_seq_len, r, H, dh);
 }
 
 int qsvd_decode_step(const qsvd_down_weight *W, const uint16_t *X, const qsvd_cache *cache, const int32_t *seq_len,
@@ -751,13 +757,13 @@ int qsvd_decode_step(const qsvd_down_weight *W, const uint16_t *X, const qsvd_ca
     if (W->rot) return fail(QSVD_EUNSUPPORTED, "decode_step: rotated weights (W->rot) need qsvd_latent_project");
     if ((W->w_bits && W->w_bits != 8) || (W->x_bits && W->x_bits != 8))
         return fail(QSVD_EUNSUPPORTED, "decode_step: 4-bit settings (W->w_bits, W->x_bits) need qsvd_latent_project");
-    const int d = W->d, r = W->r;
+    const int d = W->d, r = W->r, B = cache->B;
     if (r != cache->r) return fail(QSVD_EINVAL, "decode_step: weight rank differs from the cache's");
     if (dh != 64 && dh != 128) return fail(QSVD_EUNSUPPORTED, "decode_step: dh must be 64 or 128");
     if (H <= 0 || H * dh != d) return fail(QSVD_EINVAL, "decode_step: H * dh must equal d");
     if (d % 256 || d > 6144) return fail(QSVD_EUNSUPPORTED, "decode_step: need d %% 256 == 0 and d <= 6144");
-    if (r > 3072) return fail(QSVD_EUNSUPPORTED, "decode_step: r > 3072");
-    if (cache->B > kFuseMaxB) return fail(QSVD_EUNSUPPORTED, "decode_step: more than %d sequences", kFuseMaxB);
+    if (r > 3072 || r % 32) return fail(QSVD_EUNSUPPORTED, "decode_step: need r %% 32 == 0 and r <= 3072");
+    if (B > kPsMaxSplitTok) return fail(QSVD_EUNSUPPORTED, "decode_step: more than %d sequences", kPsMaxSplitTok);
     if (max_seq_len < 1 || max_seq_len > cache->Tmax)
         return fail(QSVD_EINVAL, "decode_step: max_seq_len outside [1, Tmax]");
     if (!(act_clip > 0.0f && act_clip <= 1.0f) || !(lat_clip > 0.0f && lat_clip <= 1.0f))
@@ -765,13 +771,37 @@ int qsvd_decode_step(const qsvd_down_weight *W, const uint16_t *X, const qsvd_ca
     const void *ptrs[] = {X, W->codes, W->scale, U_q, U_k, U_v, O, workspace};
     for (const void *p : ptrs)
         if (p && !aligned16(p)) return fail(QSVD_EINVAL, "decode_step: pointers must be 16-byte aligned");
-    const size_t need = fused_workspace_bytes(cache->B, max_seq_len, d, r, H, dh);
+    const size_t need = qsvd_decode_step_workspace_bytes(B, max_seq_len, d, r, H, dh);
     if (!workspace || workspace_bytes < need) return fail(QSVD_ENOSPC, "decode_step: workspace needs %zu bytes", need);
-    FusedArgs a{X, W->codes, W->scale, view(cache), seq_len, max_seq_len, U_q, U_k, U_v, d, H, dh,
-                act_clip, lat_clip, softmax_scale, O};
+
+    char *wsp = static_cast<char *>(workspace);
+    int *counter = reinterpret_cast<int *>(wsp);
+    int8_t *xq = reinterpret_cast<int8_t *>(wsp + 256);
+    float *xs = reinterpret_cast<float *>(wsp + 256 + align256(size_t(B) * d));
+    float *c_hat = reinterpret_cast<float *>(wsp + 256 + align256(size_t(B) * d) + align256(size_t(B) * 4));
+    char *dws = wsp + step_proj_bytes(B, d, r);
+
     prof_mark(stream, "begin");
-    cudaError_t e = launch_decode_fused(a, workspace, workspace_bytes, err, stream);
-    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "decode_step launch");
+    // a1-a2: the decode-size projection leaves the new latents in c_hat (one
+    // token: every CTA quantizes the row itself; more: each row quantized once)
+    cudaError_t e = cudaSuccess;
+    if (B < kPsSplitTok) {
+        e = launch_proj_small(X, B, d, act_clip, W->codes, W->scale, r, cache->bits, lat_clip, c_hat, counter, nullptr,
+                              nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, err, stream, nullptr,
+                              nullptr, false, 127);
+    } else {
+        e = launch_xquant(X, B, d, act_clip, xq, nullptr, xs, stream, 0, 127);
+        if (e == cudaSuccess)
+            e = launch_proj_small(X, B, d, act_clip, W->codes, W->scale, r, cache->bits, lat_clip, c_hat, counter,
+                                  nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, err, stream,
+                                  xq, xs, false, 127);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "decode_step projection launch");
+    // a3-a8: requantize and append the new latents, then attend
+    DecodeArgs a{view(cache), seq_len, max_seq_len, UpW{U_q, nullptr, 16}, UpW{U_k, nullptr, 16},
+                 UpW{U_v, nullptr, 16}, H, dh, softmax_scale, O, c_hat, lat_clip};
+    e = launch_decode(a, dws, workspace_bytes - step_proj_bytes(B, d, r), err, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "decode_step attention launch");
 }
 
 }  // extern "C"

@@ -133,12 +133,105 @@ __device__ __forceinline__ void unpack16B(const uint4 &v, float (&f)[128 / WB]) 
 // columns x NB sequences over its row group; the row groups are added in
 // shared memory, then rank k adds the kCl partials of columns
 // [k ncol/kCl, (k+1) ncol/kCl) in rank order.  CTA (0, 0) also clears qmax.
+//
+// FRESH: the current tokens' latents are not in the cache yet; c_hat holds
+// them as the projection left them (fp32, row b = sequence b).  Every CTA
+// requantizes each row the way requant_kernel does (Eq. 11's Q(C_qkv): the
+// same quantizer on the same values gives the same codes and scales), keeps
+// the dequantized values of its own rows, and the CTAs of the first cluster
+// store their rows' codes, with the scales, at position L - 1 of the
+// sequence (a4).  This saves a decode step the requantization launch and one
+// dependent round trip; the kernels that read the cache run after this grid.
 // ---------------------------------------------------------------------------
-template <int NB, int WB>
+constexpr int kFreshQuads = 3;     // float4 of a latent row per thread (r <= 3072)
+
+template <int NB>
+__device__ __forceinline__ void fresh_rows(const float *c_hat, int b0, int nb, const int *L_s, const int *Q_s,
+                                           const CacheView &c, float lat_clip, int j0, int rs, bool writer,
+                                           float *c_s, float (*red)[8]) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, r = c.r, nq = r / 4;
+    const int q_lo = j0 / 4, q_hi = (j0 + rs) / 4;      // this CTA's quads
+    float4 v[NB][kFreshQuads];
+#pragma unroll
+    for (int bi = 0; bi < NB; ++bi)
+#pragma unroll
+        for (int k = 0; k < kFreshQuads; ++k) {
+            const int qi = tid + k * 256;
+            v[bi][k] = (bi < nb && L_s[bi] > 0 && qi < nq)
+                           ? reinterpret_cast<const float4 *>(c_hat + size_t(b0 + bi) * r)[qi]
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    if (c.bits == 8) {
+        // one scale per token: the maximum over all r channels
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi) {
+            float m = 0.0f;
+#pragma unroll
+            for (int k = 0; k < kFreshQuads; ++k)
+                m = fmaxf(m, fmaxf(fmaxf(fabsf(v[bi][k].x), fabsf(v[bi][k].y)),
+                                   fmaxf(fabsf(v[bi][k].z), fabsf(v[bi][k].w))));
+            m = warp_max(m);
+            if (lane == 0) red[bi][warp] = m;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi) {
+            // rows without a valid slot hold zeros: zero scale, zero values, nothing stored
+            const bool live = bi < nb && L_s[bi] > 0;
+            float m = red[bi][0];
+#pragma unroll
+            for (int w = 1; w < 8; ++w) m = fmaxf(m, red[bi][w]);
+            const float s = quant_scale(m, lat_clip, 127.0f), inv = quant_inv_scale(s);
+            const size_t slot = live ? size_t(Q_s[bi]) * c.Tmax + (L_s[bi] - 1) : 0;
+#pragma unroll
+            for (int k = 0; k < kFreshQuads; ++k) {
+                const int qi = tid + k * 256;
+                if (qi < q_lo || qi >= q_hi) continue;
+                const int c0 = quant_code_fast(v[bi][k].x, s, inv, 127), c1 = quant_code_fast(v[bi][k].y, s, inv, 127);
+                const int c2 = quant_code_fast(v[bi][k].z, s, inv, 127), c3 = quant_code_fast(v[bi][k].w, s, inv, 127);
+                *reinterpret_cast<float4 *>(c_s + bi * rs + 4 * qi - j0) =
+                    make_float4(float(c0) * s, float(c1) * s, float(c2) * s, float(c3) * s);
+                if (writer && live)
+                    reinterpret_cast<uint32_t *>(static_cast<int8_t *>(c.codes) + slot * r)[qi] =
+                        uint32_t(c0 & 0xff) | (uint32_t(c1 & 0xff) << 8) | (uint32_t(c2 & 0xff) << 16) |
+                        (uint32_t(c3 & 0xff) << 24);
+            }
+            if (writer && live && j0 == 0 && tid == 0) static_cast<float *>(c.scales)[slot] = s;
+        }
+    } else {
+        // one fp16 scale per 128-channel group: the 32 quads of a group are one warp's lanes
+#pragma unroll
+        for (int bi = 0; bi < NB; ++bi) {
+            const bool live = bi < nb && L_s[bi] > 0;
+            const size_t slot = live ? size_t(Q_s[bi]) * c.Tmax + (L_s[bi] - 1) : 0;
+#pragma unroll
+            for (int k = 0; k < kFreshQuads; ++k) {
+                const int qi = tid + k * 256;
+                if (qi - lane >= nq) break;                 // warp-uniform
+                float m = fmaxf(fmaxf(fabsf(v[bi][k].x), fabsf(v[bi][k].y)), fmaxf(fabsf(v[bi][k].z), fabsf(v[bi][k].w)));
+                m = warp_max(m);
+                if (qi < q_lo || qi >= q_hi) continue;
+                const __half hs = int4_group_scale(m, lat_clip);
+                const float s = __half2float(hs), inv = quant_inv_scale(s);
+                const int c0 = quant_code_fast(v[bi][k].x, s, inv, 7), c1 = quant_code_fast(v[bi][k].y, s, inv, 7);
+                const int c2 = quant_code_fast(v[bi][k].z, s, inv, 7), c3 = quant_code_fast(v[bi][k].w, s, inv, 7);
+                *reinterpret_cast<float4 *>(c_s + bi * rs + 4 * qi - j0) =
+                    make_float4(float(c0) * s, float(c1) * s, float(c2) * s, float(c3) * s);
+                if (writer && live) {
+                    reinterpret_cast<uint16_t *>(static_cast<uint8_t *>(c.codes) + slot * (r / 2))[qi] =
+                        uint16_t((c0 & 0xf) | ((c1 & 0xf) << 4) | ((c2 & 0xf) << 8) | ((c3 & 0xf) << 12));
+                    if (lane == 0) static_cast<__half *>(c.scales)[slot * (r / 128) + qi / 32] = hs;
+                }
+            }
+        }
+    }
+}
+
+template <int NB, int WB, bool FRESH>
 __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(256)
 qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint8_t *__restrict__ Uq, const float *__restrict__ sq,
              CacheView c, const int32_t *__restrict__ seq_len, int B, int d, int ncol, float *__restrict__ q,
-             unsigned *__restrict__ qmax, int n_qmax, int *err) {
+             unsigned *__restrict__ qmax, int n_qmax, const float *c_hat, float lat_clip, int *err) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ int L_s[NB], Q_s[NB];   // length and cache sequence of each row
@@ -189,6 +282,10 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint8_t *__restric
             Q_s[tid] = sq;
         }
         __syncthreads();
+        if constexpr (FRESH) {
+            __shared__ float red_f[NB][8];
+            fresh_rows<NB>(c_hat, b0, nb, L_s, Q_s, c, lat_clip, j0, rs, blockIdx.y == 0, c_s, red_f);
+        } else {
         // dequantized latent rows c_{L-1}: code words and scales, every load issued first
         constexpr int kPer = (NB * 96 + 255) / 256;      // >= words per thread (rs <= 384)
         uint32_t wv[kPer];
@@ -232,6 +329,7 @@ qproj_kernel(const __grid_constant__ CUtensorMap map_u, const uint8_t *__restric
                 *reinterpret_cast<float4 *>(c_s + bi * rs + 8 * x) = make_float4(f[0], f[1], f[2], f[3]);
                 *reinterpret_cast<float4 *>(c_s + bi * rs + 8 * x + 4) = make_float4(f[4], f[5], f[6], f[7]);
             }
+        }
         }
         for (int i = nb * rs + tid; i < NB * rs; i += blockDim.x) c_s[i] = 0.0f;
         if (!ready) {
@@ -589,15 +687,17 @@ int pass_nb(int B) {
     return nb;
 }
 
-template <int NB, int WB>
+template <int NB, int WB, bool FRESH = false>
 cudaError_t qproj_nb(const CUtensorMap &map, const UpW &Uq, const CacheView &c, const int32_t *seq_len, int d, float *q,
-                     unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
+                     unsigned *qmax, int n_qmax, int *err, cudaStream_t s, const float *c_hat = nullptr,
+                     float lat_clip = 1.0f) {
     const int rs = c.r / kCl, ncol = qproj_cols(c.r), G = 256 / (ncol / 4);
     const size_t smem = size_t(rs) * ncol * WB / 8 + size_t(NB) * rs * 4 + size_t(G) * NB * ncol * 4;
-    cudaError_t e = ensure_smem(qproj_kernel<NB, WB>, smem);
+    cudaError_t e = ensure_smem(qproj_kernel<NB, WB, FRESH>, smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(qproj_kernel<NB, WB>, dim3(kCl, d / ncol), dim3(256), smem, s, map,
-                      static_cast<const uint8_t *>(Uq.w), Uq.scale, c, seq_len, c.B, d, ncol, q, qmax, n_qmax, err);
+    return launch_pdl(qproj_kernel<NB, WB, FRESH>, dim3(kCl, d / ncol), dim3(256), smem, s, map,
+                      static_cast<const uint8_t *>(Uq.w), Uq.scale, c, seq_len, c.B, d, ncol, q, qmax, n_qmax, c_hat,
+                      lat_clip, err);
 }
 
 template <int NB, int WB>
@@ -679,12 +779,26 @@ template <int NB, int WB> struct CombineF {
 
 }  // namespace
 
+bool qproj_fresh_supported(const CacheView &c, const UpW &Uq) {
+    return c.B <= kFreshMaxB && Uq.bits == 16 && c.r <= 4 * 256 * kFreshQuads;
+}
+
 cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const UpW &Uq, int d, float *q,
-                         unsigned *qmax, int n_qmax, int *err, cudaStream_t s) {
+                         unsigned *qmax, int n_qmax, int *err, cudaStream_t s, const float *c_hat, float lat_clip) {
     const int rs = c.r / kCl, ncol = qproj_cols(c.r);
+    if (c_hat && !qproj_fresh_supported(c, Uq)) return cudaErrorInvalidValue;
     CUtensorMap map;
     if (!up_map(&map, Uq, c.r, d, ncol, box_rows(rs))) return cudaErrorInvalidValue;
-    const cudaError_t e = dispatch_nb_wb<QprojF>(c.B, Uq.bits, map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s);
+    cudaError_t e;
+    if (c_hat) {
+        switch (pass_nb(c.B)) {
+            case 1: e = qproj_nb<1, 16, true>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s, c_hat, lat_clip); break;
+            case 2: e = qproj_nb<2, 16, true>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s, c_hat, lat_clip); break;
+            default: e = qproj_nb<4, 16, true>(map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s, c_hat, lat_clip); break;
+        }
+    } else {
+        e = dispatch_nb_wb<QprojF>(c.B, Uq.bits, map, Uq, c, seq_len, d, q, qmax, n_qmax, err, s);
+    }
     prof_mark(s, "qproj");
     return e;
 }

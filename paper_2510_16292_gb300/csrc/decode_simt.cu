@@ -313,11 +313,20 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
     // the warp-level attention kernel can form the per-head maxima of q~ itself (r <= 2048)
     const bool mma_attn = attn_mma_use(c, H, B, a.max_seq_len) && attn_mma_fits(c, a.max_seq_len);
     const bool local_qmax = mma_attn && r <= 2048 && r % 128 == 0;
-    if (!mma && qfuse_use(c, a.U_q, a.U_k, H, dh)) {
+    const bool qfuse = !mma && qfuse_use(c, a.U_q, a.U_k, H, dh);
+    // the step's new latents: requantized and stored by the query kernel itself
+    // where it can, else by their own launch first
+    const bool fresh_q = a.c_hat && !mma && !qfuse && qproj_fresh_supported(c, a.U_q);
+    if (a.c_hat && !fresh_q) {
+        e = launch_requant_len(a.c_hat, B, r, c.bits, a.lat_clip, c, a.seq_len, err, s);
+        if (e != cudaSuccess) return e;
+    }
+    if (qfuse) {
         e = launch_qfuse(c, a.seq_len, a.U_q, a.U_k, H, dh, w.qt, local_qmax ? nullptr : w.qmax, err, s);
     } else {
         e = mma ? launch_qproj_mma(c, a.seq_len, static_cast<const uint16_t *>(a.U_q.w), d, w.q, w.qmax, B * H, err, s)
-                : launch_qproj(c, a.seq_len, a.U_q, d, w.q, w.qmax, B * H, err, s);
+                : launch_qproj(c, a.seq_len, a.U_q, d, w.q, w.qmax, B * H, err, s, fresh_q ? a.c_hat : nullptr,
+                               a.lat_clip);
         if (e != cudaSuccess) return e;
         e = mma ? launch_qabsorb_mma(w.q, static_cast<const uint16_t *>(a.U_k.w), B, r, d, H, dh, w.qt, w.qmax, s)
                 : launch_qabsorb(w.q, a.U_k, B, r, d, H, dh, w.qt, w.qmax, err, s);
@@ -331,8 +340,7 @@ cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *e
         int ts = 16, n_sub = 1;
         ns = attn_mma_splits(c, B, H, a.max_seq_len, &ts, &n_sub);
         chunk = ts * n_sub;
-        const bool fused_q = !mma && qfuse_use(c, a.U_q, a.U_k, H, dh);
-        e = launch_attn_mma(c, a.seq_len, w.qt, fused_q && local_qmax ? nullptr : w.qmax, H, a.softmax_scale, ts,
+        e = launch_attn_mma(c, a.seq_len, w.qt, qfuse && local_qmax ? nullptr : w.qmax, H, a.softmax_scale, ts,
                             n_sub, ns, w.pm, w.pl, w.po, err, s);
         if (e != cudaSuccess) return e;
         prof_mark(s, "attn_mma");

@@ -203,6 +203,10 @@ cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float
                            void *lat_codes, void *lat_scales, const CacheView *dst,
                            const int32_t *dst_seq, const int32_t *dst_pos, int *err,
                            cudaStream_t s);
+// The same for the B rows of a decode step: row b goes to position
+// seq_len[b] - 1 of the cache sequence behind b.
+cudaError_t launch_requant_len(const float *c_hat, int B, int r, int bits, float clip, const CacheView &dst,
+                               const int32_t *seq_len, int *err, cudaStream_t s);
 
 // Copy token-major latent rows into the cache (a4).
 cudaError_t launch_append(const CacheView &c, const int32_t *seq, const int32_t *pos, int64_t n,
@@ -227,6 +231,10 @@ struct DecodeArgs {
     int H, dh;
     float softmax_scale;
     float *O;
+    // nullable: the step's new latents (fp32 [B, r]), requantized with lat_clip
+    // and stored at position seq_len[b] - 1 before the attention reads the cache
+    const float *c_hat;
+    float lat_clip;
 };
 size_t decode_workspace_bytes(int B, int max_seq_len, int r, int H, int dh);
 
@@ -274,8 +282,14 @@ cudaError_t launch_combine_mma(const int32_t *seq_len, const int32_t *seq_map, i
                                const float *pm, const float *pl, const float *po, const uint16_t *Uv, float *O,
                                cudaStream_t s);
 // The CUDA-core forms (decode_gemv.cu); they read every weight format.
+// c_hat (nullable): the step's new latents, fp32 [B, r] as the projection left
+// them; qproj then requantizes them itself and stores them at position
+// seq_len[b] - 1 (a3/a4), for up to kFreshMaxB sequences with bf16 U_q.
+constexpr int kFreshMaxB = 4;
+bool qproj_fresh_supported(const CacheView &c, const UpW &Uq);
 cudaError_t launch_qproj(const CacheView &c, const int32_t *seq_len, const UpW &Uq, int d, float *q,
-                         unsigned *qmax, int n_qmax, int *err, cudaStream_t s);
+                         unsigned *qmax, int n_qmax, int *err, cudaStream_t s, const float *c_hat = nullptr,
+                         float lat_clip = 1.0f);
 cudaError_t launch_qabsorb(const float *q, const UpW &Uk, int B, int r, int d, int H, int dh, float *qt,
                            unsigned *qmax, int *err, cudaStream_t s);
 cudaError_t launch_combine_uv(const int32_t *seq_len, const int32_t *seq_map, int nseq, int B, int Tmax, int H, int dh,
@@ -315,22 +329,6 @@ cudaError_t launch_attn_tc(const CacheView &c, const int32_t *seq_len, const flo
                            int tiles_per_split, int n_split, float *pm, float *pl, float *po, int *err,
                            cudaStream_t s);
 
-// One fused decode step (a1-a8) for B <= kFuseMaxB sequences, one new token each.
-constexpr int kFuseMaxB = 8;
-struct FusedArgs {
-    const uint16_t *X;
-    const int8_t *w_codes;
-    const float *w_scale;
-    CacheView cache;
-    const int32_t *seq_len;
-    int max_seq_len;
-    const uint16_t *U_q, *U_k, *U_v;
-    int d, H, dh;
-    float act_clip, lat_clip, softmax_scale;
-    float *O;
-};
-size_t fused_workspace_bytes(int B, int max_seq_len, int d, int r, int H, int dh);
-cudaError_t launch_decode_fused(const FusedArgs &a, void *ws, size_t ws_bytes, int *err, cudaStream_t s);
 cudaError_t launch_decode(const DecodeArgs &a, void *ws, size_t ws_bytes, int *err,
                           cudaStream_t s);
 

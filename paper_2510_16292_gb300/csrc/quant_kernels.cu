@@ -326,6 +326,34 @@ cudaError_t launch_requant(const float *c_hat, int64_t T, int r, int bits, float
     return e;
 }
 
+// The rows of a decode step: row b of c_hat is the new token of sequence b,
+// stored at position seq_len[b] - 1 of the cache sequence behind b (an
+// invalid slot is skipped and flagged).
+__global__ void __launch_bounds__(kRqThreads)
+requant_len_kernel(const float *c_hat, int r, int bits, float clip, CacheView dst,
+                   const int32_t *__restrict__ seq_len, int *err) {
+    __shared__ float red[kRqThreads / 32];
+    __shared__ int32_t seq_s, pos_s;
+    pdl_trigger();
+    pdl_wait();
+    if (threadIdx.x == 0) {
+        const int b = int(blockIdx.x);
+        seq_s = view_seq(dst, b);
+        pos_s = seq_s < 0 ? -1 : seq_len[b] - 1;
+    }
+    __syncthreads();
+    requant_row_cta(c_hat + size_t(blockIdx.x) * r, 0, r, bits, clip, nullptr, nullptr, dst, &seq_s, &pos_s, err, red);
+}
+
+cudaError_t launch_requant_len(const float *c_hat, int B, int r, int bits, float clip, const CacheView &dst,
+                               const int32_t *seq_len, int *err, cudaStream_t s) {
+    if (B <= 0) return cudaSuccess;
+    cudaError_t e = launch_pdl(requant_len_kernel, dim3(unsigned(B)), dim3(kRqThreads), 0, s, c_hat, r, bits, clip,
+                               dst, seq_len, err);
+    prof_mark(s, "requant");
+    return e;
+}
+
 // ---------------------------------------------------------------------------
 // a2/a3/a4 after a split-K projection GEMM: one CTA per token row adds the
 // splits' int32 partial sums in split order (exact: |acc| < 2^31), forms

@@ -1,5 +1,7 @@
-"""GPU parity of the single-launch decode step (qsvd_decode_step) against the
-CPU oracle: cache codes bit-exact, outputs within 2e-3 * ||o_ref||_2."""
+"""GPU parity of the one-call decode step (qsvd_decode_step) against the CPU
+oracle: cache codes bit-exact, outputs within 2e-3 * ||o_ref||_2.  Up to four
+sequences the query kernel requantizes and stores the new latents itself;
+from five on a separate requantization launch does (both are covered)."""
 import numpy as np
 import pytest
 
@@ -53,6 +55,38 @@ def test_fused_batch_ragged(bits):
     _run(wl, inp, pipeline.prepare_weights(inp), 2, {0, 1}, lens=[1, 63, 300])
 
 
+@pytest.mark.parametrize("B,bits", [(2, 8), (4, 8), (4, 4), (6, 8), (6, 4), (17, 8)])
+def test_fused_batch_sizes(B, bits):
+    """Both ways of storing the new latents (in the query kernel up to four
+    sequences, in their own launch from five) and the batched query forms."""
+    base = synthetic.WORKLOADS["llava7b"]
+    wl = synthetic.Workload("batch", base.shape, B=B, n_image=0, n_text=160, decode_steps=3, lat_bits=bits)
+    inp = synthetic.gen_layer(wl, seed=11 + B)
+    lens = [1 + (37 * b) % 160 for b in range(B)]
+    _run(wl, inp, pipeline.prepare_weights(inp), 3, {0, 2}, lens=lens)
+
+
+def test_fused_matches_two_calls_bit_for_bit():
+    """The one-call step and qsvd_latent_project + qsvd_latent_decode_attn give
+    the same cache bytes and the same outputs."""
+    base = synthetic.WORKLOADS["llava7b"]
+    for B in (1, 3):
+        wl = synthetic.Workload("pair", base.shape, B=B, n_image=0, n_text=96, decode_steps=2, lat_bits=8)
+        inp = synthetic.gen_layer(wl, seed=21 + B)
+        w = pipeline.prepare_weights(inp)
+        one, two = GpuLayer(wl.shape, w, B, wl.tmax, 8), GpuLayer(wl.shape, w, B, wl.tmax, 8)
+        for b in range(B):
+            one.prefill(b, inp.X_prefill[b])
+            two.prefill(b, inp.X_prefill[b])
+        for step in range(2):
+            o1 = one.decode_step_fused(inp.X_decode[step]).cpu().numpy()
+            o2 = two.decode_step(inp.X_decode[step]).cpu().numpy()
+            np.testing.assert_array_equal(o1, o2)
+        q().qsvd_check()
+        np.testing.assert_array_equal(one.cache.codes.cpu().numpy(), two.cache.codes.cpu().numpy())
+        np.testing.assert_array_equal(one.cache.scales.cpu().numpy(), two.cache.scales.cpu().numpy())
+
+
 def test_fused_13b_shape():
     base = synthetic.WORKLOADS["llava13b"]
     wl = synthetic.Workload("13b_small", base.shape, B=2, n_image=200, n_text=40, decode_steps=2, lat_bits=8)
@@ -63,7 +97,7 @@ def test_fused_13b_shape():
 def test_fused_rejects_large_batch():
     lib = q()
     base = synthetic.WORKLOADS["llava7b"]
-    wl = synthetic.Workload("big", base.shape, B=9, n_image=0, n_text=4, decode_steps=1, lat_bits=8)
+    wl = synthetic.Workload("big", base.shape, B=65, n_image=0, n_text=4, decode_steps=1, lat_bits=8)
     inp = synthetic.gen_layer(wl, seed=1)
     gpu = GpuLayer(wl.shape, pipeline.prepare_weights(inp), wl.B, wl.tmax, 8)
     with pytest.raises(lib.QsvdError) as e:
