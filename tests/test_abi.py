@@ -102,3 +102,22 @@ def test_prefill_row_group_sizes(lib):
     finally:
         setg(prev)
     assert setg(-1) < 0 and setg(65536) < 0
+
+
+def test_decode_step_workspace(lib):
+    """qsvd_decode_step's workspace: the projection's part (a 256-byte
+    completion counter, then the X codes, their scales and the fp32 latent rows
+    of the B new tokens, each rounded up to 256 bytes) followed by the decode
+    attention's workspace for the same B and length."""
+    sw = lib.qsvd_decode_step_workspace_bytes
+    sw.restype = ctypes.c_size_t
+    sw.argtypes = [ctypes.c_int32] * 6
+    dw = lib.qsvd_decode_workspace_bytes
+    dw.restype = ctypes.c_size_t
+    dw.argtypes = [ctypes.c_int32] * 5
+    up = lambda x: (x + 255) // 256 * 256  # noqa: E731
+    for B, L, d, r, H in ((1, 768, 4096, 1536, 32), (3, 300, 4096, 1536, 32), (16, 4352, 4096, 1536, 32),
+                          (8, 3520, 5120, 2048, 40), (64, 1024, 4096, 3072, 32)):
+        proj = 256 + up(B * d) + up(4 * B) + up(4 * B * r)
+        assert sw(B, L, d, r, H, 128) == proj + dw(B, L, r, H, 128)
+    assert sw(0, 768, 4096, 1536, 32, 128) == 0 and sw(1, 768, 4096, 1536, 0, 128) == 0

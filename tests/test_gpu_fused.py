@@ -8,7 +8,7 @@ import pytest
 import synthetic
 from oracle import pipeline
 
-from gpu_util import GpuLayer, assert_rows_close, q
+from gpu_util import GpuLayer, assert_rows_close, bf16, dev, i32, q
 
 pytestmark = pytest.mark.gpu
 
@@ -103,3 +103,41 @@ def test_fused_rejects_large_batch():
     with pytest.raises(lib.QsvdError) as e:
         gpu.decode_step_fused(inp.X_decode[0])
     assert e.value.status == lib.QSVD_EUNSUPPORTED
+
+
+@pytest.mark.parametrize("B", [2, 6])
+def test_fused_invalid_length_flagged(B):
+    """A sequence whose length is outside [1, Tmax] gets no cache row and flags
+    QSVD_ERANGE; the other sequences of the step are unaffected (both ways of
+    storing the new latents: in the query kernel at B = 2, in their own launch
+    at B = 6)."""
+    import torch
+    lib = q()
+    base = synthetic.WORKLOADS["llava7b"]
+    wl = synthetic.Workload("bad", base.shape, B=B, n_image=0, n_text=40, decode_steps=1, lat_bits=8)
+    s = wl.shape
+    inp = synthetic.gen_layer(wl, seed=31 + B)
+    w = pipeline.prepare_weights(inp)
+    ref = pipeline.OracleLayer(s, w, B, wl.tmax, 8)
+    gpu = GpuLayer(s, w, B, wl.tmax, 8)
+    for b in range(B):
+        ref.prefill(b, inp.X_prefill[b])
+        gpu.prefill(b, inp.X_prefill[b])
+    _, outs = ref.decode_step(inp.X_decode[0])
+    codes_before = gpu.cache.codes.clone()
+    lens = np.full(B, 41, dtype=np.int32)
+    lens[1] = 0
+    O = torch.empty((B, s.d), dtype=torch.float32, device=dev())
+    lib.qsvd_decode_step(gpu.W, bf16(inp.X_decode[0]), gpu.cache, i32(lens), 41, gpu.U_q, gpu.U_k, gpu.U_v, s.H,
+                         s.dh, O)
+    with pytest.raises(lib.QsvdError) as e:
+        lib.qsvd_check()
+    assert e.value.status == lib.QSVD_ERANGE
+    lib.qsvd_check()                        # the flag was cleared
+    np.testing.assert_array_equal(gpu.cache.codes[1].cpu().numpy(), codes_before[1].cpu().numpy())
+    valid = [b for b in range(B) if b != 1]
+    got = O.cpu().numpy()
+    assert_rows_close(got[valid], np.stack([outs[b] for b in valid]), "valid sequences")
+    for b in valid:
+        np.testing.assert_array_equal(gpu.cache.codes[b, :41].cpu().numpy().view(np.uint8),
+                                      ref.cache.packed_codes()[b, :41].view(np.uint8))
