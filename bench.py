@@ -60,6 +60,8 @@ def parse():
     p.add_argument("--no-prefill-attn", action="store_true")
     p.add_argument("--importance-probe", action="store_true",
                    help="only time the Eq. 10 importance scores of one 7B-shaped layer and print one line")
+    p.add_argument("--beta-probe", action="store_true",
+                   help="only time one beta of the Eq. 14 search on a 7B-shaped layer and print one line")
     p.add_argument("--u-bits", type=int, default=0, choices=[0, 8, 4],
                    help="quantize U_q, U_k, U_v per output channel to int8 or int4 (Eq. 11) and run decode "
                         "attention on the codes (qsvd_latent_decode_attn_qu); 0: bf16 up-projections")
@@ -712,6 +714,56 @@ def importance_probe(iters=3, N=1, m=4096, n=12288, k=4096):
             "peak_kind": f"{kind} bf16 x 1.1 / 2.25 (nominal tf32 / bf16)"}
 
 
+def beta_probe(iters=3, N=512, E=4096, r=1536):
+    """One beta of Eq. 14's grid search on a 7B-shaped layer (E = 4096,
+    n_out = 3E, r = 1536) with N calibration tokens: the factors of Eq. 3
+    (W_d, and Q(W^u) from fp64 Wu_r), the per-channel weight quantizer, the
+    projection of the calibration tokens (int8 latent) and the objective.
+    Inputs: seeded torch values (the time does not depend on them).  The
+    factors' kernel reads Wd_r and Wu_r in fp64 (HBM-bound); the objective is
+    an exact integer product of codes, N x 3E x r multiply-adds."""
+    import torch
+    import paper_2510_16292_gb300 as q
+    dev = torch.device("cuda", torch.cuda.current_device())
+    g = torch.Generator(device=dev)
+    g.manual_seed(98)
+    n = 3 * E
+    Wd_r = torch.randn((E, r), generator=g, device=dev, dtype=torch.float64) / E ** 0.5
+    Wu_r = torch.randn((r, n), generator=g, device=dev, dtype=torch.float64) / r ** 0.5
+    sig = torch.linspace(8.0, 0.1, r, device=dev, dtype=torch.float64)
+    fd, fu = sig ** 0.5, sig ** 0.5
+    X = (torch.randn((N, E), generator=g, device=dev) * 0.5).to(torch.bfloat16)
+    Y = torch.randn((N, n), generator=g, device=dev)
+    lc = torch.empty((N, r), dtype=torch.int8, device=dev)
+    ls = torch.empty((N,), dtype=torch.float32, device=dev)
+    E_ = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    tf, to, tt = [], [], []
+    for it in range(iters + 1):
+        e0, e1, e2, e3 = E_(), E_(), E_(), E_()
+        e0.record()
+        W_d, U = q.qsvd_beta_factors(Wd_r, Wu_r, fd, fu)
+        e1.record()
+        W = q.qsvd_quantize_weight(W_d)
+        q.qsvd_latent_project(W, X, lat_codes=lc, lat_scales=ls)
+        e2.record()
+        q.qsvd_beta_objective(Y, lc, ls, 8, r, U)
+        e3.record()
+        torch.cuda.synchronize()
+        if it:
+            tf.append(e0.elapsed_time(e1) * 1e-3)
+            to.append(e2.elapsed_time(e3) * 1e-3)
+            tt.append(e0.elapsed_time(e3) * 1e-3)
+    q.qsvd_check()
+    hbm, _, kind = peaks()
+    fbytes = E * r * (8 + 4) + r * n * (8 + 1) + n * 4
+    t_f, t_o, t_t = min(tf), min(to), min(tt)
+    return {"beta_probe": f"E={E} n_out={n} r={r} N={N}, int8 latent and Q(W^u)",
+            "factors_ms": round(t_f * 1e3, 3), "factors_gbs": round(fbytes / t_f / 1e9, 1),
+            "factors_frac_of_hbm": round(fbytes / t_f / 1e9 / hbm, 4),
+            "objective_ms": round(t_o * 1e3, 3), "objective_int_tops": round(2.0 * N * n * r / t_o / 1e12, 2),
+            "one_beta_ms": round(t_t * 1e3, 3), "peak_kind": kind}
+
+
 def cross_rank(values, op="max"):
     """Per-rank totals reduced over the ranks of the default process group
     (max: the job takes as long as its slowest rank; min: the slowest rank's
@@ -1063,6 +1115,9 @@ def main():
         return
     if args.importance_probe:
         print(json.dumps(importance_probe(iters=args.steps)), flush=True)
+        return
+    if args.beta_probe:
+        print(json.dumps(beta_probe(iters=args.steps)), flush=True)
         return
     if args.prefill_probe:
         for name in args.prefill_shapes.split(","):

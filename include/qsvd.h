@@ -215,6 +215,51 @@ int qsvd_rank_budget(const float *scores, int32_t n, int32_t k, uint8_t *keep, v
 size_t qsvd_rank_budget_workspace_bytes(void);
 
 /*
+ * The per-layer choice of beta (Sec. 3.3, Eq. 13-14), one beta at a time.
+ * Eq. 3 splits the truncated joint SVD of W_concat = [W_q W_k W_v] (E x n_out,
+ * n_out = 3E) as W_d = Wd_r Sigma^beta and W^u = Sigma^(1-beta) Wu_r; Eq. 14
+ * keeps the beta whose quantized output Y' = Q(C) Q(W^u) (Eq. 11, C = X W_d
+ * from Eq. 12) is closest to Y = X W_concat on calibration tokens.
+ *
+ * qsvd_beta_factors: the two factors at one beta from the caller's SVD
+ *   Wd_r  fp64 [E, r] row-major, Wu_r fp64 [r, n_out] row-major (the SVD is
+ *         the caller's, computed once per layer offline);
+ *   fd, fu fp64 [r]: sigma_i^beta and sigma_i^(1-beta) (the caller's powers);
+ *   W_d   fp32 [E, r] out, fp32(Wd_r[k, i] * fd[i]) (qsvd_quantize_weight's
+ *         input);
+ *   u_codes, u_scale out: Q(W^u) in the qsvd_up_weight layout (int8 [r, n_out]
+ *         or packed int4 [r, n_out/2]; fp32 [n_out]), the weight quantizer
+ *         per output channel j applied to W^u[i, j] = fu[i] * Wu_r[i, j] formed
+ *         in fp64: s_j = fp32(fp32(u_clip * max_i |W^u[i, j]|) / q_max),
+ *         code = clamp(rne(fp32(W^u[i, j] / s_j))), q_max 127 or 7.
+ *   Requirements: n_out % 128 == 0, u_bits 8 or 4, u_clip in (0, 1].
+ *
+ * qsvd_beta_objective: Eq. 14's objective for the factors of one beta,
+ *   sum over tokens n < N and channels j < n_out of (Y[n, j] - Y'[n, j])^2,
+ *   Y' = Q(C) Q(W^u).
+ *   Y          fp32 [N, n_out]: X W_concat (the caller's, once per layer);
+ *   lat_codes, lat_scales: Q(C) of the N tokens as qsvd_latent_project writes
+ *              them token-major (int8 [N, r] + fp32 [N], or packed int4
+ *              [N, r/2] + fp16 [N, r/128]; lat_bits 8 or 4);
+ *   u_codes, u_scale, u_bits: Q(W^u) as qsvd_beta_factors writes it;
+ *   objective  one fp64 out (device).  Products of codes are exact integer
+ *              sums; the scales and the squares are applied in fp64 and summed
+ *              in a fixed order (the same bits on every run).
+ *   workspace  qsvd_beta_objective_workspace_bytes(N, n_out) bytes.
+ *   Requirements: 0 < N <= 4194240, n_out % 64 == 0, r % 32 == 0 (r % 128 == 0
+ *   for an int4 latent).
+ */
+int qsvd_beta_factors(const double *Wd_r, const double *Wu_r, const double *fd, const double *fu, int32_t E,
+                      int32_t r, int32_t n_out, int32_t u_bits, float u_clip, float *W_d, void *u_codes,
+                      float *u_scale, cudaStream_t stream);
+
+int qsvd_beta_objective(const float *Y, int64_t N, int32_t n_out, const void *lat_codes, const void *lat_scales,
+                        int32_t lat_bits, int32_t r, const void *u_codes, const float *u_scale, int32_t u_bits,
+                        double *objective, void *workspace, size_t workspace_bytes, cudaStream_t stream);
+
+size_t qsvd_beta_objective_workspace_bytes(int64_t N, int32_t n_out);
+
+/*
  * The rotation H1 of Eq. 11-12 applied on the fly (for models where it is not
  * folded into the previous layer): C = Q(X H1^T) Q(H1 W_d).  H1 is the
  * block-diagonal normalized Walsh-Hadamard matrix I_{d/rot} (x) H_rot /

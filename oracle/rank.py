@@ -71,10 +71,17 @@ def quantized_qkv_error(W_q, W_k, W_v, r: int, beta: float, X, w_bits: int = 8, 
     the factors of Eq. 3 at this beta, W_d quantized per output channel,
     X per token (int8), the latent per token (lat_bits), W^u per output
     channel (u_bits).  quantize=False gives the unquantized rank-r output."""
-    X = np.asarray(X, dtype=np.float64)
     W_d, U_q, U_k, U_v, _ = svd.joint_qkv_factors(W_q, W_k, W_v, r, beta)
-    W_u = np.concatenate([U_q, U_k, U_v], axis=1)
-    Y = X @ np.concatenate([W_q, W_k, W_v], axis=1)
+    return qkv_error_from_factors(np.concatenate([W_q, W_k, W_v], axis=1), W_d,
+                                  np.concatenate([U_q, U_k, U_v], axis=1), X, w_bits, u_bits, lat_bits, quantize)
+
+
+def qkv_error_from_factors(W_concat, W_d, W_u, X, w_bits: int = 8, u_bits: int = 8, lat_bits: int = 8,
+                           quantize: bool = True):
+    """The objective of quantized_qkv_error for given factors W_d [E, r] and
+    W^u [r, n] (Eq. 3 at one beta) of W_concat [E, n]."""
+    X = np.asarray(X, dtype=np.float64)
+    Y = X @ np.asarray(W_concat, dtype=np.float64)
     if not quantize:
         return float(np.sum((Y - (X @ W_d) @ W_u) ** 2))
     Wq, s_w = quant.quantize_columns(quant.f32(W_d), w_bits)
@@ -86,7 +93,13 @@ def quantized_qkv_error(W_q, W_k, W_v, r: int, beta: float, X, w_bits: int = 8, 
 
 
 def beta_search(W_q, W_k, W_v, r: int, X, betas=tuple(np.round(np.linspace(0.0, 1.0, 11), 2)), **kw):
-    """Eq. 14 by grid search: (best beta, {beta: objective})."""
-    errs = {float(b): quantized_qkv_error(W_q, W_k, W_v, r, float(b), X, **kw) for b in betas}
+    """Eq. 14 by grid search: (best beta, {beta: objective}).  The joint SVD
+    is taken once; Eq. 3 then gives the factors of every beta."""
+    W_concat = np.concatenate([W_q, W_k, W_v], axis=1)
+    Wd_r, sig, Wu_r = svd.truncated_svd(W_concat, r)
+    errs = {}
+    for b in betas:
+        W_d, W_u = svd.factors_at_beta(Wd_r, sig, Wu_r, float(b))
+        errs[float(b)] = qkv_error_from_factors(W_concat, W_d, W_u, X, **kw)
     best = min(errs, key=lambda b: (errs[b], b))
     return best, errs

@@ -89,6 +89,16 @@ def joint_qkv_factors(W_q, W_k, W_v, r: int, beta: float):
     W_concat = np.concatenate([W_q, W_k, W_v], axis=1)
     E = W_q.shape[1]
     Wd_r, sig, Wu_r = truncated_svd(W_concat, r)
-    W_d = Wd_r * (sig ** beta)[None, :]
-    W_u = (sig ** (1.0 - beta))[:, None] * Wu_r
+    W_d, W_u = factors_at_beta(Wd_r, sig, Wu_r, beta)
     return W_d, W_u[:, :E], W_u[:, E:2 * E], W_u[:, 2 * E:], sig
+
+
+def factors_at_beta(Wd_r, sig, Wu_r, beta: float):
+    """Eq. 3 from the rank-r SVD factors: W_d = W^d_r Sigma_r^beta (E x r) and
+    W^u = Sigma_r^(1-beta) W^u_r (r x n), in fp64."""
+    if not 0.0 <= beta <= 1.0:
+        raise ValueError("beta must lie in [0, 1] (Eq. 3)")
+    sig = np.asarray(sig, dtype=np.float64)
+    W_d = np.asarray(Wd_r, dtype=np.float64) * (sig ** beta)[None, :]
+    W_u = (sig ** (1.0 - beta))[:, None] * np.asarray(Wu_r, dtype=np.float64)
+    return W_d, W_u

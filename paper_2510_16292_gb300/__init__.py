@@ -31,7 +31,9 @@ _lib = ctypes.CDLL(_LIB_PATH)
 QSVD_OK, QSVD_EINVAL, QSVD_EUNSUPPORTED, QSVD_ECUDA = 0, -1, -2, -3
 QSVD_ETIMEOUT, QSVD_ERANGE, QSVD_ENOSPC = -4, -5, -6
 EXPORTS = ("qsvd_quantize_weight", "qsvd_quantize_weight_rotated", "qsvd_quantize_weight_ex", "qsvd_importance_scores",
-           "qsvd_importance_workspace_bytes", "qsvd_rank_budget", "qsvd_rank_budget_workspace_bytes", "qsvd_latent_project", "qsvd_project_workspace_bytes",
+           "qsvd_importance_workspace_bytes", "qsvd_rank_budget", "qsvd_rank_budget_workspace_bytes",
+           "qsvd_beta_factors", "qsvd_beta_objective", "qsvd_beta_objective_workspace_bytes",
+           "qsvd_latent_project", "qsvd_project_workspace_bytes",
            "qsvd_cache_append", "qsvd_latent_decode_attn", "qsvd_decode_workspace_bytes",
            "qsvd_quantize_up", "qsvd_latent_decode_attn_qu",
            "qsvd_latent_prefill_attn", "qsvd_prefill_workspace_bytes", "qsvd_prefill_weights",
@@ -74,6 +76,10 @@ _lib.qsvd_quantize_weight_ex.argtypes = [_vp, _i32, _i32, _f32, _i32, _i32, _vp,
 _lib.qsvd_importance_scores.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _sz, _vp]
 _lib.qsvd_importance_workspace_bytes.argtypes = [_i32, _i32, _i32]
 _lib.qsvd_rank_budget.argtypes = [_vp, _i32, _i32, _vp, _vp, _sz, _vp]
+_lib.qsvd_beta_factors.argtypes = [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _i32, _f32, _vp, _vp, _vp, _vp]
+_lib.qsvd_beta_objective.argtypes = [_vp, _i64, _i32, _vp, _vp, _i32, _i32, _vp, _vp, _i32, _vp, _vp, _sz, _vp]
+_lib.qsvd_beta_objective_workspace_bytes.argtypes = [_i64, _i32]
+_lib.qsvd_beta_objective_workspace_bytes.restype = _sz
 _lib.qsvd_rank_budget_workspace_bytes.argtypes = []
 _lib.qsvd_rank_budget_workspace_bytes.restype = _sz
 _lib.qsvd_importance_workspace_bytes.restype = _sz
@@ -300,6 +306,42 @@ def qsvd_rank_budget(scores: torch.Tensor, k: int, workspace=None, stream=None) 
     _check(_lib.qsvd_rank_budget(_ptr(scores, _F32, "scores"), n, k, _ptr(keep), _ptr(workspace), workspace.numel(),
                                  _stream(stream)))
     return keep
+
+
+def qsvd_beta_factors(Wd_r: torch.Tensor, Wu_r: torch.Tensor, fd: torch.Tensor, fu: torch.Tensor, u_bits: int = 8,
+                      u_clip: float = 1.0, stream=None):
+    """Eq. 3 at one beta (Sec. 3.3): Wd_r fp64 [E, r], Wu_r fp64 [r, n_out] (the
+    truncated joint SVD), fd = sigma^beta and fu = sigma^(1-beta) fp64 [r] ->
+    (W_d fp32 [E, r], UpWeight Q(W^u) of [r, n_out])."""
+    E, r = Wd_r.shape
+    n_out = Wu_r.shape[1]
+    dev = Wd_r.device
+    W_d = torch.empty((E, r), dtype=torch.float32, device=dev)
+    codes = torch.empty((r, n_out if u_bits == 8 else n_out // 2), dtype=torch.int8 if u_bits == 8 else torch.uint8,
+                        device=dev)
+    scale = torch.empty((n_out,), dtype=torch.float32, device=dev)
+    f64 = torch.float64
+    _check(_lib.qsvd_beta_factors(_ptr(Wd_r, f64, "Wd_r"), _ptr(Wu_r, f64, "Wu_r"), _ptr(fd, f64, "fd"),
+                                  _ptr(fu, f64, "fu"), E, r, n_out, u_bits, u_clip, _ptr(W_d), _ptr(codes),
+                                  _ptr(scale), _stream(stream)))
+    return W_d, UpWeight(codes, scale, u_bits)
+
+
+def qsvd_beta_objective(Y: torch.Tensor, lat_codes: torch.Tensor, lat_scales: torch.Tensor, lat_bits: int, r: int,
+                        U: "UpWeight", workspace=None, stream=None) -> torch.Tensor:
+    """Eq. 14's objective sum (Y - Q(C) Q(W^u))^2: Y fp32 [N, n_out] = X W_concat,
+    Q(C) token-major as qsvd_latent_project writes it, U from qsvd_beta_factors.
+    Returns a one-element fp64 device tensor."""
+    N, n_out = Y.shape
+    out = torch.empty((1,), dtype=torch.float64, device=Y.device)
+    if workspace is None:
+        workspace = torch.empty(max(1, int(_lib.qsvd_beta_objective_workspace_bytes(N, n_out))), dtype=torch.uint8,
+                                device=Y.device)
+    _check(_lib.qsvd_beta_objective(_ptr(Y, _F32, "Y"), N, n_out, _ptr(lat_codes, _CODES, "lat_codes"),
+                                    _ptr(lat_scales, _SCALES, "lat_scales"), lat_bits, r,
+                                    _ptr(U.codes, _CODES, "U.codes"), _ptr(U.scale, _F32, "U.scale"), U.bits,
+                                    _ptr(out), _ptr(workspace), workspace.numel(), _stream(stream)))
+    return out
 
 
 def qsvd_project_workspace_bytes(T: int, d: int, r: int) -> int:

@@ -732,6 +732,57 @@ int qsvd_importance_scores(const float *U, const float *sigma, const float *Vt, 
     return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "importance_scores launch");
 }
 
+int qsvd_beta_factors(const double *Wd_r, const double *Wu_r, const double *fd, const double *fu, int32_t E,
+                      int32_t r, int32_t n_out, int32_t u_bits, float u_clip, float *W_d, void *u_codes,
+                      float *u_scale, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!Wd_r || !Wu_r || !fd || !fu || !W_d || !u_codes || !u_scale) return fail(QSVD_EINVAL, "beta_factors: null pointer");
+    if (E <= 0 || r <= 0 || n_out <= 0 || n_out % 128)
+        return fail(QSVD_EINVAL, "beta_factors: need E > 0, r > 0 and n_out %% 128 == 0");
+    if (u_bits != 8 && u_bits != 4) return fail(QSVD_EINVAL, "beta_factors: u_bits must be 8 or 4");
+    if (!(u_clip > 0.0f && u_clip <= 1.0f)) return fail(QSVD_EINVAL, "beta_factors: u_clip must lie in (0, 1]");
+    const void *ptrs[] = {Wd_r, Wu_r, fd, fu, W_d, u_codes, u_scale};
+    for (const void *p : ptrs)
+        if (!aligned16(p)) return fail(QSVD_EINVAL, "beta_factors: pointers must be 16-byte aligned");
+    prof_mark(stream, "begin");
+    const cudaError_t e = launch_beta_factors(Wd_r, Wu_r, fd, fu, E, r, n_out, u_bits, u_clip, W_d, u_codes, u_scale,
+                                              stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "beta_factors launch");
+}
+
+size_t qsvd_beta_objective_workspace_bytes(int64_t N, int32_t n_out) {
+    if (N <= 0 || n_out <= 0) return 0;
+    return beta_objective_partials(N, n_out) * sizeof(double);
+}
+
+int qsvd_beta_objective(const float *Y, int64_t N, int32_t n_out, const void *lat_codes, const void *lat_scales,
+                        int32_t lat_bits, int32_t r, const void *u_codes, const float *u_scale, int32_t u_bits,
+                        double *objective, void *workspace, size_t workspace_bytes, cudaStream_t stream) {
+    int *err = nullptr;
+    int st = device_setup(&err);
+    if (st) return st;
+    if (!Y || !lat_codes || !lat_scales || !u_codes || !u_scale || !objective)
+        return fail(QSVD_EINVAL, "beta_objective: null pointer");
+    if (N <= 0 || N > int64_t(65535) * 64) return fail(QSVD_EINVAL, "beta_objective: need 0 < N <= 4194240");
+    if (n_out <= 0 || n_out % 64) return fail(QSVD_EINVAL, "beta_objective: need n_out %% 64 == 0");
+    if (lat_bits != 8 && lat_bits != 4) return fail(QSVD_EINVAL, "beta_objective: lat_bits must be 8 or 4");
+    if (u_bits != 8 && u_bits != 4) return fail(QSVD_EINVAL, "beta_objective: u_bits must be 8 or 4");
+    if (r <= 0 || r % 32 || (lat_bits == 4 && r % 128))
+        return fail(QSVD_EINVAL, "beta_objective: need r %% 32 == 0 (r %% 128 == 0 for an int4 latent)");
+    const void *ptrs[] = {Y, lat_codes, lat_scales, u_codes, u_scale, objective, workspace};
+    for (const void *p : ptrs)
+        if (p && !aligned16(p)) return fail(QSVD_EINVAL, "beta_objective: pointers must be 16-byte aligned");
+    const size_t need = qsvd_beta_objective_workspace_bytes(N, n_out);
+    if (!workspace || workspace_bytes < need)
+        return fail(QSVD_ENOSPC, "beta_objective: workspace needs %zu bytes", need);
+    prof_mark(stream, "begin");
+    const cudaError_t e = launch_beta_objective(Y, N, n_out, lat_codes, lat_scales, lat_bits, r, u_codes, u_scale,
+                                                u_bits, static_cast<double *>(workspace), objective, stream);
+    return e == cudaSuccess ? QSVD_OK : cuda_fail(e, "beta_objective launch");
+}
+
 // Workspace of a decode step: the projection's part (completion counter, X
 // codes and scales, the new latents c_hat) followed by the attention's.
 static size_t step_proj_bytes(int B, int d, int r) {
