@@ -37,8 +37,9 @@ __global__ void beta_wd_kernel(const double *__restrict__ Wd_r, const double *__
         W_d[i] = __double2float_rn(Wd_r[i] * fd[i % r]);
 }
 
-// CTA: kBuTx x kBuCols consecutive output channels, rows split over kBuTy groups.
-constexpr int kBuCols = 4, kBuTx = 32, kBuTy = 8;
+// CTA: kBuTx x kBuCols consecutive output channels, rows split over kBuTy
+// groups (32 channels per CTA: n_out / 32 CTAs, 384 at the 7B shape).
+constexpr int kBuCols = 4, kBuTx = 8, kBuTy = 32;
 
 __global__ void __launch_bounds__(kBuTx * kBuTy)
 beta_up_kernel(const double *__restrict__ Wu_r, const double *__restrict__ fu, int r, int n_out, int qmax, float clip,
