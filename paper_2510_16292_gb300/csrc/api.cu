@@ -10,6 +10,7 @@
 #include <vector>
 
 #include "launch.h"
+#include "prep_beta.h"
 #include "qsvd.h"
 
 namespace qsvd {

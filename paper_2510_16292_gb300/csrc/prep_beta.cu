@@ -26,6 +26,7 @@
 
 #include "common.cuh"
 #include "launch.h"
+#include "prep_beta.h"
 
 namespace qsvd {
 
