@@ -21,6 +21,10 @@
  *   qsvd_latent_decode_attn_qu  the decode step with quantized up-projections
  *   qsvd_latent_prefill_attn causal attention of prompt tokens over that cache
  *   qsvd_latent_prefill      the same for whole prompt blocks, K and V materialised
+ *   qsvd_decode_step         project, requantize and append, and attend in one call
+ *   qsvd_beta_factors        offline Eq. 3 factors at one beta (Sec. 3.3)
+ *   qsvd_beta_objective      offline Eq. 14 objective of those factors
+ *   qsvd_latent_project_static  the decode-size projection without a workspace
  *
  * Conventions shared by every entry point:
  *   - Row-vector convention Y = X W, as in the paper.  E = d = H * dh.
