@@ -88,3 +88,21 @@ def test_latent_channel_spread_grows_with_beta():
         cn = np.linalg.norm(X @ W_d, axis=0)
         spread.append(cn.max() / cn.min())
     assert spread[0] < spread[1] < spread[2]
+
+
+def test_beta_search_matches_the_objective_per_beta():
+    """The search (one joint SVD, Eq. 3 per beta) gives, bit for bit, the
+    objective quantized_qkv_error computes from its own SVD at each beta; at
+    full rank the unquantized objective vanishes (W^d W^u = W_concat)."""
+    rng = np.random.default_rng(5)
+    E, r = 24, 10
+    Wq, Wk, Wv = (rng.standard_normal((E, E)) / np.sqrt(E) for _ in range(3))
+    X = rng.standard_normal((30, E))
+    X[:, 5] *= 20.0
+    _, errs = rank.beta_search(Wq, Wk, Wv, r, X, betas=(0.0, 0.4, 1.0))
+    for b, v in errs.items():
+        assert v == rank.quantized_qkv_error(Wq, Wk, Wv, r, b, X)
+    _, errs4 = rank.beta_search(Wq, Wk, Wv, r, X, betas=(0.3,), u_bits=4)
+    assert errs4[0.3] == rank.quantized_qkv_error(Wq, Wk, Wv, r, 0.3, X, u_bits=4)
+    full = rank.quantized_qkv_error(Wq, Wk, Wv, E, 0.5, X, quantize=False)
+    assert full <= 1e-18 * np.sum((X @ np.concatenate([Wq, Wk, Wv], axis=1)) ** 2)
