@@ -28,6 +28,19 @@ def test_host_tensors_are_refused(lib):
         lambda: lib.qsvd_prefill_weights(bf, bf, bf),
         lambda: lib.qsvd_latent_prefill(cache, [(0, 0, 4)], torch.zeros((768, 64), dtype=torch.float16), 2, 128, O,
                                         workspace=torch.zeros(16, dtype=torch.uint8)),
+        lambda: lib.qsvd_decode_step(lib.DownWeight(torch.zeros((64, 256), dtype=torch.int8),
+                                                    torch.zeros((64, 256), dtype=torch.bfloat16),
+                                                    torch.zeros(64, dtype=torch.float32)),
+                                     bf[:1], cache, i32[:1], 4, bf, bf, bf, 2, 128, O[:1],
+                                     workspace=torch.zeros(16, dtype=torch.uint8)),
+        lambda: lib.qsvd_beta_factors(torch.zeros((64, 32), dtype=torch.float64),
+                                      torch.zeros((32, 128), dtype=torch.float64),
+                                      torch.ones(32, dtype=torch.float64), torch.ones(32, dtype=torch.float64)),
+        lambda: lib.qsvd_beta_objective(torch.zeros((4, 128), dtype=torch.float32), torch.zeros((4, 32), dtype=torch.int8),
+                                        torch.zeros(4, dtype=torch.float32), 8, 32,
+                                        lib.UpWeight(torch.zeros((32, 128), dtype=torch.int8),
+                                                     torch.zeros(128, dtype=torch.float32), 8),
+                                        workspace=torch.zeros(16, dtype=torch.uint8)),
     ]
     for call in calls:
         with pytest.raises(ValueError, match="device tensor expected"):
